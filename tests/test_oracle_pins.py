@@ -1,0 +1,409 @@
+"""Pins for the fp64 oracle: each check reaches the oracle's result by another route (a
+closed form, a library routine, brute force, an invariant, or a value the paper prints), so
+a dropped term, a wrong sign, index or transposed operand in the oracle fails one of them.
+CPU only."""
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+from scipy.cluster.vq import vq
+
+from oracle import crvq_oracle as O
+import synthetic as S
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden(name):
+    rows = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                rows.append(line.split())
+    return rows
+
+
+def _spd(rng, d, cond=20.0):
+    Q, _ = np.linalg.qr(rng.standard_normal((d, d)))
+    ev = np.exp(rng.uniform(0, math.log(cond), d))
+    return ((Q * ev) @ Q.T).astype(np.float32)
+
+
+def _sym32(A):
+    A = np.asarray(A, np.float32)
+    return ((A + A.T) * np.float32(0.5)).astype(np.float32)
+
+
+# ---------------------------------------------------------------- generator pins
+def test_splitmix64_published_sequence():
+    for seed, ctr, hexv in _golden("splitmix64.txt"):
+        assert O.splitmix64(int(seed), int(ctr)) == int(hexv, 16)
+        assert int(S.splitmix64(int(seed), np.array([int(ctr)]))[0]) == int(hexv, 16)
+
+
+def test_bf16_rounding_ties_to_even():
+    a = np.array([1.0, 1.0 + 2 ** -8, 1.0 + 3 * 2 ** -8, 1.0 + 2 ** -9, -2.5], np.float32)
+    # 1 + 2^-8 is halfway between 1 and 1 + 2^-7 -> even (1.0); 1 + 3*2^-8 -> 1 + 2^-6.
+    exp = np.array([1.0, 1.0, 1.0 + 2 ** -6, 1.0, -2.5], np.float32)
+    np.testing.assert_array_equal(S.round_to_bf16(a), exp)
+
+
+# ---------------------------------------------------------------- O1 Hessian
+def test_hessian_closed_form_scaled_identity():
+    N = 16
+    X = np.sqrt(N) * np.eye(N, dtype=np.float32)    # n = N tokens: X^T X / n = I
+    H, xsq, Hb, delta = O.hessian(X, 0.25, 8)
+    np.testing.assert_allclose(H, 1.25 * np.eye(N), rtol=0, atol=1e-6)
+    np.testing.assert_allclose(xsq, np.ones(N), rtol=1e-6)
+    assert abs(float(delta) - 0.25) < 1e-7
+    np.testing.assert_allclose(Hb, np.broadcast_to(1.25 * np.eye(8), (2, 8, 8)), atol=1e-6)
+
+
+def test_hessian_matches_matrix_free_product():
+    rng = np.random.default_rng(1)
+    X = rng.standard_normal((37, 24)).astype(np.float32) * rng.uniform(0.1, 3, 24)
+    H, xsq, Hb, delta = O.hessian(X, 0.01, 8)
+    v = rng.standard_normal(24)
+    X64 = X.astype(np.float64)
+    ref = X64.T @ (X64 @ v) / 37 + float(delta) * v
+    np.testing.assert_allclose(H.astype(np.float64) @ v, ref, rtol=1e-5, atol=1e-5)
+    assert np.allclose(H, H.T)
+    np.testing.assert_allclose(xsq, (X64 ** 2).mean(axis=0), rtol=1e-6)
+    np.testing.assert_allclose(float(delta), 0.01 * (X64 ** 2).mean(), rtol=1e-6)
+    for g in range(3):
+        np.testing.assert_array_equal(Hb[g], H[8 * g:8 * g + 8, 8 * g:8 * g + 8])
+
+
+# ---------------------------------------------------------------- O2/O3 encode
+def test_encode_isotropic_is_euclidean_nearest_codeword():
+    rng = np.random.default_rng(2)
+    M, G, d, K = 40, 3, 8, 16
+    T = rng.standard_normal((M, G * d)).astype(np.float32)
+    C = rng.standard_normal((K, d)).astype(np.float32)
+    Hb = np.stack([np.float32(c) * np.eye(d, dtype=np.float32) for c in (1.0, 2.0, 0.5)])
+    codes, verr = O.encode_beam(T, d, Hb, [O.Codebook(C, None, G)], 0, 1)
+    for g in range(G):
+        ref, dist = vq(T[:, g * d:(g + 1) * d].astype(np.float64), C.astype(np.float64))
+        np.testing.assert_array_equal(codes[0][:, g], ref)
+        np.testing.assert_allclose(verr[:, g], Hb[g][0, 0] * dist ** 2, rtol=1e-5)
+
+
+def test_encode_general_H_equals_whitened_nearest_codeword():
+    """err(t,c) = ||L^T (t - c)||^2 with H = L L^T: nearest codeword after whitening."""
+    rng = np.random.default_rng(3)
+    M, G, d, K = 50, 2, 8, 32
+    T = rng.standard_normal((M, G * d)).astype(np.float32)
+    C = rng.standard_normal((K, d)).astype(np.float32)
+    Hb = np.stack([_spd(rng, d) for _ in range(G)])
+    codes, verr = O.encode_beam(T, d, Hb, [O.Codebook(C, None, G)], 0, 1)
+    for g in range(G):
+        L = np.linalg.cholesky(Hb[g].astype(np.float64))
+        ref, dist = vq(T[:, g * d:(g + 1) * d].astype(np.float64) @ L, C.astype(np.float64) @ L)
+        np.testing.assert_array_equal(codes[0][:, g], ref)
+        np.testing.assert_allclose(verr[:, g], dist ** 2, rtol=1e-5)
+
+
+def test_encode_with_fixed_codebook_equals_encode_of_residual():
+    rng = np.random.default_rng(4)
+    M, G, d = 30, 2, 4
+    T = rng.standard_normal((M, G * d)).astype(np.float32)
+    C0 = rng.standard_normal((8, d)).astype(np.float32)
+    C1 = (0.3 * rng.standard_normal((8, d))).astype(np.float32)
+    codes0 = rng.integers(0, 8, (M, G))
+    Hb = np.stack([_spd(rng, d) for _ in range(G)])
+    R = T.astype(np.float64).copy()
+    for g in range(G):
+        R[:, g * d:(g + 1) * d] -= C0[codes0[:, g]]
+    a, ea = O.encode_beam(T, d, Hb, [O.Codebook(C0, codes0, G), O.Codebook(C1, None, G)], 1, 1)
+    b, eb = O.encode_beam(R, d, Hb, [O.Codebook(C1, None, G)], 0, 1)
+    np.testing.assert_array_equal(a[1], b[0])
+    np.testing.assert_allclose(ea, eb, rtol=1e-4, atol=1e-6)
+
+
+# ---------------------------------------------------------------- O4 beam vs exhaustive
+@pytest.mark.parametrize("K,m,d", [(2, 1, 2), (4, 2, 4), (2, 3, 8), (4, 3, 2), (3, 2, 8)])
+def test_beam_with_full_width_equals_exhaustive_search(K, m, d):
+    rng = np.random.default_rng(10 * K + m + d)
+    M, G = 12, 2
+    T = rng.standard_normal((M, G * d)).astype(np.float32)
+    Cs = [(rng.standard_normal((K, d)) / (1 + s)).astype(np.float32) for s in range(m)]
+    Hb = np.stack([_spd(rng, d) for _ in range(G)])
+    B = K ** (m - 1)                                      # >= product of all but the last K
+    cbs = [O.Codebook(C, None, G) for C in Cs]
+    codes, verr = O.encode_beam(T, d, Hb, cbs, 0, B)
+    for g in range(G):
+        L = np.linalg.cholesky(Hb[g].astype(np.float64))
+        for i in range(M):
+            t = T[i, g * d:(g + 1) * d].astype(np.float64)
+            best, arg = np.inf, None
+            for tup in itertools.product(range(K), repeat=m):
+                r = t - sum(Cs[s][tup[s]].astype(np.float64) for s in range(m))
+                e = float(np.linalg.norm(L.T @ r) ** 2)
+                if e < best:
+                    best, arg = e, tup
+            assert tuple(codes[s][i, g] for s in range(m)) == arg
+            assert abs(verr[i, g] - best) <= 1e-5 * max(1.0, best)
+
+
+def test_narrow_beam_never_beats_exhaustive_and_keep_if_better_keeps_optimum():
+    rng = np.random.default_rng(11)
+    K, m, d, M, G = 4, 3, 4, 20, 1
+    T = rng.standard_normal((M, G * d)).astype(np.float32)
+    Cs = [(rng.standard_normal((K, d)) / (1 + s)).astype(np.float32) for s in range(m)]
+    Hb = np.stack([_spd(rng, d)])
+    full, efull = O.encode_beam(T, d, Hb, [O.Codebook(C, None, G) for C in Cs], 0, K ** 2)
+    narrow, enarrow = O.encode_beam(T, d, Hb, [O.Codebook(C, None, G) for C in Cs], 0, 1)
+    assert np.all(enarrow >= efull - 1e-6)
+    # seeded with the optimal tuple, the width-1 beam must keep it
+    kept, ekept = O.encode_beam(T, d, Hb, [O.Codebook(C, full[s], G) for s, C in enumerate(Cs)],
+                                0, 1, keep_if_better=True)
+    np.testing.assert_allclose(ekept, efull, rtol=1e-6)
+    for s in range(m):
+        np.testing.assert_array_equal(kept[s], full[s])
+
+
+# ---------------------------------------------------------------- O5 init
+def test_kmeans_init_strata_distinct_deterministic():
+    n, K = 1000, 37
+    a = O.kmeans_sample_indices(n, K, 123)
+    b = O.kmeans_sample_indices(n, K, 123)
+    c = O.kmeans_sample_indices(n, K, 124)
+    np.testing.assert_array_equal(a, b)
+    assert not np.array_equal(a, c)
+    assert len(set(a.tolist())) == K
+    for k, v in enumerate(a):
+        assert (k * n) // K <= v < ((k + 1) * n) // K
+    np.testing.assert_array_equal(O.kmeans_sample_indices(5, 5, 9), np.arange(5))
+
+
+def test_kmeans_init_takes_sampled_vectors_and_residuals():
+    rng = np.random.default_rng(5)
+    M, G, d, K = 10, 3, 8, 6
+    T = rng.standard_normal((M, G * d)).astype(np.float32)
+    idx = O.kmeans_sample_indices(M * G, K, 77)
+    C = O.kmeans_init(T, d, G, K, 77)
+    for k, v in enumerate(idx):
+        i, g = divmod(int(v), G)
+        np.testing.assert_array_equal(C[k], T[i, g * d:(g + 1) * d])
+    C0 = rng.standard_normal((4, d)).astype(np.float32)
+    codes0 = rng.integers(0, 4, (M, G))
+    Cr = O.kmeans_init(T, d, G, K, 77, fixed=[O.Codebook(C0, codes0, G)])
+    for k, v in enumerate(idx):
+        i, g = divmod(int(v), G)
+        np.testing.assert_allclose(Cr[k], T[i, g * d:(g + 1) * d] - C0[codes0[i, g]], atol=1e-6)
+
+
+# ---------------------------------------------------------------- O6 LS update
+def test_update_isotropic_is_cluster_mean():
+    rng = np.random.default_rng(6)
+    M, G, d, K = 60, 2, 8, 7
+    T = rng.standard_normal((M, G * d)).astype(np.float32)
+    codes = rng.integers(0, K - 1, (M, G))         # codeword K-1 stays empty
+    Cold = rng.standard_normal((K, d)).astype(np.float32)
+    Hb = np.stack([np.float32(2.0) * np.eye(d, dtype=np.float32)] * G)
+    C, counts = O.update_codebook(T, d, Hb, [O.Codebook(Cold, codes, G)], 0)
+    V = np.concatenate([T[:, g * d:(g + 1) * d] for g in range(G)])
+    code = np.concatenate([codes[:, g] for g in range(G)])
+    for k in range(K - 1):
+        np.testing.assert_allclose(C[k], V[code == k].astype(np.float64).mean(0), rtol=1e-5,
+                                   atol=1e-6)
+    np.testing.assert_array_equal(C[K - 1], Cold[K - 1])
+    np.testing.assert_array_equal(counts, np.bincount(code, minlength=K))
+
+
+def test_update_is_a_minimiser_and_single_member_is_exact():
+    rng = np.random.default_rng(7)
+    M, G, d, K = 40, 3, 8, 5
+    T = rng.standard_normal((M, G * d)).astype(np.float32)
+    codes = rng.integers(0, K, (M, G))
+    codes[0, 0] = K - 1
+    codes[(codes == K - 1)] = 0
+    codes[0, 0] = K - 1                             # codeword K-1 has exactly one member
+    Hb = np.stack([_spd(rng, d) for _ in range(G)])
+    Cold = rng.standard_normal((K, d)).astype(np.float32)
+    C, counts = O.update_codebook(T, d, Hb, [O.Codebook(Cold, codes, G)], 0)
+    assert counts[K - 1] == 1
+    np.testing.assert_allclose(C[K - 1], T[0, :d], rtol=1e-5, atol=1e-6)
+
+    def obj(k, c):
+        tot = 0.0
+        for g in range(G):
+            Dg = T[codes[:, g] == k, g * d:(g + 1) * d].astype(np.float64) - c
+            L = np.linalg.cholesky(Hb[g].astype(np.float64))
+            tot += float((np.linalg.norm(Dg @ L, axis=1) ** 2).sum())
+        return tot
+
+    for k in range(K):
+        base = obj(k, C[k].astype(np.float64))
+        for _ in range(10):
+            u = rng.standard_normal(d) * 1e-2
+            assert obj(k, C[k] + u) >= base - 1e-9 * max(1.0, base)
+
+
+def test_update_of_second_codebook_targets_residual():
+    rng = np.random.default_rng(8)
+    M, G, d = 30, 2, 4
+    T = rng.standard_normal((M, G * d)).astype(np.float32)
+    C0 = rng.standard_normal((6, d)).astype(np.float32)
+    C1 = rng.standard_normal((5, d)).astype(np.float32)
+    c0 = rng.integers(0, 6, (M, G))
+    c1 = rng.integers(0, 5, (M, G))
+    Hb = np.stack([_spd(rng, d) for _ in range(G)])
+    a, ca = O.update_codebook(T, d, Hb, [O.Codebook(C0, c0, G), O.Codebook(C1, c1, G)], 1)
+    R = T.astype(np.float64).copy()
+    for g in range(G):
+        R[:, g * d:(g + 1) * d] -= C0[c0[:, g]]
+    b, cb = O.update_codebook(R, d, Hb, [O.Codebook(C1, c1, G)], 0)
+    np.testing.assert_allclose(a, b, rtol=1e-5, atol=1e-6)
+    np.testing.assert_array_equal(ca, cb)
+
+
+def test_lloyd_objective_non_increasing():
+    rng = np.random.default_rng(9)
+    M, G, d, K = 64, 4, 8, 16
+    T = (0.02 * rng.standard_normal((M, G * d))).astype(np.float32)
+    Hb = np.stack([_spd(rng, d) for _ in range(G)])
+    C0 = O.kmeans_init(T, d, G, K, 5)
+    _, objective = O.lloyd(T, d, Hb, [], C0, G, 8)
+    assert all(b <= a * (1 + 1e-9) for a, b in zip(objective, objective[1:]))
+    assert objective[-1] < objective[0]
+
+
+# ---------------------------------------------------------------- O7/O8 importance & reorder
+def test_importance_wa_equals_literal_app_a2_sum():
+    rng = np.random.default_rng(12)
+    n, M, N = 9, 5, 16
+    X = rng.standard_normal((n, N)).astype(np.float32)
+    W = rng.standard_normal((M, N)).astype(np.float32)
+    Wq = (W + 0.1 * rng.standard_normal((M, N))).astype(np.float32)
+    _, xsq, _, _ = O.hessian(X, 0.0, 8)
+    I = O.importance(W, Wq, xsq, O.MODE_WA, 0)
+    lit = np.zeros(N)
+    for i in range(N):
+        lit[i] = max(0.5 * sum((float(X[k, i]) * (float(W[j, i]) - float(Wq[j, i]))) ** 2
+                               for k in range(n)) for j in range(M))
+    np.testing.assert_allclose(I * n, lit, rtol=1e-6)            # xsq carries the 1/n
+    np.testing.assert_allclose(O.importance(W, Wq, xsq, O.MODE_WONLY, 0),
+                               (W.astype(np.float64) ** 2).max(0))
+
+
+def test_reorder_bijection_roundtrip_and_blocks():
+    rng = np.random.default_rng(13)
+    M, N, d = 7, 32, 8
+    W = rng.standard_normal((M, N)).astype(np.float32)
+    X = rng.standard_normal((20, N)).astype(np.float32)
+    H, xsq, _, _ = O.hessian(X, 0.01, d)
+    Wq = np.round(W * 2) / 2
+    perm, I, Ws, Hb, Gc = O.select_reorder_channels(W, d, Wq, xsq, H, 0.1, O.MODE_WA, 0)
+    assert sorted(perm.tolist()) == list(range(N))
+    assert np.all(np.diff(I[perm].astype(np.float64)) <= 0)
+    inv = np.argsort(perm)
+    np.testing.assert_array_equal(Ws[:, inv], W)
+    Hp = H[np.ix_(perm, perm)]
+    for g in range(N // d):
+        np.testing.assert_array_equal(Hb[g], Hp[g * d:(g + 1) * d, g * d:(g + 1) * d])
+    assert Gc == 1
+    # random mode: a seeded permutation, deterministic
+    p1 = O.select_reorder_channels(W, d, Wq, xsq, H, 0.1, O.MODE_RANDOM, 5)[0]
+    p2 = O.select_reorder_channels(W, d, Wq, xsq, H, 0.1, O.MODE_RANDOM, 5)[0]
+    np.testing.assert_array_equal(p1, p2)
+    assert sorted(p1.tolist()) == list(range(N))
+
+
+def test_importance_ties_broken_by_index():
+    W = np.ones((3, 16), np.float32)
+    perm = O.select_reorder_channels(W, 8, np.zeros_like(W), np.ones(16, np.float32),
+                                     np.eye(16, dtype=np.float32), 0.5, O.MODE_WONLY, 0)[0]
+    np.testing.assert_array_equal(perm, np.arange(16))
+
+
+def test_n_crit_groups_closed_form():
+    for N, d, lam, gc in _golden("n_crit_groups.txt"):
+        assert O.n_crit_groups(int(N), int(d), float(lam)) == int(gc)
+    assert O.n_crit_groups(64, 8, 0.0) == 0
+    assert O.n_crit_groups(64, 8, 1.0) == 8
+
+
+def test_outlier_channels_land_in_critical_set():
+    cfg = S.C1.with_(kmeans_iters=2)
+    W, X = S.gen_W(cfg), S.gen_X(cfg)
+    d, G = cfg.d, cfg.G
+    H, xsq, Hb0, _ = O.hessian(X, cfg.damp_rel, d)
+    C0 = O.kmeans_init(W, d, G, cfg.K_base, 1)
+    pre, _ = O.lloyd(W, d, Hb0, [], C0, G, cfg.kmeans_iters)
+    W_pre = O.reconstruct_error(W, d, Hb0, None, [pre], 0)[0]
+    outl = set(S.pick_columns(cfg.seed, cfg.name + "/W/outliers", cfg.N, 8).tolist())
+    for mode in (O.MODE_WA, O.MODE_WONLY):
+        perm, _, _, _, Gc = O.select_reorder_channels(W, d, W_pre, xsq, H, cfg.crit_frac,
+                                                      mode, 0)
+        assert outl <= set(perm[:Gc * d].tolist())
+
+
+# ---------------------------------------------------------------- O10 losses & decode
+def test_loss_full_two_routes_and_block_loss_matches_encode():
+    rng = np.random.default_rng(14)
+    M, N, d, n = 6, 24, 8, 30
+    X = rng.standard_normal((n, N)).astype(np.float32)
+    W = rng.standard_normal((M, N)).astype(np.float32)
+    H, xsq, _, delta = O.hessian(X, 0.05, d)
+    perm = rng.permutation(N).astype(np.int32)
+    Ws = W[:, perm]
+    Hb = np.stack([H[np.ix_(perm[g * d:g * d + d], perm[g * d:g * d + d])] for g in range(3)])
+    C0 = rng.standard_normal((5, d)).astype(np.float32)
+    C1 = (0.2 * rng.standard_normal((4, d))).astype(np.float32)
+    cbs = [O.Codebook(C0, None, 3), O.Codebook(C1, None, 1)]
+    codes, verr = O.encode_beam(Ws, d, Hb, cbs, 0, 4)
+    cbs = [O.Codebook(C0, codes[0], 3), O.Codebook(C1, codes[1], 1)]
+    W_hat, lb, lc, lf = O.reconstruct_error(Ws, d, Hb, perm, cbs, 1, X, float(delta))
+    dW = W.astype(np.float64) - W_hat.astype(np.float64)
+    tr = float(np.trace(dW @ H.astype(np.float64) @ dW.T))
+    assert abs(lf - tr) <= 1e-5 * tr
+    assert abs(lb - float(verr.astype(np.float64).sum())) <= 1e-5 * lb
+    assert abs(lc - float(verr[:, :1].astype(np.float64).sum())) <= 1e-5 * lc
+    # reconstruction of vector (i, g) in the original order is the sum of its codewords
+    for i in range(M):
+        for g in range(3):
+            r = C0[codes[0][i, g]].astype(np.float64)
+            if g < 1:
+                r = r + C1[codes[1][i, g]]
+            np.testing.assert_allclose(W_hat[i, perm[g * d:(g + 1) * d]], r, rtol=1e-6)
+
+
+def test_codebook_holding_every_vector_gives_zero_loss():
+    rng = np.random.default_rng(15)
+    M, N, d = 4, 16, 8
+    W = rng.standard_normal((M, N)).astype(np.float32)
+    C = np.concatenate([W[:, g * d:(g + 1) * d] for g in range(2)])
+    Hb = np.stack([_spd(rng, d) for _ in range(2)])
+    codes, verr = O.encode_beam(W, d, Hb, [O.Codebook(C, None, 2)], 0, 1)
+    np.testing.assert_array_equal(verr, 0)
+    W_hat, lb, lc, _ = O.reconstruct_error(W, d, Hb, None, [O.Codebook(C, codes[0], 2)], 0)
+    np.testing.assert_array_equal(W_hat, W)
+    assert lb == 0.0 and lc == 0.0
+
+
+# ---------------------------------------------------------------- A16 bit-width (golden)
+def test_avg_bits_paper_values():
+    for e, d, m, lam, exp, dec, *_ in _golden("avg_bits.txt"):
+        v = O.avg_bits(int(e), int(d), int(m), float(lam))
+        assert round(v, int(dec)) == pytest.approx(float(exp))
+
+
+# ---------------------------------------------------------------- schedule invariants
+def test_schedule_invariants_small():
+    """Extended codebooks never raise the critical-channel loss (LS optimality vs c = 0
+    start), Lloyd objectives never rise, and one refinement round never raises the loss."""
+    cfg = S.LayerConfig("pin_small", 64, 64, 96, "outlier_cols", "lognormal", 0.5,
+                        n_outlier_cols=3, K_base=16, n_ext=2, K_ext=8, crit_frac=0.1, B=4,
+                        kmeans_iters=4)
+    out = O.quantize_layer(S.gen_W(cfg), S.gen_X(cfg), cfg)
+    cl = out["crit_loss_after_ext"]
+    assert all(b <= a * (1 + 1e-9) for a, b in zip(cl, cl[1:]))
+    ob = out["base_objective"]
+    assert all(b <= a * (1 + 1e-9) for a, b in zip(ob, ob[1:]))
+    h = out["loss_history"]
+    assert h[-1] <= h[0] * (1 + 1e-9)
+    assert out["loss_full"] > 0
