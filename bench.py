@@ -1,0 +1,335 @@
+#!/usr/bin/env python
+"""Benchmark of the CRVQ code-search hot path on GB300.
+
+A step is one weight matrix through the whole hot path (Alg. 1 lines 3-17: Hessian,
+prequantize, importance + reorder, base k-means, extended codebooks, least-squares refinement
+with beam re-encode, losses), i.e. one crvq_quantize_layer call, on the LLaMA-2-7B-shaped
+q_proj workload (W 4096 x 4096, 4096 calibration tokens, d = 8, K = 256, 1 extended codebook
+on 2% channels, B = 8, 10 Lloyd iterations). The metric is code-search throughput: scored
+(hypothesis, codeword) pairs per second over the whole step; the per-layer time is reported
+beside it.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl crvq|reference] [--config c2]
+
+With N > 1 (torchrun, one rank per GPU) every rank quantizes its own layer (independent
+problems, no collective on the data path): weak scaling; value = all ranks' scores / the
+slowest rank's time. `--impl reference` times the fp64 CPU oracle on a bounded row sample of
+the same workload (the paper ships no code; the oracle is the reference arm).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synthetic as S  # noqa: E402
+
+
+def schedule_scores(cfg, M, N):
+    """(hypothesis, codeword) pairs scored by one matrix through the schedule."""
+    d, T = cfg.d, cfg.kmeans_iters
+    G = N // d
+    Gc = min(G, int(np.ceil(np.float32(cfg.crit_frac) * N / d - 1e-12))) if cfg.crit_frac > 0 else 0
+    n_all, n_crit = M * G, M * Gc
+    s = 2 * (T + 1) * n_all * cfg.K_base                  # prequantize + base k-means
+    s += cfg.n_ext * (T + 1) * n_crit * cfg.K_ext          # extended k-means
+    beam = cfg.K_base
+    parents = min(cfg.B, cfg.K_base)
+    for _ in range(cfg.n_ext):
+        beam += parents * cfg.K_ext
+        parents = min(cfg.B, parents * cfg.K_ext)
+    s += cfg.refine_rounds * (n_crit * beam + (n_all - n_crit) * cfg.K_base)
+    return float(s)
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            return json.load(f), "measured"
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "sm_max_mhz": 2070.0}, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id):
+        self.gpu_id = gpu_id
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.gpu_id)], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.t.join(timeout=2)
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax = float(f[2])
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() in ("active", "1", "yes"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def cpu_oracle_sample(cfg, rows, X=None):
+    """Times the fp64 oracle's whole schedule on the first `rows` rows of the workload's W
+    (same X). Returns (scores/s, seconds, cores used)."""
+    from oracle import crvq_oracle as O
+    W = S.gen_W(cfg, np.arange(rows))
+    X = S.gen_X(cfg) if X is None else X
+    t0, c0 = time.perf_counter(), time.process_time()
+    O.quantize_layer(W, X, cfg)
+    wall = time.perf_counter() - t0
+    cpu = time.process_time() - c0
+    sc = schedule_scores(cfg, rows, cfg.N)
+    return sc / wall, wall, max(1, int(round(cpu / max(wall, 1e-9))))
+
+
+def dist_init():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if _cuda_ok() else "gloo")
+    return ws, rank, local
+
+
+def _cuda_ok():
+    import torch
+    return torch.cuda.is_available()
+
+
+def run_reference(args, cfg, ws, rank):
+    """Reference arm: the fp64 CPU oracle on a bounded row sample, rank 0 only."""
+    if rank != 0:
+        return
+    X = S.gen_X(cfg)
+    rows = args.ref_rows
+    for _ in range(args.warmup if args.ref_warmup else 0):
+        cpu_oracle_sample(cfg, rows, X)
+    times, cores = [], 1
+    for _ in range(args.steps):
+        _, wall, cores = cpu_oracle_sample(cfg, rows, X)
+        times.append(wall)
+    sc = schedule_scores(cfg, rows, cfg.N)
+    tot = sum(times)
+    value = sc * len(times) / tot
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "scores/s",
+        "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * tot / len(times), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": DATA,
+        "config": config_dict(cfg, rows_note=f"row sample: first {rows} of {cfg.M} rows"),
+        "cpu_baseline": {"value": value, "unit": "scores/s", "cores": cores, "kind": "oracle",
+                         "sample": f"whole schedule on rows 0..{rows - 1} of W, full X"},
+        "e2e": {"value": value, "unit": "scores/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+METRIC = "code-search scores/s (whole-layer CRVQ quantize, S1-S7)"
+DATA = ("synthetic: seeded SplitMix64/Box-Muller LLaMA-2-shaped weights and calibration "
+        "activations (no real weights or Red_Pajama text)")
+
+
+def config_dict(cfg, rows_note=None):
+    c = {"workload": cfg.name, "M": cfg.M, "N": cfg.N, "n_tok": cfg.n_tok, "d": cfg.d,
+         "K_base": cfg.K_base, "n_ext": cfg.n_ext, "K_ext": cfg.K_ext,
+         "crit_frac": cfg.crit_frac, "B": cfg.B, "kmeans_iters": cfg.kmeans_iters,
+         "refine_rounds": cfg.refine_rounds,
+         "l2": "flushed between timed steps (512 MB write)"}
+    if rows_note:
+        c["sample"] = rows_note
+    return c
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="crvq", choices=["crvq", "reference"])
+    ap.add_argument("--config", default="c2", choices=sorted(S.CONFIGS))
+    ap.add_argument("--ref-rows", type=int, default=24)
+    ap.add_argument("--ref-warmup", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    args = ap.parse_args()
+    cfg = S.CONFIGS[args.config]
+    ws, rank, local = dist_init()
+    if args.impl == "reference":
+        run_reference(args, cfg, ws, rank)
+        return
+
+    import torch
+    import paper_2412_09282_gb300 as P
+    from paper_2412_09282_gb300 import build as B
+    B.build()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    cfg_r = cfg.with_(seed=cfg.seed + rank)                # each rank: its own layer
+    Wn, Xn = S.gen_W(cfg_r), S.gen_X(cfg_r)
+    W_h = torch.from_numpy(Wn).pin_memory()
+    X_h = torch.from_numpy(Xn).pin_memory()
+    W_d, X_d = W_h.to(dev), X_h.to(dev)
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    out = None
+    for _ in range(args.warmup):
+        out = P.crvq_quantize_layer(W_d, X_d, cfg_r, out=out)
+    torch.cuda.synchronize()
+
+    def barrier():
+        if ws > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    clocks = ClockSampler(torch.cuda.get_device_properties(dev).uuid
+                          if hasattr(torch.cuda.get_device_properties(dev), "uuid") else local)
+    try:
+        clocks.gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        clocks.gpu_id = local
+    barrier()
+    clocks.start()
+    launches0 = P.crvq_launch_count()
+    P.crvq_profile_begin()
+    step_ms = []
+    scores = 0.0
+    for _ in range(args.steps):
+        flush.fill_(1.0)                                     # evict the 129 MB L2
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        out = P.crvq_quantize_layer(W_d, X_d, cfg_r, out=out)
+        b.record(stream)
+        b.synchronize()
+        step_ms.append(a.elapsed_time(b))
+        scores += out.report["scores"]
+    barrier()
+    kstats = P.crvq_profile_end()
+    launches = P.crvq_launch_count() - launches0
+    clk = clocks.stop()
+    tot_ms = sum(step_ms)
+    if ws > 1:
+        import torch.distributed as dist
+        t = torch.tensor([tot_ms, scores], dtype=torch.float64, device=dev)
+        tmax = t[:1].clone()
+        dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
+        dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
+        tot_ms_max, scores_all = float(tmax[0]), float(t[1])
+    else:
+        tot_ms_max, scores_all = tot_ms, scores
+    value = scores_all / (tot_ms_max / 1e3)
+
+    # End to end through the public C ABI with host buffers (pinned): H2D of W and X and D2H
+    # of every output inside the timed region, wall clock around a synchronizing call.
+    e2e_times = []
+    h_out = None
+    for i in range(args.e2e_steps + 1):
+        t0 = time.perf_counter()
+        h_out = P.crvq_quantize_layer(W_h, X_h, cfg_r, out=h_out)
+        dt = time.perf_counter() - t0
+        if i > 0:
+            e2e_times.append(dt)
+    e2e_scores = h_out.report["scores"]
+    h2d = W_h.numel() * 4 + X_h.numel() * 4
+    d2h = sum(t.numel() * t.element_size() for t in
+              [h_out.perm, h_out.C_base, h_out.codes_base, h_out.C_ext, h_out.codes_ext,
+               h_out.W_hat, h_out.importance] if t is not None) + 48
+    e2e_val = ws * e2e_scores / statistics.mean(e2e_times)
+
+    if rank != 0:
+        return
+    peaks, peak_src = load_peaks()
+    props = torch.cuda.get_device_properties(dev)
+    nsm = props.multi_processor_count
+    ks = sorted(kstats, key=lambda k: -k["ms"])
+    total_k = sum(k["ms"] for k in ks) or 1.0
+    top = ks[0]
+    # The dominant kernel is the SIMT fp32 score contraction: bound by the FP32 pipe.
+    fp32_peak = nsm * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+    enc = next((k for k in ks if k["name"] == "encode_argmin"), top)
+    achieved = enc["units"] * 16.0 / (enc["ms"] / 1e3) / 1e12
+    roof = {"kernel": enc["name"], "bound": "alu", "achieved": achieved, "peak": fp32_peak,
+            "unit": "TFLOP/s", "frac": achieved / fp32_peak, "traffic": None,
+            "peak_source": f"{nsm} SMs x 128 FP32 lanes x 2 flop x "
+                           f"{peaks.get('sm_max_mhz', 2070.0):.0f} MHz (sm_max_mhz, {peak_src})",
+            "work": "16 flop per scored (vector, codeword) pair",
+            "avg_launch_ms": enc["ms"] / max(enc["launches"], 1)}
+    line = {
+        "metric": METRIC, "value": value, "unit": "scores/s", "n_gpus": ws,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": tot_ms_max / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": DATA, "config": config_dict(cfg),
+        "layer_time_s": tot_ms_max / args.steps / 1e3,
+        "losses": {k: out.report[k] for k in ("loss_pre", "loss_block", "loss_crit",
+                                              "loss_full")},
+        "roofline": roof,
+        "e2e": {"value": e2e_val, "unit": "scores/s", "h2d_bytes_per_step": int(h2d),
+                "d2h_bytes_per_step": int(d2h), "ms_per_step": 1e3 * statistics.mean(e2e_times)},
+        "gpu_launches": int(launches),
+        "kernels": [{"name": k["name"], "launches": k["launches"], "ms": k["ms"],
+                     "share": k["ms"] / total_k} for k in ks[:12]],
+        "clocks": clk,
+    }
+    if ws == 1 and not args.no_cpu_baseline:
+        rows = args.ref_rows
+        v, wall, cores = cpu_oracle_sample(cfg_r, rows, Xn)
+        line["cpu_baseline"] = {"value": v, "unit": "scores/s", "cores": cores, "kind": "oracle",
+                                "sample": f"whole schedule on rows 0..{rows - 1} of W "
+                                          f"(full X), {wall:.1f} s"}
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,278 @@
+/*
+ * crvq.h - C ABI of the GB300 (sm_103a) CRVQ code-search library (libcrvq.so).
+ *
+ * CRVQ (Channel-Relaxed Vector Quantization, arXiv 2412.09282) quantizes a weight matrix W
+ * (M x N) by vector quantization of its length-d row segments, with one base codebook over
+ * all vectors and extra "extended" codebooks fitted additively on the vectors of a small set
+ * of reordered critical channels (Sec. 4, Alg. 1). This library runs the data-parallel hot
+ * path of that procedure on one GPU: the Hessian proxy, channel scoring and reordering, the
+ * vector x codeword score contraction with top-B (beam) selection, the codebook
+ * least-squares update and the error evaluation.
+ *
+ * Conventions (every call):
+ *  - Arrays are device pointers owned by the caller unless a parameter says "host". The
+ *    library keeps no pointer after the call returns. Row-major; fp32 unless stated.
+ *  - Calls enqueue work on `stream` and return without waiting, except calls that return a
+ *    value in host memory (their documentation says so): those synchronize `stream`.
+ *  - Scratch memory is taken with stream-ordered cudaMallocAsync/cudaFreeAsync on `stream`.
+ *  - Arguments are validated before any launch: a bad argument returns
+ *    CRVQ_ERR_INVALID_ARG, an unsupported size CRVQ_ERR_UNSUPPORTED, and nothing is
+ *    enqueued. crvq_last_error() then describes the problem (per host thread).
+ *  - Faults found on the device (an index out of range, a non-SPD normal matrix, a bounded
+ *    wait that ran out) set a per-device error word instead of trapping; crvq_sync() reports
+ *    and clears it.
+ *  - d (vector length) must be 8 in this version; larger d returns CRVQ_ERR_UNSUPPORTED.
+ *
+ * Vector sets. The encode/update/init calls work on a vector set: an M x (G_sub*d) block
+ * T of a row-major matrix with leading dimension ldT (floats). Vector (i, g), 0 <= i < M,
+ * 0 <= g < G_sub, is T[i*ldT + g*d .. + d) (the partition S of Sec. 3.1), and is scored with
+ * the d x d Hessian block H_blocks[g] (pass H_blocks already offset to the set's first group).
+ *
+ * Codebooks. A codebook of a vector set covers the groups g < G_cov (a prefix of the set):
+ * the base codebook covers every group, an extended codebook only the first G_c groups,
+ * where the reordered critical channels sit (Sec. 4.3, Fig. 2). The reconstruction of vector
+ * (i, g) is the sum, over the codebooks that cover g, of C[code(i, g)] (additive VQ).
+ *
+ * Score. Vector t against reconstruction r: err = (t - r)^T H_g (t - r), the block-diagonal
+ * part of the Alg. 1 loss ||W X - W_enc X||^2 written with H = X^T X / n + delta I. With
+ * H_g = c I it is the squared L2 distance of Sec. 3.1 Eq. (2)-(3). Code indices are decided
+ * exactly: scores are computed in fp32 with a rigorous error bound and any decision closer
+ * than that bound is re-taken in fp64, so codes equal those of an fp64 evaluation except
+ * for ties at fp64 rounding level (ties go to the smaller index / earlier tuple).
+ */
+#ifndef CRVQ_H
+#define CRVQ_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* crvq_stream_t; /* a cudaStream_t; NULL = the legacy default stream */
+typedef int32_t crvq_status;
+
+enum {
+  CRVQ_OK = 0,
+  CRVQ_ERR_INVALID_ARG = -1, /* a pointer, size or option is out of its documented range */
+  CRVQ_ERR_UNSUPPORTED = -2, /* a valid request this build does not implement (e.g. d != 8) */
+  CRVQ_ERR_CUDA = -3,        /* a CUDA runtime call failed */
+  CRVQ_ERR_NOMEM = -4,       /* device memory allocation failed */
+  CRVQ_ERR_TIMEOUT = -5,     /* a bounded device-side wait ran out */
+  CRVQ_ERR_NUMERIC = -6,     /* non-finite input or a normal matrix that is not SPD */
+  CRVQ_ERR_DEVICE = -7       /* a device-side index check failed (access skipped) */
+};
+
+/* Importance modes (Sec. 4.1; Table 2 "Reorder Strategy"). */
+enum { CRVQ_IMPORTANCE_WA = 0, CRVQ_IMPORTANCE_W_ONLY = 1, CRVQ_IMPORTANCE_RANDOM = 2 };
+
+/* One codebook of a vector set (see "Codebooks" above). */
+typedef struct crvq_codebook {
+  const float* C; /* K x d codewords (device) */
+  int32_t K;      /* number of codewords, 1 <= K <= 65536 */
+  int32_t _pad;
+  int32_t* codes; /* device; code of vector (i, g) is codes[i * ld + g] for g < G_cov */
+  int64_t ld;     /* leading dimension of codes, ld >= G_cov */
+  int64_t G_cov;  /* the codebook covers groups 0 <= g < G_cov of the set, G_cov <= G_sub */
+} crvq_codebook;
+
+/* Message describing the last failure on the calling host thread ("" when none). */
+const char* crvq_last_error(void);
+
+/* Waits for `stream`, then returns and clears the device error word of the current device:
+ * CRVQ_OK, CRVQ_ERR_DEVICE, CRVQ_ERR_NUMERIC or CRVQ_ERR_TIMEOUT (or CRVQ_ERR_CUDA). */
+crvq_status crvq_sync(crvq_stream_t stream);
+
+/* Library build string (compiler, architecture). Host memory, static. */
+const char* crvq_version(void);
+
+/* Per-kernel timing. Between crvq_profile_begin() and crvq_profile_end(), every kernel the
+ * library launches is bracketed by CUDA events recorded on the stream it is launched on.
+ * crvq_profile_end() waits for them and writes one entry per kernel name (host memory,
+ * at most `cap` entries, *n_stats set to the number written). `units` is the algorithmic
+ * work the launches were given (scores for the encode kernels, vectors for the update,
+ * multiply-adds for the GEMMs, bytes for the streaming kernels). */
+typedef struct crvq_kernel_stat {
+  char name[64];
+  int64_t launches;
+  double ms;     /* summed event time */
+  double units;  /* summed algorithmic work */
+} crvq_kernel_stat;
+
+crvq_status crvq_profile_begin(void);
+crvq_status crvq_profile_end(crvq_kernel_stat* stats, int32_t cap, int32_t* n_stats);
+
+/* Number of kernels this library has launched in this process (all devices). */
+int64_t crvq_launch_count(void);
+
+/*
+ * S1. Hessian proxy (Alg. 1 "Require: XX^T"; App. A.2, where X is N x O and the proxy XX^T).
+ * Here X is n_tok x N (row = token) and H = X^T X / n_tok + delta I with
+ * delta = damp_rel * mean_i (X^T X / n_tok)_ii (damping is not in the paper; it keeps the
+ * least-squares codebook solves well posed).
+ *   X        [n_tok x N] calibration activations.
+ *   H        [N x N] out, symmetric.
+ *   xsq      [N] out, undamped diagonal (X^T X / n_tok)_ii, used by the W-A importance.
+ *   H_blocks [(N/d) x d x d] out or NULL: diagonal blocks of H in the original channel order.
+ *   delta    [1] out or NULL: the damping added to the diagonal.
+ * Requires n_tok >= 1, N >= 1, N % d == 0, damp_rel >= 0 and finite.
+ */
+crvq_status crvq_hessian(const float* X, int64_t n_tok, int64_t N, int32_t d, float damp_rel,
+                         float* H, float* xsq, float* H_blocks, float* delta,
+                         crvq_stream_t stream);
+
+/*
+ * S3. Channel importance and reordering (Alg. 1 ComputeImportance, ReorderChannels;
+ * Sec. 4.1-4.2; App. A.2).
+ *   mode W-A:    I_i = 1/2 * xsq_i * max_j (W_ji - W_pre_ji)^2 (App. A.2 form; W_pre is the
+ *                prequantized W, original order).
+ *   mode W-only: I_i = max_j W_ji^2 (Sec. 4.1). W_pre and xsq may be NULL.
+ *   mode random: I_i = (SplitMix64(seed, i) >> 40) * 2^-24 (Table 2 "Random").
+ * perm sorts channels by I descending, ties by original index (perm[new] = old).
+ *   perm        [N] int32 out.      importance [N] out or NULL.
+ *   W_sorted    [M x N] out, W_sorted[:, p] = W[:, perm[p]].
+ *   H_blocks    [(N/d) x d x d] out, H_blocks[g][a][b] = H[perm[g d + a]][perm[g d + b]].
+ *   n_crit_groups  host out: G_c = min(N/d, ceil(crit_frac * N / d)) (Sec. 4.3 ratio lambda,
+ *               rounded up to whole groups of d channels).
+ * Requires 0 <= crit_frac <= 1, N % d == 0, N <= 49152.
+ */
+crvq_status crvq_select_reorder_channels(const float* W, int64_t M, int64_t N, int32_t d,
+                                         const float* W_pre, const float* xsq, const float* H,
+                                         float crit_frac, int32_t mode, uint64_t seed,
+                                         int32_t* perm, float* importance, float* W_sorted,
+                                         float* H_blocks, int64_t* n_crit_groups,
+                                         crvq_stream_t stream);
+
+/*
+ * k-means initial codebook (Eq. kmeans in Sec. 3.1; Alg. 1 KMeansCodebook). Draws one vector
+ * from each of K equal strata of the vector index range v = i * G_sub + g:
+ * v_k = floor(k n / K) + SplitMix64(seed, k) mod (floor((k+1) n / K) - floor(k n / K)),
+ * n = M * G_sub; codeword k is that vector minus the reconstruction of the `fixed`
+ * codebooks (residual, for extended codebooks), evaluated in fp64 and rounded once.
+ *   fixed  host array of n_fixed codebooks (may be NULL when n_fixed == 0).
+ *   C_out  [K x d] out.     Requires 1 <= K <= min(n, 65536).
+ */
+crvq_status crvq_kmeans_init(const float* T, int64_t ldT, int64_t M, int64_t G_sub, int32_t d,
+                             const crvq_codebook* fixed, int32_t n_fixed, int32_t K,
+                             uint64_t seed, float* C_out, crvq_stream_t stream);
+
+/*
+ * Encode / beam search (Sec. 3.1 Eq. (2)-(3); Alg. 1 VectorQuant, BeamSearchOptimize).
+ * Codebooks 0..n_fixed-1 are fixed (their codes are read); codebooks n_fixed..n_cb-1 are
+ * searched and their codes written. For each vector the target is t minus the fixed
+ * reconstruction; the searched codebooks that cover the vector are taken in order as beam
+ * stages: every kept partial tuple is extended by every codeword and the B best are kept,
+ * ordered by (err, parent rank, codeword index). The best tuple of the last stage is written.
+ * With one searched stage this is the arg-min assignment step of k-means.
+ *   keep_if_better  nonzero: the searched codes hold a tuple on entry, which is kept when
+ *                   its err is strictly smaller than the beam's best.
+ *   vec_err         [M x G_sub] out or NULL: err of the written tuple (fp64, rounded).
+ * Requires 1 <= B <= 16, 0 <= n_fixed < n_cb <= 8.
+ */
+crvq_status crvq_encode_beam(const float* T, int64_t ldT, int64_t M, int64_t G_sub, int32_t d,
+                             const float* H_blocks, const crvq_codebook* cbs, int32_t n_cb,
+                             int32_t n_fixed, int32_t B, int32_t keep_if_better,
+                             float* vec_err, crvq_stream_t stream);
+
+/*
+ * Least-squares codebook update (k-means update step; Alg. 1 FineTuneCodebook read as the
+ * closed-form minimiser). Codebook `which` is refitted with all others fixed: the members v
+ * of cluster k (vectors with code k, g < G_cov) have targets tau_v = t_v - sum over the other
+ * covering codebooks of C[code]; c_k solves (sum_v H_{g_v}) c = sum_v H_{g_v} tau_v
+ * (Cholesky, fp64 sums in a fixed order, so results are reproducible). Empty clusters keep
+ * their codeword.   C_out [K x d] out (may alias cbs[which].C).
+ *   counts [K] int32 out or NULL: cluster sizes.
+ */
+crvq_status crvq_update_codebook(const float* T, int64_t ldT, int64_t M, int64_t G_sub,
+                                 int32_t d, const float* H_blocks, const crvq_codebook* cbs,
+                                 int32_t n_cb, int32_t which, float* C_out, int32_t* counts,
+                                 crvq_stream_t stream);
+
+/*
+ * S7. Reconstruction, reverse reorder and losses (Alg. 1 QuantLoss; Sec. 4.3 "restored to
+ * their original order"). The set is all of W_sorted (M x N, G = N/d groups).
+ *   perm         [N] or NULL (identity).
+ *   W_hat        [M x N] out or NULL: the reconstruction in the original channel order.
+ *   X            [n_tok x N] or NULL (then losses[2] = NaN).
+ *   losses       HOST out [3]: loss_block = sum over vectors of err; loss_crit = the same
+ *                over groups g < n_crit_groups; loss_full = ||(W - W_hat) X^T||^2 / n_tok
+ *                + damp_delta ||W - W_hat||^2 = tr(dW H dW^T). Synchronizes `stream`.
+ */
+crvq_status crvq_reconstruct_error(const float* W_sorted, int64_t M, int64_t N, int32_t d,
+                                   const float* H_blocks, const int32_t* perm,
+                                   const crvq_codebook* cbs, int32_t n_cb,
+                                   int64_t n_crit_groups, const float* X, int64_t n_tok,
+                                   double damp_delta, float* W_hat, double* losses,
+                                   crvq_stream_t stream);
+
+/* Average bits per weight (Sec. 3.2 Eq. (bitwidth); App. A.1): e-bit codes for all M N / d
+ * vectors, plus m-1 extended codebooks on the lambda fraction, plus m codebooks of 2^e
+ * fp16 vectors of length d, plus (include_perm) a 16-bit reorder index per channel. */
+double crvq_avg_bits(int32_t e, int32_t d, int32_t m, double lambda, int64_t M, int64_t N,
+                     int32_t include_perm);
+
+/* G_c = min(N/d, ceil(crit_frac * N / d)) (0 when crit_frac == 0). */
+int64_t crvq_n_crit_groups(int64_t N, int32_t d, float crit_frac);
+
+/* Hyper-parameters of one matrix (Alg. 1 inputs m, lambda, epsilon; Sec. 3.2 e, d). */
+typedef struct crvq_config {
+  int32_t d;               /* vector length (8) */
+  int32_t K_base;          /* base codebook size 2^e */
+  int32_t n_ext;           /* extended codebooks (m - 1), 0..7 */
+  int32_t K_ext;           /* extended codebook size */
+  float crit_frac;         /* lambda */
+  int32_t B;               /* beam width of the refinement re-encode, 1..16 */
+  int32_t kmeans_iters;    /* Lloyd iterations per codebook fit */
+  int32_t refine_rounds;   /* maximum FineTuneCodebook + BeamSearch rounds */
+  float eps_rel;           /* stop refining when loss_block > (1 - eps_rel) * previous */
+  float damp_rel;          /* Hessian damping, relative to the mean diagonal */
+  int32_t importance_mode; /* CRVQ_IMPORTANCE_* */
+  int32_t _pad;
+  uint64_t seed;
+} crvq_config;
+
+/* Outputs of one matrix. Pointers may be device or host memory (host buffers are staged
+ * through the device inside the call). */
+typedef struct crvq_layer_outputs {
+  int32_t* perm;       /* [N] channel order, perm[new] = old */
+  float* C_base;       /* [K_base x d] */
+  int32_t* codes_base; /* [M x N/d], vector (i, g) in the sorted order */
+  float* C_ext;        /* [n_ext x K_ext x d] */
+  int32_t* codes_ext;  /* [n_ext x M x G_c] */
+  float* W_hat;        /* [M x N] reconstruction in the original order, or NULL */
+  float* importance;   /* [N] or NULL */
+} crvq_layer_outputs;
+
+typedef struct crvq_layer_report {
+  double loss_pre;       /* loss_block of the prequantized W (original order) */
+  double loss_block;     /* final losses (see crvq_reconstruct_error) */
+  double loss_crit;
+  double loss_full;
+  double loss_before_refine;
+  double scores;         /* (hypothesis, codeword) pairs scored by the encode passes */
+  int64_t n_crit_groups;
+  int32_t refine_rounds_done;
+  int32_t _pad;
+} crvq_layer_report;
+
+/*
+ * One weight matrix through Alg. 1 lines 3-17 (everything but block / end-to-end fine-tuning):
+ * S1 Hessian; S2 prequantize (k-means + encode in the original order); S3 importance and
+ * reorder; S4 base codebook (k-means over all vectors); S5 each extended codebook (k-means
+ * on the critical residual, greedy encode); S6 up to refine_rounds rounds of
+ * least-squares updates of every codebook followed by a joint beam re-encode (keep-if-better);
+ * S7 losses and the reconstruction in the original order. Per-phase seeds are
+ * SplitMix64(cfg->seed, phase * 1024 + codebook) with phase 1 = prequantize, 2 = base,
+ * 3 = extended, 4 = random importance. W [M x N], X [n_tok x N] may be host or device
+ * pointers. Synchronizes `stream` (the report is host memory).
+ */
+crvq_status crvq_quantize_layer(const float* W, const float* X, int64_t M, int64_t N,
+                                int64_t n_tok, const crvq_config* cfg,
+                                const crvq_layer_outputs* out, crvq_layer_report* report,
+                                crvq_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CRVQ_H */

@@ -1,0 +1,601 @@
+// C ABI of libcrvq: argument validation, status / error-word handling and the per-matrix
+// schedule (Alg. 1 lines 3-17) that strings the kernels together on one stream.
+#include <atomic>
+#include <cmath>
+#include <cstring>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace crvq {
+
+// ------------------------------------------------------------------------- status helpers
+static thread_local std::string t_last_error;
+
+void set_last_error(const char* fmt, ...) {
+  char buf[1024];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  t_last_error = buf;
+}
+
+crvq_status fail(crvq_status st, const char* fmt, ...) {
+  char buf[1024];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof(buf), fmt, ap);
+  va_end(ap);
+  t_last_error = buf;
+  return st;
+}
+
+void clear_last_error() { t_last_error.clear(); }
+
+namespace {
+std::mutex g_mu;
+std::vector<unsigned*> g_err_words;  // per device
+std::vector<int> g_sm;               // per device
+}  // namespace
+
+crvq_status device_error_word(unsigned** out) {
+  int dev = 0;
+  CRVQ_CUDA(cudaGetDevice(&dev));
+  std::lock_guard<std::mutex> lk(g_mu);
+  if ((int)g_err_words.size() <= dev) g_err_words.resize(dev + 1, nullptr);
+  if (!g_err_words[dev]) {
+    unsigned* p = nullptr;
+    CRVQ_CUDA(cudaMalloc(&p, sizeof(unsigned)));
+    CRVQ_CUDA(cudaMemset(p, 0, sizeof(unsigned)));
+    g_err_words[dev] = p;
+  }
+  *out = g_err_words[dev];
+  return CRVQ_OK;
+}
+
+int sm_count() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+  std::lock_guard<std::mutex> lk(g_mu);
+  if ((int)g_sm.size() <= dev) g_sm.resize(dev + 1, 0);
+  if (!g_sm[dev]) {
+    int n = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    g_sm[dev] = n > 0 ? n : 1;
+  }
+  return g_sm[dev];
+}
+
+// ------------------------------------------------------------------------- launch stats
+namespace {
+std::atomic<long long> g_launches{0};
+std::atomic<bool> g_prof{false};
+std::mutex g_pmu;
+struct ProfRec {
+  const char* name;
+  cudaEvent_t a, b;
+  double units;
+};
+std::vector<ProfRec> g_recs;
+}  // namespace
+
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
+ProfScope::ProfScope(const char* name, cudaStream_t s, double units)
+    : name_(name), s_(s), units_(units) {
+  if (g_prof.load(std::memory_order_relaxed)) {
+    if (cudaEventCreate(&a_) != cudaSuccess || cudaEventRecord(a_, s_) != cudaSuccess) {
+      if (a_) cudaEventDestroy(a_);
+      a_ = nullptr;
+      cudaGetLastError();
+    }
+  }
+}
+
+ProfScope::~ProfScope() {
+  if (!a_) return;
+  cudaEvent_t b = nullptr;
+  if (cudaEventCreate(&b) != cudaSuccess || cudaEventRecord(b, s_) != cudaSuccess) {
+    cudaGetLastError();
+    cudaEventDestroy(a_);
+    if (b) cudaEventDestroy(b);
+    return;
+  }
+  std::lock_guard<std::mutex> lk(g_pmu);
+  g_recs.push_back(ProfRec{name_, a_, b, units_});
+}
+
+// ------------------------------------------------------------------------- validation
+static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+static crvq_status check_d(int32_t d) {
+  if (d <= 0) return fail(CRVQ_ERR_INVALID_ARG, "d must be positive (got %d)", d);
+  if (d != kD) return fail(CRVQ_ERR_UNSUPPORTED, "only d = 8 is implemented (got %d)", d);
+  return CRVQ_OK;
+}
+
+static crvq_status check_set(const float* T, int64_t ldT, int64_t M, int64_t G_sub,
+                             const float* Hb) {
+  CRVQ_CHECK_ARG(T != nullptr, "T is NULL");
+  CRVQ_CHECK_ARG(Hb != nullptr, "H_blocks is NULL");
+  CRVQ_CHECK_ARG(M >= 1 && G_sub >= 1, "empty vector set (M=%lld, G_sub=%lld)", (long long)M,
+                 (long long)G_sub);
+  CRVQ_CHECK_ARG(ldT >= G_sub * kD, "ldT (%lld) < G_sub * d (%lld)", (long long)ldT,
+                 (long long)(G_sub * kD));
+  CRVQ_CHECK_ARG(ldT % 4 == 0, "ldT must be a multiple of 4 floats");
+  CRVQ_CHECK_ARG(aligned16(T) && aligned16(Hb), "T and H_blocks must be 16-byte aligned");
+  CRVQ_CHECK_ARG(M * G_sub < (int64_t)1 << 31, "too many vectors in one set");
+  return CRVQ_OK;
+}
+
+static crvq_status make_cblist(const crvq_codebook* cbs, int32_t n_cb, int64_t G_sub,
+                               bool need_codes_all, CbList* out) {
+  CRVQ_CHECK_ARG(n_cb >= 0 && n_cb <= kMaxCodebooks, "n_cb must be in [0, %d]", kMaxCodebooks);
+  CRVQ_CHECK_ARG(n_cb == 0 || cbs != nullptr, "codebook array is NULL");
+  out->n = n_cb;
+  for (int s = 0; s < n_cb; ++s) {
+    const crvq_codebook& c = cbs[s];
+    CRVQ_CHECK_ARG(c.C != nullptr && aligned16(c.C), "codebook %d: C is NULL or not 16-byte aligned", s);
+    CRVQ_CHECK_ARG(c.K >= 1 && c.K <= 65536, "codebook %d: K must be in [1, 65536]", s);
+    CRVQ_CHECK_ARG(c.G_cov >= 0 && c.G_cov <= G_sub, "codebook %d: G_cov out of [0, G_sub]", s);
+    CRVQ_CHECK_ARG(c.G_cov == 0 || c.ld >= c.G_cov, "codebook %d: ld < G_cov", s);
+    if (need_codes_all && c.G_cov > 0)
+      CRVQ_CHECK_ARG(c.codes != nullptr, "codebook %d: codes is NULL", s);
+    out->cb[s] = CbView{c.C, c.codes, c.ld, c.G_cov, c.K};
+  }
+  return CRVQ_OK;
+}
+
+static bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+}  // namespace crvq
+
+using namespace crvq;
+
+#define CRVQ_STR_(x) #x
+#define CRVQ_XSTR(x) CRVQ_STR_(x)
+
+// =========================================================================== C entry points
+extern "C" {
+
+const char* crvq_last_error(void) { return t_last_error.c_str(); }
+
+const char* crvq_version(void) {
+  return "libcrvq (sm_103a, CUDA " CRVQ_XSTR(__CUDACC_VER_MAJOR__) "." CRVQ_XSTR(__CUDACC_VER_MINOR__) ")";
+}
+
+int64_t crvq_launch_count(void) { return (int64_t)g_launches.load(); }
+
+crvq_status crvq_profile_begin(void) {
+  std::lock_guard<std::mutex> lk(g_pmu);
+  for (auto& r : g_recs) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  g_recs.clear();
+  g_prof.store(true);
+  return CRVQ_OK;
+}
+
+crvq_status crvq_profile_end(crvq_kernel_stat* stats, int32_t cap, int32_t* n_stats) {
+  g_prof.store(false);
+  std::vector<ProfRec> recs;
+  {
+    std::lock_guard<std::mutex> lk(g_pmu);
+    recs.swap(g_recs);
+  }
+  std::vector<crvq_kernel_stat> agg;
+  crvq_status st = CRVQ_OK;
+  for (auto& r : recs) {
+    float ms = 0.f;
+    if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess) {
+      st = fail(CRVQ_ERR_CUDA, "profiling event failed: %s", cudaGetErrorString(cudaGetLastError()));
+    }
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+    size_t j = 0;
+    for (; j < agg.size(); ++j)
+      if (strncmp(agg[j].name, r.name, sizeof(agg[j].name)) == 0) break;
+    if (j == agg.size()) {
+      crvq_kernel_stat z;
+      memset(&z, 0, sizeof(z));
+      strncpy(z.name, r.name, sizeof(z.name) - 1);
+      agg.push_back(z);
+    }
+    agg[j].launches += 1;
+    agg[j].ms += ms;
+    agg[j].units += r.units;
+  }
+  const int n = (int)std::min<size_t>(agg.size(), cap > 0 ? (size_t)cap : 0);
+  for (int i = 0; i < n; ++i) stats[i] = agg[i];
+  if (n_stats) *n_stats = n;
+  return st;
+}
+
+crvq_status crvq_sync(crvq_stream_t stream) {
+  CRVQ_CUDA(cudaStreamSynchronize((cudaStream_t)stream));
+  unsigned* w = nullptr;
+  CRVQ_TRY(device_error_word(&w));
+  unsigned h = 0;
+  CRVQ_CUDA(cudaMemcpy(&h, w, sizeof(unsigned), cudaMemcpyDeviceToHost));
+  if (h) {
+    CRVQ_CUDA(cudaMemset(w, 0, sizeof(unsigned)));
+    if (h & ERRBIT_TIMEOUT) return fail(CRVQ_ERR_TIMEOUT, "a bounded device wait ran out");
+    if (h & ERRBIT_INDEX) return fail(CRVQ_ERR_DEVICE, "a device-side index check failed");
+    return fail(CRVQ_ERR_NUMERIC, "non-finite value or non-SPD normal matrix on the device");
+  }
+  return CRVQ_OK;
+}
+
+crvq_status crvq_hessian(const float* X, int64_t n_tok, int64_t N, int32_t d, float damp_rel,
+                         float* H, float* xsq, float* H_blocks, float* delta,
+                         crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_TRY(check_d(d));
+  CRVQ_CHECK_ARG(X && H && xsq, "X, H and xsq must not be NULL");
+  CRVQ_CHECK_ARG(n_tok >= 1 && N >= 1 && N % d == 0, "need n_tok >= 1, N >= 1, N %% d == 0");
+  CRVQ_CHECK_ARG(std::isfinite(damp_rel) && damp_rel >= 0.f, "damp_rel must be finite, >= 0");
+  CRVQ_CHECK_ARG(aligned16(X), "X must be 16-byte aligned");
+  return launch_hessian(X, n_tok, N, d, damp_rel, H, xsq, H_blocks, delta,
+                        (cudaStream_t)stream);
+}
+
+int64_t crvq_n_crit_groups(int64_t N, int32_t d, float crit_frac) {
+  if (d <= 0 || N <= 0 || !(crit_frac > 0.f)) return 0;
+  const int64_t G = N / d;
+  const double x = std::ceil((double)crit_frac * (double)N / (double)d - 1e-12);
+  return std::min<int64_t>(G, (int64_t)x);
+}
+
+crvq_status crvq_select_reorder_channels(const float* W, int64_t M, int64_t N, int32_t d,
+                                         const float* W_pre, const float* xsq, const float* H,
+                                         float crit_frac, int32_t mode, uint64_t seed,
+                                         int32_t* perm, float* importance, float* W_sorted,
+                                         float* H_blocks, int64_t* n_crit_groups,
+                                         crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_TRY(check_d(d));
+  CRVQ_CHECK_ARG(W && H && perm && W_sorted && H_blocks, "required pointer is NULL");
+  CRVQ_CHECK_ARG(M >= 1 && N >= 1 && N % d == 0, "need M >= 1, N >= 1, N %% d == 0");
+  CRVQ_CHECK_ARG(N <= 49152, "N must be <= 49152");
+  CRVQ_CHECK_ARG(crit_frac >= 0.f && crit_frac <= 1.f, "crit_frac must be in [0, 1]");
+  CRVQ_CHECK_ARG(mode >= 0 && mode <= 2, "unknown importance mode %d", mode);
+  if (mode == CRVQ_IMPORTANCE_WA) CRVQ_CHECK_ARG(W_pre && xsq, "W-A mode needs W_pre and xsq");
+  CRVQ_CHECK_ARG(aligned16(W) && aligned16(W_sorted) && (!W_pre || aligned16(W_pre)),
+                 "W, W_pre and W_sorted must be 16-byte aligned");
+  if (n_crit_groups) *n_crit_groups = crvq_n_crit_groups(N, d, crit_frac);
+  return launch_select_reorder(W, M, N, d, W_pre, xsq, H, mode, seed, perm, importance,
+                               W_sorted, H_blocks, (cudaStream_t)stream);
+}
+
+crvq_status crvq_kmeans_init(const float* T, int64_t ldT, int64_t M, int64_t G_sub, int32_t d,
+                             const crvq_codebook* fixed, int32_t n_fixed, int32_t K,
+                             uint64_t seed, float* C_out, crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_TRY(check_d(d));
+  CRVQ_CHECK_ARG(T && C_out, "T and C_out must not be NULL");
+  CRVQ_CHECK_ARG(M >= 1 && G_sub >= 1 && ldT >= G_sub * d && ldT % 4 == 0 && aligned16(T),
+                 "bad vector set");
+  CRVQ_CHECK_ARG(K >= 1 && K <= 65536 && (int64_t)K <= M * G_sub,
+                 "K must be in [1, min(65536, M * G_sub)]");
+  CbList fl;
+  CRVQ_TRY(make_cblist(fixed, n_fixed, G_sub, true, &fl));
+  SetView set{T, ldT, M, G_sub, nullptr};
+  return launch_kmeans_init(set, fl, K, seed, C_out, (cudaStream_t)stream);
+}
+
+crvq_status crvq_encode_beam(const float* T, int64_t ldT, int64_t M, int64_t G_sub, int32_t d,
+                             const float* H_blocks, const crvq_codebook* cbs, int32_t n_cb,
+                             int32_t n_fixed, int32_t B, int32_t keep_if_better,
+                             float* vec_err, crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_TRY(check_d(d));
+  CRVQ_TRY(check_set(T, ldT, M, G_sub, H_blocks));
+  CRVQ_CHECK_ARG(n_cb >= 1 && n_cb <= kMaxCodebooks, "n_cb must be in [1, %d]", kMaxCodebooks);
+  CRVQ_CHECK_ARG(n_fixed >= 0 && n_fixed < n_cb, "n_fixed must be in [0, n_cb)");
+  CRVQ_CHECK_ARG(B >= 1, "B must be >= 1");
+  if (B > 16) return fail(CRVQ_ERR_UNSUPPORTED, "beam width B > 16 is not implemented");
+  CbList cl;
+  CRVQ_TRY(make_cblist(cbs, n_cb, G_sub, true, &cl));
+  SetView set{T, ldT, M, G_sub, H_blocks};
+  return launch_encode_beam(set, cl, n_fixed, B, keep_if_better != 0, vec_err, nullptr,
+                            (cudaStream_t)stream);
+}
+
+crvq_status crvq_update_codebook(const float* T, int64_t ldT, int64_t M, int64_t G_sub,
+                                 int32_t d, const float* H_blocks, const crvq_codebook* cbs,
+                                 int32_t n_cb, int32_t which, float* C_out, int32_t* counts,
+                                 crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_TRY(check_d(d));
+  CRVQ_TRY(check_set(T, ldT, M, G_sub, H_blocks));
+  CRVQ_CHECK_ARG(n_cb >= 1 && which >= 0 && which < n_cb, "which must be in [0, n_cb)");
+  CRVQ_CHECK_ARG(C_out != nullptr, "C_out is NULL");
+  CbList cl;
+  CRVQ_TRY(make_cblist(cbs, n_cb, G_sub, true, &cl));
+  SetView set{T, ldT, M, G_sub, H_blocks};
+  return launch_update_codebook(set, cl, which, C_out, counts, (cudaStream_t)stream);
+}
+
+crvq_status crvq_reconstruct_error(const float* W_sorted, int64_t M, int64_t N, int32_t d,
+                                   const float* H_blocks, const int32_t* perm,
+                                   const crvq_codebook* cbs, int32_t n_cb,
+                                   int64_t n_crit_groups, const float* X, int64_t n_tok,
+                                   double damp_delta, float* W_hat, double* losses,
+                                   crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_TRY(check_d(d));
+  CRVQ_CHECK_ARG(N >= 1 && N % d == 0, "N must be a positive multiple of d");
+  CRVQ_TRY(check_set(W_sorted, N, M, N / d, H_blocks));
+  CRVQ_CHECK_ARG(losses != nullptr, "losses is NULL");
+  CRVQ_CHECK_ARG(N <= 49152, "N must be <= 49152");
+  CRVQ_CHECK_ARG(n_crit_groups >= 0 && n_crit_groups <= N / d, "n_crit_groups out of range");
+  CRVQ_CHECK_ARG(!X || n_tok >= 1, "n_tok must be >= 1 when X is given");
+  CRVQ_CHECK_ARG(!W_hat || aligned16(W_hat), "W_hat must be 16-byte aligned");
+  CbList cl;
+  CRVQ_TRY(make_cblist(cbs, n_cb, N / d, true, &cl));
+  cudaStream_t s = (cudaStream_t)stream;
+  Scratch mem;
+  CRVQ_TRY(mem.alloc(3 * sizeof(double), s));
+  CRVQ_TRY(launch_reconstruct_error(W_sorted, M, N, H_blocks, perm, cl, n_crit_groups, X, n_tok,
+                                    damp_delta, nullptr, W_hat, mem.as<double>(), s));
+  CRVQ_CUDA(cudaMemcpyAsync(losses, mem.as<double>(), 3 * sizeof(double),
+                            cudaMemcpyDeviceToHost, s));
+  CRVQ_CUDA(cudaStreamSynchronize(s));
+  return CRVQ_OK;
+}
+
+double crvq_avg_bits(int32_t e, int32_t d, int32_t m, double lambda, int64_t M, int64_t N,
+                     int32_t include_perm) {
+  if (d <= 0 || M <= 0 || N <= 0 || m < 1 || e < 0) return std::nan("");
+  const double nvec = (double)M * (double)N / (double)d;
+  double bits = nvec * e + (double)(m - 1) * lambda * nvec * e +
+                (double)m * std::ldexp(1.0, e) * d * 16.0;
+  if (include_perm) bits += 16.0 * (double)N;
+  return bits / ((double)M * (double)N);
+}
+
+}  // extern "C"
+
+// ------------------------------------------------------------------------- layer schedule
+namespace {
+
+struct Buf {
+  Scratch s;
+  template <class T>
+  crvq_status get(T** p, size_t count, cudaStream_t st) {
+    CRVQ_TRY(s.alloc(count * sizeof(T), st));
+    *p = s.as<T>();
+    return CRVQ_OK;
+  }
+};
+
+uint64_t phase_seed(uint64_t seed, int phase, int cb) {
+  return splitmix64(seed, (uint64_t)phase * 1024u + (uint64_t)cb);
+}
+
+// Lloyd iterations for the last codebook of `cbs` (all earlier ones fixed), then a final
+// encode: T x (encode, LS update) + encode.
+crvq_status lloyd(const SetView& set, CbList cbs, int iters, double* scores, cudaStream_t s) {
+  const int j = cbs.n - 1;
+  float* C = const_cast<float*>(cbs.cb[j].C);
+  for (int it = 0; it < iters; ++it) {
+    CRVQ_TRY(launch_encode_beam(set, cbs, j, 1, false, nullptr, scores, s));
+    CRVQ_TRY(launch_update_codebook(set, cbs, j, C, nullptr, s));
+  }
+  return launch_encode_beam(set, cbs, j, 1, false, nullptr, scores, s);
+}
+
+template <class T>
+crvq_status to_device(const T* host_or_dev, size_t count, Buf& b, const T** out,
+                      cudaStream_t s) {
+  if (is_device_ptr(host_or_dev)) {
+    *out = host_or_dev;
+    return CRVQ_OK;
+  }
+  T* d = nullptr;
+  CRVQ_TRY(b.get(&d, count, s));
+  CRVQ_CUDA(cudaMemcpyAsync(d, host_or_dev, count * sizeof(T), cudaMemcpyHostToDevice, s));
+  *out = d;
+  return CRVQ_OK;
+}
+
+// Output buffer: the caller's device pointer, or a device staging buffer copied back at the end.
+template <class T>
+struct OutBuf {
+  T* user = nullptr;
+  T* dev = nullptr;
+  size_t count = 0;
+  Buf b;
+  crvq_status init(T* u, size_t n, cudaStream_t s) {
+    user = u;
+    count = n;
+    if (u && is_device_ptr(u)) {
+      dev = u;
+      return CRVQ_OK;
+    }
+    return b.get(&dev, std::max<size_t>(n, 1), s);
+  }
+  crvq_status flush(cudaStream_t s) {
+    if (user && dev != user && count)
+      CRVQ_CUDA(cudaMemcpyAsync(user, dev, count * sizeof(T), cudaMemcpyDeviceToHost, s));
+    return CRVQ_OK;
+  }
+};
+
+}  // namespace
+
+extern "C" {
+
+crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M, int64_t N,
+                                int64_t n_tok, const crvq_config* cfg,
+                                const crvq_layer_outputs* out, crvq_layer_report* report,
+                                crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_CHECK_ARG(cfg && out && report && W_in && X_in, "required pointer is NULL");
+  CRVQ_TRY(check_d(cfg->d));
+  const int d = cfg->d;
+  CRVQ_CHECK_ARG(M >= 1 && N >= 1 && N % d == 0 && n_tok >= 1, "bad matrix shape");
+  CRVQ_CHECK_ARG(N <= 49152, "N must be <= 49152");
+  const int64_t G = N / d;
+  CRVQ_CHECK_ARG(cfg->K_base >= 1 && cfg->K_base <= 65536 && cfg->K_base <= M * G,
+                 "K_base out of range");
+  CRVQ_CHECK_ARG(cfg->n_ext >= 0 && cfg->n_ext <= kMaxCodebooks - 1, "n_ext must be in [0, 7]");
+  CRVQ_CHECK_ARG(cfg->crit_frac >= 0.f && cfg->crit_frac <= 1.f, "crit_frac must be in [0, 1]");
+  CRVQ_CHECK_ARG(cfg->B >= 1 && cfg->B <= 16, "B must be in [1, 16]");
+  CRVQ_CHECK_ARG(cfg->kmeans_iters >= 0 && cfg->refine_rounds >= 0, "negative iteration count");
+  CRVQ_CHECK_ARG(cfg->importance_mode >= 0 && cfg->importance_mode <= 2, "bad importance mode");
+  CRVQ_CHECK_ARG(std::isfinite(cfg->damp_rel) && cfg->damp_rel >= 0.f, "bad damp_rel");
+  const int64_t Gc = crvq_n_crit_groups(N, d, cfg->crit_frac);
+  if (cfg->n_ext > 0) {
+    CRVQ_CHECK_ARG(Gc >= 1, "extended codebooks need at least one critical group");
+    CRVQ_CHECK_ARG(cfg->K_ext >= 1 && cfg->K_ext <= 65536 && cfg->K_ext <= M * Gc,
+                   "K_ext out of range");
+  }
+  CRVQ_CHECK_ARG(out->perm && out->C_base && out->codes_base, "perm, C_base, codes_base needed");
+  CRVQ_CHECK_ARG(cfg->n_ext == 0 || (out->C_ext && out->codes_ext), "C_ext, codes_ext needed");
+  cudaStream_t s = (cudaStream_t)stream;
+  memset(report, 0, sizeof(*report));
+  report->n_crit_groups = Gc;
+  double scores = 0.0;
+
+  Buf bW, bX;
+  const float *W = nullptr, *X = nullptr;
+  CRVQ_TRY(to_device(W_in, (size_t)M * N, bW, &W, s));
+  CRVQ_TRY(to_device(X_in, (size_t)n_tok * N, bX, &X, s));
+
+  OutBuf<int32_t> o_perm, o_codes_base, o_codes_ext;
+  OutBuf<float> o_C_base, o_C_ext, o_W_hat, o_imp;
+  CRVQ_TRY(o_perm.init(out->perm, N, s));
+  CRVQ_TRY(o_C_base.init(out->C_base, (size_t)cfg->K_base * d, s));
+  CRVQ_TRY(o_codes_base.init(out->codes_base, (size_t)M * G, s));
+  CRVQ_TRY(o_C_ext.init(out->C_ext, (size_t)cfg->n_ext * cfg->K_ext * d, s));
+  CRVQ_TRY(o_codes_ext.init(out->codes_ext, (size_t)cfg->n_ext * M * Gc, s));
+  if (out->W_hat) CRVQ_TRY(o_W_hat.init(out->W_hat, (size_t)M * N, s));
+  CRVQ_TRY(o_imp.init(out->importance, N, s));
+
+  Buf bH, bxsq, bHb0, bdelta, bC0, bcodes0, bWpre, bWs, bHb, bloss;
+  float *H, *xsq, *Hb0, *delta, *C0, *Wpre, *Ws, *Hb;
+  int32_t* codes0;
+  double* losses;
+  CRVQ_TRY(bH.get(&H, (size_t)N * N, s));
+  CRVQ_TRY(bxsq.get(&xsq, N, s));
+  CRVQ_TRY(bHb0.get(&Hb0, (size_t)G * d * d, s));
+  CRVQ_TRY(bdelta.get(&delta, 4, s));
+  CRVQ_TRY(bC0.get(&C0, (size_t)cfg->K_base * d, s));
+  CRVQ_TRY(bcodes0.get(&codes0, (size_t)M * G, s));
+  CRVQ_TRY(bWpre.get(&Wpre, (size_t)M * N, s));
+  CRVQ_TRY(bWs.get(&Ws, (size_t)M * N, s));
+  CRVQ_TRY(bHb.get(&Hb, (size_t)G * d * d, s));
+  CRVQ_TRY(bloss.get(&losses, 16, s));
+
+  // S1: Hessian proxy
+  CRVQ_TRY(launch_hessian(X, n_tok, N, d, cfg->damp_rel, H, xsq, Hb0, delta, s));
+  // S2: prequantize in the original order (Alg. 1 line 3)
+  {
+    SetView set{W, N, M, G, Hb0};
+    CbList cl{};
+    cl.n = 1;
+    cl.cb[0] = CbView{C0, codes0, G, G, cfg->K_base};
+    CRVQ_TRY(launch_kmeans_init(set, CbList{}, cfg->K_base,
+                                phase_seed(cfg->seed, 1, 0), C0, s));
+    CRVQ_TRY(lloyd(set, cl, cfg->kmeans_iters, &scores, s));
+    CRVQ_TRY(launch_reconstruct_error(W, M, N, Hb0, nullptr, cl, 0, nullptr, 0, 0.0, nullptr,
+                                      Wpre, losses + 3, s));
+  }
+  // S3: importance and reordering (Alg. 1 lines 4-5)
+  CRVQ_TRY(launch_select_reorder(W, M, N, d, Wpre, xsq, H, cfg->importance_mode,
+                                 phase_seed(cfg->seed, 4, 0), o_perm.dev, o_imp.dev, Ws, Hb, s));
+  // S4: base codebook over all vectors (Alg. 1 lines 6-7)
+  CbList all{};
+  all.n = 1 + cfg->n_ext;
+  all.cb[0] = CbView{o_C_base.dev, o_codes_base.dev, G, G, cfg->K_base};
+  for (int t = 1; t <= cfg->n_ext; ++t)
+    all.cb[t] = CbView{o_C_ext.dev + (size_t)(t - 1) * cfg->K_ext * d,
+                       o_codes_ext.dev + (size_t)(t - 1) * M * Gc, Gc, Gc, cfg->K_ext};
+  const SetView full{Ws, N, M, G, Hb};
+  {
+    CbList cl{};
+    cl.n = 1;
+    cl.cb[0] = all.cb[0];
+    CRVQ_TRY(launch_kmeans_init(full, CbList{}, cfg->K_base, phase_seed(cfg->seed, 2, 0),
+                                o_C_base.dev, s));
+    CRVQ_TRY(lloyd(full, cl, cfg->kmeans_iters, &scores, s));
+  }
+  // S5: extended codebooks on the critical residual (Alg. 1 lines 8-13)
+  if (cfg->n_ext > 0) {
+    const SetView crit{Ws, N, M, Gc, Hb};
+    for (int t = 1; t <= cfg->n_ext; ++t) {
+      CbList cl{};
+      cl.n = t + 1;
+      for (int q = 0; q <= t; ++q) {
+        cl.cb[q] = all.cb[q];
+        cl.cb[q].G_cov = Gc;
+      }
+      CbList fixed{};
+      fixed.n = t;
+      for (int q = 0; q < t; ++q) fixed.cb[q] = cl.cb[q];
+      CRVQ_TRY(launch_kmeans_init(crit, fixed, cfg->K_ext, phase_seed(cfg->seed, 3, t),
+                                  const_cast<float*>(all.cb[t].C), s));
+      CRVQ_TRY(lloyd(crit, cl, cfg->kmeans_iters, &scores, s));
+    }
+  }
+  // S6: least-squares codebook updates + joint beam re-encode (Alg. 1 lines 14-17)
+  CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o_perm.dev, all, Gc, nullptr, 0, 0.0,
+                                    nullptr, nullptr, losses + 6, s));
+  double prev = 0.0;
+  if (cfg->refine_rounds > 1) {
+    CRVQ_CUDA(cudaMemcpyAsync(&prev, losses + 6, sizeof(double), cudaMemcpyDeviceToHost, s));
+    CRVQ_CUDA(cudaStreamSynchronize(s));
+  }
+  int rounds = 0;
+  for (int r = 0; r < cfg->refine_rounds; ++r) {
+    for (int j = 0; j < all.n; ++j)
+      CRVQ_TRY(launch_update_codebook(full, all, j, const_cast<float*>(all.cb[j].C), nullptr, s));
+    CRVQ_TRY(launch_encode_beam(full, all, 0, cfg->B, true, nullptr, &scores, s));
+    ++rounds;
+    if (cfg->refine_rounds > 1 && r + 1 < cfg->refine_rounds) {
+      CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o_perm.dev, all, Gc, nullptr, 0, 0.0,
+                                        nullptr, nullptr, losses + 9, s));
+      double cur = 0.0;
+      CRVQ_CUDA(cudaMemcpyAsync(&cur, losses + 9, sizeof(double), cudaMemcpyDeviceToHost, s));
+      CRVQ_CUDA(cudaStreamSynchronize(s));
+      if (cur > (1.0 - (double)cfg->eps_rel) * prev) break;
+      prev = cur;
+    }
+  }
+  // S7: losses and the reconstruction in the original order
+  CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o_perm.dev, all, Gc, X, n_tok, 0.0, delta,
+                                    out->W_hat ? o_W_hat.dev : nullptr, losses, s));
+  CRVQ_TRY(o_perm.flush(s));
+  CRVQ_TRY(o_C_base.flush(s));
+  CRVQ_TRY(o_codes_base.flush(s));
+  CRVQ_TRY(o_C_ext.flush(s));
+  CRVQ_TRY(o_codes_ext.flush(s));
+  if (out->W_hat) CRVQ_TRY(o_W_hat.flush(s));
+  if (out->importance) CRVQ_TRY(o_imp.flush(s));
+  double hl[12];
+  CRVQ_CUDA(cudaMemcpyAsync(hl, losses, sizeof(hl), cudaMemcpyDeviceToHost, s));
+  CRVQ_CUDA(cudaStreamSynchronize(s));
+  report->loss_block = hl[0];
+  report->loss_crit = hl[1];
+  report->loss_full = hl[2];
+  report->loss_pre = hl[3];
+  report->loss_before_refine = hl[6];
+  report->scores = scores;
+  report->refine_rounds_done = rounds;
+  return CRVQ_OK;
+}
+
+}  // extern "C"

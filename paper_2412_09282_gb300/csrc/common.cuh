@@ -1,0 +1,129 @@
+// Shared host/device helpers of libcrvq: status handling, the device error word, stream-
+// ordered scratch, SplitMix64 and small device utilities.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <cstdarg>
+#include <cstdio>
+#include <string>
+
+#include "crvq.h"
+
+namespace crvq {
+
+// ---------------------------------------------------------------- host-side status
+void set_last_error(const char* fmt, ...);
+crvq_status fail(crvq_status st, const char* fmt, ...);
+void clear_last_error();
+
+#define CRVQ_CHECK_ARG(cond, ...)                                        \
+  do {                                                                   \
+    if (!(cond)) return ::crvq::fail(CRVQ_ERR_INVALID_ARG, __VA_ARGS__); \
+  } while (0)
+
+#define CRVQ_CUDA(call)                                                                     \
+  do {                                                                                      \
+    cudaError_t e_ = (call);                                                                \
+    if (e_ != cudaSuccess)                                                                  \
+      return ::crvq::fail(e_ == cudaErrorMemoryAllocation ? CRVQ_ERR_NOMEM : CRVQ_ERR_CUDA, \
+                          "%s failed: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__, \
+                          __LINE__);                                                        \
+  } while (0)
+
+#define CRVQ_TRY(expr)                    \
+  do {                                    \
+    crvq_status s_ = (expr);              \
+    if (s_ != CRVQ_OK) return s_;         \
+  } while (0)
+
+// Launch bookkeeping: counts the launch and reports a launch-configuration failure right
+// after a <<<>>> launch.
+void count_launch();
+#define CRVQ_LAUNCHED()              \
+  do {                               \
+    ::crvq::count_launch();          \
+    CRVQ_CUDA(cudaGetLastError());   \
+  } while (0)
+
+// Brackets the launches in its scope with CUDA events when profiling is on.
+class ProfScope {
+ public:
+  ProfScope(const char* name, cudaStream_t s, double units);
+  ~ProfScope();
+  ProfScope(const ProfScope&) = delete;
+  ProfScope& operator=(const ProfScope&) = delete;
+
+ private:
+  const char* name_;
+  cudaStream_t s_;
+  double units_;
+  cudaEvent_t a_ = nullptr;
+};
+
+// Error-word bits set by kernels (never a trap): decoded by crvq_sync().
+enum : unsigned { ERRBIT_INDEX = 1u, ERRBIT_NUMERIC = 2u, ERRBIT_TIMEOUT = 4u };
+
+// Device error word of the current device (allocated once per device, zeroed).
+crvq_status device_error_word(unsigned** out);
+
+// Stream-ordered scratch buffer; freed (stream-ordered) when it goes out of scope.
+class Scratch {
+ public:
+  Scratch() = default;
+  Scratch(const Scratch&) = delete;
+  Scratch& operator=(const Scratch&) = delete;
+  ~Scratch() { release(); }
+  crvq_status alloc(size_t bytes, cudaStream_t s) {
+    release();
+    stream_ = s;
+    if (bytes == 0) return CRVQ_OK;
+    CRVQ_CUDA(cudaMallocAsync(&p_, bytes, s));
+    return CRVQ_OK;
+  }
+  void release() {
+    if (p_) cudaFreeAsync(p_, stream_);
+    p_ = nullptr;
+  }
+  template <class T>
+  T* as() const { return static_cast<T*>(p_); }
+
+ private:
+  void* p_ = nullptr;
+  cudaStream_t stream_ = nullptr;
+};
+
+inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+// Number of SMs of the current device (cached per device).
+int sm_count();
+
+// ---------------------------------------------------------------- device helpers
+// SplitMix64 (Steele, Lea & Flood 2014): output `ctr` (0-based) of the stream `stream`.
+__host__ __device__ inline uint64_t splitmix64(uint64_t stream, uint64_t ctr) {
+  uint64_t z = stream + (ctr + 1ull) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
+__device__ inline void raise_error(unsigned* err, unsigned bit) {
+  if (err) atomicOr(err, bit);
+}
+
+// Codebook view passed to kernels by value (fits in kernel parameter space).
+constexpr int kMaxCodebooks = 8;
+struct CbView {
+  const float* C;
+  int32_t* codes;
+  int64_t ld;
+  int64_t G_cov;
+  int32_t K;
+};
+struct CbList {
+  CbView cb[kMaxCodebooks];
+  int n;
+};
+
+}  // namespace crvq

@@ -1,0 +1,269 @@
+// S7: reconstruction W_enc (sum of the covering codebooks' codewords), the reverse reorder
+// to the original channel order (Sec. 4.3) and the losses of Alg. 1 (QuantLoss):
+//   loss_block = sum_v (t_v - r_v)^T H_g (t_v - r_v)       (block-diagonal part)
+//   loss_crit  = the same over the critical groups g < G_c
+//   loss_full  = ||dW X^T||^2 / n + delta ||dW||^2 = tr(dW H dW^T)   (dW in original order)
+// Per-row partial sums are fp64 and reduced in a fixed order; the full loss streams
+// dW X^T tiles through a SIMT GEMM whose epilogue squares and sums them (fp64 per CTA).
+#include "common.cuh"
+#include "kernels.h"
+
+namespace crvq {
+
+namespace {
+
+// Reconstruction of vector (i, g) in fp64 (sum in codebook order), as fp32 values.
+__device__ __forceinline__ void recon(const CbList& cbs, int64_t i, int64_t g, double r[kD],
+                                      unsigned* err) {
+#pragma unroll
+  for (int j = 0; j < kD; ++j) r[j] = 0.0;
+  for (int s = 0; s < cbs.n; ++s) {
+    const CbView& cb = cbs.cb[s];
+    if (g >= cb.G_cov) continue;
+    const int32_t k = cb.codes[i * cb.ld + g];
+    if (k < 0 || k >= cb.K) {
+      raise_error(err, ERRBIT_INDEX);
+      continue;
+    }
+    const float* c = cb.C + (int64_t)k * kD;
+#pragma unroll
+    for (int j = 0; j < kD; ++j) r[j] += (double)c[j];
+  }
+}
+
+// One CTA per row: block/critical losses and ||dW||^2 of the row (fp64 partials), and the row
+// of W_hat and of dW in the original channel order (staged in shared memory).
+__global__ void __launch_bounds__(256)
+decode_row_kernel(const float* __restrict__ Ws, int64_t M, int64_t N, const float* __restrict__ Hb,
+                  const int32_t* __restrict__ perm, CbList cbs, int64_t n_crit_groups,
+                  float* __restrict__ W_hat, float* __restrict__ dW,
+                  double* __restrict__ row_part, unsigned* err) {
+  extern __shared__ __align__(16) float srow[];
+  __shared__ double red[3][256];
+  const int64_t G = N / kD;
+  for (int64_t i = blockIdx.x; i < M; i += gridDim.x) {
+    double lb = 0.0, lc = 0.0, sq = 0.0;
+    for (int pass = 0; pass < 2; ++pass) {
+      float* out = pass == 0 ? W_hat : dW;
+      if (pass == 1 && !dW) break;
+      __syncthreads();
+      for (int64_t g = threadIdx.x; g < G; g += blockDim.x) {
+        double r[kD];
+        recon(cbs, i, g, r, err);
+        const float* t = Ws + i * N + g * kD;
+        float dl[kD];
+#pragma unroll
+        for (int j = 0; j < kD; ++j) dl[j] = (float)((double)t[j] - r[j]);
+        if (pass == 0) {
+          const float* H = Hb + g * kD * kD;
+          float e = 0.f;
+#pragma unroll
+          for (int b = 0; b < kD; ++b) {
+            float hb = 0.f;
+#pragma unroll
+            for (int a = 0; a < kD; ++a) hb = fmaf(dl[a], H[a * kD + b], hb);
+            e = fmaf(hb, dl[b], e);
+          }
+          lb += (double)e;
+          if (g < n_crit_groups) lc += (double)e;
+#pragma unroll
+          for (int j = 0; j < kD; ++j) sq += (double)dl[j] * (double)dl[j];
+        }
+        if (out) {
+#pragma unroll
+          for (int j = 0; j < kD; ++j) {
+            const int64_t p = g * kD + j;
+            int64_t col = perm ? perm[p] : p;
+            if (col < 0 || col >= N) {
+              raise_error(err, ERRBIT_INDEX);
+              continue;
+            }
+            srow[col] = pass == 0 ? (float)r[j] : dl[j];
+          }
+        }
+      }
+      __syncthreads();
+      if (out) {
+        float* dst = out + i * N;
+        for (int64_t c = (int64_t)threadIdx.x * 4; c < N; c += (int64_t)blockDim.x * 4)
+          *reinterpret_cast<float4*>(dst + c) = *reinterpret_cast<const float4*>(srow + c);
+      }
+    }
+    red[0][threadIdx.x] = lb;
+    red[1][threadIdx.x] = lc;
+    red[2][threadIdx.x] = sq;
+    __syncthreads();
+    for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+      if ((int)threadIdx.x < w) {
+#pragma unroll
+        for (int q = 0; q < 3; ++q) red[q][threadIdx.x] += red[q][threadIdx.x + w];
+      }
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+      row_part[i * 3 + 0] = red[0][0];
+      row_part[i * 3 + 1] = red[1][0];
+      row_part[i * 3 + 2] = red[2][0];
+    }
+  }
+}
+
+constexpr int kT = 128, kBK = 16, kFlush = 256;
+
+// sum over a 128 x 128 tile of P = dW X^T (dW: M x N, X: n x N, both row-major) of P^2.
+__global__ void __launch_bounds__(256)
+gemm_nt_sumsq_kernel(const float* __restrict__ A, int64_t M, const float* __restrict__ X,
+                     int64_t n, int64_t N, double* __restrict__ part) {
+  __shared__ __align__(16) float As[kBK][kT];
+  __shared__ __align__(16) float Bs[kBK][kT];
+  __shared__ double red[256];
+  const int64_t a0 = (int64_t)blockIdx.x * kT, b0 = (int64_t)blockIdx.y * kT;
+  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
+  float acc[8][8], outer[8][8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[i][j] = outer[i][j] = 0.f;
+  int since = 0;
+  const int lr = tid >> 1, lk = (tid & 1) * 8;  // load: row lr, k offset lk (8 values)
+  for (int64_t k0 = 0; k0 < N; k0 += kBK) {
+    {
+      const int64_t ra = a0 + lr, rb = b0 + lr;
+      float va[8], vb[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int64_t k = k0 + lk + q;
+        va[q] = (ra < M && k < N) ? A[ra * N + k] : 0.f;
+        vb[q] = (rb < n && k < N) ? X[rb * N + k] : 0.f;
+      }
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        As[lk + q][lr] = va[q];
+        Bs[lk + q][lr] = vb[q];
+      }
+    }
+    __syncthreads();
+#pragma unroll
+    for (int kk = 0; kk < kBK; ++kk) {
+      float a[8], b[8];
+      const float4 a_lo = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
+      const float4 a_hi = *reinterpret_cast<const float4*>(&As[kk][64 + ty * 4]);
+      const float4 b_lo = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
+      const float4 b_hi = *reinterpret_cast<const float4*>(&Bs[kk][64 + tx * 4]);
+      a[0] = a_lo.x; a[1] = a_lo.y; a[2] = a_lo.z; a[3] = a_lo.w;
+      a[4] = a_hi.x; a[5] = a_hi.y; a[6] = a_hi.z; a[7] = a_hi.w;
+      b[0] = b_lo.x; b[1] = b_lo.y; b[2] = b_lo.z; b[3] = b_lo.w;
+      b[4] = b_hi.x; b[5] = b_hi.y; b[6] = b_hi.z; b[7] = b_hi.w;
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+    }
+    __syncthreads();
+    since += kBK;
+    if (since >= kFlush) {
+      since = 0;
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          outer[i][j] += acc[i][j];
+          acc[i][j] = 0.f;
+        }
+    }
+  }
+  double s = 0.0;
+#pragma unroll
+  for (int i = 0; i < 8; ++i)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const double v = (double)(outer[i][j] + acc[i][j]);
+      s += v * v;
+    }
+  red[tid] = s;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if (tid < w) red[tid] += red[tid + w];
+    __syncthreads();
+  }
+  if (tid == 0) part[(int64_t)blockIdx.y * gridDim.x + blockIdx.x] = red[0];
+}
+
+__global__ void __launch_bounds__(256)
+finalize_losses_kernel(const double* __restrict__ row_part, int64_t M,
+                       const double* __restrict__ gemm_part, int64_t n_gemm, int64_t n_tok,
+                       double delta_host, const float* __restrict__ delta_dev,
+                       double* __restrict__ losses) {
+  __shared__ double red[4][256];
+  double a = 0, b = 0, c = 0, e = 0;
+  for (int64_t i = threadIdx.x; i < M; i += blockDim.x) {
+    a += row_part[i * 3 + 0];
+    b += row_part[i * 3 + 1];
+    c += row_part[i * 3 + 2];
+  }
+  for (int64_t i = threadIdx.x; i < n_gemm; i += blockDim.x) e += gemm_part[i];
+  red[0][threadIdx.x] = a;
+  red[1][threadIdx.x] = b;
+  red[2][threadIdx.x] = c;
+  red[3][threadIdx.x] = e;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w)
+      for (int q = 0; q < 4; ++q) red[q][threadIdx.x] += red[q][threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    losses[0] = red[0][0];
+    losses[1] = red[1][0];
+    if (gemm_part) {
+      const double delta = delta_dev ? (double)*delta_dev : delta_host;
+      losses[2] = red[3][0] / (double)n_tok + delta * red[2][0];
+    } else {
+      losses[2] = __longlong_as_double(0x7ff8000000000000ll);  // NaN: no X given
+    }
+  }
+}
+
+}  // namespace
+
+crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N,
+                                     const float* Hb, const int32_t* perm, const CbList& cbs,
+                                     int64_t n_crit_groups, const float* X, int64_t n_tok,
+                                     double damp_delta, const float* delta_dev, float* W_hat,
+                                     double* losses_dev, cudaStream_t stream) {
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
+  const int nsm = sm_count();
+  const int64_t gx = ceil_div(M, kT), gy = X ? ceil_div(n_tok, kT) : 0;
+  Scratch mem;
+  const size_t dW_bytes = X ? (size_t)M * N * sizeof(float) : 0;
+  const size_t part_bytes = (size_t)M * 3 * sizeof(double) + (size_t)(gx * gy + 1) * sizeof(double);
+  CRVQ_TRY(mem.alloc(part_bytes + dW_bytes + 256, stream));
+  double* row_part = mem.as<double>();
+  double* gemm_part = row_part + M * 3;
+  float* dW = X ? reinterpret_cast<float*>(gemm_part + gx * gy + 1) : nullptr;
+  const size_t smem = (size_t)N * sizeof(float);
+  if (smem > 48 * 1024)
+    CRVQ_CUDA(cudaFuncSetAttribute(decode_row_kernel,
+                                   cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+  const int blocks = (int)std::min<int64_t>(M, (int64_t)8 * nsm);
+  {
+  ProfScope ps("decode_rows", stream,
+               (double)M * N * 4.0 * (1.0 + (W_hat ? 1.0 : 0.0) + (X ? 1.0 : 0.0)));
+  decode_row_kernel<<<blocks, 256, smem, stream>>>(W_sorted, M, N, Hb, perm, cbs,
+                                                   n_crit_groups, W_hat, dW, row_part, err);
+  CRVQ_LAUNCHED();
+  }
+  if (X) {
+    dim3 grid((unsigned)gx, (unsigned)gy);
+    ProfScope ps("loss_gemm", stream, 2.0 * (double)M * N * n_tok);
+    gemm_nt_sumsq_kernel<<<grid, 256, 0, stream>>>(dW, M, X, n_tok, N, gemm_part);
+    CRVQ_LAUNCHED();
+  }
+  finalize_losses_kernel<<<1, 256, 0, stream>>>(row_part, M, X ? gemm_part : nullptr, gx * gy,
+                                                n_tok, damp_delta, delta_dev, losses_dev);
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
+}
+
+}  // namespace crvq

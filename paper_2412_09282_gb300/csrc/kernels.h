@@ -1,0 +1,52 @@
+// Internal launchers of libcrvq (host side). Each enqueues on `stream` and returns a status.
+#pragma once
+
+#include "common.cuh"
+
+namespace crvq {
+
+constexpr int kD = 8;  // vector length supported by the kernels
+
+// A vector set: M x (G_sub * d) block of a row-major matrix (leading dimension ldT) whose
+// group g uses the Hessian block Hb[g].
+struct SetView {
+  const float* T;
+  int64_t ldT;
+  int64_t M;
+  int64_t G_sub;
+  const float* Hb;
+};
+
+crvq_status launch_hessian(const float* X, int64_t n, int64_t N, int d, float damp_rel,
+                           float* H, float* xsq, float* H_blocks, float* delta,
+                           cudaStream_t stream);
+crvq_status launch_extract_blocks(const float* H, int64_t N, int d, const int32_t* perm,
+                                  float* H_blocks, cudaStream_t stream);
+
+crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
+                                  const float* W_pre, const float* xsq, const float* H,
+                                  int mode, uint64_t seed, int32_t* perm, float* importance,
+                                  float* W_sorted, float* H_blocks, cudaStream_t stream);
+
+crvq_status launch_kmeans_init(const SetView& set, const CbList& fixed, int K, uint64_t seed,
+                               float* C_out, cudaStream_t stream);
+
+// Encode / beam (see crvq_encode_beam). `scores` (may be null) accumulates the number of
+// (hypothesis, codeword) pairs the launch scores.
+crvq_status launch_encode_beam(const SetView& set, const CbList& cbs, int n_fixed, int B,
+                               bool keep_if_better, float* vec_err, double* scores,
+                               cudaStream_t stream);
+
+crvq_status launch_update_codebook(const SetView& set, const CbList& cbs, int which,
+                                   float* C_out, int32_t* counts, cudaStream_t stream);
+
+// Decode + block losses (+ optional W_hat in original order, + optional full loss).
+// losses_dev: 3 doubles on the device [block, crit, full].
+// delta_dev (device, 1 float) overrides damp_delta when not null.
+crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N,
+                                     const float* Hb, const int32_t* perm, const CbList& cbs,
+                                     int64_t n_crit_groups, const float* X, int64_t n_tok,
+                                     double damp_delta, const float* delta_dev, float* W_hat,
+                                     double* losses_dev, cudaStream_t stream);
+
+}  // namespace crvq

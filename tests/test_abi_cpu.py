@@ -1,0 +1,88 @@
+"""CPU checks of the C ABI: the library builds, loads and exports every entry point that
+include/crvq.h declares; host-only functions agree with the oracle; argument validation
+rejects bad calls before anything reaches a GPU. No GPU needed."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from oracle import crvq_oracle as O
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2412_09282_gb300 import build
+    build.build()
+    from paper_2412_09282_gb300 import _lib
+    return _lib.load()
+
+
+def _declared_symbols():
+    src = open(os.path.join(ROOT, "include", "crvq.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(crvq_[a-z_0-9]+)\s*\(", src)))
+
+
+def test_header_declares_the_entry_points():
+    names = _declared_symbols()
+    for required in ["crvq_hessian", "crvq_select_reorder_channels", "crvq_kmeans_init",
+                     "crvq_encode_beam", "crvq_update_codebook", "crvq_reconstruct_error"]:
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    from paper_2412_09282_gb300 import _lib
+    for name in _declared_symbols():
+        assert hasattr(lib, name), name
+        assert name in _lib.SIGNATURES, f"{name} has no ctypes signature"
+
+
+def test_avg_bits_and_crit_groups_match_oracle(lib):
+    import paper_2412_09282_gb300 as P
+    for e, d, m, lam in [(8, 8, 1, 0.0), (8, 8, 4, 0.02), (10, 8, 2, 0.05), (12, 16, 3, 0.1)]:
+        for M, N in [(4096, 4096), (11008, 4096), (512, 512)]:
+            for ip in (False, True):
+                assert P.crvq_avg_bits(e, d, m, lam, M, N, ip) == pytest.approx(
+                    O.avg_bits(e, d, m, lam, M, N, ip), rel=1e-12)
+    for N, d, lam in [(512, 8, 0.02), (4096, 8, 0.02), (11008, 8, 0.01), (8192, 8, 0.05),
+                      (64, 8, 0.0), (64, 8, 1.0), (64, 8, 0.125), (8, 8, 0.5)]:
+        assert P.crvq_n_crit_groups(N, d, lam) == O.n_crit_groups(N, d, lam)
+
+
+def test_validation_rejects_before_launch(lib):
+    c = ctypes
+    # d other than 8 is unsupported; NULL pointers are invalid
+    assert lib.crvq_hessian(None, 1, 8, 16, 0.0, None, None, None, None, None) == -2
+    assert lib.crvq_hessian(None, 1, 8, 8, 0.0, None, None, None, None, None) == -1
+    assert b"NULL" in lib.crvq_last_error()
+    dummy = c.c_void_p(16)
+    # N not a multiple of d
+    assert lib.crvq_hessian(dummy, 4, 12, 8, 0.0, dummy, dummy, None, None, None) == -1
+    # negative damping
+    assert lib.crvq_hessian(dummy, 4, 16, 8, -1.0, dummy, dummy, None, None, None) == -1
+    # beam width beyond the implemented maximum
+    from paper_2412_09282_gb300 import _lib
+    cb = (_lib.crvq_codebook * 1)()
+    cb[0] = _lib.crvq_codebook(16, 4, 0, 32, 2, 2)
+    assert lib.crvq_encode_beam(dummy, 16, 2, 2, 8, dummy, cb, 1, 0, 17, 0, None, None) == -2
+    assert lib.crvq_encode_beam(dummy, 16, 2, 2, 8, dummy, cb, 1, 0, 0, 0, None, None) == -1
+    # n_fixed must leave a searched codebook
+    assert lib.crvq_encode_beam(dummy, 16, 2, 2, 8, dummy, cb, 1, 1, 1, 0, None, None) == -1
+    # ldT too small for the set
+    assert lib.crvq_encode_beam(dummy, 8, 2, 2, 8, dummy, cb, 1, 0, 1, 0, None, None) == -1
+    # codebook coverage beyond the set
+    cb[0] = _lib.crvq_codebook(16, 4, 0, 32, 4, 3)
+    assert lib.crvq_update_codebook(dummy, 16, 2, 2, 8, dummy, cb, 1, 0, dummy, None,
+                                    None) == -1
+    # K larger than the number of vectors for k-means init
+    assert lib.crvq_kmeans_init(dummy, 16, 2, 2, 8, None, 0, 5, 0, dummy, None) == -1
+    # crit_frac outside [0, 1]
+    gc = c.c_int64(0)
+    assert lib.crvq_select_reorder_channels(dummy, 2, 16, 8, dummy, dummy, dummy, 1.5, 0, 0,
+                                            dummy, None, dummy, dummy, c.byref(gc), None) == -1
+    # unknown importance mode
+    assert lib.crvq_select_reorder_channels(dummy, 2, 16, 8, dummy, dummy, dummy, 0.5, 7, 0,
+                                            dummy, None, dummy, dummy, c.byref(gc), None) == -1

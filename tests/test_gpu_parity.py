@@ -1,0 +1,358 @@
+"""GPU-vs-oracle parity of every C-ABI entry point, called through the ctypes binding on
+seeded synthetic inputs. Stepwise: each call gets byte-identical inputs on both sides.
+
+Bars: code indices and permutations bit-exact except fp64 near-ties (relative margin below
+1e-6 of err_best + t^T H t, or importance gaps below 1e-6 of max I); codebooks within 1e-4 of
+the codebook's max |value|; losses within 1e-4 relative; H within 2e-5 * sqrt(H_aa H_bb)
+(two-level fp32 accumulation over <= 4096 tokens is bounded by about 3e-5 and typically
+~1e-6); reconstructions bit-exact (fp64 sums of fp32 codewords rounded once on both sides).
+"""
+import numpy as np
+import pytest
+import torch
+
+import synthetic as S
+from oracle import crvq_oracle as O
+from parity_util import (beam_boundary_gap, check_codes_with_ties, dev, host, oracle_cbs)
+
+pytestmark = pytest.mark.gpu
+
+if torch.cuda.is_available():
+    import paper_2412_09282_gb300 as P
+    from paper_2412_09282_gb300 import Codebook
+    from paper_2412_09282_gb300 import build as _build
+    _build.build()
+
+D = 8
+
+
+@pytest.fixture(scope="module")
+def c1():
+    cfg = S.C1
+    W, X = S.gen_W(cfg), S.gen_X(cfg)
+    H, xsq, Hb0, delta = O.hessian(X, cfg.damp_rel, D)
+    return dict(cfg=cfg, W=W, X=X, H=H, xsq=xsq, Hb0=Hb0, delta=delta)
+
+
+def _sync():
+    P.crvq_sync()
+
+
+def _cmp_codebook(Cg, Co, tol=1e-4):
+    err = np.abs(Cg.astype(np.float64) - Co).max() / max(np.abs(Co).max(), 1e-30)
+    assert err <= tol, f"codebook rel err {err}"
+
+
+# ------------------------------------------------------------------------------ S1 Hessian
+@pytest.mark.parametrize("n,N", [(1024, 512), (77, 136), (300, 8), (5, 264)])
+def test_hessian_parity(n, N):
+    cfg = S.C1.with_(name=f"hess_{n}_{N}", n_tok=n, N=N)
+    X = S.gen_X(cfg)
+    H, xsq, Hb, delta = P.crvq_hessian(dev(X), cfg.damp_rel, D)
+    _sync()
+    Ho, xo, Hbo, do = O.hessian(X, cfg.damp_rel, D)
+    Hg = host(H)
+    scale = np.sqrt(np.outer(np.diag(Ho), np.diag(Ho)))
+    assert np.all(np.abs(Hg - Ho) <= 2e-5 * scale + 1e-30)
+    np.testing.assert_allclose(host(xsq), xo, rtol=2e-5)
+    assert abs(float(host(delta)[0]) - float(do)) <= 2e-5 * abs(float(do))
+    np.testing.assert_array_equal(host(Hb), np.stack(
+        [Hg[g * D:(g + 1) * D, g * D:(g + 1) * D] for g in range(N // D)]))
+    assert np.array_equal(Hg, Hg.T)
+
+
+# ------------------------------------------------------------------------------ S3 reorder
+@pytest.mark.parametrize("mode", [0, 1, 2])
+def test_select_reorder_parity(c1, mode):
+    W, H, xsq = c1["W"], c1["H"], c1["xsq"]
+    W_pre = (np.round(W * 40) / 40).astype(np.float32)
+    perm, imp, Ws, Hb, gc = P.crvq_select_reorder_channels(dev(W), D, dev(W_pre), dev(xsq),
+                                                           dev(H), 0.02, mode, seed=1234)
+    _sync()
+    po, io, Wso, Hbo, gco = O.select_reorder_channels(W, D, W_pre, xsq, H, 0.02, mode, 1234)
+    assert gc == gco
+    pg = host(perm)
+    I64 = O.importance(W, W_pre, xsq, mode, 1234)
+    np.testing.assert_allclose(host(imp), io, rtol=1e-6)
+    diff = np.nonzero(pg != po)[0]
+    for p in diff:  # only near-ties may swap
+        assert abs(I64[pg[p]] - I64[po[p]]) <= 1e-6 * I64.max()
+    assert sorted(pg.tolist()) == list(range(W.shape[1]))
+    np.testing.assert_array_equal(host(Ws), W[:, pg])
+    Hp = H[np.ix_(pg, pg)]
+    np.testing.assert_array_equal(host(Hb), np.stack(
+        [Hp[g * D:(g + 1) * D, g * D:(g + 1) * D] for g in range(W.shape[1] // D)]))
+
+
+# ------------------------------------------------------------------------------ k-means init
+def test_kmeans_init_parity(c1):
+    W = c1["W"]
+    M, N = W.shape
+    G = N // D
+    Cg = P.crvq_kmeans_init(dev(W), D, G, 256, seed=99)
+    _sync()
+    np.testing.assert_array_equal(host(Cg), O.kmeans_init(W, D, G, 256, 99))
+    # residual init on a 3-group critical slice with a fixed base codebook (bit-exact: fp64
+    # residual rounded once on both sides)
+    rng = np.random.default_rng(0)
+    Cb = (0.02 * rng.standard_normal((256, D))).astype(np.float32)
+    codes = rng.integers(0, 256, (M, G)).astype(np.int32)
+    Wd = dev(W)
+    codes_d = dev(codes)
+    fixed = [Codebook(dev(Cb), codes_d[:, :3], 3)]
+    Cr = P.crvq_kmeans_init(Wd[:, :3 * D], D, 3, 100, seed=7, fixed=fixed)
+    _sync()
+    Co = O.kmeans_init(W[:, :3 * D], D, 3, 100, 7, [O.Codebook(Cb, codes[:, :3], 3)])
+    np.testing.assert_array_equal(host(Cr), Co)
+    # K equal to the number of vectors takes every vector once
+    Ca = P.crvq_kmeans_init(Wd[:2, :2 * D], D, 2, 4, seed=3)
+    _sync()
+    np.testing.assert_array_equal(host(Ca), np.stack([W[0, :8], W[0, 8:16], W[1, :8],
+                                                      W[1, 8:16]]))
+
+
+# ------------------------------------------------------------------------------ encode
+def _codebook_for(W, G, K, seed, scale=1.0):
+    C = O.kmeans_init(W, D, G, K, seed)
+    return (C * np.float32(scale)).astype(np.float32)
+
+
+@pytest.mark.parametrize("M,K", [(512, 256), (77, 1500), (513, 1), (1, 300), (600, 4100)])
+def test_encode_argmin_parity(c1, M, K):
+    W = c1["W"][:M] if M <= 512 else np.concatenate([c1["W"], c1["W"][:M - 512] * 1.5])
+    W = np.ascontiguousarray(W, dtype=np.float32)
+    G = W.shape[1] // D
+    Hb = c1["Hb0"]
+    C = _codebook_for(W, G, min(K, W.shape[0] * G), 5)
+    if C.shape[0] < K:
+        C = np.concatenate([C, C[:K - C.shape[0]] * 1.01]).astype(np.float32)
+    codes = torch.zeros((W.shape[0], G), dtype=torch.int32, device="cuda")
+    cbs = [Codebook(dev(C), codes, G)]
+    verr = P.crvq_encode_beam(dev(W), D, dev(Hb), cbs, 0, 1, want_err=True)
+    _sync()
+    oc, oerr = O.encode_beam(W, D, Hb, [O.Codebook(C, None, G)], 0, 1)
+    check_codes_with_ties(W, D, Hb, [O.Codebook(C, None, G)], 0, [host(codes)], oc)
+    np.testing.assert_allclose(host(verr), oerr, rtol=1e-5, atol=1e-12)
+
+
+def test_encode_argmin_exact_duplicate_codewords_tie_to_smaller_index(c1):
+    W = c1["W"][:64]
+    G = W.shape[1] // D
+    C = _codebook_for(W, G, 16, 3)
+    C = np.concatenate([C, C]).astype(np.float32)       # every codeword twice
+    codes = torch.zeros((64, G), dtype=torch.int32, device="cuda")
+    P.crvq_encode_beam(dev(W), D, dev(c1["Hb0"]), [Codebook(dev(C), codes, G)], 0, 1)
+    _sync()
+    oc, _ = O.encode_beam(W, D, c1["Hb0"], [O.Codebook(C, None, G)], 0, 1)
+    np.testing.assert_array_equal(host(codes), oc[0])
+    assert host(codes).max() < 16
+
+
+def test_encode_fixed_codebooks_on_critical_slice(c1):
+    W, Hb = c1["W"], c1["Hb0"]
+    M, N = W.shape
+    G, Gc = N // D, 5
+    rng = np.random.default_rng(1)
+    Cb = _codebook_for(W, G, 256, 11)
+    cb_codes = rng.integers(0, 256, (M, G)).astype(np.int32)
+    Ce = (0.3 * _codebook_for(W, G, 64, 12)).astype(np.float32)
+    Wd = dev(W)
+    base_codes = dev(cb_codes)
+    ext_codes = torch.zeros((M, Gc), dtype=torch.int32, device="cuda")
+    cbs = [Codebook(dev(Cb), base_codes[:, :Gc], Gc), Codebook(dev(Ce), ext_codes, Gc)]
+    verr = P.crvq_encode_beam(Wd[:, :Gc * D], D, dev(Hb[:Gc]), cbs, 1, 1, want_err=True)
+    _sync()
+    ocbs = [O.Codebook(Cb, cb_codes[:, :Gc], Gc), O.Codebook(Ce, None, Gc)]
+    oc, oerr = O.encode_beam(W[:, :Gc * D], D, Hb[:Gc], ocbs, 1, 1)
+    check_codes_with_ties(W[:, :Gc * D], D, Hb[:Gc], ocbs, 1, [None, host(ext_codes)], oc)
+    np.testing.assert_allclose(host(verr), oerr, rtol=1e-5)
+
+
+@pytest.mark.parametrize("B", [1, 2, 4, 8, 16])
+def test_encode_beam_parity_mixed_coverage(c1, B):
+    """Full set: base covers every group, two extended codebooks cover the first Gc groups;
+    critical vectors get the 3-stage beam, the others the base arg-min, in one call."""
+    W, Hb = c1["W"], c1["Hb0"]
+    M, N = W.shape
+    G, Gc = N // D, 4
+    Cb = _codebook_for(W, G, 256, 21)
+    rng = np.random.default_rng(2)
+    Ce1 = (0.4 * _codebook_for(W, G, 64, 22)).astype(np.float32)
+    Ce2 = (0.15 * _codebook_for(W, G, 32, 23)).astype(np.float32)
+    codes = [torch.zeros((M, G), dtype=torch.int32, device="cuda"),
+             torch.zeros((M, Gc), dtype=torch.int32, device="cuda"),
+             torch.zeros((M, Gc), dtype=torch.int32, device="cuda")]
+    cbs = [Codebook(dev(Cb), codes[0], G), Codebook(dev(Ce1), codes[1], Gc),
+           Codebook(dev(Ce2), codes[2], Gc)]
+    verr = P.crvq_encode_beam(dev(W), D, dev(Hb), cbs, 0, B, want_err=True)
+    _sync()
+    ocbs = [O.Codebook(Cb, None, G), O.Codebook(Ce1, None, Gc), O.Codebook(Ce2, None, Gc)]
+    oc, oerr = O.encode_beam(W, D, Hb, ocbs, 0, B)
+    gpu = [host(c) for c in codes]
+    # mismatching critical vectors must come from a near-tie inside the oracle's beam
+    diff = np.zeros((M, G), bool)
+    for s in range(3):
+        diff[:, :cbs[s].G_cov] |= gpu[s] != oc[s]
+    for i, g in zip(*np.nonzero(diff)):
+        Cs = [Cb] + ([Ce1, Ce2] if g < Gc else [])
+        gap = beam_boundary_gap(W[i, g * D:(g + 1) * D].astype(np.float64), Hb[g], Cs, B)
+        assert gap < 1e-6, f"vector ({i},{g}) differs with beam gap {gap}"
+    np.testing.assert_allclose(host(verr)[~diff], oerr[~diff], rtol=1e-5)
+
+
+def test_encode_keep_if_better(c1):
+    W, Hb = c1["W"], c1["Hb0"]
+    M, N = W.shape
+    G, Gc = N // D, 3
+    Cb = _codebook_for(W, G, 128, 31)
+    Ce = (0.3 * _codebook_for(W, G, 16, 32)).astype(np.float32)
+    ocbs = [O.Codebook(Cb, None, G), O.Codebook(Ce, None, Gc)]
+    best, _ = O.encode_beam(W, D, Hb, ocbs, 0, 16)      # a (near) optimal tuple
+    # start from the optimal tuple: a width-1 beam must keep it wherever it is better
+    codes = [dev(best[0]), dev(best[1])]
+    cbs = [Codebook(dev(Cb), codes[0], G), Codebook(dev(Ce), codes[1], Gc)]
+    P.crvq_encode_beam(dev(W), D, dev(Hb), cbs, 0, 1, keep_if_better=True)
+    _sync()
+    oc, _ = O.encode_beam(W, D, Hb, [O.Codebook(Cb, best[0], G), O.Codebook(Ce, best[1], Gc)],
+                          0, 1, keep_if_better=True)
+    check_codes_with_ties(W, D, Hb, [O.Codebook(Cb, best[0], G), O.Codebook(Ce, best[1], Gc)],
+                          0, [host(c) for c in codes], oc)
+
+
+# ------------------------------------------------------------------------------ update
+@pytest.mark.parametrize("which", [0, 1])
+def test_update_codebook_parity(c1, which):
+    W, Hb = c1["W"], c1["Hb0"]
+    M, N = W.shape
+    G, Gc = N // D, 6
+    rng = np.random.default_rng(3 + which)
+    Cb = _codebook_for(W, G, 256, 41)
+    Ce = (0.3 * _codebook_for(W, G, 64, 42)).astype(np.float32)
+    cb_codes = rng.integers(0, 250, (M, G)).astype(np.int32)    # 250..255 stay empty
+    ce_codes = rng.integers(0, 60, (M, Gc)).astype(np.int32)    # 60..63 stay empty
+    cbs = [Codebook(dev(Cb), dev(cb_codes), G), Codebook(dev(Ce), dev(ce_codes), Gc)]
+    Cg, cnt = P.crvq_update_codebook(dev(W), D, dev(Hb), cbs, which)
+    _sync()
+    ocbs = [O.Codebook(Cb, cb_codes, G), O.Codebook(Ce, ce_codes, Gc)]
+    Co, co = O.update_codebook(W, D, Hb, ocbs, which)
+    np.testing.assert_array_equal(host(cnt), co)
+    _cmp_codebook(host(Cg), Co.astype(np.float64))
+    empty = co == 0
+    np.testing.assert_array_equal(host(Cg)[empty], (Cb if which == 0 else Ce)[empty])
+
+
+def test_update_codebook_in_place_and_large_K(c1):
+    W, Hb = c1["W"], c1["Hb0"]
+    M, N = W.shape
+    G = N // D
+    rng = np.random.default_rng(5)
+    K = 4096                                            # two radix passes
+    C = _codebook_for(W, G, K, 51)
+    codes = rng.integers(0, K, (M, G)).astype(np.int32)
+    Cd = dev(C)
+    cbs = [Codebook(Cd, dev(codes), G)]
+    P.crvq_update_codebook(dev(W), D, dev(Hb), cbs, 0, C_out=Cd)
+    _sync()
+    Co, _ = O.update_codebook(W, D, Hb, [O.Codebook(C, codes, G)], 0)
+    _cmp_codebook(host(Cd), Co.astype(np.float64))
+
+
+def test_update_is_deterministic(c1):
+    W, Hb = c1["W"], c1["Hb0"]
+    M, N = W.shape
+    G = N // D
+    rng = np.random.default_rng(6)
+    C = _codebook_for(W, G, 256, 61)
+    codes = dev(rng.integers(0, 256, (M, G)).astype(np.int32))
+    cbs = [Codebook(dev(C), codes, G)]
+    a, _ = P.crvq_update_codebook(dev(W), D, dev(Hb), cbs, 0)
+    b, _ = P.crvq_update_codebook(dev(W), D, dev(Hb), cbs, 0)
+    _sync()
+    assert torch.equal(a, b)
+
+
+# ------------------------------------------------------------------------------ S7 losses
+def test_reconstruct_error_parity(c1):
+    W, X, H, delta = c1["W"], c1["X"], c1["H"], float(c1["delta"])
+    M, N = W.shape
+    G, Gc = N // D, 2
+    rng = np.random.default_rng(7)
+    perm = rng.permutation(N).astype(np.int32)
+    Ws = np.ascontiguousarray(W[:, perm])
+    Hb = np.stack([H[np.ix_(perm[g * D:g * D + D], perm[g * D:g * D + D])] for g in range(G)])
+    Cb = _codebook_for(Ws, G, 256, 71)
+    Ce = (0.3 * _codebook_for(Ws, G, 32, 72)).astype(np.float32)
+    cbc = rng.integers(0, 256, (M, G)).astype(np.int32)
+    cec = rng.integers(0, 32, (M, Gc)).astype(np.int32)
+    cbs = [Codebook(dev(Cb), dev(cbc), G), Codebook(dev(Ce), dev(cec), Gc)]
+    Wh, lb, lc, lf = P.crvq_reconstruct_error(dev(Ws), D, dev(Hb), dev(perm), cbs, Gc,
+                                              X=dev(X), damp_delta=delta)
+    ocbs = [O.Codebook(Cb, cbc, G), O.Codebook(Ce, cec, Gc)]
+    Who, lbo, lco, lfo = O.reconstruct_error(Ws, D, Hb, perm, ocbs, Gc, X, delta)
+    np.testing.assert_array_equal(host(Wh), Who)
+    assert abs(lb - lbo) <= 1e-4 * lbo
+    assert abs(lc - lco) <= 1e-4 * lco
+    assert abs(lf - lfo) <= 1e-4 * lfo
+    # identity order, no X
+    Wh2, lb2, _, lf2 = P.crvq_reconstruct_error(dev(Ws), D, dev(Hb), None, cbs, Gc)
+    assert lf2 is None
+    np.testing.assert_array_equal(host(Wh2), O.reconstruct_error(Ws, D, Hb, None, ocbs, Gc)[0])
+
+
+# ------------------------------------------------------------------------------ errors
+def test_device_index_check_reports_and_recovers(c1):
+    W, Hb = c1["W"], c1["Hb0"]
+    M, N = W.shape
+    G = N // D
+    C = _codebook_for(W, G, 16, 81)
+    bad = np.zeros((M, G), np.int32)
+    bad[3, 4] = 999                                      # out of range: skipped, reported
+    with pytest.raises(P.CrvqError) as e:
+        P.crvq_update_codebook(dev(W), D, dev(Hb), [Codebook(dev(C), dev(bad), G)], 0)
+        P.crvq_sync()
+    assert e.value.status == -7
+    P.crvq_sync()                                        # the word was cleared
+    good = dev(np.zeros((M, G), np.int32))
+    P.crvq_encode_beam(dev(W), D, dev(Hb), [Codebook(dev(C), good, G)], 0, 1)
+    P.crvq_sync()
+
+
+def test_invalid_arguments_raise_before_launch(c1):
+    W = dev(c1["W"])
+    with pytest.raises(P.CrvqError) as e:
+        P.crvq_kmeans_init(W[:1, :8], D, 1, 2, seed=0)   # K > #vectors
+    assert e.value.status == -1
+    with pytest.raises(P.CrvqError) as e:
+        P.crvq_hessian(dev(c1["X"]), 0.01, d=16)
+    assert e.value.status == -2
+
+
+# ------------------------------------------------------------------------------ end to end
+def test_quantize_layer_c1_end_to_end(c1):
+    cfg = c1["cfg"]
+    out = P.crvq_quantize_layer(dev(c1["W"]), dev(c1["X"]), cfg)
+    torch.cuda.synchronize()
+    ref = O.quantize_layer(c1["W"], c1["X"], cfg)
+    rep = out.report
+    np.testing.assert_array_equal(host(out.perm), ref["perm"])
+    assert rep["n_crit_groups"] == ref["n_crit_groups"]
+    agree = (host(out.codes_base) == ref["codebooks"][0].codes).mean()
+    assert agree >= 0.999, agree
+    for key, r in [("loss_block", ref["loss_block"]), ("loss_crit", ref["loss_crit"]),
+                   ("loss_full", ref["loss_full"]), ("loss_pre", ref["loss_pre"])]:
+        assert abs(rep[key] - r) <= 1e-3 * abs(r), (key, rep[key], r)
+    _cmp_codebook(host(out.C_base), ref["codebooks"][0].C.astype(np.float64), 1e-3)
+
+
+def test_quantize_layer_host_buffers_match_device(c1):
+    cfg = c1["cfg"].with_(kmeans_iters=3)
+    a = P.crvq_quantize_layer(dev(c1["W"]), dev(c1["X"]), cfg)
+    torch.cuda.synchronize()
+    Wh = torch.from_numpy(c1["W"]).pin_memory()
+    Xh = torch.from_numpy(c1["X"]).pin_memory()
+    b = P.crvq_quantize_layer(Wh, Xh, cfg)
+    assert b.perm.device.type == "cpu"
+    np.testing.assert_array_equal(host(a.perm), b.perm.numpy())
+    np.testing.assert_array_equal(host(a.codes_base), b.codes_base.numpy())
+    np.testing.assert_array_equal(host(a.C_ext), b.C_ext.numpy())
+    assert a.report["loss_full"] == b.report["loss_full"]
