@@ -474,6 +474,7 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   const float *W = nullptr, *X = nullptr;
   CRVQ_TRY(to_device(W_in, (size_t)M * N, bW, &W, s));
   CRVQ_TRY(to_device(X_in, (size_t)n_tok * N, bX, &X, s));
+  CRVQ_CHECK_ARG(aligned16(W) && aligned16(X), "W and X must be 16-byte aligned");
 
   OutBuf<int32_t> o_perm, o_codes_base, o_codes_ext;
   OutBuf<float> o_C_base, o_C_ext, o_W_hat, o_imp;
@@ -484,6 +485,9 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   CRVQ_TRY(o_codes_ext.init(out->codes_ext, (size_t)cfg->n_ext * M * Gc, s));
   if (out->W_hat) CRVQ_TRY(o_W_hat.init(out->W_hat, (size_t)M * N, s));
   CRVQ_TRY(o_imp.init(out->importance, N, s));
+  CRVQ_CHECK_ARG(aligned16(o_C_base.dev) && aligned16(o_C_ext.dev) &&
+                     (!out->W_hat || aligned16(o_W_hat.dev)),
+                 "C_base, C_ext and W_hat must be 16-byte aligned");
 
   Buf bH, bxsq, bHb0, bdelta, bC0, bcodes0, bWpre, bWs, bHb, bloss;
   float *H, *xsq, *Hb0, *delta, *C0, *Wpre, *Ws, *Hb;

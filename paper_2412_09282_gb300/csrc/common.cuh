@@ -95,6 +95,7 @@ class Scratch {
 };
 
 inline int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // Number of SMs of the current device (cached per device).
 int sm_count();

@@ -235,13 +235,14 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   CRVQ_TRY(device_error_word(&err));
   const int nsm = sm_count();
   const int64_t gx = ceil_div(M, kT), gy = X ? ceil_div(n_tok, kT) : 0;
-  Scratch mem;
-  const size_t dW_bytes = X ? (size_t)M * N * sizeof(float) : 0;
+  // Scratch: dW (16-byte aligned for the 128-bit stores), then the fp64 partial sums.
+  const size_t dW_bytes = X ? align_up((size_t)M * N * sizeof(float), 256) : 0;
   const size_t part_bytes = (size_t)M * 3 * sizeof(double) + (size_t)(gx * gy + 1) * sizeof(double);
-  CRVQ_TRY(mem.alloc(part_bytes + dW_bytes + 256, stream));
-  double* row_part = mem.as<double>();
+  Scratch mem;
+  CRVQ_TRY(mem.alloc(dW_bytes + part_bytes, stream));
+  float* dW = X ? mem.as<float>() : nullptr;
+  double* row_part = reinterpret_cast<double*>(mem.as<char>() + dW_bytes);
   double* gemm_part = row_part + M * 3;
-  float* dW = X ? reinterpret_cast<float*>(gemm_part + gx * gy + 1) : nullptr;
   const size_t smem = (size_t)N * sizeof(float);
   if (smem > 48 * 1024)
     CRVQ_CUDA(cudaFuncSetAttribute(decode_row_kernel,
