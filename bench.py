@@ -275,18 +275,22 @@ def main():
     # of every output inside the timed region, wall clock around a synchronizing call.
     e2e_times = []
     h_out = None
-    for i in range(args.e2e_steps + 1):
+    for i in range(args.e2e_steps + 1 if args.e2e_steps > 0 else 0):
         t0 = time.perf_counter()
         h_out = P.crvq_quantize_layer(W_h, X_h, cfg_r, out=h_out)
         dt = time.perf_counter() - t0
         if i > 0:
             e2e_times.append(dt)
-    e2e_scores = h_out.report["scores"]
-    h2d = W_h.numel() * 4 + X_h.numel() * 4
-    d2h = sum(t.numel() * t.element_size() for t in
-              [h_out.perm, h_out.C_base, h_out.codes_base, h_out.C_ext, h_out.codes_ext,
-               h_out.W_hat, h_out.importance] if t is not None) + 48
-    e2e_val = ws * e2e_scores / statistics.mean(e2e_times)
+    e2e = None
+    if e2e_times:
+        h2d = W_h.numel() * 4 + X_h.numel() * 4
+        d2h = sum(t.numel() * t.element_size() for t in
+                  [h_out.perm, h_out.C_base, h_out.codes_base, h_out.C_ext, h_out.codes_ext,
+                   h_out.W_hat, h_out.importance] if t is not None) + 48
+        e2e = {"value": ws * h_out.report["scores"] / statistics.mean(e2e_times),
+               "unit": "scores/s", "h2d_bytes_per_step": int(h2d),
+               "d2h_bytes_per_step": int(d2h),
+               "ms_per_step": 1e3 * statistics.mean(e2e_times)}
 
     if rank != 0:
         return
@@ -315,8 +319,7 @@ def main():
         "losses": {k: out.report[k] for k in ("loss_pre", "loss_block", "loss_crit",
                                               "loss_full")},
         "roofline": roof,
-        "e2e": {"value": e2e_val, "unit": "scores/s", "h2d_bytes_per_step": int(h2d),
-                "d2h_bytes_per_step": int(d2h), "ms_per_step": 1e3 * statistics.mean(e2e_times)},
+        "e2e": e2e,
         "gpu_launches": int(launches),
         "kernels": [{"name": k["name"], "launches": k["launches"], "ms": k["ms"],
                      "share": k["ms"] / total_k} for k in ks[:12]],
