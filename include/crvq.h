@@ -251,6 +251,7 @@ typedef struct crvq_layer_report {
   double loss_before_refine;
   double scores;         /* (hypothesis, codeword) pairs scored by the encode passes */
   int64_t n_crit_groups;
+  int64_t flagged;       /* encode decisions re-taken in fp64 (fp32 bound not conclusive) */
   int32_t refine_rounds_done;
   int32_t _pad;
 } crvq_layer_report;

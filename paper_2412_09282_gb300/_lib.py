@@ -36,7 +36,8 @@ class crvq_layer_report(C.Structure):
     _fields_ = [("loss_pre", C.c_double), ("loss_block", C.c_double),
                 ("loss_crit", C.c_double), ("loss_full", C.c_double),
                 ("loss_before_refine", C.c_double), ("scores", C.c_double),
-                ("n_crit_groups", C.c_int64), ("refine_rounds_done", C.c_int32),
+                ("n_crit_groups", C.c_int64), ("flagged", C.c_int64),
+                ("refine_rounds_done", C.c_int32),
                 ("_pad", C.c_int32)]
 
 

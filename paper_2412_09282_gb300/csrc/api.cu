@@ -9,6 +9,7 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "stats.cuh"
 
 namespace crvq {
 
@@ -309,7 +310,7 @@ crvq_status crvq_encode_beam(const float* T, int64_t ldT, int64_t M, int64_t G_s
   CbList cl;
   CRVQ_TRY(make_cblist(cbs, n_cb, G_sub, true, &cl));
   SetView set{T, ldT, M, G_sub, H_blocks};
-  return launch_encode_beam(set, cl, n_fixed, B, keep_if_better != 0, vec_err, nullptr,
+  return launch_encode_beam(set, cl, n_fixed, B, keep_if_better != 0, vec_err, EncodeExtras{},
                             (cudaStream_t)stream);
 }
 
@@ -386,15 +387,24 @@ uint64_t phase_seed(uint64_t seed, int phase, int cb) {
 }
 
 // Lloyd iterations for the last codebook of `cbs` (all earlier ones fixed), then a final
-// encode: T x (encode, LS update) + encode.
-crvq_status lloyd(const SetView& set, CbList cbs, int iters, double* scores, cudaStream_t s) {
+// encode: T x (encode, LS update) + encode. Each encode accumulates the least-squares
+// statistics of the codes it writes, so the update is only the per-codeword solve.
+crvq_status lloyd(const SetView& set, CbList cbs, int iters, const EncodeExtras& ex0,
+                  cudaStream_t s) {
   const int j = cbs.n - 1;
   float* C = const_cast<float*>(cbs.cb[j].C);
+  Scratch mem;
+  StatsView st;
+  CRVQ_TRY(stats_alloc(mem, cbs.cb[j].G_cov, cbs.cb[j].K, &st, s));
+  CRVQ_TRY(launch_stats_prepare(set, cbs, j, st, s));  // T, H and fixed codebooks stay put
+  EncodeExtras ex = ex0;
+  ex.stats = &st;
   for (int it = 0; it < iters; ++it) {
-    CRVQ_TRY(launch_encode_beam(set, cbs, j, 1, false, nullptr, scores, s));
-    CRVQ_TRY(launch_update_codebook(set, cbs, j, C, nullptr, s));
+    if (it > 0) CRVQ_TRY(stats_zero(st, s));
+    CRVQ_TRY(launch_encode_beam(set, cbs, j, 1, false, nullptr, ex, s));
+    CRVQ_TRY(launch_stats_solve(set, st, C, C, nullptr, s));
   }
-  return launch_encode_beam(set, cbs, j, 1, false, nullptr, scores, s);
+  return launch_encode_beam(set, cbs, j, 1, false, nullptr, ex0, s);
 }
 
 template <class T>
@@ -469,6 +479,13 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   memset(report, 0, sizeof(*report));
   report->n_crit_groups = Gc;
   double scores = 0.0;
+  Buf bflag;
+  unsigned long long* flag_total = nullptr;
+  CRVQ_TRY(bflag.get(&flag_total, 1, s));
+  CRVQ_CUDA(cudaMemsetAsync(flag_total, 0, sizeof(unsigned long long), s));
+  EncodeExtras ex;
+  ex.scores = &scores;
+  ex.flag_total = flag_total;
 
   Buf bW, bX;
   const float *W = nullptr, *X = nullptr;
@@ -514,7 +531,7 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
     cl.cb[0] = CbView{C0, codes0, G, G, cfg->K_base};
     CRVQ_TRY(launch_kmeans_init(set, CbList{}, cfg->K_base,
                                 phase_seed(cfg->seed, 1, 0), C0, s));
-    CRVQ_TRY(lloyd(set, cl, cfg->kmeans_iters, &scores, s));
+    CRVQ_TRY(lloyd(set, cl, cfg->kmeans_iters, ex, s));
     CRVQ_TRY(launch_reconstruct_error(W, M, N, Hb0, nullptr, cl, 0, nullptr, 0, 0.0, nullptr,
                                       Wpre, losses + 3, s));
   }
@@ -535,7 +552,7 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
     cl.cb[0] = all.cb[0];
     CRVQ_TRY(launch_kmeans_init(full, CbList{}, cfg->K_base, phase_seed(cfg->seed, 2, 0),
                                 o_C_base.dev, s));
-    CRVQ_TRY(lloyd(full, cl, cfg->kmeans_iters, &scores, s));
+    CRVQ_TRY(lloyd(full, cl, cfg->kmeans_iters, ex, s));
   }
   // S5: extended codebooks on the critical residual (Alg. 1 lines 8-13)
   if (cfg->n_ext > 0) {
@@ -552,7 +569,7 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
       for (int q = 0; q < t; ++q) fixed.cb[q] = cl.cb[q];
       CRVQ_TRY(launch_kmeans_init(crit, fixed, cfg->K_ext, phase_seed(cfg->seed, 3, t),
                                   const_cast<float*>(all.cb[t].C), s));
-      CRVQ_TRY(lloyd(crit, cl, cfg->kmeans_iters, &scores, s));
+      CRVQ_TRY(lloyd(crit, cl, cfg->kmeans_iters, ex, s));
     }
   }
   // S6: least-squares codebook updates + joint beam re-encode (Alg. 1 lines 14-17)
@@ -567,7 +584,7 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   for (int r = 0; r < cfg->refine_rounds; ++r) {
     for (int j = 0; j < all.n; ++j)
       CRVQ_TRY(launch_update_codebook(full, all, j, const_cast<float*>(all.cb[j].C), nullptr, s));
-    CRVQ_TRY(launch_encode_beam(full, all, 0, cfg->B, true, nullptr, &scores, s));
+    CRVQ_TRY(launch_encode_beam(full, all, 0, cfg->B, true, nullptr, ex, s));
     ++rounds;
     if (cfg->refine_rounds > 1 && r + 1 < cfg->refine_rounds) {
       CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o_perm.dev, all, Gc, nullptr, 0, 0.0,
@@ -590,8 +607,11 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   if (out->W_hat) CRVQ_TRY(o_W_hat.flush(s));
   if (out->importance) CRVQ_TRY(o_imp.flush(s));
   double hl[12];
+  unsigned long long flagged = 0;
   CRVQ_CUDA(cudaMemcpyAsync(hl, losses, sizeof(hl), cudaMemcpyDeviceToHost, s));
+  CRVQ_CUDA(cudaMemcpyAsync(&flagged, flag_total, sizeof(flagged), cudaMemcpyDeviceToHost, s));
   CRVQ_CUDA(cudaStreamSynchronize(s));
+  report->flagged = (int64_t)flagged;
   report->loss_block = hl[0];
   report->loss_crit = hl[1];
   report->loss_full = hl[2];

@@ -3,18 +3,23 @@
 //
 // Score of target r against codeword c for a vector of group g:
 //   err(r, c) = (r - c)^T H_g (r - c) = r^T H_g r + n_g(c) - 2 (H_g r) . c,  n_g(c) = c^T H_g c.
-// The fast pass evaluates the expanded form in fp32 (8 FMAs per pair, the norm table of the
-// group staged in shared memory) and keeps, per vector, the best and second-best values. An
-// a-priori bound E on the fp32 error of every score (from the magnitudes of H_g, the target
-// and the codebook) certifies the arg-min when the runner-up is more than 2E away; otherwise
-// the vector goes to a fallback that re-scans it and decides among the candidates within 2E
-// in fp64. The result equals the fp64 arg-min (ties to the smaller index) except for ties at
-// fp64 rounding level.
+// The fast pass evaluates the expanded form in fp32 (8 FMAs per pair; the codewords, their
+// group norms and L1 norms staged in shared memory). Every fp32 score s_k comes with an
+// a-priori bound on its rounding error,
+//   E_k <= Et_k = u C (Na_k + 2 Pmax L1_k),   u = 2^-24,
+//   Na_k = |c_k|^T |H_g| |c_k|,  L1_k = ||c_k||_1,  Pmax = max_p sum_j |H_pj| (|t_j| + sum_f |c_f,j|),
+// and the pass ranks the lower bounds low_k = s_k - Et_k, keeping the best two. The arg-min j
+// is certified when low_2nd - low_j > 2 Et_j: every other codeword's exact score is then larger
+// than j's. Otherwise the vector is flagged; a fallback re-scores it, keeps the codewords with
+// low_k <= low_j + 2 Et_j (the exact arg-min is among them) and decides among those in fp64.
+// Codes therefore equal the fp64 arg-min (ties to the smaller index) except for ties at fp64
+// rounding level. Beam stages use the same bounds on a sorted top-(B+1) list.
 #include <algorithm>
 #include <vector>
 
 #include "common.cuh"
 #include "kernels.h"
+#include "stats.cuh"
 
 namespace crvq {
 
@@ -24,11 +29,15 @@ constexpr int kThreads = 128;
 constexpr int kChunk = 1024;            // codewords staged per shared-memory chunk
 constexpr float kU = 5.9604645e-08f;    // 2^-24
 
+// Error-bound multiplier: about twice the worst-case FMA-chain analysis (<= 37 + 2 n_fixed).
+__host__ __device__ inline float bound_mult(int n_terms) { return 64.f + 4.f * n_terms; }
+
 struct FlagList {
   int64_t* vec;      // vector index within the launch range (i * G_range + (g - g_begin))
-  float* thr;        // decision threshold b1 + 2E (fast pass value units)
+  float* thr;        // decision threshold (fast-pass value units)
   unsigned* count;
   int64_t cap;
+  unsigned long long* total;  // optional running total of flagged vectors
 };
 
 // --------------------------------------------------------------------------- device helpers
@@ -47,8 +56,8 @@ __device__ __forceinline__ bool code_ok(int32_t k, int32_t K, unsigned* err) {
   return true;
 }
 
-// fp32 target r = t - sum of the fixed codebooks covering g, and the magnitude bound
-// a_j = |t_j| + sum |c_fixed,j| of every term that went into r.
+// fp32 target r = t - sum of the fixed codebooks covering g (codebook order), and the
+// magnitude bound a_j = |t_j| + sum |c_fixed,j| of every term that went into r.
 __device__ __forceinline__ void target32(const SetView& set, const CbList& cbs, int n_fixed,
                                          int64_t i, int64_t g, float r[kD], float a[kD],
                                          unsigned* err) {
@@ -70,7 +79,7 @@ __device__ __forceinline__ void target32(const SetView& set, const CbList& cbs, 
   }
 }
 
-// fp64 target (the fixed reconstruction subtracted in fp64).
+// fp64 target (the fixed reconstruction subtracted in fp64, codebook order).
 __device__ void target64(const SetView& set, const CbList& cbs, int n_fixed, int64_t i,
                          int64_t g, double r[kD], unsigned* err) {
   const float* t = set.T + i * set.ldT + g * kD;
@@ -87,7 +96,7 @@ __device__ void target64(const SetView& set, const CbList& cbs, int n_fixed, int
   }
 }
 
-// (r - c)^T H (r - c) in fp64; H row-major d x d (fp32), c fp32.
+// (r - c)^T H (r - c) in fp64; H row-major d x d (fp32); c fp32 or null.
 __device__ double quad_err64(const double r[kD], const float* c, const float* H) {
   double dlt[kD];
 #pragma unroll
@@ -103,78 +112,107 @@ __device__ double quad_err64(const double r[kD], const float* c, const float* H)
   return e;
 }
 
-// Stage the codewords [k0, k0 + nk) of C and their group norms n_g(c) = c^T H c in shared
-// memory; also the running maxima Na = max_k |c|^T |H| |c| and cmax_j = max_k |c_kj|.
-__device__ __forceinline__ void stage_chunk(const float* __restrict__ C, int k0, int nk,
-                                            const float* sH, float* sC, float* sN,
-                                            unsigned* sNa_bits, unsigned* sCmax_bits) {
-  for (int k = threadIdx.x; k < nk; k += blockDim.x) {
-    float c[kD];
-    load_vec(C + (int64_t)(k0 + k) * kD, c);
-    float n = 0.f, na = 0.f;
+// Codeword terms of the score and of its bound: n = c^T H c (fp32, two FMA chains),
+// na = |c|^T |H| |c|, l1 = ||c||_1.
+__device__ __forceinline__ void codeword_terms(const float c[kD], const float* H, float& n,
+                                               float& na, float& l1) {
+  n = 0.f;
+  na = 0.f;
+  l1 = 0.f;
 #pragma unroll
-    for (int a = 0; a < kD; ++a) {
-      float u = 0.f, ua = 0.f;
+  for (int a = 0; a < kD; ++a) {
+    float u = 0.f, ua = 0.f;
 #pragma unroll
-      for (int b = 0; b < kD; ++b) {
-        u = fmaf(sH[a * kD + b], c[b], u);
-        ua = fmaf(fabsf(sH[a * kD + b]), fabsf(c[b]), ua);
-      }
-      n = fmaf(c[a], u, n);
-      na = fmaf(fabsf(c[a]), ua, na);
+    for (int b = 0; b < kD; ++b) {
+      u = fmaf(H[a * kD + b], c[b], u);
+      ua = fmaf(fabsf(H[a * kD + b]), fabsf(c[b]), ua);
     }
-    *reinterpret_cast<float4*>(sC + k * kD) = make_float4(c[0], c[1], c[2], c[3]);
-    *reinterpret_cast<float4*>(sC + k * kD + 4) = make_float4(c[4], c[5], c[6], c[7]);
-    sN[k] = n;
-    atomicMax(sNa_bits, __float_as_uint(na));
-#pragma unroll
-    for (int j = 0; j < kD; ++j) atomicMax(&sCmax_bits[j], __float_as_uint(fabsf(c[j])));
+    n = fmaf(c[a], u, n);
+    na = fmaf(fabsf(c[a]), ua, na);
+    l1 += fabsf(c[a]);
   }
 }
 
+// Vector terms: m2q = -2 H r (the row FMA chains of stats_htau), Pmax = max_p (|H| a)_p.
+__device__ __forceinline__ void vector_terms(const float r[kD], const float a[kD],
+                                             const float* H, float m2q[kD], float& pmax) {
+  pmax = 0.f;
+#pragma unroll
+  for (int p = 0; p < kD; ++p) {
+    float q = 0.f, pa = 0.f;
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      q = fmaf(H[p * kD + j], r[j], q);
+      pa = fmaf(fabsf(H[p * kD + j]), a[j], pa);
+    }
+    m2q[p] = -2.f * q;
+    pmax = fmaxf(pmax, pa);
+  }
+}
+
+// Stage the codewords [k0, k0 + nk): sC = c, sN = n - u C Na (the lower-bound offset of the
+// codeword part), sL = ||c||_1.
+__device__ __forceinline__ void stage_chunk(const float* __restrict__ C, int k0, int nk,
+                                            const float* sH, float cmul, float* sC, float* sN,
+                                            float* sL) {
+  for (int k = threadIdx.x; k < nk; k += blockDim.x) {
+    float c[kD];
+    load_vec(C + (int64_t)(k0 + k) * kD, c);
+    float n, na, l1;
+    codeword_terms(c, sH, n, na, l1);
+    *reinterpret_cast<float4*>(sC + k * kD) = make_float4(c[0], c[1], c[2], c[3]);
+    *reinterpret_cast<float4*>(sC + k * kD + 4) = make_float4(c[4], c[5], c[6], c[7]);
+    sN[k] = n - kU * cmul * na;
+    sL[k] = l1;
+  }
+}
+
+// fp32 lower bound low_k of the score of codeword k (same operation order as the fast pass).
+__device__ __forceinline__ float low_score(const float c[kD], const float* H, const float m2q[kD],
+                                           float nbeta, float cmul) {
+  float n, na, l1;
+  codeword_terms(c, H, n, na, l1);
+  float s = n - kU * cmul * na;
+#pragma unroll
+  for (int p = 0; p < kD; ++p) s = fmaf(m2q[p], c[p], s);
+  return fmaf(nbeta, l1, s);
+}
+
 // --------------------------------------------------------------------------- arg-min pass
-// One CTA = one group g and kThreads * VPT rows. Each thread owns VPT vectors.
+// One CTA = one group g and kThreads * VPT rows; each thread owns VPT vectors. When
+// st.cnt != null the certified codes' least-squares statistics are accumulated (stats.cuh).
 template <int VPT>
 __global__ void __launch_bounds__(kThreads)
 argmin_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
               int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0, FlagList flags,
-              unsigned* err) {
+              StatsView st, unsigned* err) {
   const int64_t g = g_begin + blockIdx.y;
   const int64_t G_range = gridDim.y;
   const int64_t row0 = (int64_t)blockIdx.x * kThreads * VPT;
   __shared__ float sH[kD * kD];
   __shared__ __align__(16) float sC[kChunk * kD];
-  __shared__ float sN[kChunk];
-  __shared__ unsigned sNa_bits, sCmax_bits[kD];
+  __shared__ float sN[kChunk], sL[kChunk];
 
   if (threadIdx.x < kD * kD) sH[threadIdx.x] = set.Hb[g * kD * kD + threadIdx.x];
-  if (threadIdx.x < kD) sCmax_bits[threadIdx.x] = 0u;
-  if (threadIdx.x == 0) sNa_bits = 0u;
   __syncthreads();
 
   const CbView cw = cbs.cb[s_idx];
-  float m2q[VPT][kD];
+  const float cmul = bound_mult(n_fixed);
+  float m2q[VPT][kD], nbeta[VPT];
   float b1[VPT], b2[VPT];
   int i1[VPT];
-  bool live[VPT];
 #pragma unroll
   for (int v = 0; v < VPT; ++v) {
     const int64_t i = row0 + threadIdx.x + (int64_t)v * kThreads;
-    live[v] = i < set.M;
-    float r[kD], a[kD];
-    if (live[v]) {
+    float r[kD], a[kD], pmax;
+    if (i < set.M) {
       target32(set, cbs, n_fixed, i, g, r, a, err);
     } else {
 #pragma unroll
       for (int j = 0; j < kD; ++j) r[j] = a[j] = 0.f;
     }
-#pragma unroll
-    for (int p = 0; p < kD; ++p) {
-      float q = 0.f;
-#pragma unroll
-      for (int j = 0; j < kD; ++j) q = fmaf(sH[p * kD + j], r[j], q);
-      m2q[v][p] = -2.f * q;
-    }
+    vector_terms(r, a, sH, m2q[v], pmax);
+    nbeta[v] = -2.f * kU * cmul * pmax;
     b1[v] = INFINITY;
     b2[v] = INFINITY;
     i1[v] = 0;
@@ -183,13 +221,13 @@ argmin_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
   for (int k0 = 0; k0 < cw.K; k0 += kChunk) {
     const int nk = min(kChunk, cw.K - k0);
     __syncthreads();
-    stage_chunk(cw.C, k0, nk, sH, sC, sN, &sNa_bits, sCmax_bits);
+    stage_chunk(cw.C, k0, nk, sH, cmul, sC, sN, sL);
     __syncthreads();
 #pragma unroll 2
     for (int k = 0; k < nk; ++k) {
       const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
       const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
-      const float n = sN[k];
+      const float n = sN[k], l1 = sL[k];
 #pragma unroll
       for (int v = 0; v < VPT; ++v) {
         float s = n;
@@ -201,6 +239,7 @@ argmin_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
         s = fmaf(m2q[v][5], c1.y, s);
         s = fmaf(m2q[v][6], c1.z, s);
         s = fmaf(m2q[v][7], c1.w, s);
+        s = fmaf(nbeta[v], l1, s);
         b2[v] = fminf(b2[v], fmaxf(s, b1[v]));
         const bool lt = s < b1[v];
         i1[v] = lt ? k0 + k : i1[v];
@@ -208,86 +247,69 @@ argmin_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
       }
     }
   }
-  __syncthreads();
-  const float Na = __uint_as_float(sNa_bits);
-  float cmax[kD];
-#pragma unroll
-  for (int j = 0; j < kD; ++j) cmax[j] = __uint_as_float(sCmax_bits[j]);
 #pragma unroll
   for (int v = 0; v < VPT; ++v) {
-    if (!live[v]) continue;
     const int64_t i = row0 + threadIdx.x + (int64_t)v * kThreads;
-    // Error bound E = C u (Na + 2 sum_p P_p cmax_p), P_p = sum_j |H_pj| (|t_j| + sum |c_f,j|).
-    float r[kD], a[kD];
-    target32(set, cbs, n_fixed, i, g, r, a, err);
-    float sc = Na;
-#pragma unroll
-    for (int p = 0; p < kD; ++p) {
-      float pa = 0.f;
-#pragma unroll
-      for (int j = 0; j < kD; ++j) pa = fmaf(fabsf(sH[p * kD + j]), a[j], pa);
-      sc = fmaf(2.f * pa, cmax[p], sc);
-    }
-    const float E = (160.f + 8.f * n_fixed) * kU * sc;
-    if (!(b2[v] - b1[v] > 2.f * E)) {
+    if (i >= set.M) continue;
+    // Winner's bound Et_j = u C (Na_j + 2 Pmax L1_j), recomputed from c_j.
+    float c[kD];
+    load_vec(cw.C + (int64_t)i1[v] * kD, c);
+    float n, na, l1;
+    codeword_terms(c, sH, n, na, l1);
+    const float Et = kU * cmul * na - 0.5f * nbeta[v] * l1;
+    const bool cert = b2[v] - b1[v] > 2.f * Et;
+    if (!cert) {
       const unsigned slot = atomicAdd(flags.count, 1u);
       if (slot < flags.cap) {
         flags.vec[slot] = i * G_range + (g - g_begin);
-        flags.thr[slot] = b1[v] + 2.f * E;
+        flags.thr[slot] = b1[v] + 2.f * Et;
       } else {
         raise_error(err, ERRBIT_INDEX);
       }
     }
     // Always write the fast-pass winner; the fallback overwrites uncertain ones.
     out_code[i * out_ld + (g - out_g0)] = i1[v];
+    if (cert && st.cnt) {
+      float q[kD];
+#pragma unroll
+      for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[v][p];
+      stats_add(st, *st.scale, g, i1[v], q);
+    }
   }
 }
 
-// Fallback: one warp per flagged vector. Re-scores every codeword in fp32; candidates whose
-// score is within the threshold are re-scored in fp64; the smallest fp64 err wins (ties to the
-// smaller index).
+// Fallback: one warp per flagged vector. Recomputes low_k for every codeword; those with
+// low_k <= threshold are re-scored in fp64 and the smallest fp64 err wins (ties to the
+// smaller index). Adds the statistics of the decided code when requested.
 __global__ void __launch_bounds__(kThreads)
 argmin_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs,
                        int n_fixed, int s_idx, int32_t* __restrict__ out_code,
-                       int64_t out_ld, int64_t out_g0, FlagList flags, unsigned* err) {
+                       int64_t out_ld, int64_t out_g0, FlagList flags, StatsView st,
+                       unsigned* err) {
   const int lane = threadIdx.x & 31;
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const unsigned cnt = min((unsigned long long)*flags.count, (unsigned long long)flags.cap);
+  if (flags.total && blockIdx.x == 0 && threadIdx.x == 0) atomicAdd(flags.total, cnt);
   const CbView cw = cbs.cb[s_idx];
+  const float cmul = bound_mult(n_fixed);
   for (int64_t f = warp; f < cnt; f += nwarps) {
     const int64_t vi = flags.vec[f];
     const int64_t i = vi / G_range, g = g_begin + vi % G_range;
     const float thr = flags.thr[f];
     const float* H = set.Hb + g * kD * kD;
-    float r[kD], a[kD], m2q[kD];
+    float r[kD], a[kD], m2q[kD], pmax;
     target32(set, cbs, n_fixed, i, g, r, a, err);
+    vector_terms(r, a, H, m2q, pmax);
+    const float nbeta = -2.f * kU * cmul * pmax;
     double r64[kD];
     target64(set, cbs, n_fixed, i, g, r64, err);
-#pragma unroll
-    for (int p = 0; p < kD; ++p) {
-      float q = 0.f;
-#pragma unroll
-      for (int j = 0; j < kD; ++j) q = fmaf(H[p * kD + j], r[j], q);
-      m2q[p] = -2.f * q;
-    }
     double best = INFINITY;
     int bestk = 0x7fffffff;
     for (int k = lane; k < cw.K; k += 32) {
       float c[kD];
       load_vec(cw.C + (int64_t)k * kD, c);
-      float n = 0.f;
-#pragma unroll
-      for (int p = 0; p < kD; ++p) {
-        float u = 0.f;
-#pragma unroll
-        for (int j = 0; j < kD; ++j) u = fmaf(H[p * kD + j], c[j], u);
-        n = fmaf(c[p], u, n);
-      }
-      float s = n;
-#pragma unroll
-      for (int p = 0; p < kD; ++p) s = fmaf(m2q[p], c[p], s);
-      if (s <= thr) {
+      if (low_score(c, H, m2q, nbeta, cmul) <= thr) {
         const double e = quad_err64(r64, cw.C + (int64_t)k * kD, H);
         if (e < best || (e == best && k < bestk)) {
           best = e;
@@ -309,6 +331,12 @@ argmin_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs
         raise_error(err, ERRBIT_NUMERIC);  // no candidate: non-finite scores
       } else {
         out_code[i * out_ld + (g - out_g0)] = bestk;
+        if (st.cnt) {
+          float q[kD];
+#pragma unroll
+          for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[p];
+          stats_add(st, *st.scale, g, bestk, q);
+        }
       }
     }
   }
@@ -332,7 +360,7 @@ struct StageDesc {
   int Bs;                 // hypotheses kept by the current stage (1 at the last stage)
 };
 
-// fp64 residual of hypothesis h before stage s: target - sum_{s' < s} C_{st[s']}[code].
+// fp64 residual of a hypothesis before stage s: target - sum_{s' < s} C_{st[s']}[code].
 __device__ void hyp_residual64(const double tgt[kD], const CbList& cbs, const StageDesc& sd,
                                const int32_t* codes, double r[kD], unsigned* err) {
 #pragma unroll
@@ -347,8 +375,33 @@ __device__ void hyp_residual64(const double tgt[kD], const CbList& cbs, const St
   }
 }
 
+// Per-hypothesis terms of the approximate err: m2q = -2 H r, rr = r^T H r (r rounded to
+// fp32), and the bound pieces Ra = |r|^T |H| |r|, Pmax = max_p (|H| |r|)_p.
+__device__ __forceinline__ void hyp_terms(const double r64[kD], const float* H, float m2q[kD],
+                                          float& rr, float& ra, float& pmax) {
+  float r[kD];
+#pragma unroll
+  for (int j = 0; j < kD; ++j) r[j] = (float)r64[j];
+  rr = 0.f;
+  ra = 0.f;
+  pmax = 0.f;
+#pragma unroll
+  for (int p = 0; p < kD; ++p) {
+    float q = 0.f, pa = 0.f;
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      q = fmaf(H[p * kD + j], r[j], q);
+      pa = fmaf(fabsf(H[p * kD + j]), fabsf(r[j]), pa);
+    }
+    m2q[p] = -2.f * q;
+    rr = fmaf(r[p], q, rr);
+    ra = fmaf(fabsf(r[p]), pa, ra);
+    pmax = fmaxf(pmax, pa);
+  }
+}
+
 // Fast stage: one thread per vector, the stage codebook chunked through shared memory, a
-// sorted top-L list (L >= B + 1) of approximate errs in registers.
+// sorted top-L list (L >= Bs + 1) of lower bounds low = approx_err - Et in registers.
 template <int L>
 __global__ void __launch_bounds__(kThreads)
 beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc sd,
@@ -360,15 +413,13 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
   const int64_t vi = live ? i * G_range + (g - g_begin) : 0;
   __shared__ float sH[kD * kD];
   __shared__ __align__(16) float sC[kChunk * kD];
-  __shared__ float sN[kChunk];
-  __shared__ unsigned sNa_bits, sCmax_bits[kD];
+  __shared__ float sN[kChunk], sL[kChunk];
   if (threadIdx.x < kD * kD) sH[threadIdx.x] = set.Hb[g * kD * kD + threadIdx.x];
-  if (threadIdx.x < kD) sCmax_bits[threadIdx.x] = 0u;
-  if (threadIdx.x == 0) sNa_bits = 0u;
   __syncthreads();
 
   const CbView cw = cbs.cb[sd.st[sd.s]];
   const int S = sd.S, B = sd.B, Bs = sd.Bs;
+  const float cmul = bound_mult(n_fixed + sd.s);
   const int Bh = (sd.s == 0) ? 1 : (live ? bb.n_in[vi] : 1);
   double tgt[kD];
   if (live) {
@@ -386,32 +437,25 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
     toph[j] = 0x7fffffff;
     topk[j] = 0x7fffffff;
   }
+
   for (int k0 = 0; k0 < cw.K; k0 += kChunk) {
     const int nk = min(kChunk, cw.K - k0);
     __syncthreads();
-    stage_chunk(cw.C, k0, nk, sH, sC, sN, &sNa_bits, sCmax_bits);
+    stage_chunk(cw.C, k0, nk, sH, cmul, sC, sN, sL);
     __syncthreads();
     if (!live) continue;
     for (int h = 0; h < Bh; ++h) {
       double r64[kD];
       const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
       hyp_residual64(tgt, cbs, sd, pc, r64, err);
-      float r[kD], m2q[kD];
-#pragma unroll
-      for (int j = 0; j < kD; ++j) r[j] = (float)r64[j];
-      float rr = 0.f;
-#pragma unroll
-      for (int p = 0; p < kD; ++p) {
-        float q = 0.f;
-#pragma unroll
-        for (int j = 0; j < kD; ++j) q = fmaf(sH[p * kD + j], r[j], q);
-        m2q[p] = -2.f * q;
-        rr = fmaf(r[p], q, rr);
-      }
+      float m2q[kD], rr, ra, pmax;
+      hyp_terms(r64, sH, m2q, rr, ra, pmax);
+      const float base = rr - kU * cmul * ra;
+      const float nbeta = -2.f * kU * cmul * pmax;
       for (int k = 0; k < nk; ++k) {
         const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
         const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
-        float s = rr + sN[k];
+        float s = base + sN[k];
         s = fmaf(m2q[0], c0.x, s);
         s = fmaf(m2q[1], c0.y, s);
         s = fmaf(m2q[2], c0.z, s);
@@ -420,6 +464,7 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
         s = fmaf(m2q[5], c1.y, s);
         s = fmaf(m2q[6], c1.z, s);
         s = fmaf(m2q[7], c1.w, s);
+        s = fmaf(nbeta, sL[k], s);
         if (s < topv[L - 1]) {
           float sv = s;
           int sh = h, sk = k0 + k;
@@ -436,106 +481,87 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
       }
     }
   }
-  __syncthreads();
   if (!live) return;
 
-  // Error bound: E = C u (Ra + Na + 2 sum_j P_j cmax_j) maximised over parents, where
-  // P_j = sum_l |H_jl| |r_l|. The P-term is recomputed here with the final cmax.
-  const float Na = __uint_as_float(sNa_bits);
-  float scale = 0.f;
-  for (int h = 0; h < Bh; ++h) {
-    double r64[kD];
-    const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
-    hyp_residual64(tgt, cbs, sd, pc, r64, err);
-    float ra = 0.f, pc2 = 0.f;
-#pragma unroll
-    for (int p = 0; p < kD; ++p) {
-      float pa = 0.f;
-#pragma unroll
-      for (int j = 0; j < kD; ++j) pa = fmaf(fabsf(sH[p * kD + j]), fabsf((float)r64[j]), pa);
-      ra = fmaf(fabsf((float)r64[p]), pa, ra);
-      pc2 = fmaf(pa, __uint_as_float(sCmax_bits[p]), pc2);
-    }
-    scale = fmaxf(scale, ra + Na + 2.f * pc2);
-  }
-  const float E = (160.f + 8.f * (n_fixed + sd.s)) * kU * scale;
-
   const int64_t total = (int64_t)Bh * cw.K;
+  const int nkept = (int)min((int64_t)L, total);
   const int keep = (int)min((int64_t)Bs, total);
   // Non-finite scores never enter the list; keep indices valid and report it.
 #pragma unroll
   for (int j = 0; j < L; ++j) {
-    if (j < min((int64_t)L, total) && (toph[j] >= Bh || topk[j] >= cw.K)) {
+    if (j < nkept && (toph[j] >= Bh || topk[j] >= cw.K)) {
       raise_error(err, ERRBIT_NUMERIC);
       toph[j] = 0;
       topk[j] = 0;
     }
   }
-  const bool all_kept = total <= L;
-  // Fast certificate: the gaps between consecutive entries j -> j+1, j < min(keep, total-1),
-  // exceed 2E (every candidate outside the list scores at least the last list entry).
-  bool ok = true;
-  const int lim = (int)min((int64_t)keep, total - 1);
-#pragma unroll
-  for (int j = 0; j < L - 1; ++j)
-    if (j < lim && !(topv[j + 1] - topv[j] > 2.f * E)) ok = false;
-
-  int32_t* out = bb.hyp_out + vi * B * S;
-  if (ok) {
-#pragma unroll
-    for (int j = 0; j < L; ++j) {
-      if (j >= keep) break;
-      const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
-      for (int q = 0; q < sd.s; ++q) out[j * S + q] = pc[q];
-      out[j * S + sd.s] = topk[j];
-    }
-    bb.n_out[vi] = keep;
-    return;
-  }
-  // Exact path on the kept candidates: fp64 errs, exact (err, h, k) order, then the boundary
-  // certificate a_L - E > e_(keep).
-  const int nkept = (int)min((int64_t)L, total);
-  double ev[L];
+  // Per-entry bound Et = u C (Ra_h + Na_k + 2 Pmax_h L1_k) for the listed entries.
+  float et[L];
 #pragma unroll
   for (int j = 0; j < L; ++j) {
-    ev[j] = INFINITY;
+    et[j] = 0.f;
     if (j < nkept) {
       double r64[kD];
       const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
       hyp_residual64(tgt, cbs, sd, pc, r64, err);
-      ev[j] = quad_err64(r64, cw.C + (int64_t)topk[j] * kD, sH);
+      float m2q[kD], rr, ra, pmax;
+      hyp_terms(r64, sH, m2q, rr, ra, pmax);
+      float c[kD], n, na, l1;
+      load_vec(cw.C + (int64_t)topk[j] * kD, c);
+      codeword_terms(c, sH, n, na, l1);
+      et[j] = kU * cmul * (ra + na + 2.f * pmax * l1);
     }
   }
-  // insertion sort by (ev, h, k)
+  // Fast certificate: low_{j+1} - low_j > 2 Et_j for j < min(keep, total - 1) (every
+  // candidate outside the list has low >= the last list entry).
+  bool ok = true;
+  const int lim = (int)min((int64_t)keep, total - 1);
 #pragma unroll
-  for (int a = 1; a < L; ++a) {
+  for (int j = 0; j < L - 1; ++j)
+    if (j < lim && !(topv[j + 1] - topv[j] > 2.f * et[j])) ok = false;
+
+  int32_t* out = bb.hyp_out + vi * B * S;
+  if (!ok) {
+    // Exact path on the listed candidates: fp64 errs, exact (err, h, k) order; then every
+    // unlisted candidate must have low >= the last listed low > the keep-th exact err.
+    double ev[L];
 #pragma unroll
-    for (int b = a; b > 0; --b) {
-      const bool sw = (ev[b] < ev[b - 1]) ||
-                      (ev[b] == ev[b - 1] &&
-                       (toph[b] < toph[b - 1] || (toph[b] == toph[b - 1] && topk[b] < topk[b - 1])));
-      if (sw) {
-        const double te = ev[b]; ev[b] = ev[b - 1]; ev[b - 1] = te;
-        const int th = toph[b]; toph[b] = toph[b - 1]; toph[b - 1] = th;
-        const int tk = topk[b]; topk[b] = topk[b - 1]; topk[b - 1] = tk;
-        const float tv = topv[b]; topv[b] = topv[b - 1]; topv[b - 1] = tv;
+    for (int j = 0; j < L; ++j) {
+      ev[j] = INFINITY;
+      if (j < nkept) {
+        double r64[kD];
+        const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
+        hyp_residual64(tgt, cbs, sd, pc, r64, err);
+        ev[j] = quad_err64(r64, cw.C + (int64_t)topk[j] * kD, sH);
       }
     }
-  }
-  float amax = -INFINITY;
+    const float last_low = topv[nkept - 1];
 #pragma unroll
-  for (int j = 0; j < L; ++j)
-    if (j < nkept) amax = fmaxf(amax, topv[j]);
-  const bool cert = all_kept || ((double)amax - (double)E > ev[keep - 1]);
-  if (!cert) {
-    const unsigned slot = atomicAdd(flags.count, 1u);
-    if (slot < flags.cap) {
-      flags.vec[slot] = vi;
-      flags.thr[slot] = 0.f;
-    } else {
-      raise_error(err, ERRBIT_INDEX);
+    for (int a = 1; a < L; ++a) {
+#pragma unroll
+      for (int b = a; b > 0; --b) {
+        const bool sw = (ev[b] < ev[b - 1]) ||
+                        (ev[b] == ev[b - 1] &&
+                         (toph[b] < toph[b - 1] ||
+                          (toph[b] == toph[b - 1] && topk[b] < topk[b - 1])));
+        if (sw) {
+          const double te = ev[b]; ev[b] = ev[b - 1]; ev[b - 1] = te;
+          const int th = toph[b]; toph[b] = toph[b - 1]; toph[b - 1] = th;
+          const int tk = topk[b]; topk[b] = topk[b - 1]; topk[b - 1] = tk;
+        }
+      }
     }
-    return;
+    const bool cert = total <= L || (double)last_low > ev[keep - 1];
+    if (!cert) {
+      const unsigned slot = atomicAdd(flags.count, 1u);
+      if (slot < flags.cap) {
+        flags.vec[slot] = vi;
+        flags.thr[slot] = 0.f;
+      } else {
+        raise_error(err, ERRBIT_INDEX);
+      }
+      return;
+    }
   }
 #pragma unroll
   for (int j = 0; j < L; ++j) {
@@ -547,16 +573,21 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
   bb.n_out[vi] = keep;
 }
 
-// Exact stage for flagged vectors: one thread per vector, every (h, k) candidate in fp64,
-// sorted top-B by (err, h, k) kept in local memory.
-__global__ void beam_stage_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range,
-                                           CbList cbs, int n_fixed, StageDesc sd, BeamBufs bb,
-                                           FlagList flags, unsigned* err) {
+// Exact stage for flagged vectors: one warp per vector; the lanes stride over the (h, k)
+// candidates in fp64 keeping a sorted local top-Bs; a warp merge then extracts the global
+// top-Bs in (err, h, k) order.
+__global__ void __launch_bounds__(kThreads)
+beam_stage_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs,
+                           int n_fixed, StageDesc sd, BeamBufs bb, FlagList flags,
+                           unsigned* err) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const unsigned cnt = min((unsigned long long)*flags.count, (unsigned long long)flags.cap);
+  if (flags.total && blockIdx.x == 0 && threadIdx.x == 0) atomicAdd(flags.total, cnt);
   const int S = sd.S, B = sd.B, Bs = sd.Bs;
   const CbView cw = cbs.cb[sd.st[sd.s]];
-  for (int64_t f = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; f < cnt;
-       f += (int64_t)gridDim.x * blockDim.x) {
+  for (int64_t f = warp; f < cnt; f += nwarps) {
     const int64_t vi = flags.vec[f];
     const int64_t i = vi / G_range, g = g_begin + vi % G_range;
     const float* H = set.Hb + g * kD * kD;
@@ -570,9 +601,10 @@ __global__ void beam_stage_fallback_kernel(SetView set, int64_t g_begin, int64_t
       double r64[kD];
       const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
       hyp_residual64(tgt, cbs, sd, pc, r64, err);
-      for (int k = 0; k < cw.K; ++k) {
+      for (int k = lane; k < cw.K; k += 32) {
         const double e = quad_err64(r64, cw.C + (int64_t)k * kD, H);
-        // candidates arrive in (h, k) order: strict comparison keeps the earlier on ties
+        // this lane sees its candidates in increasing (h, k): strict comparison keeps ties
+        // in (h, k) order
         if (nb < Bs || e < be[nb - 1]) {
           int pos = nb < Bs ? nb : Bs - 1;
           while (pos > 0 && e < be[pos - 1]) {
@@ -584,13 +616,39 @@ __global__ void beam_stage_fallback_kernel(SetView set, int64_t g_begin, int64_t
         }
       }
     }
+    // Warp merge: rounds of (min over the lanes' heads by (err, h, k)); the winner pops.
+    int head = 0;
     int32_t* out = bb.hyp_out + vi * B * S;
-    for (int j = 0; j < nb; ++j) {
-      const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + bh[j]) * S : nullptr;
-      for (int q = 0; q < sd.s; ++q) out[j * S + q] = pc[q];
-      out[j * S + sd.s] = bk[j];
+    const int total = (int)min((int64_t)Bs, (int64_t)Bh * cw.K);
+    for (int j = 0; j < total; ++j) {
+      double e = head < nb ? be[head] : INFINITY;
+      int hh = head < nb ? bh[head] : 0x7fffffff;
+      int kk = head < nb ? bk[head] : 0x7fffffff;
+      int src = lane;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const double oe = __shfl_xor_sync(0xffffffffu, e, off);
+        const int oh = __shfl_xor_sync(0xffffffffu, hh, off);
+        const int ok = __shfl_xor_sync(0xffffffffu, kk, off);
+        const int os = __shfl_xor_sync(0xffffffffu, src, off);
+        const bool take = oe < e || (oe == e && (oh < hh || (oh == hh && ok < kk)));
+        if (take) {
+          e = oe; hh = oh; kk = ok; src = os;
+        }
+      }
+      if (lane == src) ++head;
+      if (lane == 0) {
+        if (hh >= Bh || kk >= cw.K) {
+          raise_error(err, ERRBIT_NUMERIC);
+          hh = 0;
+          kk = 0;
+        }
+        const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + hh) * S : nullptr;
+        for (int q = 0; q < sd.s; ++q) out[j * S + q] = pc[q];
+        out[j * S + sd.s] = kk;
+      }
     }
-    bb.n_out[vi] = nb;
+    if (lane == 0) bb.n_out[vi] = total;
   }
 }
 
@@ -606,12 +664,12 @@ __global__ void beam_finalize_kernel(SetView set, int64_t g_begin, int64_t G_ran
        vi += (int64_t)gridDim.x * blockDim.x) {
     const int64_t i = vi / G_range, g = g_begin + vi % G_range;
     const float* H = set.Hb + g * kD * kD;
-    double tgt[kD];
-    target64(set, cbs, n_fixed, i, g, tgt, err);
     const int32_t* best = hyp + vi * B * S;
     bool use_old = false;
     double e_new = 0.0, e_old = 0.0;
     if (keep_if_better || vec_err) {
+      double tgt[kD];
+      target64(set, cbs, n_fixed, i, g, tgt, err);
       double r[kD];
 #pragma unroll
       for (int j = 0; j < kD; ++j) r[j] = tgt[j];
@@ -623,21 +681,20 @@ __global__ void beam_finalize_kernel(SetView set, int64_t g_begin, int64_t G_ran
         for (int j = 0; j < kD; ++j) r[j] -= (double)c[j];
       }
       e_new = quad_err64(r, nullptr, H);
-    }
-    if (keep_if_better) {
-      double r[kD];
+      if (keep_if_better) {
 #pragma unroll
-      for (int j = 0; j < kD; ++j) r[j] = tgt[j];
-      for (int q = 0; q < S; ++q) {
-        const CbView& cb = cbs.cb[sd.st[q]];
-        const int32_t k = cb.codes[i * cb.ld + g];
-        if (!code_ok(k, cb.K, err)) continue;
-        const float* c = cb.C + (int64_t)k * kD;
+        for (int j = 0; j < kD; ++j) r[j] = tgt[j];
+        for (int q = 0; q < S; ++q) {
+          const CbView& cb = cbs.cb[sd.st[q]];
+          const int32_t k = cb.codes[i * cb.ld + g];
+          if (!code_ok(k, cb.K, err)) continue;
+          const float* c = cb.C + (int64_t)k * kD;
 #pragma unroll
-        for (int j = 0; j < kD; ++j) r[j] -= (double)c[j];
+          for (int j = 0; j < kD; ++j) r[j] -= (double)c[j];
+        }
+        e_old = quad_err64(r, nullptr, H);
+        use_old = e_old < e_new;
       }
-      e_old = quad_err64(r, nullptr, H);
-      use_old = e_old < e_new;
     }
     if (!use_old) {
       for (int q = 0; q < S; ++q) {
@@ -649,8 +706,7 @@ __global__ void beam_finalize_kernel(SetView set, int64_t g_begin, int64_t G_ran
   }
 }
 
-// err of the tuple currently in the codes (fixed + searched) for vectors that no searched
-// codebook covers.
+// err of the tuple currently in the codes (all covering codebooks), fp64.
 __global__ void residual_err_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs,
                                     float* __restrict__ vec_err, unsigned* err) {
   const int64_t nvec = set.M * G_range;
@@ -700,9 +756,9 @@ template <int L>
 crvq_status launch_beam_stage_L(const SetView& set, int64_t g_begin, int64_t G_range,
                                 const CbList& cbs, int n_fixed, const StageDesc& sd,
                                 const BeamBufs& bb, const FlagList& fl, unsigned* err,
-                                cudaStream_t stream) {
+                                double units, cudaStream_t stream) {
   dim3 grid((unsigned)ceil_div(set.M, kThreads), (unsigned)G_range);
-  ProfScope ps("encode_beam_stage", stream, 0.0);
+  ProfScope ps("encode_beam_stage", stream, units);
   beam_stage_kernel<L><<<grid, kThreads, 0, stream>>>(set, g_begin, cbs, n_fixed, sd, bb, fl,
                                                      err);
   CRVQ_LAUNCHED();
@@ -712,19 +768,20 @@ crvq_status launch_beam_stage_L(const SetView& set, int64_t g_begin, int64_t G_r
 crvq_status launch_beam_stage(const SetView& set, int64_t g_begin, int64_t G_range,
                               const CbList& cbs, int n_fixed, const StageDesc& sd,
                               const BeamBufs& bb, const FlagList& fl, unsigned* err,
-                              cudaStream_t stream) {
+                              double units, cudaStream_t stream) {
   const int need = sd.Bs + 1;
-  if (need <= 2) return launch_beam_stage_L<2>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, stream);
-  if (need <= 3) return launch_beam_stage_L<3>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, stream);
-  if (need <= 5) return launch_beam_stage_L<5>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, stream);
-  if (need <= 9) return launch_beam_stage_L<9>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, stream);
-  return launch_beam_stage_L<17>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, stream);
+  if (need <= 2) return launch_beam_stage_L<2>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
+  if (need <= 3) return launch_beam_stage_L<3>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
+  if (need <= 5) return launch_beam_stage_L<5>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
+  if (need <= 9) return launch_beam_stage_L<9>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
+  return launch_beam_stage_L<17>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
 }
 
 // One range of groups [g_begin, g_begin + G_range) whose searched stages are sd.st[0..S).
 crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
                          const CbList& cbs, int n_fixed, StageDesc sd, bool keep_if_better,
-                         float* vec_err, double* scores, unsigned* err, cudaStream_t stream) {
+                         float* vec_err, const EncodeExtras& ex, unsigned* err,
+                         cudaStream_t stream) {
   const int64_t nvec = set.M * G_range;
   if (nvec == 0) return CRVQ_OK;
   const int nsm = sm_count();
@@ -745,6 +802,7 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
   fl.vec = reinterpret_cast<int64_t*>(flag_mem.as<char>() + 256);
   fl.thr = reinterpret_cast<float*>(fl.vec + nvec);
   fl.cap = nvec;
+  fl.total = ex.flag_total;
 
   if (sd.S == 1) {
     // Arg-min over one codebook (the k-means assignment step). Written in place unless the
@@ -761,25 +819,31 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
       out_ld = G_range;
       out_g0 = g_begin;
     }
+    StatsView st{};
+    if (ex.stats && !keep_if_better) st = *ex.stats;
     CRVQ_CUDA(cudaMemsetAsync(fl.count, 0, sizeof(unsigned), stream));
     const bool big = (ceil_div(set.M, kThreads * 4) * G_range) >= 2 * nsm;
-    ProfScope ps("encode_argmin", stream, (double)nvec * cw.K);
-    if (big) {
-      dim3 grid((unsigned)ceil_div(set.M, kThreads * 4), (unsigned)G_range);
-      argmin_kernel<4><<<grid, kThreads, 0, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                      out_ld, out_g0, fl, err);
-    } else {
-      dim3 grid((unsigned)ceil_div(set.M, kThreads), (unsigned)G_range);
-      argmin_kernel<1><<<grid, kThreads, 0, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                      out_ld, out_g0, fl, err);
+    {
+      ProfScope ps("encode_argmin", stream, (double)nvec * cw.K);
+      if (big) {
+        dim3 grid((unsigned)ceil_div(set.M, kThreads * 4), (unsigned)G_range);
+        argmin_kernel<4><<<grid, kThreads, 0, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
+                                                        out_ld, out_g0, fl, st, err);
+      } else {
+        dim3 grid((unsigned)ceil_div(set.M, kThreads), (unsigned)G_range);
+        argmin_kernel<1><<<grid, kThreads, 0, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
+                                                        out_ld, out_g0, fl, st, err);
+      }
+      CRVQ_LAUNCHED();
     }
-    CRVQ_LAUNCHED();
-    ProfScope ps2("encode_argmin_fallback", stream, 0.0);
-    argmin_fallback_kernel<<<4 * nsm, kThreads, 0, stream>>>(set, g_begin, G_range, cbs,
-                                                             n_fixed, s_idx, out, out_ld,
-                                                             out_g0, fl, err);
-    CRVQ_LAUNCHED();
-    if (scores) *scores += (double)nvec * cw.K;
+    {
+      ProfScope ps2("encode_argmin_fallback", stream, 0.0);
+      argmin_fallback_kernel<<<4 * nsm, kThreads, 0, stream>>>(set, g_begin, G_range, cbs,
+                                                               n_fixed, s_idx, out, out_ld,
+                                                               out_g0, fl, st, err);
+      CRVQ_LAUNCHED();
+    }
+    if (ex.scores) *ex.scores += (double)nvec * cw.K;
     ProfScope ps3("encode_finalize", stream, 0.0);
     if (keep_if_better) {
       StageDesc one = sd;
@@ -816,14 +880,15 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     sd.Bs = (s == S - 1) ? 1 : B;  // only the best tuple of the last stage is used
     CRVQ_CUDA(cudaMemsetAsync(fl.count, 0, sizeof(unsigned), stream));
     BeamBufs bb{in_h, in_n, out_h, out_n};
-    CRVQ_TRY(launch_beam_stage(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, stream));
+    const int K = cbs.cb[sd.st[s]].K;
+    CRVQ_TRY(launch_beam_stage(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err,
+                               (double)nvec * parents * K, stream));
     {
       ProfScope ps("encode_beam_fallback", stream, 0.0);
-      beam_stage_fallback_kernel<<<std::max(1, nsm), 128, 0, stream>>>(
+      beam_stage_fallback_kernel<<<4 * nsm, kThreads, 0, stream>>>(
           set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err);
       CRVQ_LAUNCHED();
     }
-    const int K = cbs.cb[sd.st[s]].K;
     sc += (double)nvec * parents * K;
     parents = std::min<int64_t>(B, parents * K);
     in_h = out_h;
@@ -831,7 +896,7 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     out_h = (out_h == hypA) ? hypB : hypA;
     out_n = (out_n == nA) ? nB : nA;
   }
-  if (scores) *scores += sc;
+  if (ex.scores) *ex.scores += sc;
   ProfScope ps("encode_finalize", stream, 0.0);
   beam_finalize_kernel<<<fin_blocks, 128, 0, stream>>>(set, g_begin, G_range, cbs, n_fixed, sd,
                                                        in_h, keep_if_better, vec_err, err);
@@ -842,7 +907,7 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
 }  // namespace
 
 crvq_status launch_encode_beam(const SetView& set, const CbList& cbs, int n_fixed, int B,
-                               bool keep_if_better, float* vec_err, double* scores,
+                               bool keep_if_better, float* vec_err, const EncodeExtras& ex,
                                cudaStream_t stream) {
   unsigned* err = nullptr;
   CRVQ_TRY(device_error_word(&err));
@@ -852,6 +917,8 @@ crvq_status launch_encode_beam(const SetView& set, const CbList& cbs, int n_fixe
     if (cbs.cb[s].G_cov > 0 && cbs.cb[s].G_cov < set.G_sub) cuts.push_back(cbs.cb[s].G_cov);
   std::sort(cuts.begin(), cuts.end());
   cuts.erase(std::unique(cuts.begin(), cuts.end()), cuts.end());
+  if (ex.stats && cuts.size() > 2)
+    return fail(CRVQ_ERR_UNSUPPORTED, "fused statistics need one group range");
   for (size_t r = 0; r + 1 < cuts.size(); ++r) {
     const int64_t g0 = cuts[r], g1 = cuts[r + 1];
     StageDesc sd{};
@@ -860,8 +927,8 @@ crvq_status launch_encode_beam(const SetView& set, const CbList& cbs, int n_fixe
     sd.Bs = B;
     for (int s = n_fixed; s < cbs.n; ++s)
       if (g0 < cbs.cb[s].G_cov) sd.st[sd.S++] = s;
-    CRVQ_TRY(encode_range(set, g0, g1 - g0, cbs, n_fixed, sd, keep_if_better, vec_err, scores,
-                          err, stream));
+    CRVQ_TRY(encode_range(set, g0, g1 - g0, cbs, n_fixed, sd, keep_if_better, vec_err, ex, err,
+                          stream));
   }
   return CRVQ_OK;
 }

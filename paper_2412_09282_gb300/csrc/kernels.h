@@ -31,10 +31,18 @@ crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
 crvq_status launch_kmeans_init(const SetView& set, const CbList& fixed, int K, uint64_t seed,
                                float* C_out, cudaStream_t stream);
 
-// Encode / beam (see crvq_encode_beam). `scores` (may be null) accumulates the number of
-// (hypothesis, codeword) pairs the launch scores.
+struct StatsView;
+
+// Optional extras of an encode launch.
+struct EncodeExtras {
+  double* scores = nullptr;                // host: += (hypothesis, codeword) pairs scored
+  const StatsView* stats = nullptr;        // accumulate LS statistics of the written codes
+  unsigned long long* flag_total = nullptr;  // device: += vectors sent to the fp64 fallback
+};
+
+// Encode / beam (see crvq_encode_beam).
 crvq_status launch_encode_beam(const SetView& set, const CbList& cbs, int n_fixed, int B,
-                               bool keep_if_better, float* vec_err, double* scores,
+                               bool keep_if_better, float* vec_err, const EncodeExtras& ex,
                                cudaStream_t stream);
 
 crvq_status launch_update_codebook(const SetView& set, const CbList& cbs, int which,

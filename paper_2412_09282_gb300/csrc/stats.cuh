@@ -1,0 +1,122 @@
+// Least-squares statistics of one codebook, shared by the standalone update (update.cu) and
+// the Lloyd encode pass that accumulates them for the codes it writes (encode.cu).
+//
+//   cnt[g][k]  exact count of members of code k in group g (int32)
+//   bacc[k][j] sum over members v of code k of (H_{g_v} tau_v)_j, as 64-bit fixed point
+//   scale      the power of two used for the fixed point (chosen from a bound on the terms)
+//
+// Integer accumulation makes the sums independent of the order in which threads add, so the
+// solve sees identical inputs on every run.
+#pragma once
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace crvq {
+
+struct StatsView {
+  int32_t* cnt;     // [G_cov][K]
+  long long* bacc;  // [K][d]
+  double* scale;    // device scalar
+  int64_t G_cov;
+  int K;
+};
+
+// 2^e with e the largest integer such that n * bound * 2^e < 2^62.
+__host__ __device__ inline double stats_scale_for(double bound, int64_t n) {
+  const double lim = 4.611686018427387904e18;  // 2^62
+  const double denom = bound * (double)(n > 0 ? n : 1);
+  if (!(denom > 0.0)) return 1099511627776.0;  // 2^40: nothing to scale
+  const int e = (int)floor(log2(lim / denom));
+  return ldexp(1.0, e < -1000 ? -1000 : (e > 1000 ? 1000 : e));
+}
+
+// tau = t - sum over the codebooks s != which that cover g of C_s[code] (fp32, codebook order).
+__device__ __forceinline__ void stats_target(const SetView& set, const CbList& cbs, int which,
+                                             int64_t i, int64_t g, float tau[kD],
+                                             unsigned* err) {
+  const float* t = set.T + i * set.ldT + g * kD;
+  const float4 t0 = *reinterpret_cast<const float4*>(t);
+  const float4 t1 = *reinterpret_cast<const float4*>(t + 4);
+  tau[0] = t0.x; tau[1] = t0.y; tau[2] = t0.z; tau[3] = t0.w;
+  tau[4] = t1.x; tau[5] = t1.y; tau[6] = t1.z; tau[7] = t1.w;
+  for (int s = 0; s < cbs.n; ++s) {
+    if (s == which) continue;
+    const CbView& cb = cbs.cb[s];
+    if (g >= cb.G_cov) continue;
+    const int32_t k = cb.codes[i * cb.ld + g];
+    if (k < 0 || k >= cb.K) {
+      raise_error(err, ERRBIT_INDEX);
+      continue;
+    }
+    const float* c = cb.C + (int64_t)k * kD;
+#pragma unroll
+    for (int j = 0; j < kD; ++j) tau[j] -= c[j];
+  }
+}
+
+// q = H tau, each row an FMA chain over the columns in order (the encode pass evaluates
+// H r the same way, so both paths produce bit-identical contributions).
+__device__ __forceinline__ void stats_htau(const float* H, const float tau[kD], float q[kD]) {
+#pragma unroll
+  for (int r = 0; r < kD; ++r) {
+    float a = 0.f;
+#pragma unroll
+    for (int c = 0; c < kD; ++c) a = fmaf(H[r * kD + c], tau[c], a);
+    q[r] = a;
+  }
+}
+
+__device__ __forceinline__ void stats_add(const StatsView& st, double scale, int64_t g, int k,
+                                          const float q[kD]) {
+  atomicAdd(&st.cnt[g * st.K + k], 1);
+#pragma unroll
+  for (int j = 0; j < kD; ++j) {
+    const long long v = __double2ll_rn((double)q[j] * scale);
+    atomicAdd(reinterpret_cast<unsigned long long*>(&st.bacc[(int64_t)k * kD + j]),
+              (unsigned long long)v);
+  }
+}
+
+// Solves A x = b for a symmetric positive definite 8 x 8 A given as its packed lower
+// triangle (row-major, A[r(r+1)/2 + c] for c <= r). Returns false when A is not SPD.
+__device__ inline bool cholesky_solve8(const double A[36], const double b[kD], double x[kD]) {
+  double L[36];
+  int q = 0;
+  for (int r = 0; r < kD; ++r) {
+    for (int c = 0; c <= r; ++c, ++q) {
+      double s = A[q];
+      for (int m = 0; m < c; ++m) s -= L[r * (r + 1) / 2 + m] * L[c * (c + 1) / 2 + m];
+      if (r == c) {
+        if (!(s > 0.0)) return false;
+        L[q] = sqrt(s);
+      } else {
+        L[q] = s / L[c * (c + 1) / 2 + c];
+      }
+    }
+  }
+  double y[kD];
+  for (int r = 0; r < kD; ++r) {
+    double s = b[r];
+    for (int m = 0; m < r; ++m) s -= L[r * (r + 1) / 2 + m] * y[m];
+    y[r] = s / L[r * (r + 1) / 2 + r];
+  }
+  for (int r = kD - 1; r >= 0; --r) {
+    double s = y[r];
+    for (int m = r + 1; m < kD; ++m) s -= L[m * (m + 1) / 2 + r] * x[m];
+    x[r] = s / L[r * (r + 1) / 2 + r];
+  }
+  return true;
+}
+
+// Host side (update.cu).
+crvq_status stats_alloc(Scratch& mem, int64_t G_cov, int K, StatsView* st, cudaStream_t s);
+// Zeroes cnt/bacc (scale is kept).
+crvq_status stats_zero(const StatsView& st, cudaStream_t s);
+// Computes the fixed-point scale for accumulating codebook `which` over `set`.
+crvq_status launch_stats_prepare(const SetView& set, const CbList& cbs, int which,
+                                 const StatsView& st, cudaStream_t stream);
+crvq_status launch_stats_solve(const SetView& set, const StatsView& st, const float* C_old,
+                               float* C_out, int32_t* counts, cudaStream_t stream);
+
+}  // namespace crvq

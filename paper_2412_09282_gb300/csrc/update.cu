@@ -1,339 +1,229 @@
 // Least-squares codebook update (k-means update step; Alg. 1 FineTuneCodebook in its
 // closed-form reading). For codebook `which` with all others fixed, codeword k solves
-//   (sum_{v in cluster k} H_{g_v}) c_k = sum_{v in cluster k} H_{g_v} tau_v,
+//   A_k c_k = b_k,  A_k = sum_g cnt[g][k] H_g,  b_k = sum_{v in cluster k} H_{g_v} tau_v,
 //   tau_v = t_v - sum over the other covering codebooks of C[code].
 //
-// Deterministic by construction: members are ordered by a stable LSD radix sort of the codes
-// (8-bit digits, per-tile warp-match ranks, no float atomics), every cluster is reduced by
-// one warp in a fixed lane/flush order (fp32 partials flushed into fp64 every 32 members),
-// and the 8 x 8 normal equations are solved by an fp64 Cholesky factorisation.
+// Deterministic by construction, with no sort and no float atomics: cnt[g][k] are integer
+// counts, b_k is accumulated in 64-bit fixed point (stats.cuh), A_k is summed in fp64 in a
+// fixed order (one CTA per codeword, groups split over the threads, then a fixed reduction
+// tree), and the 8 x 8 system is solved by an fp64 Cholesky factorisation. The Lloyd encode
+// pass (encode.cu) accumulates the same statistics for the codes it writes.
 #include <algorithm>
+#include <cmath>
 
 #include "common.cuh"
 #include "kernels.h"
+#include "stats.cuh"
 
 namespace crvq {
 
 namespace {
 
-constexpr int kRadixThreads = 256;
-constexpr int kRadixItems = 8;
-constexpr int kTileElems = kRadixThreads * kRadixItems;  // 2048
-constexpr int kDigits = 256;
-constexpr int kWarps = kRadixThreads / 32;
+// maxbits[0] = max |T| over the covered vectors, maxbits[1] = max row sum of |H_g|,
+// maxbits[2 + s] = max |C_s| (float bits of non-negative values, merged with atomicMax).
+__global__ void __launch_bounds__(256)
+maxabs_kernel(SetView set, int64_t G_cov, CbList cbs, int which, unsigned* __restrict__ maxbits) {
+  const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int64_t nth = (int64_t)gridDim.x * blockDim.x;
+  float tm = 0.f;
+  const int64_t nv = set.M * G_cov;
+  for (int64_t v = tid; v < nv; v += nth) {
+    const int64_t i = v / G_cov, g = v % G_cov;
+    const float4* t = reinterpret_cast<const float4*>(set.T + i * set.ldT + g * kD);
+    const float4 a = t[0], b = t[1];
+    tm = fmaxf(tm, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
+    tm = fmaxf(tm, fmaxf(fmaxf(fabsf(b.x), fabsf(b.y)), fmaxf(fabsf(b.z), fabsf(b.w))));
+  }
+  float hm = 0.f;
+  for (int64_t r = tid; r < G_cov * kD; r += nth) {
+    const float* h = set.Hb + r * kD;
+    float s = 0.f;
+#pragma unroll
+    for (int j = 0; j < kD; ++j) s += fabsf(h[j]);
+    hm = fmaxf(hm, s);
+  }
+  // warp max, then one atomic per warp
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, off));
+    hm = fmaxf(hm, __shfl_xor_sync(0xffffffffu, hm, off));
+  }
+  if ((threadIdx.x & 31) == 0) {
+    atomicMax(&maxbits[0], __float_as_uint(tm));
+    atomicMax(&maxbits[1], __float_as_uint(hm));
+  }
+  for (int s = 0; s < cbs.n; ++s) {
+    if (s == which) continue;
+    float m = 0.f;
+    for (int64_t e = tid; e < (int64_t)cbs.cb[s].K * kD; e += nth)
+      m = fmaxf(m, fabsf(cbs.cb[s].C[e]));
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+    if ((threadIdx.x & 31) == 0) atomicMax(&maxbits[2 + s], __float_as_uint(m));
+  }
+}
 
-// keys[v] = code of member v (v = i * G_cov + g), vals[v] = v.
-__global__ void gather_keys_kernel(const int32_t* __restrict__ codes, int64_t ld, int64_t M,
-                                   int64_t G_cov, int32_t K, uint32_t* __restrict__ keys,
-                                   uint32_t* __restrict__ vals, int32_t* __restrict__ counts,
+__global__ void stats_scale_kernel(const unsigned* __restrict__ maxbits, int n_cb, int which,
+                                   int64_t n_members, double* __restrict__ scale,
                                    unsigned* err) {
-  const int64_t n = M * G_cov;
+  double cs = 0.0;
+  for (int s = 0; s < n_cb; ++s)
+    if (s != which) cs += (double)__uint_as_float(maxbits[2 + s]);
+  // |H_g tau|_inf <= max row sum |H_g| * (max |t| + sum_s max |C_s|)
+  const double bound =
+      (double)__uint_as_float(maxbits[1]) * ((double)__uint_as_float(maxbits[0]) + cs) * 1.001;
+  if (!isfinite(bound)) raise_error(err, ERRBIT_NUMERIC);
+  *scale = stats_scale_for(bound, n_members);
+}
+
+__global__ void __launch_bounds__(256)
+accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsigned* err) {
+  const CbView cw = cbs.cb[which];
+  const int64_t n = set.M * cw.G_cov;
+  const double scale = *st.scale;
   for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < n;
        v += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t i = v / G_cov, g = v % G_cov;
-    int32_t k = codes[i * ld + g];
-    if (k < 0 || k >= K) {
+    const int64_t i = v / cw.G_cov, g = v % cw.G_cov;
+    const int32_t k = cw.codes[i * cw.ld + g];
+    if (k < 0 || k >= cw.K) {
       raise_error(err, ERRBIT_INDEX);
-      k = 0;
-    }
-    keys[v] = (uint32_t)k;
-    vals[v] = (uint32_t)v;
-    atomicAdd(&counts[k], 1);  // integer counts: order-independent
-  }
-}
-
-__global__ void __launch_bounds__(kRadixThreads)
-radix_hist_kernel(const uint32_t* __restrict__ keys, int64_t n, int shift,
-                  uint32_t* __restrict__ tile_hist, int64_t num_tiles) {
-  __shared__ uint32_t h[kDigits];
-  const int64_t tile = blockIdx.x;
-  h[threadIdx.x] = 0;
-  __syncthreads();
-  const int64_t base = tile * kTileElems;
-  for (int r = 0; r < kRadixItems; ++r) {
-    const int64_t e = base + (int64_t)r * kRadixThreads + threadIdx.x;
-    if (e < n) atomicAdd(&h[(keys[e] >> shift) & 0xFF], 1u);
-  }
-  __syncthreads();
-  tile_hist[(int64_t)threadIdx.x * num_tiles + tile] = h[threadIdx.x];
-}
-
-// Exclusive scan of a uint32 array in place: one CTA walks the array in coalesced blocks of
-// 4096 values (warp-shuffle scans, then a scan of the warp totals) carrying the running sum.
-__global__ void __launch_bounds__(1024)
-exclusive_scan_kernel(uint32_t* __restrict__ a, int64_t n) {
-  __shared__ uint32_t warp_sums[32];
-  __shared__ uint32_t carry;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  if (tid == 0) carry = 0;
-  __syncthreads();
-  for (int64_t base = 0; base < n; base += 4096) {
-    const int64_t e0 = base + (int64_t)tid * 4;
-    uint32_t v[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) v[j] = (e0 + j < n) ? a[e0 + j] : 0u;
-    const uint32_t s = v[0] + v[1] + v[2] + v[3];
-    uint32_t x = s;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t y = __shfl_up_sync(0xffffffffu, x, off);
-      if (lane >= off) x += y;
-    }
-    if (lane == 31) warp_sums[warp] = x;
-    __syncthreads();
-    if (warp == 0) {
-      uint32_t w = warp_sums[lane];
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const uint32_t y = __shfl_up_sync(0xffffffffu, w, off);
-        if (lane >= off) w += y;
-      }
-      warp_sums[lane] = w;
-    }
-    __syncthreads();
-    uint32_t excl = carry + (warp ? warp_sums[warp - 1] : 0u) + x - s;
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      if (e0 + j < n) a[e0 + j] = excl;
-      excl += v[j];
-    }
-    __syncthreads();
-    if (tid == 1023) carry = excl;
-    __syncthreads();
-  }
-}
-
-__global__ void __launch_bounds__(kRadixThreads)
-radix_scatter_kernel(const uint32_t* __restrict__ keys_in, const uint32_t* __restrict__ vals_in,
-                     int64_t n, int shift, const uint32_t* __restrict__ tile_off,
-                     int64_t num_tiles, uint32_t* __restrict__ keys_out,
-                     uint32_t* __restrict__ vals_out) {
-  __shared__ uint32_t cnt[kWarps][kDigits];
-  __shared__ uint32_t run[kDigits];
-  const int64_t tile = blockIdx.x;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  run[threadIdx.x] = tile_off[(int64_t)threadIdx.x * num_tiles + tile];
-  const int64_t base = tile * kTileElems;
-  const unsigned lt_mask = (1u << lane) - 1u;
-  for (int r = 0; r < kRadixItems; ++r) {
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) cnt[w][threadIdx.x] = 0;
-    __syncthreads();
-    const int64_t e = base + (int64_t)r * kRadixThreads + threadIdx.x;
-    const bool act = e < n;
-    const unsigned amask = __ballot_sync(0xffffffffu, act);
-    uint32_t key = 0, val = 0, dig = 0, rank = 0;
-    if (act) {
-      key = keys_in[e];
-      val = vals_in[e];
-      dig = (key >> shift) & 0xFF;
-      const unsigned peers = __match_any_sync(amask, dig);
-      rank = __popc(peers & lt_mask);
-      if ((peers & lt_mask) == 0) cnt[warp][dig] = __popc(peers);
-    }
-    __syncthreads();
-    {  // exclusive prefix over warps for digit = threadIdx.x, continuing the running offset
-      uint32_t p = run[threadIdx.x];
-#pragma unroll
-      for (int w = 0; w < kWarps; ++w) {
-        const uint32_t t = cnt[w][threadIdx.x];
-        cnt[w][threadIdx.x] = p;
-        p += t;
-      }
-      run[threadIdx.x] = p;
-    }
-    __syncthreads();
-    if (act) {
-      const uint32_t pos = cnt[warp][dig] + rank;
-      keys_out[pos] = key;
-      vals_out[pos] = val;
-    }
-    __syncthreads();
-  }
-}
-
-// One warp per codeword: ordered reduction of its members, then the fp64 Cholesky solve.
-__global__ void __launch_bounds__(128)
-cluster_solve_kernel(SetView set, CbList cbs, int which, const uint32_t* __restrict__ members,
-                     const uint32_t* __restrict__ seg_start, const int32_t* __restrict__ counts,
-                     float* __restrict__ C_out, unsigned* err) {
-  const int lane = threadIdx.x & 31;
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  const CbView cw = cbs.cb[which];
-  const int64_t G_cov = cw.G_cov;
-  for (int64_t k = warp; k < cw.K; k += nwarps) {
-    const int64_t beg = seg_start[k];
-    const int64_t cnt = counts[k];
-    if (cnt == 0) {
-      if (lane < kD) C_out[k * kD + lane] = cw.C[k * kD + lane];
       continue;
     }
-    double A[36], b[kD];
-    float Af[36], bf[kD];
+    float tau[kD], q[kD];
+    stats_target(set, cbs, which, i, g, tau, err);
+    stats_htau(set.Hb + g * kD * kD, tau, q);
+    stats_add(st, scale, g, k, q);
+  }
+}
+
+// One CTA per codeword: A_k = sum_g cnt[g][k] H_g in fp64 (groups strided over the threads,
+// then a fixed warp-shuffle + shared-memory tree), b_k from the fixed point, Cholesky solve.
+constexpr int kSolveThreads = 128;
+
+__global__ void __launch_bounds__(kSolveThreads)
+stats_solve_kernel(const float* __restrict__ Hb, int64_t G_cov, int K, StatsView st,
+                   const float* __restrict__ C_old, float* __restrict__ C_out,
+                   int32_t* __restrict__ counts_out, unsigned* err) {
+  __shared__ double part[kSolveThreads / 32][37];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  for (int k = blockIdx.x; k < K; k += gridDim.x) {
+    double A[37];
 #pragma unroll
-    for (int j = 0; j < 36; ++j) { A[j] = 0.0; Af[j] = 0.f; }
-#pragma unroll
-    for (int j = 0; j < kD; ++j) { b[j] = 0.0; bf[j] = 0.f; }
-    int since = 0;
-    for (int64_t p = beg + lane; p < beg + cnt; p += 32) {
-      const int64_t v = members[p];
-      const int64_t i = v / G_cov, g = v % G_cov;
-      const float* H = set.Hb + g * kD * kD;
-      float tau[kD];
-      const float* t = set.T + i * set.ldT + g * kD;
-      const float4 t0 = *reinterpret_cast<const float4*>(t);
-      const float4 t1 = *reinterpret_cast<const float4*>(t + 4);
-      tau[0] = t0.x; tau[1] = t0.y; tau[2] = t0.z; tau[3] = t0.w;
-      tau[4] = t1.x; tau[5] = t1.y; tau[6] = t1.z; tau[7] = t1.w;
-      for (int s = 0; s < cbs.n; ++s) {
-        if (s == which) continue;
-        const CbView& cb = cbs.cb[s];
-        if (g >= cb.G_cov) continue;
-        const int32_t kk = cb.codes[i * cb.ld + g];
-        if (kk < 0 || kk >= cb.K) {
-          raise_error(err, ERRBIT_INDEX);
-          continue;
-        }
-        const float* c = cb.C + (int64_t)kk * kD;
-#pragma unroll
-        for (int j = 0; j < kD; ++j) tau[j] -= c[j];
-      }
-      float h[kD * kD];
-#pragma unroll
-      for (int j = 0; j < kD * kD; ++j) h[j] = H[j];
+    for (int j = 0; j < 37; ++j) A[j] = 0.0;
+    for (int64_t g = threadIdx.x; g < G_cov; g += blockDim.x) {
+      const int c = st.cnt[g * K + k];
+      if (c == 0) continue;
+      A[36] += (double)c;
+      const float* H = Hb + g * kD * kD;
       int q = 0;
 #pragma unroll
-      for (int r = 0; r < kD; ++r) {
-        float acc = 0.f;
+      for (int r = 0; r < kD; ++r)
 #pragma unroll
-        for (int c = 0; c < kD; ++c) acc = fmaf(h[r * kD + c], tau[c], acc);
-        bf[r] += acc;
-#pragma unroll
-        for (int c = 0; c <= r; ++c) Af[q++] += h[r * kD + c];
-      }
-      if (++since == 32) {
-        since = 0;
-#pragma unroll
-        for (int j = 0; j < 36; ++j) { A[j] += (double)Af[j]; Af[j] = 0.f; }
-#pragma unroll
-        for (int j = 0; j < kD; ++j) { b[j] += (double)bf[j]; bf[j] = 0.f; }
-      }
+        for (int cc = 0; cc <= r; ++cc) A[q++] += (double)c * (double)H[r * kD + cc];
     }
 #pragma unroll
-    for (int j = 0; j < 36; ++j) A[j] += (double)Af[j];
+    for (int j = 0; j < 37; ++j)
 #pragma unroll
-    for (int j = 0; j < kD; ++j) b[j] += (double)bf[j];
-    // Fixed butterfly reduction across the warp.
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-#pragma unroll
-      for (int j = 0; j < 36; ++j) A[j] += __shfl_xor_sync(0xffffffffu, A[j], off);
-#pragma unroll
-      for (int j = 0; j < kD; ++j) b[j] += __shfl_xor_sync(0xffffffffu, b[j], off);
-    }
-    if (lane == 0) {
-      // Cholesky A = L L^T (packed lower triangle, row-major), then two triangular solves.
-      double L[36];
-      bool spd = true;
-      int q = 0;
-      for (int r = 0; r < kD; ++r) {
-        for (int c = 0; c <= r; ++c, ++q) {
-          double s = A[q];
-          for (int m = 0; m < c; ++m) s -= L[r * (r + 1) / 2 + m] * L[c * (c + 1) / 2 + m];
-          if (r == c) {
-            if (!(s > 0.0)) { spd = false; s = 1.0; }
-            L[q] = sqrt(s);
-          } else {
-            L[q] = s / L[c * (c + 1) / 2 + c];
-          }
+      for (int off = 16; off > 0; off >>= 1) A[j] += __shfl_xor_sync(0xffffffffu, A[j], off);
+    __syncthreads();
+    if (lane == 0)
+      for (int j = 0; j < 37; ++j) part[warp][j] = A[j];
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      for (int w = 1; w < kSolveThreads / 32; ++w)
+        for (int j = 0; j < 37; ++j) A[j] += part[w][j];
+      const int64_t count = (int64_t)A[36];
+      if (counts_out) counts_out[k] = (int32_t)count;
+      bool keep = count == 0;
+      if (!keep) {
+        const double scale = *st.scale;
+        double b[kD], x[kD];
+        for (int j = 0; j < kD; ++j) b[j] = (double)st.bacc[(int64_t)k * kD + j] / scale;
+        if (cholesky_solve8(A, b, x)) {
+          for (int j = 0; j < kD; ++j) C_out[(int64_t)k * kD + j] = (float)x[j];
+        } else {
+          raise_error(err, ERRBIT_NUMERIC);
+          keep = true;
         }
       }
-      if (!spd) {
-        raise_error(err, ERRBIT_NUMERIC);
-        for (int j = 0; j < kD; ++j) C_out[k * kD + j] = cw.C[k * kD + j];
-      } else {
-        double y[kD], x[kD];
-        for (int r = 0; r < kD; ++r) {
-          double s = b[r];
-          for (int m = 0; m < r; ++m) s -= L[r * (r + 1) / 2 + m] * y[m];
-          y[r] = s / L[r * (r + 1) / 2 + r];
-        }
-        for (int r = kD - 1; r >= 0; --r) {
-          double s = y[r];
-          for (int m = r + 1; m < kD; ++m) s -= L[m * (m + 1) / 2 + r] * x[m];
-          x[r] = s / L[r * (r + 1) / 2 + r];
-        }
-        for (int j = 0; j < kD; ++j) C_out[k * kD + j] = (float)x[j];
-      }
+      if (keep)
+        for (int j = 0; j < kD; ++j) C_out[(int64_t)k * kD + j] = C_old[(int64_t)k * kD + j];
     }
   }
 }
 
 }  // namespace
 
+crvq_status stats_alloc(Scratch& mem, int64_t G_cov, int K, StatsView* st, cudaStream_t s) {
+  const size_t cnt_bytes = align_up((size_t)std::max<int64_t>(G_cov, 1) * K * sizeof(int32_t), 256);
+  const size_t b_bytes = align_up((size_t)K * kD * sizeof(long long), 256);
+  const size_t max_bytes = 256;  // maxbits[2 + kMaxCodebooks] + scale
+  CRVQ_TRY(mem.alloc(cnt_bytes + b_bytes + max_bytes, s));
+  st->cnt = mem.as<int32_t>();
+  st->bacc = reinterpret_cast<long long*>(mem.as<char>() + cnt_bytes);
+  st->scale = reinterpret_cast<double*>(mem.as<char>() + cnt_bytes + b_bytes);
+  st->G_cov = G_cov;
+  st->K = K;
+  return stats_zero(*st, s);
+}
+
+crvq_status stats_zero(const StatsView& st, cudaStream_t s) {
+  const size_t cnt_bytes = align_up((size_t)std::max<int64_t>(st.G_cov, 1) * st.K * sizeof(int32_t), 256);
+  const size_t b_bytes = align_up((size_t)st.K * kD * sizeof(long long), 256);
+  CRVQ_CUDA(cudaMemsetAsync(st.cnt, 0, cnt_bytes + b_bytes, s));
+  return CRVQ_OK;
+}
+
+crvq_status launch_stats_prepare(const SetView& set, const CbList& cbs, int which,
+                                 const StatsView& st, cudaStream_t stream) {
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
+  const CbView& cw = cbs.cb[which];
+  // maxbits live right after the scale (same 256-byte block).
+  unsigned* maxbits = reinterpret_cast<unsigned*>(st.scale + 1);
+  CRVQ_CUDA(cudaMemsetAsync(maxbits, 0, (2 + kMaxCodebooks) * sizeof(unsigned), stream));
+  const int64_t n = set.M * cw.G_cov;
+  const int nsm = sm_count();
+  ProfScope ps("update_bound", stream, (double)n * kD * 4.0);
+  maxabs_kernel<<<(unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(n, 256), 4 * nsm)),
+                  256, 0, stream>>>(set, cw.G_cov, cbs, which, maxbits);
+  CRVQ_LAUNCHED();
+  stats_scale_kernel<<<1, 1, 0, stream>>>(maxbits, cbs.n, which, std::max<int64_t>(1, n),
+                                          st.scale, err);
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
+}
+
+crvq_status launch_stats_solve(const SetView& set, const StatsView& st, const float* C_old,
+                               float* C_out, int32_t* counts, cudaStream_t stream) {
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
+  ProfScope ps("update_solve", stream, (double)st.K);
+  const int blocks = (int)std::min<int64_t>(st.K, 64 * sm_count());
+  stats_solve_kernel<<<blocks, kSolveThreads, 0, stream>>>(set.Hb, st.G_cov, st.K, st, C_old,
+                                                           C_out, counts, err);
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
+}
+
 crvq_status launch_update_codebook(const SetView& set, const CbList& cbs, int which,
-                                   float* C_out, int32_t* counts_out, cudaStream_t stream) {
+                                   float* C_out, int32_t* counts, cudaStream_t stream) {
   unsigned* err = nullptr;
   CRVQ_TRY(device_error_word(&err));
   const CbView& cw = cbs.cb[which];
   const int64_t n = set.M * cw.G_cov;
-  const int K = cw.K;
-  const int nsm = sm_count();
-  const int64_t num_tiles = std::max<int64_t>(1, ceil_div(n, kTileElems));
-  const int passes = K > 256 ? 2 : 1;
-  // scratch: keys/vals x2, tile histogram, counts, segment starts
   Scratch mem;
-  const size_t nn = (size_t)std::max<int64_t>(n, 1);
-  const size_t bytes = 4 * nn * sizeof(uint32_t) + (size_t)kDigits * num_tiles * sizeof(uint32_t) +
-                       2 * (size_t)K * sizeof(uint32_t) + 256;
-  CRVQ_TRY(mem.alloc(bytes, stream));
-  uint32_t* keysA = mem.as<uint32_t>();
-  uint32_t* valsA = keysA + nn;
-  uint32_t* keysB = valsA + nn;
-  uint32_t* valsB = keysB + nn;
-  uint32_t* tile_hist = valsB + nn;
-  int32_t* counts = reinterpret_cast<int32_t*>(tile_hist + (size_t)kDigits * num_tiles);
-  uint32_t* seg = reinterpret_cast<uint32_t*>(counts + K);
-
-  CRVQ_CUDA(cudaMemsetAsync(counts, 0, (size_t)K * sizeof(int32_t), stream));
+  StatsView st;
+  CRVQ_TRY(stats_alloc(mem, cw.G_cov, cw.K, &st, stream));
+  CRVQ_TRY(launch_stats_prepare(set, cbs, which, st, stream));
   if (n > 0) {
-    ProfScope ps("update_sort", stream, (double)n);
-    gather_keys_kernel<<<(unsigned)std::min<int64_t>(ceil_div(n, 256), 16 * nsm), 256, 0,
-                         stream>>>(cw.codes, cw.ld, set.M, cw.G_cov, K, keysA, valsA, counts,
-                                   err);
+    ProfScope ps("update_accumulate", stream, (double)n);
+    const int nsm = sm_count();
+    accumulate_stats_kernel<<<(unsigned)std::min<int64_t>(ceil_div(n, 256), 16 * nsm), 256, 0,
+                              stream>>>(set, cbs, which, st, err);
     CRVQ_LAUNCHED();
-    uint32_t *kin = keysA, *vin = valsA, *kout = keysB, *vout = valsB;
-    for (int pass = 0; pass < passes; ++pass) {
-      const int shift = 8 * pass;
-      radix_hist_kernel<<<(unsigned)num_tiles, kRadixThreads, 0, stream>>>(kin, n, shift,
-                                                                          tile_hist, num_tiles);
-      CRVQ_LAUNCHED();
-      exclusive_scan_kernel<<<1, 1024, 0, stream>>>(tile_hist, (int64_t)kDigits * num_tiles);
-      CRVQ_LAUNCHED();
-      radix_scatter_kernel<<<(unsigned)num_tiles, kRadixThreads, 0, stream>>>(
-          kin, vin, n, shift, tile_hist, num_tiles, kout, vout);
-      CRVQ_LAUNCHED();
-      std::swap(kin, kout);
-      std::swap(vin, vout);
-    }
-    // sorted member list is now in (kin, vin)
-    CRVQ_CUDA(cudaMemcpyAsync(seg, counts, (size_t)K * sizeof(int32_t), cudaMemcpyDeviceToDevice,
-                              stream));
-    exclusive_scan_kernel<<<1, 1024, 0, stream>>>(seg, K);
-    CRVQ_LAUNCHED();
-    ProfScope ps2("update_solve", stream, (double)n);
-    cluster_solve_kernel<<<(unsigned)std::min<int64_t>(ceil_div((int64_t)K * 32, 128), 64 * nsm),
-                           128, 0, stream>>>(set, cbs, which, vin, seg, counts, C_out, err);
-    CRVQ_LAUNCHED();
-  } else {
-    CRVQ_CUDA(cudaMemcpyAsync(C_out, cw.C, (size_t)K * kD * sizeof(float),
-                              cudaMemcpyDeviceToDevice, stream));
   }
-  if (counts_out)
-    CRVQ_CUDA(cudaMemcpyAsync(counts_out, counts, (size_t)K * sizeof(int32_t),
-                              cudaMemcpyDeviceToDevice, stream));
-  return CRVQ_OK;
+  return launch_stats_solve(set, st, cw.C, C_out, counts, stream);
 }
 
 }  // namespace crvq

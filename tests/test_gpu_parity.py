@@ -328,20 +328,130 @@ def test_invalid_arguments_raise_before_launch(c1):
 
 
 # ------------------------------------------------------------------------------ end to end
-def test_quantize_layer_c1_end_to_end(c1):
+def _gpu_schedule_with_checks(W, X, cfg):
+    """The per-matrix schedule driven call by call through the C ABI, each step checked
+    against the oracle fed the GPU's own state (stepwise re-synced parity along the GPU's
+    trajectory). Returns the GPU state at the end."""
+    d = cfg.d
+    M, N = W.shape
+    G = N // d
+    seed = lambda ph, cb: O.phase_seed(cfg.seed, ph, cb)
+    Xd, Wd = dev(X), dev(W)
+    H, xsq, Hb0, delta = P.crvq_hessian(Xd, cfg.damp_rel, d)
+
+    def lloyd(T, Hb, fixed, C0, G_cov, Td_np, Hb_np):
+        codes = torch.zeros((M, G_cov), dtype=torch.int32, device="cuda")
+        cbs = list(fixed) + [Codebook(C0, codes, G_cov)]
+        j = len(cbs) - 1
+        for it in range(cfg.kmeans_iters + 1):
+            P.crvq_encode_beam(T, d, Hb, cbs, j, 1)
+            P.crvq_sync()
+            ocb = oracle_cbs(cbs)
+            oc, _ = O.encode_beam(Td_np, d, Hb_np, [c for c in ocb[:j]] +
+                                  [O.Codebook(ocb[j].C, None, G_cov)], j, 1)
+            check_codes_with_ties(Td_np, d, Hb_np, ocb[:j] + [O.Codebook(ocb[j].C, None, G_cov)],
+                                  j, [None] * j + [host(codes)], oc)
+            if it == cfg.kmeans_iters:
+                break
+            Cn, _ = P.crvq_update_codebook(T, d, Hb, cbs, j)
+            P.crvq_sync()
+            Co, _ = O.update_codebook(Td_np, d, Hb_np, oracle_cbs(cbs), j)
+            _cmp_codebook(host(Cn), Co.astype(np.float64))
+            cbs[j] = Codebook(Cn, codes, G_cov)
+        return cbs[j]
+
+    # S2 prequantize
+    C0 = P.crvq_kmeans_init(Wd, d, G, cfg.K_base, seed(1, 0))
+    pre = lloyd(Wd, Hb0, [], C0, G, W, host(Hb0))
+    W_pre, _, _, _ = P.crvq_reconstruct_error(Wd, d, Hb0, None, [pre], 0)
+    # S3
+    perm, imp, Ws, Hb, Gc = P.crvq_select_reorder_channels(
+        Wd, d, W_pre, xsq, H, cfg.crit_frac, cfg.importance_mode, seed(4, 0))
+    P.crvq_sync()
+    po = O.select_reorder_channels(W, d, host(W_pre), host(xsq), host(H), cfg.crit_frac,
+                                   cfg.importance_mode, seed(4, 0))
+    np.testing.assert_array_equal(host(perm), po[0])
+    Ws_np, Hb_np = host(Ws), host(Hb)
+    # S4
+    Cb0 = P.crvq_kmeans_init(Ws, d, G, cfg.K_base, seed(2, 0))
+    base = lloyd(Ws, Hb, [], Cb0, G, Ws_np, Hb_np)
+    cbs = [base]
+    # S5
+    crit = Ws[:, :Gc * d]
+    for t in range(1, cfg.n_ext + 1):
+        fixed = [Codebook(cb.C, cb.codes[:, :Gc], Gc) for cb in cbs]
+        Ct0 = P.crvq_kmeans_init(crit, d, Gc, cfg.K_ext, seed(3, t), fixed=fixed)
+        ext = lloyd(crit, Hb[:Gc], fixed, Ct0, Gc, Ws_np[:, :Gc * d], Hb_np[:Gc])
+        cbs.append(Codebook(ext.C, ext.codes, Gc))
+    # S6 (one round)
+    for r in range(cfg.refine_rounds):
+        for j in range(len(cbs)):
+            Cn, _ = P.crvq_update_codebook(Ws, d, Hb, cbs, j)
+            P.crvq_sync()
+            Co, _ = O.update_codebook(Ws_np, d, Hb_np, oracle_cbs(cbs), j)
+            _cmp_codebook(host(Cn), Co.astype(np.float64))
+            cbs[j] = Codebook(Cn, cbs[j].codes, cbs[j].G_cov)
+        before = oracle_cbs(cbs)
+        P.crvq_encode_beam(Ws, d, Hb, cbs, 0, cfg.B, keep_if_better=True)
+        P.crvq_sync()
+        oc, _ = O.encode_beam(Ws_np, d, Hb_np, before, 0, cfg.B, keep_if_better=True)
+        gpu = [host(cb.codes) for cb in cbs]
+        diff = np.zeros((M, G), bool)
+        for s in range(len(cbs)):
+            diff[:, :cbs[s].G_cov] |= gpu[s] != oc[s]
+        for i, g in zip(*np.nonzero(diff)):
+            Cs = [before[0].C] + ([cb.C for cb in before[1:]] if g < Gc else [])
+            gap = beam_boundary_gap(Ws_np[i, g * d:(g + 1) * d].astype(np.float64), Hb_np[g],
+                                    Cs, cfg.B)
+            assert gap < 1e-6, f"refinement code differs at ({i},{g}) with gap {gap}"
+    Wh, lb, lc, lf = P.crvq_reconstruct_error(Ws, d, Hb, perm, cbs, Gc, X=Xd,
+                                              damp_delta=float(host(delta)[0]))
+    ocb = oracle_cbs(cbs)
+    _, lbo, lco, lfo = O.reconstruct_error(Ws_np, d, Hb_np, host(perm), ocb, Gc, X,
+                                           float(host(delta)[0]))
+    assert abs(lb - lbo) <= 1e-4 * lbo and abs(lc - lco) <= 1e-4 * lco
+    assert abs(lf - lfo) <= 1e-4 * lfo
+    return dict(perm=host(perm), cbs=[(host(cb.C), host(cb.codes)) for cb in cbs],
+                losses=(lb, lc, lf))
+
+
+@pytest.mark.parametrize("name", ["c1", "small_B8_3ext"])
+def test_quantize_layer_matches_resynced_stepwise_schedule(c1, name):
+    """Every step of the schedule agrees with the oracle given the GPU's state, and the
+    one-call crvq_quantize_layer reproduces that trajectory exactly (same kernels, same
+    order; the fused Lloyd statistics equal the standalone update's, bit for bit)."""
+    if name == "c1":
+        cfg, W, X = c1["cfg"], c1["W"], c1["X"]
+    else:
+        cfg = S.LayerConfig("pin_med", 256, 192, 300, "outlier_cols", "lognormal", 0.5,
+                            n_outlier_cols=5, K_base=128, n_ext=3, K_ext=32, crit_frac=0.1,
+                            B=8, kmeans_iters=5)
+        W, X = S.gen_W(cfg), S.gen_X(cfg)
+    ref = _gpu_schedule_with_checks(W, X, cfg)
+    out = P.crvq_quantize_layer(dev(W), dev(X), cfg)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(host(out.perm), ref["perm"])
+    np.testing.assert_array_equal(host(out.C_base), ref["cbs"][0][0])
+    np.testing.assert_array_equal(host(out.codes_base), ref["cbs"][0][1])
+    for t in range(cfg.n_ext):
+        np.testing.assert_array_equal(host(out.C_ext[t]), ref["cbs"][t + 1][0])
+        np.testing.assert_array_equal(host(out.codes_ext[t]), ref["cbs"][t + 1][1])
+    lb, lc, lf = ref["losses"]
+    assert out.report["loss_block"] == pytest.approx(lb, rel=1e-12)
+    assert out.report["loss_full"] == pytest.approx(lf, rel=1e-12)
+
+
+def test_quantize_layer_c1_independent_oracle_run_is_close(c1):
+    """Report-level check against an independent oracle run of the whole schedule: the two
+    k-means trajectories may part at rounding-level near-ties, so only the final losses are
+    compared, loosely."""
     cfg = c1["cfg"]
     out = P.crvq_quantize_layer(dev(c1["W"]), dev(c1["X"]), cfg)
     torch.cuda.synchronize()
     ref = O.quantize_layer(c1["W"], c1["X"], cfg)
-    rep = out.report
     np.testing.assert_array_equal(host(out.perm), ref["perm"])
-    assert rep["n_crit_groups"] == ref["n_crit_groups"]
-    agree = (host(out.codes_base) == ref["codebooks"][0].codes).mean()
-    assert agree >= 0.999, agree
-    for key, r in [("loss_block", ref["loss_block"]), ("loss_crit", ref["loss_crit"]),
-                   ("loss_full", ref["loss_full"]), ("loss_pre", ref["loss_pre"])]:
-        assert abs(rep[key] - r) <= 1e-3 * abs(r), (key, rep[key], r)
-    _cmp_codebook(host(out.C_base), ref["codebooks"][0].C.astype(np.float64), 1e-3)
+    for key in ("loss_block", "loss_crit", "loss_full", "loss_pre"):
+        assert abs(out.report[key] - ref[key]) <= 2e-2 * abs(ref[key]), key
 
 
 def test_quantize_layer_host_buffers_match_device(c1):
