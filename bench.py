@@ -321,6 +321,7 @@ def main():
         "roofline": roof,
         "e2e": e2e,
         "gpu_launches": int(launches),
+        "fp64_fallback_decisions_per_step": out.report["flagged"],
         "kernels": [{"name": k["name"], "launches": k["launches"], "ms": k["ms"],
                      "share": k["ms"] / total_k} for k in ks[:12]],
         "clocks": clk,
