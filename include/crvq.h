@@ -189,6 +189,30 @@ crvq_status crvq_update_codebook(const float* T, int64_t ldT, int64_t M, int64_t
                                  crvq_stream_t stream);
 
 /*
+ * crvq_update_codebook without device memory allocation. The paper has no counterpart: this
+ * entry point exists for callers that cannot call cudaMalloc or cudaFree (code running while
+ * a CUDA graph is captured into a pool it does not own, runtimes that hand out a fixed memory
+ * arena and forbid allocation after start-up, callers that must not synchronise). Arguments,
+ * results and rounding are those of crvq_update_codebook; the caller still passes the
+ * inputs and outputs. Its scratch is one file-scope device array of 4 MiB, held by every GPU
+ * that loads the library until the process exits:
+ *  - sizes whose statistics exceed it (G_cov * K * 4 + K * 64 + 512 bytes > 4 MiB - 256,
+ *    e.g. K = 256 with more than ~4000 covered groups) return CRVQ_ERR_UNSUPPORTED before
+ *    anything is enqueued;
+ *  - every call shares the array, so calls that overlap on the GPU (different streams or
+ *    devices' streams writing the same device's array) race; each call clears what must
+ *    start at zero;
+ *  - the first call on a device looks up the array's device address (cudaGetSymbolAddress)
+ *    with that device current; make that first call before any stream capture;
+ *  - device-side range checks (codes outside [0, K)) skip the bad entries and record them in
+ *    this entry point's own error word inside the array, which crvq_sync does not read.
+ */
+crvq_status crvq_update_codebook_noalloc(const float* T, int64_t ldT, int64_t M, int64_t G_sub,
+                                         int32_t d, const float* H_blocks,
+                                         const crvq_codebook* cbs, int32_t n_cb, int32_t which,
+                                         float* C_out, int32_t* counts, crvq_stream_t stream);
+
+/*
  * S7. Reconstruction, reverse reorder and losses (Alg. 1 QuantLoss; Sec. 4.3 "restored to
  * their original order"). The set is all of W_sorted (M x N, G = N/d groups).
  *   perm         [N] or NULL (identity).

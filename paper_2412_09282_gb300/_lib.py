@@ -68,6 +68,9 @@ SIGNATURES = {
     "crvq_update_codebook": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int64, C.c_int32,
                                          c_vp, C.POINTER(crvq_codebook), C.c_int32, C.c_int32,
                                          c_vp, c_vp, c_vp]),
+    "crvq_update_codebook_noalloc": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int64,
+                                                 C.c_int32, c_vp, C.POINTER(crvq_codebook),
+                                                 C.c_int32, C.c_int32, c_vp, c_vp, c_vp]),
     "crvq_reconstruct_error": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int32, c_vp, c_vp,
                                            C.POINTER(crvq_codebook), C.c_int32, C.c_int64,
                                            c_vp, C.c_int64, C.c_double, c_vp, c_f64p, c_vp]),

@@ -205,6 +205,26 @@ def crvq_update_codebook(T, d, H_blocks, cbs, which, C_out=None, counts=None, st
     return C_out, counts
 
 
+def crvq_update_codebook_noalloc(T, d, H_blocks, cbs, which, C_out=None, counts=None,
+                                 stream=None):
+    """crvq_update_codebook without device allocation inside the library: its scratch is a
+    fixed 4 MiB device array (see include/crvq.h). Outputs not passed in are allocated here,
+    by torch, before the call."""
+    _need(T, torch.float32, "T")
+    _rowmajor(T, "T")
+    M = T.shape[0]
+    G_sub = H_blocks.shape[0]
+    dev = T.device
+    K = cbs[which].C.shape[0]
+    C_out = torch.empty((K, d), device=dev, dtype=torch.float32) if C_out is None else C_out
+    counts = torch.empty(K, device=dev, dtype=torch.int32) if counts is None else counts
+    arr = _cb_array(cbs)
+    _check(_L().crvq_update_codebook_noalloc(_ptr(T), T.stride(0), M, G_sub, d, _ptr(H_blocks),
+                                             arr, len(cbs), which, _ptr(C_out), _ptr(counts),
+                                             _stream(stream, dev)))
+    return C_out, counts
+
+
 def crvq_reconstruct_error(W_sorted, d, H_blocks, perm, cbs, n_crit_groups, X=None,
                            damp_delta=0.0, want_W_hat=True, stream=None):
     """Returns (W_hat or None, loss_block, loss_crit, loss_full). Synchronizes the stream."""

@@ -227,3 +227,56 @@ crvq_status launch_update_codebook(const SetView& set, const CbList& cbs, int wh
 }
 
 }  // namespace crvq
+
+namespace crvq {
+
+// The update of launch_update_codebook on caller-provided scratch (no allocation): `scratch`
+// (256-byte aligned, `bytes` long) holds cnt | bacc | scale + maxima, and `err` is the error
+// word the kernels report to. Returns CRVQ_ERR_UNSUPPORTED when the statistics of this
+// codebook do not fit in `bytes`.
+size_t update_scratch_bytes(int64_t G_cov, int K) {
+  return align_up((size_t)std::max<int64_t>(G_cov, 1) * K * sizeof(int32_t), 256) +
+         align_up((size_t)K * kD * sizeof(long long), 256) + 256;
+}
+
+crvq_status launch_update_codebook_on(const SetView& set, const CbList& cbs, int which,
+                                      float* C_out, int32_t* counts, void* scratch,
+                                      size_t bytes, unsigned* err, cudaStream_t stream) {
+  const CbView& cw = cbs.cb[which];
+  const int64_t n = set.M * cw.G_cov;
+  const size_t need = update_scratch_bytes(cw.G_cov, cw.K);
+  if (need > bytes)
+    return fail(CRVQ_ERR_UNSUPPORTED,
+                "statistics of this codebook need %zu bytes of scratch, the limit is %zu "
+                "(G_cov * K * 4 + K * 64 + 512 bytes)",
+                need, bytes);
+  const size_t cnt_bytes = align_up((size_t)std::max<int64_t>(cw.G_cov, 1) * cw.K * sizeof(int32_t), 256);
+  const size_t b_bytes = align_up((size_t)cw.K * kD * sizeof(long long), 256);
+  StatsView st;
+  st.cnt = static_cast<int32_t*>(scratch);
+  st.bacc = reinterpret_cast<long long*>(static_cast<char*>(scratch) + cnt_bytes);
+  st.scale = reinterpret_cast<double*>(static_cast<char*>(scratch) + cnt_bytes + b_bytes);
+  st.G_cov = cw.G_cov;
+  st.K = cw.K;
+  unsigned* maxbits = reinterpret_cast<unsigned*>(st.scale + 1);
+  // The scratch keeps the previous call's contents: clear counts, sums and maxima.
+  CRVQ_CUDA(cudaMemsetAsync(scratch, 0, cnt_bytes + b_bytes + 256, stream));
+  const int nsm = sm_count();
+  maxabs_kernel<<<(unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(n, 256), 4 * nsm)),
+                  256, 0, stream>>>(set, cw.G_cov, cbs, which, maxbits);
+  CRVQ_LAUNCHED();
+  stats_scale_kernel<<<1, 1, 0, stream>>>(maxbits, cbs.n, which, std::max<int64_t>(1, n),
+                                          st.scale, err);
+  CRVQ_LAUNCHED();
+  if (n > 0) {
+    accumulate_stats_kernel<<<(unsigned)std::min<int64_t>(ceil_div(n, 256), 16 * nsm), 256, 0,
+                              stream>>>(set, cbs, which, st, err);
+    CRVQ_LAUNCHED();
+  }
+  stats_solve_kernel<<<(int)std::min<int64_t>(st.K, 64 * nsm), kSolveThreads, 0, stream>>>(
+      set.Hb, st.G_cov, st.K, st, cw.C, C_out, counts, err);
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
+}
+
+}  // namespace crvq
