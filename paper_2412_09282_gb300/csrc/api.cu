@@ -82,6 +82,22 @@ struct ProfRec {
   double units;
 };
 std::vector<ProfRec> g_recs;
+std::vector<cudaEvent_t> g_pool;  // events reused across profiling sessions
+
+cudaEvent_t pool_get() {
+  std::lock_guard<std::mutex> lk(g_pmu);
+  if (!g_pool.empty()) {
+    cudaEvent_t e = g_pool.back();
+    g_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  if (cudaEventCreate(&e) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return e;
+}
 }  // namespace
 
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
@@ -89,21 +105,19 @@ void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 ProfScope::ProfScope(const char* name, cudaStream_t s, double units)
     : name_(name), s_(s), units_(units) {
   if (g_prof.load(std::memory_order_relaxed)) {
-    if (cudaEventCreate(&a_) != cudaSuccess || cudaEventRecord(a_, s_) != cudaSuccess) {
-      if (a_) cudaEventDestroy(a_);
-      a_ = nullptr;
+    a_ = pool_get();
+    if (a_ && cudaEventRecord(a_, s_) != cudaSuccess) {
       cudaGetLastError();
+      a_ = nullptr;
     }
   }
 }
 
 ProfScope::~ProfScope() {
   if (!a_) return;
-  cudaEvent_t b = nullptr;
-  if (cudaEventCreate(&b) != cudaSuccess || cudaEventRecord(b, s_) != cudaSuccess) {
+  cudaEvent_t b = pool_get();
+  if (!b || cudaEventRecord(b, s_) != cudaSuccess) {
     cudaGetLastError();
-    cudaEventDestroy(a_);
-    if (b) cudaEventDestroy(b);
     return;
   }
   std::lock_guard<std::mutex> lk(g_pmu);
@@ -179,12 +193,22 @@ const char* crvq_version(void) {
 int64_t crvq_launch_count(void) { return (int64_t)g_launches.load(); }
 
 crvq_status crvq_profile_begin(void) {
-  std::lock_guard<std::mutex> lk(g_pmu);
-  for (auto& r : g_recs) {
-    cudaEventDestroy(r.a);
-    cudaEventDestroy(r.b);
+  {
+    std::lock_guard<std::mutex> lk(g_pmu);
+    for (auto& r : g_recs) {
+      g_pool.push_back(r.a);
+      g_pool.push_back(r.b);
+    }
+    g_recs.clear();
   }
-  g_recs.clear();
+  // pre-create events so that recording inside the profiled region does not create any
+  std::vector<cudaEvent_t> fresh;
+  for (int i = 0; i < 1024; ++i) fresh.push_back(pool_get());
+  {
+    std::lock_guard<std::mutex> lk(g_pmu);
+    for (auto e : fresh)
+      if (e) g_pool.push_back(e);
+  }
   g_prof.store(true);
   return CRVQ_OK;
 }
@@ -203,8 +227,11 @@ crvq_status crvq_profile_end(crvq_kernel_stat* stats, int32_t cap, int32_t* n_st
     if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess) {
       st = fail(CRVQ_ERR_CUDA, "profiling event failed: %s", cudaGetErrorString(cudaGetLastError()));
     }
-    cudaEventDestroy(r.a);
-    cudaEventDestroy(r.b);
+    {
+      std::lock_guard<std::mutex> lk(g_pmu);
+      g_pool.push_back(r.a);
+      g_pool.push_back(r.b);
+    }
     size_t j = 0;
     for (; j < agg.size(); ++j)
       if (strncmp(agg[j].name, r.name, sizeof(agg[j].name)) == 0) break;

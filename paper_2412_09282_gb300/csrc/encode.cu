@@ -167,7 +167,8 @@ __device__ __forceinline__ void stage_chunk(const float* __restrict__ C, int k0,
   }
 }
 
-// fp32 lower bound low_k of the score of codeword k (same operation order as the fast pass).
+// fp32 lower bound low_k of the score of codeword k. Any evaluation covered by the same
+// error analysis is a valid lower bound; the fallback needs no more than that.
 __device__ __forceinline__ float low_score(const float c[kD], const float* H, const float m2q[kD],
                                            float nbeta, float cmul) {
   float n, na, l1;
@@ -182,7 +183,7 @@ __device__ __forceinline__ float low_score(const float c[kD], const float* H, co
 // One CTA = one group g and kThreads * VPT rows; each thread owns VPT vectors. When
 // st.cnt != null the certified codes' least-squares statistics are accumulated (stats.cuh).
 template <int VPT>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, 4)
 argmin_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
               int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0, FlagList flags,
               StatsView st, unsigned* err) {
@@ -230,16 +231,17 @@ argmin_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
       const float n = sN[k], l1 = sL[k];
 #pragma unroll
       for (int v = 0; v < VPT; ++v) {
-        float s = n;
-        s = fmaf(m2q[v][0], c0.x, s);
+        // two independent FMA chains (latency), summed once
+        float s = fmaf(m2q[v][0], c0.x, n);
+        float t = nbeta[v] * l1;
         s = fmaf(m2q[v][1], c0.y, s);
+        t = fmaf(m2q[v][4], c1.x, t);
         s = fmaf(m2q[v][2], c0.z, s);
+        t = fmaf(m2q[v][5], c1.y, t);
         s = fmaf(m2q[v][3], c0.w, s);
-        s = fmaf(m2q[v][4], c1.x, s);
-        s = fmaf(m2q[v][5], c1.y, s);
-        s = fmaf(m2q[v][6], c1.z, s);
-        s = fmaf(m2q[v][7], c1.w, s);
-        s = fmaf(nbeta[v], l1, s);
+        t = fmaf(m2q[v][6], c1.z, t);
+        t = fmaf(m2q[v][7], c1.w, t);
+        s += t;
         b2[v] = fminf(b2[v], fmaxf(s, b1[v]));
         const bool lt = s < b1[v];
         i1[v] = lt ? k0 + k : i1[v];
