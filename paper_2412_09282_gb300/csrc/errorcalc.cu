@@ -3,8 +3,8 @@
 //   loss_block = sum_v (t_v - r_v)^T H_g (t_v - r_v)       (block-diagonal part)
 //   loss_crit  = the same over the critical groups g < G_c
 //   loss_full  = ||dW X^T||^2 / n + delta ||dW||^2 = tr(dW H dW^T)   (dW in original order)
-// Per-row partial sums are fp64 and reduced in a fixed order; the full loss streams
-// dW X^T tiles through a SIMT GEMM whose epilogue squares and sums them (fp64 per CTA).
+// Per-row partial sums are fp64 and reduced in a fixed order; the full loss forms dW X^T on the
+// tensor cores (tc_gemm.cuh: tcgen05, 3xTF32, split K) and squares and sums it in fp64.
 #include "common.cuh"
 #include "kernels.h"
 
@@ -108,87 +108,6 @@ decode_row_kernel(const float* __restrict__ Ws, int64_t M, int64_t N, const floa
   }
 }
 
-constexpr int kT = 128, kBK = 16, kFlush = 256;
-
-// sum over a 128 x 128 tile of P = dW X^T (dW: M x N, X: n x N, both row-major) of P^2.
-__global__ void __launch_bounds__(256)
-gemm_nt_sumsq_kernel(const float* __restrict__ A, int64_t M, const float* __restrict__ X,
-                     int64_t n, int64_t N, double* __restrict__ part) {
-  __shared__ __align__(16) float As[kBK][kT];
-  __shared__ __align__(16) float Bs[kBK][kT];
-  __shared__ double red[256];
-  const int64_t a0 = (int64_t)blockIdx.x * kT, b0 = (int64_t)blockIdx.y * kT;
-  const int tid = threadIdx.x, tx = tid & 15, ty = tid >> 4;
-  float acc[8][8], outer[8][8];
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) acc[i][j] = outer[i][j] = 0.f;
-  int since = 0;
-  const int lr = tid >> 1, lk = (tid & 1) * 8;  // load: row lr, k offset lk (8 values)
-  for (int64_t k0 = 0; k0 < N; k0 += kBK) {
-    {
-      const int64_t ra = a0 + lr, rb = b0 + lr;
-      float va[8], vb[8];
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const int64_t k = k0 + lk + q;
-        va[q] = (ra < M && k < N) ? A[ra * N + k] : 0.f;
-        vb[q] = (rb < n && k < N) ? X[rb * N + k] : 0.f;
-      }
-#pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        As[lk + q][lr] = va[q];
-        Bs[lk + q][lr] = vb[q];
-      }
-    }
-    __syncthreads();
-#pragma unroll
-    for (int kk = 0; kk < kBK; ++kk) {
-      float a[8], b[8];
-      const float4 a_lo = *reinterpret_cast<const float4*>(&As[kk][ty * 4]);
-      const float4 a_hi = *reinterpret_cast<const float4*>(&As[kk][64 + ty * 4]);
-      const float4 b_lo = *reinterpret_cast<const float4*>(&Bs[kk][tx * 4]);
-      const float4 b_hi = *reinterpret_cast<const float4*>(&Bs[kk][64 + tx * 4]);
-      a[0] = a_lo.x; a[1] = a_lo.y; a[2] = a_lo.z; a[3] = a_lo.w;
-      a[4] = a_hi.x; a[5] = a_hi.y; a[6] = a_hi.z; a[7] = a_hi.w;
-      b[0] = b_lo.x; b[1] = b_lo.y; b[2] = b_lo.z; b[3] = b_lo.w;
-      b[4] = b_hi.x; b[5] = b_hi.y; b[6] = b_hi.z; b[7] = b_hi.w;
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
-    }
-    __syncthreads();
-    since += kBK;
-    if (since >= kFlush) {
-      since = 0;
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-          outer[i][j] += acc[i][j];
-          acc[i][j] = 0.f;
-        }
-    }
-  }
-  double s = 0.0;
-#pragma unroll
-  for (int i = 0; i < 8; ++i)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const double v = (double)(outer[i][j] + acc[i][j]);
-      s += v * v;
-    }
-  red[tid] = s;
-  __syncthreads();
-  for (int w = 128; w > 0; w >>= 1) {
-    if (tid < w) red[tid] += red[tid + w];
-    __syncthreads();
-  }
-  if (tid == 0) part[(int64_t)blockIdx.y * gridDim.x + blockIdx.x] = red[0];
-}
-
 __global__ void __launch_bounds__(256)
 finalize_losses_kernel(const double* __restrict__ row_part, int64_t M,
                        const double* __restrict__ gemm_part, int64_t n_gemm, int64_t n_tok,
@@ -234,10 +153,11 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   unsigned* err = nullptr;
   CRVQ_TRY(device_error_word(&err));
   const int nsm = sm_count();
-  const int64_t gx = ceil_div(M, kT), gy = X ? ceil_div(n_tok, kT) : 0;
+  const int64_t n_gemm_cap = X ? 8 * (int64_t)nsm : 0;  // partial sums of the full loss
+  int64_t n_gemm = 0;
   // Scratch: dW (16-byte aligned for the 128-bit stores), then the fp64 partial sums.
   const size_t dW_bytes = X ? align_up((size_t)M * N * sizeof(float), 256) : 0;
-  const size_t part_bytes = (size_t)M * 3 * sizeof(double) + (size_t)(gx * gy + 1) * sizeof(double);
+  const size_t part_bytes = (size_t)M * 3 * sizeof(double) + (size_t)(n_gemm_cap + 1) * sizeof(double);
   Scratch mem;
   CRVQ_TRY(mem.alloc(dW_bytes + part_bytes, stream));
   float* dW = X ? mem.as<float>() : nullptr;
@@ -256,12 +176,9 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   CRVQ_LAUNCHED();
   }
   if (X) {
-    dim3 grid((unsigned)gx, (unsigned)gy);
-    ProfScope ps("loss_gemm", stream, 2.0 * (double)M * N * n_tok);
-    gemm_nt_sumsq_kernel<<<grid, 256, 0, stream>>>(dW, M, X, n_tok, N, gemm_part);
-    CRVQ_LAUNCHED();
+    CRVQ_TRY(launch_tc_sumsq(dW, M, X, n_tok, N, gemm_part, n_gemm_cap, &n_gemm, stream));
   }
-  finalize_losses_kernel<<<1, 256, 0, stream>>>(row_part, M, X ? gemm_part : nullptr, gx * gy,
+  finalize_losses_kernel<<<1, 256, 0, stream>>>(row_part, M, X ? gemm_part : nullptr, n_gemm,
                                                 n_tok, damp_delta, delta_dev, losses_dev);
   CRVQ_LAUNCHED();
   return CRVQ_OK;

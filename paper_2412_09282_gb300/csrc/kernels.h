@@ -23,6 +23,14 @@ crvq_status launch_hessian(const float* X, int64_t n, int64_t N, int d, float da
 crvq_status launch_extract_blocks(const float* H, int64_t N, int d, const int32_t* perm,
                                   float* H_blocks, cudaStream_t stream);
 
+// Tensor-core (tcgen05, 3xTF32) products.
+// S = X^T X / n for X n x N row-major (S N x N, both triangles).
+crvq_status launch_tc_syrk(const float* X, int64_t n, int64_t N, float* S, cudaStream_t stream);
+// Partial sums of ||A B^T||_F^2 (A M x K, B Nb x K row-major) into part[0 .. *nparts).
+crvq_status launch_tc_sumsq(const float* A, int64_t M, const float* B, int64_t Nb, int64_t K,
+                            double* part, int64_t part_cap, int64_t* nparts,
+                            cudaStream_t stream);
+
 crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
                                   const float* W_pre, const float* xsq, const float* H,
                                   int mode, uint64_t seed, int32_t* perm, float* importance,

@@ -1,0 +1,140 @@
+// Host side of the tcgen05 3xTF32 GEMM (tc_gemm.cuh) and the fixed-order reductions of its
+// split-K partial products. The tensor core accumulates fp32 with a small systematic
+// rounding bias per accumulation step, so K is cut into chunks of at most kKChunk and the
+// chunk partials are summed afterwards in fp64, in chunk order.
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "tc_gemm.cuh"
+
+namespace crvq {
+
+namespace {
+
+constexpr int64_t kKChunk = 1024;
+
+// out[e] = scale * sum_c P[c * stride + e]  (fp64 sum, chunks in order)
+__global__ void __launch_bounds__(256)
+sum_partials_kernel(const float* __restrict__ P, int64_t count, int chunks, int64_t stride,
+                    double scale, float* __restrict__ out) {
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < count;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    double s = 0.0;
+    for (int c = 0; c < chunks; ++c) s += (double)P[c * stride + e];
+    out[e] = (float)(s * scale);
+  }
+}
+
+// part[block] = sum over this block's elements e of (sum_c P[c * stride + e])^2
+__global__ void __launch_bounds__(256)
+sumsq_partials_kernel(const float* __restrict__ P, int64_t count, int chunks, int64_t stride,
+                      double* __restrict__ part) {
+  __shared__ double red[256];
+  double acc = 0.0;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < count;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    double s = 0.0;
+    for (int c = 0; c < chunks; ++c) s += (double)P[c * stride + e];
+    acc += s * s;
+  }
+  red[threadIdx.x] = acc;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) part[blockIdx.x] = red[0];
+}
+
+crvq_status launch_gemm(tc::GemmArgs g, int64_t chunks, cudaStream_t stream) {
+  static bool attr_set[64] = {};
+  int dev = 0;
+  CRVQ_CUDA(cudaGetDevice(&dev));
+  if (dev < 64 && !attr_set[dev]) {
+    CRVQ_CUDA(cudaFuncSetAttribute(tc::gemm3xtf32_kernel,
+                                   cudaFuncAttributeMaxDynamicSharedMemorySize, tc::kSmemBytes));
+    attr_set[dev] = true;
+  }
+  const int64_t tm = ceil_div(g.A.rows, tc::kBM), tn = ceil_div(g.B.rows, tc::kBN);
+  g.tiles_n = (int)tn;
+  dim3 grid((unsigned)(tm * tn), (unsigned)chunks);
+  tc::gemm3xtf32_kernel<<<grid, tc::kThreads, tc::kSmemBytes, stream>>>(g);
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
+}
+
+}  // namespace
+
+// S = X^T X / n (X: n x N row-major) into S (N x N), both triangles, via split-K partials.
+crvq_status launch_tc_syrk(const float* X, int64_t n, int64_t N, float* S, cudaStream_t stream) {
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
+  const int64_t chunks = ceil_div(n, kKChunk);
+  Scratch mem;
+  float* P = S;
+  if (chunks > 1) {
+    CRVQ_TRY(mem.alloc((size_t)chunks * N * N * sizeof(float), stream));
+    P = mem.as<float>();
+  }
+  tc::GemmArgs g{};
+  g.A = tc::Operand{X, N, N, false};  // A(a, k) = X[k][a]
+  g.B = g.A;
+  g.K = n;
+  g.k_chunk = kKChunk;
+  g.c_chunk_stride = N * N;
+  g.mode = tc::kStoreSymmetric;
+  g.C = P;
+  g.ldc = N;
+  g.alpha = chunks > 1 ? 1.f : (float)(1.0 / (double)n);
+  g.err = err;
+  {
+    ProfScope ps("hessian_gemm_tc", stream, 2.0 * (double)n * N * N);
+    CRVQ_TRY(launch_gemm(g, chunks, stream));
+  }
+  if (chunks > 1) {
+    ProfScope ps("hessian_sum_partials", stream, (double)chunks * N * N * 4.0);
+    const int blocks = (int)std::min<int64_t>(ceil_div(N * N, 256), 16 * sm_count());
+    sum_partials_kernel<<<blocks, 256, 0, stream>>>(P, N * N, (int)chunks, N * N,
+                                                    1.0 / (double)n, S);
+    CRVQ_LAUNCHED();
+  }
+  return CRVQ_OK;
+}
+
+// part[0 .. nparts) = partial sums of ||A B^T||_F^2 with A: M x K, B: Nb x K (row-major,
+// leading dimension K); returns the number of partials written.
+crvq_status launch_tc_sumsq(const float* A, int64_t M, const float* B, int64_t Nb, int64_t K,
+                            double* part, int64_t part_cap, int64_t* nparts,
+                            cudaStream_t stream) {
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
+  const int64_t chunks = ceil_div(K, kKChunk);
+  Scratch mem;
+  CRVQ_TRY(mem.alloc((size_t)chunks * M * Nb * sizeof(float), stream));
+  float* P = mem.as<float>();
+  tc::GemmArgs g{};
+  g.A = tc::Operand{A, K, M, true};
+  g.B = tc::Operand{B, K, Nb, true};
+  g.K = K;
+  g.k_chunk = kKChunk;
+  g.c_chunk_stride = M * Nb;
+  g.mode = tc::kStore;
+  g.C = P;
+  g.ldc = Nb;
+  g.alpha = 1.f;
+  g.err = err;
+  {
+    ProfScope ps("loss_gemm_tc", stream, 2.0 * (double)M * Nb * K);
+    CRVQ_TRY(launch_gemm(g, chunks, stream));
+  }
+  const int blocks = (int)std::min<int64_t>(part_cap, std::min<int64_t>(
+                                                          ceil_div(M * Nb, 256), 8 * sm_count()));
+  ProfScope ps("loss_sumsq", stream, (double)chunks * M * Nb * 4.0);
+  sumsq_partials_kernel<<<blocks, 256, 0, stream>>>(P, M * Nb, (int)chunks, M * Nb, part);
+  CRVQ_LAUNCHED();
+  *nparts = blocks;
+  return CRVQ_OK;
+}
+
+}  // namespace crvq
