@@ -20,6 +20,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "stats.cuh"
+#include "tc_ops.cuh"
 
 namespace crvq {
 
@@ -179,104 +180,297 @@ __device__ __forceinline__ float low_score(const float c[kD], const float* H, co
   return fmaf(nbeta, l1, s);
 }
 
-// --------------------------------------------------------------------------- arg-min pass
-// One CTA = one group g and kThreads * VPT rows; each thread owns VPT vectors. When
-// st.cnt != null the certified codes' least-squares statistics are accumulated (stats.cuh).
-template <int VPT>
-__global__ void __launch_bounds__(kThreads, 4)
-argmin_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
-              int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0, FlagList flags,
-              StatsView st, unsigned* err) {
+// --------------------------------------------------------------------------- arg-min pass on
+// the tensor cores. The whole certified lower bound is one dot product of length 32:
+//   D[v][k] = sum_p q_vp c_kp + n'_k + beta_v L1_k + off_v = low_k(v) + off_v,
+//   q = -2 H_g r, n' = n - u C Na, beta = -2 u C Pmax, off >= r^T H r + bound (so D >= 0),
+// with every term split into tf32 hi + lo (3xTF32: hi*hi + hi*lo + lo*hi):
+//   A row (vector):   [q_hi x8 | q_hi x8 | q_lo x8 | 1 1 | beta_hi beta_hi beta_lo | off_hi off_lo | 0]
+//   B row (codeword): [c_hi x8 | c_lo x8 | c_hi x8 | n'_hi n'_lo | L1_hi L1_lo L1_hi | 1 1 | 0]
+// One tcgen05.mma M = 128 vectors x N = 256 codewords x K = 8, four per tile (K = 32), fp32
+// accumulator in tensor memory. The epilogue reads each row's 256 scores, packs the codeword's
+// index into the low 8 mantissa bits of the (non-negative) fp32 bound (a truncation of at most
+// 2^-15 relative) and keeps the two smallest keys with integer min / max. The certificate and
+// the fp64 fallback are those of the fp32 pass, with the bound multiplier raised to cover the
+// tensor-core products and accumulation (about 2^-22 per split product and fp32 accumulation
+// over 32 terms) and the packing.
+namespace tcenc {
+
+constexpr int kRows = 128;        // vectors per row tile (TMEM lanes)
+constexpr int kCols = 256;        // codewords per chunk (MMA N)
+constexpr int kK = 32;            // tf32 columns per row
+constexpr int kATile = kRows * kK * 4;   // 16 KB
+constexpr int kBTile = kCols * kK * 4;   // 32 KB
+constexpr float kCmul = 256.f;           // bound multiplier (about twice the analysis)
+constexpr float kPack = 3.0517578e-05f;  // 2^-15: relative truncation of the packed key
+constexpr uint32_t kIdesc = tc::idesc_tf32(kRows, kCols);
+
+__device__ __forceinline__ uint32_t koff(int r, int k) {
+  return (uint32_t)(((r >> 3) * (kK / 4) + (k >> 2)) * 128 + (r & 7) * 16 + (k & 3) * 4);
+}
+
+// Writes the 32 tf32 values v[0..31] of row r (hi parts given as fp32 values).
+__device__ __forceinline__ void put_row(char* tile, int r, const uint32_t v[kK]) {
+#pragma unroll
+  for (int q = 0; q < kK / 4; ++q)
+    *reinterpret_cast<uint4*>(tile + koff(r, 4 * q)) =
+        make_uint4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+}
+
+__device__ __forceinline__ void split(float x, uint32_t& hi, uint32_t& lo) {
+  hi = tc::to_tf32(x);
+  lo = tc::to_tf32(x - __uint_as_float(hi));
+}
+
+}  // namespace tcenc
+
+template <int R>
+__global__ void __launch_bounds__(128, 2)
+argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
+                 int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
+                 FlagList flags, StatsView st, const float* __restrict__ cbmax,
+                 unsigned* err) {
+  using namespace tcenc;
+  extern __shared__ __align__(1024) char smem_raw[];
+  char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                       ~(uintptr_t)1023);
+  char* Btile = smem;                  // 32 KB
+  char* Atiles = smem + kBTile;        // R x 16 KB
+  __shared__ float sH[kD * kD];
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ uint32_t tmem_slot;
+
   const int64_t g = g_begin + blockIdx.y;
   const int64_t G_range = gridDim.y;
-  const int64_t row0 = (int64_t)blockIdx.x * kThreads * VPT;
-  __shared__ float sH[kD * kD];
-  __shared__ __align__(16) float sC[kChunk * kD];
-  __shared__ float sN[kChunk], sL[kChunk];
-
-  if (threadIdx.x < kD * kD) sH[threadIdx.x] = set.Hb[g * kD * kD + threadIdx.x];
-  __syncthreads();
-
+  const int tid = threadIdx.x, warp = tid >> 5;
   const CbView cw = cbs.cb[s_idx];
-  const float cmul = bound_mult(n_fixed);
-  float m2q[VPT][kD], nbeta[VPT];
-  float b1[VPT], b2[VPT];
-  int i1[VPT];
+  const float cmul = kCmul + 4.f * n_fixed;
+  const float uc = kU * cmul;
+
+  if (tid < kD * kD) sH[tid] = set.Hb[g * kD * kD + tid];
+  if (warp == 0) tc::tmem_alloc(&tmem_slot, kCols);
+  if (tid == 0) {
+    tc::mbar_init(tc::smem_u32(&bar), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+
+  // Bound on Na_k over the codebook for this group: (max row sum |H_g|) L1max cinfmax.
+  float hrow = 0.f;
 #pragma unroll
-  for (int v = 0; v < VPT; ++v) {
-    const int64_t i = row0 + threadIdx.x + (int64_t)v * kThreads;
-    float r[kD], a[kD], pmax;
+  for (int a = 0; a < kD; ++a) {
+    float rs = 0.f;
+#pragma unroll
+    for (int b = 0; b < kD; ++b) rs += fabsf(sH[a * kD + b]);
+    hrow = fmaxf(hrow, rs);
+  }
+  const float l1max = cbmax[0], cinf = cbmax[1];
+
+  // Prologue: the A rows of this CTA's R row tiles (thread = row in each tile).
+  float pmax_r[R], off_r[R], q_r[R][kD];
+  uint32_t g1[R], g2[R];
+  int gch[R];
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    const int64_t i = ((int64_t)blockIdx.x * R + r) * kRows + tid;
+    float rv[kD], a[kD], m2q[kD], pmax;
     if (i < set.M) {
-      target32(set, cbs, n_fixed, i, g, r, a, err);
+      target32(set, cbs, n_fixed, i, g, rv, a, err);
     } else {
 #pragma unroll
-      for (int j = 0; j < kD; ++j) r[j] = a[j] = 0.f;
+      for (int j = 0; j < kD; ++j) rv[j] = a[j] = 0.f;
     }
-    vector_terms(r, a, sH, m2q[v], pmax);
-    nbeta[v] = -2.f * kU * cmul * pmax;
-    b1[v] = INFINITY;
-    b2[v] = INFINITY;
-    i1[v] = 0;
+    vector_terms(rv, a, sH, m2q, pmax);
+    float rr = 0.f, ra = 0.f;
+#pragma unroll
+    for (int p = 0; p < kD; ++p) {
+      rr = fmaf(rv[p], -0.5f * m2q[p], rr);
+      float pa = 0.f;
+#pragma unroll
+      for (int j = 0; j < kD; ++j) pa = fmaf(fabsf(sH[p * kD + j]), a[j], pa);
+      ra = fmaf(a[p], pa, ra);
+    }
+    // offset so that every D = low + off is >= 0, with margins for every rounding involved
+    const float off = (rr + 32.f * kU * ra + 2.f * uc * (hrow * l1max * cinf + 2.f * pmax * l1max)) *
+                          (1.f + 4.f * uc) + 1e-30f;
+    const float beta = -2.f * uc * pmax;
+    uint32_t row[kK];
+#pragma unroll
+    for (int p = 0; p < kD; ++p) {
+      uint32_t h, l;
+      split(m2q[p], h, l);
+      row[p] = h;
+      row[8 + p] = h;
+      row[16 + p] = l;
+    }
+    const uint32_t one = __float_as_uint(1.f);
+    row[24] = one;
+    row[25] = one;
+    split(beta, row[26], row[28]);
+    row[27] = row[26];
+    split(off * (1.f - uc), row[29], row[30]);
+    row[31] = 0u;
+    put_row(Atiles + r * kATile, tid, row);
+    pmax_r[r] = pmax;
+    off_r[r] = off;
+#pragma unroll
+    for (int p = 0; p < kD; ++p) q_r[r][p] = -0.5f * m2q[p];
+    g1[r] = 0xffffffffu;
+    g2[r] = 0xffffffffu;
+    gch[r] = 0;
   }
 
-  for (int k0 = 0; k0 < cw.K; k0 += kChunk) {
-    const int nk = min(kChunk, cw.K - k0);
-    __syncthreads();
-    stage_chunk(cw.C, k0, nk, sH, cmul, sC, sN, sL);
-    __syncthreads();
-#pragma unroll 2
-    for (int k = 0; k < nk; ++k) {
-      const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
-      const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
-      const float n = sN[k], l1 = sL[k];
+  uint32_t phase = 0;
+  bool ok = true;
+  for (int kc = 0; kc < cw.K; kc += kCols) {
+    // B tile: codewords kc .. kc + 255 of the stage codebook (padding rows score +1e30).
 #pragma unroll
-      for (int v = 0; v < VPT; ++v) {
-        // two independent FMA chains (latency), summed once
-        float s = fmaf(m2q[v][0], c0.x, n);
-        float t = nbeta[v] * l1;
-        s = fmaf(m2q[v][1], c0.y, s);
-        t = fmaf(m2q[v][4], c1.x, t);
-        s = fmaf(m2q[v][2], c0.z, s);
-        t = fmaf(m2q[v][5], c1.y, t);
-        s = fmaf(m2q[v][3], c0.w, s);
-        t = fmaf(m2q[v][6], c1.z, t);
-        t = fmaf(m2q[v][7], c1.w, t);
-        s += t;
-        b2[v] = fminf(b2[v], fmaxf(s, b1[v]));
-        const bool lt = s < b1[v];
-        i1[v] = lt ? k0 + k : i1[v];
-        b1[v] = lt ? s : b1[v];
+    for (int h = 0; h < kCols / 128; ++h) {
+      const int k = tid + 128 * h;
+      uint32_t row[kK];
+      if (kc + k < cw.K) {
+        float c[kD], n, na, l1;
+        load_vec(cw.C + (int64_t)(kc + k) * kD, c);
+        codeword_terms(c, sH, n, na, l1);
+#pragma unroll
+        for (int p = 0; p < kD; ++p) {
+          uint32_t hh, ll;
+          split(c[p], hh, ll);
+          row[p] = hh;
+          row[8 + p] = ll;
+          row[16 + p] = hh;
+        }
+        split(n - uc * na, row[24], row[25]);
+        split(l1, row[26], row[27]);
+        row[28] = row[26];
+      } else {
+#pragma unroll
+        for (int p = 0; p < 24; ++p) row[p] = 0u;
+        row[24] = __float_as_uint(1e30f);
+        row[25] = 0u;
+        row[26] = row[27] = row[28] = 0u;
       }
+      row[29] = row[30] = __float_as_uint(1.f);
+      row[31] = 0u;
+      put_row(Btile, k, row);
     }
-  }
+    tc::fence_async_smem();
+    __syncthreads();
+#pragma unroll 1
+    for (int r = 0; r < R; ++r) {
+      if (tid == 0 && ok) {
+        tc::tc_fence_after();
+        const uint32_t a0 = tc::smem_u32(Atiles + r * kATile), b0 = tc::smem_u32(Btile);
 #pragma unroll
-  for (int v = 0; v < VPT; ++v) {
-    const int64_t i = row0 + threadIdx.x + (int64_t)v * kThreads;
+        for (int ks = 0; ks < kK / 8; ++ks)
+          tc::mma_tf32(tmem, tc::smem_desc(a0 + ks * 256, 128, (kK / 4) * 128),
+                       tc::smem_desc(b0 + ks * 256, 128, (kK / 4) * 128), kIdesc,
+                       ks > 0 ? 1u : 0u);
+        tc::mma_commit(tc::smem_u32(&bar));
+      }
+      if (ok) ok = tc::mbar_wait(tc::smem_u32(&bar), phase, err);
+      phase ^= 1u;
+      ok = __syncthreads_and(ok);
+      tc::tc_fence_after();
+      if (ok) {
+        uint32_t t1 = 0xffffffffu, t2 = 0xffffffffu;
+#pragma unroll 1
+        for (int c0 = 0; c0 < kCols; c0 += 32) {
+          float v[32];
+          tc::tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+#pragma unroll
+          for (int j = 0; j < 32; ++j) {
+            const uint32_t key = (__float_as_uint(v[j]) & 0xffffff00u) | (uint32_t)(c0 + j);
+            const uint32_t hi = max(t1, key);
+            t1 = min(t1, key);
+            t2 = min(t2, hi);
+          }
+        }
+        if (t1 < g1[r]) {
+          g2[r] = min(g1[r], t2);
+          g1[r] = t1;
+          gch[r] = kc;
+        } else {
+          g2[r] = min(g2[r], t1);
+        }
+      }
+      tc::tc_fence_before();
+      __syncthreads();
+    }
+    if (!ok) break;
+  }
+
+  // Certificate, codes, flags and statistics per row.
+#pragma unroll
+  for (int r = 0; r < R; ++r) {
+    const int64_t i = ((int64_t)blockIdx.x * R + r) * kRows + tid;
     if (i >= set.M) continue;
-    // Winner's bound Et_j = u C (Na_j + 2 Pmax L1_j), recomputed from c_j.
-    float c[kD];
-    load_vec(cw.C + (int64_t)i1[v] * kD, c);
-    float n, na, l1;
-    codeword_terms(c, sH, n, na, l1);
-    const float Et = kU * cmul * na - 0.5f * nbeta[v] * l1;
-    const bool cert = b2[v] - b1[v] > 2.f * Et;
+    int j = gch[r] + (int)(g1[r] & 0xffu);
+    const float k1 = __uint_as_float(g1[r]), k2 = __uint_as_float(g2[r]);
+    bool cert = false;
+    float thr = INFINITY;
+    if (ok && j < cw.K) {
+      float c[kD], n, na, l1;
+      load_vec(cw.C + (int64_t)j * kD, c);
+      codeword_terms(c, sH, n, na, l1);
+      // |key - D| <= 2^-15 D; D_k <= s_k + off (every k); s_j + off <= D_j + e2 (winner).
+      const float e2 = 2.f * uc * (na + 2.f * pmax_r[r] * l1 + off_r[r]);
+      const float top = k1 * (1.f + 2.5f * kPack) + e2;   // >= s_j + off
+      cert = cw.K == 1 || (k2 * (1.f - kPack) > top);
+      thr = top - off_r[r];
+      thr += 4.f * kU * (k1 + off_r[r] + e2);
+    } else {
+      j = 0;
+    }
     if (!cert) {
       const unsigned slot = atomicAdd(flags.count, 1u);
       if (slot < flags.cap) {
         flags.vec[slot] = i * G_range + (g - g_begin);
-        flags.thr[slot] = b1[v] + 2.f * Et;
+        flags.thr[slot] = thr;
       } else {
         raise_error(err, ERRBIT_INDEX);
       }
     }
-    // Always write the fast-pass winner; the fallback overwrites uncertain ones.
-    out_code[i * out_ld + (g - out_g0)] = i1[v];
-    if (cert && st.cnt) {
-      float q[kD];
+    out_code[i * out_ld + (g - out_g0)] = j;
+    if (cert && st.cnt) stats_add(st, *st.scale, g, j, q_r[r]);
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, kCols);
+}
+
+// cbmax[0] = max_k ||c_k||_1, cbmax[1] = max_k,j |c_kj| (one CTA; maxima are order-free).
+__global__ void __launch_bounds__(256)
+cbmax_kernel(const float* __restrict__ C, int K, float* __restrict__ cbmax) {
+  __shared__ float r1[256], r2[256];
+  float l1m = 0.f, cm = 0.f;
+  for (int k = threadIdx.x; k < K; k += blockDim.x) {
+    float c[kD];
+    load_vec(C + (int64_t)k * kD, c);
+    float l1 = 0.f;
 #pragma unroll
-      for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[v][p];
-      stats_add(st, *st.scale, g, i1[v], q);
+    for (int j = 0; j < kD; ++j) {
+      l1 += fabsf(c[j]);
+      cm = fmaxf(cm, fabsf(c[j]));
     }
+    l1m = fmaxf(l1m, l1);
+  }
+  r1[threadIdx.x] = l1m;
+  r2[threadIdx.x] = cm;
+  __syncthreads();
+  for (int w = 128; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w) {
+      r1[threadIdx.x] = fmaxf(r1[threadIdx.x], r1[threadIdx.x + w]);
+      r2[threadIdx.x] = fmaxf(r2[threadIdx.x], r2[threadIdx.x + w]);
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    cbmax[0] = r1[0] * (1.f + 1e-6f);
+    cbmax[1] = r2[0];
   }
 }
 
@@ -741,6 +935,12 @@ __global__ void kmeans_init_kernel(SetView set, CbList fixed, int K, uint64_t se
 }  // namespace
 
 // =============================================================================== host side
+template <class Kern>
+static crvq_status set_smem_attr(Kern k, size_t bytes) {
+  CRVQ_CUDA(cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes));
+  return CRVQ_OK;
+}
+
 crvq_status launch_kmeans_init(const SetView& set, const CbList& fixed, int K, uint64_t seed,
                                float* C_out, cudaStream_t stream) {
   unsigned* err = nullptr;
@@ -824,17 +1024,25 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     StatsView st{};
     if (ex.stats && !keep_if_better) st = *ex.stats;
     CRVQ_CUDA(cudaMemsetAsync(fl.count, 0, sizeof(unsigned), stream));
-    const bool big = (ceil_div(set.M, kThreads * 4) * G_range) >= 2 * nsm;
+    float* cbmax = reinterpret_cast<float*>(flag_mem.as<char>() + 128);
+    cbmax_kernel<<<1, 256, 0, stream>>>(cw.C, cw.K, cbmax);
+    CRVQ_LAUNCHED();
     {
+      // R row tiles of 128 vectors per CTA share one staged codebook chunk; at most two CTAs
+      // per SM (their tensor memory, 256 columns each, fills the SM's 512).
+      const int64_t row_tiles = ceil_div(set.M, tcenc::kRows);
+      const int R = (ceil_div(row_tiles, 4) * G_range >= 2 * nsm) ? 4 : 1;
+      const size_t smem = (size_t)tcenc::kBTile + 4 * (size_t)tcenc::kATile + 1024;
+      dim3 grid((unsigned)ceil_div(row_tiles, R), (unsigned)G_range);
       ProfScope ps("encode_argmin", stream, (double)nvec * cw.K);
-      if (big) {
-        dim3 grid((unsigned)ceil_div(set.M, kThreads * 4), (unsigned)G_range);
-        argmin_kernel<4><<<grid, kThreads, 0, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                        out_ld, out_g0, fl, st, err);
+      if (R == 4) {
+        CRVQ_TRY(set_smem_attr(argmin_tc_kernel<4>, smem));
+        argmin_tc_kernel<4><<<grid, 128, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
+                                                         out_ld, out_g0, fl, st, cbmax, err);
       } else {
-        dim3 grid((unsigned)ceil_div(set.M, kThreads), (unsigned)G_range);
-        argmin_kernel<1><<<grid, kThreads, 0, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                        out_ld, out_g0, fl, st, err);
+        CRVQ_TRY(set_smem_attr(argmin_tc_kernel<1>, smem));
+        argmin_tc_kernel<1><<<grid, 128, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
+                                                         out_ld, out_g0, fl, st, cbmax, err);
       }
       CRVQ_LAUNCHED();
     }
