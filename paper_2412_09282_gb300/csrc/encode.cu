@@ -231,76 +231,50 @@ __device__ __forceinline__ void merge2(uint32_t& x1, uint32_t& x2, uint32_t y1, 
   x2 = min(hi, min(x2, y2));
 }
 
-// 8 warps: warps w and w + 4 read the same 32 tensor-memory lanes (rows) and split the 256
-// columns; two accumulator buffers (512 columns) let the MMA of the next row tile run during
-// this tile's epilogue; the codebook chunk (B tile) is double-buffered as well.
-template <int R>
-__global__ void __launch_bounds__(256, 1)
+// Two 256-thread CTAs per SM, each holding two row tiles of 128 vectors (thread t owns row
+// t % 128 of tile t / 128) and one 256-column accumulator. Warps w and w + 4 read the same 32
+// tensor-memory lanes and split the 256 codeword columns; the owner half of the tile merges
+// the two halves. While one CTA runs its FMA-heavy prologue or certificate, the other's
+// ALU-heavy epilogue and the tensor core keep the SM busy.
+constexpr int kTcRowTiles = 2;
+
+__global__ void __launch_bounds__(256, 2)
 argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
                  int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
                  FlagList flags, StatsView st, const float* __restrict__ cbmax,
                  unsigned* err) {
   using namespace tcenc;
+  constexpr int R = kTcRowTiles;
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                        ~(uintptr_t)1023);
-  char* Btiles = smem;                 // 2 x 32 KB
-  char* Atiles = smem + 2 * kBTile;    // R x 16 KB
+  char* Btile = smem;                  // 32 KB
+  char* Atiles = smem + kBTile;        // R x 16 KB
   __shared__ float sH[kD * kD];
-  __shared__ __align__(8) uint64_t bars[2];
+  __shared__ __align__(8) uint64_t bar;
   __shared__ uint32_t tmem_slot;
   __shared__ uint32_t part1[128], part2[128];
+  __shared__ float sq[8][256];  // each row's H r (least-squares statistics), column-major
 
   const int64_t g = g_begin + blockIdx.y;
   const int64_t G_range = gridDim.y;
   const int tid = threadIdx.x, warp = tid >> 5;
+  const int my_tile = tid >> 7, my_row = tid & 127;
+  const int64_t i = ((int64_t)blockIdx.x * R + my_tile) * kRows + my_row;
   const CbView cw = cbs.cb[s_idx];
   const float cmul = kCmul + 4.f * n_fixed;
   const float uc = kU * cmul;
 
   if (tid < kD * kD) sH[tid] = set.Hb[g * kD * kD + tid];
-  if (warp == 0) tc::tmem_alloc(&tmem_slot, 2 * kCols);
+  if (warp == 0) tc::tmem_alloc(&tmem_slot, kCols);
   if (tid == 0) {
-    tc::mbar_init(tc::smem_u32(&bars[0]), 1);
-    tc::mbar_init(tc::smem_u32(&bars[1]), 1);
+    tc::mbar_init(tc::smem_u32(&bar), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
   const uint32_t tmem = tmem_slot;
-
-  // Stages the B tile of chunk c (codewords c*256 .. c*256 + 255; padding rows score +1e30).
-  auto prep_B = [&](int c, char* Bt) {
-    const int k = tid;  // 256 threads, one codeword each
-    const int kk = c * kCols + k;
-    uint32_t row[kK];
-    if (kk < cw.K) {
-      float cv[kD], n, na, l1;
-      load_vec(cw.C + (int64_t)kk * kD, cv);
-      codeword_terms(cv, sH, n, na, l1);
-#pragma unroll
-      for (int p = 0; p < kD; ++p) {
-        uint32_t hh, ll;
-        split(cv[p], hh, ll);
-        row[p] = hh;
-        row[8 + p] = ll;
-        row[16 + p] = hh;
-      }
-      split(n - uc * na, row[24], row[25]);
-      split(l1, row[26], row[27]);
-      row[28] = row[26];
-    } else {
-#pragma unroll
-      for (int p = 0; p < 24; ++p) row[p] = 0u;
-      row[24] = __float_as_uint(1e30f);
-      row[25] = 0u;
-      row[26] = row[27] = row[28] = 0u;
-    }
-    row[29] = row[30] = __float_as_uint(1.f);
-    row[31] = 0u;
-    put_row(Bt, k, row);
-  };
 
   // Bound on Na_k over the codebook for this group: (max row sum |H_g|) L1max cinfmax.
   float hrow = 0.f;
@@ -313,208 +287,195 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   }
   const float l1max = cbmax[0], cinf = cbmax[1];
 
-  // Prologue (threads 0..127): the A rows of this CTA's R row tiles; per-row state.
-  float pmax_r[R], off_r[R], q_r[R][kD];
-  uint32_t g1[R], g2[R];
-  int gch[R];
+  // Prologue: this thread's A row and row state.
+  float pmax, off;
+  {
+    float rv[kD], a[kD], m2q[kD];
+    if (i < set.M) {
+      target32(set, cbs, n_fixed, i, g, rv, a, err);
+    } else {
 #pragma unroll
-  for (int r = 0; r < R; ++r) {
-    g1[r] = 0xffffffffu;
-    g2[r] = 0xffffffffu;
-    gch[r] = 0;
-    pmax_r[r] = 0.f;
-    off_r[r] = 0.f;
-#pragma unroll
-    for (int p = 0; p < kD; ++p) q_r[r][p] = 0.f;
-  }
-  if (tid < kRows) {
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int64_t i = ((int64_t)blockIdx.x * R + r) * kRows + tid;
-      float rv[kD], a[kD], m2q[kD], pmax;
-      if (i < set.M) {
-        target32(set, cbs, n_fixed, i, g, rv, a, err);
-      } else {
-#pragma unroll
-        for (int j = 0; j < kD; ++j) rv[j] = a[j] = 0.f;
-      }
-      vector_terms(rv, a, sH, m2q, pmax);
-      float rr = 0.f, ra = 0.f;
-#pragma unroll
-      for (int p = 0; p < kD; ++p) {
-        rr = fmaf(rv[p], -0.5f * m2q[p], rr);
-        float pa = 0.f;
-#pragma unroll
-        for (int j = 0; j < kD; ++j) pa = fmaf(fabsf(sH[p * kD + j]), a[j], pa);
-        ra = fmaf(a[p], pa, ra);
-      }
-      // offset making every D = low + off >= 0, with margins for every rounding involved
-      const float off =
-          (rr + 32.f * kU * ra + 2.f * uc * (hrow * l1max * cinf + 2.f * pmax * l1max)) *
-              (1.f + 4.f * uc) + 1e-30f;
-      const float beta = -2.f * uc * pmax;
-      uint32_t row[kK];
-#pragma unroll
-      for (int p = 0; p < kD; ++p) {
-        uint32_t h, l;
-        split(m2q[p], h, l);
-        row[p] = h;
-        row[8 + p] = h;
-        row[16 + p] = l;
-      }
-      const uint32_t one = __float_as_uint(1.f);
-      row[24] = one;
-      row[25] = one;
-      split(beta, row[26], row[28]);
-      row[27] = row[26];
-      split(off * (1.f - uc), row[29], row[30]);
-      row[31] = 0u;
-      put_row(Atiles + r * kATile, tid, row);
-      pmax_r[r] = pmax;
-      off_r[r] = off;
-#pragma unroll
-      for (int p = 0; p < kD; ++p) q_r[r][p] = -0.5f * m2q[p];
+      for (int j = 0; j < kD; ++j) rv[j] = a[j] = 0.f;
     }
-  }
-  prep_B(0, Btiles);
-  tc::fence_async_smem();
-  __syncthreads();
-
-  const int nch = (cw.K + kCols - 1) / kCols;
-  const int nsteps = nch * R;
-  auto issue = [&](int s) {  // MMA of step s (chunk s / R, row tile s % R) into buffer s & 1
-    tc::tc_fence_after();
-    const int c = s / R, r = s % R;
-    const uint32_t a0 = tc::smem_u32(Atiles + r * kATile);
-    const uint32_t b0 = tc::smem_u32(Btiles + (c & 1) * kBTile);
-    const uint32_t d = tmem + (uint32_t)((s & 1) * kCols);
+    vector_terms(rv, a, sH, m2q, pmax);
+    float rr = 0.f, ra = 0.f;
 #pragma unroll
-    for (int ks = 0; ks < kK / 8; ++ks)
-      tc::mma_tf32(d, tc::smem_desc(a0 + ks * 256, 128, (kK / 4) * 128),
-                   tc::smem_desc(b0 + ks * 256, 128, (kK / 4) * 128), kIdesc, ks > 0 ? 1u : 0u);
-    tc::mma_commit(tc::smem_u32(&bars[s & 1]));
-  };
-  if (tid == 0) issue(0);
-  int issued = 1, waited = 0;
-  uint32_t wpar[2] = {0u, 0u};
+    for (int p = 0; p < kD; ++p) {
+      rr = fmaf(rv[p], -0.5f * m2q[p], rr);
+      float pa = 0.f;
+#pragma unroll
+      for (int j = 0; j < kD; ++j) pa = fmaf(fabsf(sH[p * kD + j]), a[j], pa);
+      ra = fmaf(a[p], pa, ra);
+    }
+    // offset making every D = low + off >= 0, with margins for every rounding involved
+    off = (rr + 32.f * kU * ra + 2.f * uc * (hrow * l1max * cinf + 2.f * pmax * l1max)) *
+              (1.f + 4.f * uc) + 1e-30f;
+    const float beta = -2.f * uc * pmax;
+    uint32_t row[kK];
+#pragma unroll
+    for (int p = 0; p < kD; ++p) {
+      uint32_t h, l;
+      split(m2q[p], h, l);
+      row[p] = h;
+      row[8 + p] = h;
+      row[16 + p] = l;
+      sq[p][tid] = -0.5f * m2q[p];
+    }
+    const uint32_t one = __float_as_uint(1.f);
+    row[24] = one;
+    row[25] = one;
+    split(beta, row[26], row[28]);
+    row[27] = row[26];
+    split(off * (1.f - uc), row[29], row[30]);
+    row[31] = 0u;
+    put_row(Atiles + my_tile * kATile, my_row, row);
+  }
+  uint32_t g1 = 0xffffffffu, g2 = 0xffffffffu;
+  int gch = 0;
+
+  uint32_t phase = 0;
   bool ok = true;
   const int lq = warp & 3, half = warp >> 2;
-
-  for (int s = 0; s < nsteps; ++s) {
-    const int c = s / R, r = s % R, buf = s & 1;
-    if (r == 0 && c + 1 < nch) {
-      // chunk c + 1's codewords into the other B buffer (its last reader, chunk c - 1, is done)
-      prep_B(c + 1, Btiles + ((c + 1) & 1) * kBTile);
-      tc::fence_async_smem();
-      __syncthreads();
-    }
-    if (ok && s + 1 < nsteps) {
-      if (tid == 0) issue(s + 1);
-      ++issued;
-    }
-    if (ok) ok = tc::mbar_wait(tc::smem_u32(&bars[buf]), wpar[buf], err);
-    wpar[buf] ^= 1u;
-    ++waited;
-    ok = __syncthreads_and(ok);
-    if (!ok) break;
-    tc::tc_fence_after();
-    // Epilogue: 128 columns of this warp's 32 rows; four independent top-2 chains.
-    uint32_t v[4][32];
-    const uint32_t base = tmem + (uint32_t)(buf * kCols) + ((uint32_t)(lq * 32) << 16) +
-                          (uint32_t)(half * 128);
+  for (int kc = 0; kc < cw.K && ok; kc += kCols) {
+    // B tile: codewords kc .. kc + 255 (one per thread; padding rows score +1e30).
+    {
+      const int kk = kc + tid;
+      uint32_t row[kK];
+      if (kk < cw.K) {
+        float cv[kD], n, na, l1;
+        load_vec(cw.C + (int64_t)kk * kD, cv);
+        codeword_terms(cv, sH, n, na, l1);
 #pragma unroll
-    for (int b = 0; b < 4; ++b) tc::tmem_ld32_nowait(base + 32 * b, v[b]);
-    tc::tmem_wait_ld();
-    uint32_t a1[4], a2[4];
+        for (int p = 0; p < kD; ++p) {
+          uint32_t hh, ll;
+          split(cv[p], hh, ll);
+          row[p] = hh;
+          row[8 + p] = ll;
+          row[16 + p] = hh;
+        }
+        split(n - uc * na, row[24], row[25]);
+        split(l1, row[26], row[27]);
+        row[28] = row[26];
+      } else {
 #pragma unroll
-    for (int b = 0; b < 4; ++b) {
-      a1[b] = 0xffffffffu;
-      a2[b] = 0xffffffffu;
+        for (int p = 0; p < 24; ++p) row[p] = 0u;
+        row[24] = __float_as_uint(1e30f);
+        row[25] = 0u;
+        row[26] = row[27] = row[28] = 0u;
+      }
+      row[29] = row[30] = __float_as_uint(1.f);
+      row[31] = 0u;
+      put_row(Btile, tid, row);
     }
+    tc::fence_async_smem();
+    __syncthreads();
+#pragma unroll 1
+    for (int r = 0; r < R; ++r) {
+      if (tid == 0) {
+        tc::tc_fence_after();
+        const uint32_t a0 = tc::smem_u32(Atiles + r * kATile), b0 = tc::smem_u32(Btile);
 #pragma unroll
-    for (int j = 0; j < 32; ++j) {
+        for (int ks = 0; ks < kK / 8; ++ks)
+          tc::mma_tf32(tmem, tc::smem_desc(a0 + ks * 256, 128, (kK / 4) * 128),
+                       tc::smem_desc(b0 + ks * 256, 128, (kK / 4) * 128), kIdesc,
+                       ks > 0 ? 1u : 0u);
+        tc::mma_commit(tc::smem_u32(&bar));
+      }
+      ok = tc::mbar_wait(tc::smem_u32(&bar), phase, err);
+      phase ^= 1u;
+      ok = __syncthreads_and(ok);
+      if (!ok) break;
+      tc::tc_fence_after();
+      // 128 columns of this warp's 32 rows, two 64-column rounds, four top-2 chains.
+      uint32_t a1[4], a2[4];
 #pragma unroll
       for (int b = 0; b < 4; ++b) {
-        const uint32_t key = (v[b][j] & 0xffffff00u) | (uint32_t)j;
-        const uint32_t hi = max(a1[b], key);
-        a1[b] = min(a1[b], key);
-        a2[b] = min(a2[b], hi);
+        a1[b] = 0xffffffffu;
+        a2[b] = 0xffffffffu;
       }
-    }
-    // add the column base of each block (the keys' low 8 bits become the chunk column)
-    uint32_t t1 = a1[0] | (uint32_t)(half * 128), t2 = a2[0] | (uint32_t)(half * 128);
+      const uint32_t base = tmem + ((uint32_t)(lq * 32) << 16) + (uint32_t)(half * 128);
 #pragma unroll
-    for (int b = 1; b < 4; ++b)
-      merge2(t1, t2, a1[b] | (uint32_t)(half * 128 + 32 * b),
-             a2[b] | (uint32_t)(half * 128 + 32 * b));
-    if (half == 1) {
-      part1[lq * 32 + (tid & 31)] = t1;
-      part2[lq * 32 + (tid & 31)] = t2;
-    }
-    tc::tc_fence_before();
-    __syncthreads();
-    if (half == 0) {
-      merge2(t1, t2, part1[tid], part2[tid]);
-      // merge into the row state of tile r (runtime index: select by unrolled compare)
+      for (int rnd = 0; rnd < 2; ++rnd) {
+        uint32_t v0[32], v1[32];
+        tc::tmem_ld32_nowait(base + 64 * rnd, v0);
+        tc::tmem_ld32_nowait(base + 64 * rnd + 32, v1);
+        tc::tmem_wait_ld();
 #pragma unroll
-      for (int rr = 0; rr < R; ++rr) {
-        if (rr == r) {
-          if (t1 < g1[rr]) {
-            g2[rr] = min(g1[rr], t2);
-            g1[rr] = t1;
-            gch[rr] = c * kCols;
-          } else {
-            g2[rr] = min(g2[rr], t1);
-          }
+        for (int j = 0; j < 32; ++j) {
+          const uint32_t k0 = (v0[j] & 0xffffff00u) | (uint32_t)j;
+          const uint32_t k1 = (v1[j] & 0xffffff00u) | (uint32_t)j;
+          const uint32_t h0 = max(a1[2 * rnd], k0), h1 = max(a1[2 * rnd + 1], k1);
+          a1[2 * rnd] = min(a1[2 * rnd], k0);
+          a1[2 * rnd + 1] = min(a1[2 * rnd + 1], k1);
+          a2[2 * rnd] = min(a2[2 * rnd], h0);
+          a2[2 * rnd + 1] = min(a2[2 * rnd + 1], h1);
         }
       }
+      // the keys' low 8 bits become the chunk column: half * 128 + 32 * block + j
+      uint32_t t1 = a1[0] | (uint32_t)(half * 128), t2 = a2[0] | (uint32_t)(half * 128);
+#pragma unroll
+      for (int b = 1; b < 4; ++b)
+        merge2(t1, t2, a1[b] | (uint32_t)(half * 128 + 32 * b),
+               a2[b] | (uint32_t)(half * 128 + 32 * b));
+      if (half != r) {
+        part1[lq * 32 + (tid & 31)] = t1;
+        part2[lq * 32 + (tid & 31)] = t2;
+      }
+      tc::tc_fence_before();
+      __syncthreads();
+      if (half == r) {  // owner half of tile r: its threads hold the rows' state
+        merge2(t1, t2, part1[lq * 32 + (tid & 31)], part2[lq * 32 + (tid & 31)]);
+        if (t1 < g1) {
+          g2 = min(g1, t2);
+          g1 = t1;
+          gch = kc;
+        } else {
+          g2 = min(g2, t1);
+        }
+      }
+      __syncthreads();  // part1/part2 and the accumulator are free for the next tile
     }
-  }
-  // an MMA issued but not waited for (only after a timeout): wait for it, bounded
-  if (issued > waited) {
-    const int s = issued - 1;
-    tc::mbar_wait(tc::smem_u32(&bars[s & 1]), wpar[s & 1], err);
   }
 
-  // Certificate, codes, flags and statistics per row (threads 0..127).
-  if (tid < kRows) {
-#pragma unroll
-    for (int r = 0; r < R; ++r) {
-      const int64_t i = ((int64_t)blockIdx.x * R + r) * kRows + tid;
-      if (i >= set.M) continue;
-      int j = gch[r] + (int)(g1[r] & 0xffu);
-      const float k1 = __uint_as_float(g1[r]), k2 = __uint_as_float(g2[r]);
-      bool cert = false;
-      float thr = INFINITY;
-      if (ok && j < cw.K) {
-        float cv[kD], n, na, l1;
-        load_vec(cw.C + (int64_t)j * kD, cv);
-        codeword_terms(cv, sH, n, na, l1);
-        // |key - D| <= 2^-15 D; D_k <= s_k + off (every k); s_j + off <= D_j + e2 (winner).
-        const float e2 = 2.f * uc * (na + 2.f * pmax_r[r] * l1 + off_r[r]);
-        const float top = k1 * (1.f + 2.5f * kPack) + e2;   // >= s_j + off
-        cert = cw.K == 1 || (k2 * (1.f - kPack) > top);
-        thr = top - off_r[r];
-        thr += 4.f * kU * (k1 + off_r[r] + e2);
+  // Certificate, code, flag and statistics of this thread's row.
+  if (i < set.M) {
+    int j = gch + (int)(g1 & 0xffu);
+    const float k1 = __uint_as_float(g1), k2 = __uint_as_float(g2);
+    bool cert = false;
+    float thr = INFINITY;
+    if (ok && j < cw.K) {
+      float cv[kD], n, na, l1;
+      load_vec(cw.C + (int64_t)j * kD, cv);
+      codeword_terms(cv, sH, n, na, l1);
+      // |key - D| <= 2^-15 D; D_k <= s_k + off (every k); s_j + off <= D_j + e2 (winner).
+      const float e2 = 2.f * uc * (na + 2.f * pmax * l1 + off);
+      const float top = k1 * (1.f + 2.5f * kPack) + e2;   // >= s_j + off
+      cert = cw.K == 1 || (k2 * (1.f - kPack) > top);
+      thr = top - off;
+      thr += 4.f * kU * (k1 + off + e2);
+    } else {
+      j = 0;
+    }
+    if (!cert) {
+      const unsigned slot = atomicAdd(flags.count, 1u);
+      if (slot < flags.cap) {
+        flags.vec[slot] = i * G_range + (g - g_begin);
+        flags.thr[slot] = thr;
       } else {
-        j = 0;
+        raise_error(err, ERRBIT_INDEX);
       }
-      if (!cert) {
-        const unsigned slot = atomicAdd(flags.count, 1u);
-        if (slot < flags.cap) {
-          flags.vec[slot] = i * G_range + (g - g_begin);
-          flags.thr[slot] = thr;
-        } else {
-          raise_error(err, ERRBIT_INDEX);
-        }
-      }
-      out_code[i * out_ld + (g - out_g0)] = j;
-      if (cert && st.cnt) stats_add(st, *st.scale, g, j, q_r[r]);
+    }
+    out_code[i * out_ld + (g - out_g0)] = j;
+    if (cert && st.cnt) {
+      float q[kD];
+#pragma unroll
+      for (int p = 0; p < kD; ++p) q[p] = sq[p][tid];
+      stats_add(st, *st.scale, g, j, q);
     }
   }
   tc::tc_fence_before();
   __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, 2 * kCols);
+  if (warp == 0) tc::tmem_dealloc(tmem, kCols);
 }
 
 // cbmax[0] = max_k ||c_k||_1, cbmax[1] = max_k,j |c_kj| (one CTA; maxima are order-free).
@@ -1103,22 +1064,15 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     cbmax_kernel<<<1, 256, 0, stream>>>(cw.C, cw.K, cbmax);
     CRVQ_LAUNCHED();
     {
-      // R row tiles of 128 vectors per CTA share each staged codebook chunk; one CTA per SM
-      // (its two accumulator buffers take the SM's 512 tensor-memory columns).
+      // two row tiles of 128 vectors per CTA; two CTAs per SM (256 tensor-memory columns
+      // each); the dynamic shared memory request keeps a third CTA off the SM
       const int64_t row_tiles = ceil_div(set.M, tcenc::kRows);
-      const int R = (ceil_div(row_tiles, 4) * G_range >= 2 * nsm) ? 4 : 1;
-      const size_t smem = 2 * (size_t)tcenc::kBTile + (size_t)R * tcenc::kATile + 1024;
-      dim3 grid((unsigned)ceil_div(row_tiles, R), (unsigned)G_range);
+      const size_t smem = 100 * 1024;
+      dim3 grid((unsigned)ceil_div(row_tiles, kTcRowTiles), (unsigned)G_range);
       ProfScope ps("encode_argmin", stream, (double)nvec * cw.K);
-      if (R == 4) {
-        CRVQ_TRY(set_smem_attr(argmin_tc_kernel<4>, smem));
-        argmin_tc_kernel<4><<<grid, 256, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                         out_ld, out_g0, fl, st, cbmax, err);
-      } else {
-        CRVQ_TRY(set_smem_attr(argmin_tc_kernel<1>, smem));
-        argmin_tc_kernel<1><<<grid, 256, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                         out_ld, out_g0, fl, st, cbmax, err);
-      }
+      CRVQ_TRY(set_smem_attr(argmin_tc_kernel, smem));
+      argmin_tc_kernel<<<grid, 256, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
+                                                    out_ld, out_g0, fl, st, cbmax, err);
       CRVQ_LAUNCHED();
     }
     {
