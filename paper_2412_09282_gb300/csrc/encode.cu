@@ -202,7 +202,7 @@ constexpr int kK = 32;            // tf32 columns per row
 constexpr int kATile = kRows * kK * 4;   // 16 KB
 constexpr int kBTile = kCols * kK * 4;   // 32 KB
 constexpr float kCmul = 256.f;           // bound multiplier (about twice the analysis)
-constexpr float kPack = 3.0517578e-05f;  // 2^-15: relative truncation of the packed key
+constexpr float kPack = 3.8146973e-06f;  // 2^-18: relative truncation of the packed key
 constexpr uint32_t kIdesc = tc::idesc_tf32(kRows, kCols);
 
 __device__ __forceinline__ uint32_t koff(int r, int k) {
@@ -231,45 +231,103 @@ __device__ __forceinline__ void merge2(uint32_t& x1, uint32_t& x2, uint32_t y1, 
   x2 = min(hi, min(x2, y2));
 }
 
-// Two 256-thread CTAs per SM, each holding two row tiles of 128 vectors (thread t owns row
-// t % 128 of tile t / 128) and one 256-column accumulator. Warps w and w + 4 read the same 32
-// tensor-memory lanes and split the 256 codeword columns; the owner half of the tile merges
-// the two halves. While one CTA runs its FMA-heavy prologue or certificate, the other's
-// ALU-heavy epilogue and the tensor core keep the SM busy.
-constexpr int kTcRowTiles = 2;
+// Row of the B operand for codeword kk of C (K codewords): [c_hi | c_lo | c_hi | n'_hi n'_lo |
+// L1_hi L1_lo L1_hi | 1 1 | 0]; padding rows (kk >= K) score +1e30.
+__device__ __forceinline__ void build_b_row(const float* __restrict__ C, int K, int kk,
+                                            const float* H, float uc, uint32_t row[tcenc::kK]) {
+  using namespace tcenc;
+  if (kk < K) {
+    float cv[kD], n, na, l1;
+    load_vec(C + (int64_t)kk * kD, cv);
+    codeword_terms(cv, H, n, na, l1);
+#pragma unroll
+    for (int p = 0; p < kD; ++p) {
+      uint32_t hh, ll;
+      split(cv[p], hh, ll);
+      row[p] = hh;
+      row[8 + p] = ll;
+      row[16 + p] = hh;
+    }
+    split(n - uc * na, row[24], row[25]);
+    split(l1, row[26], row[27]);
+    row[28] = row[26];
+  } else {
+#pragma unroll
+    for (int p = 0; p < 24; ++p) row[p] = 0u;
+    row[24] = __float_as_uint(1e30f);
+    row[25] = 0u;
+    row[26] = row[27] = row[28] = 0u;
+  }
+  row[29] = row[30] = __float_as_uint(1.f);
+  row[31] = 0u;
+}
 
-__global__ void __launch_bounds__(256, 2)
+constexpr int kTcCols = 128;                     // codewords per chunk (MMA N)
+constexpr int kTcBTile = kTcCols * tcenc::kK * 4;  // 16 KB
+
+// B operand images of the codebook for groups [g_begin, g_begin + G_range): block
+// (g, chunk) holds 128 rows in the canonical shared-memory layout, ready for a bulk copy.
+__global__ void __launch_bounds__(128)
+prep_b_kernel(SetView set, int64_t g_begin, int64_t G_range, const float* __restrict__ C,
+              int K, int nchunk, float uc, char* __restrict__ out) {
+  const int64_t total = G_range * nchunk * (int64_t)kTcCols;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int row = (int)(e % kTcCols);
+    const int64_t blk = e / kTcCols;  // g_rel * nchunk + chunk
+    const int chunk = (int)(blk % nchunk);
+    const int64_t g = g_begin + blk / nchunk;
+    uint32_t v[tcenc::kK];
+    build_b_row(C, K, chunk * kTcCols + row, set.Hb + g * kD * kD, uc, v);
+    tcenc::put_row(out + blk * kTcBTile, row, v);
+  }
+}
+
+// One 128-thread CTA per row tile (thread = row = tensor-memory lane), four CTAs per SM, each
+// with a 128-column accumulator. Codeword chunks of 128 stream through two shared-memory
+// buffers: bulk copies of precomputed B images when given (bpre), built in place otherwise.
+// Keys carry the column within a 32-column block in their low 5 bits (2^-18 relative
+// truncation); the block is tracked by the merge.
+__global__ void __launch_bounds__(128, 4)
 argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
                  int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
                  FlagList flags, StatsView st, const float* __restrict__ cbmax,
-                 unsigned* err) {
+                 const char* __restrict__ bpre, unsigned* err) {
   using namespace tcenc;
-  constexpr int R = kTcRowTiles;
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                        ~(uintptr_t)1023);
-  char* Btile = smem;                  // 32 KB
-  char* Atiles = smem + kBTile;        // R x 16 KB
+  char* Atile = smem;                  // 16 KB
+  char* Bbuf = smem + kATile;          // 2 x 16 KB
   __shared__ float sH[kD * kD];
-  __shared__ __align__(8) uint64_t bar;
+  __shared__ __align__(8) uint64_t bar_mma, bar_b[2];
   __shared__ uint32_t tmem_slot;
-  __shared__ uint32_t part1[128], part2[128];
-  __shared__ float sq[8][256];  // each row's H r (least-squares statistics), column-major
+  __shared__ float sq[kD][128];        // each row's H r (least-squares statistics)
 
   const int64_t g = g_begin + blockIdx.y;
   const int64_t G_range = gridDim.y;
   const int tid = threadIdx.x, warp = tid >> 5;
-  const int my_tile = tid >> 7, my_row = tid & 127;
-  const int64_t i = ((int64_t)blockIdx.x * R + my_tile) * kRows + my_row;
+  const int64_t i = (int64_t)blockIdx.x * kRows + tid;
   const CbView cw = cbs.cb[s_idx];
   const float cmul = kCmul + 4.f * n_fixed;
   const float uc = kU * cmul;
+  const int nchunk = (cw.K + kTcCols - 1) / kTcCols;
+  const char* bimg = bpre ? bpre + (size_t)(g - g_begin) * nchunk * kTcBTile : nullptr;
 
   if (tid < kD * kD) sH[tid] = set.Hb[g * kD * kD + tid];
-  if (warp == 0) tc::tmem_alloc(&tmem_slot, kCols);
+  if (warp == 0) tc::tmem_alloc(&tmem_slot, kTcCols);
   if (tid == 0) {
-    tc::mbar_init(tc::smem_u32(&bar), 1);
+    tc::mbar_init(tc::smem_u32(&bar_mma), 1);
+    tc::mbar_init(tc::smem_u32(&bar_b[0]), 1);
+    tc::mbar_init(tc::smem_u32(&bar_b[1]), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    if (bimg) {
+      for (int c = 0; c < 2 && c < nchunk; ++c) {
+        tc::mbar_expect_tx(tc::smem_u32(&bar_b[c]), kTcBTile);
+        tc::bulk_copy_g2s(tc::smem_u32(Bbuf + c * kTcBTile), bimg + (size_t)c * kTcBTile,
+                          kTcBTile, tc::smem_u32(&bar_b[c]));
+      }
+    }
   }
   tc::tc_fence_before();
   __syncthreads();
@@ -287,7 +345,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   }
   const float l1max = cbmax[0], cinf = cbmax[1];
 
-  // Prologue: this thread's A row and row state.
+  // Prologue: this thread's A row.
   float pmax, off;
   {
     float rv[kD], a[kD], m2q[kD];
@@ -328,118 +386,103 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
     row[27] = row[26];
     split(off * (1.f - uc), row[29], row[30]);
     row[31] = 0u;
-    put_row(Atiles + my_tile * kATile, my_row, row);
+    put_row(Atile, tid, row);
   }
-  uint32_t g1 = 0xffffffffu, g2 = 0xffffffffu;
-  int gch = 0;
+  tc::fence_async_smem();
+  __syncthreads();
 
-  uint32_t phase = 0;
+  uint32_t g1 = 0xffffffffu, g2 = 0xffffffffu;
+  int gidx = 0;
   bool ok = true;
-  const int lq = warp & 3, half = warp >> 2;
-  for (int kc = 0; kc < cw.K && ok; kc += kCols) {
-    // B tile: codewords kc .. kc + 255 (one per thread; padding rows score +1e30).
-    {
-      const int kk = kc + tid;
-      uint32_t row[kK];
-      if (kk < cw.K) {
-        float cv[kD], n, na, l1;
-        load_vec(cw.C + (int64_t)kk * kD, cv);
-        codeword_terms(cv, sH, n, na, l1);
-#pragma unroll
-        for (int p = 0; p < kD; ++p) {
-          uint32_t hh, ll;
-          split(cv[p], hh, ll);
-          row[p] = hh;
-          row[8 + p] = ll;
-          row[16 + p] = hh;
-        }
-        split(n - uc * na, row[24], row[25]);
-        split(l1, row[26], row[27]);
-        row[28] = row[26];
-      } else {
-#pragma unroll
-        for (int p = 0; p < 24; ++p) row[p] = 0u;
-        row[24] = __float_as_uint(1e30f);
-        row[25] = 0u;
-        row[26] = row[27] = row[28] = 0u;
-      }
-      row[29] = row[30] = __float_as_uint(1.f);
-      row[31] = 0u;
-      put_row(Btile, tid, row);
-    }
-    tc::fence_async_smem();
-    __syncthreads();
-#pragma unroll 1
-    for (int r = 0; r < R; ++r) {
-      if (tid == 0) {
-        tc::tc_fence_after();
-        const uint32_t a0 = tc::smem_u32(Atiles + r * kATile), b0 = tc::smem_u32(Btile);
-#pragma unroll
-        for (int ks = 0; ks < kK / 8; ++ks)
-          tc::mma_tf32(tmem, tc::smem_desc(a0 + ks * 256, 128, (kK / 4) * 128),
-                       tc::smem_desc(b0 + ks * 256, 128, (kK / 4) * 128), kIdesc,
-                       ks > 0 ? 1u : 0u);
-        tc::mma_commit(tc::smem_u32(&bar));
-      }
-      ok = tc::mbar_wait(tc::smem_u32(&bar), phase, err);
-      phase ^= 1u;
-      ok = __syncthreads_and(ok);
-      if (!ok) break;
-      tc::tc_fence_after();
-      // 128 columns of this warp's 32 rows, two 64-column rounds, four top-2 chains.
-      uint32_t a1[4], a2[4];
-#pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        a1[b] = 0xffffffffu;
-        a2[b] = 0xffffffffu;
-      }
-      const uint32_t base = tmem + ((uint32_t)(lq * 32) << 16) + (uint32_t)(half * 128);
-#pragma unroll
-      for (int rnd = 0; rnd < 2; ++rnd) {
-        uint32_t v0[32], v1[32];
-        tc::tmem_ld32_nowait(base + 64 * rnd, v0);
-        tc::tmem_ld32_nowait(base + 64 * rnd + 32, v1);
-        tc::tmem_wait_ld();
-#pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const uint32_t k0 = (v0[j] & 0xffffff00u) | (uint32_t)j;
-          const uint32_t k1 = (v1[j] & 0xffffff00u) | (uint32_t)j;
-          const uint32_t h0 = max(a1[2 * rnd], k0), h1 = max(a1[2 * rnd + 1], k1);
-          a1[2 * rnd] = min(a1[2 * rnd], k0);
-          a1[2 * rnd + 1] = min(a1[2 * rnd + 1], k1);
-          a2[2 * rnd] = min(a2[2 * rnd], h0);
-          a2[2 * rnd + 1] = min(a2[2 * rnd + 1], h1);
-        }
-      }
-      // the keys' low 8 bits become the chunk column: half * 128 + 32 * block + j
-      uint32_t t1 = a1[0] | (uint32_t)(half * 128), t2 = a2[0] | (uint32_t)(half * 128);
-#pragma unroll
-      for (int b = 1; b < 4; ++b)
-        merge2(t1, t2, a1[b] | (uint32_t)(half * 128 + 32 * b),
-               a2[b] | (uint32_t)(half * 128 + 32 * b));
-      if (half != r) {
-        part1[lq * 32 + (tid & 31)] = t1;
-        part2[lq * 32 + (tid & 31)] = t2;
-      }
-      tc::tc_fence_before();
+  constexpr uint32_t idesc = tc::idesc_tf32(kRows, kTcCols);
+  // bulk copies issued / waited per buffer (the same count in every thread)
+  int b_issued[2] = {bimg ? 1 : 0, (bimg && nchunk > 1) ? 1 : 0}, b_waited[2] = {0, 0};
+  for (int c = 0; c < nchunk; ++c) {
+    const int buf = c & 1;
+    char* Bt = Bbuf + buf * kTcBTile;
+    if (bimg) {
+      if (ok) ok = tc::mbar_wait(tc::smem_u32(&bar_b[buf]), (uint32_t)((c >> 1) & 1), err);
+      ++b_waited[buf];
+    } else {
+      uint32_t v[kK];
+      build_b_row(cw.C, cw.K, c * kTcCols + tid, sH, uc, v);
+      put_row(Bt, tid, v);
+      tc::fence_async_smem();
       __syncthreads();
-      if (half == r) {  // owner half of tile r: its threads hold the rows' state
-        merge2(t1, t2, part1[lq * 32 + (tid & 31)], part2[lq * 32 + (tid & 31)]);
-        if (t1 < g1) {
-          g2 = min(g1, t2);
-          g1 = t1;
-          gch = kc;
-        } else {
-          g2 = min(g2, t1);
-        }
-      }
-      __syncthreads();  // part1/part2 and the accumulator are free for the next tile
     }
+    ok = __syncthreads_and(ok);
+    if (!ok) break;
+    if (tid == 0) {
+      tc::tc_fence_after();
+      const uint32_t a0 = tc::smem_u32(Atile), b0 = tc::smem_u32(Bt);
+#pragma unroll
+      for (int ks = 0; ks < kK / 8; ++ks)
+        tc::mma_tf32(tmem, tc::smem_desc(a0 + ks * 256, 128, (kK / 4) * 128),
+                     tc::smem_desc(b0 + ks * 256, 128, (kK / 4) * 128), idesc,
+                     ks > 0 ? 1u : 0u);
+      tc::mma_commit(tc::smem_u32(&bar_mma));
+    }
+    ok = tc::mbar_wait(tc::smem_u32(&bar_mma), (uint32_t)(c & 1), err);
+    ok = __syncthreads_and(ok);
+    if (!ok) break;
+    if (bimg && c + 2 < nchunk) {  // this buffer is free again: fetch chunk c + 2
+      if (tid == 0) {
+        tc::mbar_expect_tx(tc::smem_u32(&bar_b[buf]), kTcBTile);
+        tc::bulk_copy_g2s(tc::smem_u32(Bt), bimg + (size_t)(c + 2) * kTcBTile, kTcBTile,
+                          tc::smem_u32(&bar_b[buf]));
+      }
+      ++b_issued[buf];
+    }
+    tc::tc_fence_after();
+    // Epilogue: this warp's 32 rows x 128 columns, four 32-column blocks, one top-2 chain each.
+    uint32_t a1[4], a2[4];
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      a1[b] = 0xffffffffu;
+      a2[b] = 0xffffffffu;
+    }
+    const uint32_t base = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll
+    for (int rnd = 0; rnd < 2; ++rnd) {
+      uint32_t v0[32], v1[32];
+      tc::tmem_ld32_nowait(base + 64 * rnd, v0);
+      tc::tmem_ld32_nowait(base + 64 * rnd + 32, v1);
+      tc::tmem_wait_ld();
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const uint32_t k0 = (v0[j] & 0xffffffe0u) | (uint32_t)j;
+        const uint32_t k1 = (v1[j] & 0xffffffe0u) | (uint32_t)j;
+        const uint32_t h0 = max(a1[2 * rnd], k0), h1 = max(a1[2 * rnd + 1], k1);
+        a1[2 * rnd] = min(a1[2 * rnd], k0);
+        a1[2 * rnd + 1] = min(a1[2 * rnd + 1], k1);
+        a2[2 * rnd] = min(a2[2 * rnd], h0);
+        a2[2 * rnd + 1] = min(a2[2 * rnd + 1], h1);
+      }
+    }
+#pragma unroll
+    for (int b = 0; b < 4; ++b) {
+      if (a1[b] < g1) {
+        g2 = min(g1, a2[b]);
+        g1 = a1[b];
+        gidx = c * kTcCols + 32 * b + (int)(a1[b] & 31u);
+      } else {
+        g2 = min(g2, a1[b]);
+      }
+    }
+    tc::tc_fence_before();
+    __syncthreads();  // the accumulator is free for the next chunk
   }
+
+  // After a timeout: let copies still in flight into this CTA's shared memory land (bounded).
+  for (int b = 0; b < 2; ++b)
+    while (b_waited[b] < b_issued[b]) {
+      tc::mbar_wait(tc::smem_u32(&bar_b[b]), (uint32_t)(b_waited[b] & 1), err);
+      ++b_waited[b];
+    }
 
   // Certificate, code, flag and statistics of this thread's row.
   if (i < set.M) {
-    int j = gch + (int)(g1 & 0xffu);
+    int j = gidx;
     const float k1 = __uint_as_float(g1), k2 = __uint_as_float(g2);
     bool cert = false;
     float thr = INFINITY;
@@ -447,7 +490,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       float cv[kD], n, na, l1;
       load_vec(cw.C + (int64_t)j * kD, cv);
       codeword_terms(cv, sH, n, na, l1);
-      // |key - D| <= 2^-15 D; D_k <= s_k + off (every k); s_j + off <= D_j + e2 (winner).
+      // |key - D| <= 2^-18 D; D_k <= s_k + off (every k); s_j + off <= D_j + e2 (winner).
       const float e2 = 2.f * uc * (na + 2.f * pmax * l1 + off);
       const float top = k1 * (1.f + 2.5f * kPack) + e2;   // >= s_j + off
       cert = cw.K == 1 || (k2 * (1.f - kPack) > top);
@@ -475,7 +518,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   }
   tc::tc_fence_before();
   __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, kCols);
+  if (warp == 0) tc::tmem_dealloc(tmem, kTcCols);
 }
 
 // cbmax[0] = max_k ||c_k||_1, cbmax[1] = max_k,j |c_kj| (one CTA; maxima are order-free).
@@ -1064,15 +1107,29 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     cbmax_kernel<<<1, 256, 0, stream>>>(cw.C, cw.K, cbmax);
     CRVQ_LAUNCHED();
     {
-      // two row tiles of 128 vectors per CTA; two CTAs per SM (256 tensor-memory columns
-      // each); the dynamic shared memory request keeps a third CTA off the SM
-      const int64_t row_tiles = ceil_div(set.M, tcenc::kRows);
-      const size_t smem = 100 * 1024;
-      dim3 grid((unsigned)ceil_div(row_tiles, kTcRowTiles), (unsigned)G_range);
+      // one row tile of 128 vectors per CTA, four CTAs per SM (128 tensor-memory columns
+      // each); the codebook's B images are precomputed per group when they fit in 256 MB
+      const int nchunk = (int)ceil_div(cw.K, kTcCols);
+      const size_t bbytes = (size_t)G_range * nchunk * kTcBTile;
+      Scratch bmem;
+      const char* bpre = nullptr;
+      const float uc = kU * (tcenc::kCmul + 4.f * n_fixed);
+      if (bbytes <= (size_t(256) << 20)) {
+        CRVQ_TRY(bmem.alloc(bbytes, stream));
+        ProfScope pb("encode_prep_b", stream, (double)G_range * nchunk * kTcCols);
+        const int64_t rows = (int64_t)G_range * nchunk * kTcCols;
+        prep_b_kernel<<<(unsigned)std::min<int64_t>(ceil_div(rows, 128), 16 * nsm), 128, 0,
+                        stream>>>(set, g_begin, G_range, cw.C, cw.K, nchunk, uc,
+                                  bmem.as<char>());
+        CRVQ_LAUNCHED();
+        bpre = bmem.as<char>();
+      }
+      const size_t smem = (size_t)tcenc::kATile + 2 * (size_t)kTcBTile + 1024;
+      dim3 grid((unsigned)ceil_div(set.M, tcenc::kRows), (unsigned)G_range);
       ProfScope ps("encode_argmin", stream, (double)nvec * cw.K);
       CRVQ_TRY(set_smem_attr(argmin_tc_kernel, smem));
-      argmin_tc_kernel<<<grid, 256, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                    out_ld, out_g0, fl, st, cbmax, err);
+      argmin_tc_kernel<<<grid, 128, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
+                                                    out_ld, out_g0, fl, st, cbmax, bpre, err);
       CRVQ_LAUNCHED();
     }
     {
