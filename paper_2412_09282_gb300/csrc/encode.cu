@@ -283,56 +283,59 @@ prep_b_kernel(SetView set, int64_t g_begin, int64_t G_range, const float* __rest
   }
 }
 
-// One 128-thread CTA per row tile (thread = row = tensor-memory lane), four CTAs per SM, each
-// with a 128-column accumulator. Codeword chunks of 128 stream through two shared-memory
-// buffers: bulk copies of precomputed B images when given (bpre), built in place otherwise.
-// Keys carry the column within a 32-column block in their low 5 bits (2^-18 relative
-// truncation); the block is tracked by the merge.
-__global__ void __launch_bounds__(128, 4)
+// A 128-thread CTA walks `tiles` consecutive row tiles of one group (thread = row = tensor-
+// memory lane), with a 128-column accumulator; three CTAs per SM. Codeword chunks of 128 come
+// from precomputed B images by bulk copy (bpre) or are built in place; with at most two chunks
+// they stay resident for all the CTA's tiles. Keys carry the column within a 32-column block in
+// their low 5 bits (2^-18 relative truncation); the block is tracked by the merge. The Lloyd
+// statistics of certified rows are summed in shared memory (integer atomics) and flushed once.
+constexpr int kTcSmemStatsK = 256;  // codebooks up to this size aggregate statistics in smem
+
+__global__ void __launch_bounds__(128, 3)
 argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
                  int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
                  FlagList flags, StatsView st, const float* __restrict__ cbmax,
-                 const char* __restrict__ bpre, unsigned* err) {
+                 const char* __restrict__ bpre, int tiles, unsigned* err) {
   using namespace tcenc;
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                        ~(uintptr_t)1023);
   char* Atile = smem;                  // 16 KB
   char* Bbuf = smem + kATile;          // 2 x 16 KB
+  long long* s_bacc = reinterpret_cast<long long*>(Bbuf + 2 * kTcBTile);  // [256][8]
+  int* s_cnt = reinterpret_cast<int*>(s_bacc + kTcSmemStatsK * kD);       // [256]
   __shared__ float sH[kD * kD];
   __shared__ __align__(8) uint64_t bar_mma, bar_b[2];
   __shared__ uint32_t tmem_slot;
-  __shared__ float sq[kD][128];        // each row's H r (least-squares statistics)
 
   const int64_t g = g_begin + blockIdx.y;
   const int64_t G_range = gridDim.y;
   const int tid = threadIdx.x, warp = tid >> 5;
-  const int64_t i = (int64_t)blockIdx.x * kRows + tid;
   const CbView cw = cbs.cb[s_idx];
   const float cmul = kCmul + 4.f * n_fixed;
   const float uc = kU * cmul;
   const int nchunk = (cw.K + kTcCols - 1) / kTcCols;
+  const bool resident = nchunk <= 2;
   const char* bimg = bpre ? bpre + (size_t)(g - g_begin) * nchunk * kTcBTile : nullptr;
+  const bool smem_stats = st.cnt && cw.K <= kTcSmemStatsK;
 
   if (tid < kD * kD) sH[tid] = set.Hb[g * kD * kD + tid];
+  if (smem_stats) {
+    for (int e = tid; e < kTcSmemStatsK * kD; e += blockDim.x) s_bacc[e] = 0;
+    for (int e = tid; e < kTcSmemStatsK; e += blockDim.x) s_cnt[e] = 0;
+  }
   if (warp == 0) tc::tmem_alloc(&tmem_slot, kTcCols);
   if (tid == 0) {
     tc::mbar_init(tc::smem_u32(&bar_mma), 1);
     tc::mbar_init(tc::smem_u32(&bar_b[0]), 1);
     tc::mbar_init(tc::smem_u32(&bar_b[1]), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    if (bimg) {
-      for (int c = 0; c < 2 && c < nchunk; ++c) {
-        tc::mbar_expect_tx(tc::smem_u32(&bar_b[c]), kTcBTile);
-        tc::bulk_copy_g2s(tc::smem_u32(Bbuf + c * kTcBTile), bimg + (size_t)c * kTcBTile,
-                          kTcBTile, tc::smem_u32(&bar_b[c]));
-      }
-    }
   }
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
   const uint32_t tmem = tmem_slot;
+  const double scale = st.cnt ? *st.scale : 0.0;
 
   // Bound on Na_k over the codebook for this group: (max row sum |H_g|) L1max cinfmax.
   float hrow = 0.f;
@@ -344,176 +347,225 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
     hrow = fmaxf(hrow, rs);
   }
   const float l1max = cbmax[0], cinf = cbmax[1];
-
-  // Prologue: this thread's A row.
-  float pmax, off;
-  {
-    float rv[kD], a[kD], m2q[kD];
-    if (i < set.M) {
-      target32(set, cbs, n_fixed, i, g, rv, a, err);
-    } else {
-#pragma unroll
-      for (int j = 0; j < kD; ++j) rv[j] = a[j] = 0.f;
-    }
-    vector_terms(rv, a, sH, m2q, pmax);
-    float rr = 0.f, ra = 0.f;
-#pragma unroll
-    for (int p = 0; p < kD; ++p) {
-      rr = fmaf(rv[p], -0.5f * m2q[p], rr);
-      float pa = 0.f;
-#pragma unroll
-      for (int j = 0; j < kD; ++j) pa = fmaf(fabsf(sH[p * kD + j]), a[j], pa);
-      ra = fmaf(a[p], pa, ra);
-    }
-    // offset making every D = low + off >= 0, with margins for every rounding involved
-    off = (rr + 32.f * kU * ra + 2.f * uc * (hrow * l1max * cinf + 2.f * pmax * l1max)) *
-              (1.f + 4.f * uc) + 1e-30f;
-    const float beta = -2.f * uc * pmax;
-    uint32_t row[kK];
-#pragma unroll
-    for (int p = 0; p < kD; ++p) {
-      uint32_t h, l;
-      split(m2q[p], h, l);
-      row[p] = h;
-      row[8 + p] = h;
-      row[16 + p] = l;
-      sq[p][tid] = -0.5f * m2q[p];
-    }
-    const uint32_t one = __float_as_uint(1.f);
-    row[24] = one;
-    row[25] = one;
-    split(beta, row[26], row[28]);
-    row[27] = row[26];
-    split(off * (1.f - uc), row[29], row[30]);
-    row[31] = 0u;
-    put_row(Atile, tid, row);
-  }
-  tc::fence_async_smem();
-  __syncthreads();
-
-  uint32_t g1 = 0xffffffffu, g2 = 0xffffffffu;
-  int gidx = 0;
-  bool ok = true;
   constexpr uint32_t idesc = tc::idesc_tf32(kRows, kTcCols);
-  // bulk copies issued / waited per buffer (the same count in every thread)
-  int b_issued[2] = {bimg ? 1 : 0, (bimg && nchunk > 1) ? 1 : 0}, b_waited[2] = {0, 0};
-  for (int c = 0; c < nchunk; ++c) {
-    const int buf = c & 1;
-    char* Bt = Bbuf + buf * kTcBTile;
-    if (bimg) {
-      if (ok) ok = tc::mbar_wait(tc::smem_u32(&bar_b[buf]), (uint32_t)((c >> 1) & 1), err);
-      ++b_waited[buf];
-    } else {
-      uint32_t v[kK];
-      build_b_row(cw.C, cw.K, c * kTcCols + tid, sH, uc, v);
-      put_row(Bt, tid, v);
-      tc::fence_async_smem();
-      __syncthreads();
-    }
-    ok = __syncthreads_and(ok);
-    if (!ok) break;
-    if (tid == 0) {
-      tc::tc_fence_after();
-      const uint32_t a0 = tc::smem_u32(Atile), b0 = tc::smem_u32(Bt);
-#pragma unroll
-      for (int ks = 0; ks < kK / 8; ++ks)
-        tc::mma_tf32(tmem, tc::smem_desc(a0 + ks * 256, 128, (kK / 4) * 128),
-                     tc::smem_desc(b0 + ks * 256, 128, (kK / 4) * 128), idesc,
-                     ks > 0 ? 1u : 0u);
-      tc::mma_commit(tc::smem_u32(&bar_mma));
-    }
-    ok = tc::mbar_wait(tc::smem_u32(&bar_mma), (uint32_t)(c & 1), err);
-    ok = __syncthreads_and(ok);
-    if (!ok) break;
-    if (bimg && c + 2 < nchunk) {  // this buffer is free again: fetch chunk c + 2
-      if (tid == 0) {
-        tc::mbar_expect_tx(tc::smem_u32(&bar_b[buf]), kTcBTile);
-        tc::bulk_copy_g2s(tc::smem_u32(Bt), bimg + (size_t)(c + 2) * kTcBTile, kTcBTile,
-                          tc::smem_u32(&bar_b[buf]));
-      }
-      ++b_issued[buf];
-    }
-    tc::tc_fence_after();
-    // Epilogue: this warp's 32 rows x 128 columns, four 32-column blocks, one top-2 chain each.
-    uint32_t a1[4], a2[4];
-#pragma unroll
-    for (int b = 0; b < 4; ++b) {
-      a1[b] = 0xffffffffu;
-      a2[b] = 0xffffffffu;
-    }
-    const uint32_t base = tmem + ((uint32_t)(warp * 32) << 16);
-#pragma unroll
-    for (int rnd = 0; rnd < 2; ++rnd) {
-      uint32_t v0[32], v1[32];
-      tc::tmem_ld32_nowait(base + 64 * rnd, v0);
-      tc::tmem_ld32_nowait(base + 64 * rnd + 32, v1);
-      tc::tmem_wait_ld();
-#pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        const uint32_t k0 = (v0[j] & 0xffffffe0u) | (uint32_t)j;
-        const uint32_t k1 = (v1[j] & 0xffffffe0u) | (uint32_t)j;
-        const uint32_t h0 = max(a1[2 * rnd], k0), h1 = max(a1[2 * rnd + 1], k1);
-        a1[2 * rnd] = min(a1[2 * rnd], k0);
-        a1[2 * rnd + 1] = min(a1[2 * rnd + 1], k1);
-        a2[2 * rnd] = min(a2[2 * rnd], h0);
-        a2[2 * rnd + 1] = min(a2[2 * rnd + 1], h1);
-      }
-    }
-#pragma unroll
-    for (int b = 0; b < 4; ++b) {
-      if (a1[b] < g1) {
-        g2 = min(g1, a2[b]);
-        g1 = a1[b];
-        gidx = c * kTcCols + 32 * b + (int)(a1[b] & 31u);
-      } else {
-        g2 = min(g2, a1[b]);
-      }
-    }
-    tc::tc_fence_before();
-    __syncthreads();  // the accumulator is free for the next chunk
-  }
 
+  // this CTA's row tiles (the last CTA of a column may have fewer)
+  const int64_t row_tiles = (set.M + kRows - 1) / kRows;
+  const int my_tiles = (int)min((int64_t)tiles, row_tiles - (int64_t)blockIdx.x * tiles);
+  // Chunk uses are numbered u = t * nchunk + c. Resident chunks sit in buffer c; otherwise use u
+  // reads buffer u & 1, and the copy for use u + 2 starts when use u is done. Bulk copies
+  // issued / waited per buffer (the same count in every thread).
+  const int n_uses = resident ? nchunk : my_tiles * nchunk;
+  int b_issued[2] = {0, 0}, b_waited[2] = {0, 0};
+  auto fetch = [&](int u) {  // chunk u % nchunk into buffer u & 1 (bimg only)
+    const int b = u & 1;
+    if (tid == 0) {
+      tc::mbar_expect_tx(tc::smem_u32(&bar_b[b]), kTcBTile);
+      tc::bulk_copy_g2s(tc::smem_u32(Bbuf + b * kTcBTile),
+                        bimg + (size_t)(u % nchunk) * kTcBTile, kTcBTile,
+                        tc::smem_u32(&bar_b[b]));
+    }
+    ++b_issued[b];
+  };
+  if (bimg) {
+    fetch(0);
+    if (n_uses > 1) fetch(1);
+  }
+  bool ok = true;
+  int mma_count = 0;
+
+  for (int t = 0; t < my_tiles && ok; ++t) {
+    const int64_t i = ((int64_t)blockIdx.x * tiles + t) * kRows + tid;
+    // Prologue: this thread's A row.
+    float pmax, off;
+    {
+      float rv[kD], a[kD], m2q[kD];
+      if (i < set.M) {
+        target32(set, cbs, n_fixed, i, g, rv, a, err);
+      } else {
+#pragma unroll
+        for (int j = 0; j < kD; ++j) rv[j] = a[j] = 0.f;
+      }
+      vector_terms(rv, a, sH, m2q, pmax);
+      float rr = 0.f, ra = 0.f;
+#pragma unroll
+      for (int p = 0; p < kD; ++p) {
+        rr = fmaf(rv[p], -0.5f * m2q[p], rr);
+        float pa = 0.f;
+#pragma unroll
+        for (int j = 0; j < kD; ++j) pa = fmaf(fabsf(sH[p * kD + j]), a[j], pa);
+        ra = fmaf(a[p], pa, ra);
+      }
+      // offset making every D = low + off >= 0, with margins for every rounding involved
+      off = (rr + 32.f * kU * ra + 2.f * uc * (hrow * l1max * cinf + 2.f * pmax * l1max)) *
+                (1.f + 4.f * uc) + 1e-30f;
+      const float beta = -2.f * uc * pmax;
+      uint32_t row[kK];
+#pragma unroll
+      for (int p = 0; p < kD; ++p) {
+        uint32_t h, l;
+        split(m2q[p], h, l);
+        row[p] = h;
+        row[8 + p] = h;
+        row[16 + p] = l;
+      }
+      const uint32_t one = __float_as_uint(1.f);
+      row[24] = one;
+      row[25] = one;
+      split(beta, row[26], row[28]);
+      row[27] = row[26];
+      split(off * (1.f - uc), row[29], row[30]);
+      row[31] = 0u;
+      put_row(Atile, tid, row);
+    }
+    tc::fence_async_smem();
+    __syncthreads();
+
+    uint32_t g1 = 0xffffffffu, g2 = 0xffffffffu;
+    int gidx = 0;
+    for (int c = 0; c < nchunk; ++c) {
+      const int u = t * nchunk + c;
+      const int buf = resident ? c : (u & 1);
+      char* Bt = Bbuf + buf * kTcBTile;
+      if (bimg) {
+        if (b_waited[buf] < b_issued[buf]) {
+          if (ok) ok = tc::mbar_wait(tc::smem_u32(&bar_b[buf]), (uint32_t)(b_waited[buf] & 1), err);
+          ++b_waited[buf];
+        }
+      } else if (!resident || t == 0) {
+        uint32_t v[kK];
+        build_b_row(cw.C, cw.K, c * kTcCols + tid, sH, uc, v);
+        put_row(Bt, tid, v);
+        tc::fence_async_smem();
+        __syncthreads();
+      }
+      ok = __syncthreads_and(ok);
+      if (!ok) break;
+      if (tid == 0) {
+        tc::tc_fence_after();
+        const uint32_t a0 = tc::smem_u32(Atile), b0 = tc::smem_u32(Bt);
+#pragma unroll
+        for (int ks = 0; ks < kK / 8; ++ks)
+          tc::mma_tf32(tmem, tc::smem_desc(a0 + ks * 256, 128, (kK / 4) * 128),
+                       tc::smem_desc(b0 + ks * 256, 128, (kK / 4) * 128), idesc,
+                       ks > 0 ? 1u : 0u);
+        tc::mma_commit(tc::smem_u32(&bar_mma));
+      }
+      ok = tc::mbar_wait(tc::smem_u32(&bar_mma), (uint32_t)(mma_count & 1), err);
+      ++mma_count;
+      ok = __syncthreads_and(ok);
+      if (!ok) break;
+      if (bimg && !resident && u + 2 < n_uses) fetch(u + 2);  // this buffer is free again
+      tc::tc_fence_after();
+      // Epilogue: this warp's 32 rows x 128 columns, four 32-column blocks, one top-2 chain
+      // each.
+      uint32_t a1[4], a2[4];
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        a1[b] = 0xffffffffu;
+        a2[b] = 0xffffffffu;
+      }
+      const uint32_t base = tmem + ((uint32_t)(warp * 32) << 16);
+#pragma unroll
+      for (int rnd = 0; rnd < 2; ++rnd) {
+        uint32_t v0[32], v1[32];
+        tc::tmem_ld32_nowait(base + 64 * rnd, v0);
+        tc::tmem_ld32_nowait(base + 64 * rnd + 32, v1);
+        tc::tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const uint32_t k0 = (v0[j] & 0xffffffe0u) | (uint32_t)j;
+          const uint32_t k1 = (v1[j] & 0xffffffe0u) | (uint32_t)j;
+          const uint32_t h0 = max(a1[2 * rnd], k0), h1 = max(a1[2 * rnd + 1], k1);
+          a1[2 * rnd] = min(a1[2 * rnd], k0);
+          a1[2 * rnd + 1] = min(a1[2 * rnd + 1], k1);
+          a2[2 * rnd] = min(a2[2 * rnd], h0);
+          a2[2 * rnd + 1] = min(a2[2 * rnd + 1], h1);
+        }
+      }
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        if (a1[b] < g1) {
+          g2 = min(g1, a2[b]);
+          g1 = a1[b];
+          gidx = c * kTcCols + 32 * b + (int)(a1[b] & 31u);
+        } else {
+          g2 = min(g2, a1[b]);
+        }
+      }
+      tc::tc_fence_before();
+      __syncthreads();  // the accumulator is free for the next MMA
+    }
+    if (!ok) break;
+
+    // Certificate, code, flag and statistics of this thread's row.
+    if (i < set.M) {
+      int j = gidx;
+      const float k1 = __uint_as_float(g1), k2 = __uint_as_float(g2);
+      bool cert = false;
+      float thr = INFINITY;
+      float cv[kD];
+      if (j < cw.K) {
+        float n, na, l1;
+        load_vec(cw.C + (int64_t)j * kD, cv);
+        codeword_terms(cv, sH, n, na, l1);
+        // |key - D| <= 2^-18 D; D_k <= s_k + off (every k); s_j + off <= D_j + e2 (winner).
+        const float e2 = 2.f * uc * (na + 2.f * pmax * l1 + off);
+        const float top = k1 * (1.f + 2.5f * kPack) + e2;   // >= s_j + off
+        cert = cw.K == 1 || (k2 * (1.f - kPack) > top);
+        thr = top - off;
+        thr += 4.f * kU * (k1 + off + e2);
+      } else {
+        j = 0;
+      }
+      if (!cert) {
+        const unsigned slot = atomicAdd(flags.count, 1u);
+        if (slot < flags.cap) {
+          flags.vec[slot] = i * G_range + (g - g_begin);
+          flags.thr[slot] = thr;
+        } else {
+          raise_error(err, ERRBIT_INDEX);
+        }
+      }
+      out_code[i * out_ld + (g - out_g0)] = j;
+      if (cert && st.cnt) {
+        // the fallback's target / H r (bit-identical to the standalone update's)
+        float rv[kD], a[kD], m2q[kD], pm;
+        target32(set, cbs, n_fixed, i, g, rv, a, err);
+        vector_terms(rv, a, sH, m2q, pm);
+        if (smem_stats) {
+          atomicAdd(&s_cnt[j], 1);
+#pragma unroll
+          for (int p = 0; p < kD; ++p) {
+            const long long v = __double2ll_rn((double)(-0.5f * m2q[p]) * scale);
+            atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[j * kD + p]),
+                      (unsigned long long)v);
+          }
+        } else {
+          float q[kD];
+#pragma unroll
+          for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[p];
+          stats_add(st, scale, g, j, q);
+        }
+      }
+    }
+  }
   // After a timeout: let copies still in flight into this CTA's shared memory land (bounded).
   for (int b = 0; b < 2; ++b)
     while (b_waited[b] < b_issued[b]) {
       tc::mbar_wait(tc::smem_u32(&bar_b[b]), (uint32_t)(b_waited[b] & 1), err);
       ++b_waited[b];
     }
-
-  // Certificate, code, flag and statistics of this thread's row.
-  if (i < set.M) {
-    int j = gidx;
-    const float k1 = __uint_as_float(g1), k2 = __uint_as_float(g2);
-    bool cert = false;
-    float thr = INFINITY;
-    if (ok && j < cw.K) {
-      float cv[kD], n, na, l1;
-      load_vec(cw.C + (int64_t)j * kD, cv);
-      codeword_terms(cv, sH, n, na, l1);
-      // |key - D| <= 2^-18 D; D_k <= s_k + off (every k); s_j + off <= D_j + e2 (winner).
-      const float e2 = 2.f * uc * (na + 2.f * pmax * l1 + off);
-      const float top = k1 * (1.f + 2.5f * kPack) + e2;   // >= s_j + off
-      cert = cw.K == 1 || (k2 * (1.f - kPack) > top);
-      thr = top - off;
-      thr += 4.f * kU * (k1 + off + e2);
-    } else {
-      j = 0;
-    }
-    if (!cert) {
-      const unsigned slot = atomicAdd(flags.count, 1u);
-      if (slot < flags.cap) {
-        flags.vec[slot] = i * G_range + (g - g_begin);
-        flags.thr[slot] = thr;
-      } else {
-        raise_error(err, ERRBIT_INDEX);
-      }
-    }
-    out_code[i * out_ld + (g - out_g0)] = j;
-    if (cert && st.cnt) {
-      float q[kD];
+  __syncthreads();
+  if (smem_stats) {  // one flush of this CTA's statistics (integer sums: order-free)
+    for (int k = tid; k < cw.K; k += blockDim.x) {
+      const int c = s_cnt[k];
+      if (c == 0) continue;
+      atomicAdd(&st.cnt[g * st.K + k], c);
 #pragma unroll
-      for (int p = 0; p < kD; ++p) q[p] = sq[p][tid];
-      stats_add(st, *st.scale, g, j, q);
+      for (int p = 0; p < kD; ++p)
+        atomicAdd(reinterpret_cast<unsigned long long*>(&st.bacc[(int64_t)k * kD + p]),
+                  (unsigned long long)s_bacc[k * kD + p]);
     }
   }
   tc::tc_fence_before();
@@ -1104,11 +1156,14 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     if (ex.stats && !keep_if_better) st = *ex.stats;
     CRVQ_CUDA(cudaMemsetAsync(fl.count, 0, sizeof(unsigned), stream));
     float* cbmax = reinterpret_cast<float*>(flag_mem.as<char>() + 128);
-    cbmax_kernel<<<1, 256, 0, stream>>>(cw.C, cw.K, cbmax);
-    CRVQ_LAUNCHED();
     {
-      // one row tile of 128 vectors per CTA, four CTAs per SM (128 tensor-memory columns
-      // each); the codebook's B images are precomputed per group when they fit in 256 MB
+      ProfScope pc("encode_cbmax", stream, 0.0);
+      cbmax_kernel<<<1, 256, 0, stream>>>(cw.C, cw.K, cbmax);
+      CRVQ_LAUNCHED();
+    }
+    {
+      // 128-row tiles, three CTAs per SM (128 tensor-memory columns each); the codebook's B
+      // images are precomputed per group when they fit in 256 MB
       const int nchunk = (int)ceil_div(cw.K, kTcCols);
       const size_t bbytes = (size_t)G_range * nchunk * kTcBTile;
       Scratch bmem;
@@ -1124,12 +1179,21 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
         CRVQ_LAUNCHED();
         bpre = bmem.as<char>();
       }
-      const size_t smem = (size_t)tcenc::kATile + 2 * (size_t)kTcBTile + 1024;
-      dim3 grid((unsigned)ceil_div(set.M, tcenc::kRows), (unsigned)G_range);
-      ProfScope ps("encode_argmin", stream, (double)nvec * cw.K);
+      const size_t smem = (size_t)tcenc::kATile + 2 * (size_t)kTcBTile +
+                          (size_t)kTcSmemStatsK * (kD * 8 + 4) + 1024;
+      // row tiles per CTA: about eight waves of three CTAs per SM (a fine-grained tail),
+      // each CTA reusing its group's resident codebook operand over several tiles
+      const int64_t row_tiles = ceil_div(set.M, tcenc::kRows);
+      const int64_t want_ctas = 24 * (int64_t)nsm;
+      const int64_t per_group = std::max<int64_t>(1, want_ctas / std::max<int64_t>(1, G_range));
+      const int tiles = (int)std::max<int64_t>(1, ceil_div(row_tiles, per_group));
+      dim3 grid((unsigned)ceil_div(row_tiles, tiles), (unsigned)G_range);
+      ProfScope ps(st.cnt ? "encode_argmin_lloyd" : "encode_argmin", stream,
+                   (double)nvec * cw.K);
       CRVQ_TRY(set_smem_attr(argmin_tc_kernel, smem));
       argmin_tc_kernel<<<grid, 128, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                    out_ld, out_g0, fl, st, cbmax, bpre, err);
+                                                    out_ld, out_g0, fl, st, cbmax, bpre, tiles,
+                                                    err);
       CRVQ_LAUNCHED();
     }
     {
