@@ -102,6 +102,12 @@ typedef struct crvq_kernel_stat {
 crvq_status crvq_profile_begin(void);
 crvq_status crvq_profile_end(crvq_kernel_stat* stats, int32_t cap, int32_t* n_stats);
 
+/* Restricts the next profiling sessions to kernel names starting with `prefix` (host string,
+ * copied; at most 63 characters); NULL or "" profiles every kernel again. Recording events
+ * costs host time per launch, so a narrow filter keeps a timed region close to unprofiled.
+ * Returns CRVQ_ERR_INVALID_ARG while a session is running or for a longer prefix. */
+crvq_status crvq_profile_filter(const char* prefix);
+
 /* Number of kernels this library has launched in this process (all devices). */
 int64_t crvq_launch_count(void);
 
@@ -196,9 +202,10 @@ crvq_status crvq_update_codebook(const float* T, int64_t ldT, int64_t M, int64_t
  * results and rounding are those of crvq_update_codebook; the caller still passes the
  * inputs and outputs. Its scratch is one file-scope device array of 4 MiB, held by every GPU
  * that loads the library until the process exits:
- *  - sizes whose statistics exceed it (G_cov * K * 4 + K * 64 + 512 bytes > 4 MiB - 256,
- *    e.g. K = 256 with more than ~4000 covered groups) return CRVQ_ERR_UNSUPPORTED before
- *    anything is enqueued;
+ *  - sizes whose statistics exceed it (G_cov * K * 4 + K * 64 + 256 + S * 296 * K bytes,
+ *    S = min(32, ceil(G_cov / 32)) group slices, each part rounded up to 256 bytes, above
+ *    4 MiB - 256; e.g. K = 256 with more than ~1600 covered groups) return
+ *    CRVQ_ERR_UNSUPPORTED before anything is enqueued;
  *  - every call shares the array, so calls that overlap on the GPU (different streams or
  *    devices' streams writing the same device's array) race; each call clears what must
  *    start at zero;

@@ -53,6 +53,7 @@ SIGNATURES = {
     "crvq_sync": (C.c_int32, [c_vp]),
     "crvq_profile_begin": (C.c_int32, []),
     "crvq_profile_end": (C.c_int32, [C.POINTER(crvq_kernel_stat), C.c_int32, c_i32p]),
+    "crvq_profile_filter": (C.c_int32, [C.c_char_p]),
     "crvq_launch_count": (C.c_int64, []),
     "crvq_hessian": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int32, C.c_float, c_vp, c_vp,
                                  c_vp, c_vp, c_vp]),

@@ -102,6 +102,11 @@ def crvq_profile_begin():
     _check(_L().crvq_profile_begin())
 
 
+def crvq_profile_filter(prefix=None):
+    """Profile only kernels whose name starts with `prefix` (None: every kernel)."""
+    _check(_L().crvq_profile_filter(None if not prefix else prefix.encode()))
+
+
 def crvq_profile_end() -> list[dict]:
     """Stop profiling; per kernel name: launches, summed event ms, summed algorithmic units."""
     arr = (_lib.crvq_kernel_stat * 64)()

@@ -76,6 +76,7 @@ namespace {
 std::atomic<long long> g_launches{0};
 std::atomic<bool> g_prof{false};
 std::mutex g_pmu;
+char g_filter[64] = {0};  // profiled name prefix ("" = all); changed only between sessions
 struct ProfRec {
   const char* name;
   cudaEvent_t a, b;
@@ -104,7 +105,8 @@ void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
 ProfScope::ProfScope(const char* name, cudaStream_t s, double units)
     : name_(name), s_(s), units_(units) {
-  if (g_prof.load(std::memory_order_relaxed)) {
+  if (g_prof.load(std::memory_order_relaxed) &&
+      strncmp(name, g_filter, strlen(g_filter)) == 0) {
     a_ = pool_get();
     if (a_ && cudaEventRecord(a_, s_) != cudaSuccess) {
       cudaGetLastError();
@@ -210,6 +212,18 @@ crvq_status crvq_profile_begin(void) {
       if (e) g_pool.push_back(e);
   }
   g_prof.store(true);
+  return CRVQ_OK;
+}
+
+crvq_status crvq_profile_filter(const char* prefix) {
+  if (g_prof.load()) return fail(CRVQ_ERR_INVALID_ARG, "crvq_profile_filter: a session is running");
+  const size_t n = prefix ? strlen(prefix) : 0;
+  if (n >= sizeof(g_filter))
+    return fail(CRVQ_ERR_INVALID_ARG, "crvq_profile_filter: prefix longer than %zu characters",
+                sizeof(g_filter) - 1);
+  std::lock_guard<std::mutex> lk(g_pmu);
+  memset(g_filter, 0, sizeof(g_filter));
+  if (n) memcpy(g_filter, prefix, n);
   return CRVQ_OK;
 }
 

@@ -168,16 +168,30 @@ __device__ __forceinline__ void stage_chunk(const float* __restrict__ C, int k0,
   }
 }
 
-// fp32 lower bound low_k of the score of codeword k. Any evaluation covered by the same
-// error analysis is a valid lower bound; the fallback needs no more than that.
+// fp32 lower / upper bounds s_k -+ Et_k of the score of codeword k from its terms t = (n, Na,
+// L1) (codeword_terms): s_k = n + sum_p m2q_p c_p, Et_k = u C (Na + 2 Pmax L1). Any
+// evaluation covered by the same error analysis is a valid bound; the fallback needs no more.
+__device__ __forceinline__ float low_from(float n, float na, float l1, const float c[kD],
+                                          const float m2q[kD], float nbeta, float cmul) {
+  float s = fmaf(-kU * cmul, na, n);
+#pragma unroll
+  for (int p = 0; p < kD; ++p) s = fmaf(m2q[p], c[p], s);
+  return fmaf(nbeta, l1, s);
+}
+
+__device__ __forceinline__ float up_from(float n, float na, float l1, const float c[kD],
+                                         const float m2q[kD], float pmax, float cmul) {
+  float s = fmaf(kU * cmul, na, n);
+#pragma unroll
+  for (int p = 0; p < kD; ++p) s = fmaf(m2q[p], c[p], s);
+  return fmaf(2.f * kU * cmul * pmax, l1, s);
+}
+
 __device__ __forceinline__ float low_score(const float c[kD], const float* H, const float m2q[kD],
                                            float nbeta, float cmul) {
   float n, na, l1;
   codeword_terms(c, H, n, na, l1);
-  float s = n - kU * cmul * na;
-#pragma unroll
-  for (int p = 0; p < kD; ++p) s = fmaf(m2q[p], c[p], s);
-  return fmaf(nbeta, l1, s);
+  return low_from(n, na, l1, c, m2q, nbeta, cmul);
 }
 
 // --------------------------------------------------------------------------- arg-min pass on
@@ -187,23 +201,21 @@ __device__ __forceinline__ float low_score(const float c[kD], const float* H, co
 // with every term split into tf32 hi + lo (3xTF32: hi*hi + hi*lo + lo*hi):
 //   A row (vector):   [q_hi x8 | q_hi x8 | q_lo x8 | 1 1 | beta_hi beta_hi beta_lo | off_hi off_lo | 0]
 //   B row (codeword): [c_hi x8 | c_lo x8 | c_hi x8 | n'_hi n'_lo | L1_hi L1_lo L1_hi | 1 1 | 0]
-// One tcgen05.mma M = 128 vectors x N = 256 codewords x K = 8, four per tile (K = 32), fp32
-// accumulator in tensor memory. The epilogue reads each row's 256 scores, packs the codeword's
-// index into the low 8 mantissa bits of the (non-negative) fp32 bound (a truncation of at most
-// 2^-15 relative) and keeps the two smallest keys with integer min / max. The certificate and
-// the fp64 fallback are those of the fp32 pass, with the bound multiplier raised to cover the
+// One tcgen05.mma M = 128 vectors x N = 128 codewords x K = 8, four per chunk (K = 32), fp32
+// accumulator in tensor memory. The epilogue reads each row's 128 scores in blocks of 32,
+// packs the column within its block into the low 5 mantissa bits of the (non-negative) fp32
+// bound (a truncation of at most 2^-18 relative) and keeps the two smallest keys of each
+// block with integer min / max; the block is tracked by the merge. The certificate and the
+// fp64 fallback are those of the fp32 pass, with the bound multiplier raised to cover the
 // tensor-core products and accumulation (about 2^-22 per split product and fp32 accumulation
 // over 32 terms) and the packing.
 namespace tcenc {
 
 constexpr int kRows = 128;        // vectors per row tile (TMEM lanes)
-constexpr int kCols = 256;        // codewords per chunk (MMA N)
 constexpr int kK = 32;            // tf32 columns per row
 constexpr int kATile = kRows * kK * 4;   // 16 KB
-constexpr int kBTile = kCols * kK * 4;   // 32 KB
 constexpr float kCmul = 256.f;           // bound multiplier (about twice the analysis)
 constexpr float kPack = 3.8146973e-06f;  // 2^-18: relative truncation of the packed key
-constexpr uint32_t kIdesc = tc::idesc_tf32(kRows, kCols);
 
 __device__ __forceinline__ uint32_t koff(int r, int k) {
   return (uint32_t)(((r >> 3) * (kK / 4) + (k >> 2)) * 128 + (r & 7) * 16 + (k & 3) * 4);
@@ -223,13 +235,6 @@ __device__ __forceinline__ void split(float x, uint32_t& hi, uint32_t& lo) {
 }
 
 }  // namespace tcenc
-
-// Top-2 merge of two (best, second) key pairs.
-__device__ __forceinline__ void merge2(uint32_t& x1, uint32_t& x2, uint32_t y1, uint32_t y2) {
-  const uint32_t hi = max(x1, y1);
-  x1 = min(x1, y1);
-  x2 = min(hi, min(x2, y2));
-}
 
 // Row of the B operand for codeword kk of C (K codewords): [c_hi | c_lo | c_hi | n'_hi n'_lo |
 // L1_hi L1_lo L1_hi | 1 1 | 0]; padding rows (kk >= K) score +1e30.
@@ -267,9 +272,10 @@ constexpr int kTcBTile = kTcCols * tcenc::kK * 4;  // 16 KB
 
 // B operand images of the codebook for groups [g_begin, g_begin + G_range): block
 // (g, chunk) holds 128 rows in the canonical shared-memory layout, ready for a bulk copy.
+// terms[(g - g_begin) K + k] = (n, Na, L1, 0) of codeword k in group g (codeword_terms).
 __global__ void __launch_bounds__(128)
 prep_b_kernel(SetView set, int64_t g_begin, int64_t G_range, const float* __restrict__ C,
-              int K, int nchunk, float uc, char* __restrict__ out) {
+              int K, int nchunk, float uc, char* __restrict__ out, float4* __restrict__ terms) {
   const int64_t total = G_range * nchunk * (int64_t)kTcCols;
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
        e += (int64_t)gridDim.x * blockDim.x) {
@@ -278,8 +284,15 @@ prep_b_kernel(SetView set, int64_t g_begin, int64_t G_range, const float* __rest
     const int chunk = (int)(blk % nchunk);
     const int64_t g = g_begin + blk / nchunk;
     uint32_t v[tcenc::kK];
-    build_b_row(C, K, chunk * kTcCols + row, set.Hb + g * kD * kD, uc, v);
+    const int kk = chunk * kTcCols + row;
+    build_b_row(C, K, kk, set.Hb + g * kD * kD, uc, v);
     tcenc::put_row(out + blk * kTcBTile, row, v);
+    if (kk < K) {
+      float cv[kD], n, na, l1;
+      load_vec(C + (int64_t)kk * kD, cv);
+      codeword_terms(cv, set.Hb + g * kD * kD, n, na, l1);
+      terms[(g - g_begin) * K + kk] = make_float4(n, na, l1, 0.f);
+    }
   }
 }
 
@@ -295,7 +308,8 @@ __global__ void __launch_bounds__(128, 3)
 argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
                  int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
                  FlagList flags, StatsView st, const float* __restrict__ cbmax,
-                 const char* __restrict__ bpre, int tiles, unsigned* err) {
+                 const char* __restrict__ bpre, const float4* __restrict__ terms, int tiles,
+                 unsigned* err) {
   using namespace tcenc;
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -304,6 +318,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   char* Bbuf = smem + kATile;          // 2 x 16 KB
   long long* s_bacc = reinterpret_cast<long long*>(Bbuf + 2 * kTcBTile);  // [256][8]
   int* s_cnt = reinterpret_cast<int*>(s_bacc + kTcSmemStatsK * kD);       // [256]
+  float* sQ = reinterpret_cast<float*>(s_cnt + kTcSmemStatsK);            // [128][8] H r
   __shared__ float sH[kD * kD];
   __shared__ __align__(8) uint64_t bar_mma, bar_b[2];
   __shared__ uint32_t tmem_slot;
@@ -317,6 +332,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   const int nchunk = (cw.K + kTcCols - 1) / kTcCols;
   const bool resident = nchunk <= 2;
   const char* bimg = bpre ? bpre + (size_t)(g - g_begin) * nchunk * kTcBTile : nullptr;
+  const float4* gterms = terms ? terms + (g - g_begin) * cw.K : nullptr;
   const bool smem_stats = st.cnt && cw.K <= kTcSmemStatsK;
 
   if (tid < kD * kD) sH[tid] = set.Hb[g * kD * kD + tid];
@@ -335,7 +351,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   __syncthreads();
   tc::tc_fence_after();
   const uint32_t tmem = tmem_slot;
-  const double scale = st.cnt ? *st.scale : 0.0;
+  const int sexp = st.cnt ? stats_scale_exp(*st.scale) : 0;
 
   // Bound on Na_k over the codebook for this group: (max row sum |H_g|) L1max cinfmax.
   float hrow = 0.f;
@@ -400,6 +416,12 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       off = (rr + 32.f * kU * ra + 2.f * uc * (hrow * l1max * cinf + 2.f * pmax * l1max)) *
                 (1.f + 4.f * uc) + 1e-30f;
       const float beta = -2.f * uc * pmax;
+      if (st.cnt) {  // H r of this row, kept for the statistics (-m2q / 2, exact)
+        *reinterpret_cast<float4*>(sQ + tid * kD) =
+            make_float4(-0.5f * m2q[0], -0.5f * m2q[1], -0.5f * m2q[2], -0.5f * m2q[3]);
+        *reinterpret_cast<float4*>(sQ + tid * kD + 4) =
+            make_float4(-0.5f * m2q[4], -0.5f * m2q[5], -0.5f * m2q[6], -0.5f * m2q[7]);
+      }
       uint32_t row[kK];
 #pragma unroll
       for (int p = 0; p < kD; ++p) {
@@ -504,11 +526,18 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       const float k1 = __uint_as_float(g1), k2 = __uint_as_float(g2);
       bool cert = false;
       float thr = INFINITY;
-      float cv[kD];
       if (j < cw.K) {
         float n, na, l1;
-        load_vec(cw.C + (int64_t)j * kD, cv);
-        codeword_terms(cv, sH, n, na, l1);
+        if (gterms) {
+          const float4 tj = gterms[j];
+          n = tj.x;
+          na = tj.y;
+          l1 = tj.z;
+        } else {
+          float cv[kD];
+          load_vec(cw.C + (int64_t)j * kD, cv);
+          codeword_terms(cv, sH, n, na, l1);
+        }
         // |key - D| <= 2^-18 D; D_k <= s_k + off (every k); s_j + off <= D_j + e2 (winner).
         const float e2 = 2.f * uc * (na + 2.f * pmax * l1 + off);
         const float top = k1 * (1.f + 2.5f * kPack) + e2;   // >= s_j + off
@@ -529,23 +558,20 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       }
       out_code[i * out_ld + (g - out_g0)] = j;
       if (cert && st.cnt) {
-        // the fallback's target / H r (bit-identical to the standalone update's)
-        float rv[kD], a[kD], m2q[kD], pm;
-        target32(set, cbs, n_fixed, i, g, rv, a, err);
-        vector_terms(rv, a, sH, m2q, pm);
+        // H r from the prologue (bit-identical to the standalone update's H tau)
+        float q[kD];
+        const float4 q0 = *reinterpret_cast<const float4*>(sQ + tid * kD);
+        const float4 q1 = *reinterpret_cast<const float4*>(sQ + tid * kD + 4);
+        q[0] = q0.x; q[1] = q0.y; q[2] = q0.z; q[3] = q0.w;
+        q[4] = q1.x; q[5] = q1.y; q[6] = q1.z; q[7] = q1.w;
         if (smem_stats) {
           atomicAdd(&s_cnt[j], 1);
 #pragma unroll
-          for (int p = 0; p < kD; ++p) {
-            const long long v = __double2ll_rn((double)(-0.5f * m2q[p]) * scale);
+          for (int p = 0; p < kD; ++p)
             atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[j * kD + p]),
-                      (unsigned long long)v);
-          }
+                      (unsigned long long)fix_rn(q[p], sexp));
         } else {
-          float q[kD];
-#pragma unroll
-          for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[p];
-          stats_add(st, scale, g, j, q);
+          stats_add(st, sexp, g, j, q);
         }
       }
     }
@@ -605,21 +631,27 @@ cbmax_kernel(const float* __restrict__ C, int K, float* __restrict__ cbmax) {
   }
 }
 
-// Fallback: one warp per flagged vector. Recomputes low_k for every codeword; those with
-// low_k <= threshold are re-scored in fp64 and the smallest fp64 err wins (ties to the
-// smaller index). Adds the statistics of the decided code when requested.
+// Fallback: one warp per flagged vector. A first sweep takes U = the smallest fp32 upper
+// bound s_k + Et_k over the codebook (and the fast pass's threshold); every codeword whose
+// lower bound s_k - Et_k is at most U is a candidate (the exact arg-min always is: its err
+// is at most U). Candidates are queued in shared memory and re-scored in fp64 one per lane,
+// so the fp64 work of a warp is one pass per 32 candidates; the smallest fp64 err wins (ties
+// to the smaller index). Adds the statistics of the decided code when requested.
 __global__ void __launch_bounds__(kThreads)
 argmin_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs,
                        int n_fixed, int s_idx, int32_t* __restrict__ out_code,
                        int64_t out_ld, int64_t out_g0, FlagList flags, StatsView st,
-                       unsigned* err) {
+                       const float4* __restrict__ terms, unsigned* err) {
+  __shared__ int queue[kThreads / 32][32];
   const int lane = threadIdx.x & 31;
+  int* q = queue[threadIdx.x >> 5];
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const unsigned cnt = min((unsigned long long)*flags.count, (unsigned long long)flags.cap);
   if (flags.total && blockIdx.x == 0 && threadIdx.x == 0) atomicAdd(flags.total, cnt);
   const CbView cw = cbs.cb[s_idx];
   const float cmul = bound_mult(n_fixed);
+  const unsigned lt_mask = (1u << lane) - 1u;
   for (int64_t f = warp; f < cnt; f += nwarps) {
     const int64_t vi = flags.vec[f];
     const int64_t i = vi / G_range, g = g_begin + vi % G_range;
@@ -631,19 +663,58 @@ argmin_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs
     const float nbeta = -2.f * kU * cmul * pmax;
     double r64[kD];
     target64(set, cbs, n_fixed, i, g, r64, err);
+    const float4* gterms = terms ? terms + (g - g_begin) * cw.K : nullptr;
+    auto terms_of = [&](int k, const float c[kD], float& n, float& na, float& l1) {
+      if (gterms) {
+        const float4 t = gterms[k];
+        n = t.x;
+        na = t.y;
+        l1 = t.z;
+      } else {
+        codeword_terms(c, H, n, na, l1);
+      }
+    };
+    float U = thr;
+    for (int k = lane; k < cw.K; k += 32) {
+      float c[kD], n, na, l1;
+      load_vec(cw.C + (int64_t)k * kD, c);
+      terms_of(k, c, n, na, l1);
+      U = fminf(U, up_from(n, na, l1, c, m2q, pmax, cmul));
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) U = fminf(U, __shfl_xor_sync(0xffffffffu, U, off));
     double best = INFINITY;
     int bestk = 0x7fffffff;
-    for (int k = lane; k < cw.K; k += 32) {
-      float c[kD];
-      load_vec(cw.C + (int64_t)k * kD, c);
-      if (low_score(c, H, m2q, nbeta, cmul) <= thr) {
+    int qn = 0;  // queued candidates (the same in every lane)
+    auto drain = [&]() {
+      __syncwarp();
+      if (lane < qn) {
+        const int k = q[lane];
         const double e = quad_err64(r64, cw.C + (int64_t)k * kD, H);
         if (e < best || (e == best && k < bestk)) {
           best = e;
           bestk = k;
         }
       }
+      __syncwarp();
+      qn = 0;
+    };
+    for (int k0 = 0; k0 < cw.K; k0 += 32) {
+      const int k = k0 + lane;
+      bool cand = false;
+      if (k < cw.K) {
+        float c[kD], n, na, l1;
+        load_vec(cw.C + (int64_t)k * kD, c);
+        terms_of(k, c, n, na, l1);
+        cand = low_from(n, na, l1, c, m2q, nbeta, cmul) <= U;
+      }
+      const unsigned m = __ballot_sync(0xffffffffu, cand);
+      const int n = __popc(m);
+      if (qn + n > 32) drain();
+      if (cand) q[qn + __popc(m & lt_mask)] = k;
+      qn += n;
     }
+    drain();
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
       const double ob = __shfl_xor_sync(0xffffffffu, best, off);
@@ -659,10 +730,10 @@ argmin_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs
       } else {
         out_code[i * out_ld + (g - out_g0)] = bestk;
         if (st.cnt) {
-          float q[kD];
+          float qv[kD];
 #pragma unroll
-          for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[p];
-          stats_add(st, *st.scale, g, bestk, q);
+          for (int p = 0; p < kD; ++p) qv[p] = -0.5f * m2q[p];
+          stats_add(st, stats_scale_exp(*st.scale), g, bestk, qv);
         }
       }
     }
@@ -883,7 +954,8 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
       const unsigned slot = atomicAdd(flags.count, 1u);
       if (slot < flags.cap) {
         flags.vec[slot] = vi;
-        flags.thr[slot] = 0.f;
+        // every member of the exact top-keep has err <= the keep-th listed exact err
+        flags.thr[slot] = isfinite(ev[keep - 1]) ? __double2float_ru(ev[keep - 1]) : INFINITY;
       } else {
         raise_error(err, ERRBIT_INDEX);
       }
@@ -901,13 +973,18 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
 }
 
 // Exact stage for flagged vectors: one warp per vector; the lanes stride over the (h, k)
-// candidates in fp64 keeping a sorted local top-Bs; a warp merge then extracts the global
-// top-Bs in (err, h, k) order.
+// candidates, re-score in fp64 those whose fp32 lower bound is at most the vector's
+// threshold (the keep-th exact err among the fast pass's listed candidates, which bounds
+// every member of the exact top-Bs) and keep a sorted local top-Bs; a warp merge then
+// extracts the global top-Bs in (err, h, k) order.
 __global__ void __launch_bounds__(kThreads)
 beam_stage_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs,
                            int n_fixed, StageDesc sd, BeamBufs bb, FlagList flags,
                            unsigned* err) {
+  __shared__ int queue[kThreads / 32][32], queue_h[kThreads / 32][32];
   const int lane = threadIdx.x & 31;
+  int* q = queue[threadIdx.x >> 5];
+  int* qh = queue_h[threadIdx.x >> 5];
   const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
   const unsigned cnt = min((unsigned long long)*flags.count, (unsigned long long)flags.cap);
@@ -921,17 +998,25 @@ beam_stage_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList
     double tgt[kD];
     target64(set, cbs, n_fixed, i, g, tgt, err);
     const int Bh = (sd.s == 0) ? 1 : bb.n_in[vi];
+    const float thr = flags.thr[f];
+    const float cmul = bound_mult(n_fixed + sd.s);
     double be[16];
     int bh[16], bk[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) be[j] = INFINITY;
     int nb = 0;
-    for (int h = 0; h < Bh; ++h) {
-      double r64[kD];
-      const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
-      hyp_residual64(tgt, cbs, sd, pc, r64, err);
-      for (int k = lane; k < cw.K; k += 32) {
+    // Candidates (h, k) are queued in increasing (h, k) order and scored one per lane, so
+    // every lane still sees its own candidates in increasing (h, k): strict comparison in
+    // the insertion keeps ties in (h, k) order.
+    int qn = 0;
+    auto drain = [&]() {
+      __syncwarp();
+      if (lane < qn) {
+        const int h = qh[lane], k = q[lane];
+        double r64[kD];
+        const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
+        hyp_residual64(tgt, cbs, sd, pc, r64, err);
         const double e = quad_err64(r64, cw.C + (int64_t)k * kD, H);
-        // this lane sees its candidates in increasing (h, k): strict comparison keeps ties
-        // in (h, k) order
         if (nb < Bs || e < be[nb - 1]) {
           int pos = nb < Bs ? nb : Bs - 1;
           while (pos > 0 && e < be[pos - 1]) {
@@ -942,7 +1027,37 @@ beam_stage_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList
           if (nb < Bs) ++nb;
         }
       }
+      __syncwarp();
+      qn = 0;
+    };
+    for (int h = 0; h < Bh; ++h) {
+      double r64[kD];
+      const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
+      hyp_residual64(tgt, cbs, sd, pc, r64, err);
+      float m2q[kD], rr, ra, pmax;
+      hyp_terms(r64, H, m2q, rr, ra, pmax);
+      const float base = rr - kU * cmul * ra;
+      const float nbeta = -2.f * kU * cmul * pmax;
+      for (int k0 = 0; k0 < cw.K; k0 += 32) {
+        const int k = k0 + lane;
+        bool cand = false;
+        if (k < cw.K) {
+          float c[kD];
+          load_vec(cw.C + (int64_t)k * kD, c);
+          cand = base + low_score(c, H, m2q, nbeta, cmul) <= thr;
+        }
+        const unsigned m = __ballot_sync(0xffffffffu, cand);
+        const int n = __popc(m);
+        if (qn + n > 32) drain();
+        if (cand) {
+          const int pos = qn + __popc(m & ((1u << lane) - 1u));
+          q[pos] = k;
+          qh[pos] = h;
+        }
+        qn += n;
+      }
     }
+    drain();
     // Warp merge: rounds of (min over the lanes' heads by (err, h, k)); the winner pops.
     int head = 0;
     int32_t* out = bb.hyp_out + vi * B * S;
@@ -979,8 +1094,48 @@ beam_stage_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList
   }
 }
 
+// fp32 err of a whole tuple for vector (i, g): the fixed codebooks' codes, then for each
+// searched stage q the code sc[q] (or, with sc null, the code already stored), with a bound
+// on its distance from the exact err: the residual's rounding (m subtractions) and the two
+// FMA chains of the quadratic form stay below (16 + 2 m) u a^T |H| a, a_j = |t_j| + sum of
+// the |c_j| subtracted; the bound uses the multiplier of the score bounds, about twice that.
+__device__ void tuple_err32(const SetView& set, const CbList& cbs, int n_fixed,
+                            const StageDesc& sd, int64_t i, int64_t g, const int32_t* sc,
+                            const float* H, float& e, float& bnd, unsigned* err) {
+  float r[kD], a[kD];
+  target32(set, cbs, n_fixed, i, g, r, a, err);
+  for (int q = 0; q < sd.S; ++q) {
+    const CbView& cb = cbs.cb[sd.st[q]];
+    const int32_t k = sc ? sc[q] : cb.codes[i * cb.ld + g];
+    if (!code_ok(k, cb.K, err)) continue;
+    float c[kD];
+    load_vec(cb.C + (int64_t)k * kD, c);
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      r[j] -= c[j];
+      a[j] += fabsf(c[j]);
+    }
+  }
+  float ee = 0.f, na = 0.f;
+#pragma unroll
+  for (int b = 0; b < kD; ++b) {
+    float hb = 0.f, hab = 0.f;
+#pragma unroll
+    for (int a2 = 0; a2 < kD; ++a2) {
+      hb = fmaf(r[a2], H[a2 * kD + b], hb);
+      hab = fmaf(a[a2], fabsf(H[a2 * kD + b]), hab);
+    }
+    ee = fmaf(hb, r[b], ee);
+    na = fmaf(hab, a[b], na);
+  }
+  e = ee;
+  bnd = kU * bound_mult(n_fixed + sd.S + 1) * na;
+}
+
 // Final step of a multi-stage (or keep-if-better) encode: write the best tuple, or keep the
-// tuple already in the codes when its fp64 err is strictly smaller; optional vec_err.
+// tuple already in the codes when its err is strictly smaller. The comparison is decided by
+// fp32 errs with bounds when they separate, in fp64 otherwise; an unchanged tuple needs no
+// comparison. vec_err (optional) is the fp64 err of the tuple kept.
 __global__ void beam_finalize_kernel(SetView set, int64_t g_begin, int64_t G_range,
                                      CbList cbs, int n_fixed, StageDesc sd,
                                      const int32_t* __restrict__ hyp, bool keep_if_better,
@@ -993,8 +1148,25 @@ __global__ void beam_finalize_kernel(SetView set, int64_t g_begin, int64_t G_ran
     const float* H = set.Hb + g * kD * kD;
     const int32_t* best = hyp + vi * B * S;
     bool use_old = false;
-    double e_new = 0.0, e_old = 0.0;
-    if (keep_if_better || vec_err) {
+    bool exact = vec_err != nullptr;
+    if (keep_if_better) {
+      bool same = true;
+      for (int q = 0; q < S; ++q) {
+        const CbView& cb = cbs.cb[sd.st[q]];
+        same = same && cb.codes[i * cb.ld + g] == best[q];
+      }
+      if (!same) {
+        float en, bn, eo, bo;
+        tuple_err32(set, cbs, n_fixed, sd, i, g, best, H, en, bn, err);
+        tuple_err32(set, cbs, n_fixed, sd, i, g, nullptr, H, eo, bo, err);
+        if (eo + bo < en - bn) {
+          use_old = true;
+        } else if (!(eo - bo >= en + bn)) {
+          exact = true;  // not separated (or not finite): decide in fp64
+        }
+      }
+    }
+    if (exact) {
       double tgt[kD];
       target64(set, cbs, n_fixed, i, g, tgt, err);
       double r[kD];
@@ -1007,7 +1179,8 @@ __global__ void beam_finalize_kernel(SetView set, int64_t g_begin, int64_t G_ran
 #pragma unroll
         for (int j = 0; j < kD; ++j) r[j] -= (double)c[j];
       }
-      e_new = quad_err64(r, nullptr, H);
+      const double e_new = quad_err64(r, nullptr, H);
+      double e_old = e_new;
       if (keep_if_better) {
 #pragma unroll
         for (int j = 0; j < kD; ++j) r[j] = tgt[j];
@@ -1022,6 +1195,7 @@ __global__ void beam_finalize_kernel(SetView set, int64_t g_begin, int64_t G_ran
         e_old = quad_err64(r, nullptr, H);
         use_old = e_old < e_new;
       }
+      if (vec_err) vec_err[i * set.G_sub + g] = (float)(use_old ? e_old : e_new);
     }
     if (!use_old) {
       for (int q = 0; q < S; ++q) {
@@ -1029,7 +1203,6 @@ __global__ void beam_finalize_kernel(SetView set, int64_t g_begin, int64_t G_ran
         cb.codes[i * cb.ld + g] = best[q];
       }
     }
-    if (vec_err) vec_err[i * set.G_sub + g] = (float)(use_old ? e_old : e_new);
   }
 }
 
@@ -1161,26 +1334,31 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
       cbmax_kernel<<<1, 256, 0, stream>>>(cw.C, cw.K, cbmax);
       CRVQ_LAUNCHED();
     }
-    {
-      // 128-row tiles, three CTAs per SM (128 tensor-memory columns each); the codebook's B
-      // images are precomputed per group when they fit in 256 MB
-      const int nchunk = (int)ceil_div(cw.K, kTcCols);
-      const size_t bbytes = (size_t)G_range * nchunk * kTcBTile;
-      Scratch bmem;
-      const char* bpre = nullptr;
+    // The codebook's B images per group (when they fit in 256 MB) and its per-group terms
+    // (n, Na, L1), read by the arg-min pass and its fallback.
+    const int nchunk = (int)ceil_div(cw.K, kTcCols);
+    const size_t bbytes = (size_t)G_range * nchunk * kTcBTile;
+    const size_t tbytes = align_up((size_t)G_range * cw.K * sizeof(float4), 256);
+    Scratch bmem;
+    const char* bpre = nullptr;
+    const float4* terms = nullptr;
+    if (bbytes <= (size_t(256) << 20)) {
+      CRVQ_TRY(bmem.alloc(bbytes + tbytes, stream));
       const float uc = kU * (tcenc::kCmul + 4.f * n_fixed);
-      if (bbytes <= (size_t(256) << 20)) {
-        CRVQ_TRY(bmem.alloc(bbytes, stream));
-        ProfScope pb("encode_prep_b", stream, (double)G_range * nchunk * kTcCols);
-        const int64_t rows = (int64_t)G_range * nchunk * kTcCols;
-        prep_b_kernel<<<(unsigned)std::min<int64_t>(ceil_div(rows, 128), 16 * nsm), 128, 0,
-                        stream>>>(set, g_begin, G_range, cw.C, cw.K, nchunk, uc,
-                                  bmem.as<char>());
-        CRVQ_LAUNCHED();
-        bpre = bmem.as<char>();
-      }
+      ProfScope pb("encode_prep_b", stream, (double)G_range * nchunk * kTcCols);
+      const int64_t rows = (int64_t)G_range * nchunk * kTcCols;
+      float4* tout = reinterpret_cast<float4*>(bmem.as<char>() + bbytes);
+      prep_b_kernel<<<(unsigned)std::min<int64_t>(ceil_div(rows, 128), 16 * nsm), 128, 0,
+                      stream>>>(set, g_begin, G_range, cw.C, cw.K, nchunk, uc, bmem.as<char>(),
+                                tout);
+      CRVQ_LAUNCHED();
+      bpre = bmem.as<char>();
+      terms = tout;
+    }
+    {
+      // 128-row tiles, three CTAs per SM (128 tensor-memory columns each)
       const size_t smem = (size_t)tcenc::kATile + 2 * (size_t)kTcBTile +
-                          (size_t)kTcSmemStatsK * (kD * 8 + 4) + 1024;
+                          (size_t)kTcSmemStatsK * (kD * 8 + 4) + tcenc::kRows * kD * 4 + 1024;
       // row tiles per CTA: about eight waves of three CTAs per SM (a fine-grained tail),
       // each CTA reusing its group's resident codebook operand over several tiles
       const int64_t row_tiles = ceil_div(set.M, tcenc::kRows);
@@ -1192,15 +1370,15 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
                    (double)nvec * cw.K);
       CRVQ_TRY(set_smem_attr(argmin_tc_kernel, smem));
       argmin_tc_kernel<<<grid, 128, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                    out_ld, out_g0, fl, st, cbmax, bpre, tiles,
-                                                    err);
+                                                    out_ld, out_g0, fl, st, cbmax, bpre, terms,
+                                                    tiles, err);
       CRVQ_LAUNCHED();
     }
     {
       ProfScope ps2("encode_argmin_fallback", stream, 0.0);
       argmin_fallback_kernel<<<4 * nsm, kThreads, 0, stream>>>(set, g_begin, G_range, cbs,
                                                                n_fixed, s_idx, out, out_ld,
-                                                               out_g0, fl, st, err);
+                                                               out_g0, fl, st, terms, err);
       CRVQ_LAUNCHED();
     }
     if (ex.scores) *ex.scores += (double)nvec * cw.K;

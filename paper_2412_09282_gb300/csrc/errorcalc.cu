@@ -12,11 +12,14 @@ namespace crvq {
 
 namespace {
 
-// Reconstruction of vector (i, g) in fp64 (sum in codebook order), as fp32 values.
-__device__ __forceinline__ void recon(const CbList& cbs, int64_t i, int64_t g, double r[kD],
+// Reconstruction of vector (i, g): the sum of the covering codebooks' codewords (codebook
+// order), correctly rounded to fp32 like the fp64 sum rounded once. With at most two terms the
+// fp32 sum is that value (the exact sum of two fp32 values rounds to fp32 the same way
+// whether or not it first passes through fp64); three or more terms are summed in fp64.
+__device__ __forceinline__ void recon(const CbList& cbs, int64_t i, int64_t g, float r[kD],
                                       unsigned* err) {
-#pragma unroll
-  for (int j = 0; j < kD; ++j) r[j] = 0.0;
+  const float* cw[kMaxCodebooks];
+  int n = 0;
   for (int s = 0; s < cbs.n; ++s) {
     const CbView& cb = cbs.cb[s];
     if (g >= cb.G_cov) continue;
@@ -25,85 +28,125 @@ __device__ __forceinline__ void recon(const CbList& cbs, int64_t i, int64_t g, d
       raise_error(err, ERRBIT_INDEX);
       continue;
     }
-    const float* c = cb.C + (int64_t)k * kD;
+    cw[n++] = cb.C + (int64_t)k * kD;
+  }
+  if (n <= 2) {
 #pragma unroll
-    for (int j = 0; j < kD; ++j) r[j] += (double)c[j];
+    for (int j = 0; j < kD; ++j) r[j] = 0.f;
+    for (int q = 0; q < n; ++q) {
+      const float4 a = *reinterpret_cast<const float4*>(cw[q]);
+      const float4 b = *reinterpret_cast<const float4*>(cw[q] + 4);
+      r[0] += a.x; r[1] += a.y; r[2] += a.z; r[3] += a.w;
+      r[4] += b.x; r[5] += b.y; r[6] += b.z; r[7] += b.w;
+    }
+  } else {
+    double d[kD];
+#pragma unroll
+    for (int j = 0; j < kD; ++j) d[j] = 0.0;
+    for (int q = 0; q < n; ++q)
+#pragma unroll
+      for (int j = 0; j < kD; ++j) d[j] += (double)cw[q][j];
+#pragma unroll
+    for (int j = 0; j < kD; ++j) r[j] = (float)d[j];
   }
 }
 
-// One CTA per row: block/critical losses and ||dW||^2 of the row (fp64 partials), and the row
-// of W_hat and of dW in the original channel order (staged in shared memory).
+// One CTA per row (grid-strided): the row of W_hat and of dW = W - W_hat in the original
+// channel order (staged in shared memory, then stored with 16-byte writes), and the row's
+// block loss, critical loss and ||dW||^2. Each vector's terms are fp32 (the quadratic form as
+// two FMA chains); the thread's running sums and the row reduction are fp64.
 __global__ void __launch_bounds__(256)
 decode_row_kernel(const float* __restrict__ Ws, int64_t M, int64_t N, const float* __restrict__ Hb,
                   const int32_t* __restrict__ perm, CbList cbs, int64_t n_crit_groups,
                   float* __restrict__ W_hat, float* __restrict__ dW,
                   double* __restrict__ row_part, unsigned* err) {
-  extern __shared__ __align__(16) float srow[];
-  __shared__ double red[3][256];
+  extern __shared__ __align__(16) float srow[];  // [N] W_hat row (if any), then [N] dW row
+  float* s_hat = srow;
+  float* s_dw = srow + (W_hat ? N : 0);
+  __shared__ double red[3][256 / 32];
   const int64_t G = N / kD;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int64_t i = blockIdx.x; i < M; i += gridDim.x) {
     double lb = 0.0, lc = 0.0, sq = 0.0;
-    for (int pass = 0; pass < 2; ++pass) {
-      float* out = pass == 0 ? W_hat : dW;
-      if (pass == 1 && !dW) break;
-      __syncthreads();
-      for (int64_t g = threadIdx.x; g < G; g += blockDim.x) {
-        double r[kD];
-        recon(cbs, i, g, r, err);
-        const float* t = Ws + i * N + g * kD;
-        float dl[kD];
+    __syncthreads();  // the previous row's stores have read the staging rows
+    for (int64_t g = threadIdx.x; g < G; g += blockDim.x) {
+      float r[kD], t[kD], dl[kD];
+      recon(cbs, i, g, r, err);
+      const float4 t0 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD);
+      const float4 t1 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD + 4);
+      t[0] = t0.x; t[1] = t0.y; t[2] = t0.z; t[3] = t0.w;
+      t[4] = t1.x; t[5] = t1.y; t[6] = t1.z; t[7] = t1.w;
+      float q2 = 0.f;
 #pragma unroll
-        for (int j = 0; j < kD; ++j) dl[j] = (float)((double)t[j] - r[j]);
-        if (pass == 0) {
-          const float* H = Hb + g * kD * kD;
-          float e = 0.f;
-#pragma unroll
-          for (int b = 0; b < kD; ++b) {
-            float hb = 0.f;
-#pragma unroll
-            for (int a = 0; a < kD; ++a) hb = fmaf(dl[a], H[a * kD + b], hb);
-            e = fmaf(hb, dl[b], e);
-          }
-          lb += (double)e;
-          if (g < n_crit_groups) lc += (double)e;
-#pragma unroll
-          for (int j = 0; j < kD; ++j) sq += (double)dl[j] * (double)dl[j];
-        }
-        if (out) {
-#pragma unroll
-          for (int j = 0; j < kD; ++j) {
-            const int64_t p = g * kD + j;
-            int64_t col = perm ? perm[p] : p;
-            if (col < 0 || col >= N) {
-              raise_error(err, ERRBIT_INDEX);
-              continue;
-            }
-            srow[col] = pass == 0 ? (float)r[j] : dl[j];
-          }
-        }
+      for (int j = 0; j < kD; ++j) {
+        dl[j] = t[j] - r[j];
+        q2 = fmaf(dl[j], dl[j], q2);
       }
-      __syncthreads();
-      if (out) {
-        float* dst = out + i * N;
-        for (int64_t c = (int64_t)threadIdx.x * 4; c < N; c += (int64_t)blockDim.x * 4)
-          *reinterpret_cast<float4*>(dst + c) = *reinterpret_cast<const float4*>(srow + c);
+      const float4* H4 = reinterpret_cast<const float4*>(Hb + g * kD * kD);
+      float e = 0.f;
+#pragma unroll
+      for (int a = 0; a < kD; ++a) {
+        const float4 h0 = __ldg(H4 + 2 * a), h1 = __ldg(H4 + 2 * a + 1);
+        float hb = dl[0] * h0.x;
+        hb = fmaf(dl[1], h0.y, hb);
+        hb = fmaf(dl[2], h0.z, hb);
+        hb = fmaf(dl[3], h0.w, hb);
+        hb = fmaf(dl[4], h1.x, hb);
+        hb = fmaf(dl[5], h1.y, hb);
+        hb = fmaf(dl[6], h1.z, hb);
+        hb = fmaf(dl[7], h1.w, hb);
+        e = fmaf(hb, dl[a], e);
+      }
+      lb += (double)e;
+      if (g < n_crit_groups) lc += (double)e;
+      sq += (double)q2;
+#pragma unroll
+      for (int j = 0; j < kD; ++j) {
+        const int64_t p = g * kD + j;
+        const int64_t col = perm ? perm[p] : p;
+        if (col < 0 || col >= N) {
+          raise_error(err, ERRBIT_INDEX);
+          continue;
+        }
+        if (W_hat) s_hat[col] = r[j];
+        if (dW) s_dw[col] = dl[j];
       }
     }
-    red[0][threadIdx.x] = lb;
-    red[1][threadIdx.x] = lc;
-    red[2][threadIdx.x] = sq;
     __syncthreads();
-    for (int w = blockDim.x / 2; w > 0; w >>= 1) {
-      if ((int)threadIdx.x < w) {
-#pragma unroll
-        for (int q = 0; q < 3; ++q) red[q][threadIdx.x] += red[q][threadIdx.x + w];
+    {
+      if (W_hat) {
+        float* dst = W_hat + i * N;
+        for (int64_t c = (int64_t)threadIdx.x * 4; c < N; c += (int64_t)blockDim.x * 4)
+          *reinterpret_cast<float4*>(dst + c) = *reinterpret_cast<const float4*>(s_hat + c);
       }
-      __syncthreads();
+      if (dW) {
+        float* dd = dW + i * N;
+        for (int64_t c = (int64_t)threadIdx.x * 4; c < N; c += (int64_t)blockDim.x * 4)
+          *reinterpret_cast<float4*>(dd + c) = *reinterpret_cast<const float4*>(s_dw + c);
+      }
     }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      lb += __shfl_xor_sync(0xffffffffu, lb, off);
+      lc += __shfl_xor_sync(0xffffffffu, lc, off);
+      sq += __shfl_xor_sync(0xffffffffu, sq, off);
+    }
+    if (lane == 0) {
+      red[0][warp] = lb;
+      red[1][warp] = lc;
+      red[2][warp] = sq;
+    }
+    __syncthreads();
     if (threadIdx.x == 0) {
-      row_part[i * 3 + 0] = red[0][0];
-      row_part[i * 3 + 1] = red[1][0];
-      row_part[i * 3 + 2] = red[2][0];
+      double a = 0.0, b = 0.0, c = 0.0;
+      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+        a += red[0][w];
+        b += red[1][w];
+        c += red[2][w];
+      }
+      row_part[i * 3 + 0] = a;
+      row_part[i * 3 + 1] = b;
+      row_part[i * 3 + 2] = c;
     }
   }
 }
@@ -163,7 +206,11 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   float* dW = X ? mem.as<float>() : nullptr;
   double* row_part = reinterpret_cast<double*>(mem.as<char>() + dW_bytes);
   double* gemm_part = row_part + M * 3;
-  const size_t smem = (size_t)N * sizeof(float);
+  const size_t smem = (size_t)N * sizeof(float) * ((W_hat ? 1 : 0) + (dW ? 1 : 0));
+  if (smem > (size_t)227 * 1024)
+    return fail(CRVQ_ERR_UNSUPPORTED,
+                "crvq_reconstruct_error: N = %lld channels need %zu bytes of shared memory per "
+                "row (227 KB available)", (long long)N, smem);
   if (smem > 48 * 1024)
     CRVQ_CUDA(cudaFuncSetAttribute(decode_row_kernel,
                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));

@@ -10,6 +10,7 @@
 #pragma once
 
 #include "common.cuh"
+#include "fixed_point.cuh"
 #include "kernels.h"
 
 namespace crvq {
@@ -17,10 +18,46 @@ namespace crvq {
 struct StatsView {
   int32_t* cnt;     // [G_cov][K]
   long long* bacc;  // [K][d]
-  double* scale;    // device scalar
+  double* scale;    // device scalar (followed by the maxima of the scale bound)
+  double* apart;    // [gsplit][kNA][K] fp64 partial sums of A_k over slices of the groups
   int64_t G_cov;
   int K;
+  int gsplit;
 };
+
+constexpr int kNA = 37;  // packed lower triangle of the 8 x 8 A_k (36 entries) + the count
+
+// Memory of the statistics of one codebook: cnt | bacc | scale + maxima (256 B) | apart, each
+// part 256-byte aligned. The groups are cut into gsplit slices of about 32 groups each.
+struct StatsLayout {
+  size_t cnt, bacc, head, apart, total;
+  int gsplit;
+};
+
+inline StatsLayout stats_layout(int64_t G_cov, int K) {
+  StatsLayout L;
+  const int64_t G = G_cov > 1 ? G_cov : 1;
+  L.gsplit = (int)(G < 32 * 32 ? (G + 31) / 32 : 32);
+  L.cnt = align_up((size_t)G * K * sizeof(int32_t), 256);
+  L.bacc = align_up((size_t)K * kD * sizeof(long long), 256);
+  L.head = 256;
+  L.apart = align_up((size_t)L.gsplit * kNA * K * sizeof(double), 256);
+  L.total = L.cnt + L.bacc + L.head + L.apart;
+  return L;
+}
+
+// Points st at the statistics laid out in `base` (stats_layout(G_cov, K).total bytes).
+inline void stats_bind(void* base, int64_t G_cov, int K, StatsView* st) {
+  const StatsLayout L = stats_layout(G_cov, K);
+  char* p = static_cast<char*>(base);
+  st->cnt = reinterpret_cast<int32_t*>(p);
+  st->bacc = reinterpret_cast<long long*>(p + L.cnt);
+  st->scale = reinterpret_cast<double*>(p + L.cnt + L.bacc);
+  st->apart = reinterpret_cast<double*>(p + L.cnt + L.bacc + L.head);
+  st->G_cov = G_cov;
+  st->K = K;
+  st->gsplit = L.gsplit;
+}
 
 // 2^e with e the largest integer such that n * bound * 2^e < 2^62.
 __host__ __device__ inline double stats_scale_for(double bound, int64_t n) {
@@ -67,15 +104,18 @@ __device__ __forceinline__ void stats_htau(const float* H, const float tau[kD], 
   }
 }
 
-__device__ __forceinline__ void stats_add(const StatsView& st, double scale, int64_t g, int k,
+// Exponent e of the fixed-point scale 2^e (an exact power of two, normal).
+__device__ __forceinline__ int stats_scale_exp(double scale) {
+  return (int)((__double_as_longlong(scale) >> 52) & 0x7ff) - 1023;
+}
+
+__device__ __forceinline__ void stats_add(const StatsView& st, int sexp, int64_t g, int k,
                                           const float q[kD]) {
   atomicAdd(&st.cnt[g * st.K + k], 1);
 #pragma unroll
-  for (int j = 0; j < kD; ++j) {
-    const long long v = __double2ll_rn((double)q[j] * scale);
+  for (int j = 0; j < kD; ++j)
     atomicAdd(reinterpret_cast<unsigned long long*>(&st.bacc[(int64_t)k * kD + j]),
-              (unsigned long long)v);
-  }
+              (unsigned long long)fix_rn(q[j], sexp));
 }
 
 // Solves A x = b for a symmetric positive definite 8 x 8 A given as its packed lower

@@ -1,7 +1,8 @@
 // Host side of the tcgen05 3xTF32 GEMM (tc_gemm.cuh) and the fixed-order reductions of its
 // split-K partial products. The tensor core accumulates fp32 with a small systematic
 // rounding bias per accumulation step, so K is cut into chunks of at most kKChunk and the
-// chunk partials are summed afterwards in fp64, in chunk order.
+// few chunk partials of an element are summed afterwards in fp32, in chunk order (a relative
+// error of a few u); the sums of squares over elements are reduced in fp64.
 #include <algorithm>
 
 #include "common.cuh"
@@ -14,15 +15,15 @@ namespace {
 
 constexpr int64_t kKChunk = 1024;
 
-// out[e] = scale * sum_c P[c * stride + e]  (fp64 sum, chunks in order)
+// out[e] = scale * sum_c P[c * stride + e]  (chunks in order)
 __global__ void __launch_bounds__(256)
 sum_partials_kernel(const float* __restrict__ P, int64_t count, int chunks, int64_t stride,
-                    double scale, float* __restrict__ out) {
+                    float scale, float* __restrict__ out) {
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < count;
        e += (int64_t)gridDim.x * blockDim.x) {
-    double s = 0.0;
-    for (int c = 0; c < chunks; ++c) s += (double)P[c * stride + e];
-    out[e] = (float)(s * scale);
+    float s = 0.f;
+    for (int c = 0; c < chunks; ++c) s += P[c * stride + e];
+    out[e] = s * scale;
   }
 }
 
@@ -31,13 +32,15 @@ __global__ void __launch_bounds__(256)
 sumsq_partials_kernel(const float* __restrict__ P, int64_t count, int chunks, int64_t stride,
                       double* __restrict__ part) {
   __shared__ double red[256];
-  double acc = 0.0;
+  float acc_f = 0.f;  // a few hundred non-negative terms per thread
+  double acc;
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < count;
        e += (int64_t)gridDim.x * blockDim.x) {
-    double s = 0.0;
-    for (int c = 0; c < chunks; ++c) s += (double)P[c * stride + e];
-    acc += s * s;
+    float s = 0.f;
+    for (int c = 0; c < chunks; ++c) s += P[c * stride + e];
+    acc_f = fmaf(s, s, acc_f);
   }
+  acc = (double)acc_f;
   red[threadIdx.x] = acc;
   __syncthreads();
   for (int w = 128; w > 0; w >>= 1) {
@@ -96,7 +99,7 @@ crvq_status launch_tc_syrk(const float* X, int64_t n, int64_t N, float* S, cudaS
     ProfScope ps("hessian_sum_partials", stream, (double)chunks * N * N * 4.0);
     const int blocks = (int)std::min<int64_t>(ceil_div(N * N, 256), 16 * sm_count());
     sum_partials_kernel<<<blocks, 256, 0, stream>>>(P, N * N, (int)chunks, N * N,
-                                                    1.0 / (double)n, S);
+                                                    (float)(1.0 / (double)n), S);
     CRVQ_LAUNCHED();
   }
   return CRVQ_OK;

@@ -4,9 +4,11 @@
 //   tau_v = t_v - sum over the other covering codebooks of C[code].
 //
 // Deterministic by construction, with no sort and no float atomics: cnt[g][k] are integer
-// counts, b_k is accumulated in 64-bit fixed point (stats.cuh), A_k is summed in fp64 in a
-// fixed order (one CTA per codeword, groups split over the threads, then a fixed reduction
-// tree), and the 8 x 8 system is solved by an fp64 Cholesky factorisation. The Lloyd encode
+// counts, b_k is accumulated in 64-bit fixed point (stats.cuh), A_k is summed as fp32 pairs in
+// a fixed order (partial sums over fixed slices of the groups, added in slice order), and the
+// 8 x 8 system is solved to fp64 accuracy by mixed-precision iterative refinement, one thread
+// per codeword. GB300's fp64 pipe is a small fraction of its fp32 rate, so none of this
+// arithmetic runs per element in fp64. The Lloyd encode
 // pass (encode.cu) accumulates the same statistics for the codes it writes.
 #include <algorithm>
 #include <cmath>
@@ -76,101 +78,271 @@ __global__ void stats_scale_kernel(const unsigned* __restrict__ maxbits, int n_c
   *scale = stats_scale_for(bound, n_members);
 }
 
+// Statistics of every covered vector from its current code. CTA (x, y): groups y,
+// y + gridDim.y, ..., rows x, x + gridDim.x, ... of each; with K <= kSmemStatsK the CTA sums its counts and fixed-point terms
+// in shared memory (integer atomics) and adds them to the global sums once; larger codebooks
+// add each vector's terms to the global sums directly. Integer sums: the order is immaterial.
+constexpr int kSmemStatsK = 256;
+
 __global__ void __launch_bounds__(256)
 accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsigned* err) {
+  __shared__ long long s_bacc[kSmemStatsK * kD];
+  __shared__ int s_cnt[kSmemStatsK];
   const CbView cw = cbs.cb[which];
-  const int64_t n = set.M * cw.G_cov;
-  const double scale = *st.scale;
-  for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < n;
-       v += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t i = v / cw.G_cov, g = v % cw.G_cov;
-    const int32_t k = cw.codes[i * cw.ld + g];
-    if (k < 0 || k >= cw.K) {
-      raise_error(err, ERRBIT_INDEX);
-      continue;
+  const int sexp = stats_scale_exp(*st.scale);
+  const bool smem = cw.K <= kSmemStatsK;
+  for (int64_t g = blockIdx.y; g < cw.G_cov; g += gridDim.y) {
+    if (smem) {
+      __syncthreads();  // the previous group's flush has read the sums
+      for (int e = threadIdx.x; e < kSmemStatsK * kD; e += blockDim.x) s_bacc[e] = 0;
+      for (int e = threadIdx.x; e < kSmemStatsK; e += blockDim.x) s_cnt[e] = 0;
+      __syncthreads();
     }
-    float tau[kD], q[kD];
-    stats_target(set, cbs, which, i, g, tau, err);
-    stats_htau(set.Hb + g * kD * kD, tau, q);
-    stats_add(st, scale, g, k, q);
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < set.M;
+         i += (int64_t)gridDim.x * blockDim.x) {
+      const int32_t k = cw.codes[i * cw.ld + g];
+      if (k < 0 || k >= cw.K) {
+        raise_error(err, ERRBIT_INDEX);
+        continue;
+      }
+      float tau[kD], q[kD];
+      stats_target(set, cbs, which, i, g, tau, err);
+      stats_htau(set.Hb + g * kD * kD, tau, q);
+      if (smem) {
+        atomicAdd(&s_cnt[k], 1);
+#pragma unroll
+        for (int j = 0; j < kD; ++j)
+          atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[k * kD + j]),
+                    (unsigned long long)fix_rn(q[j], sexp));
+      } else {
+        stats_add(st, sexp, g, k, q);
+      }
+    }
+    if (smem) {
+      __syncthreads();
+      for (int k = threadIdx.x; k < cw.K; k += blockDim.x) {
+        const int c = s_cnt[k];
+        if (c == 0) continue;
+        atomicAdd(&st.cnt[g * st.K + k], c);
+#pragma unroll
+        for (int j = 0; j < kD; ++j)
+          atomicAdd(reinterpret_cast<unsigned long long*>(&st.bacc[(int64_t)k * kD + j]),
+                    (unsigned long long)s_bacc[k * kD + j]);
+      }
+    }
   }
 }
 
-// One CTA per codeword: A_k = sum_g cnt[g][k] H_g in fp64 (groups strided over the threads,
-// then a fixed warp-shuffle + shared-memory tree), b_k from the fixed point, Cholesky solve.
-constexpr int kSolveThreads = 128;
+// Grid of accumulate_stats_kernel: one column of CTAs per group, enough rows per CTA that
+// the flush stays small, at least ~4 CTAs per SM overall.
+dim3 accumulate_grid(int64_t M, int64_t G_cov, int nsm) {
+  const int64_t want = std::max<int64_t>(1, ceil_div(4 * (int64_t)nsm, std::max<int64_t>(G_cov, 1)));
+  const int64_t rows_x = std::max<int64_t>(1, std::min<int64_t>(want, ceil_div(M, 1024)));
+  return dim3((unsigned)rows_x, (unsigned)std::min<int64_t>(std::max<int64_t>(G_cov, 1), 65535));
+}
 
-__global__ void __launch_bounds__(kSolveThreads)
-stats_solve_kernel(const float* __restrict__ Hb, int64_t G_cov, int K, StatsView st,
-                   const float* __restrict__ C_old, float* __restrict__ C_out,
-                   int32_t* __restrict__ counts_out, unsigned* err) {
-  __shared__ double part[kSolveThreads / 32][37];
+// A_k = sum_g cnt[g][k] H_g as partial sums over slices of the groups, without the fp64
+// pipe: every product cnt * H is split exactly into fp32 hi + lo (cnt < 2^24), and the sum is
+// kept as an unevaluated fp32 pair (Knuth's TwoSum for the high part, the low parts added),
+// about 2^-44 relative after a few thousand terms. CTA (kb, gs): lane = codeword 32 kb + lane
+// (coalesced counts), the groups of slice gs strided over the warps (H_g read once per warp,
+// the same address in every lane), then the warps' pairs added in fp64 in warp order. The
+// fixed assignment and order make the result identical on every run.
+constexpr int kGramWarps = 4;
+
+__global__ void __launch_bounds__(32 * kGramWarps)
+stats_gram_kernel(const float* __restrict__ Hb, StatsView st) {
+  __shared__ double red[kGramWarps - 1][kNA][32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int k = blockIdx.x; k < K; k += gridDim.x) {
-    double A[37];
+  const int K = st.K;
+  const int k = blockIdx.x * 32 + lane;
+  const int64_t gper = (st.G_cov + st.gsplit - 1) / st.gsplit;
+  const int64_t g0 = (int64_t)blockIdx.y * gper;
+  const int64_t g1 = min(st.G_cov, g0 + gper);
+  float hi[kNA - 1], lo[kNA - 1];
 #pragma unroll
-    for (int j = 0; j < 37; ++j) A[j] = 0.0;
-    for (int64_t g = threadIdx.x; g < G_cov; g += blockDim.x) {
-      const int c = st.cnt[g * K + k];
-      if (c == 0) continue;
-      A[36] += (double)c;
-      const float* H = Hb + g * kD * kD;
-      int q = 0;
+  for (int e = 0; e < kNA - 1; ++e) hi[e] = lo[e] = 0.f;
+  int count = 0;
+  for (int64_t g = g0 + warp; g < g1; g += kGramWarps) {
+    const int c = k < K ? st.cnt[g * K + k] : 0;
+    if (!__any_sync(0xffffffffu, c != 0)) continue;
+    const float* H = Hb + g * kD * kD;
+    const float fc = (float)c;  // exact: counts stay below 2^24
+    count += c;
+    int q = 0;
 #pragma unroll
-      for (int r = 0; r < kD; ++r)
+    for (int r = 0; r < kD; ++r)
 #pragma unroll
-        for (int cc = 0; cc <= r; ++cc) A[q++] += (double)c * (double)H[r * kD + cc];
-    }
-#pragma unroll
-    for (int j = 0; j < 37; ++j)
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) A[j] += __shfl_xor_sync(0xffffffffu, A[j], off);
-    __syncthreads();
-    if (lane == 0)
-      for (int j = 0; j < 37; ++j) part[warp][j] = A[j];
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      for (int w = 1; w < kSolveThreads / 32; ++w)
-        for (int j = 0; j < 37; ++j) A[j] += part[w][j];
-      const int64_t count = (int64_t)A[36];
-      if (counts_out) counts_out[k] = (int32_t)count;
-      bool keep = count == 0;
-      if (!keep) {
-        const double scale = *st.scale;
-        double b[kD], x[kD];
-        for (int j = 0; j < kD; ++j) b[j] = (double)st.bacc[(int64_t)k * kD + j] / scale;
-        if (cholesky_solve8(A, b, x)) {
-          for (int j = 0; j < kD; ++j) C_out[(int64_t)k * kD + j] = (float)x[j];
-        } else {
-          raise_error(err, ERRBIT_NUMERIC);
-          keep = true;
-        }
+      for (int cc = 0; cc <= r; ++cc, ++q) {
+        const float h = __ldg(H + r * kD + cc);
+        const float p = __fmul_rn(fc, h);
+        const float pe = fmaf(fc, h, -p);           // fc * h = p + pe exactly
+        const float sum = __fadd_rn(hi[q], p);       // TwoSum(hi, p) = sum + t exactly
+        const float bp = __fsub_rn(sum, hi[q]);
+        const float t = __fadd_rn(__fsub_rn(hi[q], __fsub_rn(sum, bp)), __fsub_rn(p, bp));
+        hi[q] = sum;
+        lo[q] = __fadd_rn(lo[q], __fadd_rn(t, pe));
       }
-      if (keep)
-        for (int j = 0; j < kD; ++j) C_out[(int64_t)k * kD + j] = C_old[(int64_t)k * kD + j];
-    }
   }
+  double A[kNA];
+#pragma unroll
+  for (int e = 0; e < kNA - 1; ++e) A[e] = (double)hi[e] + (double)lo[e];
+  A[kNA - 1] = (double)count;
+  if (warp > 0)
+#pragma unroll
+    for (int e = 0; e < kNA; ++e) red[warp - 1][e][lane] = A[e];
+  __syncthreads();
+  if (warp == 0 && k < K) {
+    for (int w = 0; w < kGramWarps - 1; ++w)
+#pragma unroll
+      for (int e = 0; e < kNA; ++e) A[e] += red[w][e][lane];
+#pragma unroll
+    for (int e = 0; e < kNA; ++e) st.apart[((int64_t)blockIdx.y * kNA + e) * K + k] = A[e];
+  }
+}
+
+// fp32 Cholesky factor of the packed lower triangle (false unless every pivot is positive),
+// and the solve L L^T x = b with it.
+__device__ inline bool chol8_f32(const float A[36], float L[36]) {
+  int q = 0;
+#pragma unroll
+  for (int r = 0; r < kD; ++r)
+#pragma unroll
+    for (int c = 0; c <= r; ++c, ++q) {
+      float s = A[q];
+#pragma unroll
+      for (int m = 0; m < c; ++m) s = fmaf(-L[r * (r + 1) / 2 + m], L[c * (c + 1) / 2 + m], s);
+      if (r == c) {
+        if (!(s > 0.f)) return false;
+        L[q] = sqrtf(s);
+      } else {
+        L[q] = s / L[c * (c + 1) / 2 + c];
+      }
+    }
+  return true;
+}
+
+__device__ inline void chol8_solve_f32(const float L[36], const float b[kD], float x[kD]) {
+  float y[kD];
+#pragma unroll
+  for (int r = 0; r < kD; ++r) {
+    float s = b[r];
+#pragma unroll
+    for (int m = 0; m < r; ++m) s = fmaf(-L[r * (r + 1) / 2 + m], y[m], s);
+    y[r] = s / L[r * (r + 1) / 2 + r];
+  }
+#pragma unroll
+  for (int r = kD - 1; r >= 0; --r) {
+    float s = y[r];
+#pragma unroll
+    for (int m = r + 1; m < kD; ++m) s = fmaf(-L[m * (m + 1) / 2 + r], x[m], s);
+    x[r] = s / L[r * (r + 1) / 2 + r];
+  }
+}
+
+// One thread per codeword: A_k = the slices' partial sums added in slice order, b_k from the
+// fixed point. The system is solved by mixed-precision iterative refinement: an fp32
+// Cholesky factor, then x += L^-T L^-1 (b - A x) with the residual in fp64 until the
+// correction is below 2^-40 of x (cond(A) u_32 < 1 makes each step gain about
+// -log2(cond(A) u_32) bits). A factor that fails or a refinement that does not settle falls
+// back to the fp64 Cholesky solve. Codewords without members keep their old value.
+__global__ void __launch_bounds__(32)
+stats_chol_kernel(StatsView st, const float* C_old, float* C_out, int32_t* __restrict__ counts_out,
+                  unsigned* err) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= st.K) return;
+  const int K = st.K;
+  double A[kNA];
+#pragma unroll
+  for (int e = 0; e < kNA; ++e) A[e] = 0.0;
+  for (int gs = 0; gs < st.gsplit; ++gs)
+#pragma unroll
+    for (int e = 0; e < kNA; ++e) A[e] += st.apart[((int64_t)gs * kNA + e) * K + k];
+  const int64_t count = (int64_t)A[36];
+  if (counts_out) counts_out[k] = (int32_t)count;
+  bool keep = count == 0;
+  float out[kD];
+  if (!keep) {
+    const double inv_scale = 1.0 / *st.scale;  // a power of two: exact
+    double b[kD], x[kD];
+#pragma unroll
+    for (int j = 0; j < kD; ++j) b[j] = (double)st.bacc[(int64_t)k * kD + j] * inv_scale;
+    float Af[36], Lf[36];
+#pragma unroll
+    for (int e = 0; e < 36; ++e) Af[e] = (float)A[e];
+    bool solved = false;
+    if (chol8_f32(Af, Lf)) {
+      float bf[kD], xf[kD];
+#pragma unroll
+      for (int j = 0; j < kD; ++j) bf[j] = (float)b[j];
+      chol8_solve_f32(Lf, bf, xf);
+#pragma unroll
+      for (int j = 0; j < kD; ++j) x[j] = (double)xf[j];
+      for (int it = 0; it < 6 && !solved; ++it) {
+        float rf[kD], dx[kD];
+#pragma unroll
+        for (int r = 0; r < kD; ++r) {
+          double s = b[r];
+#pragma unroll
+          for (int c = 0; c < kD; ++c) {
+            const double a = r >= c ? A[r * (r + 1) / 2 + c] : A[c * (c + 1) / 2 + r];
+            s = fma(-a, x[c], s);
+          }
+          rf[r] = (float)s;
+        }
+        chol8_solve_f32(Lf, rf, dx);
+        float xm = 0.f, dm = 0.f;
+#pragma unroll
+        for (int j = 0; j < kD; ++j) {
+          x[j] += (double)dx[j];
+          xm = fmaxf(xm, fabsf((float)x[j]));
+          dm = fmaxf(dm, fabsf(dx[j]));
+        }
+        solved = dm <= 9.094947e-13f * xm;  // 2^-40
+      }
+    }
+    if (!solved && !cholesky_solve8(A, b, x)) {
+      raise_error(err, ERRBIT_NUMERIC);
+      keep = true;
+    }
+    if (!keep)
+#pragma unroll
+      for (int j = 0; j < kD; ++j) out[j] = (float)x[j];
+  }
+  if (keep)
+#pragma unroll
+    for (int j = 0; j < kD; ++j) out[j] = C_old[(int64_t)k * kD + j];
+#pragma unroll
+  for (int j = 0; j < kD; ++j) C_out[(int64_t)k * kD + j] = out[j];
+}
+
+crvq_status launch_solve_kernels(const float* Hb, const StatsView& st, const float* C_old,
+                                 float* C_out, int32_t* counts, unsigned* err,
+                                 cudaStream_t stream) {
+  {
+    ProfScope ps("update_gram", stream, (double)st.G_cov * st.K);
+    stats_gram_kernel<<<dim3((unsigned)ceil_div(st.K, 32), (unsigned)st.gsplit), 32 * kGramWarps,
+                        0, stream>>>(Hb, st);
+    CRVQ_LAUNCHED();
+  }
+  ProfScope ps("update_solve", stream, (double)st.K);
+  stats_chol_kernel<<<(unsigned)ceil_div(st.K, 32), 32, 0, stream>>>(st, C_old, C_out, counts,
+                                                                     err);
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
 }
 
 }  // namespace
 
 crvq_status stats_alloc(Scratch& mem, int64_t G_cov, int K, StatsView* st, cudaStream_t s) {
-  const size_t cnt_bytes = align_up((size_t)std::max<int64_t>(G_cov, 1) * K * sizeof(int32_t), 256);
-  const size_t b_bytes = align_up((size_t)K * kD * sizeof(long long), 256);
-  const size_t max_bytes = 256;  // maxbits[2 + kMaxCodebooks] + scale
-  CRVQ_TRY(mem.alloc(cnt_bytes + b_bytes + max_bytes, s));
-  st->cnt = mem.as<int32_t>();
-  st->bacc = reinterpret_cast<long long*>(mem.as<char>() + cnt_bytes);
-  st->scale = reinterpret_cast<double*>(mem.as<char>() + cnt_bytes + b_bytes);
-  st->G_cov = G_cov;
-  st->K = K;
+  CRVQ_TRY(mem.alloc(stats_layout(G_cov, K).total, s));
+  stats_bind(mem.as<char>(), G_cov, K, st);
   return stats_zero(*st, s);
 }
 
 crvq_status stats_zero(const StatsView& st, cudaStream_t s) {
-  const size_t cnt_bytes = align_up((size_t)std::max<int64_t>(st.G_cov, 1) * st.K * sizeof(int32_t), 256);
-  const size_t b_bytes = align_up((size_t)st.K * kD * sizeof(long long), 256);
-  CRVQ_CUDA(cudaMemsetAsync(st.cnt, 0, cnt_bytes + b_bytes, s));
+  const StatsLayout L = stats_layout(st.G_cov, st.K);
+  CRVQ_CUDA(cudaMemsetAsync(st.cnt, 0, L.cnt + L.bacc, s));
   return CRVQ_OK;
 }
 
@@ -198,12 +370,7 @@ crvq_status launch_stats_solve(const SetView& set, const StatsView& st, const fl
                                float* C_out, int32_t* counts, cudaStream_t stream) {
   unsigned* err = nullptr;
   CRVQ_TRY(device_error_word(&err));
-  ProfScope ps("update_solve", stream, (double)st.K);
-  const int blocks = (int)std::min<int64_t>(st.K, 64 * sm_count());
-  stats_solve_kernel<<<blocks, kSolveThreads, 0, stream>>>(set.Hb, st.G_cov, st.K, st, C_old,
-                                                           C_out, counts, err);
-  CRVQ_LAUNCHED();
-  return CRVQ_OK;
+  return launch_solve_kernels(set.Hb, st, C_old, C_out, counts, err, stream);
 }
 
 crvq_status launch_update_codebook(const SetView& set, const CbList& cbs, int which,
@@ -219,8 +386,8 @@ crvq_status launch_update_codebook(const SetView& set, const CbList& cbs, int wh
   if (n > 0) {
     ProfScope ps("update_accumulate", stream, (double)n);
     const int nsm = sm_count();
-    accumulate_stats_kernel<<<(unsigned)std::min<int64_t>(ceil_div(n, 256), 16 * nsm), 256, 0,
-                              stream>>>(set, cbs, which, st, err);
+    accumulate_stats_kernel<<<accumulate_grid(set.M, cw.G_cov, nsm), 256, 0, stream>>>(
+        set, cbs, which, st, err);
     CRVQ_LAUNCHED();
   }
   return launch_stats_solve(set, st, cw.C, C_out, counts, stream);
@@ -234,10 +401,7 @@ namespace crvq {
 // (256-byte aligned, `bytes` long) holds cnt | bacc | scale + maxima, and `err` is the error
 // word the kernels report to. Returns CRVQ_ERR_UNSUPPORTED when the statistics of this
 // codebook do not fit in `bytes`.
-size_t update_scratch_bytes(int64_t G_cov, int K) {
-  return align_up((size_t)std::max<int64_t>(G_cov, 1) * K * sizeof(int32_t), 256) +
-         align_up((size_t)K * kD * sizeof(long long), 256) + 256;
-}
+size_t update_scratch_bytes(int64_t G_cov, int K) { return stats_layout(G_cov, K).total; }
 
 crvq_status launch_update_codebook_on(const SetView& set, const CbList& cbs, int which,
                                       float* C_out, int32_t* counts, void* scratch,
@@ -248,19 +412,14 @@ crvq_status launch_update_codebook_on(const SetView& set, const CbList& cbs, int
   if (need > bytes)
     return fail(CRVQ_ERR_UNSUPPORTED,
                 "statistics of this codebook need %zu bytes of scratch, the limit is %zu "
-                "(G_cov * K * 4 + K * 64 + 512 bytes)",
+                "(G_cov * K * 4 + K * 64 + 256 + gsplit * 296 * K bytes, 256-byte aligned)",
                 need, bytes);
-  const size_t cnt_bytes = align_up((size_t)std::max<int64_t>(cw.G_cov, 1) * cw.K * sizeof(int32_t), 256);
-  const size_t b_bytes = align_up((size_t)cw.K * kD * sizeof(long long), 256);
+  const StatsLayout L = stats_layout(cw.G_cov, cw.K);
   StatsView st;
-  st.cnt = static_cast<int32_t*>(scratch);
-  st.bacc = reinterpret_cast<long long*>(static_cast<char*>(scratch) + cnt_bytes);
-  st.scale = reinterpret_cast<double*>(static_cast<char*>(scratch) + cnt_bytes + b_bytes);
-  st.G_cov = cw.G_cov;
-  st.K = cw.K;
+  stats_bind(scratch, cw.G_cov, cw.K, &st);
   unsigned* maxbits = reinterpret_cast<unsigned*>(st.scale + 1);
   // The scratch keeps the previous call's contents: clear counts, sums and maxima.
-  CRVQ_CUDA(cudaMemsetAsync(scratch, 0, cnt_bytes + b_bytes + 256, stream));
+  CRVQ_CUDA(cudaMemsetAsync(scratch, 0, L.cnt + L.bacc + L.head, stream));
   const int nsm = sm_count();
   maxabs_kernel<<<(unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(n, 256), 4 * nsm)),
                   256, 0, stream>>>(set, cw.G_cov, cbs, which, maxbits);
@@ -269,14 +428,11 @@ crvq_status launch_update_codebook_on(const SetView& set, const CbList& cbs, int
                                           st.scale, err);
   CRVQ_LAUNCHED();
   if (n > 0) {
-    accumulate_stats_kernel<<<(unsigned)std::min<int64_t>(ceil_div(n, 256), 16 * nsm), 256, 0,
-                              stream>>>(set, cbs, which, st, err);
+    accumulate_stats_kernel<<<accumulate_grid(set.M, cw.G_cov, nsm), 256, 0, stream>>>(
+        set, cbs, which, st, err);
     CRVQ_LAUNCHED();
   }
-  stats_solve_kernel<<<(int)std::min<int64_t>(st.K, 64 * nsm), kSolveThreads, 0, stream>>>(
-      set.Hb, st.G_cov, st.K, st, cw.C, C_out, counts, err);
-  CRVQ_LAUNCHED();
-  return CRVQ_OK;
+  return launch_solve_kernels(set.Hb, st, cw.C, C_out, counts, err, stream);
 }
 
 }  // namespace crvq
