@@ -264,7 +264,8 @@ def main():
         step_ms.append(a.elapsed_time(b))
         scores += out.report["scores"]
     barrier()
-    argmin_stats = [k for k in P.crvq_profile_end() if k["name"] != "encode_argmin_fallback"]
+    argmin_stats = [k for k in P.crvq_profile_end()
+                    if k["name"] in ("encode_argmin", "encode_argmin_lloyd")]
     launches = P.crvq_launch_count() - launches0
     clk = clocks.stop()
     # per-kernel breakdown: one more step, untimed, every launch bracketed

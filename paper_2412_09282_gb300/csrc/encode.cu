@@ -267,6 +267,42 @@ __device__ __forceinline__ void build_b_row(const float* __restrict__ C, int K, 
   row[31] = 0u;
 }
 
+// cbmax[0] = max_k ||c_k||_1 (raised by 1e-6 relative), cbmax[1] = max_k,j |c_kj|: one CTA
+// of any size up to 1024 threads (maxima are order-free).
+__device__ void cbmax_block(const float* __restrict__ C, int K, float* __restrict__ cbmax) {
+  __shared__ float r1[32], r2[32];
+  float l1m = 0.f, cm = 0.f;
+  for (int k = threadIdx.x; k < K; k += blockDim.x) {
+    float c[kD];
+    load_vec(C + (int64_t)k * kD, c);
+    float l1 = 0.f;
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      l1 += fabsf(c[j]);
+      cm = fmaxf(cm, fabsf(c[j]));
+    }
+    l1m = fmaxf(l1m, l1);
+  }
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    l1m = fmaxf(l1m, __shfl_xor_sync(0xffffffffu, l1m, off));
+    cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, off));
+  }
+  if ((threadIdx.x & 31) == 0) {
+    r1[threadIdx.x >> 5] = l1m;
+    r2[threadIdx.x >> 5] = cm;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int w = 1; w < (int)((blockDim.x + 31) >> 5); ++w) {
+      l1m = fmaxf(l1m, r1[w]);
+      cm = fmaxf(cm, r2[w]);
+    }
+    cbmax[0] = l1m * (1.f + 1e-6f);
+    cbmax[1] = cm;
+  }
+}
+
 constexpr int kTcCols = 128;                     // codewords per chunk (MMA N)
 constexpr int kTcBTile = kTcCols * tcenc::kK * 4;  // 16 KB
 
@@ -275,10 +311,15 @@ constexpr int kTcBTile = kTcCols * tcenc::kK * 4;  // 16 KB
 // terms[(g - g_begin) K + k] = (n, Na, L1, 0) of codeword k in group g (codeword_terms).
 __global__ void __launch_bounds__(128)
 prep_b_kernel(SetView set, int64_t g_begin, int64_t G_range, const float* __restrict__ C,
-              int K, int nchunk, float uc, char* __restrict__ out, float4* __restrict__ terms) {
+              int K, int nchunk, float uc, char* __restrict__ out, float4* __restrict__ terms,
+              float* __restrict__ cbmax) {
+  if (blockIdx.x == gridDim.x - 1) {  // the last CTA: the codebook maxima
+    cbmax_block(C, K, cbmax);
+    return;
+  }
   const int64_t total = G_range * nchunk * (int64_t)kTcCols;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
-       e += (int64_t)gridDim.x * blockDim.x) {
+  const int64_t nth = (int64_t)(gridDim.x - 1) * blockDim.x;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total; e += nth) {
     const int row = (int)(e % kTcCols);
     const int64_t blk = e / kTcCols;  // g_rel * nchunk + chunk
     const int chunk = (int)(blk % nchunk);
@@ -296,13 +337,106 @@ prep_b_kernel(SetView set, int64_t g_begin, int64_t G_range, const float* __rest
   }
 }
 
-// A 128-thread CTA walks `tiles` consecutive row tiles of one group (thread = row = tensor-
-// memory lane), with a 128-column accumulator; three CTAs per SM. Codeword chunks of 128 come
-// from precomputed B images by bulk copy (bpre) or are built in place; with at most two chunks
-// they stay resident for all the CTA's tiles. Keys carry the column within a 32-column block in
-// their low 5 bits (2^-18 relative truncation); the block is tracked by the merge. The Lloyd
-// statistics of certified rows are summed in shared memory (integer atomics) and flushed once.
+// Exact scoring in unevaluated fp32 pairs ("double-float"): GB300's fp64 pipe is a small
+// fraction of its fp32 rate, so the few decisions that the certified bounds leave open are
+// settled with error-free transformations (Knuth's TwoSum, the FMA-based TwoProduct) on the
+// fp32 pipe instead. The residual r = t - sum of the fixed codewords is held exactly as
+// rh + rl; the err (r - c)^T H (r - c) comes out within a few 2^-48 of |r - c|^T |H| |r - c|,
+// far inside the near-tie margin at which fp64 itself stops deciding.
+namespace dfl {
+
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+  s = __fadd_rn(a, b);
+  const float bp = __fsub_rn(s, a);
+  e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bp)), __fsub_rn(b, bp));
+}
+
+// (rh + rl) = t - sum of the fixed codebooks' codewords covering g (codebook order).
+__device__ __forceinline__ void target(const SetView& set, const CbList& cbs, int n_fixed,
+                                       int64_t i, int64_t g, float rh[kD], float rl[kD],
+                                       unsigned* err) {
+  load_vec(set.T + i * set.ldT + g * kD, rh);
+#pragma unroll
+  for (int j = 0; j < kD; ++j) rl[j] = 0.f;
+  for (int s = 0; s < n_fixed; ++s) {
+    const CbView& cb = cbs.cb[s];
+    if (g >= cb.G_cov) continue;
+    const int32_t k = cb.codes[i * cb.ld + g];
+    if (!code_ok(k, cb.K, err)) continue;
+    float c[kD];
+    load_vec(cb.C + (int64_t)k * kD, c);
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      float sj, ej;
+      two_sum(rh[j], -c[j], sj, ej);
+      rh[j] = sj;
+      rl[j] = __fadd_rn(rl[j], ej);
+    }
+  }
+}
+
+// err = (r - c)^T H (r - c) as a normalised pair (eh, el), r = rh + rl.
+__device__ __forceinline__ void quad_err(const float rh[kD], const float rl[kD],
+                                         const float c[kD], const float* H, float& eh,
+                                         float& el) {
+  float dh[kD], dl[kD];
+#pragma unroll
+  for (int j = 0; j < kD; ++j) {
+    float e;
+    two_sum(rh[j], -c[j], dh[j], e);
+    dl[j] = __fadd_rn(rl[j], e);
+  }
+  float yh[kD], yl[kD];
+#pragma unroll
+  for (int b = 0; b < kD; ++b) yh[b] = yl[b] = 0.f;
+#pragma unroll
+  for (int a = 0; a < kD; ++a)
+#pragma unroll
+    for (int b = 0; b < kD; ++b) {
+      const float h = H[a * kD + b];
+      const float p = __fmul_rn(dh[a], h);
+      const float pe = __fmaf_rn(dh[a], h, -p);  // dh h = p + pe exactly
+      float s, t;
+      two_sum(yh[b], p, s, t);
+      yh[b] = s;
+      yl[b] = __fadd_rn(yl[b], __fadd_rn(t, __fmaf_rn(dl[a], h, pe)));
+    }
+  float sh = 0.f, sl = 0.f;
+#pragma unroll
+  for (int b = 0; b < kD; ++b) {
+    const float p = __fmul_rn(dh[b], yh[b]);
+    const float pe = __fmaf_rn(dh[b], yh[b], -p);
+    float s, t;
+    two_sum(sh, p, s, t);
+    sh = s;
+    sl = __fadd_rn(sl, __fadd_rn(t, __fmaf_rn(dh[b], yl[b], __fmaf_rn(dl[b], yh[b], pe))));
+  }
+  eh = __fadd_rn(sh, sl);
+  el = __fsub_rn(sl, __fsub_rn(eh, sh));
+}
+
+__device__ __forceinline__ bool less(float ah, float al, int ak, float bh, float bl, int bk) {
+  return ah < bh || (ah == bh && (al < bl || (al == bl && ak < bk)));
+}
+
+}  // namespace dfl
+
+// Arg-min over one codebook on the tensor cores. A 128-thread CTA walks `tiles` consecutive
+// row tiles of one group (thread = row = tensor-memory lane), with a 128-column accumulator;
+// three CTAs per SM, whose phases (A rows, MMA, epilogue, certificate) interleave on the SM.
+// Codeword chunks of 128 come from precomputed B images by bulk copy (bpre) or are built in
+// place; with at most two chunks they stay resident for all the CTA's tiles. Keys carry the
+// column within a 32-column block in their low 5 bits (2^-18 relative truncation); the block
+// is tracked by the merge. Rows the bounds do not certify go to the flag list (decided exactly
+// by argmin_exact_kernel). The Lloyd statistics of certified rows are summed in shared memory
+// (integer atomics, [component][code] so that a warp's lanes hit spread banks) and flushed
+// once.
 constexpr int kTcSmemStatsK = 256;  // codebooks up to this size aggregate statistics in smem
+
+// dynamic shared memory of argmin_tc_kernel: A tile, two B chunks, statistics, H r, alignment
+constexpr size_t kArgminSmem = (size_t)tcenc::kATile + 2 * (size_t)kTcBTile +
+                               (size_t)kTcSmemStatsK * (kD * 8 + 4) + tcenc::kRows * kD * 4 +
+                               1024;
 
 __global__ void __launch_bounds__(128, 3)
 argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
@@ -312,11 +446,11 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
                  unsigned* err) {
   using namespace tcenc;
   extern __shared__ __align__(1024) char smem_raw[];
-  char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                       ~(uintptr_t)1023);
+  // 1024-byte aligned base, derived from the shared array (keeps the shared address space)
+  char* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
   char* Atile = smem;                  // 16 KB
   char* Bbuf = smem + kATile;          // 2 x 16 KB
-  long long* s_bacc = reinterpret_cast<long long*>(Bbuf + 2 * kTcBTile);  // [256][8]
+  long long* s_bacc = reinterpret_cast<long long*>(Bbuf + 2 * kTcBTile);  // [8][256]
   int* s_cnt = reinterpret_cast<int*>(s_bacc + kTcSmemStatsK * kD);       // [256]
   float* sQ = reinterpret_cast<float*>(s_cnt + kTcSmemStatsK);            // [128][8] H r
   __shared__ float sH[kD * kD];
@@ -369,10 +503,11 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   const int64_t row_tiles = (set.M + kRows - 1) / kRows;
   const int my_tiles = (int)min((int64_t)tiles, row_tiles - (int64_t)blockIdx.x * tiles);
   // Chunk uses are numbered u = t * nchunk + c. Resident chunks sit in buffer c; otherwise use u
-  // reads buffer u & 1, and the copy for use u + 2 starts when use u is done. Bulk copies
-  // issued / waited per buffer (the same count in every thread).
+  // reads buffer u & 1, and the copy for use u + 2 starts when use u is done. At most one copy
+  // per buffer is outstanding; every thread tracks the same state.
   const int n_uses = resident ? nchunk : my_tiles * nchunk;
-  int b_issued[2] = {0, 0}, b_waited[2] = {0, 0};
+  // per buffer (bit b): a copy outstanding, and the parity of its wait (registers, not arrays)
+  uint32_t b_pend = 0, b_par = 0;
   auto fetch = [&](int u) {  // chunk u % nchunk into buffer u & 1 (bimg only)
     const int b = u & 1;
     if (tid == 0) {
@@ -381,7 +516,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
                         bimg + (size_t)(u % nchunk) * kTcBTile, kTcBTile,
                         tc::smem_u32(&bar_b[b]));
     }
-    ++b_issued[b];
+    b_pend |= 1u << b;
   };
   if (bimg) {
     fetch(0);
@@ -450,9 +585,10 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       const int buf = resident ? c : (u & 1);
       char* Bt = Bbuf + buf * kTcBTile;
       if (bimg) {
-        if (b_waited[buf] < b_issued[buf]) {
-          if (ok) ok = tc::mbar_wait(tc::smem_u32(&bar_b[buf]), (uint32_t)(b_waited[buf] & 1), err);
-          ++b_waited[buf];
+        if ((b_pend >> buf) & 1u) {
+          if (ok) ok = tc::mbar_wait(tc::smem_u32(&bar_b[buf]), (b_par >> buf) & 1u, err);
+          b_par ^= 1u << buf;
+          b_pend &= ~(1u << buf);
         }
       } else if (!resident || t == 0) {
         uint32_t v[kK];
@@ -490,10 +626,10 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       const uint32_t base = tmem + ((uint32_t)(warp * 32) << 16);
 #pragma unroll
       for (int rnd = 0; rnd < 2; ++rnd) {
-        uint32_t v0[32], v1[32];
-        tc::tmem_ld32_nowait(base + 64 * rnd, v0);
-        tc::tmem_ld32_nowait(base + 64 * rnd + 32, v1);
-        tc::tmem_wait_ld();
+        uint32_t v[64];
+        tc::tmem_ld64_wait(base + 64 * rnd, v);
+        const uint32_t* v0 = v;
+        const uint32_t* v1 = v + 32;
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
           const uint32_t k0 = (v0[j] & 0xffffffe0u) | (uint32_t)j;
@@ -568,7 +704,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
           atomicAdd(&s_cnt[j], 1);
 #pragma unroll
           for (int p = 0; p < kD; ++p)
-            atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[j * kD + p]),
+            atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[p * kTcSmemStatsK + j]),
                       (unsigned long long)fix_rn(q[p], sexp));
         } else {
           stats_add(st, sexp, g, j, q);
@@ -578,9 +714,8 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   }
   // After a timeout: let copies still in flight into this CTA's shared memory land (bounded).
   for (int b = 0; b < 2; ++b)
-    while (b_waited[b] < b_issued[b]) {
-      tc::mbar_wait(tc::smem_u32(&bar_b[b]), (uint32_t)(b_waited[b] & 1), err);
-      ++b_waited[b];
+    if ((b_pend >> b) & 1u) {
+      tc::mbar_wait(tc::smem_u32(&bar_b[b]), (b_par >> b) & 1u, err);
     }
   __syncthreads();
   if (smem_stats) {  // one flush of this CTA's statistics (integer sums: order-free)
@@ -591,7 +726,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
 #pragma unroll
       for (int p = 0; p < kD; ++p)
         atomicAdd(reinterpret_cast<unsigned long long*>(&st.bacc[(int64_t)k * kD + p]),
-                  (unsigned long long)s_bacc[k * kD + p]);
+                  (unsigned long long)s_bacc[p * kTcSmemStatsK + k]);
     }
   }
   tc::tc_fence_before();
@@ -599,146 +734,129 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   if (warp == 0) tc::tmem_dealloc(tmem, kTcCols);
 }
 
-// cbmax[0] = max_k ||c_k||_1, cbmax[1] = max_k,j |c_kj| (one CTA; maxima are order-free).
-__global__ void __launch_bounds__(256)
-cbmax_kernel(const float* __restrict__ C, int K, float* __restrict__ cbmax) {
-  __shared__ float r1[256], r2[256];
-  float l1m = 0.f, cm = 0.f;
-  for (int k = threadIdx.x; k < K; k += blockDim.x) {
-    float c[kD];
-    load_vec(C + (int64_t)k * kD, c);
-    float l1 = 0.f;
-#pragma unroll
-    for (int j = 0; j < kD; ++j) {
-      l1 += fabsf(c[j]);
-      cm = fmaxf(cm, fabsf(c[j]));
-    }
-    l1m = fmaxf(l1m, l1);
-  }
-  r1[threadIdx.x] = l1m;
-  r2[threadIdx.x] = cm;
-  __syncthreads();
-  for (int w = 128; w > 0; w >>= 1) {
-    if ((int)threadIdx.x < w) {
-      r1[threadIdx.x] = fmaxf(r1[threadIdx.x], r1[threadIdx.x + w]);
-      r2[threadIdx.x] = fmaxf(r2[threadIdx.x], r2[threadIdx.x + w]);
-    }
-    __syncthreads();
-  }
-  if (threadIdx.x == 0) {
-    cbmax[0] = r1[0] * (1.f + 1e-6f);
-    cbmax[1] = r2[0];
-  }
-}
-
-// Fallback: one warp per flagged vector. A first sweep takes U = the smallest fp32 upper
-// bound s_k + Et_k over the codebook (and the fast pass's threshold); every codeword whose
-// lower bound s_k - Et_k is at most U is a candidate (the exact arg-min always is: its err
-// is at most U). Candidates are queued in shared memory and re-scored in fp64 one per lane,
-// so the fp64 work of a warp is one pass per 32 candidates; the smallest fp64 err wins (ties
-// to the smaller index). Adds the statistics of the decided code when requested.
-__global__ void __launch_bounds__(kThreads)
-argmin_fallback_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs,
-                       int n_fixed, int s_idx, int32_t* __restrict__ out_code,
-                       int64_t out_ld, int64_t out_g0, FlagList flags, StatsView st,
-                       const float4* __restrict__ terms, unsigned* err) {
-  __shared__ int queue[kThreads / 32][32];
-  const int lane = threadIdx.x & 31;
-  int* q = queue[threadIdx.x >> 5];
-  const int64_t warp = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int64_t nwarps = ((int64_t)gridDim.x * blockDim.x) >> 5;
+// Exact decision for the rows the arg-min pass flagged: one CTA per flagged vector. The
+// threads stride over the codebook for U = min(fast-pass threshold, smallest fp32 upper
+// bound); every codeword whose fp32 lower bound is at most U is a candidate (the exact
+// arg-min always is) and is re-scored exactly in fp32 pairs (dfl) by one thread; the
+// smallest (err, index) wins. Adds the statistics of the decided code when requested.
+__global__ void __launch_bounds__(128)
+argmin_exact_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs, int n_fixed,
+                    int s_idx, int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
+                    FlagList flags, StatsView st, const float4* __restrict__ terms,
+                    unsigned* err) {
+  __shared__ float sH[kD * kD];
+  __shared__ float redf[4];
+  __shared__ int cand[256];
+  __shared__ int ncand;
+  __shared__ float bh_s[4], bl_s[4];
+  __shared__ int bk_s[4];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const unsigned cnt = min((unsigned long long)*flags.count, (unsigned long long)flags.cap);
-  if (flags.total && blockIdx.x == 0 && threadIdx.x == 0) atomicAdd(flags.total, cnt);
+  if (flags.total && blockIdx.x == 0 && tid == 0) atomicAdd(flags.total, cnt);
   const CbView cw = cbs.cb[s_idx];
   const float cmul = bound_mult(n_fixed);
-  const unsigned lt_mask = (1u << lane) - 1u;
-  for (int64_t f = warp; f < cnt; f += nwarps) {
+  for (unsigned f = blockIdx.x; f < cnt; f += gridDim.x) {
     const int64_t vi = flags.vec[f];
-    const int64_t i = vi / G_range, g = g_begin + vi % G_range;
+    const int64_t i = vi / G_range, grel = vi % G_range, g = g_begin + grel;
     const float thr = flags.thr[f];
-    const float* H = set.Hb + g * kD * kD;
-    float r[kD], a[kD], m2q[kD], pmax;
-    target32(set, cbs, n_fixed, i, g, r, a, err);
-    vector_terms(r, a, H, m2q, pmax);
+    __syncthreads();
+    if (tid < kD * kD) sH[tid] = set.Hb[g * kD * kD + tid];
+    if (tid == 0) ncand = 0;
+    __syncthreads();
+    float rv[kD], av[kD], m2q[kD], pmax;
+    target32(set, cbs, n_fixed, i, g, rv, av, err);
+    vector_terms(rv, av, sH, m2q, pmax);
     const float nbeta = -2.f * kU * cmul * pmax;
-    double r64[kD];
-    target64(set, cbs, n_fixed, i, g, r64, err);
-    const float4* gterms = terms ? terms + (g - g_begin) * cw.K : nullptr;
-    auto terms_of = [&](int k, const float c[kD], float& n, float& na, float& l1) {
-      if (gterms) {
-        const float4 t = gterms[k];
-        n = t.x;
+    const float4* gt = terms ? terms + grel * cw.K : nullptr;
+    auto terms_of = [&](int k, const float cv[kD], float& nn, float& na, float& l1) {
+      if (gt) {
+        const float4 t = gt[k];
+        nn = t.x;
         na = t.y;
         l1 = t.z;
       } else {
-        codeword_terms(c, H, n, na, l1);
+        codeword_terms(cv, sH, nn, na, l1);
       }
     };
     float U = thr;
-    for (int k = lane; k < cw.K; k += 32) {
-      float c[kD], n, na, l1;
-      load_vec(cw.C + (int64_t)k * kD, c);
-      terms_of(k, c, n, na, l1);
-      U = fminf(U, up_from(n, na, l1, c, m2q, pmax, cmul));
+    for (int k = tid; k < cw.K; k += blockDim.x) {
+      float cv[kD], nn, na, l1;
+      load_vec(cw.C + (int64_t)k * kD, cv);
+      terms_of(k, cv, nn, na, l1);
+      U = fminf(U, up_from(nn, na, l1, cv, m2q, pmax, cmul));
     }
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) U = fminf(U, __shfl_xor_sync(0xffffffffu, U, off));
-    double best = INFINITY;
-    int bestk = 0x7fffffff;
-    int qn = 0;  // queued candidates (the same in every lane)
-    auto drain = [&]() {
-      __syncwarp();
-      if (lane < qn) {
-        const int k = q[lane];
-        const double e = quad_err64(r64, cw.C + (int64_t)k * kD, H);
-        if (e < best || (e == best && k < bestk)) {
-          best = e;
-          bestk = k;
+    for (int o = 16; o > 0; o >>= 1) U = fminf(U, __shfl_xor_sync(0xffffffffu, U, o));
+    if (lane == 0) redf[warp] = U;
+    __syncthreads();
+    U = fminf(fminf(redf[0], redf[1]), fminf(redf[2], redf[3]));
+    float rh[kD], rl[kD];
+    dfl::target(set, cbs, n_fixed, i, g, rh, rl, err);
+    float bh = INFINITY, bl = 0.f;
+    int bk = 0x7fffffff;
+    for (int k0 = 0; k0 < cw.K; k0 += 256) {
+      for (int k = k0 + tid; k < min(cw.K, k0 + 256); k += blockDim.x) {
+        float cv[kD], nn, na, l1;
+        load_vec(cw.C + (int64_t)k * kD, cv);
+        terms_of(k, cv, nn, na, l1);
+        if (low_from(nn, na, l1, cv, m2q, nbeta, cmul) <= U) cand[atomicAdd(&ncand, 1)] = k;
+      }
+      __syncthreads();
+      const int nc = ncand;
+      for (int q = tid; q < nc; q += blockDim.x) {
+        const int k = cand[q];
+        float cv[kD], eh, el;
+        load_vec(cw.C + (int64_t)k * kD, cv);
+        dfl::quad_err(rh, rl, cv, sH, eh, el);
+        if (dfl::less(eh, el, k, bh, bl, bk)) {
+          bh = eh;
+          bl = el;
+          bk = k;
         }
       }
-      __syncwarp();
-      qn = 0;
-    };
-    for (int k0 = 0; k0 < cw.K; k0 += 32) {
-      const int k = k0 + lane;
-      bool cand = false;
-      if (k < cw.K) {
-        float c[kD], n, na, l1;
-        load_vec(cw.C + (int64_t)k * kD, c);
-        terms_of(k, c, n, na, l1);
-        cand = low_from(n, na, l1, c, m2q, nbeta, cmul) <= U;
-      }
-      const unsigned m = __ballot_sync(0xffffffffu, cand);
-      const int n = __popc(m);
-      if (qn + n > 32) drain();
-      if (cand) q[qn + __popc(m & lt_mask)] = k;
-      qn += n;
+      __syncthreads();
+      if (tid == 0) ncand = 0;
+      __syncthreads();
     }
-    drain();
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const double ob = __shfl_xor_sync(0xffffffffu, best, off);
-      const int ok = __shfl_xor_sync(0xffffffffu, bestk, off);
-      if (ob < best || (ob == best && ok < bestk)) {
-        best = ob;
-        bestk = ok;
+    for (int o = 16; o > 0; o >>= 1) {
+      const float oh = __shfl_xor_sync(0xffffffffu, bh, o);
+      const float ol = __shfl_xor_sync(0xffffffffu, bl, o);
+      const int ok = __shfl_xor_sync(0xffffffffu, bk, o);
+      if (dfl::less(oh, ol, ok, bh, bl, bk)) {
+        bh = oh;
+        bl = ol;
+        bk = ok;
       }
     }
     if (lane == 0) {
-      if (bestk == 0x7fffffff) {
+      bh_s[warp] = bh;
+      bl_s[warp] = bl;
+      bk_s[warp] = bk;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      for (int w = 1; w < 4; ++w)
+        if (dfl::less(bh_s[w], bl_s[w], bk_s[w], bh, bl, bk)) {
+          bh = bh_s[w];
+          bl = bl_s[w];
+          bk = bk_s[w];
+        }
+      if (bk == 0x7fffffff) {
         raise_error(err, ERRBIT_NUMERIC);  // no candidate: non-finite scores
       } else {
-        out_code[i * out_ld + (g - out_g0)] = bestk;
+        out_code[i * out_ld + (g - out_g0)] = bk;
         if (st.cnt) {
-          float qv[kD];
+          float q[kD];
 #pragma unroll
-          for (int p = 0; p < kD; ++p) qv[p] = -0.5f * m2q[p];
-          stats_add(st, stats_scale_exp(*st.scale), g, bestk, qv);
+          for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[p];
+          stats_add(st, stats_scale_exp(*st.scale), g, bk, q);
         }
       }
     }
   }
 }
+
 
 // --------------------------------------------------------------------------- beam stages
 // Hypotheses of a vector: up to B partial tuples (codes of the first s+1 searched codebooks)
@@ -1300,16 +1418,6 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     }
     return CRVQ_OK;
   }
-  Scratch flag_mem;
-  const size_t fl_bytes = (size_t)nvec * (sizeof(int64_t) + sizeof(float)) + 256;
-  CRVQ_TRY(flag_mem.alloc(fl_bytes, stream));
-  FlagList fl;
-  fl.count = flag_mem.as<unsigned>();
-  fl.vec = reinterpret_cast<int64_t*>(flag_mem.as<char>() + 256);
-  fl.thr = reinterpret_cast<float*>(fl.vec + nvec);
-  fl.cap = nvec;
-  fl.total = ex.flag_total;
-
   if (sd.S == 1) {
     // Arg-min over one codebook (the k-means assignment step). Written in place unless the
     // old code may be kept, in which case into a scratch tuple buffer that the finalize step
@@ -1327,63 +1435,67 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     }
     StatsView st{};
     if (ex.stats && !keep_if_better) st = *ex.stats;
-    CRVQ_CUDA(cudaMemsetAsync(fl.count, 0, sizeof(unsigned), stream));
-    float* cbmax = reinterpret_cast<float*>(flag_mem.as<char>() + 128);
-    {
-      ProfScope pc("encode_cbmax", stream, 0.0);
-      cbmax_kernel<<<1, 256, 0, stream>>>(cw.C, cw.K, cbmax);
-      CRVQ_LAUNCHED();
-    }
-    // The codebook's B images per group (when they fit in 256 MB) and its per-group terms
-    // (n, Na, L1), read by the arg-min pass and its fallback.
+    // Groups in sub-ranges whose B images (the codebook's tensor-core operand per group) take
+    // at most 256 MB; per sub-range: images + per-group codeword terms (prep_b, which also
+    // writes the codebook maxima), the arg-min pass, and the exact decision of flagged rows.
     const int nchunk = (int)ceil_div(cw.K, kTcCols);
-    const size_t bbytes = (size_t)G_range * nchunk * kTcBTile;
-    const size_t tbytes = align_up((size_t)G_range * cw.K * sizeof(float4), 256);
+    const int64_t per_group = (int64_t)nchunk * kTcBTile;
+    const int64_t G_sub = std::max<int64_t>(1, std::min<int64_t>(G_range, (int64_t(256) << 20) /
+                                                                              per_group));
+    const size_t bbytes = (size_t)G_sub * per_group;
+    const size_t tbytes = align_up((size_t)G_sub * cw.K * sizeof(float4), 256);
+    const size_t fbytes = align_up((size_t)set.M * G_sub * (sizeof(int64_t) + sizeof(float)), 256);
     Scratch bmem;
-    const char* bpre = nullptr;
-    const float4* terms = nullptr;
-    if (bbytes <= (size_t(256) << 20)) {
-      CRVQ_TRY(bmem.alloc(bbytes + tbytes, stream));
-      const float uc = kU * (tcenc::kCmul + 4.f * n_fixed);
-      ProfScope pb("encode_prep_b", stream, (double)G_range * nchunk * kTcCols);
-      const int64_t rows = (int64_t)G_range * nchunk * kTcCols;
-      float4* tout = reinterpret_cast<float4*>(bmem.as<char>() + bbytes);
-      prep_b_kernel<<<(unsigned)std::min<int64_t>(ceil_div(rows, 128), 16 * nsm), 128, 0,
-                      stream>>>(set, g_begin, G_range, cw.C, cw.K, nchunk, uc, bmem.as<char>(),
-                                tout);
-      CRVQ_LAUNCHED();
-      bpre = bmem.as<char>();
-      terms = tout;
-    }
-    {
-      // 128-row tiles, three CTAs per SM (128 tensor-memory columns each)
-      const size_t smem = (size_t)tcenc::kATile + 2 * (size_t)kTcBTile +
-                          (size_t)kTcSmemStatsK * (kD * 8 + 4) + tcenc::kRows * kD * 4 + 1024;
-      // row tiles per CTA: about eight waves of three CTAs per SM (a fine-grained tail),
-      // each CTA reusing its group's resident codebook operand over several tiles
-      const int64_t row_tiles = ceil_div(set.M, tcenc::kRows);
-      const int64_t want_ctas = 24 * (int64_t)nsm;
-      const int64_t per_group = std::max<int64_t>(1, want_ctas / std::max<int64_t>(1, G_range));
-      const int tiles = (int)std::max<int64_t>(1, ceil_div(row_tiles, per_group));
-      dim3 grid((unsigned)ceil_div(row_tiles, tiles), (unsigned)G_range);
-      ProfScope ps(st.cnt ? "encode_argmin_lloyd" : "encode_argmin", stream,
-                   (double)nvec * cw.K);
-      CRVQ_TRY(set_smem_attr(argmin_tc_kernel, smem));
-      argmin_tc_kernel<<<grid, 128, smem, stream>>>(set, g_begin, cbs, n_fixed, s_idx, out,
-                                                    out_ld, out_g0, fl, st, cbmax, bpre, terms,
-                                                    tiles, err);
-      CRVQ_LAUNCHED();
-    }
-    {
-      ProfScope ps2("encode_argmin_fallback", stream, 0.0);
-      argmin_fallback_kernel<<<4 * nsm, kThreads, 0, stream>>>(set, g_begin, G_range, cbs,
-                                                               n_fixed, s_idx, out, out_ld,
-                                                               out_g0, fl, st, terms, err);
-      CRVQ_LAUNCHED();
+    CRVQ_TRY(bmem.alloc(256 + bbytes + tbytes + 256 + fbytes, stream));
+    float* cbmax = bmem.as<float>();
+    char* bimg = bmem.as<char>() + 256;
+    float4* tout = reinterpret_cast<float4*>(bimg + bbytes);
+    FlagList fl;
+    fl.count = reinterpret_cast<unsigned*>(bmem.as<char>() + 256 + bbytes + tbytes);
+    fl.vec = reinterpret_cast<int64_t*>(bmem.as<char>() + 256 + bbytes + tbytes + 256);
+    fl.cap = set.M * G_sub;
+    fl.thr = reinterpret_cast<float*>(fl.vec + fl.cap);
+    fl.total = ex.flag_total;
+    const float uc = kU * (tcenc::kCmul + 4.f * n_fixed);
+    CRVQ_TRY(set_smem_attr(argmin_tc_kernel, kArgminSmem));
+    for (int64_t gs = g_begin; gs < g_begin + G_range; gs += G_sub) {
+      const int64_t gn = std::min<int64_t>(G_sub, g_begin + G_range - gs);
+      const int64_t nv = set.M * gn;
+      fl.cap = nv;
+      fl.thr = reinterpret_cast<float*>(fl.vec + nv);
+      CRVQ_CUDA(cudaMemsetAsync(fl.count, 0, sizeof(unsigned), stream));
+      {
+        ProfScope pb("encode_prep_b", stream, (double)gn * nchunk * kTcCols);
+        const int64_t rows = gn * nchunk * kTcCols;
+        prep_b_kernel<<<(unsigned)std::min<int64_t>(ceil_div(rows, 128), 16 * nsm) + 1, 128, 0,
+                        stream>>>(set, gs, gn, cw.C, cw.K, nchunk, uc, bimg, tout, cbmax);
+        CRVQ_LAUNCHED();
+      }
+      {
+        // row tiles per CTA: about eight waves of three CTAs per SM (a fine-grained tail),
+        // each CTA reusing its group's resident codebook operand over several tiles
+        const int64_t row_tiles = ceil_div(set.M, tcenc::kRows);
+        const int64_t want_ctas = 24 * (int64_t)nsm;
+        const int64_t per_group = std::max<int64_t>(1, want_ctas / std::max<int64_t>(1, gn));
+        const int tiles = (int)std::max<int64_t>(1, ceil_div(row_tiles, per_group));
+        const dim3 grid((unsigned)ceil_div(row_tiles, tiles), (unsigned)gn);
+        ProfScope ps(st.cnt ? "encode_argmin_lloyd" : "encode_argmin", stream,
+                     (double)nv * cw.K);
+        argmin_tc_kernel<<<grid, 128, kArgminSmem, stream>>>(set, gs, cbs, n_fixed, s_idx, out,
+                                                             out_ld, out_g0, fl, st, cbmax,
+                                                             bimg, tout, tiles, err);
+        CRVQ_LAUNCHED();
+      }
+      {
+        ProfScope pf("encode_argmin_exact", stream, 0.0);
+        argmin_exact_kernel<<<(unsigned)std::min<int64_t>(nv, 16 * nsm), 128, 0, stream>>>(
+            set, gs, gn, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, tout, err);
+        CRVQ_LAUNCHED();
+      }
     }
     if (ex.scores) *ex.scores += (double)nvec * cw.K;
-    ProfScope ps3("encode_finalize", stream, 0.0);
     if (keep_if_better) {
+      ProfScope ps3("encode_finalize", stream, 0.0);
       StageDesc one = sd;
       one.B = 1;
       one.Bs = 1;
@@ -1391,12 +1503,23 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
                                                            one, out, true, vec_err, err);
       CRVQ_LAUNCHED();
     } else if (vec_err) {
+      ProfScope ps3("encode_finalize", stream, 0.0);
       residual_err_kernel<<<fin_blocks, 128, 0, stream>>>(set, g_begin, G_range, cbs, vec_err,
                                                           err);
       CRVQ_LAUNCHED();
     }
     return CRVQ_OK;
   }
+
+  Scratch flag_mem;
+  const size_t fl_bytes = (size_t)nvec * (sizeof(int64_t) + sizeof(float)) + 256;
+  CRVQ_TRY(flag_mem.alloc(fl_bytes, stream));
+  FlagList fl;
+  fl.count = flag_mem.as<unsigned>();
+  fl.vec = reinterpret_cast<int64_t*>(flag_mem.as<char>() + 256);
+  fl.thr = reinterpret_cast<float*>(fl.vec + nvec);
+  fl.cap = nvec;
+  fl.total = ex.flag_total;
 
   // Beam over S >= 2 stages: stage kernels over double-buffered hypothesis arrays.
   Scratch hyp_mem;

@@ -113,8 +113,8 @@ struct GemmArgs {
 
 __global__ void __launch_bounds__(kThreads, 1) gemm3xtf32_kernel(GemmArgs a) {
   extern __shared__ __align__(1024) char smem_raw[];
-  char* smem = reinterpret_cast<char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
-                                       ~(uintptr_t)1023);
+  // 1024-byte aligned base, derived from the shared array (keeps the shared address space)
+  char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kStages);
   __shared__ double red[kThreads];

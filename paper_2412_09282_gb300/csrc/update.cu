@@ -86,7 +86,8 @@ constexpr int kSmemStatsK = 256;
 
 __global__ void __launch_bounds__(256)
 accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsigned* err) {
-  __shared__ long long s_bacc[kSmemStatsK * kD];
+  __shared__ long long s_bacc[kD * kSmemStatsK];  // [component][code]: lanes of a warp
+                                                  // adding one component hit spread banks
   __shared__ int s_cnt[kSmemStatsK];
   const CbView cw = cbs.cb[which];
   const int sexp = stats_scale_exp(*st.scale);
@@ -112,7 +113,7 @@ accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsign
         atomicAdd(&s_cnt[k], 1);
 #pragma unroll
         for (int j = 0; j < kD; ++j)
-          atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[k * kD + j]),
+          atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[j * kSmemStatsK + k]),
                     (unsigned long long)fix_rn(q[j], sexp));
       } else {
         stats_add(st, sexp, g, k, q);
@@ -127,7 +128,7 @@ accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsign
 #pragma unroll
         for (int j = 0; j < kD; ++j)
           atomicAdd(reinterpret_cast<unsigned long long*>(&st.bacc[(int64_t)k * kD + j]),
-                    (unsigned long long)s_bacc[k * kD + j]);
+                    (unsigned long long)s_bacc[j * kSmemStatsK + k]);
       }
     }
   }
