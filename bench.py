@@ -52,9 +52,10 @@ def schedule_scores(cfg, M, N):
     return float(s)
 
 
-# dram__bytes_read.sum + dram__bytes_write.sum of one arg-min launch (ncu, a Lloyd pass of
-# the c2 workload; null whenever the kernel has changed since the counters were taken)
-ARGMIN_TRAFFIC = None
+# dram__bytes_read.sum + dram__bytes_write.sum of one arg-min launch (ncu --set full, a Lloyd
+# pass over the base codebook of the c2 workload: 86.7 MB read + 5.3 MB written; set to None
+# whenever the kernel changes until the counters are taken again)
+ARGMIN_TRAFFIC = 92.02e6
 
 
 def load_peaks():
@@ -198,11 +199,11 @@ def config_dict(cfg, rows_note=None):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="crvq", choices=["crvq", "reference"])
     ap.add_argument("--config", default="c2", choices=sorted(S.CONFIGS))
-    ap.add_argument("--ref-rows", type=int, default=24)
+    ap.add_argument("--ref-rows", type=int, default=64)
     ap.add_argument("--ref-warmup", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
