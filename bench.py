@@ -245,12 +245,17 @@ def main():
         clocks.gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
     except Exception:
         clocks.gpu_id = local
+    # events only around the arg-min launches (the roofline kernel): the other launches of
+    # the timed steps run unbracketed. The library replays a captured CUDA graph of the layer
+    # per profiling state; one untimed call captures the one the timed steps use.
+    P.crvq_profile_filter("encode_argmin")
+    P.crvq_profile_begin()
+    out = P.crvq_quantize_layer(W_d, X_d, cfg_r, out=out)
+    torch.cuda.synchronize()
+    P.crvq_profile_end()
     barrier()
     clocks.start()
     launches0 = P.crvq_launch_count()
-    # events only around the arg-min launches (the roofline kernel): the other launches of
-    # the timed steps run unbracketed
-    P.crvq_profile_filter("encode_argmin")
     P.crvq_profile_begin()
     step_ms = []
     scores = 0.0

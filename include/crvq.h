@@ -202,10 +202,9 @@ crvq_status crvq_update_codebook(const float* T, int64_t ldT, int64_t M, int64_t
  * results and rounding are those of crvq_update_codebook; the caller still passes the
  * inputs and outputs. Its scratch is one file-scope device array of 4 MiB, held by every GPU
  * that loads the library until the process exits:
- *  - sizes whose statistics exceed it (G_cov * K * 4 + K * 64 + 256 + S * 296 * K bytes,
- *    S = min(32, ceil(G_cov / 32)) group slices, each part rounded up to 256 bytes, above
- *    4 MiB - 256; e.g. K = 256 with more than ~1600 covered groups) return
- *    CRVQ_ERR_UNSUPPORTED before anything is enqueued;
+ *  - sizes whose statistics exceed it (G_cov * K * 4 + K * 64 + 256 bytes, each part rounded
+ *    up to 256 bytes, above 4 MiB - 256; e.g. K = 256 with more than ~4000 covered groups)
+ *    return CRVQ_ERR_UNSUPPORTED before anything is enqueued;
  *  - every call shares the array, so calls that overlap on the GPU (different streams or
  *    devices' streams writing the same device's array) race; each call clears what must
  *    start at zero;
@@ -297,6 +296,12 @@ typedef struct crvq_layer_report {
  * SplitMix64(cfg->seed, phase * 1024 + codebook) with phase 1 = prequantize, 2 = base,
  * 3 = extended, 4 = random importance. W [M x N], X [n_tok x N] may be host or device
  * pointers. Synchronizes `stream` (the report is host memory).
+ * When W, X and every output are device pointers and refine_rounds <= 1, the schedule has no
+ * host synchronisation inside: it is captured into a CUDA graph on the first call for a given
+ * (device, stream, shapes, configuration, pointers, profiling state) and replayed on later
+ * calls, which reads the current contents of W and X (up to 4 graphs are kept per process,
+ * least recently used evicted; their scratch stays reserved while they are kept). Setting
+ * CRVQ_GRAPHS=0 in the environment runs every call directly. Results are identical either way.
  */
 crvq_status crvq_quantize_layer(const float* W, const float* X, int64_t M, int64_t N,
                                 int64_t n_tok, const crvq_config* cfg,

@@ -83,6 +83,12 @@ struct ProfRec {
   double units;
 };
 std::vector<ProfRec> g_recs;
+struct ProfDone {  // a launch timed inside a replayed layer graph
+  const char* name;
+  float ms;
+  double units;
+};
+std::vector<ProfDone> g_graph_recs;
 std::vector<cudaEvent_t> g_pool;  // events reused across profiling sessions
 
 cudaEvent_t pool_get() {
@@ -103,10 +109,25 @@ cudaEvent_t pool_get() {
 
 void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
 
+// Layer graph being captured on this thread (ProfScope then records external event nodes
+// owned by it instead of pooled events).
+struct CapturedEvents {
+  std::vector<ProfRec> recs;
+};
+thread_local CapturedEvents* t_capture = nullptr;
+
 ProfScope::ProfScope(const char* name, cudaStream_t s, double units)
     : name_(name), s_(s), units_(units) {
   if (g_prof.load(std::memory_order_relaxed) &&
       strncmp(name, g_filter, strlen(g_filter)) == 0) {
+    if (t_capture) {  // an event node of the graph, recorded on every replay
+      if (cudaEventCreate(&a_) != cudaSuccess ||
+          cudaEventRecordWithFlags(a_, s_, cudaEventRecordExternal) != cudaSuccess) {
+        cudaGetLastError();
+        a_ = nullptr;
+      }
+      return;
+    }
     a_ = pool_get();
     if (a_ && cudaEventRecord(a_, s_) != cudaSuccess) {
       cudaGetLastError();
@@ -117,6 +138,16 @@ ProfScope::ProfScope(const char* name, cudaStream_t s, double units)
 
 ProfScope::~ProfScope() {
   if (!a_) return;
+  if (t_capture) {
+    cudaEvent_t b = nullptr;
+    if (cudaEventCreate(&b) != cudaSuccess ||
+        cudaEventRecordWithFlags(b, s_, cudaEventRecordExternal) != cudaSuccess) {
+      cudaGetLastError();
+      return;
+    }
+    t_capture->recs.push_back(ProfRec{name_, a_, b, units_});
+    return;
+  }
   cudaEvent_t b = pool_get();
   if (!b || cudaEventRecord(b, s_) != cudaSuccess) {
     cudaGetLastError();
@@ -202,6 +233,7 @@ crvq_status crvq_profile_begin(void) {
       g_pool.push_back(r.b);
     }
     g_recs.clear();
+    g_graph_recs.clear();
   }
   // pre-create events so that recording inside the profiled region does not create any
   std::vector<cudaEvent_t> fresh;
@@ -230,12 +262,29 @@ crvq_status crvq_profile_filter(const char* prefix) {
 crvq_status crvq_profile_end(crvq_kernel_stat* stats, int32_t cap, int32_t* n_stats) {
   g_prof.store(false);
   std::vector<ProfRec> recs;
+  std::vector<ProfDone> done;
   {
     std::lock_guard<std::mutex> lk(g_pmu);
     recs.swap(g_recs);
+    done.swap(g_graph_recs);
   }
   std::vector<crvq_kernel_stat> agg;
   crvq_status st = CRVQ_OK;
+  auto add = [&](const char* name, double ms, double units) {
+    size_t j = 0;
+    for (; j < agg.size(); ++j)
+      if (strncmp(agg[j].name, name, sizeof(agg[j].name)) == 0) break;
+    if (j == agg.size()) {
+      crvq_kernel_stat z;
+      memset(&z, 0, sizeof(z));
+      strncpy(z.name, name, sizeof(z.name) - 1);
+      agg.push_back(z);
+    }
+    agg[j].launches += 1;
+    agg[j].ms += ms;
+    agg[j].units += units;
+  };
+  for (auto& r : done) add(r.name, r.ms, r.units);
   for (auto& r : recs) {
     float ms = 0.f;
     if (cudaEventSynchronize(r.b) != cudaSuccess || cudaEventElapsedTime(&ms, r.a, r.b) != cudaSuccess) {
@@ -246,18 +295,7 @@ crvq_status crvq_profile_end(crvq_kernel_stat* stats, int32_t cap, int32_t* n_st
       g_pool.push_back(r.a);
       g_pool.push_back(r.b);
     }
-    size_t j = 0;
-    for (; j < agg.size(); ++j)
-      if (strncmp(agg[j].name, r.name, sizeof(agg[j].name)) == 0) break;
-    if (j == agg.size()) {
-      crvq_kernel_stat z;
-      memset(&z, 0, sizeof(z));
-      strncpy(z.name, r.name, sizeof(z.name) - 1);
-      agg.push_back(z);
-    }
-    agg[j].launches += 1;
-    agg[j].ms += ms;
-    agg[j].units += r.units;
+    add(r.name, ms, r.units);
   }
   const int n = (int)std::min<size_t>(agg.size(), cap > 0 ? (size_t)cap : 0);
   for (int i = 0; i < n; ++i) stats[i] = agg[i];
@@ -487,6 +525,289 @@ struct OutBuf {
 
 }  // namespace
 
+namespace {
+
+// Device outputs of one layer (every pointer on the device; C_ext / codes_ext NULL when
+// n_ext = 0, W_hat and imp may be NULL).
+struct LayerDev {
+  int32_t* perm;
+  float* C_base;
+  int32_t* codes_base;
+  float* C_ext;
+  int32_t* codes_ext;
+  float* W_hat;
+  float* imp;
+};
+
+// S1-S7 on device pointers: losses[0..11] (block, crit, full | pre | before refinement) and
+// *flag_total are written on the device; *scores and *rounds on the host. No host
+// synchronisation unless cfg->refine_rounds > 1 (the early stop reads the loss).
+crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, int64_t n_tok,
+                         const crvq_config* cfg, int64_t Gc, const LayerDev& o, double* losses,
+                         unsigned long long* flag_total, double* scores_out, int* rounds_out,
+                         cudaStream_t s) {
+  const int d = cfg->d;
+  const int64_t G = N / d;
+  double scores = 0.0;
+  CRVQ_CUDA(cudaMemsetAsync(flag_total, 0, sizeof(unsigned long long), s));
+  EncodeExtras ex;
+  ex.scores = &scores;
+  ex.flag_total = flag_total;
+
+  Buf bH, bxsq, bHb0, bdelta, bC0, bcodes0, bWpre, bWs, bHb;
+  float *H, *xsq, *Hb0, *delta, *C0, *Wpre, *Ws, *Hb;
+  int32_t* codes0;
+  CRVQ_TRY(bH.get(&H, (size_t)N * N, s));
+  CRVQ_TRY(bxsq.get(&xsq, N, s));
+  CRVQ_TRY(bHb0.get(&Hb0, (size_t)G * d * d, s));
+  CRVQ_TRY(bdelta.get(&delta, 4, s));
+  CRVQ_TRY(bC0.get(&C0, (size_t)cfg->K_base * d, s));
+  CRVQ_TRY(bcodes0.get(&codes0, (size_t)M * G, s));
+  CRVQ_TRY(bWpre.get(&Wpre, (size_t)M * N, s));
+  CRVQ_TRY(bWs.get(&Ws, (size_t)M * N, s));
+  CRVQ_TRY(bHb.get(&Hb, (size_t)G * d * d, s));
+
+  // S1: Hessian proxy
+  CRVQ_TRY(launch_hessian(X, n_tok, N, d, cfg->damp_rel, H, xsq, Hb0, delta, s));
+  // S2: prequantize in the original order (Alg. 1 line 3)
+  {
+    SetView set{W, N, M, G, Hb0};
+    CbList cl{};
+    cl.n = 1;
+    cl.cb[0] = CbView{C0, codes0, G, G, cfg->K_base};
+    CRVQ_TRY(launch_kmeans_init(set, CbList{}, cfg->K_base,
+                                phase_seed(cfg->seed, 1, 0), C0, s));
+    CRVQ_TRY(lloyd(set, cl, cfg->kmeans_iters, ex, s));
+    CRVQ_TRY(launch_reconstruct_error(W, M, N, Hb0, nullptr, cl, 0, nullptr, 0, 0.0, nullptr,
+                                      Wpre, losses + 3, s));
+  }
+  // S3: importance and reordering (Alg. 1 lines 4-5)
+  CRVQ_TRY(launch_select_reorder(W, M, N, d, Wpre, xsq, H, cfg->importance_mode,
+                                 phase_seed(cfg->seed, 4, 0), o.perm, o.imp, Ws, Hb, s));
+  // S4: base codebook over all vectors (Alg. 1 lines 6-7)
+  CbList all{};
+  all.n = 1 + cfg->n_ext;
+  all.cb[0] = CbView{o.C_base, o.codes_base, G, G, cfg->K_base};
+  for (int t = 1; t <= cfg->n_ext; ++t)
+    all.cb[t] = CbView{o.C_ext + (size_t)(t - 1) * cfg->K_ext * d,
+                       o.codes_ext + (size_t)(t - 1) * M * Gc, Gc, Gc, cfg->K_ext};
+  const SetView full{Ws, N, M, G, Hb};
+  {
+    CbList cl{};
+    cl.n = 1;
+    cl.cb[0] = all.cb[0];
+    CRVQ_TRY(launch_kmeans_init(full, CbList{}, cfg->K_base, phase_seed(cfg->seed, 2, 0),
+                                o.C_base, s));
+    CRVQ_TRY(lloyd(full, cl, cfg->kmeans_iters, ex, s));
+  }
+  // S5: extended codebooks on the critical residual (Alg. 1 lines 8-13)
+  if (cfg->n_ext > 0) {
+    const SetView crit{Ws, N, M, Gc, Hb};
+    for (int t = 1; t <= cfg->n_ext; ++t) {
+      CbList cl{};
+      cl.n = t + 1;
+      for (int q = 0; q <= t; ++q) {
+        cl.cb[q] = all.cb[q];
+        cl.cb[q].G_cov = Gc;
+      }
+      CbList fixed{};
+      fixed.n = t;
+      for (int q = 0; q < t; ++q) fixed.cb[q] = cl.cb[q];
+      CRVQ_TRY(launch_kmeans_init(crit, fixed, cfg->K_ext, phase_seed(cfg->seed, 3, t),
+                                  const_cast<float*>(all.cb[t].C), s));
+      CRVQ_TRY(lloyd(crit, cl, cfg->kmeans_iters, ex, s));
+    }
+  }
+  // S6: least-squares codebook updates + joint beam re-encode (Alg. 1 lines 14-17)
+  CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o.perm, all, Gc, nullptr, 0, 0.0, nullptr,
+                                    nullptr, losses + 6, s));
+  double prev = 0.0;
+  if (cfg->refine_rounds > 1) {
+    CRVQ_CUDA(cudaMemcpyAsync(&prev, losses + 6, sizeof(double), cudaMemcpyDeviceToHost, s));
+    CRVQ_CUDA(cudaStreamSynchronize(s));
+  }
+  int rounds = 0;
+  for (int r = 0; r < cfg->refine_rounds; ++r) {
+    for (int j = 0; j < all.n; ++j)
+      CRVQ_TRY(launch_update_codebook(full, all, j, const_cast<float*>(all.cb[j].C), nullptr, s));
+    CRVQ_TRY(launch_encode_beam(full, all, 0, cfg->B, true, nullptr, ex, s));
+    ++rounds;
+    if (cfg->refine_rounds > 1 && r + 1 < cfg->refine_rounds) {
+      CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o.perm, all, Gc, nullptr, 0, 0.0,
+                                        nullptr, nullptr, losses + 9, s));
+      double cur = 0.0;
+      CRVQ_CUDA(cudaMemcpyAsync(&cur, losses + 9, sizeof(double), cudaMemcpyDeviceToHost, s));
+      CRVQ_CUDA(cudaStreamSynchronize(s));
+      if (cur > (1.0 - (double)cfg->eps_rel) * prev) break;
+      prev = cur;
+    }
+  }
+  // S7: losses and the reconstruction in the original order
+  CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o.perm, all, Gc, X, n_tok, 0.0, delta,
+                                    o.W_hat, losses, s));
+  *scores_out = scores;
+  *rounds_out = rounds;
+  return CRVQ_OK;
+}
+
+void fill_report(crvq_layer_report* report, const double hl[12], unsigned long long flagged,
+                 double scores, int rounds) {
+  report->flagged = (int64_t)flagged;
+  report->loss_block = hl[0];
+  report->loss_crit = hl[1];
+  report->loss_full = hl[2];
+  report->loss_pre = hl[3];
+  report->loss_before_refine = hl[6];
+  report->scores = scores;
+  report->refine_rounds_done = rounds;
+}
+
+// ---- replay of whole-layer CUDA graphs
+// A layer whose inputs and outputs all live on the device, with at most one refinement round,
+// runs without host synchronisation between its ~240 launches; it is captured once into a
+// CUDA graph per (device, stream, shapes, configuration, pointers, profiling state) and
+// replayed, which removes the host launch gaps. Up to kGraphs graphs are kept (least recently
+// used evicted). CRVQ_GRAPHS=0 in the environment turns this off.
+struct LayerGraph {
+  int dev = -1;
+  cudaStream_t stream = nullptr;
+  int64_t M = 0, N = 0, n_tok = 0;
+  crvq_config cfg;
+  const float* W = nullptr;
+  const float* X = nullptr;
+  LayerDev o{};
+  bool prof = false;
+  char filter[64] = {0};
+  cudaGraphExec_t exec = nullptr;
+  double* losses = nullptr;                 // persistent device buffers read after a replay
+  unsigned long long* flag_total = nullptr;
+  double scores = 0.0;
+  int rounds = 0;
+  int64_t launches = 0;                     // kernels in the graph
+  CapturedEvents events;                    // arg-min event nodes when captured while profiling
+  uint64_t used = 0;
+};
+constexpr int kGraphs = 4;
+std::mutex g_graph_mu;
+std::vector<LayerGraph*> g_graphs;
+uint64_t g_graph_clock = 0;
+
+void destroy_graph(LayerGraph* e) {
+  if (e->exec) cudaGraphExecDestroy(e->exec);
+  if (e->losses) cudaFree(e->losses);
+  for (auto& r : e->events.recs) {
+    cudaEventDestroy(r.a);
+    cudaEventDestroy(r.b);
+  }
+  cudaGetLastError();
+  delete e;
+}
+
+bool graphs_enabled() {
+  const char* v = getenv("CRVQ_GRAPHS");
+  return !(v && v[0] == '0');
+}
+
+bool same_key(const LayerGraph& e, int dev, cudaStream_t st, int64_t M, int64_t N, int64_t n_tok,
+              const crvq_config* cfg, const float* W, const float* X, const LayerDev& o,
+              bool prof) {
+  return e.dev == dev && e.stream == st && e.M == M && e.N == N && e.n_tok == n_tok &&
+         memcmp(&e.cfg, cfg, sizeof(crvq_config)) == 0 && e.W == W && e.X == X &&
+         memcmp(&e.o, &o, sizeof(LayerDev)) == 0 && e.prof == prof &&
+         (!prof || strncmp(e.filter, g_filter, sizeof(e.filter)) == 0);
+}
+
+crvq_status run_graph(const float* W, const float* X, int64_t M, int64_t N, int64_t n_tok,
+                      const crvq_config* cfg, int64_t Gc, const LayerDev& o,
+                      crvq_layer_report* report, cudaStream_t s, bool* done) {
+  *done = false;
+  int dev = 0;
+  CRVQ_CUDA(cudaGetDevice(&dev));
+  const bool prof = g_prof.load();
+  std::lock_guard<std::mutex> lk(g_graph_mu);
+  LayerGraph* e = nullptr;
+  for (auto* c : g_graphs)
+    if (same_key(*c, dev, s, M, N, n_tok, cfg, W, X, o, prof)) e = c;
+  if (!e) {
+    // Everything that allocates or initialises lazily happens before the capture.
+    unsigned* err = nullptr;
+    CRVQ_TRY(device_error_word(&err));
+    sm_count();
+    e = new LayerGraph;
+    e->dev = dev;
+    e->stream = s;
+    e->M = M;
+    e->N = N;
+    e->n_tok = n_tok;
+    e->cfg = *cfg;
+    e->W = W;
+    e->X = X;
+    e->o = o;
+    e->prof = prof;
+    strncpy(e->filter, g_filter, sizeof(e->filter) - 1);
+    if (cudaMalloc(&e->losses, 16 * sizeof(double) + 64) != cudaSuccess) {
+      cudaGetLastError();
+      delete e;
+      return CRVQ_OK;  // not done: the caller runs the schedule directly
+    }
+    e->flag_total = reinterpret_cast<unsigned long long*>(e->losses + 16);
+    const long long l0 = g_launches.load();
+    cudaGraph_t graph = nullptr;
+    crvq_status st = CRVQ_OK;
+    if (cudaStreamBeginCapture(s, cudaStreamCaptureModeRelaxed) == cudaSuccess) {
+      t_capture = &e->events;
+      st = run_schedule(W, X, M, N, n_tok, cfg, Gc, o, e->losses, e->flag_total, &e->scores,
+                        &e->rounds, s);
+      t_capture = nullptr;
+      const cudaError_t ce = cudaStreamEndCapture(s, &graph);
+      if (ce != cudaSuccess) st = CRVQ_ERR_CUDA;
+    } else {
+      st = CRVQ_ERR_CUDA;
+    }
+    e->launches = g_launches.load() - l0;
+    g_launches.fetch_sub(e->launches);  // counted when replayed
+    if (st == CRVQ_OK && cudaGraphInstantiate(&e->exec, graph, 0) != cudaSuccess) st = CRVQ_ERR_CUDA;
+    if (graph) cudaGraphDestroy(graph);
+    cudaGetLastError();
+    if (st != CRVQ_OK) {  // capture not possible here: run the schedule directly
+      destroy_graph(e);
+      clear_last_error();
+      return CRVQ_OK;
+    }
+    if ((int)g_graphs.size() >= kGraphs) {
+      size_t lru = 0;
+      for (size_t q = 1; q < g_graphs.size(); ++q)
+        if (g_graphs[q]->used < g_graphs[lru]->used) lru = q;
+      destroy_graph(g_graphs[lru]);
+      g_graphs.erase(g_graphs.begin() + lru);
+    }
+    g_graphs.push_back(e);
+  }
+  e->used = ++g_graph_clock;
+  CRVQ_CUDA(cudaGraphLaunch(e->exec, s));
+  g_launches.fetch_add(e->launches);
+  double hl[12];
+  unsigned long long flagged = 0;
+  CRVQ_CUDA(cudaMemcpyAsync(hl, e->losses, sizeof(hl), cudaMemcpyDeviceToHost, s));
+  CRVQ_CUDA(cudaMemcpyAsync(&flagged, e->flag_total, sizeof(flagged), cudaMemcpyDeviceToHost, s));
+  CRVQ_CUDA(cudaStreamSynchronize(s));
+  if (prof && g_prof.load()) {  // the event nodes of this replay have completed
+    std::lock_guard<std::mutex> lk2(g_pmu);
+    for (auto& r : e->events.recs) {
+      float ms = 0.f;
+      if (cudaEventElapsedTime(&ms, r.a, r.b) == cudaSuccess)
+        g_graph_recs.push_back(ProfDone{r.name, ms, r.units});
+      else
+        cudaGetLastError();
+    }
+  }
+  fill_report(report, hl, flagged, e->scores, e->rounds);
+  *done = true;
+  return CRVQ_OK;
+}
+
+}  // namespace
+
 extern "C" {
 
 crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M, int64_t N,
@@ -519,21 +840,34 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   cudaStream_t s = (cudaStream_t)stream;
   memset(report, 0, sizeof(*report));
   report->n_crit_groups = Gc;
-  double scores = 0.0;
-  Buf bflag;
-  unsigned long long* flag_total = nullptr;
-  CRVQ_TRY(bflag.get(&flag_total, 1, s));
-  CRVQ_CUDA(cudaMemsetAsync(flag_total, 0, sizeof(unsigned long long), s));
-  EncodeExtras ex;
-  ex.scores = &scores;
-  ex.flag_total = flag_total;
 
-  Buf bW, bX;
+  const bool dev_in = is_device_ptr(W_in) && is_device_ptr(X_in);
+  const bool dev_out = is_device_ptr(out->perm) && is_device_ptr(out->C_base) &&
+                       is_device_ptr(out->codes_base) &&
+                       (cfg->n_ext == 0 || (is_device_ptr(out->C_ext) &&
+                                            is_device_ptr(out->codes_ext))) &&
+                       (!out->W_hat || is_device_ptr(out->W_hat)) &&
+                       (!out->importance || is_device_ptr(out->importance));
+  if (dev_in && dev_out && cfg->refine_rounds <= 1 && graphs_enabled() &&
+      aligned16(W_in) && aligned16(X_in) && aligned16(out->C_base) &&
+      (cfg->n_ext == 0 || aligned16(out->C_ext)) && (!out->W_hat || aligned16(out->W_hat))) {
+    const LayerDev o{out->perm, out->C_base, out->codes_base,
+                     cfg->n_ext ? out->C_ext : nullptr, cfg->n_ext ? out->codes_ext : nullptr,
+                     out->W_hat, out->importance};
+    bool done = false;
+    CRVQ_TRY(run_graph(W_in, X_in, M, N, n_tok, cfg, Gc, o, report, s, &done));
+    if (done) {
+      report->n_crit_groups = Gc;
+      return CRVQ_OK;
+    }
+  }
+
+  // Direct path: host inputs / outputs are staged through device buffers.
+  Buf bW, bX, bloss;
   const float *W = nullptr, *X = nullptr;
   CRVQ_TRY(to_device(W_in, (size_t)M * N, bW, &W, s));
   CRVQ_TRY(to_device(X_in, (size_t)n_tok * N, bX, &X, s));
   CRVQ_CHECK_ARG(aligned16(W) && aligned16(X), "W and X must be 16-byte aligned");
-
   OutBuf<int32_t> o_perm, o_codes_base, o_codes_ext;
   OutBuf<float> o_C_base, o_C_ext, o_W_hat, o_imp;
   CRVQ_TRY(o_perm.init(out->perm, N, s));
@@ -546,100 +880,14 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   CRVQ_CHECK_ARG(aligned16(o_C_base.dev) && aligned16(o_C_ext.dev) &&
                      (!out->W_hat || aligned16(o_W_hat.dev)),
                  "C_base, C_ext and W_hat must be 16-byte aligned");
-
-  Buf bH, bxsq, bHb0, bdelta, bC0, bcodes0, bWpre, bWs, bHb, bloss;
-  float *H, *xsq, *Hb0, *delta, *C0, *Wpre, *Ws, *Hb;
-  int32_t* codes0;
-  double* losses;
-  CRVQ_TRY(bH.get(&H, (size_t)N * N, s));
-  CRVQ_TRY(bxsq.get(&xsq, N, s));
-  CRVQ_TRY(bHb0.get(&Hb0, (size_t)G * d * d, s));
-  CRVQ_TRY(bdelta.get(&delta, 4, s));
-  CRVQ_TRY(bC0.get(&C0, (size_t)cfg->K_base * d, s));
-  CRVQ_TRY(bcodes0.get(&codes0, (size_t)M * G, s));
-  CRVQ_TRY(bWpre.get(&Wpre, (size_t)M * N, s));
-  CRVQ_TRY(bWs.get(&Ws, (size_t)M * N, s));
-  CRVQ_TRY(bHb.get(&Hb, (size_t)G * d * d, s));
-  CRVQ_TRY(bloss.get(&losses, 16, s));
-
-  // S1: Hessian proxy
-  CRVQ_TRY(launch_hessian(X, n_tok, N, d, cfg->damp_rel, H, xsq, Hb0, delta, s));
-  // S2: prequantize in the original order (Alg. 1 line 3)
-  {
-    SetView set{W, N, M, G, Hb0};
-    CbList cl{};
-    cl.n = 1;
-    cl.cb[0] = CbView{C0, codes0, G, G, cfg->K_base};
-    CRVQ_TRY(launch_kmeans_init(set, CbList{}, cfg->K_base,
-                                phase_seed(cfg->seed, 1, 0), C0, s));
-    CRVQ_TRY(lloyd(set, cl, cfg->kmeans_iters, ex, s));
-    CRVQ_TRY(launch_reconstruct_error(W, M, N, Hb0, nullptr, cl, 0, nullptr, 0, 0.0, nullptr,
-                                      Wpre, losses + 3, s));
-  }
-  // S3: importance and reordering (Alg. 1 lines 4-5)
-  CRVQ_TRY(launch_select_reorder(W, M, N, d, Wpre, xsq, H, cfg->importance_mode,
-                                 phase_seed(cfg->seed, 4, 0), o_perm.dev, o_imp.dev, Ws, Hb, s));
-  // S4: base codebook over all vectors (Alg. 1 lines 6-7)
-  CbList all{};
-  all.n = 1 + cfg->n_ext;
-  all.cb[0] = CbView{o_C_base.dev, o_codes_base.dev, G, G, cfg->K_base};
-  for (int t = 1; t <= cfg->n_ext; ++t)
-    all.cb[t] = CbView{o_C_ext.dev + (size_t)(t - 1) * cfg->K_ext * d,
-                       o_codes_ext.dev + (size_t)(t - 1) * M * Gc, Gc, Gc, cfg->K_ext};
-  const SetView full{Ws, N, M, G, Hb};
-  {
-    CbList cl{};
-    cl.n = 1;
-    cl.cb[0] = all.cb[0];
-    CRVQ_TRY(launch_kmeans_init(full, CbList{}, cfg->K_base, phase_seed(cfg->seed, 2, 0),
-                                o_C_base.dev, s));
-    CRVQ_TRY(lloyd(full, cl, cfg->kmeans_iters, ex, s));
-  }
-  // S5: extended codebooks on the critical residual (Alg. 1 lines 8-13)
-  if (cfg->n_ext > 0) {
-    const SetView crit{Ws, N, M, Gc, Hb};
-    for (int t = 1; t <= cfg->n_ext; ++t) {
-      CbList cl{};
-      cl.n = t + 1;
-      for (int q = 0; q <= t; ++q) {
-        cl.cb[q] = all.cb[q];
-        cl.cb[q].G_cov = Gc;
-      }
-      CbList fixed{};
-      fixed.n = t;
-      for (int q = 0; q < t; ++q) fixed.cb[q] = cl.cb[q];
-      CRVQ_TRY(launch_kmeans_init(crit, fixed, cfg->K_ext, phase_seed(cfg->seed, 3, t),
-                                  const_cast<float*>(all.cb[t].C), s));
-      CRVQ_TRY(lloyd(crit, cl, cfg->kmeans_iters, ex, s));
-    }
-  }
-  // S6: least-squares codebook updates + joint beam re-encode (Alg. 1 lines 14-17)
-  CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o_perm.dev, all, Gc, nullptr, 0, 0.0,
-                                    nullptr, nullptr, losses + 6, s));
-  double prev = 0.0;
-  if (cfg->refine_rounds > 1) {
-    CRVQ_CUDA(cudaMemcpyAsync(&prev, losses + 6, sizeof(double), cudaMemcpyDeviceToHost, s));
-    CRVQ_CUDA(cudaStreamSynchronize(s));
-  }
+  double* losses = nullptr;
+  CRVQ_TRY(bloss.get(&losses, 16 + 8, s));
+  unsigned long long* flag_total = reinterpret_cast<unsigned long long*>(losses + 16);
+  const LayerDev o{o_perm.dev, o_C_base.dev, o_codes_base.dev, o_C_ext.dev, o_codes_ext.dev,
+                   out->W_hat ? o_W_hat.dev : nullptr, o_imp.dev};
+  double scores = 0.0;
   int rounds = 0;
-  for (int r = 0; r < cfg->refine_rounds; ++r) {
-    for (int j = 0; j < all.n; ++j)
-      CRVQ_TRY(launch_update_codebook(full, all, j, const_cast<float*>(all.cb[j].C), nullptr, s));
-    CRVQ_TRY(launch_encode_beam(full, all, 0, cfg->B, true, nullptr, ex, s));
-    ++rounds;
-    if (cfg->refine_rounds > 1 && r + 1 < cfg->refine_rounds) {
-      CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o_perm.dev, all, Gc, nullptr, 0, 0.0,
-                                        nullptr, nullptr, losses + 9, s));
-      double cur = 0.0;
-      CRVQ_CUDA(cudaMemcpyAsync(&cur, losses + 9, sizeof(double), cudaMemcpyDeviceToHost, s));
-      CRVQ_CUDA(cudaStreamSynchronize(s));
-      if (cur > (1.0 - (double)cfg->eps_rel) * prev) break;
-      prev = cur;
-    }
-  }
-  // S7: losses and the reconstruction in the original order
-  CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o_perm.dev, all, Gc, X, n_tok, 0.0, delta,
-                                    out->W_hat ? o_W_hat.dev : nullptr, losses, s));
+  CRVQ_TRY(run_schedule(W, X, M, N, n_tok, cfg, Gc, o, losses, flag_total, &scores, &rounds, s));
   CRVQ_TRY(o_perm.flush(s));
   CRVQ_TRY(o_C_base.flush(s));
   CRVQ_TRY(o_codes_base.flush(s));
@@ -652,14 +900,7 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   CRVQ_CUDA(cudaMemcpyAsync(hl, losses, sizeof(hl), cudaMemcpyDeviceToHost, s));
   CRVQ_CUDA(cudaMemcpyAsync(&flagged, flag_total, sizeof(flagged), cudaMemcpyDeviceToHost, s));
   CRVQ_CUDA(cudaStreamSynchronize(s));
-  report->flagged = (int64_t)flagged;
-  report->loss_block = hl[0];
-  report->loss_crit = hl[1];
-  report->loss_full = hl[2];
-  report->loss_pre = hl[3];
-  report->loss_before_refine = hl[6];
-  report->scores = scores;
-  report->refine_rounds_done = rounds;
+  fill_report(report, hl, flagged, scores, rounds);
   return CRVQ_OK;
 }
 

@@ -19,30 +19,25 @@ struct StatsView {
   int32_t* cnt;     // [G_cov][K]
   long long* bacc;  // [K][d]
   double* scale;    // device scalar (followed by the maxima of the scale bound)
-  double* apart;    // [gsplit][kNA][K] fp64 partial sums of A_k over slices of the groups
   int64_t G_cov;
   int K;
-  int gsplit;
 };
 
 constexpr int kNA = 37;  // packed lower triangle of the 8 x 8 A_k (36 entries) + the count
 
-// Memory of the statistics of one codebook: cnt | bacc | scale + maxima (256 B) | apart, each
-// part 256-byte aligned. The groups are cut into gsplit slices of about 32 groups each.
+// Memory of the statistics of one codebook: cnt | bacc | scale + maxima (256 B), each part
+// 256-byte aligned.
 struct StatsLayout {
-  size_t cnt, bacc, head, apart, total;
-  int gsplit;
+  size_t cnt, bacc, head, total;
 };
 
 inline StatsLayout stats_layout(int64_t G_cov, int K) {
   StatsLayout L;
   const int64_t G = G_cov > 1 ? G_cov : 1;
-  L.gsplit = (int)(G < 32 * 32 ? (G + 31) / 32 : 32);
   L.cnt = align_up((size_t)G * K * sizeof(int32_t), 256);
   L.bacc = align_up((size_t)K * kD * sizeof(long long), 256);
   L.head = 256;
-  L.apart = align_up((size_t)L.gsplit * kNA * K * sizeof(double), 256);
-  L.total = L.cnt + L.bacc + L.head + L.apart;
+  L.total = L.cnt + L.bacc + L.head;
   return L;
 }
 
@@ -53,10 +48,8 @@ inline void stats_bind(void* base, int64_t G_cov, int K, StatsView* st) {
   st->cnt = reinterpret_cast<int32_t*>(p);
   st->bacc = reinterpret_cast<long long*>(p + L.cnt);
   st->scale = reinterpret_cast<double*>(p + L.cnt + L.bacc);
-  st->apart = reinterpret_cast<double*>(p + L.cnt + L.bacc + L.head);
   st->G_cov = G_cov;
   st->K = K;
-  st->gsplit = L.gsplit;
 }
 
 // 2^e with e the largest integer such that n * bound * 2^e < 2^62.

@@ -6,8 +6,8 @@
 // Deterministic by construction, with no sort and no float atomics: cnt[g][k] are integer
 // counts, b_k is accumulated in 64-bit fixed point (stats.cuh), A_k is summed as fp32 pairs in
 // a fixed order (partial sums over fixed slices of the groups, added in slice order), and the
-// 8 x 8 system is solved to fp64 accuracy by mixed-precision iterative refinement, one thread
-// per codeword. GB300's fp64 pipe is a small fraction of its fp32 rate, so none of this
+// 8 x 8 system is solved to fp64 accuracy by mixed-precision iterative refinement, in one
+// kernel. GB300's fp64 pipe is a small fraction of its fp32 rate, so none of this
 // arithmetic runs per element in fp64. The Lloyd encode
 // pass (encode.cu) accumulates the same statistics for the codes it writes.
 #include <algorithm>
@@ -142,69 +142,10 @@ dim3 accumulate_grid(int64_t M, int64_t G_cov, int nsm) {
   return dim3((unsigned)rows_x, (unsigned)std::min<int64_t>(std::max<int64_t>(G_cov, 1), 65535));
 }
 
-// A_k = sum_g cnt[g][k] H_g as partial sums over slices of the groups, without the fp64
-// pipe: every product cnt * H is split exactly into fp32 hi + lo (cnt < 2^24), and the sum is
-// kept as an unevaluated fp32 pair (Knuth's TwoSum for the high part, the low parts added),
-// about 2^-44 relative after a few thousand terms. CTA (kb, gs): lane = codeword 32 kb + lane
-// (coalesced counts), the groups of slice gs strided over the warps (H_g read once per warp,
-// the same address in every lane), then the warps' pairs added in fp64 in warp order. The
-// fixed assignment and order make the result identical on every run.
-constexpr int kGramWarps = 4;
-
-__global__ void __launch_bounds__(32 * kGramWarps)
-stats_gram_kernel(const float* __restrict__ Hb, StatsView st) {
-  __shared__ double red[kGramWarps - 1][kNA][32];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int K = st.K;
-  const int k = blockIdx.x * 32 + lane;
-  const int64_t gper = (st.G_cov + st.gsplit - 1) / st.gsplit;
-  const int64_t g0 = (int64_t)blockIdx.y * gper;
-  const int64_t g1 = min(st.G_cov, g0 + gper);
-  float hi[kNA - 1], lo[kNA - 1];
-#pragma unroll
-  for (int e = 0; e < kNA - 1; ++e) hi[e] = lo[e] = 0.f;
-  int count = 0;
-  for (int64_t g = g0 + warp; g < g1; g += kGramWarps) {
-    const int c = k < K ? st.cnt[g * K + k] : 0;
-    if (!__any_sync(0xffffffffu, c != 0)) continue;
-    const float* H = Hb + g * kD * kD;
-    const float fc = (float)c;  // exact: counts stay below 2^24
-    count += c;
-    int q = 0;
-#pragma unroll
-    for (int r = 0; r < kD; ++r)
-#pragma unroll
-      for (int cc = 0; cc <= r; ++cc, ++q) {
-        const float h = __ldg(H + r * kD + cc);
-        const float p = __fmul_rn(fc, h);
-        const float pe = fmaf(fc, h, -p);           // fc * h = p + pe exactly
-        const float sum = __fadd_rn(hi[q], p);       // TwoSum(hi, p) = sum + t exactly
-        const float bp = __fsub_rn(sum, hi[q]);
-        const float t = __fadd_rn(__fsub_rn(hi[q], __fsub_rn(sum, bp)), __fsub_rn(p, bp));
-        hi[q] = sum;
-        lo[q] = __fadd_rn(lo[q], __fadd_rn(t, pe));
-      }
-  }
-  double A[kNA];
-#pragma unroll
-  for (int e = 0; e < kNA - 1; ++e) A[e] = (double)hi[e] + (double)lo[e];
-  A[kNA - 1] = (double)count;
-  if (warp > 0)
-#pragma unroll
-    for (int e = 0; e < kNA; ++e) red[warp - 1][e][lane] = A[e];
-  __syncthreads();
-  if (warp == 0 && k < K) {
-    for (int w = 0; w < kGramWarps - 1; ++w)
-#pragma unroll
-      for (int e = 0; e < kNA; ++e) A[e] += red[w][e][lane];
-#pragma unroll
-    for (int e = 0; e < kNA; ++e) st.apart[((int64_t)blockIdx.y * kNA + e) * K + k] = A[e];
-  }
-}
-
-// fp32 Cholesky factor of the packed lower triangle (false unless every pivot is positive),
-// and the solve L L^T x = b with it.
-__device__ inline bool chol8_f32(const float A[36], float L[36]) {
+// fp32 Cholesky factor of the packed lower triangle (false unless every pivot is positive)
+// with the reciprocals of its diagonal, and the solve L L^T x = b with them: 8 divisions per
+// factor, none per solve (the refinement absorbs the rounding of the reciprocals).
+__device__ inline bool chol8_f32(const float A[36], float L[36], float inv[kD]) {
   int q = 0;
 #pragma unroll
   for (int r = 0; r < kD; ++r)
@@ -216,49 +157,137 @@ __device__ inline bool chol8_f32(const float A[36], float L[36]) {
       if (r == c) {
         if (!(s > 0.f)) return false;
         L[q] = sqrtf(s);
+        inv[r] = 1.f / L[q];
       } else {
-        L[q] = s / L[c * (c + 1) / 2 + c];
+        L[q] = s * inv[c];
       }
     }
   return true;
 }
 
-__device__ inline void chol8_solve_f32(const float L[36], const float b[kD], float x[kD]) {
+__device__ inline void chol8_solve_f32(const float L[36], const float inv[kD], const float b[kD],
+                                       float x[kD]) {
   float y[kD];
 #pragma unroll
   for (int r = 0; r < kD; ++r) {
     float s = b[r];
 #pragma unroll
     for (int m = 0; m < r; ++m) s = fmaf(-L[r * (r + 1) / 2 + m], y[m], s);
-    y[r] = s / L[r * (r + 1) / 2 + r];
+    y[r] = s * inv[r];
   }
 #pragma unroll
   for (int r = kD - 1; r >= 0; --r) {
     float s = y[r];
 #pragma unroll
     for (int m = r + 1; m < kD; ++m) s = fmaf(-L[m * (m + 1) / 2 + r], x[m], s);
-    x[r] = s / L[r * (r + 1) / 2 + r];
+    x[r] = s * inv[r];
   }
 }
 
-// One thread per codeword: A_k = the slices' partial sums added in slice order, b_k from the
-// fixed point. The system is solved by mixed-precision iterative refinement: an fp32
-// Cholesky factor, then x += L^-T L^-1 (b - A x) with the residual in fp64 until the
-// correction is below 2^-40 of x (cond(A) u_32 < 1 makes each step gain about
-// -log2(cond(A) u_32) bits). A factor that fails or a refinement that does not settle falls
-// back to the fp64 Cholesky solve. Codewords without members keep their old value.
-__global__ void __launch_bounds__(32)
-stats_chol_kernel(StatsView st, const float* C_old, float* C_out, int32_t* __restrict__ counts_out,
-                  unsigned* err) {
-  const int k = blockIdx.x * blockDim.x + threadIdx.x;
-  if (k >= st.K) return;
+// Solves A x = b (A packed lower triangle, fp64) by mixed-precision iterative refinement: an
+// fp32 Cholesky factor, then x += L^-T L^-1 (b - A x) with the residual in fp64 until the
+// correction is below 2^-40 of x (each step gains about -log2(cond(A) u_32) bits). A factor
+// that fails or a refinement that does not settle falls back to the fp64 Cholesky solve.
+__device__ bool solve8_refined(const double A[36], const double b[kD], double x[kD]) {
+  float Af[36], Lf[36], inv[kD];
+#pragma unroll
+  for (int e = 0; e < 36; ++e) Af[e] = (float)A[e];
+  if (chol8_f32(Af, Lf, inv)) {
+    float bf[kD], xf[kD];
+#pragma unroll
+    for (int j = 0; j < kD; ++j) bf[j] = (float)b[j];
+    chol8_solve_f32(Lf, inv, bf, xf);
+#pragma unroll
+    for (int j = 0; j < kD; ++j) x[j] = (double)xf[j];
+    for (int it = 0; it < 6; ++it) {
+      float rf[kD], dx[kD];
+#pragma unroll
+      for (int r = 0; r < kD; ++r) {
+        double s = b[r];
+#pragma unroll
+        for (int c = 0; c < kD; ++c) {
+          const double a = r >= c ? A[r * (r + 1) / 2 + c] : A[c * (c + 1) / 2 + r];
+          s = fma(-a, x[c], s);
+        }
+        rf[r] = (float)s;
+      }
+      chol8_solve_f32(Lf, inv, rf, dx);
+      float xm = 0.f, dm = 0.f;
+#pragma unroll
+      for (int j = 0; j < kD; ++j) {
+        x[j] += (double)dx[j];
+        xm = fmaxf(xm, fabsf((float)x[j]));
+        dm = fmaxf(dm, fabsf(dx[j]));
+      }
+      if (dm <= 9.094947e-13f * xm) return true;  // 2^-40
+    }
+  }
+  return cholesky_solve8(A, b, x);
+}
+
+// The least-squares solve of every codeword, one kernel. CTA = kSolveK codewords; thread =
+// (codeword, entry e of A_k's packed lower triangle or the count, slice of the groups). Each
+// thread sums cnt[g][k] * H_g[e] over its slice as an unevaluated fp32 pair (every product is
+// split exactly: cnt < 2^24; TwoSum for the high part), so no fp64 arithmetic runs per group;
+// the slices are added in a fixed order in fp64; then one thread per codeword solves
+// A_k c_k = b_k (b_k from the fixed point) by refined Cholesky. The fixed assignment and
+// order make the result identical on every run. Codewords without members keep their old
+// value.
+constexpr int kSolveK = 4;
+constexpr int kSolveSlices = 4;
+constexpr int kSolveThreads = kSolveK * kSolveSlices * kNA;  // 592
+
+__global__ void __launch_bounds__(kSolveThreads)
+stats_solve_kernel(const float* __restrict__ Hb, StatsView st, const float* C_old, float* C_out,
+                   int32_t* __restrict__ counts_out, unsigned* err) {
+  __shared__ double part[kSolveK][kSolveSlices][kNA];
+  const int tid = threadIdx.x;
+  const int kk = tid / (kSolveSlices * kNA);
+  const int sl = (tid / kNA) % kSolveSlices;
+  const int e = tid % kNA;
   const int K = st.K;
+  const int k = blockIdx.x * kSolveK + kk;
+  // entry e of the packed lower triangle: row r, column c (c <= r); e = 36 is the count
+  int r = 0;
+  while ((r + 1) * (r + 2) / 2 <= e && r < kD - 1) ++r;
+  const int c = e - r * (r + 1) / 2;
+  const int hoff = r * kD + c;
+  float hi = 0.f, lo = 0.f;
+  if (k < K) {
+    const int64_t gper = (st.G_cov + kSolveSlices - 1) / kSolveSlices;
+    const int64_t g0 = sl * gper, g1 = min(st.G_cov, g0 + gper);
+    constexpr int kBatch = 8;  // loads of 8 groups in flight together; no branches
+    for (int64_t gb = g0; gb < g1; gb += kBatch) {
+      float fc[kBatch], h[kBatch];
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u) {
+        const int64_t g = gb + u;
+        const bool in = g < g1;
+        fc[u] = in ? (float)st.cnt[g * K + k] : 0.f;  // exact: counts stay below 2^24
+        h[u] = in ? (e < 36 ? __ldg(Hb + g * kD * kD + hoff) : 1.f) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < kBatch; ++u) {
+        const float p = __fmul_rn(fc[u], h[u]);
+        const float pe = __fmaf_rn(fc[u], h[u], -p);  // fc h = p + pe exactly
+        const float sum = __fadd_rn(hi, p);            // TwoSum(hi, p) = sum + t exactly
+        const float bp = __fsub_rn(sum, hi);
+        const float t = __fadd_rn(__fsub_rn(hi, __fsub_rn(sum, bp)), __fsub_rn(p, bp));
+        hi = sum;
+        lo = __fadd_rn(lo, __fadd_rn(t, pe));
+      }
+    }
+  }
+  part[kk][sl][e] = (double)hi + (double)lo;
+  __syncthreads();
+  if (sl != 0 || e != 0 || k >= K) return;
   double A[kNA];
 #pragma unroll
-  for (int e = 0; e < kNA; ++e) A[e] = 0.0;
-  for (int gs = 0; gs < st.gsplit; ++gs)
-#pragma unroll
-    for (int e = 0; e < kNA; ++e) A[e] += st.apart[((int64_t)gs * kNA + e) * K + k];
+  for (int q = 0; q < kNA; ++q) {
+    double a = part[kk][0][q];
+    for (int s2 = 1; s2 < kSolveSlices; ++s2) a += part[kk][s2][q];
+    A[q] = a;
+  }
   const int64_t count = (int64_t)A[36];
   if (counts_out) counts_out[k] = (int32_t)count;
   bool keep = count == 0;
@@ -268,47 +297,13 @@ stats_chol_kernel(StatsView st, const float* C_old, float* C_out, int32_t* __res
     double b[kD], x[kD];
 #pragma unroll
     for (int j = 0; j < kD; ++j) b[j] = (double)st.bacc[(int64_t)k * kD + j] * inv_scale;
-    float Af[36], Lf[36];
+    if (solve8_refined(A, b, x)) {
 #pragma unroll
-    for (int e = 0; e < 36; ++e) Af[e] = (float)A[e];
-    bool solved = false;
-    if (chol8_f32(Af, Lf)) {
-      float bf[kD], xf[kD];
-#pragma unroll
-      for (int j = 0; j < kD; ++j) bf[j] = (float)b[j];
-      chol8_solve_f32(Lf, bf, xf);
-#pragma unroll
-      for (int j = 0; j < kD; ++j) x[j] = (double)xf[j];
-      for (int it = 0; it < 6 && !solved; ++it) {
-        float rf[kD], dx[kD];
-#pragma unroll
-        for (int r = 0; r < kD; ++r) {
-          double s = b[r];
-#pragma unroll
-          for (int c = 0; c < kD; ++c) {
-            const double a = r >= c ? A[r * (r + 1) / 2 + c] : A[c * (c + 1) / 2 + r];
-            s = fma(-a, x[c], s);
-          }
-          rf[r] = (float)s;
-        }
-        chol8_solve_f32(Lf, rf, dx);
-        float xm = 0.f, dm = 0.f;
-#pragma unroll
-        for (int j = 0; j < kD; ++j) {
-          x[j] += (double)dx[j];
-          xm = fmaxf(xm, fabsf((float)x[j]));
-          dm = fmaxf(dm, fabsf(dx[j]));
-        }
-        solved = dm <= 9.094947e-13f * xm;  // 2^-40
-      }
-    }
-    if (!solved && !cholesky_solve8(A, b, x)) {
+      for (int j = 0; j < kD; ++j) out[j] = (float)x[j];
+    } else {
       raise_error(err, ERRBIT_NUMERIC);
       keep = true;
     }
-    if (!keep)
-#pragma unroll
-      for (int j = 0; j < kD; ++j) out[j] = (float)x[j];
   }
   if (keep)
 #pragma unroll
@@ -320,15 +315,9 @@ stats_chol_kernel(StatsView st, const float* C_old, float* C_out, int32_t* __res
 crvq_status launch_solve_kernels(const float* Hb, const StatsView& st, const float* C_old,
                                  float* C_out, int32_t* counts, unsigned* err,
                                  cudaStream_t stream) {
-  {
-    ProfScope ps("update_gram", stream, (double)st.G_cov * st.K);
-    stats_gram_kernel<<<dim3((unsigned)ceil_div(st.K, 32), (unsigned)st.gsplit), 32 * kGramWarps,
-                        0, stream>>>(Hb, st);
-    CRVQ_LAUNCHED();
-  }
   ProfScope ps("update_solve", stream, (double)st.K);
-  stats_chol_kernel<<<(unsigned)ceil_div(st.K, 32), 32, 0, stream>>>(st, C_old, C_out, counts,
-                                                                     err);
+  stats_solve_kernel<<<(unsigned)ceil_div(st.K, kSolveK), kSolveThreads, 0, stream>>>(
+      Hb, st, C_old, C_out, counts, err);
   CRVQ_LAUNCHED();
   return CRVQ_OK;
 }
@@ -413,7 +402,7 @@ crvq_status launch_update_codebook_on(const SetView& set, const CbList& cbs, int
   if (need > bytes)
     return fail(CRVQ_ERR_UNSUPPORTED,
                 "statistics of this codebook need %zu bytes of scratch, the limit is %zu "
-                "(G_cov * K * 4 + K * 64 + 256 + gsplit * 296 * K bytes, 256-byte aligned)",
+                "(G_cov * K * 4 + K * 64 + 256 bytes, each part 256-byte aligned)",
                 need, bytes);
   const StatsLayout L = stats_layout(cw.G_cov, cw.K);
   StatsView st;

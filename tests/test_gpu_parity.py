@@ -473,3 +473,32 @@ def test_quantize_layer_host_buffers_match_device(c1):
     np.testing.assert_array_equal(host(a.codes_base), b.codes_base.numpy())
     np.testing.assert_array_equal(host(a.C_ext), b.C_ext.numpy())
     assert a.report["loss_full"] == b.report["loss_full"]
+
+
+def test_quantize_layer_graph_replay_matches_direct_run(c1, monkeypatch):
+    """With device buffers the layer is captured into a CUDA graph on the first call and
+    replayed on later ones: a replay equals the direct (uncaptured) run bit for bit, also after
+    the contents of W change in place, and counts the same launches."""
+    cfg = c1["cfg"].with_(kmeans_iters=3)
+    W = dev(c1["W"])
+    X = dev(c1["X"])
+    first = P.crvq_quantize_layer(W, X, cfg)                     # captured
+    n0 = P.crvq_launch_count()
+    again = P.crvq_quantize_layer(W, X, cfg, out=first)          # replayed
+    torch.cuda.synchronize()
+    n_graph = P.crvq_launch_count() - n0
+    W.mul_(1.5)                                                  # same pointer, new values
+    replay = P.crvq_quantize_layer(W, X, cfg, out=again)
+    torch.cuda.synchronize()
+    got = {k: host(getattr(replay, k)).copy() for k in ("perm", "C_base", "codes_base",
+                                                          "C_ext", "codes_ext", "W_hat")}
+    rep = dict(replay.report)
+    monkeypatch.setenv("CRVQ_GRAPHS", "0")
+    n1 = P.crvq_launch_count()
+    direct = P.crvq_quantize_layer(W, X, cfg)
+    torch.cuda.synchronize()
+    assert P.crvq_launch_count() - n1 == n_graph
+    for k, v in got.items():
+        np.testing.assert_array_equal(v, host(getattr(direct, k)), err_msg=k)
+    for k in ("loss_block", "loss_crit", "loss_full", "loss_pre", "scores", "flagged"):
+        assert rep[k] == direct.report[k], k
