@@ -50,6 +50,26 @@ sumsq_partials_kernel(const float* __restrict__ P, int64_t count, int chunks, in
   if (threadIdx.x == 0) part[blockIdx.x] = red[0];
 }
 
+// out[a][k] = X[k][a] (X: n x N row-major) for a < N, k < n; columns k in [n, ldt) are 0.
+__global__ void __launch_bounds__(256)
+transpose_kernel(const float* __restrict__ X, int64_t n, int64_t N, float* __restrict__ out,
+                 int64_t ldt) {
+  __shared__ float t[32][33];
+  const int64_t k0 = (int64_t)blockIdx.x * 32, a0 = (int64_t)blockIdx.y * 32;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 32 x 8
+#pragma unroll
+  for (int r = ty; r < 32; r += 8) {
+    const int64_t k = k0 + r, a = a0 + tx;
+    t[r][tx] = (k < n && a < N) ? X[k * N + a] : 0.f;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int r = ty; r < 32; r += 8) {
+    const int64_t a = a0 + r, k = k0 + tx;
+    if (a < N && k < ldt) out[a * ldt + k] = t[tx][r];
+  }
+}
+
 crvq_status launch_gemm(tc::GemmArgs g, int64_t chunks, cudaStream_t stream) {
   static bool attr_set[64] = {};
   int dev = 0;
@@ -74,14 +94,24 @@ crvq_status launch_tc_syrk(const float* X, int64_t n, int64_t N, float* S, cudaS
   unsigned* err = nullptr;
   CRVQ_TRY(device_error_word(&err));
   const int64_t chunks = ceil_div(n, kKChunk);
-  Scratch mem;
+  Scratch mem, xt_mem;
   float* P = S;
   if (chunks > 1) {
     CRVQ_TRY(mem.alloc((size_t)chunks * N * N * sizeof(float), stream));
     P = mem.as<float>();
   }
+  // X^T with rows padded to a multiple of 4 floats: both operands K-major, loaded with 16-byte
+  // loads (A(a, k) = X[k][a])
+  const int64_t ldt = (n + 3) / 4 * 4;
+  CRVQ_TRY(xt_mem.alloc((size_t)N * ldt * sizeof(float), stream));
+  {
+    ProfScope ps("hessian_transpose", stream, 8.0 * (double)n * N);
+    transpose_kernel<<<dim3((unsigned)ceil_div(ldt, 32), (unsigned)ceil_div(N, 32)), 256, 0,
+                       stream>>>(X, n, N, xt_mem.as<float>(), ldt);
+    CRVQ_LAUNCHED();
+  }
   tc::GemmArgs g{};
-  g.A = tc::Operand{X, N, N, false};  // A(a, k) = X[k][a]
+  g.A = tc::Operand{xt_mem.as<float>(), ldt, N, true};
   g.B = g.A;
   g.K = n;
   g.k_chunk = kKChunk;

@@ -7,9 +7,10 @@
 // lo parts are ~2^-22 relative), accumulated in fp32 by the tensor core.
 //
 // CTA tile 128 x 256 (one tcgen05.mma M = 128, N = 256, K = 8 per instruction), K staged 16
-// at a time through two shared-memory stages. All 128 threads load and split the next stage
-// while the tensor core works on the previous one; thread 0 issues the MMAs and commits them
-// to the stage's mbarrier. Operands sit in shared memory in the canonical K-major layout
+// at a time through two shared-memory stages. All 128 threads split and store a stage while
+// the tensor core works on the previous one, with the global loads of the next stage already
+// in flight in registers (software pipeline); thread 0 issues the MMAs and commits them to the
+// stage's mbarrier. Operands sit in shared memory in the canonical K-major layout
 // without swizzle: 8-row x 16-byte core matrices, consecutive along K (LBO = 128 B), 8-row
 // groups SBO = (BK / 4) * 128 B apart. Every wait on an mbarrier is bounded (~2 s of
 // %globaltimer); on expiry the kernel records ERRBIT_TIMEOUT, stops issuing and exits
@@ -43,44 +44,53 @@ struct Operand {
   bool kmajor;
 };
 
-// Loads rows [r0, r0 + R) x k [k0, k0 + kBK) of the operand, splits each value into tf32
-// hi / lo and stores both tiles (zero outside the matrix). Thread t handles rows t, t + 128...
+// Loads rows [r0, r0 + R) x k [k0, k0 + kBK) of the operand into registers (zero outside the
+// matrix). Thread t handles rows t, t + 128, ...
 template <int R>
-__device__ __forceinline__ void load_split(const Operand& op, int64_t r0, int64_t k0,
-                                           int64_t K, char* hi, char* lo) {
+__device__ __forceinline__ void load_tile(const Operand& op, int64_t r0, int64_t k0, int64_t K,
+                                          float v[R / kThreads][kBK]) {
 #pragma unroll
   for (int rr = 0; rr < R / kThreads; ++rr) {
     const int r = threadIdx.x + rr * kThreads;
     const int64_t row = r0 + r;
-    float v[kBK];
     if (row < op.rows) {
       if (op.kmajor) {
         const float* src = op.p + row * op.ld + k0;
         if (k0 + kBK <= K && (op.ld & 3) == 0 && ((uintptr_t)op.p & 15) == 0) {
 #pragma unroll
           for (int q = 0; q < kBK / 4; ++q) {
-            const float4 x = reinterpret_cast<const float4*>(src)[q];
-            v[4 * q] = x.x; v[4 * q + 1] = x.y; v[4 * q + 2] = x.z; v[4 * q + 3] = x.w;
+            const float4 x = __ldg(reinterpret_cast<const float4*>(src) + q);
+            v[rr][4 * q] = x.x; v[rr][4 * q + 1] = x.y; v[rr][4 * q + 2] = x.z; v[rr][4 * q + 3] = x.w;
           }
         } else {
 #pragma unroll
-          for (int q = 0; q < kBK; ++q) v[q] = (k0 + q < K) ? src[q] : 0.f;
+          for (int q = 0; q < kBK; ++q) v[rr][q] = (k0 + q < K) ? src[q] : 0.f;
         }
       } else {
 #pragma unroll
-        for (int q = 0; q < kBK; ++q) v[q] = (k0 + q < K) ? op.p[(k0 + q) * op.ld + row] : 0.f;
+        for (int q = 0; q < kBK; ++q)
+          v[rr][q] = (k0 + q < K) ? op.p[(k0 + q) * op.ld + row] : 0.f;
       }
     } else {
 #pragma unroll
-      for (int q = 0; q < kBK; ++q) v[q] = 0.f;
+      for (int q = 0; q < kBK; ++q) v[rr][q] = 0.f;
     }
+  }
+}
+
+// Splits the loaded values into tf32 hi / lo and stores both tiles.
+template <int R>
+__device__ __forceinline__ void split_store(const float v[R / kThreads][kBK], char* hi, char* lo) {
+#pragma unroll
+  for (int rr = 0; rr < R / kThreads; ++rr) {
+    const int r = threadIdx.x + rr * kThreads;
 #pragma unroll
     for (int q = 0; q < kBK / 4; ++q) {
       uint32_t h[4], l[4];
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
-        h[j] = to_tf32(v[4 * q + j]);
-        l[j] = to_tf32(v[4 * q + j] - __uint_as_float(h[j]));
+        h[j] = to_tf32(v[rr][4 * q + j]);
+        l[j] = to_tf32(v[rr][4 * q + j] - __uint_as_float(h[j]));
       }
       const uint32_t off = tile_off(r, 4 * q);
       *reinterpret_cast<uint4*>(hi + off) = make_uint4(h[0], h[1], h[2], h[3]);
@@ -140,8 +150,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemm3xtf32_kernel(GemmArgs a) {
   const uint32_t tmem = *tmem_slot;
 
   const int64_t nkt = (kend - kbeg + kBK - 1) / kBK;
-  uint32_t waits[kStages] = {0, 0};
+  uint32_t par = 0;  // parity of the next wait per stage (bit = stage)
   bool ok = true;
+  // Software pipeline: the global loads of step kt + 1 are in flight while step kt is split,
+  // stored and multiplied.
+  float va[kBM / kThreads][kBK], vb[kBN / kThreads][kBK];
+  if (nkt > 0) {
+    load_tile<kBM>(a.A, m0, kbeg, kend, va);
+    load_tile<kBN>(a.B, n0, kbeg, kend, vb);
+  }
   for (int64_t kt = 0; kt < nkt; ++kt) {
     const int s = (int)(kt & 1);
     char* st = smem + s * kStageBytes;
@@ -151,13 +168,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemm3xtf32_kernel(GemmArgs a) {
     char* b_lo = b_hi + kBStageBytes;
     if (kt >= kStages) {
       // the MMAs issued two stages ago read this buffer: wait for them (bounded)
-      if (ok) ok = mbar_wait(smem_u32(&bars[s]), waits[s] & 1, a.err);
-      ++waits[s];
+      if (ok) ok = mbar_wait(smem_u32(&bars[s]), (par >> s) & 1u, a.err);
+      par ^= 1u << s;
     }
     ok = __syncthreads_and(ok);
     if (!ok) break;
-    load_split<kBM>(a.A, m0, kbeg + kt * kBK, kend, a_hi, a_lo);
-    load_split<kBN>(a.B, n0, kbeg + kt * kBK, kend, b_hi, b_lo);
+    split_store<kBM>(va, a_hi, a_lo);
+    split_store<kBN>(vb, b_hi, b_lo);
+    if (kt + 1 < nkt) {
+      load_tile<kBM>(a.A, m0, kbeg + (kt + 1) * kBK, kend, va);
+      load_tile<kBN>(a.B, n0, kbeg + (kt + 1) * kBK, kend, vb);
+    }
     fence_async_smem();
     __syncthreads();
     if (threadIdx.x == 0) {
@@ -180,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm3xtf32_kernel(GemmArgs a) {
   // wait for the last commit (it covers every earlier MMA of this thread)
   if (ok && nkt > 0) {
     const int s = (int)((nkt - 1) & 1);
-    ok = mbar_wait(smem_u32(&bars[s]), waits[s] & 1, a.err);
+    ok = mbar_wait(smem_u32(&bars[s]), (par >> s) & 1u, a.err);
   }
   ok = __syncthreads_and(ok);
   tc_fence_after();
