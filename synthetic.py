@@ -19,6 +19,9 @@ from __future__ import annotations
 import dataclasses
 from dataclasses import dataclass, field
 
+import os
+from concurrent.futures import ThreadPoolExecutor
+
 import numpy as np
 
 _GAMMA = np.uint64(0x9E3779B97F4A7C15)
@@ -117,9 +120,23 @@ class LayerConfig:
         return dataclasses.replace(self, **kw)
 
 
+def _by_row_chunks(fn, n_rows: int, chunk: int = 2048) -> np.ndarray:
+    """fn(rows) over row chunks on a thread pool (numpy releases the GIL in its loops). The
+    generators are counter-based, so every element depends only on its own indices and the
+    chunked result equals the one-shot one."""
+    if n_rows <= chunk:
+        return fn(np.arange(n_rows))
+    parts = [np.arange(r0, min(n_rows, r0 + chunk)) for r0 in range(0, n_rows, chunk)]
+    workers = min(len(parts), os.cpu_count() or 1, 16)
+    with ThreadPoolExecutor(max_workers=workers) as ex:
+        return np.ascontiguousarray(np.concatenate(list(ex.map(fn, parts)), axis=0))
+
+
 def gen_W(cfg: LayerConfig, rows: np.ndarray | None = None) -> np.ndarray:
     """Weights: N(0, 0.02^2), with the configured outlier columns; fp32 M x N (or a row subset)."""
-    rows = np.arange(cfg.M) if rows is None else np.asarray(rows)
+    if rows is None:
+        return _by_row_chunks(lambda r: gen_W(cfg, r), cfg.M)
+    rows = np.asarray(rows)
     s = stream_key(cfg.seed, cfg.name + "/W")
     W = 0.02 * _matrix_normals(s, rows, cfg.N)
     if cfg.w_kind == "outlier_cols":
@@ -142,7 +159,9 @@ def gen_W(cfg: LayerConfig, rows: np.ndarray | None = None) -> np.ndarray:
 
 def gen_X(cfg: LayerConfig, rows: np.ndarray | None = None) -> np.ndarray:
     """Calibration activations: n_tok x N fp32, row = token, per-channel LogNormal scales."""
-    rows = np.arange(cfg.n_tok) if rows is None else np.asarray(rows)
+    if rows is None:
+        return _by_row_chunks(lambda r: gen_X(cfg, r), cfg.n_tok)
+    rows = np.asarray(rows)
     tag = cfg.x_tag or cfg.name
     s_scale = stream_key(cfg.seed, tag + "/X/scale")
     scale = np.exp(cfg.x_sigma * normal(s_scale, np.arange(cfg.N)))
