@@ -7,7 +7,9 @@ with beam re-encode, losses), i.e. one crvq_quantize_layer call, on the LLaMA-2-
 q_proj workload (W 4096 x 4096, 4096 calibration tokens, d = 8, K = 256, 1 extended codebook
 on 2% channels, B = 8, 10 Lloyd iterations). The metric is code-search throughput: scored
 (hypothesis, codeword) pairs per second over the whole step; the per-layer time is reported
-beside it.
+beside it. `--config c5` makes a step the seven matrices of a LLaMA-2-7B decoder block
+(q, k, v, o, gate, up 4096-wide inputs sharing one X; down_proj 11008-wide with its own X),
+and reports the block time as well.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl crvq|reference] [--config c2]
 
@@ -122,18 +124,52 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def cpu_oracle_sample(cfg, rows, X=None):
-    """Times the fp64 oracle's whole schedule on the first `rows` rows of the workload's W
-    (same X). Returns (scores/s, seconds, cores used)."""
+# Rough fp64-oracle throughput on a few host cores, only to size the CPU samples below.
+ORACLE_RATE_EST = 1.5e7
+
+
+def cpu_oracle_sample(cfg, X=None, budget_s=20.0, max_rows=64):
+    """Times the fp64 oracle, as it stands, on a bounded sample of the workload (about
+    `budget_s` of CPU work). The whole schedule on the first rows of W (full X) when enough rows
+    for K fit the budget; otherwise (a 65536-entry codebook needs 65536 vectors) one encode
+    pass, the schedule's dominant step, of the first rows over the first 32 groups against a
+    seeded K_base-entry codebook. Returns (scores/s, seconds, cores used, description)."""
     from oracle import crvq_oracle as O
-    W = S.gen_W(cfg, np.arange(rows))
+    d = cfg.d
+    G = cfg.N // d
+    Gc = O.n_crit_groups(cfg.N, d, cfg.crit_frac)
+    need = max(cfg.K_base / G, cfg.K_ext / Gc if cfg.n_ext > 0 and Gc > 0 else 0.0)
+    per_row = schedule_scores(cfg, 1, cfg.N)
+    fit = int(budget_s * ORACLE_RATE_EST / per_row)
+    rows = min(cfg.M, max(int(np.ceil(need)), min(fit, max_rows)))
     X = S.gen_X(cfg) if X is None else X
-    t0, c0 = time.perf_counter(), time.process_time()
-    O.quantize_layer(W, X, cfg)
-    wall = time.perf_counter() - t0
+    c0 = time.process_time()
+    if rows >= need and per_row * rows <= 3.0 * budget_s * ORACLE_RATE_EST:
+        W = S.gen_W(cfg, np.arange(rows))
+        t0 = time.perf_counter()
+        O.quantize_layer(W, X, cfg)
+        wall = time.perf_counter() - t0
+        sc = schedule_scores(cfg, rows, cfg.N)
+        desc = f"whole schedule on rows 0..{rows - 1} of {cfg.name} (full X)"
+    else:
+        gs = min(G, 32)
+        _, _, Hb, _ = O.hessian(np.ascontiguousarray(X[:, :gs * d]), cfg.damp_rel, d)
+        C = np.random.default_rng(0).normal(0.0, 0.02, (cfg.K_base, d)).astype(np.float32)
+        W1 = np.ascontiguousarray(S.gen_W(cfg, np.arange(1))[:, :gs * d])
+        t0 = time.perf_counter()                       # one row sizes the sample
+        O.encode_beam(W1, d, Hb, [O.Codebook(C, None, gs)], 0, 1)
+        t1 = time.perf_counter() - t0
+        rows = max(1, min(cfg.M, max_rows, int(budget_s / max(t1, 1e-6))))
+        W = np.ascontiguousarray(S.gen_W(cfg, np.arange(rows))[:, :gs * d])
+        c0 = time.process_time()
+        t0 = time.perf_counter()
+        O.encode_beam(W, d, Hb, [O.Codebook(C, None, gs)], 0, 1)
+        wall = time.perf_counter() - t0
+        sc = float(rows) * gs * cfg.K_base
+        desc = (f"one encode pass of rows 0..{rows - 1} x groups 0..{gs - 1} of {cfg.name} "
+                f"against a seeded {cfg.K_base}-entry codebook")
     cpu = time.process_time() - c0
-    sc = schedule_scores(cfg, rows, cfg.N)
-    return sc / wall, wall, max(1, int(round(cpu / max(wall, 1e-9))))
+    return sc / wall, wall, max(1, int(round(cpu / max(wall, 1e-9)))), desc
 
 
 def dist_init():
@@ -151,29 +187,31 @@ def _cuda_ok():
     return torch.cuda.is_available()
 
 
-def run_reference(args, cfg, ws, rank):
-    """Reference arm: the fp64 CPU oracle on a bounded row sample, rank 0 only."""
+def run_reference(args, layers, ws, rank):
+    """Reference arm: the fp64 CPU oracle on a bounded sample of the workload's first matrix
+    (sized so the whole run stays within a few minutes), rank 0 only."""
     if rank != 0:
         return
+    cfg = layers[0]
     X = S.gen_X(cfg)
-    rows = args.ref_rows
+    budget = min(20.0, max(2.0, 150.0 / max(1, args.steps + (args.warmup if args.ref_warmup
+                                                              else 0))))
     for _ in range(args.warmup if args.ref_warmup else 0):
-        cpu_oracle_sample(cfg, rows, X)
-    times, cores = [], 1
+        cpu_oracle_sample(cfg, X, budget, args.ref_rows)
+    tot, sc_tot, cores, desc = 0.0, 0.0, 1, ""
     for _ in range(args.steps):
-        _, wall, cores = cpu_oracle_sample(cfg, rows, X)
-        times.append(wall)
-    sc = schedule_scores(cfg, rows, cfg.N)
-    tot = sum(times)
-    value = sc * len(times) / tot
+        v, wall, cores, desc = cpu_oracle_sample(cfg, X, budget, args.ref_rows)
+        tot += wall
+        sc_tot += v * wall
+    value = sc_tot / tot
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "scores/s",
         "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": 1e3 * tot / len(times), "higher_is_better": True, "scaling": "weak",
+        "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": DATA,
-        "config": config_dict(cfg, rows_note=f"row sample: first {rows} of {cfg.M} rows"),
+        "config": workload_dict(args.config, layers, rows_note=desc),
         "cpu_baseline": {"value": value, "unit": "scores/s", "cores": cores, "kind": "oracle",
-                         "sample": f"whole schedule on rows 0..{rows - 1} of W, full X"},
+                         "sample": desc},
         "e2e": {"value": value, "unit": "scores/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -196,22 +234,43 @@ def config_dict(cfg, rows_note=None):
     return c
 
 
+def workload_dict(name, layers, rows_note=None):
+    """config of the JSON line: the layer's settings, or the block's matrices."""
+    if len(layers) == 1:
+        return config_dict(layers[0], rows_note)
+    c = config_dict(layers[0], rows_note)
+    c["workload"] = "c5_llama2_7b_decoder_block (7 matrices, one step = the whole block)"
+    c["matrices"] = [{"name": L.name.split("/")[-1], "M": L.M, "N": L.N} for L in layers]
+    c["shared_X"] = "q,k,v,o,gate,up share one 4096 x 4096 X; down_proj its own 4096 x 11008"
+    for k in ("M", "N"):
+        c.pop(k)
+    return c
+
+
+def workload_layers(name):
+    """The matrices one step quantizes: one layer, or the seven matrices of the decoder block."""
+    if name == "c5":
+        return list(S.C5)
+    return [S.CONFIGS[name]]
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="crvq", choices=["crvq", "reference"])
-    ap.add_argument("--config", default="c2", choices=sorted(S.CONFIGS))
-    ap.add_argument("--ref-rows", type=int, default=64)
+    ap.add_argument("--config", default="c2", choices=sorted(S.CONFIGS) + ["c5"])
+    ap.add_argument("--ref-rows", type=int, default=64,
+                    help="most rows a whole-schedule oracle sample takes beyond what K needs")
     ap.add_argument("--ref-warmup", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
     args = ap.parse_args()
-    cfg = S.CONFIGS[args.config]
+    layers = workload_layers(args.config)
     ws, rank, local = dist_init()
     if args.impl == "reference":
-        run_reference(args, cfg, ws, rank)
+        run_reference(args, layers, ws, rank)
         return
 
     import torch
@@ -220,17 +279,38 @@ def main():
     B.build()
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    cfg_r = cfg.with_(seed=cfg.seed + rank)                # each rank: its own layer
-    Wn, Xn = S.gen_W(cfg_r), S.gen_X(cfg_r)
-    W_h = torch.from_numpy(Wn).pin_memory()
-    X_h = torch.from_numpy(Xn).pin_memory()
-    W_d, X_d = W_h.to(dev), X_h.to(dev)
+    # each rank quantizes its own matrices; layers of a block that share X share one buffer
+    xs = {}
+    work = []
+    for cfg in layers:
+        cfg_r = cfg.with_(seed=cfg.seed + rank)
+        tag = cfg_r.x_tag or cfg_r.name
+        if tag not in xs:
+            Xn = S.gen_X(cfg_r)
+            X_h = torch.from_numpy(Xn).pin_memory()
+            xs[tag] = (Xn, X_h, X_h.to(dev))
+        Xn, X_h, X_d = xs[tag]
+        W_h = torch.from_numpy(S.gen_W(cfg_r)).pin_memory()
+        work.append({"cfg": cfg_r, "W_h": W_h, "W_d": W_h.to(dev), "X_h": X_h, "X_d": X_d,
+                     "Xn": Xn, "out": None, "h_out": None})
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
 
-    out = None
+    def run_step(host=False):
+        """One step: every matrix of the workload through crvq_quantize_layer. Returns the
+        scores of the step."""
+        sc = 0.0
+        for w in work:
+            if host:
+                w["h_out"] = P.crvq_quantize_layer(w["W_h"], w["X_h"], w["cfg"], out=w["h_out"])
+                sc += w["h_out"].report["scores"]
+            else:
+                w["out"] = P.crvq_quantize_layer(w["W_d"], w["X_d"], w["cfg"], out=w["out"])
+                sc += w["out"].report["scores"]
+        return sc
+
     for _ in range(args.warmup):
-        out = P.crvq_quantize_layer(W_d, X_d, cfg_r, out=out)
+        run_step()
     torch.cuda.synchronize()
 
     def barrier():
@@ -239,18 +319,17 @@ def main():
             dist.barrier()
         torch.cuda.synchronize()
 
-    clocks = ClockSampler(torch.cuda.get_device_properties(dev).uuid
-                          if hasattr(torch.cuda.get_device_properties(dev), "uuid") else local)
+    clocks = ClockSampler(local)
     try:
         clocks.gpu_id = "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
     except Exception:
         clocks.gpu_id = local
     # events only around the arg-min launches (the roofline kernel): the other launches of
-    # the timed steps run unbracketed. The library replays a captured CUDA graph of the layer
-    # per profiling state; one untimed call captures the one the timed steps use.
+    # the timed steps run unbracketed. The library replays a captured CUDA graph of each
+    # matrix per profiling state; one untimed step captures the ones the timed steps use.
     P.crvq_profile_filter("encode_argmin")
     P.crvq_profile_begin()
-    out = P.crvq_quantize_layer(W_d, X_d, cfg_r, out=out)
+    run_step()
     torch.cuda.synchronize()
     P.crvq_profile_end()
     barrier()
@@ -264,11 +343,10 @@ def main():
         a = torch.cuda.Event(enable_timing=True)
         b = torch.cuda.Event(enable_timing=True)
         a.record(stream)
-        out = P.crvq_quantize_layer(W_d, X_d, cfg_r, out=out)
+        scores += run_step()
         b.record(stream)
         b.synchronize()
         step_ms.append(a.elapsed_time(b))
-        scores += out.report["scores"]
     barrier()
     argmin_stats = [k for k in P.crvq_profile_end()
                     if k["name"] in ("encode_argmin", "encode_argmin_lloyd")]
@@ -277,7 +355,7 @@ def main():
     # per-kernel breakdown: one more step, untimed, every launch bracketed
     P.crvq_profile_filter(None)
     P.crvq_profile_begin()
-    out = P.crvq_quantize_layer(W_d, X_d, cfg_r, out=out)
+    run_step()
     torch.cuda.synchronize()
     kstats = P.crvq_profile_end()
     tot_ms = sum(step_ms)
@@ -293,22 +371,26 @@ def main():
     value = scores_all / (tot_ms_max / 1e3)
 
     # End to end through the public C ABI with host buffers (pinned): H2D of W and X and D2H
-    # of every output inside the timed region, wall clock around a synchronizing call.
+    # of every output inside the timed region, wall clock around synchronizing calls.
     e2e_times = []
-    h_out = None
+    e2e_scores = 0.0
     for i in range(args.e2e_steps + 1 if args.e2e_steps > 0 else 0):
         t0 = time.perf_counter()
-        h_out = P.crvq_quantize_layer(W_h, X_h, cfg_r, out=h_out)
+        sc = run_step(host=True)
         dt = time.perf_counter() - t0
         if i > 0:
             e2e_times.append(dt)
+            e2e_scores = sc
     e2e = None
     if e2e_times:
-        h2d = W_h.numel() * 4 + X_h.numel() * 4
-        d2h = sum(t.numel() * t.element_size() for t in
-                  [h_out.perm, h_out.C_base, h_out.codes_base, h_out.C_ext, h_out.codes_ext,
-                   h_out.W_hat, h_out.importance] if t is not None) + 48
-        e2e = {"value": ws * h_out.report["scores"] / statistics.mean(e2e_times),
+        h2d = sum(w["W_h"].numel() * 4 + w["X_h"].numel() * 4 for w in work)
+        d2h = 0
+        for w in work:
+            o = w["h_out"]
+            d2h += sum(t.numel() * t.element_size() for t in
+                       [o.perm, o.C_base, o.codes_base, o.C_ext, o.codes_ext, o.W_hat,
+                        o.importance] if t is not None) + 48
+        e2e = {"value": ws * e2e_scores / statistics.mean(e2e_times),
                "unit": "scores/s", "h2d_bytes_per_step": int(h2d),
                "d2h_bytes_per_step": int(d2h),
                "ms_per_step": 1e3 * statistics.mean(e2e_times)}
@@ -320,7 +402,6 @@ def main():
     nsm = props.multi_processor_count
     ks = sorted(kstats, key=lambda k: -k["ms"])
     total_k = sum(k["ms"] for k in ks) or 1.0
-    top = ks[0]
     # The dominant kernel is the tensor-core arg-min: tcgen05 computes every certified score
     # bound (a 3xTF32 dot product of length 32), and its epilogue keeps the two smallest of
     # each row with four integer ALU operations per score (key packing, min, max, min). The
@@ -336,7 +417,7 @@ def main():
     tensor_tflops = enc_units * 64.0 / (enc_ms / 1e3) / 1e12 if enc_ms > 0 else 0.0
     roof = {"kernel": "encode_argmin (all passes)", "bound": "alu", "achieved": achieved,
             "peak": alu_peak, "unit": "TOP/s", "frac": achieved / alu_peak,
-            "traffic": ARGMIN_TRAFFIC,
+            "traffic": ARGMIN_TRAFFIC if args.config == "c2" else None,
             "peak_source": f"{nsm} SMs x 64 ALU lanes x {mhz:.0f} MHz (sm_max_mhz, {peak_src})",
             "work": "4 integer ALU ops per scored (vector, codeword) pair",
             "avg_launch_ms": enc_ms / max(enc_launches, 1), "launches": enc_launches,
@@ -344,28 +425,34 @@ def main():
                        "peak": tf32_peak, "frac": tensor_tflops / tf32_peak,
                        "work": "64 tf32 flop per scored pair (K = 32 split operands)",
                        "peak_source": f"0.5 x bf16 {peak_src} ({peaks.get('bf16_tflops')})"}}
+    last = work[-1]["out"].report if len(work) == 1 else None
     line = {
         "metric": METRIC, "value": value, "unit": "scores/s", "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": tot_ms_max / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-        "data": DATA, "config": config_dict(cfg),
-        "layer_time_s": tot_ms_max / args.steps / 1e3,
-        "losses": {k: out.report[k] for k in ("loss_pre", "loss_block", "loss_crit",
-                                              "loss_full")},
+        "data": DATA, "config": workload_dict(args.config, layers),
+        "layer_time_s": tot_ms_max / args.steps / 1e3 / len(work),
         "roofline": roof,
         "e2e": e2e,
         "gpu_launches": int(launches),
-        "fp64_fallback_decisions_per_step": out.report["flagged"],
+        "fp64_fallback_decisions_per_step": sum(w["out"].report["flagged"] for w in work),
         "kernels": [{"name": k["name"], "launches": k["launches"], "ms": k["ms"],
                      "share": k["ms"] / total_k} for k in ks[:12]],
         "clocks": clk,
     }
+    if last is not None:
+        line["losses"] = {k: last[k] for k in ("loss_pre", "loss_block", "loss_crit",
+                                                "loss_full")}
+    else:
+        line["block_time_s"] = tot_ms_max / args.steps / 1e3
+        line["losses"] = {w["cfg"].name: {k: w["out"].report[k] for k in
+                                          ("loss_pre", "loss_block", "loss_crit", "loss_full")}
+                          for w in work}
     if ws == 1 and not args.no_cpu_baseline:
-        rows = args.ref_rows
-        v, wall, cores = cpu_oracle_sample(cfg_r, rows, Xn)
+        w0 = work[0]
+        v, wall, cores, desc = cpu_oracle_sample(w0["cfg"], w0["Xn"], 20.0, args.ref_rows)
         line["cpu_baseline"] = {"value": v, "unit": "scores/s", "cores": cores, "kind": "oracle",
-                                "sample": f"whole schedule on rows 0..{rows - 1} of W "
-                                          f"(full X), {wall:.1f} s"}
+                                "sample": f"{desc}, {wall:.1f} s"}
     print(json.dumps(line), flush=True)
 
 

@@ -128,6 +128,26 @@ crvq_status crvq_hessian(const float* X, int64_t n_tok, int64_t N, int32_t d, fl
                          crvq_stream_t stream);
 
 /*
+ * S1 / S3 without the dense H: the diagonal d x d blocks of H = X^T X / n_tok + delta I (as
+ * crvq_hessian defines it) for the channel order `perm`:
+ *   H_blocks[g][a][b] = H[perm[g*d + a]][perm[g*d + b]]   (perm NULL: the stored order).
+ * The method reads H only through these blocks (the vector scores of Sec. 3.1 under the
+ * block-diagonal reading of the Alg. 1 loss) and its diagonal (App. A.2 importance), so a
+ * layer needs N * n_tok floats of scratch here instead of the N x N matrix. The values equal
+ * crvq_hessian's dense H entries bit for bit (same tensor-core products, same split-K order).
+ *   X        [n_tok x N] device, 16-byte aligned.
+ *   perm     [N] device int32 channel order, or NULL. Entries outside [0, N) are reported as
+ *            CRVQ_ERR_DEVICE by crvq_sync (the affected block rows are left unwritten).
+ *   xsq      [N] out or NULL: the undamped diagonal, stored order.
+ *   delta    [1] out or NULL.
+ *   H_blocks [(N/d) x d x d] out.
+ * Requires n_tok >= 1, N >= 1, N % d == 0, damp_rel >= 0 and finite; d = 8.
+ */
+crvq_status crvq_hessian_blocks(const float* X, int64_t n_tok, int64_t N, int32_t d,
+                                float damp_rel, const int32_t* perm, float* xsq, float* delta,
+                                float* H_blocks, crvq_stream_t stream);
+
+/*
  * S3. Channel importance and reordering (Alg. 1 ComputeImportance, ReorderChannels;
  * Sec. 4.1-4.2; App. A.2).
  *   mode W-A:    I_i = 1/2 * xsq_i * max_j (W_ji - W_pre_ji)^2 (App. A.2 form; W_pre is the
@@ -299,7 +319,7 @@ typedef struct crvq_layer_report {
  * When W, X and every output are device pointers and refine_rounds <= 1, the schedule has no
  * host synchronisation inside: it is captured into a CUDA graph on the first call for a given
  * (device, stream, shapes, configuration, pointers, profiling state) and replayed on later
- * calls, which reads the current contents of W and X (up to 4 graphs are kept per process,
+ * calls, which reads the current contents of W and X (up to 16 graphs are kept per process,
  * least recently used evicted; their scratch stays reserved while they are kept). Setting
  * CRVQ_GRAPHS=0 in the environment runs every call directly. Results are identical either way.
  */

@@ -144,6 +144,26 @@ def crvq_hessian(X, damp_rel, d=8, H=None, xsq=None, H_blocks=None, delta=None, 
     return H, xsq, H_blocks, delta
 
 
+def crvq_hessian_blocks(X, damp_rel, d=8, perm=None, xsq=None, delta=None, H_blocks=None,
+                        stream=None):
+    """S1 / S3 blocks only: returns (H_blocks in the order perm (None: stored order), xsq,
+    delta[1]) without forming the dense N x N H."""
+    _need(X, torch.float32, "X")
+    X = X.contiguous()
+    n, N = X.shape
+    dev = X.device
+    if perm is not None:
+        _need(perm, torch.int32, "perm")
+    xsq = torch.empty(N, device=dev, dtype=torch.float32) if xsq is None else xsq
+    delta = torch.empty(1, device=dev, dtype=torch.float32) if delta is None else delta
+    if H_blocks is None:
+        H_blocks = torch.empty((N // d, d, d), device=dev, dtype=torch.float32)
+    _check(_L().crvq_hessian_blocks(_ptr(X), n, N, d, float(damp_rel),
+                                    _ptr(perm), _ptr(xsq),
+                                    _ptr(delta), _ptr(H_blocks), _stream(stream, dev)))
+    return H_blocks, xsq, delta
+
+
 def crvq_select_reorder_channels(W, d, W_pre, xsq, H, crit_frac, mode=IMPORTANCE_WA, seed=0,
                                  stream=None):
     """S3: returns (perm, importance, W_sorted, H_blocks, n_crit_groups)."""

@@ -331,6 +331,41 @@ crvq_status crvq_hessian(const float* X, int64_t n_tok, int64_t N, int32_t d, fl
                         (cudaStream_t)stream);
 }
 
+crvq_status crvq_hessian_blocks(const float* X, int64_t n_tok, int64_t N, int32_t d,
+                                float damp_rel, const int32_t* perm, float* xsq, float* delta,
+                                float* H_blocks, crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_TRY(check_d(d));
+  CRVQ_CHECK_ARG(X && H_blocks, "X and H_blocks must not be NULL");
+  CRVQ_CHECK_ARG(n_tok >= 1 && N >= 1 && N % d == 0, "need n_tok >= 1, N >= 1, N %% d == 0");
+  CRVQ_CHECK_ARG(N <= INT32_MAX, "N must fit in int32");
+  CRVQ_CHECK_ARG(std::isfinite(damp_rel) && damp_rel >= 0.f, "damp_rel must be finite, >= 0");
+  CRVQ_CHECK_ARG(aligned16(X), "X must be 16-byte aligned");
+  cudaStream_t s = (cudaStream_t)stream;
+  const int64_t ldt = (n_tok + 3) / 4 * 4;
+  Scratch mXt, md64, mxsq, mHb;
+  CRVQ_TRY(mXt.alloc((size_t)N * ldt * sizeof(float), s));
+  CRVQ_TRY(md64.alloc(sizeof(double), s));
+  float* Xt = mXt.as<float>();
+  double* delta64 = md64.as<double>();
+  if (!xsq) {
+    CRVQ_TRY(mxsq.alloc((size_t)N * sizeof(float), s));
+    xsq = mxsq.as<float>();
+  }
+  float* Hb0 = H_blocks;
+  if (perm) {
+    CRVQ_TRY(mHb.alloc((size_t)N * d * sizeof(float), s));
+    Hb0 = mHb.as<float>();
+  }
+  CRVQ_TRY(launch_transpose(X, n_tok, N, Xt, ldt, s));
+  CRVQ_TRY(launch_tc_hessian_blocks(Xt, ldt, n_tok, N, nullptr, false, damp_rel, xsq, delta,
+                                    delta64, Hb0, s));
+  if (perm)
+    CRVQ_TRY(launch_tc_hessian_blocks(Xt, ldt, n_tok, N, perm, true, 0.f, nullptr, nullptr,
+                                      delta64, H_blocks, s));
+  return CRVQ_OK;
+}
+
 int64_t crvq_n_crit_groups(int64_t N, int32_t d, float crit_frac) {
   if (d <= 0 || N <= 0 || !(crit_frac > 0.f)) return 0;
   const int64_t G = N / d;
@@ -554,10 +589,16 @@ crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, i
   ex.scores = &scores;
   ex.flag_total = flag_total;
 
-  Buf bH, bxsq, bHb0, bdelta, bC0, bcodes0, bWpre, bWs, bHb;
-  float *H, *xsq, *Hb0, *delta, *C0, *Wpre, *Ws, *Hb;
+  // Only the 8 x 8 diagonal blocks of H (original and sorted order) and its diagonal are read,
+  // so the dense N x N product is never formed: X^T is kept from S1 to S3 and each order's
+  // blocks are taken on the tensor cores from it (the same values as the dense H's).
+  const int64_t ldt = (n_tok + 3) / 4 * 4;
+  Buf bXt, bd64, bxsq, bHb0, bdelta, bC0, bcodes0, bWpre, bWs, bHb;
+  float *Xt, *xsq, *Hb0, *delta, *C0, *Wpre, *Ws, *Hb;
+  double* delta64;
   int32_t* codes0;
-  CRVQ_TRY(bH.get(&H, (size_t)N * N, s));
+  CRVQ_TRY(bXt.get(&Xt, (size_t)N * ldt, s));
+  CRVQ_TRY(bd64.get(&delta64, 1, s));
   CRVQ_TRY(bxsq.get(&xsq, N, s));
   CRVQ_TRY(bHb0.get(&Hb0, (size_t)G * d * d, s));
   CRVQ_TRY(bdelta.get(&delta, 4, s));
@@ -567,8 +608,10 @@ crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, i
   CRVQ_TRY(bWs.get(&Ws, (size_t)M * N, s));
   CRVQ_TRY(bHb.get(&Hb, (size_t)G * d * d, s));
 
-  // S1: Hessian proxy
-  CRVQ_TRY(launch_hessian(X, n_tok, N, d, cfg->damp_rel, H, xsq, Hb0, delta, s));
+  // S1: Hessian proxy (diagonal blocks, xsq and delta)
+  CRVQ_TRY(launch_transpose(X, n_tok, N, Xt, ldt, s));
+  CRVQ_TRY(launch_tc_hessian_blocks(Xt, ldt, n_tok, N, nullptr, false, cfg->damp_rel, xsq,
+                                    delta, delta64, Hb0, s));
   // S2: prequantize in the original order (Alg. 1 line 3)
   {
     SetView set{W, N, M, G, Hb0};
@@ -582,8 +625,10 @@ crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, i
                                       Wpre, losses + 3, s));
   }
   // S3: importance and reordering (Alg. 1 lines 4-5)
-  CRVQ_TRY(launch_select_reorder(W, M, N, d, Wpre, xsq, H, cfg->importance_mode,
-                                 phase_seed(cfg->seed, 4, 0), o.perm, o.imp, Ws, Hb, s));
+  CRVQ_TRY(launch_select_reorder(W, M, N, d, Wpre, xsq, nullptr, cfg->importance_mode,
+                                 phase_seed(cfg->seed, 4, 0), o.perm, o.imp, Ws, nullptr, s));
+  CRVQ_TRY(launch_tc_hessian_blocks(Xt, ldt, n_tok, N, o.perm, true, 0.f, nullptr, nullptr,
+                                    delta64, Hb, s));
   // S4: base codebook over all vectors (Alg. 1 lines 6-7)
   CbList all{};
   all.n = 1 + cfg->n_ext;
@@ -687,7 +732,7 @@ struct LayerGraph {
   CapturedEvents events;                    // arg-min event nodes when captured while profiling
   uint64_t used = 0;
 };
-constexpr int kGraphs = 4;
+constexpr int kGraphs = 16;  // a 7-matrix decoder block in both profiling states
 std::mutex g_graph_mu;
 std::vector<LayerGraph*> g_graphs;
 uint64_t g_graph_clock = 0;

@@ -858,6 +858,107 @@ argmin_exact_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs, i
 }
 
 
+// Exact decision of flagged rows, one warp per row, for codebooks of up to kExactWarpK
+// entries: the bounds and fp32-pair scores of argmin_exact_kernel without block barriers.
+// Lane l takes codewords l, l + 32, ...; the fp32 upper bounds give U, every codeword whose
+// lower bound reaches U is scored in fp32 pairs by the lane that holds it, and the best
+// (value, index) is reduced across the warp with the same total order, so the decision is the
+// one argmin_exact_kernel makes.
+constexpr int kExactWarpK = 1024;
+
+__global__ void __launch_bounds__(128)
+argmin_exact_warp_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs,
+                         int n_fixed, int s_idx, int32_t* __restrict__ out_code, int64_t out_ld,
+                         int64_t out_g0, FlagList flags, StatsView st,
+                         const float4* __restrict__ terms, unsigned* err) {
+  __shared__ float sHw[4][kD * kD];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const unsigned cnt = min((unsigned long long)*flags.count, (unsigned long long)flags.cap);
+  if (flags.total && blockIdx.x == 0 && threadIdx.x == 0) atomicAdd(flags.total, cnt);
+  const CbView cw = cbs.cb[s_idx];
+  const float cmul = bound_mult(n_fixed);
+  float* sH = sHw[warp];
+  for (unsigned f = blockIdx.x * 4u + warp; f < cnt; f += gridDim.x * 4u) {
+    const int64_t vi = flags.vec[f];
+    const int64_t i = vi / G_range, grel = vi % G_range, g = g_begin + grel;
+    const float thr = flags.thr[f];
+    __syncwarp();
+    sH[lane] = set.Hb[g * kD * kD + lane];
+    sH[lane + 32] = set.Hb[g * kD * kD + lane + 32];
+    __syncwarp();
+    float rv[kD], av[kD], m2q[kD], pmax;
+    target32(set, cbs, n_fixed, i, g, rv, av, err);
+    vector_terms(rv, av, sH, m2q, pmax);
+    const float nbeta = -2.f * kU * cmul * pmax;
+    const float4* gt = terms ? terms + grel * cw.K : nullptr;
+    float U = thr;
+    for (int k = lane; k < cw.K; k += 32) {
+      float cv[kD], nn, na, l1;
+      load_vec(cw.C + (int64_t)k * kD, cv);
+      if (gt) {
+        const float4 t = gt[k];
+        nn = t.x;
+        na = t.y;
+        l1 = t.z;
+      } else {
+        codeword_terms(cv, sH, nn, na, l1);
+      }
+      U = fminf(U, up_from(nn, na, l1, cv, m2q, pmax, cmul));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) U = fminf(U, __shfl_xor_sync(0xffffffffu, U, o));
+    float rh[kD], rl[kD];
+    dfl::target(set, cbs, n_fixed, i, g, rh, rl, err);
+    float bh = INFINITY, bl = 0.f;
+    int bk = 0x7fffffff;
+    for (int k = lane; k < cw.K; k += 32) {
+      float cv[kD], nn, na, l1;
+      load_vec(cw.C + (int64_t)k * kD, cv);
+      if (gt) {
+        const float4 t = gt[k];
+        nn = t.x;
+        na = t.y;
+        l1 = t.z;
+      } else {
+        codeword_terms(cv, sH, nn, na, l1);
+      }
+      if (low_from(nn, na, l1, cv, m2q, nbeta, cmul) <= U) {
+        float eh, el;
+        dfl::quad_err(rh, rl, cv, sH, eh, el);
+        if (dfl::less(eh, el, k, bh, bl, bk)) {
+          bh = eh;
+          bl = el;
+          bk = k;
+        }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float oh = __shfl_xor_sync(0xffffffffu, bh, o);
+      const float ol = __shfl_xor_sync(0xffffffffu, bl, o);
+      const int ok = __shfl_xor_sync(0xffffffffu, bk, o);
+      if (dfl::less(oh, ol, ok, bh, bl, bk)) {
+        bh = oh;
+        bl = ol;
+        bk = ok;
+      }
+    }
+    if (lane == 0) {
+      if (bk == 0x7fffffff) {
+        raise_error(err, ERRBIT_NUMERIC);  // no candidate: non-finite scores
+      } else {
+        out_code[i * out_ld + (g - out_g0)] = bk;
+        if (st.cnt) {
+          float q[kD];
+#pragma unroll
+          for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[p];
+          stats_add(st, stats_scale_exp(*st.scale), g, bk, q);
+        }
+      }
+    }
+  }
+}
+
 // --------------------------------------------------------------------------- beam stages
 // Hypotheses of a vector: up to B partial tuples (codes of the first s+1 searched codebooks)
 // in rank order. hyp layout: [vector][B][S] int32; hyp_n[vector] = number kept.
@@ -1488,8 +1589,14 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
       }
       {
         ProfScope pf("encode_argmin_exact", stream, 0.0);
-        argmin_exact_kernel<<<(unsigned)std::min<int64_t>(nv, 16 * nsm), 128, 0, stream>>>(
-            set, gs, gn, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, tout, err);
+        if (cw.K <= kExactWarpK) {
+          argmin_exact_warp_kernel<<<(unsigned)std::min<int64_t>(ceil_div(nv, 4), 16 * nsm),
+                                     128, 0, stream>>>(set, gs, gn, cbs, n_fixed, s_idx, out,
+                                                       out_ld, out_g0, fl, st, tout, err);
+        } else {
+          argmin_exact_kernel<<<(unsigned)std::min<int64_t>(nv, 16 * nsm), 128, 0, stream>>>(
+              set, gs, gn, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, tout, err);
+        }
         CRVQ_LAUNCHED();
       }
     }

@@ -26,6 +26,17 @@ crvq_status launch_extract_blocks(const float* H, int64_t N, int d, const int32_
 // Tensor-core (tcgen05, 3xTF32) products.
 // S = X^T X / n for X n x N row-major (S N x N, both triangles).
 crvq_status launch_tc_syrk(const float* X, int64_t n, int64_t N, float* S, cudaStream_t stream);
+// Xt = X^T (N x ldt, columns [n, ldt) zero) for X n x N row-major.
+crvq_status launch_transpose(const float* X, int64_t n, int64_t N, float* Xt, int64_t ldt,
+                             cudaStream_t stream);
+// The 8 x 8 diagonal blocks of X^T X / n + delta I only, in the channel order perm (NULL: the
+// stored order), bit-identical to the blocks of launch_hessian's dense H. delta_known: the
+// damping is read from delta64; otherwise (stored order only) xsq, delta and delta64 are
+// written.
+crvq_status launch_tc_hessian_blocks(const float* Xt, int64_t ldt, int64_t n, int64_t N,
+                                     const int32_t* perm, bool delta_known, float damp_rel,
+                                     float* xsq, float* delta, double* delta64, float* Hb,
+                                     cudaStream_t stream);
 // Partial sums of ||A B^T||_F^2 (A M x K, B Nb x K row-major) into part[0 .. *nparts).
 crvq_status launch_tc_sumsq(const float* A, int64_t M, const float* B, int64_t Nb, int64_t K,
                             double* part, int64_t part_cap, int64_t* nparts,

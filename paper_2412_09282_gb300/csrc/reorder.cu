@@ -168,7 +168,7 @@ crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
   ProfScope ps("reorder_gather", stream, (double)M * N * 8.0);
   gather_cols_kernel<<<blocks, 256, smem, stream>>>(W, M, N, perm, W_sorted, err);
   CRVQ_LAUNCHED();
-  CRVQ_TRY(launch_extract_blocks(H, N, d, perm, H_blocks, stream));
+  if (H_blocks) CRVQ_TRY(launch_extract_blocks(H, N, d, perm, H_blocks, stream));
   return CRVQ_OK;
 }
 

@@ -15,15 +15,64 @@ namespace {
 
 constexpr int64_t kKChunk = 1024;
 
-// out[e] = scale * sum_c P[c * stride + e]  (chunks in order)
+// scale * sum_c P[c * stride + e], chunks in order (the one rounding sequence every split-K
+// product of this file uses, so its dense and block-only forms agree bit for bit)
+__device__ __forceinline__ float chunk_sum(const float* __restrict__ P, int chunks,
+                                           int64_t stride, int64_t e, float scale) {
+  float s = 0.f;
+  for (int c = 0; c < chunks; ++c) s += P[c * stride + e];
+  return s * scale;
+}
+
 __global__ void __launch_bounds__(256)
 sum_partials_kernel(const float* __restrict__ P, int64_t count, int chunks, int64_t stride,
                     float scale, float* __restrict__ out) {
   for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < count;
+       e += (int64_t)gridDim.x * blockDim.x)
+    out[e] = chunk_sum(P, chunks, stride, e, scale);
+}
+
+// Original-order blocks, one CTA: xsq[i] = the undamped diagonal, delta = damp_rel * mean(xsq)
+// by the dense path's fixed-order fp64 reduction (1024 strided partials, then a tree), and the
+// blocks with delta added on their diagonals (rounded once from fp64, as the dense path does).
+__global__ void __launch_bounds__(1024)
+blocks_finalize_kernel(const float* __restrict__ P, int chunks, int64_t stride, float scale,
+                       int64_t N, float damp_rel, float* __restrict__ xsq,
+                       float* __restrict__ delta_out, double* __restrict__ delta64,
+                       float* __restrict__ Hb) {
+  __shared__ double part[1024];
+  double s = 0.0;
+  for (int64_t i = threadIdx.x; i < N; i += blockDim.x) {
+    const float v = chunk_sum(P, chunks, stride, i * 8 + (i & 7), scale);
+    xsq[i] = v;
+    s += (double)v;
+  }
+  part[threadIdx.x] = s;
+  __syncthreads();
+  for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+    if ((int)threadIdx.x < w) part[threadIdx.x] += part[threadIdx.x + w];
+    __syncthreads();
+  }
+  const double delta = (double)damp_rel * (part[0] / (double)N);
+  for (int64_t e = threadIdx.x; e < N * 8; e += blockDim.x) {
+    const float v = chunk_sum(P, chunks, stride, e, scale);
+    Hb[e] = ((e >> 3) & 7) == (e & 7) ? (float)((double)v + delta) : v;
+  }
+  if (threadIdx.x == 0) {
+    if (delta_out) *delta_out = (float)delta;
+    *delta64 = delta;
+  }
+}
+
+// Blocks of a given channel order with a known delta.
+__global__ void __launch_bounds__(256)
+blocks_damp_kernel(const float* __restrict__ P, int chunks, int64_t stride, float scale,
+                   int64_t N, const double* __restrict__ delta64, float* __restrict__ Hb) {
+  const double delta = *delta64;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < N * 8;
        e += (int64_t)gridDim.x * blockDim.x) {
-    float s = 0.f;
-    for (int c = 0; c < chunks; ++c) s += P[c * stride + e];
-    out[e] = s * scale;
+    const float v = chunk_sum(P, chunks, stride, e, scale);
+    Hb[e] = ((e >> 3) & 7) == (e & 7) ? (float)((double)v + delta) : v;
   }
 }
 
@@ -104,12 +153,7 @@ crvq_status launch_tc_syrk(const float* X, int64_t n, int64_t N, float* S, cudaS
   // loads (A(a, k) = X[k][a])
   const int64_t ldt = (n + 3) / 4 * 4;
   CRVQ_TRY(xt_mem.alloc((size_t)N * ldt * sizeof(float), stream));
-  {
-    ProfScope ps("hessian_transpose", stream, 8.0 * (double)n * N);
-    transpose_kernel<<<dim3((unsigned)ceil_div(ldt, 32), (unsigned)ceil_div(N, 32)), 256, 0,
-                       stream>>>(X, n, N, xt_mem.as<float>(), ldt);
-    CRVQ_LAUNCHED();
-  }
+  CRVQ_TRY(launch_transpose(X, n, N, xt_mem.as<float>(), ldt, stream));
   tc::GemmArgs g{};
   g.A = tc::Operand{xt_mem.as<float>(), ldt, N, true};
   g.B = g.A;
@@ -167,6 +211,68 @@ crvq_status launch_tc_sumsq(const float* A, int64_t M, const float* B, int64_t N
   sumsq_partials_kernel<<<blocks, 256, 0, stream>>>(P, M * Nb, (int)chunks, M * Nb, part);
   CRVQ_LAUNCHED();
   *nparts = blocks;
+  return CRVQ_OK;
+}
+
+crvq_status launch_transpose(const float* X, int64_t n, int64_t N, float* Xt, int64_t ldt,
+                             cudaStream_t stream) {
+  ProfScope ps("hessian_transpose", stream, 8.0 * (double)n * N);
+  transpose_kernel<<<dim3((unsigned)ceil_div(ldt, 32), (unsigned)ceil_div(N, 32)), 256, 0,
+                     stream>>>(X, n, N, Xt, ldt);
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
+}
+
+// Diagonal 8 x 8 blocks of X^T X / n (+ delta I) for the channel order `perm` (NULL = the
+// stored order), from Xt = X^T (N x ldt, ldt a multiple of 4). delta_known: delta64 (fp64) is
+// read; otherwise perm must be NULL and xsq, delta (float, may be NULL) and delta64 are
+// written. The entries equal those of launch_tc_syrk's dense S plus the damping bit for bit.
+crvq_status launch_tc_hessian_blocks(const float* Xt, int64_t ldt, int64_t n, int64_t N,
+                                     const int32_t* perm, bool delta_known, float damp_rel,
+                                     float* xsq, float* delta, double* delta64, float* Hb,
+                                     cudaStream_t stream) {
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
+  static bool attr_set[64] = {};
+  int dev = 0;
+  CRVQ_CUDA(cudaGetDevice(&dev));
+  if (dev < 64 && !attr_set[dev]) {
+    CRVQ_CUDA(cudaFuncSetAttribute(tc::syrk_diag_kernel,
+                                   cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                   tc::kDiagSmemBytes));
+    attr_set[dev] = true;
+  }
+  const int64_t chunks = std::max<int64_t>(1, ceil_div(n, kKChunk));
+  const int64_t stride = N * 8;
+  Scratch mem;
+  CRVQ_TRY(mem.alloc((size_t)chunks * stride * sizeof(float), stream));
+  tc::DiagArgs a{};
+  a.A = tc::Operand{Xt, ldt, N, true, perm};
+  a.K = n;
+  a.k_chunk = kKChunk;
+  a.out = mem.as<float>();
+  a.chunk_stride = stride;
+  a.alpha = chunks > 1 ? 1.f : (float)(1.0 / (double)n);
+  a.err = err;
+  const float scale = chunks > 1 ? (float)(1.0 / (double)n) : 1.f;
+  {
+    ProfScope ps(perm ? "reorder_blocks_tc" : "hessian_blocks_tc", stream,
+                 6.0 * (double)n * N * tc::kBM);
+    dim3 grid((unsigned)ceil_div(N, tc::kBM), (unsigned)chunks);
+    tc::syrk_diag_kernel<<<grid, tc::kThreads, tc::kDiagSmemBytes, stream>>>(a);
+    CRVQ_LAUNCHED();
+  }
+  ProfScope ps("hessian_blocks_finalize", stream, (double)chunks * stride * 4.0);
+  if (!delta_known) {
+    if (perm) return fail(CRVQ_ERR_UNSUPPORTED, "hessian blocks: delta needs the stored order");
+    blocks_finalize_kernel<<<1, 1024, 0, stream>>>(mem.as<float>(), (int)chunks, stride, scale,
+                                                   N, damp_rel, xsq, delta, delta64, Hb);
+  } else {
+    const int blocks = (int)std::min<int64_t>(ceil_div(stride, 256), 4 * sm_count());
+    blocks_damp_kernel<<<blocks, 256, 0, stream>>>(mem.as<float>(), (int)chunks, stride, scale,
+                                                   N, delta64, Hb);
+  }
+  CRVQ_LAUNCHED();
   return CRVQ_OK;
 }
 

@@ -233,8 +233,8 @@ __device__ bool solve8_refined(const double A[36], const double b[kD], double x[
 // A_k c_k = b_k (b_k from the fixed point) by refined Cholesky. The fixed assignment and
 // order make the result identical on every run. Codewords without members keep their old
 // value.
-constexpr int kSolveK = 4;
-constexpr int kSolveSlices = 4;
+constexpr int kSolveK = 1;        // one codeword per CTA: K CTAs share the GPU
+constexpr int kSolveSlices = 16;  // groups split 16 ways: short dependent chains per thread
 constexpr int kSolveThreads = kSolveK * kSolveSlices * kNA;  // 592
 
 __global__ void __launch_bounds__(kSolveThreads)

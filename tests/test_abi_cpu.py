@@ -63,6 +63,11 @@ def test_validation_rejects_before_launch(lib):
     assert lib.crvq_hessian(dummy, 4, 12, 8, 0.0, dummy, dummy, None, None, None) == -1
     # negative damping
     assert lib.crvq_hessian(dummy, 4, 16, 8, -1.0, dummy, dummy, None, None, None) == -1
+    # blocks-only Hessian: same rules, H_blocks required
+    assert lib.crvq_hessian_blocks(None, 1, 8, 16, 0.0, None, None, None, None, None) == -2
+    assert lib.crvq_hessian_blocks(dummy, 4, 16, 8, 0.0, None, None, None, None, None) == -1
+    assert lib.crvq_hessian_blocks(dummy, 4, 12, 8, 0.0, None, None, None, dummy, None) == -1
+    assert lib.crvq_hessian_blocks(dummy, 0, 16, 8, 0.0, None, None, None, dummy, None) == -1
     # beam width beyond the implemented maximum
     from paper_2412_09282_gb300 import _lib
     cb = (_lib.crvq_codebook * 1)()

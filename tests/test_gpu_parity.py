@@ -5,7 +5,9 @@ Bars: code indices and permutations bit-exact except fp64 near-ties (relative ma
 1e-6 of err_best + t^T H t, or importance gaps below 1e-6 of max I); codebooks within 1e-4 of
 the codebook's max |value|; losses within 1e-4 relative; H within 2e-5 * sqrt(H_aa H_bb)
 (3xTF32 tensor-core products accumulated in fp32 over chunks of at most 1024 tokens, chunks
-summed in fp64: about 1e-6 typical, under 1e-5 including the accumulator's rounding bias); reconstructions bit-exact (fp64 sums of fp32 codewords rounded once on both sides).
+summed in fp32 in chunk order: about 1e-6 typical, under 1e-5 including the accumulator's
+rounding bias); reconstructions bit-exact (fp64 sums of fp32 codewords rounded once on both
+sides).
 """
 import numpy as np
 import pytest
@@ -59,6 +61,42 @@ def test_hessian_parity(n, N):
     np.testing.assert_array_equal(host(Hb), np.stack(
         [Hg[g * D:(g + 1) * D, g * D:(g + 1) * D] for g in range(N // D)]))
     assert np.array_equal(Hg, Hg.T)
+
+
+@pytest.mark.parametrize("n,N", [(1024, 512), (77, 136), (300, 8), (2500, 264), (4096, 1032)])
+def test_hessian_blocks_equal_dense_blocks(n, N):
+    """The blocks-only path (no N x N matrix) returns the dense H's diagonal blocks bit for bit,
+    in the stored order and through a channel permutation (1, 3 and 4 token chunks; a ragged
+    last 128-channel tile), with the same xsq and delta."""
+    cfg = S.C1.with_(name=f"hessb_{n}_{N}", n_tok=n, N=N)
+    X = S.gen_X(cfg)
+    Xd = dev(X)
+    H, xsq, Hb, delta = P.crvq_hessian(Xd, cfg.damp_rel, D)
+    Hb2, xsq2, delta2 = P.crvq_hessian_blocks(Xd, cfg.damp_rel, D)
+    perm = np.random.default_rng(n + N).permutation(N).astype(np.int32)
+    Hb3, xsq3, delta3 = P.crvq_hessian_blocks(Xd, cfg.damp_rel, D, perm=dev(perm))
+    _sync()
+    Hg = host(H)
+    np.testing.assert_array_equal(host(Hb2), host(Hb))
+    for a in (xsq2, xsq3):
+        np.testing.assert_array_equal(host(a), host(xsq))
+    for a in (delta2, delta3):
+        np.testing.assert_array_equal(host(a), host(delta))
+    want = np.stack([Hg[np.ix_(perm[g * D:(g + 1) * D], perm[g * D:(g + 1) * D])]
+                     for g in range(N // D)])
+    np.testing.assert_array_equal(host(Hb3), want)
+
+
+def test_hessian_blocks_reports_out_of_range_channel():
+    cfg = S.C1.with_(name="hessb_bad", n_tok=64, N=64)
+    X = dev(S.gen_X(cfg))
+    perm = np.arange(64, dtype=np.int32)
+    perm[5] = 64
+    P.crvq_hessian_blocks(X, cfg.damp_rel, D, perm=dev(perm))
+    with pytest.raises(P.CrvqError):
+        P.crvq_sync()
+    P.crvq_hessian_blocks(X, cfg.damp_rel, D)   # the context is still usable
+    P.crvq_sync()
 
 
 # ------------------------------------------------------------------------------ S3 reorder
