@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstring>
 #include <mutex>
+#include <type_traits>
 #include <string>
 #include <vector>
 
@@ -762,9 +763,17 @@ bool same_key(const LayerGraph& e, int dev, cudaStream_t st, int64_t M, int64_t 
          (!prof || strncmp(e.filter, g_filter, sizeof(e.filter)) == 0);
 }
 
+// A device-to-host copy enqueued after a replay, before its synchronisation.
+struct HostCopy {
+  void* dst;
+  const void* src;
+  size_t bytes;
+};
+
 crvq_status run_graph(const float* W, const float* X, int64_t M, int64_t N, int64_t n_tok,
                       const crvq_config* cfg, int64_t Gc, const LayerDev& o,
-                      crvq_layer_report* report, cudaStream_t s, bool* done) {
+                      crvq_layer_report* report, cudaStream_t s, bool* done,
+                      const HostCopy* d2h = nullptr, int n_d2h = 0) {
   *done = false;
   int dev = 0;
   CRVQ_CUDA(cudaGetDevice(&dev));
@@ -835,6 +844,9 @@ crvq_status run_graph(const float* W, const float* X, int64_t M, int64_t N, int6
   unsigned long long flagged = 0;
   CRVQ_CUDA(cudaMemcpyAsync(hl, e->losses, sizeof(hl), cudaMemcpyDeviceToHost, s));
   CRVQ_CUDA(cudaMemcpyAsync(&flagged, e->flag_total, sizeof(flagged), cudaMemcpyDeviceToHost, s));
+  for (int q = 0; q < n_d2h; ++q)
+    if (d2h[q].bytes)
+      CRVQ_CUDA(cudaMemcpyAsync(d2h[q].dst, d2h[q].src, d2h[q].bytes, cudaMemcpyDeviceToHost, s));
   CRVQ_CUDA(cudaStreamSynchronize(s));
   if (prof && g_prof.load()) {  // the event nodes of this replay have completed
     std::lock_guard<std::mutex> lk2(g_pmu);
@@ -849,6 +861,92 @@ crvq_status run_graph(const float* W, const float* X, int64_t M, int64_t N, int6
   fill_report(report, hl, flagged, e->scores, e->rounds);
   *done = true;
   return CRVQ_OK;
+}
+
+// Persistent device staging for layers called with host inputs or outputs: the host data is
+// copied into buffers that outlive the call, so that the graph captured on them (keyed by
+// pointers) is replayed by later calls of the same shapes, as for device buffers. Up to
+// kStagings sets are kept (least recently used freed; never one a call is using).
+struct Staging {
+  int dev = -1;
+  int64_t M = 0, N = 0, n_tok = 0, K_base = 0, n_ext = 0, K_ext = 0, Gc = 0;
+  float *W = nullptr, *X = nullptr, *C_base = nullptr, *C_ext = nullptr, *W_hat = nullptr,
+        *imp = nullptr;
+  int32_t *perm = nullptr, *codes_base = nullptr, *codes_ext = nullptr;
+  uint64_t used = 0;
+  int users = 0;
+};
+constexpr int kStagings = 4;
+std::mutex g_stage_mu;
+std::vector<Staging*> g_stagings;
+uint64_t g_stage_clock = 0;
+
+void free_staging(Staging* sg) {
+  for (void* p : {(void*)sg->W, (void*)sg->X, (void*)sg->C_base, (void*)sg->C_ext,
+                  (void*)sg->W_hat, (void*)sg->imp, (void*)sg->perm, (void*)sg->codes_base,
+                  (void*)sg->codes_ext})
+    if (p) cudaFree(p);
+  cudaGetLastError();
+  delete sg;
+}
+
+crvq_status acquire_staging(int dev, int64_t M, int64_t N, int64_t n_tok, const crvq_config* cfg,
+                            int64_t Gc, Staging** out) {
+  std::lock_guard<std::mutex> lk(g_stage_mu);
+  const int d = cfg->d;
+  for (auto* sg : g_stagings)
+    if (sg->dev == dev && sg->M == M && sg->N == N && sg->n_tok == n_tok &&
+        sg->K_base == cfg->K_base && sg->n_ext == cfg->n_ext &&
+        sg->K_ext == (cfg->n_ext ? cfg->K_ext : 0) && sg->Gc == Gc && sg->users == 0) {
+      sg->used = ++g_stage_clock;
+      sg->users = 1;
+      *out = sg;
+      return CRVQ_OK;
+    }
+  if ((int)g_stagings.size() >= kStagings) {
+    int lru = -1;
+    for (int q = 0; q < (int)g_stagings.size(); ++q)
+      if (g_stagings[q]->users == 0 && (lru < 0 || g_stagings[q]->used < g_stagings[lru]->used))
+        lru = q;
+    if (lru >= 0) {
+      free_staging(g_stagings[lru]);
+      g_stagings.erase(g_stagings.begin() + lru);
+    }
+  }
+  Staging* sg = new Staging;
+  sg->dev = dev;
+  sg->M = M;
+  sg->N = N;
+  sg->n_tok = n_tok;
+  sg->K_base = cfg->K_base;
+  sg->n_ext = cfg->n_ext;
+  sg->K_ext = cfg->n_ext ? cfg->K_ext : 0;
+  sg->Gc = Gc;
+  const int64_t G = N / d;
+  bool ok = cudaMalloc(&sg->W, (size_t)M * N * 4) == cudaSuccess &&
+            cudaMalloc(&sg->X, (size_t)n_tok * N * 4) == cudaSuccess &&
+            cudaMalloc(&sg->C_base, (size_t)cfg->K_base * d * 4) == cudaSuccess &&
+            cudaMalloc(&sg->W_hat, (size_t)M * N * 4) == cudaSuccess &&
+            cudaMalloc(&sg->imp, (size_t)N * 4) == cudaSuccess &&
+            cudaMalloc(&sg->perm, (size_t)N * 4) == cudaSuccess &&
+            cudaMalloc(&sg->codes_base, (size_t)M * G * 4) == cudaSuccess;
+  if (ok && cfg->n_ext > 0)
+    ok = cudaMalloc(&sg->C_ext, (size_t)cfg->n_ext * cfg->K_ext * d * 4) == cudaSuccess &&
+         cudaMalloc(&sg->codes_ext, (size_t)cfg->n_ext * M * Gc * 4) == cudaSuccess;
+  if (!ok) {
+    free_staging(sg);
+    return fail(CRVQ_ERR_NOMEM, "staging buffers for a host-buffer layer call");
+  }
+  sg->used = ++g_stage_clock;
+  sg->users = 1;
+  g_stagings.push_back(sg);
+  *out = sg;
+  return CRVQ_OK;
+}
+
+void release_staging(Staging* sg) {
+  std::lock_guard<std::mutex> lk(g_stage_mu);
+  sg->users = 0;
 }
 
 }  // namespace
@@ -905,6 +1003,61 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
       report->n_crit_groups = Gc;
       return CRVQ_OK;
     }
+  } else if (cfg->refine_rounds <= 1 && graphs_enabled()) {
+    // Host inputs or outputs: the same graph replay on persistent staging buffers, with the
+    // host copies around it (device pointers of the caller are used in place).
+    const bool ok_align = (!is_device_ptr(W_in) || aligned16(W_in)) &&
+                          (!is_device_ptr(X_in) || aligned16(X_in)) &&
+                          (!is_device_ptr(out->C_base) || aligned16(out->C_base)) &&
+                          (cfg->n_ext == 0 || !is_device_ptr(out->C_ext) ||
+                           aligned16(out->C_ext)) &&
+                          (!out->W_hat || !is_device_ptr(out->W_hat) || aligned16(out->W_hat));
+    int dev = 0;
+    CRVQ_CUDA(cudaGetDevice(&dev));
+    Staging* sg = nullptr;
+    if (ok_align && acquire_staging(dev, M, N, n_tok, cfg, Gc, &sg) == CRVQ_OK) {
+      struct Release {
+        Staging* p;
+        ~Release() { release_staging(p); }
+      } rel{sg};
+      const float* Wd = W_in;
+      const float* Xd = X_in;
+      if (!is_device_ptr(W_in)) {
+        CRVQ_CUDA(cudaMemcpyAsync(sg->W, W_in, (size_t)M * N * 4, cudaMemcpyHostToDevice, s));
+        Wd = sg->W;
+      }
+      if (!is_device_ptr(X_in)) {
+        CRVQ_CUDA(cudaMemcpyAsync(sg->X, X_in, (size_t)n_tok * N * 4, cudaMemcpyHostToDevice,
+                                  s));
+        Xd = sg->X;
+      }
+      HostCopy cp[7];
+      int ncp = 0;
+      auto place = [&](auto* user, auto* stage, size_t count) {
+        using T = std::remove_pointer_t<decltype(stage)>;
+        if (!user) return (T*)nullptr;
+        if (is_device_ptr(user)) return (T*)user;
+        cp[ncp++] = HostCopy{(void*)user, (const void*)stage, count * sizeof(T)};
+        return stage;
+      };
+      LayerDev o{};
+      o.perm = place(out->perm, sg->perm, (size_t)N);
+      o.C_base = place(out->C_base, sg->C_base, (size_t)cfg->K_base * d);
+      o.codes_base = place(out->codes_base, sg->codes_base, (size_t)M * G);
+      if (cfg->n_ext) {
+        o.C_ext = place(out->C_ext, sg->C_ext, (size_t)cfg->n_ext * cfg->K_ext * d);
+        o.codes_ext = place(out->codes_ext, sg->codes_ext, (size_t)cfg->n_ext * M * Gc);
+      }
+      o.W_hat = place(out->W_hat, sg->W_hat, (size_t)M * N);
+      o.imp = out->importance ? place(out->importance, sg->imp, (size_t)N) : sg->imp;
+      bool done = false;
+      CRVQ_TRY(run_graph(Wd, Xd, M, N, n_tok, cfg, Gc, o, report, s, &done, cp, ncp));
+      if (done) {
+        report->n_crit_groups = Gc;
+        return CRVQ_OK;
+      }
+    }
+    clear_last_error();
   }
 
   // Direct path: host inputs / outputs are staged through device buffers.

@@ -485,7 +485,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   __syncthreads();
   tc::tc_fence_after();
   const uint32_t tmem = tmem_slot;
-  const int sexp = st.cnt ? stats_scale_exp(*st.scale) : 0;
+  const float sscale = st.cnt ? stats_scale_f(st) : 1.f;
 
   // Bound on Na_k over the codebook for this group: (max row sum |H_g|) L1max cinfmax.
   float hrow = 0.f;
@@ -705,9 +705,9 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
 #pragma unroll
           for (int p = 0; p < kD; ++p)
             atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[p * kTcSmemStatsK + j]),
-                      (unsigned long long)fix_rn(q[p], sexp));
+                      (unsigned long long)fix_rn_small(q[p], sscale));
         } else {
-          stats_add(st, sexp, g, j, q);
+          stats_add(st, sscale, g, j, q);
         }
       }
     }
@@ -850,7 +850,7 @@ argmin_exact_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs, i
           float q[kD];
 #pragma unroll
           for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[p];
-          stats_add(st, stats_scale_exp(*st.scale), g, bk, q);
+          stats_add(st, stats_scale_f(st), g, bk, q);
         }
       }
     }
@@ -952,7 +952,7 @@ argmin_exact_warp_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList c
           float q[kD];
 #pragma unroll
           for (int p = 0; p < kD; ++p) q[p] = -0.5f * m2q[p];
-          stats_add(st, stats_scale_exp(*st.scale), g, bk, q);
+          stats_add(st, stats_scale_f(st), g, bk, q);
         }
       }
     }

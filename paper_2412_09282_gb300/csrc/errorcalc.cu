@@ -51,10 +51,26 @@ __device__ __forceinline__ void recon(const CbList& cbs, int64_t i, int64_t g, f
   }
 }
 
+// Unevaluated fp32 pair (h, l) += x, and the merge of two pairs (TwoSum of the high parts).
+__device__ __forceinline__ void pair_add(float& h, float& l, float x) {
+  const float s = __fadd_rn(h, x);
+  const float bp = __fsub_rn(s, h);
+  const float e = __fadd_rn(__fsub_rn(h, __fsub_rn(s, bp)), __fsub_rn(x, bp));
+  h = s;
+  l = __fadd_rn(l, e);
+}
+
+__device__ __forceinline__ void pair_merge(float& h, float& l, float oh, float ol) {
+  pair_add(h, l, oh);
+  l = __fadd_rn(l, ol);
+}
+
 // One CTA per row (grid-strided): the row of W_hat and of dW = W - W_hat in the original
 // channel order (staged in shared memory, then stored with 16-byte writes), and the row's
 // block loss, critical loss and ||dW||^2. Each vector's terms are fp32 (the quadratic form as
-// two FMA chains); the thread's running sums and the row reduction are fp64.
+// two FMA chains); the thread's running sums and the row reduction are fp32 pairs in a fixed
+// order (about 2^-44 relative; a chain of dependent fp64 additions would cost about 180
+// cycles per step on this part), rounded to fp64 once per row.
 __global__ void __launch_bounds__(256)
 decode_row_kernel(const float* __restrict__ Ws, int64_t M, int64_t N, const float* __restrict__ Hb,
                   const int32_t* __restrict__ perm, CbList cbs, int64_t n_crit_groups,
@@ -63,11 +79,11 @@ decode_row_kernel(const float* __restrict__ Ws, int64_t M, int64_t N, const floa
   extern __shared__ __align__(16) float srow[];  // [N] W_hat row (if any), then [N] dW row
   float* s_hat = srow;
   float* s_dw = srow + (W_hat ? N : 0);
-  __shared__ double red[3][256 / 32];
+  __shared__ float red_h[3][256 / 32], red_l[3][256 / 32];
   const int64_t G = N / kD;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   for (int64_t i = blockIdx.x; i < M; i += gridDim.x) {
-    double lb = 0.0, lc = 0.0, sq = 0.0;
+    float lb = 0.f, lbl = 0.f, lc = 0.f, lcl = 0.f, sq = 0.f, sql = 0.f;
     __syncthreads();  // the previous row's stores have read the staging rows
     for (int64_t g = threadIdx.x; g < G; g += blockDim.x) {
       float r[kD], t[kD], dl[kD];
@@ -97,9 +113,9 @@ decode_row_kernel(const float* __restrict__ Ws, int64_t M, int64_t N, const floa
         hb = fmaf(dl[7], h1.w, hb);
         e = fmaf(hb, dl[a], e);
       }
-      lb += (double)e;
-      if (g < n_crit_groups) lc += (double)e;
-      sq += (double)q2;
+      pair_add(lb, lbl, e);
+      if (g < n_crit_groups) pair_add(lc, lcl, e);
+      pair_add(sq, sql, q2);
 #pragma unroll
       for (int j = 0; j < kD; ++j) {
         const int64_t p = g * kD + j;
@@ -127,36 +143,41 @@ decode_row_kernel(const float* __restrict__ Ws, int64_t M, int64_t N, const floa
     }
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
-      lb += __shfl_xor_sync(0xffffffffu, lb, off);
-      lc += __shfl_xor_sync(0xffffffffu, lc, off);
-      sq += __shfl_xor_sync(0xffffffffu, sq, off);
+      const float a0 = __shfl_xor_sync(0xffffffffu, lb, off);
+      const float a1 = __shfl_xor_sync(0xffffffffu, lbl, off);
+      const float b0 = __shfl_xor_sync(0xffffffffu, lc, off);
+      const float b1 = __shfl_xor_sync(0xffffffffu, lcl, off);
+      const float c0 = __shfl_xor_sync(0xffffffffu, sq, off);
+      const float c1 = __shfl_xor_sync(0xffffffffu, sql, off);
+      pair_merge(lb, lbl, a0, a1);
+      pair_merge(lc, lcl, b0, b1);
+      pair_merge(sq, sql, c0, c1);
     }
     if (lane == 0) {
-      red[0][warp] = lb;
-      red[1][warp] = lc;
-      red[2][warp] = sq;
+      red_h[0][warp] = lb;
+      red_l[0][warp] = lbl;
+      red_h[1][warp] = lc;
+      red_l[1][warp] = lcl;
+      red_h[2][warp] = sq;
+      red_l[2][warp] = sql;
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-      double a = 0.0, b = 0.0, c = 0.0;
-      for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
-        a += red[0][w];
-        b += red[1][w];
-        c += red[2][w];
-      }
-      row_part[i * 3 + 0] = a;
-      row_part[i * 3 + 1] = b;
-      row_part[i * 3 + 2] = c;
+    if (threadIdx.x < 3) {
+      const int q = threadIdx.x;
+      float h = red_h[q][0], l = red_l[q][0];
+      for (int w = 1; w < (int)(blockDim.x >> 5); ++w) pair_merge(h, l, red_h[q][w], red_l[q][w]);
+      row_part[i * 3 + q] = (double)h + (double)l;
     }
   }
 }
 
-__global__ void __launch_bounds__(256)
+// One CTA of 1024 threads (short dependent fp64 chains: strided partials, then a tree).
+__global__ void __launch_bounds__(1024)
 finalize_losses_kernel(const double* __restrict__ row_part, int64_t M,
                        const double* __restrict__ gemm_part, int64_t n_gemm, int64_t n_tok,
                        double delta_host, const float* __restrict__ delta_dev,
                        double* __restrict__ losses) {
-  __shared__ double red[4][256];
+  __shared__ double red[4][1024];
   double a = 0, b = 0, c = 0, e = 0;
   for (int64_t i = threadIdx.x; i < M; i += blockDim.x) {
     a += row_part[i * 3 + 0];
@@ -169,7 +190,7 @@ finalize_losses_kernel(const double* __restrict__ row_part, int64_t M,
   red[2][threadIdx.x] = c;
   red[3][threadIdx.x] = e;
   __syncthreads();
-  for (int w = 128; w > 0; w >>= 1) {
+  for (int w = 512; w > 0; w >>= 1) {
     if ((int)threadIdx.x < w)
       for (int q = 0; q < 4; ++q) red[q][threadIdx.x] += red[q][threadIdx.x + w];
     __syncthreads();
@@ -196,7 +217,8 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   unsigned* err = nullptr;
   CRVQ_TRY(device_error_word(&err));
   const int nsm = sm_count();
-  const int64_t n_gemm_cap = X ? 8 * (int64_t)nsm : 0;  // partial sums of the full loss
+  // partial sums of the full loss: one per 128 x 256 tile of dW X^T
+  const int64_t n_gemm_cap = X ? ceil_div(M, (int64_t)128) * ceil_div(n_tok, (int64_t)256) : 0;
   int64_t n_gemm = 0;
   // Scratch: dW (16-byte aligned for the 128-bit stores), then the fp64 partial sums.
   const size_t dW_bytes = X ? align_up((size_t)M * N * sizeof(float), 256) : 0;
@@ -225,7 +247,7 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   if (X) {
     CRVQ_TRY(launch_tc_sumsq(dW, M, X, n_tok, N, gemm_part, n_gemm_cap, &n_gemm, stream));
   }
-  finalize_losses_kernel<<<1, 256, 0, stream>>>(row_part, M, X ? gemm_part : nullptr, n_gemm,
+  finalize_losses_kernel<<<1, 1024, 0, stream>>>(row_part, M, X ? gemm_part : nullptr, n_gemm,
                                                 n_tok, damp_delta, delta_dev, losses_dev);
   CRVQ_LAUNCHED();
   return CRVQ_OK;

@@ -3,6 +3,7 @@
 // conversion it replaces.
 #pragma once
 
+#include <cmath>
 #include <cstdint>
 
 namespace crvq {
@@ -42,6 +43,19 @@ __host__ __device__ inline long long fix_rn(float q, int e) {
     r = q0 + ((rem > half || (rem == half && (q0 & 1u))) ? 1u : 0u);
   }
   return (b >> 31) ? -(long long)r : (long long)r;
+}
+
+// llrint(q * 2^e) when 2^e = scale is a normal fp32 number and |q * 2^e| < 2^31 (the
+// statistics scale keeps every term below 2^30): the product is exact, or below 2^-126 where
+// both give 0, and the conversion rounds half to even. Equals fix_rn(q, e) under those
+// conditions, in two instructions (an FMUL and a round-to-nearest F2I) instead of an integer
+// sequence with data-dependent branches.
+__host__ __device__ inline long long fix_rn_small(float q, float scale) {
+#ifdef __CUDA_ARCH__
+  return (long long)__float2int_rn(q * scale);
+#else
+  return (long long)std::lrintf(q * scale);  // default rounding: half to even
+#endif
 }
 
 }  // namespace crvq

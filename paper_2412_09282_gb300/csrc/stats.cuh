@@ -52,13 +52,19 @@ inline void stats_bind(void* base, int64_t G_cov, int K, StatsView* st) {
   st->K = K;
 }
 
-// 2^e with e the largest integer such that n * bound * 2^e < 2^62.
+// 2^e with e the largest integer such that every term stays below 2^30 (bound * 2^e < 2^30,
+// so that one fp32 multiply and one round-to-nearest conversion make it exact: fix_rn_small)
+// and no sum of n terms can overflow (n * bound * 2^e < 2^62); e within [-126, 126] so that
+// 2^e is a normal fp32 number. With terms resolved to 2^-30 of the bound, a sum's quantisation
+// error is far below the fp32 precision of its terms.
 __host__ __device__ inline double stats_scale_for(double bound, int64_t n) {
   const double lim = 4.611686018427387904e18;  // 2^62
   const double denom = bound * (double)(n > 0 ? n : 1);
   if (!(denom > 0.0)) return 1099511627776.0;  // 2^40: nothing to scale
-  const int e = (int)floor(log2(lim / denom));
-  return ldexp(1.0, e < -1000 ? -1000 : (e > 1000 ? 1000 : e));
+  int e = (int)floor(log2(lim / denom));
+  const int e_term = (int)floor(log2(1073741824.0 / bound));  // 2^30 / bound
+  if (e_term < e) e = e_term;
+  return ldexp(1.0, e < -126 ? -126 : (e > 126 ? 126 : e));
 }
 
 // tau = t - sum over the codebooks s != which that cover g of C_s[code] (fp32, codebook order).
@@ -102,13 +108,16 @@ __device__ __forceinline__ int stats_scale_exp(double scale) {
   return (int)((__double_as_longlong(scale) >> 52) & 0x7ff) - 1023;
 }
 
-__device__ __forceinline__ void stats_add(const StatsView& st, int sexp, int64_t g, int k,
+// The fixed-point scale as an fp32 number (an exact power of two in the normal range).
+__device__ __forceinline__ float stats_scale_f(const StatsView& st) { return (float)*st.scale; }
+
+__device__ __forceinline__ void stats_add(const StatsView& st, float scale, int64_t g, int k,
                                           const float q[kD]) {
   atomicAdd(&st.cnt[g * st.K + k], 1);
 #pragma unroll
   for (int j = 0; j < kD; ++j)
     atomicAdd(reinterpret_cast<unsigned long long*>(&st.bacc[(int64_t)k * kD + j]),
-              (unsigned long long)fix_rn(q[j], sexp));
+              (unsigned long long)fix_rn_small(q[j], scale));
 }
 
 // Solves A x = b for a symmetric positive definite 8 x 8 A given as its packed lower

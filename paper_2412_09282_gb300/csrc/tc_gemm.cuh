@@ -1,6 +1,6 @@
 // Tensor-core (tcgen05, sm_103a) fp32-accurate GEMM D = A B^T via the 3xTF32 split, with the
-// accumulator in tensor memory, used for the Hessian proxy X^T X (App. A.2) and for the full
-// loss ||dW X^T||^2 (Alg. 1 QuantLoss).
+// accumulator in tensor memory, used for the dense Hessian proxy X^T X (App. A.2) and, in a
+// block-diagonal form, for its d x d diagonal blocks alone.
 //
 // Each fp32 operand x is split into x_hi = tf32(x) and x_lo = tf32(x - x_hi); the product
 // uses a_hi b_hi + a_hi b_lo + a_lo b_hi (the dropped a_lo b_lo term and the rounding of the
@@ -106,13 +106,13 @@ __device__ __forceinline__ void split_store(const float v[R / kThreads][kBK], ch
 }
 
 // Epilogues.
-enum Mode { kStoreSymmetric = 0, kSumSquares = 1, kStore = 2 };
+enum Mode { kStoreSymmetric = 0, kStore = 2 };
 
 struct GemmArgs {
   Operand A, B;   // D[m][n] = sum_k A(m, k) B(n, k); M = A.rows, N = B.rows
   int64_t K;
   // Split K: blockIdx.y = chunk c covers k in [c * k_chunk, min(K, (c + 1) * k_chunk)) and
-  // writes to C + c * c_chunk_stride (kStore / kStoreSymmetric) or part + c * tiles.
+  // writes to C + c * c_chunk_stride.
   int64_t k_chunk;
   int64_t c_chunk_stride;
   int mode;
@@ -121,8 +121,6 @@ struct GemmArgs {
   float* C;
   int64_t ldc;
   float alpha;
-  // kSumSquares: part[tile] = sum over the tile of D^2 (fp64)
-  double* part;
   int tiles_n;    // tiles along N (grid is linear; tile = bm * tiles_n + bn)
   unsigned* err;
 };
@@ -133,7 +131,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm3xtf32_kernel(GemmArgs a) {
   char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kStages * kStageBytes);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kStages);
-  __shared__ double red[kThreads];
 
   const int tile = blockIdx.x;
   const int bm = tile / a.tiles_n, bn = tile % a.tiles_n;
@@ -212,7 +209,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm3xtf32_kernel(GemmArgs a) {
   ok = __syncthreads_and(ok);
   tc_fence_after();
 
-  double sq = 0.0;
   if (ok) {
     const int row = warp * 32 + lane;
     const int64_t m = m0 + row;
@@ -220,10 +216,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemm3xtf32_kernel(GemmArgs a) {
     for (int c0 = 0; c0 < kBN; c0 += 32) {
       float v[32];
       tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
-      if (a.mode == kSumSquares) {
-#pragma unroll
-        for (int j = 0; j < 32; ++j) sq += (double)v[j] * (double)v[j];
-      } else if (a.mode == kStore) {
+      if (a.mode == kStore) {
         if (m < a.A.rows) {
 #pragma unroll
           for (int j = 0; j < 32; ++j) {
@@ -243,16 +236,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemm3xtf32_kernel(GemmArgs a) {
         }
       }
     }
-  }
-  if (a.mode == kSumSquares) {
-    red[threadIdx.x] = sq;
-    __syncthreads();
-    for (int w = kThreads / 2; w > 0; w >>= 1) {
-      if ((int)threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
-      __syncthreads();
-    }
-    if (threadIdx.x == 0)
-      a.part[(int64_t)blockIdx.y * gridDim.x + tile] = ok ? red[0] : 0.0;
   }
   tc_fence_before();
   __syncthreads();

@@ -90,7 +90,7 @@ accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsign
                                                   // adding one component hit spread banks
   __shared__ int s_cnt[kSmemStatsK];
   const CbView cw = cbs.cb[which];
-  const int sexp = stats_scale_exp(*st.scale);
+  const float sscale = stats_scale_f(st);
   const bool smem = cw.K <= kSmemStatsK;
   for (int64_t g = blockIdx.y; g < cw.G_cov; g += gridDim.y) {
     if (smem) {
@@ -114,9 +114,9 @@ accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsign
 #pragma unroll
         for (int j = 0; j < kD; ++j)
           atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[j * kSmemStatsK + k]),
-                    (unsigned long long)fix_rn(q[j], sexp));
+                    (unsigned long long)fix_rn_small(q[j], sscale));
       } else {
-        stats_add(st, sexp, g, k, q);
+        stats_add(st, sscale, g, k, q);
       }
     }
     if (smem) {
@@ -184,55 +184,93 @@ __device__ inline void chol8_solve_f32(const float L[36], const float inv[kD], c
   }
 }
 
-// Solves A x = b (A packed lower triangle, fp64) by mixed-precision iterative refinement: an
-// fp32 Cholesky factor, then x += L^-T L^-1 (b - A x) with the residual in fp64 until the
-// correction is below 2^-40 of x (each step gains about -log2(cond(A) u_32) bits). A factor
-// that fails or a refinement that does not settle falls back to the fp64 Cholesky solve.
-__device__ bool solve8_refined(const double A[36], const double b[kD], double x[kD]) {
+__device__ __forceinline__ void pair_two_sum(float a, float b, float& s, float& e) {
+  s = __fadd_rn(a, b);
+  const float bp = __fsub_rn(s, a);
+  e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bp)), __fsub_rn(b, bp));
+}
+
+// Solves A x = b with A (packed lower triangle) and b given as unevaluated fp32 pairs
+// (hi + lo), by iterative refinement around an fp32 Cholesky factor: each step forms the
+// residual r = b - A x in fp32 pairs (every product split exactly by an FMA, TwoSum
+// accumulation, about 2^-44 relative), solves L L^T dx = r in fp32 and adds dx to x, which is
+// kept as a pair, until the correction is below 2^-40 of x (each step gains about
+// -log2(cond(A) u_32) bits) or after 12 steps. No fp64 arithmetic: a dependent fp64 operation
+// costs about 180 cycles on this part, and one thread solves each codeword. Returns false
+// when A has no fp32 Cholesky factor.
+__device__ bool solve8_pairs(const float Ah[36], const float Al[36], const float bh[kD],
+                             const float bl[kD], float x_out[kD]) {
   float Af[36], Lf[36], inv[kD];
 #pragma unroll
-  for (int e = 0; e < 36; ++e) Af[e] = (float)A[e];
-  if (chol8_f32(Af, Lf, inv)) {
-    float bf[kD], xf[kD];
+  for (int e = 0; e < 36; ++e) Af[e] = __fadd_rn(Ah[e], Al[e]);
+  if (!chol8_f32(Af, Lf, inv)) return false;
+  float bf[kD], xh[kD], xl[kD];
 #pragma unroll
-    for (int j = 0; j < kD; ++j) bf[j] = (float)b[j];
-    chol8_solve_f32(Lf, inv, bf, xf);
-#pragma unroll
-    for (int j = 0; j < kD; ++j) x[j] = (double)xf[j];
-    for (int it = 0; it < 6; ++it) {
-      float rf[kD], dx[kD];
-#pragma unroll
-      for (int r = 0; r < kD; ++r) {
-        double s = b[r];
-#pragma unroll
-        for (int c = 0; c < kD; ++c) {
-          const double a = r >= c ? A[r * (r + 1) / 2 + c] : A[c * (c + 1) / 2 + r];
-          s = fma(-a, x[c], s);
-        }
-        rf[r] = (float)s;
-      }
-      chol8_solve_f32(Lf, inv, rf, dx);
-      float xm = 0.f, dm = 0.f;
-#pragma unroll
-      for (int j = 0; j < kD; ++j) {
-        x[j] += (double)dx[j];
-        xm = fmaxf(xm, fabsf((float)x[j]));
-        dm = fmaxf(dm, fabsf(dx[j]));
-      }
-      if (dm <= 9.094947e-13f * xm) return true;  // 2^-40
-    }
+  for (int j = 0; j < kD; ++j) {
+    bf[j] = __fadd_rn(bh[j], bl[j]);
+    xl[j] = 0.f;
   }
-  return cholesky_solve8(A, b, x);
+  chol8_solve_f32(Lf, inv, bf, xh);
+  for (int it = 0; it < 12; ++it) {
+    float rf[kD];
+#pragma unroll
+    for (int r = 0; r < kD; ++r) {
+      float h = bh[r], l = bl[r];
+#pragma unroll
+      for (int c = 0; c < kD; ++c) {
+        const int q = r >= c ? r * (r + 1) / 2 + c : c * (c + 1) / 2 + r;
+        const float p = __fmul_rn(Ah[q], xh[c]);
+        const float pe = __fmaf_rn(Ah[q], xh[c], -p);  // Ah xh = p + pe exactly
+        const float cross = __fmaf_rn(Ah[q], xl[c], __fmul_rn(Al[q], xh[c]));
+        float sum, t;
+        pair_two_sum(h, -p, sum, t);
+        h = sum;
+        l = __fadd_rn(l, __fsub_rn(t, __fadd_rn(pe, cross)));
+      }
+      rf[r] = __fadd_rn(h, l);
+    }
+    float dx[kD];
+    chol8_solve_f32(Lf, inv, rf, dx);
+    float xm = 0.f, dm = 0.f;
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      float sum, t;
+      pair_two_sum(xh[j], dx[j], sum, t);
+      const float lo = __fadd_rn(xl[j], t);
+      xh[j] = __fadd_rn(sum, lo);                      // renormalise the pair
+      xl[j] = __fsub_rn(lo, __fsub_rn(xh[j], sum));
+      xm = fmaxf(xm, fabsf(xh[j]));
+      dm = fmaxf(dm, fabsf(dx[j]));
+    }
+    if (dm <= 9.094947e-13f * xm) break;  // 2^-40
+  }
+#pragma unroll
+  for (int j = 0; j < kD; ++j) x_out[j] = __fadd_rn(xh[j], xl[j]);
+  return true;
+}
+
+// b_j = bacc_j / 2^sexp as an fp32 pair: the int64 fixed-point sum split into three exact
+// 24-bit pieces, added by TwoSum, scaled by a power of two.
+__device__ __forceinline__ void fixed_to_pair(long long v, int sexp, float& h, float& l) {
+  const int a2 = (int)(v >> 48);                    // |a2| < 2^15
+  const int a1 = (int)((v >> 24) & 0xffffff);
+  const int a0 = (int)(v & 0xffffff);
+  float s, t;
+  pair_two_sum((float)a2 * 281474976710656.f, (float)a1 * 16777216.f, s, t);  // 2^48, 2^24
+  float s2, t2;
+  pair_two_sum(s, (float)a0, s2, t2);
+  h = ldexpf(s2, -sexp);
+  l = ldexpf(__fadd_rn(t, t2), -sexp);
 }
 
 // The least-squares solve of every codeword, one kernel. CTA = kSolveK codewords; thread =
 // (codeword, entry e of A_k's packed lower triangle or the count, slice of the groups). Each
 // thread sums cnt[g][k] * H_g[e] over its slice as an unevaluated fp32 pair (every product is
 // split exactly: cnt < 2^24; TwoSum for the high part), so no fp64 arithmetic runs per group;
-// the slices are added in a fixed order in fp64; then one thread per codeword solves
-// A_k c_k = b_k (b_k from the fixed point) by refined Cholesky. The fixed assignment and
-// order make the result identical on every run. Codewords without members keep their old
-// value.
+// the slices are added in a fixed order as fp32 pairs; then one thread per codeword solves
+// A_k c_k = b_k (b_k from the fixed point) by Cholesky with refinement in fp32 pairs. The
+// fixed assignment and order make the result identical on every run. Codewords without
+// members keep their old value.
 constexpr int kSolveK = 1;        // one codeword per CTA: K CTAs share the GPU
 constexpr int kSolveSlices = 16;  // groups split 16 ways: short dependent chains per thread
 constexpr int kSolveThreads = kSolveK * kSolveSlices * kNA;  // 592
@@ -240,7 +278,7 @@ constexpr int kSolveThreads = kSolveK * kSolveSlices * kNA;  // 592
 __global__ void __launch_bounds__(kSolveThreads)
 stats_solve_kernel(const float* __restrict__ Hb, StatsView st, const float* C_old, float* C_out,
                    int32_t* __restrict__ counts_out, unsigned* err) {
-  __shared__ double part[kSolveK][kSolveSlices][kNA];
+  __shared__ float part_h[kSolveK][kSolveSlices][kNA], part_l[kSolveK][kSolveSlices][kNA];
   const int tid = threadIdx.x;
   const int kk = tid / (kSolveSlices * kNA);
   const int sl = (tid / kNA) % kSolveSlices;
@@ -278,31 +316,53 @@ stats_solve_kernel(const float* __restrict__ Hb, StatsView st, const float* C_ol
       }
     }
   }
-  part[kk][sl][e] = (double)hi + (double)lo;
+  // Slices are merged per entry by its own thread in fp32 pairs (TwoSum of the high parts, low
+  // parts added), in slice order: no serial fp64 chain (a dependent fp64 operation costs
+  // about 180 cycles on this part).
+  part_h[kk][sl][e] = hi;
+  part_l[kk][sl][e] = lo;
+  __syncthreads();
+  if (sl == 0 && k < K) {
+    float h = part_h[kk][0][e], l = part_l[kk][0][e];
+    for (int s2 = 1; s2 < kSolveSlices; ++s2) {
+      const float p = part_h[kk][s2][e];
+      const float sum = __fadd_rn(h, p);
+      const float bp = __fsub_rn(sum, h);
+      const float t = __fadd_rn(__fsub_rn(h, __fsub_rn(sum, bp)), __fsub_rn(p, bp));
+      h = sum;
+      l = __fadd_rn(l, __fadd_rn(t, part_l[kk][s2][e]));
+    }
+    part_h[kk][0][e] = h;
+    part_l[kk][0][e] = l;
+  }
   __syncthreads();
   if (sl != 0 || e != 0 || k >= K) return;
-  double A[kNA];
-#pragma unroll
-  for (int q = 0; q < kNA; ++q) {
-    double a = part[kk][0][q];
-    for (int s2 = 1; s2 < kSolveSlices; ++s2) a += part[kk][s2][q];
-    A[q] = a;
-  }
-  const int64_t count = (int64_t)A[36];
+  const float* Ah = part_h[kk][0];
+  const float* Al = part_l[kk][0];
+  // the count: an exact integer held by the pair
+  const int64_t count = (int64_t)Ah[36] + (int64_t)Al[36];
   if (counts_out) counts_out[k] = (int32_t)count;
   bool keep = count == 0;
   float out[kD];
   if (!keep) {
-    const double inv_scale = 1.0 / *st.scale;  // a power of two: exact
-    double b[kD], x[kD];
+    const int sexp = stats_scale_exp(*st.scale);
+    float bh[kD], bl[kD];
 #pragma unroll
-    for (int j = 0; j < kD; ++j) b[j] = (double)st.bacc[(int64_t)k * kD + j] * inv_scale;
-    if (solve8_refined(A, b, x)) {
+    for (int j = 0; j < kD; ++j) fixed_to_pair(st.bacc[(int64_t)k * kD + j], sexp, bh[j], bl[j]);
+    if (!solve8_pairs(Ah, Al, bh, bl, out)) {
+      // no fp32 factor (cond(A) beyond fp32): the fp64 Cholesky solve
+      double A[36], b[kD], x[kD];
 #pragma unroll
-      for (int j = 0; j < kD; ++j) out[j] = (float)x[j];
-    } else {
-      raise_error(err, ERRBIT_NUMERIC);
-      keep = true;
+      for (int q = 0; q < 36; ++q) A[q] = (double)Ah[q] + (double)Al[q];
+#pragma unroll
+      for (int j = 0; j < kD; ++j) b[j] = (double)bh[j] + (double)bl[j];
+      if (cholesky_solve8(A, b, x)) {
+#pragma unroll
+        for (int j = 0; j < kD; ++j) out[j] = (float)x[j];
+      } else {
+        raise_error(err, ERRBIT_NUMERIC);
+        keep = true;
+      }
     }
   }
   if (keep)

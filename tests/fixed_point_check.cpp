@@ -1,6 +1,6 @@
-// Host check of crvq::fix_rn (fixed_point.cuh) against the fp64 route it replaces:
-// llrint of the exact product q * 2^e, saturated to the int64 range. Exit status 0 when every
-// case agrees; prints the first disagreements otherwise.
+// Host check of crvq::fix_rn and crvq::fix_rn_small (fixed_point.cuh) against the fp64 route
+// they replace: llrint of the exact product q * 2^e, saturated to the int64 range. Exit
+// status 0 when every case agrees; prints the first disagreements otherwise.
 #define __host__
 #define __device__
 #include <cmath>
@@ -63,6 +63,37 @@ int main() {
     float q;
     std::memcpy(&q, &b, 4);
     check(q, 149 + (int)(rng() % 40) - 20);
+  }
+  // fix_rn_small, the kernels' form: every e whose 2^e is a normal fp32 number and every q
+  // with |q 2^e| < 2^31 (random bit patterns placed in that range, ties and their neighbours)
+  auto check_small = [&](float q, int e) {
+    if (!std::isfinite(q) || e < -126 || e > 127) return;
+    if (std::fabs((double)q * std::ldexp(1.0, e)) >= 2147483648.0) return;
+    ++n;
+    const long long v = crvq::fix_rn_small(q, std::ldexp(1.f, e)), r = reference(q, e);
+    const long long w = crvq::fix_rn(q, e);
+    if (v != r || w != r) {
+      if (bad < 8) std::printf("q=%a e=%d fix_rn_small=%lld reference=%lld\n", q, e, v, r);
+      ++bad;
+    }
+  };
+  for (int it = 0; it < 2000000; ++it) {
+    uint32_t b = (uint32_t)rng();
+    float q;
+    std::memcpy(&q, &b, 4);
+    const int ex = (int)((b >> 23) & 0xff);
+    check_small(q, (150 - ex) + (int)(rng() % 56) - 40);
+  }
+  for (int it = 0; it < 500000; ++it) {
+    const int bits = 1 + (int)(rng() % 23);
+    const long long j = (long long)(rng() % (1ull << bits));
+    const float q0 = (float)((double)j + 0.5);
+    const int e = (int)(rng() % 120) - 60;
+    const float q = std::ldexp(q0, -e);
+    check_small(q, e);
+    check_small(-q, e);
+    check_small(std::nextafter(q, 0.f), e);
+    check_small(std::nextafter(q, 1e30f), e);
   }
   std::printf("cases=%lld disagreements=%lld\n", n, bad);
   return bad != 0;

@@ -1,6 +1,7 @@
-"""fix_rn, the integer float-to-fixed-point conversion of the least-squares statistics, equals
-the fp64 route (llrint of the exact product q * 2^e, saturated) bit for bit: compiled for the
-host with g++ from the same header the kernels include. No GPU needed."""
+"""fix_rn and fix_rn_small, the float-to-fixed-point conversions of the least-squares
+statistics, equal the fp64 route (llrint of the exact product q * 2^e, saturated) bit for bit
+(fix_rn_small in its range: 2^e a normal fp32 number, |q 2^e| < 2^31): compiled for the host
+with g++ from the same header the kernels include. No GPU needed."""
 import os
 import shutil
 import subprocess

@@ -337,7 +337,9 @@ def test_reconstruct_error_parity(c1, shape):
     np.testing.assert_array_equal(host(Wh), Who)
     assert abs(lb - lbo) <= 1e-4 * lbo
     assert abs(lc - lco) <= 1e-4 * lco
-    assert abs(lf - lfo) <= 1e-4 * lfo
+    # the full loss: 3xTF32 products, fp32 accumulation in chunks of 1024 channels summed in
+    # order, fp32 sums of squares per row: a few 1e-6 relative
+    assert abs(lf - lfo) <= 2e-5 * lfo
     # identity order, no X
     Wh2, lb2, _, lf2 = P.crvq_reconstruct_error(dev(Ws), D, dev(Hb), None, cbs, Gc)
     assert lf2 is None
