@@ -2,9 +2,11 @@
 // to the original channel order (Sec. 4.3) and the losses of Alg. 1 (QuantLoss):
 //   loss_block = sum_v (t_v - r_v)^T H_g (t_v - r_v)       (block-diagonal part)
 //   loss_crit  = the same over the critical groups g < G_c
-//   loss_full  = ||dW X^T||^2 / n + delta ||dW||^2 = tr(dW H dW^T)   (dW in original order)
-// Per-row partial sums are fp64 and reduced in a fixed order; the full loss forms dW X^T on the
-// tensor cores (tc_gemm.cuh: tcgen05, 3xTF32, split K) and squares and sums it in fp64.
+//   loss_full  = ||dW X^T||^2 / n + delta ||dW||^2 = tr(dW H dW^T)
+// The reconstruction is formed in the sorted channel order and gathered back to the original
+// order; per-(row, group slice) sums are fp32 pairs, reduced in fp64 in a fixed order. The full
+// loss takes dW and X's columns in the sorted order (a permutation of the channel sum) on the
+// tensor cores (tc_gemm.cu: tf32 operand images, tcgen05 3xTF32).
 #include "common.cuh"
 #include "kernels.h"
 
@@ -65,44 +67,57 @@ __device__ __forceinline__ void pair_merge(float& h, float& l, float oh, float o
   l = __fadd_rn(l, ol);
 }
 
-// One CTA per row (grid-strided): the row of W_hat and of dW = W - W_hat in the original
-// channel order (staged in shared memory, then stored with 16-byte writes), and the row's
-// block loss, critical loss and ||dW||^2. Each vector's terms are fp32 (the quadratic form as
-// two FMA chains); the thread's running sums and the row reduction are fp32 pairs in a fixed
-// order (about 2^-44 relative; a chain of dependent fp64 additions would cost about 180
-// cycles per step on this part), rounded to fp64 once per row.
-__global__ void __launch_bounds__(256)
-decode_row_kernel(const float* __restrict__ Ws, int64_t M, int64_t N, const float* __restrict__ Hb,
-                  const int32_t* __restrict__ perm, CbList cbs, int64_t n_crit_groups,
-                  float* __restrict__ W_hat, float* __restrict__ dW,
-                  double* __restrict__ row_part, unsigned* err) {
-  extern __shared__ __align__(16) float srow[];  // [N] W_hat row (if any), then [N] dW row
-  float* s_hat = srow;
-  float* s_dw = srow + (W_hat ? N : 0);
-  __shared__ float red_h[3][256 / 32], red_l[3][256 / 32];
+constexpr int kDecRows = 4;   // rows per warp: each H block is loaded once for all of them
+constexpr int kDecWarps = 8;  // warps per CTA
+
+// One warp = kDecRows rows x one slice of the groups, lanes across the groups: the
+// reconstruction in the sorted order (32-byte stores, consecutive lanes on consecutive
+// vectors), each vector's error under H_g (the block loaded once for the warp's rows; the
+// quadratic form as two FMA chains in fp32) and, per (row, slice), the block loss, the
+// critical loss and ||dW||^2 as fp32 pairs in a fixed order, rounded to fp64 once:
+// row_part[(row * slices + slice) * 3 + {0, 1, 2}]. No shared memory and no block barrier:
+// the kernel is bound by the latency of its loads, which full occupancy hides.
+__global__ void __launch_bounds__(kDecWarps * 32)
+decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
+                  const float* __restrict__ Hb, CbList cbs, int64_t n_crit_groups, int slices,
+                  float* __restrict__ W_rec, double* __restrict__ row_part, unsigned* err) {
+  const int lane = threadIdx.x & 31;
+  const int64_t wid = (int64_t)blockIdx.x * kDecWarps + (threadIdx.x >> 5);
   const int64_t G = N / kD;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  for (int64_t i = blockIdx.x; i < M; i += gridDim.x) {
-    float lb = 0.f, lbl = 0.f, lc = 0.f, lcl = 0.f, sq = 0.f, sql = 0.f;
-    __syncthreads();  // the previous row's stores have read the staging rows
-    for (int64_t g = threadIdx.x; g < G; g += blockDim.x) {
-      float r[kD], t[kD], dl[kD];
-      recon(cbs, i, g, r, err);
+  const int64_t row_blocks = (M + kDecRows - 1) / kDecRows;
+  if (wid >= row_blocks * slices) return;  // whole warps
+  const int64_t rb = wid / slices;
+  const int sl = (int)(wid % slices);
+  const int64_t gs = (G + slices - 1) / slices;
+  const int64_t g0 = sl * gs, g1 = min(G, g0 + gs);
+  const int64_t i0 = rb * kDecRows;
+  const int nr = (int)min((int64_t)kDecRows, M - i0);
+  float lb[kDecRows], lbl[kDecRows], lc[kDecRows], lcl[kDecRows], sq[kDecRows], sql[kDecRows];
+#pragma unroll
+  for (int r = 0; r < kDecRows; ++r) lb[r] = lbl[r] = lc[r] = lcl[r] = sq[r] = sql[r] = 0.f;
+  for (int64_t g = g0 + lane; g < g1; g += 32) {
+    float4 H4[2 * kD];
+#pragma unroll
+    for (int q = 0; q < 2 * kD; ++q) H4[q] = __ldg(reinterpret_cast<const float4*>(Hb + g * kD * kD) + q);
+#pragma unroll
+    for (int r = 0; r < kDecRows; ++r) {
+      if (r >= nr) break;
+      const int64_t i = i0 + r;
+      float rv[kD], dl[kD];
+      recon(cbs, i, g, rv, err);
       const float4 t0 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD);
       const float4 t1 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD + 4);
-      t[0] = t0.x; t[1] = t0.y; t[2] = t0.z; t[3] = t0.w;
-      t[4] = t1.x; t[5] = t1.y; t[6] = t1.z; t[7] = t1.w;
+      const float t[kD] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w};
       float q2 = 0.f;
 #pragma unroll
       for (int j = 0; j < kD; ++j) {
-        dl[j] = t[j] - r[j];
+        dl[j] = t[j] - rv[j];
         q2 = fmaf(dl[j], dl[j], q2);
       }
-      const float4* H4 = reinterpret_cast<const float4*>(Hb + g * kD * kD);
       float e = 0.f;
 #pragma unroll
       for (int a = 0; a < kD; ++a) {
-        const float4 h0 = __ldg(H4 + 2 * a), h1 = __ldg(H4 + 2 * a + 1);
+        const float4 h0 = H4[2 * a], h1 = H4[2 * a + 1];
         float hb = dl[0] * h0.x;
         hb = fmaf(dl[1], h0.y, hb);
         hb = fmaf(dl[2], h0.z, hb);
@@ -113,61 +128,50 @@ decode_row_kernel(const float* __restrict__ Ws, int64_t M, int64_t N, const floa
         hb = fmaf(dl[7], h1.w, hb);
         e = fmaf(hb, dl[a], e);
       }
-      pair_add(lb, lbl, e);
-      if (g < n_crit_groups) pair_add(lc, lcl, e);
-      pair_add(sq, sql, q2);
+      pair_add(lb[r], lbl[r], e);
+      if (g < n_crit_groups) pair_add(lc[r], lcl[r], e);
+      pair_add(sq[r], sql[r], q2);
+      if (W_rec) {
+        float* o = W_rec + i * N + g * kD;
+        *reinterpret_cast<float4*>(o) = make_float4(rv[0], rv[1], rv[2], rv[3]);
+        *reinterpret_cast<float4*>(o + 4) = make_float4(rv[4], rv[5], rv[6], rv[7]);
+      }
+    }
+  }
 #pragma unroll
-      for (int j = 0; j < kD; ++j) {
-        const int64_t p = g * kD + j;
-        const int64_t col = perm ? perm[p] : p;
-        if (col < 0 || col >= N) {
-          raise_error(err, ERRBIT_INDEX);
-          continue;
-        }
-        if (W_hat) s_hat[col] = r[j];
-        if (dW) s_dw[col] = dl[j];
-      }
-    }
-    __syncthreads();
-    {
-      if (W_hat) {
-        float* dst = W_hat + i * N;
-        for (int64_t c = (int64_t)threadIdx.x * 4; c < N; c += (int64_t)blockDim.x * 4)
-          *reinterpret_cast<float4*>(dst + c) = *reinterpret_cast<const float4*>(s_hat + c);
-      }
-      if (dW) {
-        float* dd = dW + i * N;
-        for (int64_t c = (int64_t)threadIdx.x * 4; c < N; c += (int64_t)blockDim.x * 4)
-          *reinterpret_cast<float4*>(dd + c) = *reinterpret_cast<const float4*>(s_dw + c);
-      }
-    }
+  for (int r = 0; r < kDecRows; ++r) {
 #pragma unroll
     for (int off = 16; off > 0; off >>= 1) {
-      const float a0 = __shfl_xor_sync(0xffffffffu, lb, off);
-      const float a1 = __shfl_xor_sync(0xffffffffu, lbl, off);
-      const float b0 = __shfl_xor_sync(0xffffffffu, lc, off);
-      const float b1 = __shfl_xor_sync(0xffffffffu, lcl, off);
-      const float c0 = __shfl_xor_sync(0xffffffffu, sq, off);
-      const float c1 = __shfl_xor_sync(0xffffffffu, sql, off);
-      pair_merge(lb, lbl, a0, a1);
-      pair_merge(lc, lcl, b0, b1);
-      pair_merge(sq, sql, c0, c1);
+      const float a0 = __shfl_xor_sync(0xffffffffu, lb[r], off);
+      const float a1 = __shfl_xor_sync(0xffffffffu, lbl[r], off);
+      const float b0 = __shfl_xor_sync(0xffffffffu, lc[r], off);
+      const float b1 = __shfl_xor_sync(0xffffffffu, lcl[r], off);
+      const float c0 = __shfl_xor_sync(0xffffffffu, sq[r], off);
+      const float c1 = __shfl_xor_sync(0xffffffffu, sql[r], off);
+      pair_merge(lb[r], lbl[r], a0, a1);
+      pair_merge(lc[r], lcl[r], b0, b1);
+      pair_merge(sq[r], sql[r], c0, c1);
     }
-    if (lane == 0) {
-      red_h[0][warp] = lb;
-      red_l[0][warp] = lbl;
-      red_h[1][warp] = lc;
-      red_l[1][warp] = lcl;
-      red_h[2][warp] = sq;
-      red_l[2][warp] = sql;
+    if (lane == 0 && r < nr) {
+      double* o = row_part + ((i0 + r) * slices + sl) * 3;
+      o[0] = (double)lb[r] + (double)lbl[r];
+      o[1] = (double)lc[r] + (double)lcl[r];
+      o[2] = (double)sq[r] + (double)sql[r];
     }
-    __syncthreads();
-    if (threadIdx.x < 3) {
-      const int q = threadIdx.x;
-      float h = red_h[q][0], l = red_l[q][0];
-      for (int w = 1; w < (int)(blockDim.x >> 5); ++w) pair_merge(h, l, red_h[q][w], red_l[q][w]);
-      row_part[i * 3 + q] = (double)h + (double)l;
+  }
+}
+
+// inv[perm[p]] = p; entries outside [0, N) are reported and skipped.
+__global__ void invert_perm_kernel(const int32_t* __restrict__ perm, int64_t N,
+                                   int32_t* __restrict__ inv, unsigned* err) {
+  for (int64_t p = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; p < N;
+       p += (int64_t)gridDim.x * blockDim.x) {
+    const int32_t c = perm[p];
+    if (c < 0 || c >= N) {
+      raise_error(err, ERRBIT_INDEX);
+      continue;
     }
+    inv[c] = (int32_t)p;
   }
 }
 
@@ -217,38 +221,54 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   unsigned* err = nullptr;
   CRVQ_TRY(device_error_word(&err));
   const int nsm = sm_count();
+  const int64_t G = N / kD;
+  // warps: kDecRows rows x a slice of the groups; enough slices for ~16 warps per SM
+  const int64_t row_blocks = ceil_div(M, (int64_t)kDecRows);
+  const int slices = (int)std::max<int64_t>(
+      1, std::min<int64_t>(ceil_div(16 * (int64_t)nsm * kDecWarps, row_blocks),
+                           ceil_div(G, (int64_t)32)));
   // partial sums of the full loss: one per 128 x 256 tile of dW X^T
   const int64_t n_gemm_cap = X ? ceil_div(M, (int64_t)128) * ceil_div(n_tok, (int64_t)256) : 0;
   int64_t n_gemm = 0;
-  // Scratch: dW (16-byte aligned for the 128-bit stores), then the fp64 partial sums.
-  const size_t dW_bytes = X ? align_up((size_t)M * N * sizeof(float), 256) : 0;
-  const size_t part_bytes = (size_t)M * 3 * sizeof(double) + (size_t)(n_gemm_cap + 1) * sizeof(double);
+  // Scratch: the reconstruction in the sorted order when it is not W_hat itself, the inverse
+  // order, and the fp64 partial sums.
+  const bool need_rec = W_hat || X;
+  const bool rec_is_out = W_hat && !perm;
+  const size_t rec_bytes = (need_rec && !rec_is_out) ? align_up((size_t)M * N * 4, 256) : 0;
+  const size_t inv_bytes = (W_hat && perm) ? align_up((size_t)N * 4, 256) : 0;
+  const size_t part_bytes = (size_t)M * slices * 3 * sizeof(double) +
+                            (size_t)(n_gemm_cap + 1) * sizeof(double);
   Scratch mem;
-  CRVQ_TRY(mem.alloc(dW_bytes + part_bytes, stream));
-  float* dW = X ? mem.as<float>() : nullptr;
-  double* row_part = reinterpret_cast<double*>(mem.as<char>() + dW_bytes);
-  double* gemm_part = row_part + M * 3;
-  const size_t smem = (size_t)N * sizeof(float) * ((W_hat ? 1 : 0) + (dW ? 1 : 0));
-  if (smem > (size_t)227 * 1024)
-    return fail(CRVQ_ERR_UNSUPPORTED,
-                "crvq_reconstruct_error: N = %lld channels need %zu bytes of shared memory per "
-                "row (227 KB available)", (long long)N, smem);
-  if (smem > 48 * 1024)
-    CRVQ_CUDA(cudaFuncSetAttribute(decode_row_kernel,
-                                   cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-  const int blocks = (int)std::min<int64_t>(M, (int64_t)8 * nsm);
+  CRVQ_TRY(mem.alloc(rec_bytes + inv_bytes + part_bytes, stream));
+  float* W_rec = rec_is_out ? W_hat : (need_rec ? mem.as<float>() : nullptr);
+  int32_t* inv = inv_bytes ? reinterpret_cast<int32_t*>(mem.as<char>() + rec_bytes) : nullptr;
+  double* row_part = reinterpret_cast<double*>(mem.as<char>() + rec_bytes + inv_bytes);
+  double* gemm_part = row_part + M * slices * 3;
   {
-  ProfScope ps("decode_rows", stream,
-               (double)M * N * 4.0 * (1.0 + (W_hat ? 1.0 : 0.0) + (X ? 1.0 : 0.0)));
-  decode_row_kernel<<<blocks, 256, smem, stream>>>(W_sorted, M, N, Hb, perm, cbs,
-                                                   n_crit_groups, W_hat, dW, row_part, err);
-  CRVQ_LAUNCHED();
+    ProfScope ps("decode_rows", stream,
+                 (double)M * N * 4.0 * (1.0 + (W_rec ? 1.0 : 0.0)));
+    const int64_t warps = row_blocks * slices;
+    decode_vec_kernel<<<(unsigned)ceil_div(warps, (int64_t)kDecWarps), kDecWarps * 32, 0,
+                        stream>>>(W_sorted, M, N, Hb, cbs, n_crit_groups, slices, W_rec,
+                                  row_part, err);
+    CRVQ_LAUNCHED();
+  }
+  if (W_hat && perm) {  // back to the original channel order: W_hat[:, c] = W_rec[:, inv[c]]
+    ProfScope ps("decode_unpermute", stream, (double)M * N * 8.0);
+    invert_perm_kernel<<<(unsigned)std::min<int64_t>(ceil_div(N, 256), 4 * nsm), 256, 0,
+                         stream>>>(perm, N, inv, err);
+    CRVQ_LAUNCHED();
+    CRVQ_TRY(launch_gather_cols(W_rec, M, N, inv, W_hat, stream));
   }
   if (X) {
-    CRVQ_TRY(launch_tc_sumsq(dW, M, X, n_tok, N, gemm_part, n_gemm_cap, &n_gemm, stream));
+    // ||dW X^T||^2 with dW and X's columns both in the sorted order (the same sum over the
+    // channels, in another order)
+    CRVQ_TRY(launch_tc_sumsq(W_sorted, W_rec, M, X, perm, n_tok, N, gemm_part, n_gemm_cap,
+                             &n_gemm, stream));
   }
-  finalize_losses_kernel<<<1, 1024, 0, stream>>>(row_part, M, X ? gemm_part : nullptr, n_gemm,
-                                                n_tok, damp_delta, delta_dev, losses_dev);
+  finalize_losses_kernel<<<1, 1024, 0, stream>>>(row_part, M * slices, X ? gemm_part : nullptr,
+                                                 n_gemm, n_tok, damp_delta, delta_dev,
+                                                 losses_dev);
   CRVQ_LAUNCHED();
   return CRVQ_OK;
 }

@@ -37,10 +37,15 @@ crvq_status launch_tc_hessian_blocks(const float* Xt, int64_t ldt, int64_t n, in
                                      const int32_t* perm, bool delta_known, float damp_rel,
                                      float* xsq, float* delta, double* delta64, float* Hb,
                                      cudaStream_t stream);
-// Partial sums of ||A B^T||_F^2 (A M x K, B Nb x K row-major) into part[0 .. *nparts).
-crvq_status launch_tc_sumsq(const float* A, int64_t M, const float* B, int64_t Nb, int64_t K,
-                            double* part, int64_t part_cap, int64_t* nparts,
-                            cudaStream_t stream);
+// dst[i][p] = src[i][idx[p]] for every row (M x N row-major; idx a permutation of 0..N-1,
+// entries outside [0, N) reported and read as 0).
+crvq_status launch_gather_cols(const float* src, int64_t M, int64_t N, const int32_t* idx,
+                               float* dst, cudaStream_t stream);
+// Partial sums of ||(A - A_sub) B'^T||_F^2 into part[0 .. *nparts): A, A_sub (optional) M x K,
+// B Nb x K row-major, B' = B with its columns taken in the order B_cols (optional).
+crvq_status launch_tc_sumsq(const float* A, const float* A_sub, int64_t M, const float* B,
+                            const int32_t* B_cols, int64_t Nb, int64_t K, double* part,
+                            int64_t part_cap, int64_t* nparts, cudaStream_t stream);
 
 crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
                                   const float* W_pre, const float* xsq, const float* H,

@@ -160,15 +160,25 @@ crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
     rank_kernel<<<(unsigned)ceil_div(N, 256), 256, 0, stream>>>(I, N, perm);
     CRVQ_LAUNCHED();
   }
+  {
+    ProfScope ps("reorder_gather", stream, (double)M * N * 8.0);
+    CRVQ_TRY(launch_gather_cols(W, M, N, perm, W_sorted, stream));
+  }
+  if (H_blocks) CRVQ_TRY(launch_extract_blocks(H, N, d, perm, H_blocks, stream));
+  return CRVQ_OK;
+}
+
+crvq_status launch_gather_cols(const float* src, int64_t M, int64_t N, const int32_t* idx,
+                               float* dst, cudaStream_t stream) {
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
   const size_t smem = (size_t)N * sizeof(float);
   if (smem > 48 * 1024)
     CRVQ_CUDA(cudaFuncSetAttribute(gather_cols_kernel,
                                    cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-  const int blocks = (int)std::min<int64_t>(M, (int64_t)8 * nsm);
-  ProfScope ps("reorder_gather", stream, (double)M * N * 8.0);
-  gather_cols_kernel<<<blocks, 256, smem, stream>>>(W, M, N, perm, W_sorted, err);
+  const int blocks = (int)std::min<int64_t>(M, (int64_t)8 * sm_count());
+  gather_cols_kernel<<<blocks, 256, smem, stream>>>(src, M, N, idx, dst, err);
   CRVQ_LAUNCHED();
-  if (H_blocks) CRVQ_TRY(launch_extract_blocks(H, N, d, perm, H_blocks, stream));
   return CRVQ_OK;
 }
 

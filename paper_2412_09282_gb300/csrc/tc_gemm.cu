@@ -127,9 +127,12 @@ __host__ __device__ inline int64_t img_off(int64_t r, int64_t k, int64_t nslab) 
 }
 
 // One warp = 8 rows x one 16-column slab: reads 8 x 64 B, writes 512 contiguous bytes per
-// image. Rows >= rows and columns >= K are written as zeros (the padding of the images).
+// image. Element (r, k) is src[r][k] - sub[r][k] (sub optional, same layout), or
+// src[r][cols[k]] with a column order (entries outside [0, K) read as 0; the caller checks
+// the order). Rows >= rows and columns >= K are written as zeros (the images' padding).
 __global__ void __launch_bounds__(256)
-image_kernel(const float* __restrict__ src, int64_t rows, int64_t K, int64_t ld,
+image_kernel(const float* __restrict__ src, const float* __restrict__ sub,
+             const int32_t* __restrict__ cols, int64_t rows, int64_t K, int64_t ld,
              int64_t rows_pad, int64_t nslab, char* __restrict__ hi, char* __restrict__ lo) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t r = (int64_t)blockIdx.x * 8 + (lane & 7);
@@ -138,13 +141,25 @@ image_kernel(const float* __restrict__ src, int64_t rows, int64_t K, int64_t ld,
   const int64_t k = sl * kSlabK + (lane >> 3) * 4;
   float v[4] = {0.f, 0.f, 0.f, 0.f};
   if (r < rows) {
-    const float* p = src + r * ld + k;
-    if (k + 4 <= K && (ld & 3) == 0 && ((uintptr_t)src & 15) == 0) {
-      const float4 x = __ldg(reinterpret_cast<const float4*>(p));
+    const float* p = src + r * ld;
+    if (cols) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int32_t c = (k + j < K) ? cols[k + j] : -1;
+        v[j] = (c >= 0 && c < K) ? p[c] : 0.f;
+      }
+    } else if (k + 4 <= K && (ld & 3) == 0 && ((uintptr_t)src & 15) == 0 &&
+               (!sub || ((uintptr_t)sub & 15) == 0)) {
+      const float4 x = __ldg(reinterpret_cast<const float4*>(p + k));
       v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+      if (sub) {
+        const float4 y = __ldg(reinterpret_cast<const float4*>(sub + r * ld + k));
+        v[0] -= y.x; v[1] -= y.y; v[2] -= y.z; v[3] -= y.w;
+      }
     } else {
 #pragma unroll
-      for (int j = 0; j < 4; ++j) v[j] = (k + j < K) ? p[j] : 0.f;
+      for (int j = 0; j < 4; ++j)
+        v[j] = (k + j < K) ? (sub ? p[k + j] - sub[r * ld + k + j] : p[k + j]) : 0.f;
     }
   }
   uint32_t h[4], l[4];
@@ -365,12 +380,13 @@ crvq_status launch_tc_syrk(const float* X, int64_t n, int64_t N, float* S, cudaS
   return CRVQ_OK;
 }
 
-// part[0 .. nparts) = partial sums of ||A B^T||_F^2 with A: M x K, B: Nb x K (row-major,
-// leading dimension K), one per 128 x 256 tile; part_cap must hold ceil(M / 128) *
-// ceil(Nb / 256) values. Returns the number of partials written.
-crvq_status launch_tc_sumsq(const float* A, int64_t M, const float* B, int64_t Nb, int64_t K,
-                            double* part, int64_t part_cap, int64_t* nparts,
-                            cudaStream_t stream) {
+// part[0 .. nparts) = partial sums of ||(A - A_sub) B'^T||_F^2 with A, A_sub: M x K, B: Nb x K
+// (row-major, leading dimension K; B' = B with columns in the order B_cols when given), one
+// per 128 x 256 tile; part_cap must hold ceil(M / 128) * ceil(Nb / 256) values. Returns the
+// number of partials written.
+crvq_status launch_tc_sumsq(const float* A, const float* A_sub, int64_t M, const float* B,
+                            const int32_t* B_cols, int64_t Nb, int64_t K, double* part,
+                            int64_t part_cap, int64_t* nparts, cudaStream_t stream) {
   unsigned* err = nullptr;
   CRVQ_TRY(device_error_word(&err));
   static bool attr_set[64] = {};
@@ -401,10 +417,10 @@ crvq_status launch_tc_sumsq(const float* A, int64_t M, const float* B, int64_t N
   {
     ProfScope ps("loss_images", stream, 12.0 * (double)(M + Nb) * K);
     img::image_kernel<<<dim3((unsigned)(am / 8), (unsigned)ceil_div(nslab, 8)), 256, 0,
-                        stream>>>(A, M, K, K, am, nslab, a_hi, a_lo);
+                        stream>>>(A, A_sub, nullptr, M, K, K, am, nslab, a_hi, a_lo);
     CRVQ_LAUNCHED();
     img::image_kernel<<<dim3((unsigned)(bm / 8), (unsigned)ceil_div(nslab, 8)), 256, 0,
-                        stream>>>(B, Nb, K, K, bm, nslab, b_hi, b_lo);
+                        stream>>>(B, nullptr, B_cols, Nb, K, K, bm, nslab, b_hi, b_lo);
     CRVQ_LAUNCHED();
   }
   img::SumsqArgs g{a_hi, a_lo, b_hi, b_lo, nslab, (int)tiles_n, part, err};
