@@ -421,24 +421,53 @@ __device__ __forceinline__ bool less(float ah, float al, int ak, float bh, float
 
 }  // namespace dfl
 
-// Arg-min over one codebook on the tensor cores. A 128-thread CTA walks `tiles` consecutive
-// row tiles of one group (thread = row = tensor-memory lane), with a 128-column accumulator;
-// three CTAs per SM, whose phases (A rows, MMA, epilogue, certificate) interleave on the SM.
-// Codeword chunks of 128 come from precomputed B images by bulk copy (bpre) or are built in
-// place; with at most two chunks they stay resident for all the CTA's tiles. Keys carry the
-// column within a 32-column block in their low 5 bits (2^-18 relative truncation); the block
-// is tracked by the merge. Rows the bounds do not certify go to the flag list (decided exactly
-// by argmin_exact_kernel). The Lloyd statistics of certified rows are summed in shared memory
-// (integer atomics, [component][code] so that a warp's lanes hit spread banks) and flushed
-// once.
+// Arg-min over one codebook on the tensor cores. A CTA walks `tiles` consecutive row tiles of
+// one group (thread = row = tensor-memory lane) with a 128-column accumulator per tile in
+// flight. HALVES = 1: 128 threads, three CTAs per SM, any codebook size (codeword chunks of 128
+// come from the precomputed B images by bulk copy; with at most two chunks they stay resident
+// for all the CTA's tiles). HALVES = 2 (codebooks of at most 256 codewords): 256 threads in two
+// halves of 128 that run independently (each its own tiles, named barriers, MMA issue and
+// accumulator) and share the resident codebook operand and the statistics; two CTAs per SM,
+// so four tile pipelines per SM interleave their phases (A rows, MMA, epilogue, certificate).
+// Keys carry the column within a 32-column block in their low 5 bits (2^-18 relative
+// truncation); the block is tracked by the merge. Rows the bounds do not certify go to the flag
+// list (decided exactly by the exact kernels). The Lloyd statistics of certified rows are summed
+// in shared memory (integer atomics, [component][code] so that a warp's lanes hit spread banks)
+// and flushed once.
 constexpr int kTcSmemStatsK = 256;  // codebooks up to this size aggregate statistics in smem
 
-// dynamic shared memory of argmin_tc_kernel: A tile, two B chunks, statistics, H r, alignment
-constexpr size_t kArgminSmem = (size_t)tcenc::kATile + 2 * (size_t)kTcBTile +
-                               (size_t)kTcSmemStatsK * (kD * 8 + 4) + tcenc::kRows * kD * 4 +
-                               1024;
+// dynamic shared memory of argmin_tc_kernel<HALVES>: A tiles, two B chunks, statistics, H r,
+// alignment
+constexpr size_t argmin_smem(int halves) {
+  return (size_t)halves * tcenc::kATile + 2 * (size_t)kTcBTile +
+         (size_t)kTcSmemStatsK * (kD * 8 + 4) + (size_t)halves * tcenc::kRows * kD * 4 + 1024;
+}
 
-__global__ void __launch_bounds__(128, 3)
+// Barrier over this half's 128 threads (named barrier 1 + half), or the whole CTA.
+template <int HALVES>
+__device__ __forceinline__ void half_sync(int half) {
+  if (HALVES == 1) {
+    __syncthreads();
+  } else {
+    asm volatile("bar.sync %0, 128;" ::"r"(1 + half) : "memory");
+  }
+}
+
+template <int HALVES>
+__device__ __forceinline__ bool half_sync_and(int half, bool v) {
+  if (HALVES == 1) return __syncthreads_and(v);
+  int r;
+  asm volatile(
+      "{\n .reg .pred p, q;\n setp.ne.b32 q, %1, 0;\n bar.red.and.pred p, %2, 128, q;\n"
+      " selp.s32 %0, 1, 0, p;\n}\n"
+      : "=r"(r)
+      : "r"((int)v), "r"(1 + half)
+      : "memory");
+  return r != 0;
+}
+
+template <int HALVES>
+__global__ void __launch_bounds__(128 * HALVES, HALVES == 1 ? 3 : 2)
 argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
                  int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
                  FlagList flags, StatsView st, const float* __restrict__ cbmax,
@@ -448,18 +477,21 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   extern __shared__ __align__(1024) char smem_raw[];
   // 1024-byte aligned base, derived from the shared array (keeps the shared address space)
   char* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
-  char* Atile = smem;                  // 16 KB
-  char* Bbuf = smem + kATile;          // 2 x 16 KB
+  char* Atiles = smem;                          // HALVES x 16 KB
+  char* Bbuf = smem + HALVES * kATile;          // 2 x 16 KB
   long long* s_bacc = reinterpret_cast<long long*>(Bbuf + 2 * kTcBTile);  // [8][256]
   int* s_cnt = reinterpret_cast<int*>(s_bacc + kTcSmemStatsK * kD);       // [256]
-  float* sQ = reinterpret_cast<float*>(s_cnt + kTcSmemStatsK);            // [128][8] H r
+  float* sQ = reinterpret_cast<float*>(s_cnt + kTcSmemStatsK);            // [128 HALVES][8]
   __shared__ float sH[kD * kD];
-  __shared__ __align__(8) uint64_t bar_mma, bar_b[2];
+  __shared__ __align__(8) uint64_t bar_mma_s[HALVES], bar_b[2];
   __shared__ uint32_t tmem_slot;
 
   const int64_t g = g_begin + blockIdx.y;
   const int64_t G_range = gridDim.y;
   const int tid = threadIdx.x, warp = tid >> 5;
+  const int half = HALVES == 1 ? 0 : (tid >> 7), rrow = tid & (kRows - 1);
+  char* Atile = Atiles + half * kATile;
+  uint64_t& bar_mma = bar_mma_s[half];
   const CbView cw = cbs.cb[s_idx];
   const float cmul = kCmul + 4.f * n_fixed;
   const float uc = kU * cmul;
@@ -474,9 +506,9 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
     for (int e = tid; e < kTcSmemStatsK * kD; e += blockDim.x) s_bacc[e] = 0;
     for (int e = tid; e < kTcSmemStatsK; e += blockDim.x) s_cnt[e] = 0;
   }
-  if (warp == 0) tc::tmem_alloc(&tmem_slot, kTcCols);
+  if (warp == 0) tc::tmem_alloc(&tmem_slot, HALVES * kTcCols);
   if (tid == 0) {
-    tc::mbar_init(tc::smem_u32(&bar_mma), 1);
+    for (int h = 0; h < HALVES; ++h) tc::mbar_init(tc::smem_u32(&bar_mma_s[h]), 1);
     tc::mbar_init(tc::smem_u32(&bar_b[0]), 1);
     tc::mbar_init(tc::smem_u32(&bar_b[1]), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -484,7 +516,8 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   tc::tc_fence_before();
   __syncthreads();
   tc::tc_fence_after();
-  const uint32_t tmem = tmem_slot;
+  // this half's accumulator: columns [128 half, 128 half + 128)
+  const uint32_t tmem = tmem_slot + (uint32_t)(half * kTcCols);
   const float sscale = st.cnt ? stats_scale_f(st) : 1.f;
 
   // Bound on Na_k over the codebook for this group: (max row sum |H_g|) L1max cinfmax.
@@ -499,13 +532,15 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   const float l1max = cbmax[0], cinf = cbmax[1];
   constexpr uint32_t idesc = tc::idesc_tf32(kRows, kTcCols);
 
-  // this CTA's row tiles (the last CTA of a column may have fewer)
+  // this CTA's row tiles (the last CTA of a column may have fewer); with two halves, half h
+  // takes tiles h, h + 2, ...
   const int64_t row_tiles = (set.M + kRows - 1) / kRows;
   const int my_tiles = (int)min((int64_t)tiles, row_tiles - (int64_t)blockIdx.x * tiles);
+  const int steps = (my_tiles + HALVES - 1) / HALVES;
   // Chunk uses are numbered u = t * nchunk + c. Resident chunks sit in buffer c; otherwise use u
-  // reads buffer u & 1, and the copy for use u + 2 starts when use u is done. At most one copy
-  // per buffer is outstanding; every thread tracks the same state.
-  const int n_uses = resident ? nchunk : my_tiles * nchunk;
+  // reads buffer u & 1, and the copy for use u + 2 starts when use u is done (one half only).
+  // At most one copy per buffer is outstanding; every thread tracks the same state.
+  const int n_uses = resident ? nchunk : steps * nchunk;
   // per buffer (bit b): a copy outstanding, and the parity of its wait (registers, not arrays)
   uint32_t b_pend = 0, b_par = 0;
   auto fetch = [&](int u) {  // chunk u % nchunk into buffer u & 1 (bimg only)
@@ -525,13 +560,15 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   bool ok = true;
   int mma_count = 0;
 
-  for (int t = 0; t < my_tiles && ok; ++t) {
-    const int64_t i = ((int64_t)blockIdx.x * tiles + t) * kRows + tid;
+  for (int t = 0; t < steps && ok; ++t) {
+    const int my_tile = HALVES * t + half;  // past my_tiles: a half without rows this step
+    const int64_t i = ((int64_t)blockIdx.x * tiles + my_tile) * kRows + rrow;
+    const bool row_ok = my_tile < my_tiles && i < set.M;
     // Prologue: this thread's A row.
     float pmax, off;
     {
       float rv[kD], a[kD], m2q[kD];
-      if (i < set.M) {
+      if (row_ok) {
         target32(set, cbs, n_fixed, i, g, rv, a, err);
       } else {
 #pragma unroll
@@ -573,10 +610,10 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       row[27] = row[26];
       split(off * (1.f - uc), row[29], row[30]);
       row[31] = 0u;
-      put_row(Atile, tid, row);
+      put_row(Atile, rrow, row);
     }
     tc::fence_async_smem();
-    __syncthreads();
+    half_sync<HALVES>(half);
 
     uint32_t g1 = 0xffffffffu, g2 = 0xffffffffu;
     int gidx = 0;
@@ -590,16 +627,16 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
           b_par ^= 1u << buf;
           b_pend &= ~(1u << buf);
         }
-      } else if (!resident || t == 0) {
+      } else if (!resident || t == 0) {  // (one half only: the host passes B images with two)
         uint32_t v[kK];
-        build_b_row(cw.C, cw.K, c * kTcCols + tid, sH, uc, v);
-        put_row(Bt, tid, v);
+        build_b_row(cw.C, cw.K, c * kTcCols + rrow, sH, uc, v);
+        put_row(Bt, rrow, v);
         tc::fence_async_smem();
-        __syncthreads();
+        half_sync<HALVES>(half);
       }
-      ok = __syncthreads_and(ok);
+      ok = half_sync_and<HALVES>(half, ok);
       if (!ok) break;
-      if (tid == 0) {
+      if (rrow == 0) {
         tc::tc_fence_after();
         const uint32_t a0 = tc::smem_u32(Atile), b0 = tc::smem_u32(Bt);
 #pragma unroll
@@ -611,7 +648,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       }
       ok = tc::mbar_wait(tc::smem_u32(&bar_mma), (uint32_t)(mma_count & 1), err);
       ++mma_count;
-      ok = __syncthreads_and(ok);
+      ok = half_sync_and<HALVES>(half, ok);
       if (!ok) break;
       if (bimg && !resident && u + 2 < n_uses) fetch(u + 2);  // this buffer is free again
       tc::tc_fence_after();
@@ -623,7 +660,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
         a1[b] = 0xffffffffu;
         a2[b] = 0xffffffffu;
       }
-      const uint32_t base = tmem + ((uint32_t)(warp * 32) << 16);
+      const uint32_t base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
 #pragma unroll
       for (int rnd = 0; rnd < 2; ++rnd) {
         uint32_t v[64];
@@ -652,12 +689,12 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
         }
       }
       tc::tc_fence_before();
-      __syncthreads();  // the accumulator is free for the next MMA
+      half_sync<HALVES>(half);  // the accumulator is free for the next MMA
     }
     if (!ok) break;
 
     // Certificate, code, flag and statistics of this thread's row.
-    if (i < set.M) {
+    if (row_ok) {
       int j = gidx;
       const float k1 = __uint_as_float(g1), k2 = __uint_as_float(g2);
       bool cert = false;
@@ -731,7 +768,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   }
   tc::tc_fence_before();
   __syncthreads();
-  if (warp == 0) tc::tmem_dealloc(tmem, kTcCols);
+  if (warp == 0) tc::tmem_dealloc(tmem_slot, HALVES * kTcCols);
 }
 
 // Exact decision for the rows the arg-min pass flagged: one CTA per flagged vector. The
@@ -1017,6 +1054,58 @@ __device__ __forceinline__ void hyp_terms(const double r64[kD], const float* H, 
   }
 }
 
+// fp32-pair residual of a hypothesis before stage s: (rh + rl) = (th + tl) - sum_{s' < s}
+// C_{st[s']}[code] (TwoSum per subtraction, about 2^-48 relative; no fp64 arithmetic).
+__device__ __forceinline__ void hyp_residual_pair(const float th[kD], const float tl[kD],
+                                                  const CbList& cbs, const StageDesc& sd,
+                                                  const int32_t* codes, float rh[kD],
+                                                  float rl[kD], unsigned* err) {
+#pragma unroll
+  for (int j = 0; j < kD; ++j) {
+    rh[j] = th[j];
+    rl[j] = tl[j];
+  }
+  for (int q = 0; q < sd.s; ++q) {
+    const CbView& cb = cbs.cb[sd.st[q]];
+    const int32_t k = codes[q];
+    if (!code_ok(k, cb.K, err)) continue;
+    float c[kD];
+    load_vec(cb.C + (int64_t)k * kD, c);
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      float sj, ej;
+      dfl::two_sum(rh[j], -c[j], sj, ej);
+      rh[j] = sj;
+      rl[j] = __fadd_rn(rl[j], ej);
+    }
+  }
+}
+
+// hyp_terms of a pair residual, rounded once to fp32.
+__device__ __forceinline__ void hyp_terms_pair(const float rh[kD], const float rl[kD],
+                                               const float* H, float m2q[kD], float& rr,
+                                               float& ra, float& pmax) {
+  float r[kD];
+#pragma unroll
+  for (int j = 0; j < kD; ++j) r[j] = __fadd_rn(rh[j], rl[j]);
+  rr = 0.f;
+  ra = 0.f;
+  pmax = 0.f;
+#pragma unroll
+  for (int p = 0; p < kD; ++p) {
+    float q = 0.f, pa = 0.f;
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      q = fmaf(H[p * kD + j], r[j], q);
+      pa = fmaf(fabsf(H[p * kD + j]), fabsf(r[j]), pa);
+    }
+    m2q[p] = -2.f * q;
+    rr = fmaf(r[p], q, rr);
+    ra = fmaf(fabsf(r[p]), pa, ra);
+    pmax = fmaxf(pmax, pa);
+  }
+}
+
 // Fast stage: one thread per vector, the stage codebook chunked through shared memory, a
 // sorted top-L list (L >= Bs + 1) of lower bounds low = approx_err - Et in registers.
 template <int L>
@@ -1038,12 +1127,12 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
   const int S = sd.S, B = sd.B, Bs = sd.Bs;
   const float cmul = bound_mult(n_fixed + sd.s);
   const int Bh = (sd.s == 0) ? 1 : (live ? bb.n_in[vi] : 1);
-  double tgt[kD];
+  float th[kD], tl[kD];  // target as an fp32 pair (t - the fixed codebooks' codewords)
   if (live) {
-    target64(set, cbs, n_fixed, i, g, tgt, err);
+    dfl::target(set, cbs, n_fixed, i, g, th, tl, err);
   } else {
 #pragma unroll
-    for (int j = 0; j < kD; ++j) tgt[j] = 0.0;
+    for (int j = 0; j < kD; ++j) th[j] = tl[j] = 0.f;
   }
 
   float topv[L];
@@ -1062,11 +1151,11 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
     __syncthreads();
     if (!live) continue;
     for (int h = 0; h < Bh; ++h) {
-      double r64[kD];
+      float rh[kD], rl[kD];
       const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
-      hyp_residual64(tgt, cbs, sd, pc, r64, err);
+      hyp_residual_pair(th, tl, cbs, sd, pc, rh, rl, err);
       float m2q[kD], rr, ra, pmax;
-      hyp_terms(r64, sH, m2q, rr, ra, pmax);
+      hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
       const float base = rr - kU * cmul * ra;
       const float nbeta = -2.f * kU * cmul * pmax;
       for (int k = 0; k < nk; ++k) {
@@ -1118,11 +1207,11 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
   for (int j = 0; j < L; ++j) {
     et[j] = 0.f;
     if (j < nkept) {
-      double r64[kD];
+      float rh[kD], rl[kD];
       const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
-      hyp_residual64(tgt, cbs, sd, pc, r64, err);
+      hyp_residual_pair(th, tl, cbs, sd, pc, rh, rl, err);
       float m2q[kD], rr, ra, pmax;
-      hyp_terms(r64, sH, m2q, rr, ra, pmax);
+      hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
       float c[kD], n, na, l1;
       load_vec(cw.C + (int64_t)topk[j] * kD, c);
       codeword_terms(c, sH, n, na, l1);
@@ -1139,17 +1228,20 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
 
   int32_t* out = bb.hyp_out + vi * B * S;
   if (!ok) {
-    // Exact path on the listed candidates: fp64 errs, exact (err, h, k) order; then every
-    // unlisted candidate must have low >= the last listed low > the keep-th exact err.
-    double ev[L];
+    // Exact path on the listed candidates: errs as fp32 pairs (about 2^-44 relative; no fp64),
+    // (err, h, k) order; then every unlisted candidate must have low >= the last listed low,
+    // which must exceed an upper bound of the keep-th err.
+    float evh[L], evl[L];
 #pragma unroll
     for (int j = 0; j < L; ++j) {
-      ev[j] = INFINITY;
+      evh[j] = INFINITY;
+      evl[j] = 0.f;
       if (j < nkept) {
-        double r64[kD];
+        float rh[kD], rl[kD], c[kD];
         const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
-        hyp_residual64(tgt, cbs, sd, pc, r64, err);
-        ev[j] = quad_err64(r64, cw.C + (int64_t)topk[j] * kD, sH);
+        hyp_residual_pair(th, tl, cbs, sd, pc, rh, rl, err);
+        load_vec(cw.C + (int64_t)topk[j] * kD, c);
+        dfl::quad_err(rh, rl, c, sH, evh[j], evl[j]);
       }
     }
     const float last_low = topv[nkept - 1];
@@ -1157,24 +1249,31 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
     for (int a = 1; a < L; ++a) {
 #pragma unroll
       for (int b = a; b > 0; --b) {
-        const bool sw = (ev[b] < ev[b - 1]) ||
-                        (ev[b] == ev[b - 1] &&
-                         (toph[b] < toph[b - 1] ||
-                          (toph[b] == toph[b - 1] && topk[b] < topk[b - 1])));
+        const bool sw = (evh[b] < evh[b - 1]) ||
+                        (evh[b] == evh[b - 1] &&
+                         (evl[b] < evl[b - 1] ||
+                          (evl[b] == evl[b - 1] &&
+                           (toph[b] < toph[b - 1] ||
+                            (toph[b] == toph[b - 1] && topk[b] < topk[b - 1])))));
         if (sw) {
-          const double te = ev[b]; ev[b] = ev[b - 1]; ev[b - 1] = te;
-          const int th = toph[b]; toph[b] = toph[b - 1]; toph[b - 1] = th;
+          const float t0 = evh[b]; evh[b] = evh[b - 1]; evh[b - 1] = t0;
+          const float t1 = evl[b]; evl[b] = evl[b - 1]; evl[b - 1] = t1;
+          const int th_ = toph[b]; toph[b] = toph[b - 1]; toph[b - 1] = th_;
           const int tk = topk[b]; topk[b] = topk[b - 1]; topk[b - 1] = tk;
         }
       }
     }
-    const bool cert = total <= L || (double)last_low > ev[keep - 1];
+    // upper bound of the keep-th listed err (the pair's own error is far below 1e-7)
+    const float ev_up = isfinite(evh[keep - 1])
+                            ? __fmul_ru(__fadd_ru(evh[keep - 1], evl[keep - 1]), 1.0000002f)
+                            : INFINITY;
+    const bool cert = total <= L || last_low > ev_up;
     if (!cert) {
       const unsigned slot = atomicAdd(flags.count, 1u);
       if (slot < flags.cap) {
         flags.vec[slot] = vi;
-        // every member of the exact top-keep has err <= the keep-th listed exact err
-        flags.thr[slot] = isfinite(ev[keep - 1]) ? __double2float_ru(ev[keep - 1]) : INFINITY;
+        // every member of the exact top-keep has err <= the keep-th listed err
+        flags.thr[slot] = ev_up;
       } else {
         raise_error(err, ERRBIT_INDEX);
       }
@@ -1558,7 +1657,10 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     fl.thr = reinterpret_cast<float*>(fl.vec + fl.cap);
     fl.total = ex.flag_total;
     const float uc = kU * (tcenc::kCmul + 4.f * n_fixed);
-    CRVQ_TRY(set_smem_attr(argmin_tc_kernel, kArgminSmem));
+    // two independent 128-thread halves per CTA when the codebook stays resident (K <= 256)
+    const bool two_halves = nchunk <= 2;
+    CRVQ_TRY(set_smem_attr(argmin_tc_kernel<1>, argmin_smem(1)));
+    CRVQ_TRY(set_smem_attr(argmin_tc_kernel<2>, argmin_smem(2)));
     for (int64_t gs = g_begin; gs < g_begin + G_range; gs += G_sub) {
       const int64_t gn = std::min<int64_t>(G_sub, g_begin + G_range - gs);
       const int64_t nv = set.M * gn;
@@ -1573,18 +1675,25 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
         CRVQ_LAUNCHED();
       }
       {
-        // row tiles per CTA: about eight waves of three CTAs per SM (a fine-grained tail),
-        // each CTA reusing its group's resident codebook operand over several tiles
+        // row tiles per CTA: about eight waves of CTAs (three per SM with one half, two with
+        // two) for a fine-grained tail, each CTA reusing its group's resident codebook operand
+        // over several tiles (an even count with two halves)
         const int64_t row_tiles = ceil_div(set.M, tcenc::kRows);
-        const int64_t want_ctas = 24 * (int64_t)nsm;
+        const int64_t want_ctas = (two_halves ? 16 : 24) * (int64_t)nsm;
         const int64_t per_group = std::max<int64_t>(1, want_ctas / std::max<int64_t>(1, gn));
-        const int tiles = (int)std::max<int64_t>(1, ceil_div(row_tiles, per_group));
+        int tiles = (int)std::max<int64_t>(1, ceil_div(row_tiles, per_group));
+        if (two_halves) tiles += tiles & 1;
         const dim3 grid((unsigned)ceil_div(row_tiles, tiles), (unsigned)gn);
         ProfScope ps(st.cnt ? "encode_argmin_lloyd" : "encode_argmin", stream,
                      (double)nv * cw.K);
-        argmin_tc_kernel<<<grid, 128, kArgminSmem, stream>>>(set, gs, cbs, n_fixed, s_idx, out,
-                                                             out_ld, out_g0, fl, st, cbmax,
-                                                             bimg, tout, tiles, err);
+        if (two_halves)
+          argmin_tc_kernel<2><<<grid, 256, argmin_smem(2), stream>>>(
+              set, gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax, bimg, tout,
+              tiles, err);
+        else
+          argmin_tc_kernel<1><<<grid, 128, argmin_smem(1), stream>>>(
+              set, gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax, bimg, tout,
+              tiles, err);
         CRVQ_LAUNCHED();
       }
       {

@@ -74,13 +74,14 @@ constexpr int kDecWarps = 8;  // warps per CTA
 // reconstruction in the sorted order (32-byte stores, consecutive lanes on consecutive
 // vectors), each vector's error under H_g (the block loaded once for the warp's rows; the
 // quadratic form as two FMA chains in fp32) and, per (row, slice), the block loss, the
-// critical loss and ||dW||^2 as fp32 pairs in a fixed order, rounded to fp64 once:
-// row_part[(row * slices + slice) * 3 + {0, 1, 2}]. No shared memory and no block barrier:
+// critical loss and ||dW||^2 as fp32 pairs in a fixed order:
+// row_part[(row * slices + slice) * 3 + {0, 1, 2}] = (hi, lo). No shared memory and no block
+// barrier:
 // the kernel is bound by the latency of its loads, which full occupancy hides.
 __global__ void __launch_bounds__(kDecWarps * 32)
 decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
                   const float* __restrict__ Hb, CbList cbs, int64_t n_crit_groups, int slices,
-                  float* __restrict__ W_rec, double* __restrict__ row_part, unsigned* err) {
+                  float* __restrict__ W_rec, float2* __restrict__ row_part, unsigned* err) {
   const int lane = threadIdx.x & 31;
   const int64_t wid = (int64_t)blockIdx.x * kDecWarps + (threadIdx.x >> 5);
   const int64_t G = N / kD;
@@ -153,10 +154,10 @@ decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
       pair_merge(sq[r], sql[r], c0, c1);
     }
     if (lane == 0 && r < nr) {
-      double* o = row_part + ((i0 + r) * slices + sl) * 3;
-      o[0] = (double)lb[r] + (double)lbl[r];
-      o[1] = (double)lc[r] + (double)lcl[r];
-      o[2] = (double)sq[r] + (double)sql[r];
+      float2* o = row_part + ((i0 + r) * slices + sl) * 3;
+      o[0] = make_float2(lb[r], lbl[r]);
+      o[1] = make_float2(lc[r], lcl[r]);
+      o[2] = make_float2(sq[r], sql[r]);
     }
   }
 }
@@ -175,36 +176,51 @@ __global__ void invert_perm_kernel(const int32_t* __restrict__ perm, int64_t N,
   }
 }
 
-// One CTA of 1024 threads (short dependent fp64 chains: strided partials, then a tree).
+// One CTA of 1024 threads: the (row, slice) partials summed as fp32 pairs (strided, then a
+// tree; no dependent fp64 chain), the loss-product partials in fp64 (a few per thread).
 __global__ void __launch_bounds__(1024)
-finalize_losses_kernel(const double* __restrict__ row_part, int64_t M,
+finalize_losses_kernel(const float2* __restrict__ row_part, int64_t n_rows,
                        const double* __restrict__ gemm_part, int64_t n_gemm, int64_t n_tok,
                        double delta_host, const float* __restrict__ delta_dev,
                        double* __restrict__ losses) {
-  __shared__ double red[4][1024];
-  double a = 0, b = 0, c = 0, e = 0;
-  for (int64_t i = threadIdx.x; i < M; i += blockDim.x) {
-    a += row_part[i * 3 + 0];
-    b += row_part[i * 3 + 1];
-    c += row_part[i * 3 + 2];
+  __shared__ float red_h[3][1024], red_l[3][1024];
+  __shared__ double red_e[1024];
+  float h[3] = {0.f, 0.f, 0.f}, l[3] = {0.f, 0.f, 0.f};
+  for (int64_t i = threadIdx.x; i < n_rows; i += blockDim.x) {
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+      const float2 v = row_part[i * 3 + q];
+      pair_merge(h[q], l[q], v.x, v.y);
+    }
   }
+  double e = 0.0;
   for (int64_t i = threadIdx.x; i < n_gemm; i += blockDim.x) e += gemm_part[i];
-  red[0][threadIdx.x] = a;
-  red[1][threadIdx.x] = b;
-  red[2][threadIdx.x] = c;
-  red[3][threadIdx.x] = e;
+#pragma unroll
+  for (int q = 0; q < 3; ++q) {
+    red_h[q][threadIdx.x] = h[q];
+    red_l[q][threadIdx.x] = l[q];
+  }
+  red_e[threadIdx.x] = e;
   __syncthreads();
   for (int w = 512; w > 0; w >>= 1) {
-    if ((int)threadIdx.x < w)
-      for (int q = 0; q < 4; ++q) red[q][threadIdx.x] += red[q][threadIdx.x + w];
+    if ((int)threadIdx.x < w) {
+#pragma unroll
+      for (int q = 0; q < 3; ++q) {
+        float hh = red_h[q][threadIdx.x], ll = red_l[q][threadIdx.x];
+        pair_merge(hh, ll, red_h[q][threadIdx.x + w], red_l[q][threadIdx.x + w]);
+        red_h[q][threadIdx.x] = hh;
+        red_l[q][threadIdx.x] = ll;
+      }
+      red_e[threadIdx.x] += red_e[threadIdx.x + w];
+    }
     __syncthreads();
   }
   if (threadIdx.x == 0) {
-    losses[0] = red[0][0];
-    losses[1] = red[1][0];
+    losses[0] = (double)red_h[0][0] + (double)red_l[0][0];
+    losses[1] = (double)red_h[1][0] + (double)red_l[1][0];
     if (gemm_part) {
       const double delta = delta_dev ? (double)*delta_dev : delta_host;
-      losses[2] = red[3][0] / (double)n_tok + delta * red[2][0];
+      losses[2] = red_e[0] / (double)n_tok + delta * ((double)red_h[2][0] + (double)red_l[2][0]);
     } else {
       losses[2] = __longlong_as_double(0x7ff8000000000000ll);  // NaN: no X given
     }
@@ -236,14 +252,15 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   const bool rec_is_out = W_hat && !perm;
   const size_t rec_bytes = (need_rec && !rec_is_out) ? align_up((size_t)M * N * 4, 256) : 0;
   const size_t inv_bytes = (W_hat && perm) ? align_up((size_t)N * 4, 256) : 0;
-  const size_t part_bytes = (size_t)M * slices * 3 * sizeof(double) +
+  const size_t part_bytes = align_up((size_t)M * slices * 3 * sizeof(float2), 256) +
                             (size_t)(n_gemm_cap + 1) * sizeof(double);
   Scratch mem;
   CRVQ_TRY(mem.alloc(rec_bytes + inv_bytes + part_bytes, stream));
   float* W_rec = rec_is_out ? W_hat : (need_rec ? mem.as<float>() : nullptr);
   int32_t* inv = inv_bytes ? reinterpret_cast<int32_t*>(mem.as<char>() + rec_bytes) : nullptr;
-  double* row_part = reinterpret_cast<double*>(mem.as<char>() + rec_bytes + inv_bytes);
-  double* gemm_part = row_part + M * slices * 3;
+  float2* row_part = reinterpret_cast<float2*>(mem.as<char>() + rec_bytes + inv_bytes);
+  double* gemm_part = reinterpret_cast<double*>(
+      reinterpret_cast<char*>(row_part) + align_up((size_t)M * slices * 3 * sizeof(float2), 256));
   {
     ProfScope ps("decode_rows", stream,
                  (double)M * N * 4.0 * (1.0 + (W_rec ? 1.0 : 0.0)));
