@@ -294,7 +294,7 @@ stats_solve_kernel(const float* __restrict__ Hb, StatsView st, const float* C_ol
   if (k < K) {
     const int64_t gper = (st.G_cov + kSolveSlices - 1) / kSolveSlices;
     const int64_t g0 = sl * gper, g1 = min(st.G_cov, g0 + gper);
-    constexpr int kBatch = 8;  // loads of 8 groups in flight together; no branches
+    constexpr int kBatch = 16;  // loads of 16 groups in flight together; no branches
     for (int64_t gb = g0; gb < g1; gb += kBatch) {
       float fc[kBatch], h[kBatch];
 #pragma unroll
@@ -340,7 +340,7 @@ stats_solve_kernel(const float* __restrict__ Hb, StatsView st, const float* C_ol
   const float* Ah = part_h[kk][0];
   const float* Al = part_l[kk][0];
   // the count: an exact integer held by the pair
-  const int64_t count = (int64_t)Ah[36] + (int64_t)Al[36];
+  const int64_t count = (int64_t)__float2int_rn(Ah[36]) + (int64_t)__float2int_rn(Al[36]);
   if (counts_out) counts_out[k] = (int32_t)count;
   bool keep = count == 0;
   float out[kD];
