@@ -151,6 +151,32 @@ __device__ __forceinline__ void vector_terms(const float r[kD], const float a[kD
   }
 }
 
+// vector_terms plus rr = r^T (H r) and Ra = a^T (|H| a), each row of H read once as two
+// float4 (H 16-byte aligned): the same FMA chains, so the same values as computing them apart.
+__device__ __forceinline__ void vector_terms_rr(const float r[kD], const float a[kD],
+                                                const float* H, float m2q[kD], float& pmax,
+                                                float& rr, float& ra) {
+  pmax = 0.f;
+  rr = 0.f;
+  ra = 0.f;
+#pragma unroll
+  for (int p = 0; p < kD; ++p) {
+    const float4 h0 = *reinterpret_cast<const float4*>(H + p * kD);
+    const float4 h1 = *reinterpret_cast<const float4*>(H + p * kD + 4);
+    const float hr[kD] = {h0.x, h0.y, h0.z, h0.w, h1.x, h1.y, h1.z, h1.w};
+    float q = 0.f, pa = 0.f;
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      q = fmaf(hr[j], r[j], q);
+      pa = fmaf(fabsf(hr[j]), a[j], pa);
+    }
+    m2q[p] = -2.f * q;
+    pmax = fmaxf(pmax, pa);
+    rr = fmaf(r[p], q, rr);
+    ra = fmaf(a[p], pa, ra);
+  }
+}
+
 // Stage the codewords [k0, k0 + nk): sC = c, sN = n - u C Na (the lower-bound offset of the
 // codeword part), sL = ||c||_1.
 __device__ __forceinline__ void stage_chunk(const float* __restrict__ C, int k0, int nk,
@@ -482,7 +508,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   long long* s_bacc = reinterpret_cast<long long*>(Bbuf + 2 * kTcBTile);  // [8][256]
   int* s_cnt = reinterpret_cast<int*>(s_bacc + kTcSmemStatsK * kD);       // [256]
   float* sQ = reinterpret_cast<float*>(s_cnt + kTcSmemStatsK);            // [128 HALVES][8]
-  __shared__ float sH[kD * kD];
+  __shared__ __align__(16) float sH[kD * kD];
   __shared__ __align__(8) uint64_t bar_mma_s[HALVES], bar_b[2];
   __shared__ uint32_t tmem_slot;
 
@@ -574,16 +600,8 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
 #pragma unroll
         for (int j = 0; j < kD; ++j) rv[j] = a[j] = 0.f;
       }
-      vector_terms(rv, a, sH, m2q, pmax);
-      float rr = 0.f, ra = 0.f;
-#pragma unroll
-      for (int p = 0; p < kD; ++p) {
-        rr = fmaf(rv[p], -0.5f * m2q[p], rr);
-        float pa = 0.f;
-#pragma unroll
-        for (int j = 0; j < kD; ++j) pa = fmaf(fabsf(sH[p * kD + j]), a[j], pa);
-        ra = fmaf(a[p], pa, ra);
-      }
+      float rr, ra;
+      vector_terms_rr(rv, a, sH, m2q, pmax, rr, ra);
       // offset making every D = low + off >= 0, with margins for every rounding involved
       off = (rr + 32.f * kU * ra + 2.f * uc * (hrow * l1max * cinf + 2.f * pmax * l1max)) *
                 (1.f + 4.f * uc) + 1e-30f;
@@ -1109,7 +1127,7 @@ __device__ __forceinline__ void hyp_terms_pair(const float rh[kD], const float r
 // Fast stage: one thread per vector, the stage codebook chunked through shared memory, a
 // sorted top-L list (L >= Bs + 1) of lower bounds low = approx_err - Et in registers.
 template <int L>
-__global__ void __launch_bounds__(kThreads)
+__global__ void __launch_bounds__(kThreads, L <= 9 ? 3 : 2)
 beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc sd,
                   BeamBufs bb, FlagList flags, unsigned* err) {
   const int64_t g = g_begin + blockIdx.y;

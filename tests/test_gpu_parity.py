@@ -310,12 +310,16 @@ def test_update_is_deterministic(c1):
 
 
 # ------------------------------------------------------------------------------ S7 losses
-@pytest.mark.parametrize("shape", ["c1", "wide"])
+@pytest.mark.parametrize("shape", ["c1", "wide", "ragged"])
 def test_reconstruct_error_parity(c1, shape):
     if shape == "c1":
         W, X, H, delta = c1["W"], c1["X"], c1["H"], float(c1["delta"])
-    else:  # N = 2056 channels: the full-loss product is split over three K chunks
-        cfg = S.C1.with_(name="recon_wide", M=200, N=2056, n_tok=300)
+    else:
+        # wide: N = 2056 channels, the full-loss product over three K chunks; ragged: M = 203
+        # rows (not a multiple of the decode's 4 rows per warp), G = 33 groups (a ragged last
+        # group slice), n_tok = 77
+        M_, N_, n_ = (200, 2056, 300) if shape == "wide" else (203, 264, 77)
+        cfg = S.C1.with_(name=f"recon_{shape}", M=M_, N=N_, n_tok=n_)
         W, X = S.gen_W(cfg), S.gen_X(cfg)
         H, _, _, delta = O.hessian(X, cfg.damp_rel, D)
         delta = float(delta)
@@ -344,6 +348,13 @@ def test_reconstruct_error_parity(c1, shape):
     Wh2, lb2, _, lf2 = P.crvq_reconstruct_error(dev(Ws), D, dev(Hb), None, cbs, Gc)
     assert lf2 is None
     np.testing.assert_array_equal(host(Wh2), O.reconstruct_error(Ws, D, Hb, None, ocbs, Gc)[0])
+    # identity order with X's columns taken in the sorted order beforehand: the same full loss
+    # (the channel sum of the loss product in another order)
+    Xs = np.ascontiguousarray(X[:, perm])
+    _, lb3, lc3, lf3 = P.crvq_reconstruct_error(dev(Ws), D, dev(Hb), None, cbs, Gc, X=dev(Xs),
+                                                damp_delta=delta)
+    assert lb3 == lb and lc3 == lc
+    assert abs(lf3 - lfo) <= 2e-5 * lfo
 
 
 # ------------------------------------------------------------------------------ errors
