@@ -182,6 +182,21 @@ def dist_init():
     return ws, rank, local
 
 
+def rank_aggregate(tot_ms, scores, ws, device):
+    """Whole-job figures of a weak-scaling run: the slowest rank's time and every rank's scores
+    (value = all ranks' scores / the slowest rank's time). One process per GPU; the two
+    reductions go through torch.distributed (NCCL on GPUs, gloo on CPU)."""
+    if ws <= 1:
+        return float(tot_ms), float(scores)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([tot_ms], dtype=torch.float64, device=device)
+    sc = torch.tensor([scores], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(sc, op=dist.ReduceOp.SUM)
+    return float(t[0]), float(sc[0])
+
+
 def _cuda_ok():
     import torch
     return torch.cuda.is_available()
@@ -358,16 +373,7 @@ def main():
     run_step()
     torch.cuda.synchronize()
     kstats = P.crvq_profile_end()
-    tot_ms = sum(step_ms)
-    if ws > 1:
-        import torch.distributed as dist
-        t = torch.tensor([tot_ms, scores], dtype=torch.float64, device=dev)
-        tmax = t[:1].clone()
-        dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
-        dist.all_reduce(t[1:], op=dist.ReduceOp.SUM)
-        tot_ms_max, scores_all = float(tmax[0]), float(t[1])
-    else:
-        tot_ms_max, scores_all = tot_ms, scores
+    tot_ms_max, scores_all = rank_aggregate(sum(step_ms), scores, ws, dev)
     value = scores_all / (tot_ms_max / 1e3)
 
     # End to end through the public C ABI with host buffers (pinned): H2D of W and X and D2H
