@@ -55,7 +55,7 @@ typedef int32_t crvq_status;
 enum {
   CRVQ_OK = 0,
   CRVQ_ERR_INVALID_ARG = -1, /* a pointer, size or option is out of its documented range */
-  CRVQ_ERR_UNSUPPORTED = -2, /* a valid request this build does not implement (e.g. d != 8) */
+  CRVQ_ERR_UNSUPPORTED = -2, /* a valid request the library does not implement (e.g. d != 8) */
   CRVQ_ERR_CUDA = -3,        /* a CUDA runtime call failed */
   CRVQ_ERR_NOMEM = -4,       /* device memory allocation failed */
   CRVQ_ERR_TIMEOUT = -5,     /* a bounded device-side wait ran out */
