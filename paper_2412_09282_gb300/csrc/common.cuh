@@ -47,6 +47,32 @@ void count_launch();
     CRVQ_CUDA(cudaGetLastError());   \
   } while (0)
 
+// Programmatic dependent launch. A kernel launched by launch_pdl may be scheduled while its
+// stream predecessor (a kernel) is still running: it lets its own dependents launch
+// (pdl_trigger) and then waits for the predecessor to complete with its memory visible
+// (pdl_wait) before it reads anything or allocates tensor memory. Both are no-ops in a kernel
+// launched without the attribute. Removes the launch gap between dependent kernels of a layer.
+__device__ __forceinline__ void pdl_trigger() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t stream, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 // Brackets the launches in its scope with CUDA events when profiling is on.
 class ProfScope {
  public:

@@ -339,6 +339,8 @@ __global__ void __launch_bounds__(128)
 prep_b_kernel(SetView set, int64_t g_begin, int64_t G_range, const float* __restrict__ C,
               int K, int nchunk, float uc, char* __restrict__ out, float4* __restrict__ terms,
               float* __restrict__ cbmax) {
+  pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
+  pdl_wait();
   if (blockIdx.x == gridDim.x - 1) {  // the last CTA: the codebook maxima
     cbmax_block(C, K, cbmax);
     return;
@@ -499,6 +501,8 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
                  FlagList flags, StatsView st, const float* __restrict__ cbmax,
                  const char* __restrict__ bpre, const float4* __restrict__ terms, int tiles,
                  unsigned* err) {
+  pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
+  pdl_wait();
   using namespace tcenc;
   extern __shared__ __align__(1024) char smem_raw[];
   // 1024-byte aligned base, derived from the shared array (keeps the shared address space)
@@ -799,6 +803,8 @@ argmin_exact_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs, i
                     int s_idx, int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
                     FlagList flags, StatsView st, const float4* __restrict__ terms,
                     unsigned* err) {
+  pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
+  pdl_wait();
   __shared__ float sH[kD * kD];
   __shared__ float redf[4];
   __shared__ int cand[256];
@@ -926,6 +932,8 @@ argmin_exact_warp_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList c
                          int n_fixed, int s_idx, int32_t* __restrict__ out_code, int64_t out_ld,
                          int64_t out_g0, FlagList flags, StatsView st,
                          const float4* __restrict__ terms, unsigned* err) {
+  pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
+  pdl_wait();
   __shared__ float sHw[4][kD * kD];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const unsigned cnt = min((unsigned long long)*flags.count, (unsigned long long)flags.cap);
@@ -1688,8 +1696,10 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
       {
         ProfScope pb("encode_prep_b", stream, (double)gn * nchunk * kTcCols);
         const int64_t rows = gn * nchunk * kTcCols;
-        prep_b_kernel<<<(unsigned)std::min<int64_t>(ceil_div(rows, 128), 16 * nsm) + 1, 128, 0,
-                        stream>>>(set, gs, gn, cw.C, cw.K, nchunk, uc, bimg, tout, cbmax);
+        CRVQ_CUDA(launch_pdl(prep_b_kernel,
+                             dim3((unsigned)std::min<int64_t>(ceil_div(rows, 128), 16 * nsm) + 1),
+                             dim3(128), 0, stream, set, gs, gn, cw.C, cw.K, nchunk, uc, bimg,
+                             tout, cbmax));
         CRVQ_LAUNCHED();
       }
       {
@@ -1705,24 +1715,27 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
         ProfScope ps(st.cnt ? "encode_argmin_lloyd" : "encode_argmin", stream,
                      (double)nv * cw.K);
         if (two_halves)
-          argmin_tc_kernel<2><<<grid, 256, argmin_smem(2), stream>>>(
-              set, gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax, bimg, tout,
-              tiles, err);
+          CRVQ_CUDA(launch_pdl(argmin_tc_kernel<2>, grid, dim3(256), argmin_smem(2), stream, set,
+                               gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax,
+                               bimg, tout, tiles, err));
         else
-          argmin_tc_kernel<1><<<grid, 128, argmin_smem(1), stream>>>(
-              set, gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax, bimg, tout,
-              tiles, err);
+          CRVQ_CUDA(launch_pdl(argmin_tc_kernel<1>, grid, dim3(128), argmin_smem(1), stream, set,
+                               gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax,
+                               bimg, tout, tiles, err));
         CRVQ_LAUNCHED();
       }
       {
         ProfScope pf("encode_argmin_exact", stream, 0.0);
         if (cw.K <= kExactWarpK) {
-          argmin_exact_warp_kernel<<<(unsigned)std::min<int64_t>(ceil_div(nv, 4), 16 * nsm),
-                                     128, 0, stream>>>(set, gs, gn, cbs, n_fixed, s_idx, out,
-                                                       out_ld, out_g0, fl, st, tout, err);
+          CRVQ_CUDA(launch_pdl(argmin_exact_warp_kernel,
+                               dim3((unsigned)std::min<int64_t>(ceil_div(nv, 4), 16 * nsm)),
+                               dim3(128), 0, stream, set, gs, gn, cbs, n_fixed, s_idx, out,
+                               out_ld, out_g0, fl, st, tout, err));
         } else {
-          argmin_exact_kernel<<<(unsigned)std::min<int64_t>(nv, 16 * nsm), 128, 0, stream>>>(
-              set, gs, gn, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, tout, err);
+          CRVQ_CUDA(launch_pdl(argmin_exact_kernel,
+                               dim3((unsigned)std::min<int64_t>(nv, 16 * nsm)), dim3(128), 0,
+                               stream, set, gs, gn, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl,
+                               st, tout, err));
         }
         CRVQ_LAUNCHED();
       }

@@ -278,6 +278,8 @@ constexpr int kSolveThreads = kSolveK * kSolveSlices * kNA;  // 592
 __global__ void __launch_bounds__(kSolveThreads)
 stats_solve_kernel(const float* __restrict__ Hb, StatsView st, const float* C_old, float* C_out,
                    int32_t* __restrict__ counts_out, unsigned* err) {
+  pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
+  pdl_wait();
   __shared__ float part_h[kSolveK][kSolveSlices][kNA], part_l[kSolveK][kSolveSlices][kNA];
   const int tid = threadIdx.x;
   const int kk = tid / (kSolveSlices * kNA);
@@ -376,8 +378,8 @@ crvq_status launch_solve_kernels(const float* Hb, const StatsView& st, const flo
                                  float* C_out, int32_t* counts, unsigned* err,
                                  cudaStream_t stream) {
   ProfScope ps("update_solve", stream, (double)st.K);
-  stats_solve_kernel<<<(unsigned)ceil_div(st.K, kSolveK), kSolveThreads, 0, stream>>>(
-      Hb, st, C_old, C_out, counts, err);
+  CRVQ_CUDA(launch_pdl(stats_solve_kernel, dim3((unsigned)ceil_div(st.K, kSolveK)),
+                       dim3(kSolveThreads), 0, stream, Hb, st, C_old, C_out, counts, err));
   CRVQ_LAUNCHED();
   return CRVQ_OK;
 }
