@@ -429,7 +429,9 @@ def main():
             "avg_launch_ms": enc_ms / max(enc_launches, 1), "launches": enc_launches,
             "tensor": {"achieved": tensor_tflops, "unit": "TFLOP/s",
                        "peak": tf32_peak, "frac": tensor_tflops / tf32_peak,
-                       "work": "64 tf32 flop per scored pair (K = 32 split operands)",
+                       "work": "64 tf32 flop per scored pair issued (K = 32 split operands)",
+                       "algorithmic_frac": tensor_tflops / 4.0 / tf32_peak,
+                       "algorithmic_work": "2 d = 16 flop per scored pair",
                        "peak_source": f"0.5 x bf16 {peak_src} ({peaks.get('bf16_tflops')})"}}
     last = work[-1]["out"].report if len(work) == 1 else None
     line = {
