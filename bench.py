@@ -443,7 +443,7 @@ def main():
         "roofline": roof,
         "e2e": e2e,
         "gpu_launches": int(launches),
-        "fp64_fallback_decisions_per_step": sum(w["out"].report["flagged"] for w in work),
+        "exact_fallback_decisions_per_step": sum(w["out"].report["flagged"] for w in work),
         "kernels": [{"name": k["name"], "launches": k["launches"], "ms": k["ms"],
                      "share": k["ms"] / total_k} for k in ks[:12]],
         "clocks": clk,

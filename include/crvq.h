@@ -36,9 +36,11 @@
  * Score. Vector t against reconstruction r: err = (t - r)^T H_g (t - r), the block-diagonal
  * part of the Alg. 1 loss ||W X - W_enc X||^2 written with H = X^T X / n + delta I. With
  * H_g = c I it is the squared L2 distance of Sec. 3.1 Eq. (2)-(3). Code indices are decided
- * exactly: scores are computed in fp32 with a rigorous error bound and any decision closer
- * than that bound is re-taken in fp64, so codes equal those of an fp64 evaluation except
- * for ties at fp64 rounding level (ties go to the smaller index / earlier tuple).
+ * exactly: scores are computed in fp32 (on the tensor cores for one searched codebook) with
+ * a rigorous error bound, and any decision closer than that bound is re-taken exactly (errs
+ * as unevaluated fp32 pairs, about 2^-44 relative, or in fp64), so codes equal those of an
+ * fp64 evaluation except for ties at rounding level (ties go to the smaller index / earlier
+ * tuple).
  */
 #ifndef CRVQ_H
 #define CRVQ_H
@@ -205,8 +207,9 @@ crvq_status crvq_encode_beam(const float* T, int64_t ldT, int64_t M, int64_t G_s
  * closed-form minimiser). Codebook `which` is refitted with all others fixed: the members v
  * of cluster k (vectors with code k, g < G_cov) have targets tau_v = t_v - sum over the other
  * covering codebooks of C[code]; c_k solves (sum_v H_{g_v}) c = sum_v H_{g_v} tau_v
- * (Cholesky, fp64 sums in a fixed order, so results are reproducible). Empty clusters keep
- * their codeword.   C_out [K x d] out (may alias cbs[which].C).
+ * (right side in 64-bit fixed point, normal matrix as fp32 pairs, both summed in a fixed order;
+ * Cholesky with refinement in fp32 pairs, so results are reproducible bit for bit). Empty
+ * clusters keep their codeword.   C_out [K x d] out (may alias cbs[which].C).
  *   counts [K] int32 out or NULL: cluster sizes.
  */
 crvq_status crvq_update_codebook(const float* T, int64_t ldT, int64_t M, int64_t G_sub,
@@ -301,7 +304,7 @@ typedef struct crvq_layer_report {
   double loss_before_refine;
   double scores;         /* (hypothesis, codeword) pairs scored by the encode passes */
   int64_t n_crit_groups;
-  int64_t flagged;       /* encode decisions re-taken in fp64 (fp32 bound not conclusive) */
+  int64_t flagged;       /* encode decisions re-taken exactly (fp32 bound not conclusive) */
   int32_t refine_rounds_done;
   int32_t _pad;
 } crvq_layer_report;
