@@ -1703,11 +1703,13 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
         CRVQ_LAUNCHED();
       }
       {
-        // row tiles per CTA: about eight waves of CTAs (three per SM with one half, two with
-        // two) for a fine-grained tail, each CTA reusing its group's resident codebook operand
-        // over several tiles (an even count with two halves)
+        // row tiles per CTA: about eight waves of three CTAs per SM with one half (a
+        // fine-grained tail); with two halves about four waves of two (fewer statistics
+        // flushes and codebook fetches; measured 3% faster than eight waves, 10% faster than
+        // sixteen), each CTA reusing its group's resident codebook operand over several tiles
+        // (an even count with two halves)
         const int64_t row_tiles = ceil_div(set.M, tcenc::kRows);
-        const int64_t want_ctas = (two_halves ? 16 : 24) * (int64_t)nsm;
+        const int64_t want_ctas = (two_halves ? 8 : 24) * (int64_t)nsm;
         const int64_t per_group = std::max<int64_t>(1, want_ctas / std::max<int64_t>(1, gn));
         int tiles = (int)std::max<int64_t>(1, ceil_div(row_tiles, per_group));
         if (two_halves) tiles += tiles & 1;
