@@ -55,9 +55,9 @@ def schedule_scores(cfg, M, N):
 
 
 # dram__bytes_read.sum + dram__bytes_write.sum of one arg-min launch (ncu --set full, a Lloyd
-# pass over the prequantize codebook of the c2 workload: 86.7 MB read + 5.0 MB written; set to None
+# pass over the prequantize codebook of the c2 workload: 86.7 MB read + 4.8 MB written; set to None
 # whenever the kernel changes until the counters are taken again)
-ARGMIN_TRAFFIC = 91.69e6
+ARGMIN_TRAFFIC = 91.48e6
 
 
 def load_peaks():
