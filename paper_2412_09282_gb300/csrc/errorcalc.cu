@@ -4,9 +4,10 @@
 //   loss_crit  = the same over the critical groups g < G_c
 //   loss_full  = ||dW X^T||^2 / n + delta ||dW||^2 = tr(dW H dW^T)
 // The reconstruction is formed in the sorted channel order and gathered back to the original
-// order; per-(row, group slice) sums are fp32 pairs, reduced in fp64 in a fixed order. The full
-// loss takes dW and X's columns in the sorted order (a permutation of the channel sum) on the
-// tensor cores (tc_gemm.cu: tf32 operand images, tcgen05 3xTF32).
+// order; per-(row, group slice) sums are fp32 pairs, reduced as fp32 pairs in a fixed order
+// and rounded to fp64 once. The full loss takes dW and X's columns in the sorted order (a
+// permutation of the channel sum) on the tensor cores (tc_gemm.cu: tf32 operand images,
+// tcgen05 3xTF32).
 #include "common.cuh"
 #include "kernels.h"
 

@@ -1,9 +1,11 @@
 // S1: Hessian proxy H = X^T X / n + delta I (App. A.2; the paper's X is N x O and its proxy
 // XX^T is the same matrix as our X^T X).
 //
-// The product X^T X runs on the tensor cores (tc_gemm.cuh: tcgen05, 3xTF32, tiles on or above
-// the diagonal, mirrored; K split into 1024-token chunks summed in fp64). A single CTA then
-// takes the diagonal, the damping and the original-order diagonal blocks.
+// The dense product X^T X (the crvq_hessian entry) runs on the tensor cores (tc_gemm.cuh:
+// tcgen05, 3xTF32, tiles on or above the diagonal, mirrored; K split into 1024-token chunks
+// summed in fp32 in chunk order). A single CTA then takes the diagonal, the damping and the
+// original-order diagonal blocks. The layer schedule forms only the diagonal blocks
+// (launch_tc_hessian_blocks in tc_gemm.cu), with the same values.
 #include "common.cuh"
 #include "kernels.h"
 

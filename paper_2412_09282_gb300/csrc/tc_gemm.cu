@@ -1,8 +1,9 @@
-// Host side of the tcgen05 3xTF32 GEMM (tc_gemm.cuh) and the fixed-order reductions of its
-// split-K partial products. The tensor core accumulates fp32 with a small systematic
-// rounding bias per accumulation step, so K is cut into chunks of at most kKChunk and the
-// few chunk partials of an element are summed afterwards in fp32, in chunk order (a relative
-// error of a few u); the sums of squares over elements are reduced in fp64.
+// Host side of the tcgen05 3xTF32 products: the dense symmetric X^T X and its diagonal blocks
+// alone (tc_gemm.cuh), and the image-fed sum of squares ||(A - A_sub) B^T||^2 of the full loss
+// (img:: below). The tensor core accumulates fp32 with a small systematic rounding bias per
+// accumulation step, so K is cut into chunks of at most kKChunk and the few chunk partials of
+// an element are summed afterwards in fp32, in chunk order (a relative error of a few u); the
+// squares are summed per row in fp32 and per tile in fp64.
 #include <algorithm>
 
 #include "common.cuh"

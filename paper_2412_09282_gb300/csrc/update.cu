@@ -6,10 +6,11 @@
 // Deterministic by construction, with no sort and no float atomics: cnt[g][k] are integer
 // counts, b_k is accumulated in 64-bit fixed point (stats.cuh), A_k is summed as fp32 pairs in
 // a fixed order (partial sums over fixed slices of the groups, added in slice order), and the
-// 8 x 8 system is solved to fp64 accuracy by mixed-precision iterative refinement, in one
-// kernel. GB300's fp64 pipe is a small fraction of its fp32 rate, so none of this
-// arithmetic runs per element in fp64. The Lloyd encode
-// pass (encode.cu) accumulates the same statistics for the codes it writes.
+// 8 x 8 system is solved by an fp32 Cholesky factor with iterative refinement whose residual
+// is formed in fp32 pairs (to 2^-40 of the solution), in one kernel. GB300's fp64 pipe is a
+// small fraction of its fp32 rate and a dependent fp64 operation costs about 180 cycles, so
+// none of this arithmetic runs in fp64. The Lloyd encode pass (encode.cu) accumulates the
+// same statistics for the codes it writes.
 #include <algorithm>
 #include <cmath>
 
