@@ -91,3 +91,42 @@ def test_validation_rejects_before_launch(lib):
     # unknown importance mode
     assert lib.crvq_select_reorder_channels(dummy, 2, 16, 8, dummy, dummy, dummy, 0.5, 7, 0,
                                             dummy, None, dummy, dummy, c.byref(gc), None) == -1
+
+
+def test_quantize_layer_rejects_bad_shapes_and_options_before_launch(lib):
+    """crvq_quantize_layer validates its shapes and configuration before any CUDA call."""
+    from paper_2412_09282_gb300 import _lib
+    c = ctypes
+    dummy = c.c_void_p(16)
+    outs = _lib.crvq_layer_outputs(dummy, dummy, dummy, dummy, dummy, None, None)
+    rep = _lib.crvq_layer_report()
+
+    def cfg(**kw):
+        base = dict(d=8, K_base=256, n_ext=1, K_ext=256, crit_frac=0.02, B=8, kmeans_iters=10,
+                    refine_rounds=1, eps_rel=1e-3, damp_rel=0.01, importance_mode=0, seed=0)
+        base.update(kw)
+        return _lib.crvq_config(**base)
+
+    def call(M=512, N=512, n_tok=64, **kw):
+        cf = cfg(**kw)
+        return lib.crvq_quantize_layer(dummy, dummy, M, N, n_tok, c.byref(cf), c.byref(outs),
+                                       c.byref(rep), None)
+
+    assert call(d=16) == -2                       # only d = 8 is implemented
+    assert call(N=500) == -1                      # N % d != 0
+    assert call(N=49160) == -1                    # beyond the channel limit
+    assert call(M=0) == -1
+    assert call(n_tok=0) == -1
+    assert call(K_base=0) == -1
+    assert call(M=4, N=64, K_base=64) == -1       # K_base > M * G (32 vectors)
+    assert call(n_ext=8) == -1                    # at most 7 extended codebooks
+    assert call(crit_frac=1.5) == -1
+    assert call(B=17) == -1
+    assert call(kmeans_iters=-1) == -1
+    assert call(importance_mode=3) == -1
+    assert call(damp_rel=-1.0) == -1
+    assert call(crit_frac=0.0) == -1              # extended codebooks need a critical group
+    assert b"critical" in lib.crvq_last_error()
+    # a NULL required pointer
+    assert lib.crvq_quantize_layer(None, dummy, 512, 512, 64, c.byref(cfg()), c.byref(outs),
+                                   c.byref(rep), None) == -1
