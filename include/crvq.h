@@ -88,6 +88,14 @@ crvq_status crvq_sync(crvq_stream_t stream);
 /* Library build string (compiler, architecture). Host memory, static. */
 const char* crvq_version(void);
 
+/* Self-test of the failure path of every bounded device wait: one thread waits on an
+ * mbarrier that nothing ever arrives on, with the same bounded wait the tensor-core kernels
+ * use (2 s of %globaltimer); it gives up, records the timeout in the device error word and
+ * exits, so the context stays usable. The next crvq_sync on the device returns
+ * CRVQ_ERR_TIMEOUT (and clears it). Enqueues on `stream`; no trap, no fault, no unbounded
+ * spin. */
+crvq_status crvq_selftest_bounded_wait(crvq_stream_t stream);
+
 /* Per-kernel timing. Between crvq_profile_begin() and crvq_profile_end(), every kernel the
  * library launches is bracketed by CUDA events recorded on the stream it is launched on.
  * crvq_profile_end() waits for them and writes one entry per kernel name (host memory,
@@ -310,7 +318,8 @@ typedef struct crvq_layer_report {
 } crvq_layer_report;
 
 /*
- * One weight matrix through Alg. 1 lines 3-17 (everything but block / end-to-end fine-tuning):
+ * One weight matrix through Alg. 1, prequantization through the refinement loop (everything
+ * but block / end-to-end fine-tuning):
  * S1 Hessian; S2 prequantize (k-means + encode in the original order); S3 importance and
  * reorder; S4 base codebook (k-means over all vectors); S5 each extended codebook (k-means
  * on the critical residual, greedy encode); S6 up to refine_rounds rounds of

@@ -358,7 +358,7 @@ def avg_bits(e, d, m, lam, M=4096, N=4096, include_perm=False):
 
 
 # --------------------------------------------------------------------------------------
-# S1-S7: one weight matrix through Alg. 1 lines 3-17
+# S1-S7: one weight matrix through Alg. 1, prequantization through the refinement loop
 # --------------------------------------------------------------------------------------
 PHASE_PREQUANT, PHASE_BASE, PHASE_EXT, PHASE_RANDOM = 1, 2, 3, 4
 
@@ -385,7 +385,7 @@ def lloyd(T, d, H_blocks, fixed, C0, G_cov, iters, seed_unused=None):
 
 
 def quantize_layer(W, X, cfg):
-    """The whole per-matrix schedule (Alg. 1 lines 3-17) with the readings above.
+    """The whole per-matrix schedule (Alg. 1, prequantization through the refinement loop) with the readings above.
 
     cfg has attributes d, K_base, n_ext, K_ext, crit_frac, B, kmeans_iters, refine_rounds,
     eps_rel, damp_rel, importance_mode, seed. Returns a dict of every intermediate result."""
@@ -397,22 +397,22 @@ def quantize_layer(W, X, cfg):
     # S1
     H, xsq, Hb0, delta = hessian(X, cfg.damp_rel, d)
     out.update(H=H, xsq=xsq, H_blocks_orig=Hb0, delta=delta)
-    # S2: prequantize in the original order (Alg. 1 line 3)
+    # S2: prequantize in the original order (Alg. 1, prequantization step)
     C0 = kmeans_init(W, d, G, cfg.K_base, phase_seed(cfg.seed, PHASE_PREQUANT, 0))
     pre, _ = lloyd(W, d, Hb0, [], C0, G, cfg.kmeans_iters)
     W_pre, pre_loss, _, _ = reconstruct_error(W, d, Hb0, None, [pre], 0)
     out.update(C_pre=pre.C, codes_pre=pre.codes, W_pre=W_pre, loss_pre=pre_loss)
-    # S3 (Alg. 1 lines 4-5)
+    # S3 (Alg. 1, importance and reordering steps)
     perm, I, Ws, Hb, Gc = select_reorder_channels(
         W, d, W_pre, xsq, H, cfg.crit_frac, cfg.importance_mode,
         phase_seed(cfg.seed, PHASE_RANDOM, 0))
     out.update(perm=perm, importance=I, W_sorted=Ws, H_blocks=Hb, n_crit_groups=Gc)
-    # S4 (Alg. 1 lines 6-7)
+    # S4 (Alg. 1, base codebook steps)
     Cb0 = kmeans_init(Ws, d, G, cfg.K_base, phase_seed(cfg.seed, PHASE_BASE, 0))
     base, obj = lloyd(Ws, d, Hb, [], Cb0, G, cfg.kmeans_iters)
     out["base_objective"] = obj
     cbs = [base]
-    # S5 (Alg. 1 lines 8-13): extended codebooks on the critical residual
+    # S5 (Alg. 1, extended-codebook loop): extended codebooks on the critical residual
     crit_losses = [reconstruct_error(Ws, d, Hb, perm, cbs, Gc)[2]]
     Tc = Ws[:, :Gc * d]
     Hbc = Hb[:Gc]
@@ -423,7 +423,7 @@ def quantize_layer(W, X, cfg):
         cbs.append(Codebook(ext.C, ext.codes, Gc))
         crit_losses.append(reconstruct_error(Ws, d, Hb, perm, cbs, Gc)[2])
     out["crit_loss_after_ext"] = crit_losses
-    # S6 (Alg. 1 lines 14-17): LS codebook updates + joint beam re-encode
+    # S6 (Alg. 1, refinement loop): LS codebook updates + joint beam re-encode
     _, lb, _, _ = reconstruct_error(Ws, d, Hb, perm, cbs, Gc)
     history = [lb]
     for _ in range(cfg.refine_rounds):

@@ -55,6 +55,7 @@ SIGNATURES = {
     "crvq_profile_end": (C.c_int32, [C.POINTER(crvq_kernel_stat), C.c_int32, c_i32p]),
     "crvq_profile_filter": (C.c_int32, [C.c_char_p]),
     "crvq_launch_count": (C.c_int64, []),
+    "crvq_selftest_bounded_wait": (C.c_int32, [c_vp]),
     "crvq_hessian": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int32, C.c_float, c_vp, c_vp,
                                  c_vp, c_vp, c_vp]),
     "crvq_hessian_blocks": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int32, C.c_float,

@@ -97,6 +97,12 @@ def crvq_sync(stream=None, device=None):
     _check(_L().crvq_sync(_stream(stream, dev)))
 
 
+def crvq_selftest_bounded_wait(stream=None, device=None):
+    """Enqueue the bounded-wait self-test: the next crvq_sync raises CRVQ_ERR_TIMEOUT."""
+    dev = device if device is not None else torch.cuda.current_device()
+    _check(_L().crvq_selftest_bounded_wait(_stream(stream, dev)))
+
+
 def crvq_profile_begin():
     """Start bracketing every library kernel launch with CUDA events."""
     _check(_L().crvq_profile_begin())
@@ -288,7 +294,7 @@ def _cfg_struct(cfg) -> _lib.crvq_config:
 
 
 def crvq_quantize_layer(W, X, cfg, want_W_hat=True, out=None, stream=None, device=None):
-    """Alg. 1 lines 3-17 for one matrix. W, X: torch tensors on the GPU, or pinned/pageable
+    """Alg. 1, prequantization through the refinement loop for one matrix. W, X: torch tensors on the GPU, or pinned/pageable
     CPU tensors (then the library stages them and the outputs are CPU tensors)."""
     M, N = W.shape
     n_tok = X.shape[0]

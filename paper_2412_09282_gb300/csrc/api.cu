@@ -1,5 +1,5 @@
 // C ABI of libcrvq: argument validation, status / error-word handling and the per-matrix
-// schedule (Alg. 1 lines 3-17) that strings the kernels together on one stream.
+// schedule (Alg. 1, prequantization through the refinement loop) that strings the kernels together on one stream.
 #include <atomic>
 #include <cmath>
 #include <cstring>
@@ -11,6 +11,7 @@
 #include "common.cuh"
 #include "kernels.h"
 #include "stats.cuh"
+#include "tc_ops.cuh"
 
 namespace crvq {
 
@@ -208,6 +209,20 @@ static bool is_device_ptr(const void* p) {
   return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
 }
 
+namespace {
+
+// One thread waits on an mbarrier nothing arrives on (crvq_selftest_bounded_wait).
+__global__ void selftest_wait_kernel(unsigned* err) {
+  __shared__ __align__(8) uint64_t bar;
+  if (threadIdx.x == 0) {
+    tc::mbar_init(tc::smem_u32(&bar), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    tc::mbar_wait(tc::smem_u32(&bar), 0u, err);  // gives up after the bound: ERRBIT_TIMEOUT
+  }
+}
+
+}  // namespace
+
 }  // namespace crvq
 
 using namespace crvq;
@@ -302,6 +317,15 @@ crvq_status crvq_profile_end(crvq_kernel_stat* stats, int32_t cap, int32_t* n_st
   for (int i = 0; i < n; ++i) stats[i] = agg[i];
   if (n_stats) *n_stats = n;
   return st;
+}
+
+crvq_status crvq_selftest_bounded_wait(crvq_stream_t stream) {
+  clear_last_error();
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
+  selftest_wait_kernel<<<1, 32, 0, (cudaStream_t)stream>>>(err);
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
 }
 
 crvq_status crvq_sync(crvq_stream_t stream) {
@@ -613,7 +637,7 @@ crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, i
   CRVQ_TRY(launch_transpose(X, n_tok, N, Xt, ldt, s));
   CRVQ_TRY(launch_tc_hessian_blocks(Xt, ldt, n_tok, N, nullptr, false, cfg->damp_rel, xsq,
                                     delta, delta64, Hb0, s));
-  // S2: prequantize in the original order (Alg. 1 line 3)
+  // S2: prequantize in the original order (Alg. 1, prequantization step)
   {
     SetView set{W, N, M, G, Hb0};
     CbList cl{};
@@ -625,12 +649,12 @@ crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, i
     CRVQ_TRY(launch_reconstruct_error(W, M, N, Hb0, nullptr, cl, 0, nullptr, 0, 0.0, nullptr,
                                       Wpre, losses + 3, s));
   }
-  // S3: importance and reordering (Alg. 1 lines 4-5)
+  // S3: importance and reordering (Alg. 1, importance and reordering steps)
   CRVQ_TRY(launch_select_reorder(W, M, N, d, Wpre, xsq, nullptr, cfg->importance_mode,
                                  phase_seed(cfg->seed, 4, 0), o.perm, o.imp, Ws, nullptr, s));
   CRVQ_TRY(launch_tc_hessian_blocks(Xt, ldt, n_tok, N, o.perm, true, 0.f, nullptr, nullptr,
                                     delta64, Hb, s));
-  // S4: base codebook over all vectors (Alg. 1 lines 6-7)
+  // S4: base codebook over all vectors (Alg. 1, base codebook steps)
   CbList all{};
   all.n = 1 + cfg->n_ext;
   all.cb[0] = CbView{o.C_base, o.codes_base, G, G, cfg->K_base};
@@ -646,7 +670,7 @@ crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, i
                                 o.C_base, s));
     CRVQ_TRY(lloyd(full, cl, cfg->kmeans_iters, ex, s));
   }
-  // S5: extended codebooks on the critical residual (Alg. 1 lines 8-13)
+  // S5: extended codebooks on the critical residual (Alg. 1, extended-codebook loop)
   if (cfg->n_ext > 0) {
     const SetView crit{Ws, N, M, Gc, Hb};
     for (int t = 1; t <= cfg->n_ext; ++t) {
@@ -664,7 +688,7 @@ crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, i
       CRVQ_TRY(lloyd(crit, cl, cfg->kmeans_iters, ex, s));
     }
   }
-  // S6: least-squares codebook updates + joint beam re-encode (Alg. 1 lines 14-17)
+  // S6: least-squares codebook updates + joint beam re-encode (Alg. 1, refinement loop)
   CRVQ_TRY(launch_reconstruct_error(Ws, M, N, Hb, o.perm, all, Gc, nullptr, 0, 0.0, nullptr,
                                     nullptr, losses + 6, s));
   double prev = 0.0;
