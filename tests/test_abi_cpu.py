@@ -130,3 +130,65 @@ def test_quantize_layer_rejects_bad_shapes_and_options_before_launch(lib):
     # a NULL required pointer
     assert lib.crvq_quantize_layer(None, dummy, 512, 512, 64, c.byref(cfg()), c.byref(outs),
                                    c.byref(rep), None) == -1
+
+
+_STRUCTS = ["crvq_codebook", "crvq_kernel_stat", "crvq_config", "crvq_layer_outputs",
+            "crvq_layer_report"]
+
+
+def _header_fields(struct):
+    """Field names of `struct` as declared in include/crvq.h (comments removed)."""
+    src = open(os.path.join(ROOT, "include", "crvq.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    body = re.search(r"typedef struct " + struct + r"\s*\{(.*?)\}\s*" + struct + ";", src,
+                     flags=re.S).group(1)
+    return [re.search(r"\**\s*(\w+)\s*(\[\d+\])?$", decl.strip()).group(1)
+            for decl in body.split(";") if decl.strip()]
+
+
+def test_ctypes_structs_match_the_header_layout(tmp_path):
+    """sizeof / offsetof of every struct of the ABI, as gcc lays out include/crvq.h, against the
+    binding's ctypes declarations (field names in the same order)."""
+    import shutil
+    import subprocess
+    from paper_2412_09282_gb300 import _lib
+    if shutil.which("gcc") is None:
+        pytest.skip("gcc not available")
+    lines = ['#include <stddef.h>', '#include <stdio.h>', '#include "crvq.h"', 'int main(void) {']
+    for s in _STRUCTS:
+        lines.append(f'  printf("{s} size %zu\\n", sizeof({s}));')
+        for f in _header_fields(s):
+            lines.append(f'  printf("{s} {f} %zu\\n", offsetof({s}, {f}));')
+    lines += ["  return 0;", "}"]
+    src = tmp_path / "layout.c"
+    src.write_text("\n".join(lines) + "\n")
+    exe = tmp_path / "layout"
+    subprocess.run(["gcc", "-std=c11", "-I", os.path.join(ROOT, "include"), str(src), "-o",
+                    str(exe)], check=True)
+    out = subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout
+    got = {tuple(l.split()[:-1]): int(l.split()[-1]) for l in out.splitlines()}
+    for s in _STRUCTS:
+        cls = getattr(_lib, s)
+        assert [n for n, _ in cls._fields_] == _header_fields(s), s
+        assert ctypes.sizeof(cls) == got[(s, "size")], s
+        for n, _ in cls._fields_:
+            assert getattr(cls, n).offset == got[(s, n)], (s, n)
+
+
+def test_binding_raises_when_the_library_is_missing(tmp_path):
+    """No CPU fallback: with the shared library absent, the first call raises ImportError."""
+    import subprocess
+    import sys
+    code = (
+        "import sys; sys.path.insert(0, %r)\n"
+        "from paper_2412_09282_gb300 import _lib\n"
+        "_lib.LIB_PATH = %r; _lib._lib = None\n"
+        "try:\n"
+        "    _lib.load()\n"
+        "except ImportError as e:\n"
+        "    print('raised', 'no CPU fallback' in str(e))\n"
+        "else:\n"
+        "    print('loaded')\n" % (ROOT, str(tmp_path / "libcrvq.so")))
+    out = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True,
+                         timeout=300)
+    assert out.stdout.strip() == "raised True", out.stdout + out.stderr
