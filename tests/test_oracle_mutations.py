@@ -1,0 +1,244 @@
+"""Planted mistakes in the oracle, on the CPU: each plausible slip (a dropped term or factor,
+a wrong sign, index or scale, an operand left unpermuted, a sampling rule broken) is patched
+into one oracle function for the duration of a test, and at least one of the pins in
+test_oracle_pins.py must then fail. This checks that the pins constrain the oracle rather
+than restate it. CPU only."""
+import importlib.util
+import os
+
+import numpy as np
+import pytest
+
+from oracle import crvq_oracle as O
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_spec = importlib.util.spec_from_file_location("oracle_pins_for_mutation",
+                                               os.path.join(_HERE, "test_oracle_pins.py"))
+pins = importlib.util.module_from_spec(_spec)
+_spec.loader.exec_module(pins)
+
+
+# ------------------------------------------------------------------ the planted mistakes
+def _hessian_without_1_over_n(orig):
+    def f(X, damp_rel, d):
+        H, xsq, Hb, delta = orig(X, damp_rel, d)
+        n = np.asarray(X).shape[0]
+        return ((H * n).astype(np.float32), (xsq * n).astype(np.float32),
+                (Hb * n).astype(np.float32), np.float32(delta * n))
+    return f
+
+
+def _hessian_damping_everywhere(orig):
+    def f(X, damp_rel, d):
+        H, xsq, Hb, delta = orig(X, damp_rel, d)
+        N = H.shape[0]
+        H2 = (H + float(delta) * (np.ones((N, N)) - np.eye(N))).astype(np.float32)
+        Hb2 = np.stack([H2[g * d:(g + 1) * d, g * d:(g + 1) * d] for g in range(N // d)])
+        return H2, xsq, Hb2, delta
+    return f
+
+
+def _hessian_delta_from_sum(orig):
+    def f(X, damp_rel, d):
+        H, xsq, Hb, delta = orig(X, damp_rel, d)
+        N = H.shape[0]
+        extra = float(delta) * (N - 1)
+        return ((H + extra * np.eye(N)).astype(np.float32), xsq,
+                (Hb + extra * np.eye(d)).astype(np.float32), np.float32(delta * N))
+    return f
+
+
+def _encode_plus_instead_of_minus(orig):
+    """err = (t + c)^T H (t + c): the codeword's sign flipped in the residual."""
+    def f(T, d, H_blocks, cbs, n_fixed, B, keep_if_better=False, **kw):
+        neg = [O.Codebook(-np.asarray(cb.C), cb.codes, cb.G_cov) for cb in cbs]
+        return orig(T, d, H_blocks, neg, n_fixed, B, keep_if_better, **kw)
+    return f
+
+
+def _encode_ignores_H(orig):
+    def f(T, d, H_blocks, cbs, n_fixed, B, keep_if_better=False, **kw):
+        eye = np.broadcast_to(np.eye(d, dtype=np.float32), np.shape(H_blocks)).copy()
+        return orig(T, d, eye, cbs, n_fixed, B, keep_if_better, **kw)
+    return f
+
+
+def _encode_ignores_fixed(orig):
+    """The fixed codebooks' codewords are not subtracted from the target."""
+    def f(T, d, H_blocks, cbs, n_fixed, B, keep_if_better=False, **kw):
+        if n_fixed == 0:
+            return orig(T, d, H_blocks, cbs, n_fixed, B, keep_if_better, **kw)
+        free = [O.Codebook(cb.C, None if not keep_if_better else cb.codes, cb.G_cov)
+                for cb in cbs[n_fixed:]]
+        codes, verr = orig(T, d, H_blocks, free, 0, B, keep_if_better, **kw)
+        return [cb.codes for cb in cbs[:n_fixed]] + list(codes), verr
+    return f
+
+
+def _update_ignores_H(orig):
+    def f(T, d, H_blocks, cbs, which):
+        eye = np.broadcast_to(np.eye(d, dtype=np.float32), np.shape(H_blocks)).copy()
+        return orig(T, d, eye, cbs, which)
+    return f
+
+
+def _update_zeroes_empty_clusters(orig):
+    def f(T, d, H_blocks, cbs, which):
+        C, counts = orig(T, d, H_blocks, cbs, which)
+        C = np.array(C, copy=True)
+        C[np.asarray(counts) == 0] = 0
+        return C, counts
+    return f
+
+
+def _update_residual_sign(orig):
+    """The other codebooks' codewords are added to the target instead of subtracted."""
+    def f(T, d, H_blocks, cbs, which):
+        flipped = [cb if s == which else O.Codebook(-np.asarray(cb.C), cb.codes, cb.G_cov)
+                   for s, cb in enumerate(cbs)]
+        return orig(T, d, H_blocks, flipped, which)
+    return f
+
+
+def _importance_without_half(orig):
+    def f(W, W_pre, xsq, mode, seed):
+        return orig(W, W_pre, xsq, mode, seed) * 2.0
+    return f
+
+
+def _importance_mean_over_rows(orig):
+    """Mean over the output rows instead of the maximum."""
+    def f(W, W_pre, xsq, mode, seed):
+        if mode != O.MODE_WA:
+            return orig(W, W_pre, xsq, mode, seed)
+        dW = np.asarray(W, np.float64) - np.asarray(W_pre, np.float64)
+        return 0.5 * np.asarray(xsq, np.float64) * (dW ** 2).mean(axis=0)
+    return f
+
+
+def _reorder_ascending(orig):
+    def f(W, d, W_pre, xsq, H, crit_frac, mode, seed):
+        perm, I, Ws, Hb, Gc = orig(W, d, W_pre, xsq, H, crit_frac, mode, seed)
+        p = np.ascontiguousarray(perm[::-1])
+        Hp = np.asarray(H)[np.ix_(p, p)]
+        Hb2 = np.stack([Hp[g * d:(g + 1) * d, g * d:(g + 1) * d] for g in range(len(p) // d)])
+        return p, I, np.asarray(W)[:, p], Hb2, Gc
+    return f
+
+
+def _reorder_blocks_unpermuted(orig):
+    def f(W, d, W_pre, xsq, H, crit_frac, mode, seed):
+        perm, I, Ws, Hb, Gc = orig(W, d, W_pre, xsq, H, crit_frac, mode, seed)
+        H = np.asarray(H)
+        Hb2 = np.stack([H[g * d:(g + 1) * d, g * d:(g + 1) * d] for g in range(len(perm) // d)])
+        return perm, I, Ws, Hb2, Gc
+    return f
+
+
+def _loss_full_block_only(orig):
+    def f(W_sorted, d, H_blocks, perm, cbs, G_c, X=None, delta=0.0):
+        W_hat, lb, lc, lf = orig(W_sorted, d, H_blocks, perm, cbs, G_c, X, delta)
+        return W_hat, lb, lc, (lb if lf is not None else lf)
+    return f
+
+
+def _loss_full_without_damping(orig):
+    def f(W_sorted, d, H_blocks, perm, cbs, G_c, X=None, delta=0.0):
+        return orig(W_sorted, d, H_blocks, perm, cbs, G_c, X, 0.0)
+    return f
+
+
+def _sample_indices_not_stratified(orig):
+    def f(n, K, seed):
+        return np.sort(np.random.default_rng(seed).choice(n, K, replace=False))
+    return f
+
+
+def _init_residual_sign(orig):
+    def f(T, d, G_sub, K, seed, fixed=()):
+        flipped = [O.Codebook(-np.asarray(cb.C), cb.codes, cb.G_cov) for cb in fixed]
+        return orig(T, d, G_sub, K, seed, fixed=flipped)
+    return f
+
+
+def _avg_bits_without_extended(orig):
+    def f(e, d, m, lam, M=4096, N=4096, include_perm=False):
+        return orig(e, d, 1, lam, M, N, include_perm)
+    return f
+
+
+def _crit_groups_floor(orig):
+    def f(N, d, crit_frac):
+        return min(N // d, int(np.floor(np.float32(crit_frac) * N / d)))
+    return f
+
+
+def _splitmix64_wrong_constant(orig):
+    def f(stream, counter):
+        return orig(stream, counter) ^ 1
+    return f
+
+
+# (name, oracle attribute, planted version, pins that must catch it)
+MUTATIONS = [
+    ("hessian: 1/n dropped", "hessian", _hessian_without_1_over_n,
+     ["test_hessian_closed_form_scaled_identity", "test_hessian_matches_matrix_free_product"]),
+    ("hessian: damping on every entry", "hessian", _hessian_damping_everywhere,
+     ["test_hessian_closed_form_scaled_identity", "test_hessian_matches_matrix_free_product"]),
+    ("hessian: delta from the sum, not the mean", "hessian", _hessian_delta_from_sum,
+     ["test_hessian_closed_form_scaled_identity", "test_hessian_matches_matrix_free_product"]),
+    ("encode: t + c instead of t - c", "encode_beam", _encode_plus_instead_of_minus,
+     ["test_encode_isotropic_is_euclidean_nearest_codeword",
+      "test_encode_general_H_equals_whitened_nearest_codeword"]),
+    ("encode: H ignored", "encode_beam", _encode_ignores_H,
+     ["test_encode_isotropic_is_euclidean_nearest_codeword",
+      "test_encode_general_H_equals_whitened_nearest_codeword"]),
+    ("encode: fixed codebooks not subtracted", "encode_beam", _encode_ignores_fixed,
+     ["test_encode_with_fixed_codebook_equals_encode_of_residual"]),
+    ("update: H ignored (plain cluster mean)", "update_codebook", _update_ignores_H,
+     ["test_update_is_a_minimiser_and_single_member_is_exact"]),
+    ("update: empty clusters zeroed", "update_codebook", _update_zeroes_empty_clusters,
+     ["test_update_isotropic_is_cluster_mean"]),
+    ("update: residual with the wrong sign", "update_codebook", _update_residual_sign,
+     ["test_update_of_second_codebook_targets_residual"]),
+    ("importance: factor 1/2 dropped", "importance", _importance_without_half,
+     ["test_importance_wa_equals_literal_app_a2_sum"]),
+    ("importance: mean over rows instead of max", "importance", _importance_mean_over_rows,
+     ["test_importance_wa_equals_literal_app_a2_sum"]),
+    ("reorder: ascending importance", "select_reorder_channels", _reorder_ascending,
+     ["test_reorder_bijection_roundtrip_and_blocks"]),
+    ("reorder: H blocks taken unpermuted", "select_reorder_channels",
+     _reorder_blocks_unpermuted, ["test_reorder_bijection_roundtrip_and_blocks"]),
+    ("losses: loss_full without cross-group terms", "reconstruct_error", _loss_full_block_only,
+     ["test_loss_full_two_routes_and_block_loss_matches_encode"]),
+    ("losses: damping left out of the X route", "reconstruct_error",
+     _loss_full_without_damping, ["test_loss_full_two_routes_and_block_loss_matches_encode"]),
+    ("init: indices not stratified", "kmeans_sample_indices", _sample_indices_not_stratified,
+     ["test_kmeans_init_strata_distinct_deterministic"]),
+    ("init: residual with the wrong sign", "kmeans_init", _init_residual_sign,
+     ["test_kmeans_init_takes_sampled_vectors_and_residuals"]),
+    ("bit-width: extended codebooks dropped", "avg_bits", _avg_bits_without_extended,
+     ["test_avg_bits_paper_values"]),
+    ("critical groups: floor instead of ceiling", "n_crit_groups", _crit_groups_floor,
+     ["test_n_crit_groups_closed_form"]),
+    ("splitmix64: wrong output", "splitmix64", _splitmix64_wrong_constant,
+     ["test_splitmix64_published_sequence"]),
+]
+
+
+def test_every_pin_named_here_passes_on_the_unmodified_oracle():
+    for name in sorted({p for *_, ps in MUTATIONS for p in ps}):
+        getattr(pins, name)()
+
+
+@pytest.mark.parametrize("label,attr,plant,pin_names", MUTATIONS,
+                         ids=[m[0] for m in MUTATIONS])
+def test_planted_mistake_fails_a_pin(monkeypatch, label, attr, plant, pin_names):
+    monkeypatch.setattr(O, attr, plant(getattr(O, attr)))
+    caught = []
+    for name in pin_names:
+        try:
+            getattr(pins, name)()
+        except AssertionError:  # a pin's own check, not an error of the planted code
+            caught.append(name)
+    assert caught, f"no pin caught the planted mistake: {label}"
