@@ -179,7 +179,33 @@ def _splitmix64_wrong_constant(orig):
     return f
 
 
-# (name, oracle attribute, planted version, pins that must catch it)
+def _beam_width_ignored(orig):
+    def f(T, d, H_blocks, cbs, n_fixed, B, keep_if_better=False, **kw):
+        return orig(T, d, H_blocks, cbs, n_fixed, 1, keep_if_better, **kw)
+    return f
+
+
+def _keep_if_better_ignored(orig):
+    def f(T, d, H_blocks, cbs, n_fixed, B, keep_if_better=False, **kw):
+        if keep_if_better:
+            cbs = [cb if s < n_fixed else O.Codebook(cb.C, None, cb.G_cov)
+                   for s, cb in enumerate(cbs)]
+        return orig(T, d, H_blocks, cbs, n_fixed, B, False, **kw)
+    return f
+
+
+def _reconstruction_forward_perm(orig):
+    """The sorted reconstruction is scattered back with perm instead of its inverse."""
+    def f(W_sorted, d, H_blocks, perm, cbs, G_c, X=None, delta=0.0):
+        W_hat, lb, lc, lf = orig(W_sorted, d, H_blocks, perm, cbs, G_c, X, delta)
+        if perm is not None:
+            W_hat = np.asarray(W_hat)[:, perm][:, perm]
+        return W_hat, lb, lc, lf
+    return f
+
+
+# (name, oracle attribute, planted version, pins that must catch it: a test name, or a test
+# name with its arguments)
 MUTATIONS = [
     ("hessian: 1/n dropped", "hessian", _hessian_without_1_over_n,
      ["test_hessian_closed_form_scaled_identity", "test_hessian_matches_matrix_free_product"]),
@@ -223,12 +249,24 @@ MUTATIONS = [
      ["test_n_crit_groups_closed_form"]),
     ("splitmix64: wrong output", "splitmix64", _splitmix64_wrong_constant,
      ["test_splitmix64_published_sequence"]),
+    ("beam: width ignored", "encode_beam", _beam_width_ignored,
+     [("test_beam_with_full_width_equals_exhaustive_search", (4, 2, 4)),
+      ("test_beam_with_full_width_equals_exhaustive_search", (4, 3, 2))]),
+    ("beam: keep-if-better ignored", "encode_beam", _keep_if_better_ignored,
+     ["test_narrow_beam_never_beats_exhaustive_and_keep_if_better_keeps_optimum"]),
+    ("losses: reconstruction scattered with perm, not its inverse", "reconstruct_error",
+     _reconstruction_forward_perm, ["test_loss_full_two_routes_and_block_loss_matches_encode"]),
 ]
 
 
+def _run_pin(spec):
+    name, args = (spec, ()) if isinstance(spec, str) else spec
+    getattr(pins, name)(*args)
+
+
 def test_every_pin_named_here_passes_on_the_unmodified_oracle():
-    for name in sorted({p for *_, ps in MUTATIONS for p in ps}):
-        getattr(pins, name)()
+    for spec in sorted({p for *_, ps in MUTATIONS for p in ps}, key=str):
+        _run_pin(spec)
 
 
 @pytest.mark.parametrize("label,attr,plant,pin_names", MUTATIONS,
@@ -236,9 +274,9 @@ def test_every_pin_named_here_passes_on_the_unmodified_oracle():
 def test_planted_mistake_fails_a_pin(monkeypatch, label, attr, plant, pin_names):
     monkeypatch.setattr(O, attr, plant(getattr(O, attr)))
     caught = []
-    for name in pin_names:
+    for spec in pin_names:
         try:
-            getattr(pins, name)()
+            _run_pin(spec)
         except AssertionError:  # a pin's own check, not an error of the planted code
-            caught.append(name)
+            caught.append(spec)
     assert caught, f"no pin caught the planted mistake: {label}"
