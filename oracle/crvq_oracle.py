@@ -28,7 +28,10 @@ Readings where the paper is silent or ambiguous (all listed in the design notes)
   * Importance uses the App. A.2 form I_i = max_j 1/2 sum_k (x_ik dw_ji)^2
     = 1/2 * xsq_i * max_j dw_ji^2 (with xsq the mean of squares, a constant factor 1/n);
     Eq. (wa) in Sec. 4.1 divides by an inverse-Hessian diagonal instead, which the App. A.2
-    expansion does not reproduce; the App. A.2 form is the one used here.
+    expansion does not reproduce; the App. A.2 form is the default. Eq. (wa) as printed is
+    the mode MODE_WA_INV, with the inverse taken of the damped proxy H (the undamped X^T X is
+    singular whenever there are fewer tokens than channels; the factor 1/n scales every I_i
+    alike and leaves the order unchanged).
   * Damping: H = X^T X / n + delta I, delta = damp_rel * mean_i xsq_i (the paper has none;
     it keeps the LS codebook solves well posed).
   * k-means init: one vector drawn from each of K equal strata of the vector index range,
@@ -44,8 +47,8 @@ import math
 
 import numpy as np
 
-# Importance modes (Sec. 4.1 and Sec. 6.3 / Table 2).
-MODE_WA, MODE_WONLY, MODE_RANDOM = 0, 1, 2
+# Importance modes (Sec. 4.1 and Sec. 6.3 / Table 2); MODE_WA_INV is Eq. (wa) as printed.
+MODE_WA, MODE_WONLY, MODE_RANDOM, MODE_WA_INV = 0, 1, 2, 3
 
 _GAMMA = 0x9E3779B97F4A7C15
 _MASK = 0xFFFFFFFFFFFFFFFF
@@ -106,17 +109,32 @@ def n_crit_groups(N, d, crit_frac):
     return min(N // d, int(math.ceil(lam * N / d - 1e-12))) if lam > 0 else 0
 
 
-def importance(W, W_pre, xsq, mode, seed):
+def hinv_diag(H):
+    """diag(H^-1) of a symmetric positive definite H (fp64): with the Cholesky factor
+    H = L L^T, H^-1 = L^-T L^-1, so [H^-1]_ii = sum_k (L^-1)_ki^2 (the denominator of Eq. (wa),
+    Sec. 4.1)."""
+    import scipy.linalg
+    H = np.asarray(H, dtype=np.float64)
+    L = np.linalg.cholesky(H)
+    Linv = scipy.linalg.solve_triangular(L, np.eye(H.shape[0]), lower=True)
+    return np.sum(Linv * Linv, axis=0)
+
+
+def importance(W, W_pre, xsq, mode, seed, hinv=None):
     """Per-channel importance I (fp64).
 
     W-A  (App. A.2): I_i = max_j 1/2 * xsq_i * (w_ji - VQ(w_ji))^2.
     W-only (Sec. 4.1): I_i = max_j w_ji^2.
-    random (Table 2): I_i = a 24-bit uniform from SplitMix64(seed, i)."""
+    random (Table 2): I_i = a 24-bit uniform from SplitMix64(seed, i).
+    W-A inverse (Eq. (wa)): I_i = max_j (w_ji - VQ(w_ji))^2 / (2 [H^-1]_ii), hinv = diag(H^-1)."""
     W = np.asarray(W, dtype=np.float64)
     M, N = W.shape
     if mode == MODE_WA:
         dW = W - np.asarray(W_pre, dtype=np.float64)
         return 0.5 * np.asarray(xsq, np.float64) * np.max(dW * dW, axis=0)
+    if mode == MODE_WA_INV:
+        dW = W - np.asarray(W_pre, dtype=np.float64)
+        return np.max(dW * dW, axis=0) / (2.0 * np.asarray(hinv, np.float64))
     if mode == MODE_WONLY:
         return np.max(W * W, axis=0)
     if mode == MODE_RANDOM:
@@ -132,7 +150,8 @@ def select_reorder_channels(W, d, W_pre, xsq, H, crit_frac, mode, seed):
     Returns (perm int32, importance fp32, W_sorted fp32, H_blocks fp32, n_crit_groups)."""
     W = np.asarray(W, dtype=np.float32)
     M, N = W.shape
-    I = importance(W, W_pre, xsq, mode, seed)
+    hinv = hinv_diag(H) if mode == MODE_WA_INV else None
+    I = importance(W, W_pre, xsq, mode, seed, hinv)
     perm = np.lexsort((np.arange(N), -I)).astype(np.int32)
     Ws = W[:, perm]
     H = np.asarray(H, dtype=np.float32)

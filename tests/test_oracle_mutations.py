@@ -101,16 +101,16 @@ def _update_residual_sign(orig):
 
 
 def _importance_without_half(orig):
-    def f(W, W_pre, xsq, mode, seed):
-        return orig(W, W_pre, xsq, mode, seed) * 2.0
+    def f(W, W_pre, xsq, mode, seed, hinv=None):
+        return orig(W, W_pre, xsq, mode, seed, hinv) * 2.0
     return f
 
 
 def _importance_mean_over_rows(orig):
     """Mean over the output rows instead of the maximum."""
-    def f(W, W_pre, xsq, mode, seed):
+    def f(W, W_pre, xsq, mode, seed, hinv=None):
         if mode != O.MODE_WA:
-            return orig(W, W_pre, xsq, mode, seed)
+            return orig(W, W_pre, xsq, mode, seed, hinv)
         dW = np.asarray(W, np.float64) - np.asarray(W_pre, np.float64)
         return 0.5 * np.asarray(xsq, np.float64) * (dW ** 2).mean(axis=0)
     return f
@@ -176,6 +176,30 @@ def _crit_groups_floor(orig):
 def _splitmix64_wrong_constant(orig):
     def f(stream, counter):
         return orig(stream, counter) ^ 1
+    return f
+
+
+def _hinv_is_diag_of_H(orig):
+    """The inverse forgotten: diag(H) instead of diag(H^-1)."""
+    def f(H):
+        return np.diag(np.asarray(H, np.float64)).copy()
+    return f
+
+
+def _hinv_ignores_correlations(orig):
+    """1 / H_ii: the inverse of the diagonal, not the diagonal of the inverse."""
+    def f(H):
+        return 1.0 / np.diag(np.asarray(H, np.float64))
+    return f
+
+
+def _eq_wa_multiplies(orig):
+    """Eq. (wa) with the inverse-Hessian diagonal in the numerator."""
+    def f(W, W_pre, xsq, mode, seed, hinv=None):
+        if mode != O.MODE_WA_INV:
+            return orig(W, W_pre, xsq, mode, seed, hinv)
+        dW = np.asarray(W, np.float64) - np.asarray(W_pre, np.float64)
+        return np.max(dW * dW, axis=0) * np.asarray(hinv, np.float64) / 2.0
     return f
 
 
@@ -256,6 +280,12 @@ MUTATIONS = [
      ["test_narrow_beam_never_beats_exhaustive_and_keep_if_better_keeps_optimum"]),
     ("losses: reconstruction scattered with perm, not its inverse", "reconstruct_error",
      _reconstruction_forward_perm, ["test_loss_full_two_routes_and_block_loss_matches_encode"]),
+    ("Eq. (wa): diag(H) for diag(H^-1)", "hinv_diag", _hinv_is_diag_of_H,
+     ["test_hinv_diag_closed_forms", "test_hinv_diag_equals_schur_complement"]),
+    ("Eq. (wa): 1 / H_ii for [H^-1]_ii", "hinv_diag", _hinv_ignores_correlations,
+     ["test_hinv_diag_closed_forms", "test_hinv_diag_equals_schur_complement"]),
+    ("Eq. (wa): inverse diagonal multiplied, not divided", "importance", _eq_wa_multiplies,
+     ["test_importance_eq_wa_is_app_a2_for_uncorrelated_channels"]),
 ]
 
 

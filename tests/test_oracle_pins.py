@@ -290,6 +290,64 @@ def test_importance_wa_equals_literal_app_a2_sum():
                                (W.astype(np.float64) ** 2).max(0))
 
 
+def test_hinv_diag_closed_forms():
+    """diag(H^-1) of Eq. (wa): a diagonal H, 2 x 2 blocks, and delta I + u u^T
+    (Sherman-Morrison: [H^-1]_ii = 1/delta - u_i^2 / (delta (delta + |u|^2)))."""
+    h = np.array([0.5, 2.0, 4.0, 1.25])
+    np.testing.assert_allclose(O.hinv_diag(np.diag(h)), 1.0 / h, rtol=1e-14)
+    a, b, c = 3.0, -1.2, 2.0
+    H = np.kron(np.eye(3), np.array([[a, b], [b, c]]))
+    det = a * c - b * b
+    np.testing.assert_allclose(O.hinv_diag(H), np.tile([c / det, a / det], 3), rtol=1e-13)
+    rng = np.random.default_rng(21)
+    u, delta = rng.standard_normal(9), 0.3
+    exp = 1.0 / delta - u * u / (delta * (delta + u @ u))
+    np.testing.assert_allclose(O.hinv_diag(delta * np.eye(9) + np.outer(u, u)), exp, rtol=1e-12)
+
+
+def test_hinv_diag_equals_schur_complement():
+    """OBS identity: 1 / [H^-1]_ii = H_ii - H_i,r H_r,r^-1 H_r,i (r = every other index), the
+    least value of z^T H z over z with z_i = 1; computed by a linear solve on the rest."""
+    rng = np.random.default_rng(22)
+    N = 12
+    X = rng.standard_normal((30, N)) * rng.uniform(0.2, 3.0, N)
+    H = X.T @ X / 30 + 0.01 * np.eye(N)
+    got = O.hinv_diag(H)
+    for i in range(N):
+        r = [j for j in range(N) if j != i]
+        s = H[i, i] - H[i, r] @ np.linalg.solve(H[np.ix_(r, r)], H[r, i])
+        assert abs(1.0 / got[i] - s) <= 1e-10 * s
+        z = np.zeros(N)
+        z[i] = 1.0
+        z[r] = -np.linalg.solve(H[np.ix_(r, r)], H[r, i])
+        assert abs(z @ H @ z - s) <= 1e-10 * s
+
+
+def test_importance_eq_wa_is_app_a2_for_uncorrelated_channels():
+    """Eq. (wa) with a diagonal X^T X (orthogonal channels, no damping) is the App. A.2 form:
+    1 / [H^-1]_ii = H_ii = xsq_i. With correlated channels the two differ."""
+    rng = np.random.default_rng(23)
+    n, M, N = 24, 6, 16
+    Q, _ = np.linalg.qr(rng.standard_normal((n, N)))
+    X = (Q * rng.uniform(0.5, 4.0, N)).astype(np.float32)
+    W = rng.standard_normal((M, N)).astype(np.float32)
+    Wq = (W + 0.1 * rng.standard_normal((M, N))).astype(np.float32)
+    H, xsq, _, _ = O.hessian(X, 0.0, 8)
+    I_inv = O.importance(W, Wq, xsq, O.MODE_WA_INV, 0, O.hinv_diag(H))
+    I_a2 = O.importance(W, Wq, xsq, O.MODE_WA, 0)
+    np.testing.assert_allclose(I_inv, I_a2, rtol=1e-4)
+    dW = W.astype(np.float64) - Wq
+    lit = np.array([max(dW[j, i] ** 2 for j in range(M)) / (2.0 * np.linalg.inv(
+        H.astype(np.float64))[i, i]) for i in range(N)])
+    np.testing.assert_allclose(I_inv, lit, rtol=1e-5)
+    Xc = X + 0.5 * X[:, :1]                          # channel 0 mixed into every channel
+    Hc, xc, _, _ = O.hessian(Xc, 0.0, 8)
+    assert not np.allclose(O.importance(W, Wq, xc, O.MODE_WA_INV, 0, O.hinv_diag(Hc)),
+                           O.importance(W, Wq, xc, O.MODE_WA, 0), rtol=1e-2)
+    perm = O.select_reorder_channels(W, 8, Wq, xsq, H, 0.25, O.MODE_WA_INV, 0)[0]
+    np.testing.assert_array_equal(perm, np.lexsort((np.arange(N), -I_inv)))
+
+
 def test_reorder_bijection_roundtrip_and_blocks():
     rng = np.random.default_rng(13)
     M, N, d = 7, 32, 8
