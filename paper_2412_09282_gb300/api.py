@@ -294,8 +294,9 @@ def _cfg_struct(cfg) -> _lib.crvq_config:
 
 
 def crvq_quantize_layer(W, X, cfg, want_W_hat=True, out=None, stream=None, device=None):
-    """Alg. 1, prequantization through the refinement loop for one matrix. W, X: torch tensors on the GPU, or pinned/pageable
-    CPU tensors (then the library stages them and the outputs are CPU tensors)."""
+    """Alg. 1, prequantization through the refinement loop, for one matrix. W, X: torch
+    tensors on the GPU, or pinned/pageable CPU tensors (then the library stages them and the
+    outputs are CPU tensors)."""
     M, N = W.shape
     n_tok = X.shape[0]
     d = cfg.d
