@@ -203,7 +203,8 @@ crvq_status crvq_kmeans_init(const float* T, int64_t ldT, int64_t M, int64_t G_s
  *   keep_if_better  nonzero: the searched codes hold a tuple on entry, which is kept when
  *                   its err is strictly smaller than the beam's best.
  *   vec_err         [M x G_sub] out or NULL: err of the written tuple (fp64, rounded).
- * Requires 1 <= B <= 16, 0 <= n_fixed < n_cb <= 8.
+ * Requires 1 <= B <= 16, 0 <= n_fixed < n_cb <= 8. Sets of more than 65535 groups return
+ * CRVQ_ERR_UNSUPPORTED (a beam stage launches one grid row per group).
  */
 crvq_status crvq_encode_beam(const float* T, int64_t ldT, int64_t M, int64_t G_sub, int32_t d,
                              const float* H_blocks, const crvq_codebook* cbs, int32_t n_cb,

@@ -442,6 +442,9 @@ crvq_status crvq_encode_beam(const float* T, int64_t ldT, int64_t M, int64_t G_s
   clear_last_error();
   CRVQ_TRY(check_d(d));
   CRVQ_TRY(check_set(T, ldT, M, G_sub, H_blocks));
+  if (G_sub > 65535)  // beam stages launch one grid row (gridDim.y) per group
+    return fail(CRVQ_ERR_UNSUPPORTED, "vector sets of more than 65535 groups are not implemented "
+                "(got %lld)", (long long)G_sub);
   CRVQ_CHECK_ARG(n_cb >= 1 && n_cb <= kMaxCodebooks, "n_cb must be in [1, %d]", kMaxCodebooks);
   CRVQ_CHECK_ARG(n_fixed >= 0 && n_fixed < n_cb, "n_fixed must be in [0, n_cb)");
   CRVQ_CHECK_ARG(B >= 1, "B must be >= 1");

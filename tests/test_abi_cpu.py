@@ -78,6 +78,13 @@ def test_validation_rejects_before_launch(lib):
     assert lib.crvq_encode_beam(dummy, 16, 2, 2, 8, dummy, cb, 1, 1, 1, 0, None, None) == -1
     # ldT too small for the set
     assert lib.crvq_encode_beam(dummy, 8, 2, 2, 8, dummy, cb, 1, 0, 1, 0, None, None) == -1
+    # more groups than a grid row per group allows
+    big = 65536
+    cb[0] = _lib.crvq_codebook(16, 4, 0, 32, big, big)
+    assert lib.crvq_encode_beam(dummy, 8 * big, 1, big, 8, dummy, cb, 1, 0, 2, 0, None,
+                                None) == -2
+    assert b"65535 groups" in lib.crvq_last_error()
+    cb[0] = _lib.crvq_codebook(16, 4, 0, 32, 2, 2)
     # codebook coverage beyond the set
     cb[0] = _lib.crvq_codebook(16, 4, 0, 32, 4, 3)
     assert lib.crvq_update_codebook(dummy, 16, 2, 2, 8, dummy, cb, 1, 0, dummy, None,
