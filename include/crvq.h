@@ -11,7 +11,10 @@
  *
  * Conventions (every call):
  *  - Arrays are device pointers owned by the caller unless a parameter says "host". The
- *    library keeps no pointer after the call returns. Row-major; fp32 unless stated.
+ *    library keeps no pointer after the call returns. Row-major; fp32 unless stated. The
+ *    step calls (crvq_hessian ... crvq_reconstruct_error, but not the no-allocation update)
+ *    check that each device array is device or managed memory and return
+ *    CRVQ_ERR_INVALID_ARG for a host pointer; crvq_quantize_layer accepts either.
  *  - Calls enqueue work on `stream` and return without waiting, except calls that return a
  *    value in host memory (their documentation says so): those synchronize `stream`.
  *  - Scratch memory is taken with stream-ordered cudaMallocAsync/cudaFreeAsync on `stream`.

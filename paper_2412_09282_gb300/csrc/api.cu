@@ -3,9 +3,11 @@
 #include <atomic>
 #include <cmath>
 #include <cstring>
+#include <initializer_list>
 #include <mutex>
 #include <type_traits>
 #include <string>
+#include <utility>
 #include <vector>
 
 #include "common.cuh"
@@ -209,6 +211,25 @@ static bool is_device_ptr(const void* p) {
   return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
 }
 
+// The kernels dereference these pointers: each non-null one must be device (or managed)
+// memory. A host pointer is refused here instead of reaching a kernel.
+static crvq_status check_dev(std::initializer_list<std::pair<const void*, const char*>> ps) {
+  for (const auto& p : ps)
+    if (p.first && !is_device_ptr(p.first))
+      return fail(CRVQ_ERR_INVALID_ARG, "%s is not device memory", p.second);
+  return CRVQ_OK;
+}
+
+static crvq_status check_dev_cbs(const crvq_codebook* cbs, int32_t n) {
+  for (int32_t s = 0; s < n; ++s) {
+    if (!is_device_ptr(cbs[s].C))
+      return fail(CRVQ_ERR_INVALID_ARG, "codebook %d: C is not device memory", s);
+    if (cbs[s].codes && !is_device_ptr(cbs[s].codes))
+      return fail(CRVQ_ERR_INVALID_ARG, "codebook %d: codes is not device memory", s);
+  }
+  return CRVQ_OK;
+}
+
 namespace {
 
 // One thread waits on an mbarrier nothing arrives on (crvq_selftest_bounded_wait).
@@ -352,6 +373,8 @@ crvq_status crvq_hessian(const float* X, int64_t n_tok, int64_t N, int32_t d, fl
   CRVQ_CHECK_ARG(n_tok >= 1 && N >= 1 && N % d == 0, "need n_tok >= 1, N >= 1, N %% d == 0");
   CRVQ_CHECK_ARG(std::isfinite(damp_rel) && damp_rel >= 0.f, "damp_rel must be finite, >= 0");
   CRVQ_CHECK_ARG(aligned16(X), "X must be 16-byte aligned");
+  CRVQ_TRY(check_dev({{X, "X"}, {H, "H"}, {xsq, "xsq"}, {H_blocks, "H_blocks"},
+                      {delta, "delta"}}));
   return launch_hessian(X, n_tok, N, d, damp_rel, H, xsq, H_blocks, delta,
                         (cudaStream_t)stream);
 }
@@ -366,6 +389,8 @@ crvq_status crvq_hessian_blocks(const float* X, int64_t n_tok, int64_t N, int32_
   CRVQ_CHECK_ARG(N <= INT32_MAX, "N must fit in int32");
   CRVQ_CHECK_ARG(std::isfinite(damp_rel) && damp_rel >= 0.f, "damp_rel must be finite, >= 0");
   CRVQ_CHECK_ARG(aligned16(X), "X must be 16-byte aligned");
+  CRVQ_TRY(check_dev({{X, "X"}, {perm, "perm"}, {xsq, "xsq"}, {delta, "delta"},
+                      {H_blocks, "H_blocks"}}));
   cudaStream_t s = (cudaStream_t)stream;
   const int64_t ldt = (n_tok + 3) / 4 * 4;
   Scratch mXt, md64, mxsq, mHb;
@@ -414,6 +439,9 @@ crvq_status crvq_select_reorder_channels(const float* W, int64_t M, int64_t N, i
   if (mode == CRVQ_IMPORTANCE_WA) CRVQ_CHECK_ARG(W_pre && xsq, "W-A mode needs W_pre and xsq");
   CRVQ_CHECK_ARG(aligned16(W) && aligned16(W_sorted) && (!W_pre || aligned16(W_pre)),
                  "W, W_pre and W_sorted must be 16-byte aligned");
+  CRVQ_TRY(check_dev({{W, "W"}, {W_pre, "W_pre"}, {xsq, "xsq"}, {H, "H"}, {perm, "perm"},
+                      {importance, "importance"}, {W_sorted, "W_sorted"},
+                      {H_blocks, "H_blocks"}}));
   if (n_crit_groups) *n_crit_groups = crvq_n_crit_groups(N, d, crit_frac);
   return launch_select_reorder(W, M, N, d, W_pre, xsq, H, mode, seed, perm, importance,
                                W_sorted, H_blocks, (cudaStream_t)stream);
@@ -431,6 +459,8 @@ crvq_status crvq_kmeans_init(const float* T, int64_t ldT, int64_t M, int64_t G_s
                  "K must be in [1, min(65536, M * G_sub)]");
   CbList fl;
   CRVQ_TRY(make_cblist(fixed, n_fixed, G_sub, true, &fl));
+  CRVQ_TRY(check_dev({{T, "T"}, {C_out, "C_out"}}));
+  CRVQ_TRY(check_dev_cbs(fixed, n_fixed));
   SetView set{T, ldT, M, G_sub, nullptr};
   return launch_kmeans_init(set, fl, K, seed, C_out, (cudaStream_t)stream);
 }
@@ -451,6 +481,8 @@ crvq_status crvq_encode_beam(const float* T, int64_t ldT, int64_t M, int64_t G_s
   if (B > 16) return fail(CRVQ_ERR_UNSUPPORTED, "beam width B > 16 is not implemented");
   CbList cl;
   CRVQ_TRY(make_cblist(cbs, n_cb, G_sub, true, &cl));
+  CRVQ_TRY(check_dev({{T, "T"}, {H_blocks, "H_blocks"}, {vec_err, "vec_err"}}));
+  CRVQ_TRY(check_dev_cbs(cbs, n_cb));
   SetView set{T, ldT, M, G_sub, H_blocks};
   return launch_encode_beam(set, cl, n_fixed, B, keep_if_better != 0, vec_err, EncodeExtras{},
                             (cudaStream_t)stream);
@@ -467,6 +499,8 @@ crvq_status crvq_update_codebook(const float* T, int64_t ldT, int64_t M, int64_t
   CRVQ_CHECK_ARG(C_out != nullptr, "C_out is NULL");
   CbList cl;
   CRVQ_TRY(make_cblist(cbs, n_cb, G_sub, true, &cl));
+  CRVQ_TRY(check_dev({{T, "T"}, {H_blocks, "H_blocks"}, {C_out, "C_out"}, {counts, "counts"}}));
+  CRVQ_TRY(check_dev_cbs(cbs, n_cb));
   SetView set{T, ldT, M, G_sub, H_blocks};
   return launch_update_codebook(set, cl, which, C_out, counts, (cudaStream_t)stream);
 }
@@ -488,6 +522,9 @@ crvq_status crvq_reconstruct_error(const float* W_sorted, int64_t M, int64_t N, 
   CRVQ_CHECK_ARG(!W_hat || aligned16(W_hat), "W_hat must be 16-byte aligned");
   CbList cl;
   CRVQ_TRY(make_cblist(cbs, n_cb, N / d, true, &cl));
+  CRVQ_TRY(check_dev({{W_sorted, "W_sorted"}, {H_blocks, "H_blocks"}, {perm, "perm"},
+                      {X, "X"}, {W_hat, "W_hat"}}));
+  CRVQ_TRY(check_dev_cbs(cbs, n_cb));
   cudaStream_t s = (cudaStream_t)stream;
   Scratch mem;
   CRVQ_TRY(mem.alloc(3 * sizeof(double), s));

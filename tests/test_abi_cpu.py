@@ -100,6 +100,32 @@ def test_validation_rejects_before_launch(lib):
                                             dummy, None, dummy, dummy, c.byref(gc), None) == -1
 
 
+def test_step_calls_refuse_host_memory_before_launch(lib):
+    """Valid shapes and options but host pointers: every step call returns
+    CRVQ_ERR_INVALID_ARG naming the array, instead of handing the pointer to a kernel."""
+    from paper_2412_09282_gb300 import _lib
+    c = ctypes
+    buf = (c.c_float * 4096)()
+    host = c.c_void_p((c.addressof(buf) + 15) // 16 * 16)       # 16-byte aligned host memory
+    cb = (_lib.crvq_codebook * 1)()
+    cb[0] = _lib.crvq_codebook(host.value, 4, 0, host.value, 2, 2)
+    gc = c.c_int64(0)
+    calls = [
+        lambda: lib.crvq_hessian(host, 4, 16, 8, 0.0, host, host, None, None, None),
+        lambda: lib.crvq_hessian_blocks(host, 4, 16, 8, 0.0, None, None, None, host, None),
+        lambda: lib.crvq_select_reorder_channels(host, 2, 16, 8, host, host, host, 0.5, 0, 0,
+                                                 host, None, host, host, c.byref(gc), None),
+        lambda: lib.crvq_kmeans_init(host, 16, 2, 2, 8, None, 0, 2, 0, host, None),
+        lambda: lib.crvq_encode_beam(host, 16, 2, 2, 8, host, cb, 1, 0, 1, 0, None, None),
+        lambda: lib.crvq_update_codebook(host, 16, 2, 2, 8, host, cb, 1, 0, host, None, None),
+        lambda: lib.crvq_reconstruct_error(host, 2, 16, 8, host, None, cb, 1, 0, None, 0, 0.0,
+                                           None, (c.c_double * 3)(), None),
+    ]
+    for call in calls:
+        assert call() == -1
+        assert b"not device memory" in lib.crvq_last_error()
+
+
 def test_quantize_layer_rejects_bad_shapes_and_options_before_launch(lib):
     """crvq_quantize_layer validates its shapes and configuration before any CUDA call."""
     from paper_2412_09282_gb300 import _lib
