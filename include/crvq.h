@@ -338,6 +338,8 @@ typedef struct crvq_layer_report {
  * calls, which reads the current contents of W and X (up to 16 graphs are kept per process,
  * least recently used evicted; their scratch stays reserved while they are kept). Setting
  * CRVQ_GRAPHS=0 in the environment runs every call directly. Results are identical either way.
+ * What the kernels report on the device (a non-finite input, a refused index, a bounded wait
+ * that ran out) is returned by the next crvq_sync on the device, not by this call.
  */
 crvq_status crvq_quantize_layer(const float* W, const float* X, int64_t M, int64_t N,
                                 int64_t n_tok, const crvq_config* cfg,
