@@ -319,6 +319,53 @@ def update_codebook(T, d, H_blocks, cbs, which):
 # --------------------------------------------------------------------------------------
 # Reconstruction, inverse reorder and losses (Alg. 1 QuantLoss; Sec. 4.3 reverse reorder)
 # --------------------------------------------------------------------------------------
+# NEXT-1: Hessian-coupled code search (the full Alg. 1 loss, cross-group terms included)
+# --------------------------------------------------------------------------------------
+def full_loss(W_sorted, H_sorted, cbs):
+    """tr(dW H dW^T) with dW = W_sorted - decode(cbs) and H in the same (sorted) channel order:
+    the Alg. 1 loss ||W X - W_enc X||^2 up to the factor n."""
+    W = np.asarray(W_sorted, dtype=np.float64)
+    dW = W - decode(W.shape[0], W.shape[1], cbs[0].C.shape[1], cbs)
+    return float(np.einsum("ij,jk,ik->", dW, np.asarray(H_sorted, np.float64), dW))
+
+
+def coupled_sweep(W_sorted, d, H_sorted, cbs, which, sweeps=1):
+    """Gauss-Seidel over the groups of codebook `which` under the full loss (others fixed).
+
+    The loss separates over rows. For row i and group g, with every other group fixed,
+      L = D_g^T H_gg D_g + 2 D_g^T b_g + const,   b_g = sum_{g' != g} H_gg' D_g',
+    where D = w_i - w_enc_i. Writing D_g = t_g - c (t_g: the row's segment minus the other
+    codebooks' codewords) and completing the square, the best codeword c minimises
+      (t_g + H_gg^-1 b_g - c)^T H_gg (t_g + H_gg^-1 b_g - c),
+    the block-diagonal score of Sec. 3.1 / Alg. 1 for a shifted target (ties: smaller index).
+    Groups are visited in order, each with the others' current codes, so the loss never rises.
+    Returns (new codes of `which` (M x G_cov int64), loss after each group step)."""
+    W = np.asarray(W_sorted, dtype=np.float64)
+    H = np.asarray(H_sorted, dtype=np.float64)
+    M, N = W.shape
+    cb = cbs[which]
+    C = cb.C.astype(np.float64)
+    codes = cb.codes.copy()
+    cur = [Codebook(c.C, c.codes, c.G_cov) for c in cbs]
+    cur[which] = Codebook(cb.C, codes, cb.G_cov)
+    D = W - decode(M, N, d, cur)                      # current error, all rows
+    history = []
+    for _ in range(sweeps):
+        for g in range(cb.G_cov):
+            sl = slice(g * d, (g + 1) * d)
+            Hgg = H[sl, sl]
+            b = D @ H[:, sl] - D[:, sl] @ Hgg         # sum over g' != g of D_g' H_g'g (rows)
+            t = D[:, sl] + C[codes[:, g]]             # segment minus the other codebooks
+            shift = np.linalg.solve(Hgg, b.T).T       # H_gg^-1 b_g (H symmetric)
+            err = quad_err(t + shift, C, Hgg)
+            k = np.argmin(err, axis=1)                # first minimum: the smaller index
+            codes[:, g] = k
+            D[:, sl] = t - C[k]
+            history.append(float(np.einsum("ij,jk,ik->", D, H, D)))
+    return codes, history
+
+
+# --------------------------------------------------------------------------------------
 def decode(M, N, d, cbs):
     """W_enc in the sorted channel order: sum of the covering codebooks' codewords."""
     G = N // d

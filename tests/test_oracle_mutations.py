@@ -203,6 +203,37 @@ def _eq_wa_multiplies(orig):
     return f
 
 
+def _coupled_variant(shift_sign, exclude_own_block):
+    """The coupled Gauss-Seidel sweep with one slip: the shift H_gg^-1 b_g subtracted instead
+    of added, or b_g formed with the group's own block left in."""
+    def plant(orig):
+        def f(W_sorted, d, H_sorted, cbs, which, sweeps=1):
+            W = np.asarray(W_sorted, np.float64)
+            H = np.asarray(H_sorted, np.float64)
+            M, N = W.shape
+            cb = cbs[which]
+            C = cb.C.astype(np.float64)
+            codes = cb.codes.copy()
+            cur = [O.Codebook(c.C, c.codes, c.G_cov) for c in cbs]
+            cur[which] = O.Codebook(cb.C, codes, cb.G_cov)
+            D = W - O.decode(M, N, d, cur)
+            hist = []
+            for _ in range(sweeps):
+                for g in range(cb.G_cov):
+                    sl = slice(g * d, (g + 1) * d)
+                    Hgg = H[sl, sl]
+                    b = D @ H[:, sl] - (D[:, sl] @ Hgg if exclude_own_block else 0.0)
+                    t = D[:, sl] + C[codes[:, g]]
+                    shift = shift_sign * np.linalg.solve(Hgg, b.T).T
+                    k = np.argmin(O.quad_err(t + shift, C, Hgg), axis=1)
+                    codes[:, g] = k
+                    D[:, sl] = t - C[k]
+                    hist.append(float(np.einsum("ij,jk,ik->", D, H, D)))
+            return codes, hist
+        return f
+    return plant
+
+
 def _beam_width_ignored(orig):
     def f(T, d, H_blocks, cbs, n_fixed, B, keep_if_better=False, **kw):
         return orig(T, d, H_blocks, cbs, n_fixed, 1, keep_if_better, **kw)
@@ -286,6 +317,15 @@ MUTATIONS = [
      ["test_hinv_diag_closed_forms", "test_hinv_diag_equals_schur_complement"]),
     ("Eq. (wa): inverse diagonal multiplied, not divided", "importance", _eq_wa_multiplies,
      ["test_importance_eq_wa_is_app_a2_for_uncorrelated_channels"]),
+    ("coupled search: shift subtracted", "coupled_sweep", _coupled_variant(-1.0, True),
+     ["test_coupled_sweep_never_raises_the_full_loss",
+      "test_coupled_sweep_fixed_point_is_optimal_per_group_by_brute_force",
+      "test_coupled_sweep_between_exhaustive_optimum_and_block_diagonal_start"]),
+    ("coupled search: own block left in the coupling", "coupled_sweep",
+     _coupled_variant(1.0, False),
+     ["test_coupled_sweep_never_raises_the_full_loss",
+      "test_coupled_sweep_fixed_point_is_optimal_per_group_by_brute_force",
+      "test_coupled_sweep_between_exhaustive_optimum_and_block_diagonal_start"]),
 ]
 
 

@@ -465,3 +465,91 @@ def test_schedule_invariants_small():
     h = out["loss_history"]
     assert h[-1] <= h[0] * (1 + 1e-9)
     assert out["loss_full"] > 0
+
+
+# ---------------------------------------------------------------- NEXT-1 coupled search
+def _coupled_case(seed, M=6, G=3, d=4, K=5, n=40):
+    rng = np.random.default_rng(seed)
+    N = G * d
+    X = rng.standard_normal((n, N)) @ rng.standard_normal((N, N)) * 0.4   # correlated channels
+    H = X.T @ X / n + 0.05 * np.eye(N)
+    W = rng.standard_normal((M, N)).astype(np.float32)
+    C = rng.standard_normal((K, d)).astype(np.float32)
+    codes = rng.integers(0, K, (M, G))
+    return W, H, C, codes, d, G
+
+
+def _row_loss(w, H, rec):
+    D = np.asarray(w, np.float64) - rec
+    return float(D @ H @ D)
+
+
+def test_coupled_sweep_never_raises_the_full_loss():
+    W, H, C, codes, d, G = _coupled_case(31)
+    cbs = [O.Codebook(C, codes, G)]
+    before = O.full_loss(W, H, cbs)
+    new, hist = O.coupled_sweep(W, d, H, cbs, 0, sweeps=3)
+    seq = [before] + hist
+    assert all(b <= a * (1 + 1e-12) for a, b in zip(seq, seq[1:]))
+    assert hist[-1] < before
+    assert abs(O.full_loss(W, H, [O.Codebook(C, new, G)]) - hist[-1]) <= 1e-9 * hist[-1]
+
+
+def test_coupled_sweep_with_block_diagonal_H_is_the_plain_encode():
+    W, H, C, codes, d, G = _coupled_case(32)
+    Hb = np.zeros_like(H)
+    for g in range(G):
+        Hb[g * d:(g + 1) * d, g * d:(g + 1) * d] = H[g * d:(g + 1) * d, g * d:(g + 1) * d]
+    new, _ = O.coupled_sweep(W, d, Hb, [O.Codebook(C, codes, G)], 0)
+    blocks = np.stack([Hb[g * d:(g + 1) * d, g * d:(g + 1) * d] for g in range(G)])
+    ref, _ = O.encode_beam(W, d, blocks.astype(np.float32), [O.Codebook(C, None, G)], 0, 1)
+    np.testing.assert_array_equal(new, ref[0])
+
+
+def test_coupled_sweep_fixed_point_is_optimal_per_group_by_brute_force():
+    """Swept to a fixed point, no single (row, group) code change lowers the row's full loss,
+    evaluated directly as (w - w_enc)^T H (w - w_enc)."""
+    W, H, C, codes, d, G = _coupled_case(33)
+    cbs = [O.Codebook(C, codes, G)]
+    for _ in range(20):
+        new, _ = O.coupled_sweep(W, d, H, cbs, 0)
+        done = np.array_equal(new, cbs[0].codes)
+        cbs = [O.Codebook(C, new, G)]
+        if done:
+            break
+    assert done
+    C64 = C.astype(np.float64)
+    for i in range(W.shape[0]):
+        rec = np.concatenate([C64[new[i, g]] for g in range(G)])
+        base = _row_loss(W[i], H, rec)
+        for g in range(G):
+            for k in range(C.shape[0]):
+                trial = rec.copy()
+                trial[g * d:(g + 1) * d] = C64[k]
+                assert _row_loss(W[i], H, trial) >= base * (1 - 1e-12) - 1e-12
+
+
+def test_coupled_sweep_between_exhaustive_optimum_and_block_diagonal_start():
+    W, H, C, codes, d, G = _coupled_case(34, M=3, G=2, K=4)
+    blocks = np.stack([H[g * d:(g + 1) * d, g * d:(g + 1) * d] for g in range(G)])
+    start, _ = O.encode_beam(W, d, blocks.astype(np.float32), [O.Codebook(C, None, G)], 0, 1)
+    new, _ = O.coupled_sweep(W, d, H, [O.Codebook(C, start[0], G)], 0, sweeps=4)
+    C64 = C.astype(np.float64)
+    for i in range(W.shape[0]):
+        best = min(_row_loss(W[i], H, np.concatenate([C64[a], C64[b]]))
+                   for a in range(4) for b in range(4))
+        got = _row_loss(W[i], H, np.concatenate([C64[new[i, 0]], C64[new[i, 1]]]))
+        init = _row_loss(W[i], H, np.concatenate([C64[start[0][i, 0]], C64[start[0][i, 1]]]))
+        assert best * (1 - 1e-12) <= got <= init * (1 + 1e-12)
+
+
+def test_coupled_sweep_of_second_codebook_is_the_sweep_on_the_residual():
+    W, H, C, codes, d, G = _coupled_case(35)
+    rng = np.random.default_rng(36)
+    C0 = rng.standard_normal((7, d)).astype(np.float32)
+    c0 = rng.integers(0, 7, (W.shape[0], G))
+    a, ha = O.coupled_sweep(W, d, H, [O.Codebook(C0, c0, G), O.Codebook(C, codes, G)], 1)
+    R = W.astype(np.float64) - np.concatenate([C0[c0[:, g]] for g in range(G)], axis=1)
+    b, hb = O.coupled_sweep(R, d, H, [O.Codebook(C, codes, G)], 0)
+    np.testing.assert_array_equal(a, b)
+    np.testing.assert_allclose(ha, hb, rtol=1e-9)
