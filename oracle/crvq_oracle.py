@@ -319,6 +319,28 @@ def update_codebook(T, d, H_blocks, cbs, which):
 # --------------------------------------------------------------------------------------
 # Reconstruction, inverse reorder and losses (Alg. 1 QuantLoss; Sec. 4.3 reverse reorder)
 # --------------------------------------------------------------------------------------
+# NEXT-3: inference product with the quantized matrix (no W_enc formed)
+# --------------------------------------------------------------------------------------
+def lut_matvec(Xin, perm, cbs, d):
+    """Y = Xin W_hat^T for a batch of inputs Xin (b x N, original channel order), with W_hat
+    given by its codes: the inputs are permuted once (x_sorted[p] = x[perm[p]]), each codebook
+    s and group g get a lookup table T_s,g[k] = <C_s[k], x_sorted,g>, and
+    y_i = sum over the covering codebooks and groups of T_s,g[codes_s[i, g]]."""
+    Xin = np.atleast_2d(np.asarray(Xin, dtype=np.float64))
+    b, N = Xin.shape
+    G = N // d
+    Xs = Xin[:, np.asarray(perm)] if perm is not None else Xin
+    M = cbs[0].codes.shape[0]
+    Y = np.zeros((b, M))
+    for cb in cbs:
+        C = cb.C.astype(np.float64)
+        for g in range(cb.G_cov):
+            T = Xs[:, g * d:(g + 1) * d] @ C.T          # b x K lookup table
+            Y += T[:, cb.codes[:, g]]
+    return Y
+
+
+# --------------------------------------------------------------------------------------
 # NEXT-1: Hessian-coupled code search (the full Alg. 1 loss, cross-group terms included)
 # --------------------------------------------------------------------------------------
 def full_loss(W_sorted, H_sorted, cbs):

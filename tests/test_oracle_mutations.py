@@ -234,6 +234,20 @@ def _coupled_variant(shift_sign, exclude_own_block):
     return plant
 
 
+def _lut_inverse_perm(orig):
+    """Inputs permuted with the inverse order."""
+    def f(Xin, perm, cbs, d):
+        return orig(Xin, None if perm is None else np.argsort(perm), cbs, d)
+    return f
+
+
+def _lut_base_only(orig):
+    """Extended codebooks left out of the product."""
+    def f(Xin, perm, cbs, d):
+        return orig(Xin, perm, cbs[:1], d)
+    return f
+
+
 def _beam_width_ignored(orig):
     def f(T, d, H_blocks, cbs, n_fixed, B, keep_if_better=False, **kw):
         return orig(T, d, H_blocks, cbs, n_fixed, 1, keep_if_better, **kw)
@@ -317,6 +331,10 @@ MUTATIONS = [
      ["test_hinv_diag_closed_forms", "test_hinv_diag_equals_schur_complement"]),
     ("Eq. (wa): inverse diagonal multiplied, not divided", "importance", _eq_wa_multiplies,
      ["test_importance_eq_wa_is_app_a2_for_uncorrelated_channels"]),
+    ("inference: inputs permuted with the inverse order", "lut_matvec", _lut_inverse_perm,
+     ["test_lut_matvec_equals_the_reconstructed_matrix_times_the_input"]),
+    ("inference: extended codebooks left out", "lut_matvec", _lut_base_only,
+     ["test_lut_matvec_equals_the_reconstructed_matrix_times_the_input"]),
     ("coupled search: shift subtracted", "coupled_sweep", _coupled_variant(-1.0, True),
      ["test_coupled_sweep_never_raises_the_full_loss",
       "test_coupled_sweep_fixed_point_is_optimal_per_group_by_brute_force",

@@ -553,3 +553,30 @@ def test_coupled_sweep_of_second_codebook_is_the_sweep_on_the_residual():
     b, hb = O.coupled_sweep(R, d, H, [O.Codebook(C, codes, G)], 0)
     np.testing.assert_array_equal(a, b)
     np.testing.assert_allclose(ha, hb, rtol=1e-9)
+
+
+# ---------------------------------------------------------------- NEXT-3 inference product
+def test_lut_matvec_equals_the_reconstructed_matrix_times_the_input():
+    """Lookup-table product vs the explicit route: W_hat (reconstruct_error, original order)
+    times the inputs by a matrix product."""
+    rng = np.random.default_rng(41)
+    M, N, d, Gc = 7, 32, 8, 2
+    W = rng.standard_normal((M, N)).astype(np.float32)
+    perm = rng.permutation(N).astype(np.int32)
+    C0 = rng.standard_normal((9, d)).astype(np.float32)
+    C1 = (0.3 * rng.standard_normal((5, d))).astype(np.float32)
+    cbs = [O.Codebook(C0, rng.integers(0, 9, (M, N // d)), N // d),
+           O.Codebook(C1, rng.integers(0, 5, (M, Gc)), Gc)]
+    Hb = np.stack([np.eye(d, dtype=np.float32)] * (N // d))
+    W_hat = O.reconstruct_error(W[:, perm], d, Hb, perm, cbs, Gc)[0]
+    Xin = rng.standard_normal((3, N))
+    np.testing.assert_allclose(O.lut_matvec(Xin, perm, cbs, d),
+                               Xin @ W_hat.astype(np.float64).T, rtol=1e-6, atol=1e-6)
+    # without a permutation the sorted order is the original one
+    W_id = O.reconstruct_error(W, d, Hb, None, cbs, Gc)[0]
+    np.testing.assert_allclose(O.lut_matvec(Xin, None, cbs, d),
+                               Xin @ W_id.astype(np.float64).T, rtol=1e-6, atol=1e-6)
+    # a permuted input channel moves with its weight column
+    e = np.zeros(N)
+    e[perm[5]] = 1.0
+    np.testing.assert_allclose(O.lut_matvec(e, perm, cbs, d)[0], W_hat[:, perm[5]], rtol=1e-6)
