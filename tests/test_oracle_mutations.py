@@ -248,6 +248,19 @@ def _lut_base_only(orig):
     return f
 
 
+def _ties_to_larger_index(orig):
+    """Equal errors resolved toward the larger codeword index (codebooks searched reversed)."""
+    def f(T, d, H_blocks, cbs, n_fixed, B, keep_if_better=False, **kw):
+        rev = []
+        for s, cb in enumerate(cbs):
+            K = cb.C.shape[0]
+            codes = None if cb.codes is None else (K - 1 - cb.codes)
+            rev.append(O.Codebook(cb.C[::-1], codes, cb.G_cov))
+        codes, verr = orig(T, d, H_blocks, rev, n_fixed, B, keep_if_better, **kw)
+        return [cb.C.shape[0] - 1 - c for cb, c in zip(cbs, codes)], verr
+    return f
+
+
 def _beam_width_ignored(orig):
     def f(T, d, H_blocks, cbs, n_fixed, B, keep_if_better=False, **kw):
         return orig(T, d, H_blocks, cbs, n_fixed, 1, keep_if_better, **kw)
@@ -321,6 +334,8 @@ MUTATIONS = [
     ("beam: width ignored", "encode_beam", _beam_width_ignored,
      [("test_beam_with_full_width_equals_exhaustive_search", (4, 2, 4)),
       ("test_beam_with_full_width_equals_exhaustive_search", (4, 3, 2))]),
+    ("encode: ties to the larger index", "encode_beam", _ties_to_larger_index,
+     ["test_beam_ties_follow_err_then_parent_rank_then_index"]),
     ("beam: keep-if-better ignored", "encode_beam", _keep_if_better_ignored,
      ["test_narrow_beam_never_beats_exhaustive_and_keep_if_better_keeps_optimum"]),
     ("losses: reconstruction scattered with perm, not its inverse", "reconstruct_error",

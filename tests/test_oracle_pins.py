@@ -580,3 +580,22 @@ def test_lut_matvec_equals_the_reconstructed_matrix_times_the_input():
     e = np.zeros(N)
     e[perm[5]] = 1.0
     np.testing.assert_allclose(O.lut_matvec(e, perm, cbs, d)[0], W_hat[:, perm[5]], rtol=1e-6)
+
+
+def test_beam_ties_follow_err_then_parent_rank_then_index():
+    """Exact ties (integer codewords, H = I): stage 0 orders equal errors by codeword index;
+    the last stage orders equal errors by parent rank, then index."""
+    d = 2
+    C0 = np.array([[0, 0], [2, 0]], np.float32)       # both at err 1 from t = (1, 0)
+    C1 = np.array([[1, 0], [-1, 0]], np.float32)      # (0, 0) and (1, 1) both reach err 0
+    T = np.array([[1, 0]], np.float32)
+    Hb = np.eye(d, dtype=np.float32)[None]
+    for B in (1, 2, 4):
+        codes, verr = O.encode_beam(T, d, Hb, [O.Codebook(C0, None, 1),
+                                               O.Codebook(C1, None, 1)], 0, B)
+        assert (codes[0][0, 0], codes[1][0, 0]) == (0, 0), B
+        assert verr[0, 0] == 0.0
+    # a single codebook with two equal codewords: the smaller index
+    codes, _ = O.encode_beam(T, d, Hb, [O.Codebook(np.array([[1, 1], [1, -1], [1, 1]],
+                                                            np.float32), None, 1)], 0, 1)
+    assert codes[0][0, 0] == 0
