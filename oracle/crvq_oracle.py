@@ -40,6 +40,12 @@ Readings where the paper is silent or ambiguous (all listed in the design notes)
     the others fixed, under the same H-weighted objective.
   * BeamSearchOptimize (Alg. 1) is a stage-wise beam over the codebooks that cover a
     vector, in codebook order, keeping the B best partial tuples by (err, parent rank, k).
+
+Beyond the current GPU path (each pinned in the tests, ahead of its kernel):
+  * MODE_WA_INV / hinv_diag: Eq. (wa) with the inverse-Hessian diagonal;
+  * coupled_sweep / full_loss: code search under the full Alg. 1 loss, cross-group terms
+    included (Gauss-Seidel over groups);
+  * lut_matvec: the inference product from codes, without forming W_enc.
 """
 from __future__ import annotations
 
