@@ -323,6 +323,18 @@ def test_hinv_diag_equals_schur_complement():
         assert abs(z @ H @ z - s) <= 1e-10 * s
 
 
+def test_hinv_diag_equals_woodbury_when_tokens_are_fewer_than_channels():
+    """H = delta I + X^T X / n with n < N: [H^-1]_ii = (1 - x_i^T (n delta I + X X^T)^-1 x_i)
+    / delta (Woodbury), from an n x n system instead of the N x N factor."""
+    rng = np.random.default_rng(24)
+    n, N, delta = 7, 20, 0.05
+    X = rng.standard_normal((n, N)) * rng.uniform(0.3, 2.0, N)
+    H = X.T @ X / n + delta * np.eye(N)
+    A = n * delta * np.eye(n) + X @ X.T
+    q = np.einsum("ki,ki->i", X, np.linalg.solve(A, X))
+    np.testing.assert_allclose(O.hinv_diag(H), (1.0 - q) / delta, rtol=1e-10)
+
+
 def test_importance_eq_wa_is_app_a2_for_uncorrelated_channels():
     """Eq. (wa) with a diagonal X^T X (orthogonal channels, no damping) is the App. A.2 form:
     1 / [H^-1]_ii = H_ii = xsq_i. With correlated channels the two differ."""
