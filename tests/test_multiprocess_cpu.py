@@ -76,3 +76,4 @@ def test_each_rank_quantizes_its_own_matrix():
     w0 = S.gen_W(cfg.with_(seed=cfg.seed + 0), np.arange(4))
     w1 = S.gen_W(cfg.with_(seed=cfg.seed + 1), np.arange(4))
     assert w0.shape == w1.shape and not np.array_equal(w0, w1)
+
