@@ -479,7 +479,8 @@ def lloyd(T, d, H_blocks, fixed, C0, G_cov, iters, seed_unused=None):
 
 
 def quantize_layer(W, X, cfg):
-    """The whole per-matrix schedule (Alg. 1, prequantization through the refinement loop) with the readings above.
+    """The whole per-matrix schedule (Alg. 1, prequantization through the refinement loop)
+    with the readings above.
 
     cfg has attributes d, K_base, n_ext, K_ext, crit_frac, B, kmeans_iters, refine_rounds,
     eps_rel, damp_rel, importance_mode, seed. Returns a dict of every intermediate result."""

@@ -1,5 +1,6 @@
 // C ABI of libcrvq: argument validation, status / error-word handling and the per-matrix
-// schedule (Alg. 1, prequantization through the refinement loop) that strings the kernels together on one stream.
+// schedule (Alg. 1, prequantization through the refinement loop) that strings the kernels
+// together on one stream.
 #include <atomic>
 #include <cmath>
 #include <cstring>
