@@ -7,9 +7,9 @@ least-squares refinement with beam re-encode, losses), i.e. one crvq_quantize_la
 the LLaMA-2-7B-shaped q_proj workload (W 4096 x 4096, 4096 calibration tokens, d = 8, K = 256,
 1 extended codebook on 2% channels, B = 8, 10 Lloyd iterations). The metric is code-search
 throughput: scored (hypothesis, codeword) pairs per second over the whole step; the per-layer
-time is reported beside it. `--config c5` makes a step the seven matrices of a LLaMA-2-7B decoder block
-(q, k, v, o, gate, up 4096-wide inputs sharing one X; down_proj 11008-wide with its own X),
-and reports the block time as well.
+time is reported beside it. `--config c5` makes a step the seven matrices of a LLaMA-2-7B
+decoder block (q, k, v, o, gate, up 4096-wide inputs sharing one X; down_proj 11008-wide with
+its own X), and reports the block time as well.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl crvq|reference] [--config c2]
 
