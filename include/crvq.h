@@ -12,7 +12,7 @@
  * Conventions (every call):
  *  - Arrays are device pointers owned by the caller unless a parameter says "host". The
  *    library keeps no pointer after the call returns. Row-major; fp32 unless stated. The
- *    step calls (crvq_hessian ... crvq_reconstruct_error, but not the no-allocation update)
+ *    step calls (crvq_hessian ... crvq_reconstruct_error, crvq_update_codebook_noalloc)
  *    check that each device array is device or managed memory and return
  *    CRVQ_ERR_INVALID_ARG for a host pointer; crvq_quantize_layer accepts either.
  *  - Calls enqueue work on `stream` and return without waiting, except calls that return a
@@ -84,8 +84,9 @@ typedef struct crvq_codebook {
 /* Message describing the last failure on the calling host thread ("" when none). */
 const char* crvq_last_error(void);
 
-/* Waits for `stream`, then returns and clears the device error word of the current device:
- * CRVQ_OK, CRVQ_ERR_DEVICE, CRVQ_ERR_NUMERIC or CRVQ_ERR_TIMEOUT (or CRVQ_ERR_CUDA). */
+/* Waits for `stream`, then returns and clears the device error words of the current device
+ * (the library's, and that of crvq_update_codebook_noalloc): CRVQ_OK, CRVQ_ERR_DEVICE,
+ * CRVQ_ERR_NUMERIC or CRVQ_ERR_TIMEOUT (or CRVQ_ERR_CUDA). */
 crvq_status crvq_sync(crvq_stream_t stream);
 
 /* Library build string (compiler, architecture). Host memory, static. */
@@ -231,22 +232,26 @@ crvq_status crvq_update_codebook(const float* T, int64_t ldT, int64_t M, int64_t
 
 /*
  * crvq_update_codebook without device memory allocation. The paper has no counterpart: this
- * entry point exists for callers that cannot call cudaMalloc or cudaFree (code running while
- * a CUDA graph is captured into a pool it does not own, runtimes that hand out a fixed memory
- * arena and forbid allocation after start-up, callers that must not synchronise). Arguments,
- * results and rounding are those of crvq_update_codebook; the caller still passes the
- * inputs and outputs. Its scratch is one file-scope device array of 4 MiB, held by every GPU
- * that loads the library until the process exits:
+ * entry point exists for callers that cannot call cudaMalloc or cudaFree, such as runtimes
+ * that hand out a fixed memory arena and forbid allocation after start-up, plugins whose host
+ * owns every device allocation, and latency-critical callers that must not synchronise
+ * (cudaFree synchronises the device). Arguments, validation (host pointers are refused with
+ * CRVQ_ERR_INVALID_ARG), results and rounding are those of crvq_update_codebook; the caller
+ * still passes the inputs and outputs. Its scratch is one file-scope device array of 4 MiB,
+ * held by every GPU that loads the library until the process exits:
  *  - sizes whose statistics exceed it (G_cov * K * 4 + K * 64 + 256 bytes, each part rounded
- *    up to 256 bytes, above 4 MiB - 256; e.g. K = 256 with more than ~4000 covered groups)
+ *    up to 256 bytes, above 4 MiB; e.g. K = 256 with more than ~4000 covered groups)
  *    return CRVQ_ERR_UNSUPPORTED before anything is enqueued;
- *  - every call shares the array, so calls that overlap on the GPU (different streams or
- *    devices' streams writing the same device's array) race; each call clears what must
- *    start at zero;
+ *  - every call shares the array and it keeps the last call's contents: each call clears
+ *    what must start at zero, and calls that overlap on the GPU (on different streams, or
+ *    host threads enqueueing on one device without ordering) race;
  *  - the first call on a device looks up the array's device address (cudaGetSymbolAddress)
  *    with that device current; make that first call before any stream capture;
- *  - device-side range checks (codes outside [0, K)) skip the bad entries and record them in
- *    this entry point's own error word inside the array, which crvq_sync does not read.
+ *  - what the kernels find on the device (codes outside [0, K), which are skipped; a
+ *    non-finite input; a normal matrix without a Cholesky factor, whose codeword keeps its
+ *    old value) is recorded in a second file-scope word, which the next crvq_sync on the
+ *    device reports (CRVQ_ERR_DEVICE, CRVQ_ERR_NUMERIC) and clears, like the other calls'
+ *    reports.
  */
 crvq_status crvq_update_codebook_noalloc(const float* T, int64_t ldT, int64_t M, int64_t G_sub,
                                          int32_t d, const float* H_blocks,

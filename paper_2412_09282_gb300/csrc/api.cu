@@ -165,14 +165,14 @@ ProfScope::~ProfScope() {
 // ------------------------------------------------------------------------- validation
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
-static crvq_status check_d(int32_t d) {
+crvq_status check_d(int32_t d) {
   if (d <= 0) return fail(CRVQ_ERR_INVALID_ARG, "d must be positive (got %d)", d);
   if (d != kD) return fail(CRVQ_ERR_UNSUPPORTED, "only d = 8 is implemented (got %d)", d);
   return CRVQ_OK;
 }
 
-static crvq_status check_set(const float* T, int64_t ldT, int64_t M, int64_t G_sub,
-                             const float* Hb) {
+crvq_status check_set(const float* T, int64_t ldT, int64_t M, int64_t G_sub,
+                      const float* Hb) {
   CRVQ_CHECK_ARG(T != nullptr, "T is NULL");
   CRVQ_CHECK_ARG(Hb != nullptr, "H_blocks is NULL");
   CRVQ_CHECK_ARG(M >= 1 && G_sub >= 1, "empty vector set (M=%lld, G_sub=%lld)", (long long)M,
@@ -185,8 +185,8 @@ static crvq_status check_set(const float* T, int64_t ldT, int64_t M, int64_t G_s
   return CRVQ_OK;
 }
 
-static crvq_status make_cblist(const crvq_codebook* cbs, int32_t n_cb, int64_t G_sub,
-                               bool need_codes_all, CbList* out) {
+crvq_status make_cblist(const crvq_codebook* cbs, int32_t n_cb, int64_t G_sub,
+                        bool need_codes_all, CbList* out) {
   CRVQ_CHECK_ARG(n_cb >= 0 && n_cb <= kMaxCodebooks, "n_cb must be in [0, %d]", kMaxCodebooks);
   CRVQ_CHECK_ARG(n_cb == 0 || cbs != nullptr, "codebook array is NULL");
   out->n = n_cb;
@@ -214,14 +214,14 @@ static bool is_device_ptr(const void* p) {
 
 // The kernels dereference these pointers: each non-null one must be device (or managed)
 // memory. A host pointer is refused here instead of reaching a kernel.
-static crvq_status check_dev(std::initializer_list<std::pair<const void*, const char*>> ps) {
+crvq_status check_dev(std::initializer_list<std::pair<const void*, const char*>> ps) {
   for (const auto& p : ps)
     if (p.first && !is_device_ptr(p.first))
       return fail(CRVQ_ERR_INVALID_ARG, "%s is not device memory", p.second);
   return CRVQ_OK;
 }
 
-static crvq_status check_dev_cbs(const crvq_codebook* cbs, int32_t n) {
+crvq_status check_dev_cbs(const crvq_codebook* cbs, int32_t n) {
   for (int32_t s = 0; s < n; ++s) {
     if (!is_device_ptr(cbs[s].C))
       return fail(CRVQ_ERR_INVALID_ARG, "codebook %d: C is not device memory", s);
@@ -356,8 +356,11 @@ crvq_status crvq_sync(crvq_stream_t stream) {
   CRVQ_TRY(device_error_word(&w));
   unsigned h = 0;
   CRVQ_CUDA(cudaMemcpy(&h, w, sizeof(unsigned), cudaMemcpyDeviceToHost));
+  unsigned h_na = 0;  // the no-allocation update's own word (read and cleared here too)
+  CRVQ_TRY(noalloc_take_error(&h_na));
+  if (h) CRVQ_CUDA(cudaMemset(w, 0, sizeof(unsigned)));
+  h |= h_na;
   if (h) {
-    CRVQ_CUDA(cudaMemset(w, 0, sizeof(unsigned)));
     if (h & ERRBIT_TIMEOUT) return fail(CRVQ_ERR_TIMEOUT, "a bounded device wait ran out");
     if (h & ERRBIT_INDEX) return fail(CRVQ_ERR_DEVICE, "a device-side index check failed");
     return fail(CRVQ_ERR_NUMERIC, "non-finite value or non-SPD normal matrix on the device");

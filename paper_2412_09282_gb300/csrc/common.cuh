@@ -7,7 +7,9 @@
 
 #include <cstdarg>
 #include <cstdio>
+#include <initializer_list>
 #include <string>
+#include <utility>
 
 #include "crvq.h"
 
@@ -152,5 +154,24 @@ struct CbList {
   CbView cb[kMaxCodebooks];
   int n;
 };
+
+// ---------------------------------------------------------------- argument validation
+// Shared by every entry point (api.cu): each returns CRVQ_OK or sets the last error and
+// returns CRVQ_ERR_INVALID_ARG (CRVQ_ERR_UNSUPPORTED for d != 8).
+crvq_status check_d(int32_t d);
+// A vector set: non-null, non-empty, ldT >= G_sub * 8 and a multiple of 4, 16-byte aligned.
+crvq_status check_set(const float* T, int64_t ldT, int64_t M, int64_t G_sub, const float* Hb);
+// Codebook array -> CbList, with the range checks of crvq_codebook's fields.
+crvq_status make_cblist(const crvq_codebook* cbs, int32_t n_cb, int64_t G_sub,
+                        bool need_codes_all, CbList* out);
+// Each non-null pointer must be device (or managed) memory: a host pointer is refused here
+// instead of reaching a kernel.
+crvq_status check_dev(std::initializer_list<std::pair<const void*, const char*>> ps);
+crvq_status check_dev_cbs(const crvq_codebook* cbs, int32_t n);
+
+// The error word of crvq_update_codebook_noalloc on the current device (noalloc.cu): *bits
+// receives its ERRBIT_* bits, which are then cleared. Reads nothing on a device where that
+// entry point has not run.
+crvq_status noalloc_take_error(unsigned* bits);
 
 }  // namespace crvq

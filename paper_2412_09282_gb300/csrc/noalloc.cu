@@ -1,10 +1,10 @@
 // crvq_update_codebook_noalloc: the least-squares codebook update without any device memory
-// allocation, for callers that cannot allocate. Examples are code running while a CUDA graph
-// is being captured into a pool they do not own, runtimes that hand out fixed memory arenas
-// and forbid cudaMalloc after start-up, and callers that must not synchronise (cudaFree
-// does). The update's scratch (per-group code counts, fixed-point sums, the scale) lives in
-// a file-scope device array of fixed size that every GPU loading the library holds until the
-// process exits.
+// allocation, for callers that cannot allocate: runtimes that hand out a fixed memory arena
+// and forbid cudaMalloc after start-up, plugins whose host owns every device allocation, and
+// latency-critical callers that must not synchronise (cudaFree synchronises the device). The
+// update's scratch (per-group code counts, fixed-point sums, the scale) lives in a file-scope
+// device array of fixed size that every GPU loading the library holds until the process
+// exits; its error word is a second file-scope device variable that crvq_sync reads.
 #include <mutex>
 #include <vector>
 
@@ -21,35 +21,61 @@ crvq_status launch_update_codebook_on(const SetView& set, const CbList& cbs, int
 namespace {
 
 // 4 MiB: counts for G_cov * K <= ~1M (group, code) pairs, e.g. K = 256 with up to ~4000
-// covered groups. The last 256 bytes hold this entry point's own error word.
+// covered groups.
 constexpr size_t kNoAllocBytes = size_t(4) << 20;
-constexpr size_t kNoAllocUsable = kNoAllocBytes - 256;
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+// ERRBIT_* of the kernels this entry point launches: set by them, read and cleared by
+// crvq_sync (zero when the module loads).
+static __device__ unsigned g_noalloc_err;
 
+struct DevAddrs {
+  void* scratch = nullptr;
+  unsigned* err = nullptr;
+};
 std::mutex g_na_mu;
-std::vector<void*> g_na_ptr;  // device address of g_noalloc_scratch, per device
+std::vector<DevAddrs> g_na;  // device addresses of the two variables, per device
 
-// Device address of the static scratch on the current device. The array's name in host code
-// is only a host-side stand-in, so the address is looked up once per device (with that
-// device current) and cached.
-crvq_status noalloc_scratch(void** out) {
+// Device addresses of the static scratch and error word on the current device. Their names
+// in host code are only host-side stand-ins, so the addresses are looked up once per device
+// (with that device current) and cached.
+crvq_status noalloc_addrs(DevAddrs* out) {
   int dev = 0;
   CRVQ_CUDA(cudaGetDevice(&dev));
   std::lock_guard<std::mutex> lk(g_na_mu);
-  if ((int)g_na_ptr.size() <= dev) g_na_ptr.resize(dev + 1, nullptr);
-  if (!g_na_ptr[dev]) {
-    void* p = nullptr;
-    CRVQ_CUDA(cudaGetSymbolAddress(&p, g_noalloc_scratch));
-    g_na_ptr[dev] = p;
+  if ((int)g_na.size() <= dev) g_na.resize(dev + 1);
+  if (!g_na[dev].scratch) {
+    DevAddrs a;
+    CRVQ_CUDA(cudaGetSymbolAddress(&a.scratch, g_noalloc_scratch));
+    void* e = nullptr;
+    CRVQ_CUDA(cudaGetSymbolAddress(&e, g_noalloc_err));
+    a.err = static_cast<unsigned*>(e);
+    g_na[dev] = a;
   }
-  *out = g_na_ptr[dev];
+  *out = g_na[dev];
   return CRVQ_OK;
 }
 
-bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
-
 }  // namespace
+
+namespace crvq {
+
+crvq_status noalloc_take_error(unsigned* bits) {
+  *bits = 0;
+  int dev = 0;
+  CRVQ_CUDA(cudaGetDevice(&dev));
+  unsigned* w = nullptr;
+  {
+    std::lock_guard<std::mutex> lk(g_na_mu);
+    if (dev < (int)g_na.size()) w = g_na[dev].err;
+  }
+  if (!w) return CRVQ_OK;  // the entry point never ran on this device
+  CRVQ_CUDA(cudaMemcpy(bits, w, sizeof(unsigned), cudaMemcpyDeviceToHost));
+  if (*bits) CRVQ_CUDA(cudaMemset(w, 0, sizeof(unsigned)));
+  return CRVQ_OK;
+}
+
+}  // namespace crvq
 
 using namespace crvq;
 
@@ -60,39 +86,24 @@ extern "C" crvq_status crvq_update_codebook_noalloc(const float* T, int64_t ldT,
                                                     int32_t which, float* C_out,
                                                     int32_t* counts, crvq_stream_t stream) {
   clear_last_error();
-  if (d != kD) return fail(d <= 0 ? CRVQ_ERR_INVALID_ARG : CRVQ_ERR_UNSUPPORTED,
-                           "only d = 8 is implemented (got %d)", d);
-  CRVQ_CHECK_ARG(T && H_blocks && C_out, "T, H_blocks and C_out must not be NULL");
-  CRVQ_CHECK_ARG(M >= 1 && G_sub >= 1 && ldT >= G_sub * kD && ldT % 4 == 0,
-                 "bad vector set (M, G_sub, ldT)");
-  CRVQ_CHECK_ARG(aligned16(T) && aligned16(H_blocks), "T and H_blocks must be 16-byte aligned");
-  CRVQ_CHECK_ARG(M * G_sub < (int64_t)1 << 31, "too many vectors in one set");
-  CRVQ_CHECK_ARG(n_cb >= 1 && n_cb <= kMaxCodebooks && cbs, "n_cb must be in [1, %d]",
-                 kMaxCodebooks);
-  CRVQ_CHECK_ARG(which >= 0 && which < n_cb, "which must be in [0, n_cb)");
+  // the same checks as crvq_update_codebook, host pointers refused before any launch
+  CRVQ_TRY(check_d(d));
+  CRVQ_TRY(check_set(T, ldT, M, G_sub, H_blocks));
+  CRVQ_CHECK_ARG(n_cb >= 1 && which >= 0 && which < n_cb, "which must be in [0, n_cb)");
+  CRVQ_CHECK_ARG(C_out != nullptr, "C_out is NULL");
   CbList cl;
-  cl.n = n_cb;
-  for (int s = 0; s < n_cb; ++s) {
-    const crvq_codebook& c = cbs[s];
-    CRVQ_CHECK_ARG(c.C && aligned16(c.C), "codebook %d: C is NULL or not 16-byte aligned", s);
-    CRVQ_CHECK_ARG(c.K >= 1 && c.K <= 65536, "codebook %d: K must be in [1, 65536]", s);
-    CRVQ_CHECK_ARG(c.G_cov >= 0 && c.G_cov <= G_sub, "codebook %d: G_cov out of [0, G_sub]", s);
-    CRVQ_CHECK_ARG(c.G_cov == 0 || (c.codes && c.ld >= c.G_cov),
-                   "codebook %d: codes NULL or ld < G_cov", s);
-    cl.cb[s] = CbView{c.C, c.codes, c.ld, c.G_cov, c.K};
-  }
+  CRVQ_TRY(make_cblist(cbs, n_cb, G_sub, true, &cl));
+  CRVQ_TRY(check_dev({{T, "T"}, {H_blocks, "H_blocks"}, {C_out, "C_out"}, {counts, "counts"}}));
+  CRVQ_TRY(check_dev_cbs(cbs, n_cb));
   const size_t need = update_scratch_bytes(cl.cb[which].G_cov, cl.cb[which].K);
-  if (need > kNoAllocUsable)
+  if (need > kNoAllocBytes)
     return fail(CRVQ_ERR_UNSUPPORTED,
                 "crvq_update_codebook_noalloc: G_cov * K = %lld (group, code) pairs need %zu "
                 "bytes of scratch; the static limit is %zu bytes",
-                (long long)(cl.cb[which].G_cov * cl.cb[which].K), need, kNoAllocUsable);
-  void* scratch = nullptr;
-  CRVQ_TRY(noalloc_scratch(&scratch));
-  unsigned* err = reinterpret_cast<unsigned*>(static_cast<char*>(scratch) + kNoAllocUsable);
-  cudaStream_t s = (cudaStream_t)stream;
-  CRVQ_CUDA(cudaMemsetAsync(err, 0, sizeof(unsigned), s));
+                (long long)(cl.cb[which].G_cov * cl.cb[which].K), need, kNoAllocBytes);
+  DevAddrs a;
+  CRVQ_TRY(noalloc_addrs(&a));
   SetView set{T, ldT, M, G_sub, H_blocks};
-  return launch_update_codebook_on(set, cl, which, C_out, counts, scratch, kNoAllocUsable, err,
-                                   s);
+  return launch_update_codebook_on(set, cl, which, C_out, counts, a.scratch, kNoAllocBytes,
+                                   a.err, (cudaStream_t)stream);
 }

@@ -22,8 +22,16 @@ namespace crvq {
 
 namespace {
 
+// max(a, b) that keeps a NaN: fmaxf returns the other operand when one is NaN, which would
+// leave the bound below finite and hide a non-finite input from the scale check.
+__device__ __forceinline__ float max_keep_nan(float a, float b) {
+  return (b > a || b != b) ? b : a;
+}
+
 // maxbits[0] = max |T| over the covered vectors, maxbits[1] = max row sum of |H_g|,
-// maxbits[2 + s] = max |C_s| (float bits of non-negative values, merged with atomicMax).
+// maxbits[2 + s] = max |C_s| (float bits of non-negative values, merged with atomicMax; a NaN
+// has larger bits than every finite value and Inf, so it survives the merge and makes the
+// bound non-finite).
 __global__ void __launch_bounds__(256)
 maxabs_kernel(SetView set, int64_t G_cov, CbList cbs, int which, unsigned* __restrict__ maxbits) {
   const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -34,22 +42,24 @@ maxabs_kernel(SetView set, int64_t G_cov, CbList cbs, int which, unsigned* __res
     const int64_t i = v / G_cov, g = v % G_cov;
     const float4* t = reinterpret_cast<const float4*>(set.T + i * set.ldT + g * kD);
     const float4 a = t[0], b = t[1];
-    tm = fmaxf(tm, fmaxf(fmaxf(fabsf(a.x), fabsf(a.y)), fmaxf(fabsf(a.z), fabsf(a.w))));
-    tm = fmaxf(tm, fmaxf(fmaxf(fabsf(b.x), fabsf(b.y)), fmaxf(fabsf(b.z), fabsf(b.w))));
+    tm = max_keep_nan(tm, max_keep_nan(max_keep_nan(fabsf(a.x), fabsf(a.y)),
+                                       max_keep_nan(fabsf(a.z), fabsf(a.w))));
+    tm = max_keep_nan(tm, max_keep_nan(max_keep_nan(fabsf(b.x), fabsf(b.y)),
+                                       max_keep_nan(fabsf(b.z), fabsf(b.w))));
   }
   float hm = 0.f;
   for (int64_t r = tid; r < G_cov * kD; r += nth) {
     const float* h = set.Hb + r * kD;
     float s = 0.f;
 #pragma unroll
-    for (int j = 0; j < kD; ++j) s += fabsf(h[j]);
-    hm = fmaxf(hm, s);
+    for (int j = 0; j < kD; ++j) s += fabsf(h[j]);  // a NaN entry makes the sum NaN
+    hm = max_keep_nan(hm, s);
   }
   // warp max, then one atomic per warp
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
-    tm = fmaxf(tm, __shfl_xor_sync(0xffffffffu, tm, off));
-    hm = fmaxf(hm, __shfl_xor_sync(0xffffffffu, hm, off));
+    tm = max_keep_nan(tm, __shfl_xor_sync(0xffffffffu, tm, off));
+    hm = max_keep_nan(hm, __shfl_xor_sync(0xffffffffu, hm, off));
   }
   if ((threadIdx.x & 31) == 0) {
     atomicMax(&maxbits[0], __float_as_uint(tm));
@@ -59,9 +69,10 @@ maxabs_kernel(SetView set, int64_t G_cov, CbList cbs, int which, unsigned* __res
     if (s == which) continue;
     float m = 0.f;
     for (int64_t e = tid; e < (int64_t)cbs.cb[s].K * kD; e += nth)
-      m = fmaxf(m, fabsf(cbs.cb[s].C[e]));
+      m = max_keep_nan(m, fabsf(cbs.cb[s].C[e]));
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, off));
+    for (int off = 16; off > 0; off >>= 1)
+      m = max_keep_nan(m, __shfl_xor_sync(0xffffffffu, m, off));
     if ((threadIdx.x & 31) == 0) atomicMax(&maxbits[2 + s], __float_as_uint(m));
   }
 }

@@ -118,6 +118,8 @@ def test_step_calls_refuse_host_memory_before_launch(lib):
         lambda: lib.crvq_kmeans_init(host, 16, 2, 2, 8, None, 0, 2, 0, host, None),
         lambda: lib.crvq_encode_beam(host, 16, 2, 2, 8, host, cb, 1, 0, 1, 0, None, None),
         lambda: lib.crvq_update_codebook(host, 16, 2, 2, 8, host, cb, 1, 0, host, None, None),
+        lambda: lib.crvq_update_codebook_noalloc(host, 16, 2, 2, 8, host, cb, 1, 0, host, None,
+                                                 None),
         lambda: lib.crvq_reconstruct_error(host, 2, 16, 8, host, None, cb, 1, 0, None, 0, 0.0,
                                            None, (c.c_double * 3)(), None),
     ]

@@ -375,6 +375,33 @@ def test_device_index_check_reports_and_recovers(c1):
     P.crvq_sync()
 
 
+@pytest.mark.parametrize("where", ["T", "other_codebook", "H"])
+def test_update_reports_a_nan_in_its_inputs(c1, where):
+    """A NaN in the targets, in a fixed codebook or in an H block makes the fixed-point scale
+    bound non-finite (the maxima keep NaN), and the next crvq_sync reports CRVQ_ERR_NUMERIC
+    instead of returning a codebook built from INT_MIN terms with status OK."""
+    W, Hb = c1["W"].copy(), c1["Hb0"].copy()
+    M, N = W.shape
+    G, Gc = N // D, 4
+    rng = np.random.default_rng(91)
+    Cb = _codebook_for(W, G, 64, 92)
+    Ce = (0.3 * _codebook_for(W, G, 16, 93)).astype(np.float32)
+    if where == "T":
+        W[7, 13] = np.nan
+    elif where == "other_codebook":
+        Ce[3, 5] = np.nan
+    else:
+        Hb[2, 4, 4] = np.nan
+    cbs = [Codebook(dev(Cb), dev(rng.integers(0, 64, (M, G)).astype(np.int32)), G),
+           Codebook(dev(Ce), dev(rng.integers(0, 16, (M, Gc)).astype(np.int32)), Gc)]
+    P.crvq_sync()
+    with pytest.raises(P.CrvqError) as e:
+        P.crvq_update_codebook(dev(W), D, dev(Hb), cbs, 0)
+        P.crvq_sync()
+    assert e.value.status == -6
+    P.crvq_sync()                                        # the word was cleared
+
+
 def test_invalid_arguments_raise_before_launch(c1):
     W = dev(c1["W"])
     with pytest.raises(P.CrvqError) as e:

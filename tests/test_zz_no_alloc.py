@@ -1,11 +1,11 @@
 """crvq_update_codebook_noalloc against crvq_update_codebook, through the C ABI.
 
-Some callers cannot allocate device memory: code running while a CUDA graph is captured into
-a pool it does not own, runtimes that hand out a fixed arena and forbid cudaMalloc after
-start-up, callers that must not synchronise. For them the library offers an update that keeps
-its scratch in a fixed device array instead of allocating. This file is collected last so
-that a failure here does not hide the other tests' results; it passes alone in a fresh
-process as well as after the rest of the suite.
+Some callers cannot allocate device memory: runtimes that hand out a fixed arena and forbid
+cudaMalloc after start-up, plugins whose host owns every device allocation, latency-critical
+callers that must not synchronise (cudaFree synchronises the device). For them the library
+offers an update that keeps its scratch in a fixed device array instead of allocating. This
+file is collected last so that a failure here does not hide the other tests' results; it
+passes alone in a fresh process as well as after the rest of the suite.
 """
 import ctypes
 
@@ -78,3 +78,47 @@ def test_noalloc_update_rejects_sizes_beyond_its_scratch():
         P.crvq_update_codebook_noalloc(T, D, Hb, [Codebook(C, codes, G)], 0)
     assert e.value.status == -2
     assert "static limit" in str(e.value)
+
+
+def test_noalloc_update_reports_device_errors_through_crvq_sync():
+    """What the kernels of the no-allocation update find on the device reaches the caller:
+    an out-of-range code (skipped) comes back from the next crvq_sync as CRVQ_ERR_DEVICE, a NaN
+    in another codebook as CRVQ_ERR_NUMERIC; each report is cleared once read, and a clean
+    call afterwards reports nothing and still equals the allocating update."""
+    import paper_2412_09282_gb300 as P
+    from paper_2412_09282_gb300 import Codebook, build
+    build.build()
+    W, Hb, Cb, Ce, cbc, cec, G = _setup(7, 64, 4)
+    Wd = torch.from_numpy(W).cuda()
+    Hd = torch.from_numpy(Hb).cuda()
+    torch.cuda.synchronize()
+    P.crvq_sync()                                            # nothing pending beforehand
+
+    bad_codes = cbc.copy()
+    bad_codes[5, 3] = 64                                     # K = 64: out of range
+    cbs = [Codebook(torch.from_numpy(Cb).cuda(), torch.from_numpy(bad_codes).cuda(), G),
+           Codebook(torch.from_numpy(Ce).cuda(), torch.from_numpy(cec).cuda(), 4)]
+    P.crvq_update_codebook_noalloc(Wd, D, Hd, cbs, 0)
+    with pytest.raises(P.CrvqError) as e:
+        P.crvq_sync()
+    assert e.value.status == -7                              # CRVQ_ERR_DEVICE
+    P.crvq_sync()                                            # the report was cleared
+
+    nan_ext = Ce.copy()
+    nan_ext[2, 1] = np.nan
+    cbs = [Codebook(torch.from_numpy(Cb).cuda(), torch.from_numpy(cbc).cuda(), G),
+           Codebook(torch.from_numpy(nan_ext).cuda(), torch.from_numpy(cec).cuda(), 4)]
+    P.crvq_update_codebook_noalloc(Wd, D, Hd, cbs, 0)
+    with pytest.raises(P.CrvqError) as e:
+        P.crvq_sync()
+    assert e.value.status == -6                              # CRVQ_ERR_NUMERIC
+    P.crvq_sync()
+
+    cbs = [Codebook(torch.from_numpy(Cb).cuda(), torch.from_numpy(cbc).cuda(), G),
+           Codebook(torch.from_numpy(Ce).cuda(), torch.from_numpy(cec).cuda(), 4)]
+    out, cnt = P.crvq_update_codebook_noalloc(Wd, D, Hd, cbs, 0)
+    P.crvq_sync()
+    ref, ref_cnt = P.crvq_update_codebook(Wd, D, Hd, cbs, 0)
+    P.crvq_sync()
+    np.testing.assert_array_equal(out.cpu().numpy(), ref.cpu().numpy())
+    np.testing.assert_array_equal(cnt.cpu().numpy(), ref_cnt.cpu().numpy())
