@@ -286,6 +286,69 @@ def _reconstruction_forward_perm(orig):
     return f
 
 
+def _schedule_variant(slip):
+    """The per-matrix schedule with one wiring slip: the base codebook fitted on W instead of
+    the reordered W ("base_on_W"), warm-started from the prequantize codebook ("warm_start"),
+    extended codebooks fitted on the raw critical vectors instead of the residual of the base
+    ("ext_without_base"), or the refinement updating the codebooks in reverse order
+    ("refine_reversed"). Otherwise the same steps as the oracle's quantize_layer."""
+    def plant(orig):
+        def f(W, X, cfg):
+            d = cfg.d
+            W = np.asarray(W, dtype=np.float32)
+            M, N = W.shape
+            G = N // d
+            out = {}
+            H, xsq, Hb0, delta = O.hessian(X, cfg.damp_rel, d)
+            C0 = O.kmeans_init(W, d, G, cfg.K_base, O.phase_seed(cfg.seed, O.PHASE_PREQUANT, 0))
+            pre, _ = O.lloyd(W, d, Hb0, [], C0, G, cfg.kmeans_iters)
+            W_pre, pre_loss, _, _ = O.reconstruct_error(W, d, Hb0, None, [pre], 0)
+            out.update(C_pre=pre.C, codes_pre=pre.codes, W_pre=W_pre, loss_pre=pre_loss)
+            perm, I, Ws, Hb, Gc = O.select_reorder_channels(
+                W, d, W_pre, xsq, H, cfg.crit_frac, cfg.importance_mode,
+                O.phase_seed(cfg.seed, O.PHASE_RANDOM, 0))
+            out.update(perm=perm, importance=I, W_sorted=Ws, H_blocks=Hb, n_crit_groups=Gc)
+            T_base = W if slip == "base_on_W" else Ws
+            if slip == "warm_start":
+                Cb0 = pre.C
+            else:
+                Cb0 = O.kmeans_init(T_base, d, G, cfg.K_base,
+                                    O.phase_seed(cfg.seed, O.PHASE_BASE, 0))
+            base, obj = O.lloyd(T_base, d, Hb, [], Cb0, G, cfg.kmeans_iters)
+            out["base_objective"] = obj
+            cbs = [base]
+            Tc, Hbc = Ws[:, :Gc * d], Hb[:Gc]
+            for t in range(1, cfg.n_ext + 1):
+                fixed = [] if slip == "ext_without_base" else \
+                    [O.Codebook(cb.C, cb.codes[:, :Gc], Gc) for cb in cbs]
+                Ct0 = O.kmeans_init(Tc, d, Gc, cfg.K_ext, O.phase_seed(cfg.seed, O.PHASE_EXT, t),
+                                    fixed)
+                ext, _ = O.lloyd(Tc, d, Hbc, fixed, Ct0, Gc, cfg.kmeans_iters)
+                cbs.append(O.Codebook(ext.C, ext.codes, Gc))
+            _, lb, _, _ = O.reconstruct_error(Ws, d, Hb, perm, cbs, Gc)
+            history = [lb]
+            order = range(len(cbs))
+            for _ in range(cfg.refine_rounds):
+                for j in (reversed(order) if slip == "refine_reversed" else order):
+                    C, _ = O.update_codebook(Ws, d, Hb, cbs, j)
+                    cbs[j] = O.Codebook(C, cbs[j].codes, cbs[j].G_cov)
+                codes, _ = O.encode_beam(Ws, d, Hb, cbs, n_fixed=0, B=cfg.B, keep_if_better=True)
+                cbs = [O.Codebook(cb.C, codes[q], cb.G_cov) for q, cb in enumerate(cbs)]
+                _, lb, _, _ = O.reconstruct_error(Ws, d, Hb, perm, cbs, Gc)
+                history.append(lb)
+            out["loss_history"] = history
+            W_hat, lb, lc, lf = O.reconstruct_error(Ws, d, Hb, perm, cbs, Gc, X, float(delta))
+            out.update(codebooks=cbs, W_hat=W_hat, loss_block=lb, loss_crit=lc, loss_full=lf)
+            return out
+        return f
+    return plant
+
+
+_SCHEDULE_PINS = ["test_schedule_with_one_codeword_per_codebook_is_a_sequence_of_weighted_means",
+                  "test_schedule_without_lloyd_iterations_keeps_the_sampled_codewords",
+                  "test_schedule_with_a_codeword_per_vector_reconstructs_exactly"]
+
+
 # (name, oracle attribute, planted version, pins that must catch it: a test name, or a test
 # name with its arguments)
 MUTATIONS = [
@@ -359,6 +422,14 @@ MUTATIONS = [
      ["test_coupled_sweep_never_raises_the_full_loss",
       "test_coupled_sweep_fixed_point_is_optimal_per_group_by_brute_force",
       "test_coupled_sweep_between_exhaustive_optimum_and_block_diagonal_start"]),
+    ("schedule: base codebook fitted on W, not the reordered W", "quantize_layer",
+     _schedule_variant("base_on_W"), _SCHEDULE_PINS),
+    ("schedule: base k-means warm-started from the prequantize codebook", "quantize_layer",
+     _schedule_variant("warm_start"), _SCHEDULE_PINS),
+    ("schedule: extended codebooks fitted without subtracting the base", "quantize_layer",
+     _schedule_variant("ext_without_base"), _SCHEDULE_PINS),
+    ("schedule: refinement updates the codebooks in reverse order", "quantize_layer",
+     _schedule_variant("refine_reversed"), _SCHEDULE_PINS),
 ]
 
 

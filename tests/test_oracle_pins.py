@@ -479,6 +479,190 @@ def test_schedule_invariants_small():
     assert out["loss_full"] > 0
 
 
+# ---------------------------------------------------------------- schedule wiring pins
+# These restate the per-matrix schedule (Alg. 1, prequantization through the refinement loop)
+# by hand on cases whose result has a closed form, so that a wiring slip (a step fed the
+# wrong matrix, Hessian blocks, seed, residual or order) fails one of them. They use only
+# numpy and the synthetic generator, none of the oracle's step functions.
+def _h64(X, damp_rel):
+    """H = X^T X / n + delta I in fp64, the undamped diagonal and delta (App. A.2 proxy with
+    the damping reading)."""
+    X = np.asarray(X, np.float64)
+    S_ = X.T @ X / X.shape[0]
+    xsq = np.diag(S_).copy()
+    delta = float(np.float32(damp_rel)) * xsq.mean()
+    return S_ + delta * np.eye(S_.shape[0]), xsq, delta
+
+
+def _blocks(H, perm, d):
+    Hp = H[np.ix_(perm, perm)]
+    return [Hp[g * d:(g + 1) * d, g * d:(g + 1) * d] for g in range(len(perm) // d)]
+
+
+def _wmean(pairs):
+    """argmin_c sum (t - c)^T H (t - c) over (H, t) pairs: (sum H)^-1 sum H t."""
+    A = sum(H for H, _ in pairs)
+    b = sum(H @ t for H, t in pairs)
+    return np.linalg.solve(A, b)
+
+
+def _seed(seed, phase, cb):
+    return int(S.splitmix64(seed, np.array([phase * 1024 + cb]))[0])
+
+
+def _strata(n, K, seed):
+    """One vector index per stratum [floor(k n / K), floor((k+1) n / K))."""
+    out = []
+    for k in range(K):
+        lo, hi = (k * n) // K, ((k + 1) * n) // K
+        out.append(lo + int(S.splitmix64(seed, np.array([k]))[0]) % (hi - lo))
+    return out
+
+
+def _nearest(t, C, Hg):
+    e = [float((t - c) @ Hg @ (t - c)) for c in np.asarray(C, np.float64)]
+    return int(np.argmin(e))
+
+
+def _importance_perm(W, W_pre, xsq):
+    I = 0.5 * xsq * np.max((np.asarray(W, np.float64) - W_pre) ** 2, axis=0)
+    return np.array(sorted(range(len(I)), key=lambda j: (-I[j], j)))
+
+
+def test_schedule_with_one_codeword_per_codebook_is_a_sequence_of_weighted_means():
+    """K_base = K_ext = 1: every code is 0, so each Lloyd fit is the H-weighted mean of its
+    targets (Sec. 3.1 Eq. kmeans with one cluster) and the schedule is a fixed sequence of
+    such means: prequantize in the original order, importance from that reconstruction
+    (App. A.2), base on the reordered W with the reordered H blocks, each extended codebook on
+    the critical residual of the base and earlier extended codebooks (Sec. 4.3), then one
+    refinement round updating base, ext 1, ext 2 in that order with the others fixed."""
+    cfg = S.LayerConfig("pin_k1", 6, 32, 48, "outlier_cols", "lognormal", 0.5,
+                        n_outlier_cols=2, K_base=1, n_ext=2, K_ext=1, crit_frac=0.3, B=2,
+                        kmeans_iters=2, refine_rounds=1)
+    W, X = S.gen_W(cfg), S.gen_X(cfg)
+    out = O.quantize_layer(W, X, cfg)
+    d, M, N = 8, cfg.M, cfg.N
+    G = N // d
+    Gc = 2                                             # ceil(0.3 * 32 / 8)
+    H, xsq, delta = _h64(X, cfg.damp_rel)
+    W64 = W.astype(np.float64)
+    vec = lambda A, i, g: A[i, g * d:(g + 1) * d]
+    H0 = _blocks(H, np.arange(N), d)
+    c_pre = _wmean([(H0[g], vec(W64, i, g)) for i in range(M) for g in range(G)])
+    perm = _importance_perm(W, np.tile(c_pre, G)[None, :], xsq)
+    Ws = W64[:, perm]
+    Hs = _blocks(H, perm, d)
+    c_b = _wmean([(Hs[g], vec(Ws, i, g)) for i in range(M) for g in range(G)])
+    crit = [(i, g) for i in range(M) for g in range(Gc)]
+    c_1 = _wmean([(Hs[g], vec(Ws, i, g) - c_b) for i, g in crit])
+    c_2 = _wmean([(Hs[g], vec(Ws, i, g) - c_b - c_1) for i, g in crit])
+    # one refinement round: base, then ext 1, then ext 2, each with the others fixed
+    c_b = _wmean([(Hs[g], vec(Ws, i, g) - (c_1 + c_2 if g < Gc else 0.0))
+                  for i in range(M) for g in range(G)])
+    c_1 = _wmean([(Hs[g], vec(Ws, i, g) - c_b - c_2) for i, g in crit])
+    c_2 = _wmean([(Hs[g], vec(Ws, i, g) - c_b - c_1) for i, g in crit])
+
+    scale = np.abs(c_pre).max()   # the second extended codeword is ~0 (its residual's
+                                  # weighted mean is zero once ext 1 fits it): absolute scale
+
+    def close(a, b):
+        np.testing.assert_allclose(np.asarray(a, np.float64).reshape(-1), b, rtol=0,
+                                   atol=2e-5 * scale)
+    close(out["C_pre"], c_pre)
+    np.testing.assert_array_equal(out["perm"], perm)
+    assert out["n_crit_groups"] == Gc
+    cbs = out["codebooks"]
+    close(cbs[0].C, c_b)
+    close(cbs[1].C, c_1)
+    close(cbs[2].C, c_2)
+    rec = np.tile(c_b, G)
+    rec[:Gc * d] += np.tile(c_1 + c_2, Gc)
+    D = Ws - rec[None, :]
+    lb = sum(float(vec(D, i, g) @ Hs[g] @ vec(D, i, g)) for i in range(M) for g in range(G))
+    lc = sum(float(vec(D, i, g) @ Hs[g] @ vec(D, i, g)) for i, g in crit)
+    Dorig = np.empty_like(D)
+    Dorig[:, perm] = D
+    lf = float(np.einsum("ij,jk,ik->", Dorig, H, Dorig))
+    assert out["loss_block"] == pytest.approx(lb, rel=1e-5)
+    assert out["loss_crit"] == pytest.approx(lc, rel=1e-5)
+    assert out["loss_full"] == pytest.approx(lf, rel=1e-5)
+
+
+def test_schedule_without_lloyd_iterations_keeps_the_sampled_codewords():
+    """kmeans_iters = 0 and no refinement: each codebook is its k-means initialisation, the
+    vectors (or critical residuals) drawn from the strata with that phase's seed, and the
+    codes are the arg-min encodes. The prequantize codebook comes from W in the original order
+    (phase 1), the base from the reordered W (phase 2, a fresh draw, not the prequantize
+    codebook), extended codebook t from the critical residual after the base and the earlier
+    extended codebooks (phase 3, codebook t)."""
+    cfg = S.LayerConfig("pin_t0", 8, 32, 40, "outlier_cols", "lognormal", 0.5,
+                        n_outlier_cols=2, K_base=8, n_ext=2, K_ext=4, crit_frac=0.3, B=2,
+                        kmeans_iters=0, refine_rounds=0, seed=5)
+    W, X = S.gen_W(cfg), S.gen_X(cfg)
+    out = O.quantize_layer(W, X, cfg)
+    d, M, N = 8, cfg.M, cfg.N
+    G, Gc = N // d, 2
+    H, xsq, _ = _h64(X, cfg.damp_rel)
+    W64 = W.astype(np.float64)
+    vec = lambda A, v, Gs: A[v // Gs, (v % Gs) * d:(v % Gs + 1) * d]
+    H0 = _blocks(H, np.arange(N), d)
+    C_pre = np.stack([vec(W64, v, G) for v in _strata(M * G, 8, _seed(5, 1, 0))])
+    W_pre = np.concatenate([C_pre[[_nearest(vec(W64, i * G + g, G), C_pre, H0[g])
+                                   for i in range(M)]] for g in range(G)], axis=1)
+    perm = _importance_perm(W, W_pre, xsq)
+    Ws = W64[:, perm]
+    Hs = _blocks(H, perm, d)
+    C_b = np.stack([vec(Ws, v, G) for v in _strata(M * G, 8, _seed(5, 2, 0))])
+    code_b = np.array([[_nearest(vec(Ws, i * G + g, G), C_b, Hs[g]) for g in range(G)]
+                       for i in range(M)])
+    res = np.stack([vec(Ws, i * G + g, G) - C_b[code_b[i, g]] for i in range(M)
+                    for g in range(Gc)])               # critical residual, vector i * Gc + g
+    C_e, code_e = [], []
+    for t in (1, 2):
+        Ct = res[_strata(M * Gc, 4, _seed(5, 3, t))]
+        ct = np.array([_nearest(res[v], Ct, Hs[v % Gc]) for v in range(M * Gc)])
+        res = res - Ct[ct]
+        C_e.append(Ct)
+        code_e.append(ct.reshape(M, Gc))
+    np.testing.assert_array_equal(out["C_pre"], C_pre.astype(np.float32))
+    np.testing.assert_array_equal(out["perm"], perm)
+    cbs = out["codebooks"]
+    np.testing.assert_array_equal(cbs[0].C, C_b.astype(np.float32))
+    np.testing.assert_array_equal(cbs[0].codes, code_b)
+    for t in range(2):
+        np.testing.assert_allclose(cbs[t + 1].C, C_e[t], rtol=0, atol=1e-7)
+        np.testing.assert_array_equal(cbs[t + 1].codes, code_e[t])
+
+
+def test_schedule_with_a_codeword_per_vector_reconstructs_exactly():
+    """K_base equal to the number of vectors: the strata hold one vector each, so the base
+    k-means starts from every vector of the reordered W and the reconstruction is exact; the
+    extended codebooks then fit a zero residual. Every loss is zero and W_hat equals W."""
+    cfg = S.LayerConfig("pin_kall", 4, 32, 40, "outlier_cols", "lognormal", 0.5,
+                        n_outlier_cols=2, K_base=16, n_ext=1, K_ext=2, crit_frac=0.3, B=2,
+                        kmeans_iters=2, refine_rounds=1)
+    W, X = S.gen_W(cfg), S.gen_X(cfg)
+    out = O.quantize_layer(W, X, cfg)
+    assert out["loss_block"] == 0.0 and out["loss_crit"] == 0.0
+    assert abs(out["loss_full"]) <= 1e-12 * float((W.astype(np.float64) ** 2).sum())
+    np.testing.assert_array_equal(out["W_hat"], W)
+
+
+def test_schedule_puts_a_dominant_channel_first():
+    """One input channel whose weights and activations dwarf the rest has the largest App. A.2
+    importance, so the reorder puts it first and the critical set is ceil(lambda N / d) whole
+    groups."""
+    cfg = S.LayerConfig("pin_dom", 16, 64, 64, "plain", "lognormal", 0.3, K_base=4, n_ext=1,
+                        K_ext=2, crit_frac=0.05, B=2, kmeans_iters=2, refine_rounds=1)
+    W, X = S.gen_W(cfg), S.gen_X(cfg)
+    W[:, 37] *= 100.0
+    X[:, 37] *= 100.0
+    out = O.quantize_layer(W, X, cfg)
+    assert out["perm"][0] == 37
+    assert out["n_crit_groups"] == 1                   # ceil(0.05 * 64 / 8)
+    np.testing.assert_array_equal(np.sort(out["perm"]), np.arange(64))
+
+
 # ---------------------------------------------------------------- NEXT-1 coupled search
 def _coupled_case(seed, M=6, G=3, d=4, K=5, n=40):
     rng = np.random.default_rng(seed)
