@@ -1,22 +1,23 @@
 #!/usr/bin/env python
 """Benchmark of the CRVQ code-search hot path on GB300.
 
-A step is one weight matrix through the whole hot path (Alg. 1 from prequantization to the
-refinement loop: Hessian, prequantize, importance + reorder, base k-means, extended codebooks,
-least-squares refinement with beam re-encode, losses), i.e. one crvq_quantize_layer call, on
-the LLaMA-2-7B-shaped q_proj workload (W 4096 x 4096, 4096 calibration tokens, d = 8, K = 256,
-1 extended codebook on 2% channels, B = 8, 10 Lloyd iterations). The metric is code-search
-throughput: scored (hypothesis, codeword) pairs per second over the whole step; the per-layer
-time is reported beside it. `--config c5` makes a step the seven matrices of a LLaMA-2-7B
-decoder block (q, k, v, o, gate, up 4096-wide inputs sharing one X; down_proj 11008-wide with
-its own X), and reports the block time as well.
+A step is the whole hot path (Alg. 1 from prequantization to the refinement loop: Hessian,
+prequantize, importance + reorder, base k-means, extended codebooks, least-squares refinement
+with beam re-encode, losses) over one workload, through crvq_quantize_layer. The default
+workload is the largest one that fits a GPU: the seven matrices of a LLaMA-2-7B decoder block
+(q, k, v, o 4096 x 4096 and gate, up 11008 x 4096 sharing one 4096-token X; down 4096 x 11008
+with its own SwiGLU-like X; d = 8, K = 256, 2 extended codebooks on 2% channels, B = 8, 10
+Lloyd iterations). `--config c1..c4` runs a single matrix instead. The metric is code-search
+throughput: scored (hypothesis, codeword) pairs per second over the whole step; the per-step
+(block) time is reported beside it.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl crvq|reference] [--config c2]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl crvq|reference] [--config c5]
 
-With N > 1 (torchrun, one rank per GPU) every rank quantizes its own layer (independent
+With N > 1 (torchrun, one rank per GPU) every rank quantizes its own block (independent
 problems, no collective on the data path): weak scaling; value = all ranks' scores / the
-slowest rank's time. `--impl reference` times the fp64 CPU oracle on a bounded row sample of
-the same workload (the paper ships no code; the oracle is the reference arm).
+slowest rank's time. `--impl reference` times the fp64 CPU oracle on bounded row samples of
+the same workload on every host core (the paper ships no code; the oracle is the reference
+arm).
 """
 from __future__ import annotations
 
@@ -54,10 +55,16 @@ def schedule_scores(cfg, M, N):
     return float(s)
 
 
-# dram__bytes_read.sum + dram__bytes_write.sum of one arg-min launch (ncu --set full, a Lloyd
-# pass over the prequantize codebook of the c2 workload: 86.7 MB read + 4.8 MB written; set to None
-# whenever the kernel changes until the counters are taken again)
-ARGMIN_TRAFFIC = 91.48e6
+# dram__bytes_read.sum + dram__bytes_write.sum per arg-min launch, averaged over every
+# argmin_tc_kernel launch of one step of the workload (one ncu capture of the launch list with
+# the two DRAM counters; the summary is kept with the other profiles). None for a workload
+# whose counters have not been taken, and whenever the kernel changes until they are taken
+# again.
+ARGMIN_TRAFFIC = {}
+
+# The tf32 tensor rate relative to bf16 (nominal dense figures of the part: 1.1 vs 2.25
+# PFLOP/s). Only the bf16 rate is measured; the arg-min's MMAs are kind::tf32.
+TF32_PER_BF16 = 1.1 / 2.25
 
 
 def load_peaks():
@@ -172,6 +179,75 @@ def cpu_oracle_sample(cfg, X=None, budget_s=20.0, max_rows=64):
     return sc / wall, wall, max(1, int(round(cpu / max(wall, 1e-9)))), desc
 
 
+def _pool_init(cfg, threads_env):
+    os.environ.update(threads_env)
+    global _POOL_X
+    _POOL_X = S.gen_X(cfg)
+
+
+def _pool_job(cfg, r0, rows):
+    """One worker's sample: the whole schedule of the oracle on rows r0 .. r0 + rows - 1."""
+    from oracle import crvq_oracle as O
+    W = S.gen_W(cfg, np.arange(r0, r0 + rows))
+    t0 = time.perf_counter()
+    O.quantize_layer(W, _POOL_X, cfg)
+    return t0, time.perf_counter()
+
+
+class OraclePool:
+    """The fp64 oracle, as it stands, on every host core: one process per core (started with
+    spawn, so that it is safe after CUDA initialisation), each running the whole schedule on its
+    own block of rows of the workload's first matrix with the full X. Throughput = all samples'
+    scores / the wall time from the first start to the last end."""
+
+    def __init__(self, cfg, workers=None):
+        import multiprocessing as mp
+        from concurrent.futures import ProcessPoolExecutor
+        self.cfg = cfg
+        self.workers = workers or len(os.sched_getaffinity(0))
+        env = {k: "1" for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")}
+        self.ex = ProcessPoolExecutor(max_workers=self.workers,
+                                      mp_context=mp.get_context("spawn"),
+                                      initializer=_pool_init, initargs=(cfg, env))
+        list(self.ex.map(int, range(self.workers)))   # start the workers, build their X
+
+    def rows_for(self, budget_s):
+        cfg = self.cfg
+        need = rows_needed(cfg)
+        per_row = schedule_scores(cfg, 1, cfg.N)
+        rate = ORACLE_RATE_EST / 1.5                  # per process, every core busy
+        return min(cfg.M // self.workers, max(need, int(budget_s * rate / per_row)))
+
+    def run(self, budget_s):
+        rows = self.rows_for(budget_s)
+        futs = [self.ex.submit(_pool_job, self.cfg, w * rows, rows) for w in range(self.workers)]
+        spans = [f.result() for f in futs]
+        wall = max(b for _, b in spans) - min(a for a, _ in spans)
+        sc = self.workers * schedule_scores(self.cfg, rows, self.cfg.N)
+        desc = (f"whole schedule on {self.workers} row blocks of {rows} rows of {self.cfg.name} "
+                f"(full X), one process per host core")
+        return sc / wall, wall, self.workers, desc
+
+    def close(self):
+        self.ex.shutdown()
+
+
+def rows_needed(cfg):
+    """Rows a whole-schedule sample needs so that every codebook can draw its K vectors."""
+    G = cfg.N // cfg.d
+    Gc = min(G, int(np.ceil(np.float32(cfg.crit_frac) * cfg.N / cfg.d - 1e-12)))
+    return int(np.ceil(max(cfg.K_base / G, cfg.K_ext / Gc if cfg.n_ext > 0 else 0.0)))
+
+
+def pool_workers(cfg):
+    """Host cores the pool can use: one block of rows each, each block large enough for K
+    (0 or 1: run one process; a 65536-entry codebook needs 65536 vectors per sample)."""
+    need = rows_needed(cfg)
+    if need > 64:
+        return 0
+    return min(len(os.sched_getaffinity(0)), cfg.M // max(need, 1))
+
+
 def dist_init():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -203,21 +279,33 @@ def _cuda_ok():
 
 
 def run_reference(args, layers, ws, rank):
-    """Reference arm: the fp64 CPU oracle on a bounded sample of the workload's first matrix
-    (sized so the whole run stays within a few minutes), rank 0 only."""
+    """Reference arm: the fp64 CPU oracle on bounded samples of the workload's first matrix on
+    every host core (one process per core, each its own rows; sized so the whole run stays
+    within a few minutes), rank 0 only. Workloads whose codebook needs more rows than a sample
+    can hold (K = 65536) time one encode pass in one process instead."""
     if rank != 0:
         return
     cfg = layers[0]
-    X = S.gen_X(cfg)
     budget = min(20.0, max(2.0, 150.0 / max(1, args.steps + (args.warmup if args.ref_warmup
                                                               else 0))))
+    workers = pool_workers(cfg)
+    pool = OraclePool(cfg, workers) if workers > 1 else None
+    X = None if pool else S.gen_X(cfg)
+
+    def sample():
+        if pool:
+            return pool.run(budget)
+        return cpu_oracle_sample(cfg, X, budget, args.ref_rows)
+
     for _ in range(args.warmup if args.ref_warmup else 0):
-        cpu_oracle_sample(cfg, X, budget, args.ref_rows)
+        sample()
     tot, sc_tot, cores, desc = 0.0, 0.0, 1, ""
     for _ in range(args.steps):
-        v, wall, cores, desc = cpu_oracle_sample(cfg, X, budget, args.ref_rows)
+        v, wall, cores, desc = sample()
         tot += wall
         sc_tot += v * wall
+    if pool:
+        pool.close()
     value = sc_tot / tot
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": "scores/s",
@@ -272,10 +360,10 @@ def workload_layers(name):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="crvq", choices=["crvq", "reference"])
-    ap.add_argument("--config", default="c2", choices=sorted(S.CONFIGS) + ["c5"])
+    ap.add_argument("--config", default="c5", choices=sorted(S.CONFIGS) + ["c5"])
     ap.add_argument("--ref-rows", type=int, default=64,
                     help="most rows a whole-schedule oracle sample takes beyond what K needs")
     ap.add_argument("--ref-warmup", action="store_true")
@@ -408,31 +496,39 @@ def main():
     nsm = props.multi_processor_count
     ks = sorted(kstats, key=lambda k: -k["ms"])
     total_k = sum(k["ms"] for k in ks) or 1.0
-    # The dominant kernel is the tensor-core arg-min: tcgen05 computes every certified score
-    # bound (a 3xTF32 dot product of length 32), and its epilogue keeps the two smallest of
-    # each row with four integer ALU operations per score (key packing, min, max, min). The
-    # ALU pipe (64 lanes per SM per clock on sm_103) is the binding unit; the roofline is
-    # those ALU operations against that pipe, timed over the timed region's arg-min launches.
-    mhz = peaks.get("sm_max_mhz", 2070.0)
-    alu_peak = nsm * 64 * mhz * 1e6 / 1e12
+    # The dominant kernel is the tensor-core arg-min (argmin_tc_kernel): tcgen05 computes the
+    # certified lower bound of every (vector, codeword) score as a 3xTF32 dot product of length
+    # 32 (64 tf32 flop issued per score), and its epilogue keeps the two smallest of each row.
+    # The roofline is the score contraction's algorithmic work, 2 d = 16 flop per score, against
+    # the tf32 tensor peak (the measured bf16 rate scaled by the nominal tf32 / bf16 ratio; the
+    # sustained figure, since the kernel is timed inside a long step). The issued-flop fraction
+    # and the integer ALU pipe that binds the epilogue are reported beside it.
     enc_ms = sum(k["ms"] for k in argmin_stats)
     enc_units = sum(k["units"] for k in argmin_stats)
     enc_launches = sum(k["launches"] for k in argmin_stats)
-    achieved = enc_units * 4.0 / (enc_ms / 1e3) / 1e12 if enc_ms > 0 else 0.0
-    tf32_peak = 0.5 * peaks.get("bf16_tflops", 1900.0)
-    tensor_tflops = enc_units * 64.0 / (enc_ms / 1e3) / 1e12 if enc_ms > 0 else 0.0
-    roof = {"kernel": "encode_argmin (all passes)", "bound": "alu", "achieved": achieved,
-            "peak": alu_peak, "unit": "TOP/s", "frac": achieved / alu_peak,
-            "traffic": ARGMIN_TRAFFIC if args.config == "c2" else None,
-            "peak_source": f"{nsm} SMs x 64 ALU lanes x {mhz:.0f} MHz (sm_max_mhz, {peak_src})",
-            "work": "4 integer ALU ops per scored (vector, codeword) pair",
+    sec = enc_ms / 1e3 if enc_ms > 0 else float("inf")
+    bf16 = peaks.get("bf16_tflops_sustained", peaks.get("bf16_tflops", 1700.0))
+    tf32_peak = TF32_PER_BF16 * bf16
+    alg_tflops = enc_units * 16.0 / sec / 1e12
+    issued_tflops = enc_units * 64.0 / sec / 1e12
+    mhz = peaks.get("sm_max_mhz", 2070.0)
+    alu_peak = nsm * 64 * mhz * 1e6 / 1e12
+    alu_achieved = enc_units * 4.0 / sec / 1e12
+    traffic = ARGMIN_TRAFFIC.get(args.config)
+    roof = {"kernel": "argmin_tc_kernel (tensor-core arg-min, all passes of the step)",
+            "bound": "tensor", "achieved": alg_tflops, "peak": tf32_peak, "unit": "TFLOP/s",
+            "frac": alg_tflops / tf32_peak, "traffic": traffic,
+            "work": "2 d = 16 flop per scored (vector, codeword) pair (the score contraction)",
+            "peak_source": (f"tf32 = {TF32_PER_BF16:.4f} x bf16 sustained {bf16} TFLOP/s "
+                            f"({peak_src}, MEASURED_PEAKS.json) of measured"),
             "avg_launch_ms": enc_ms / max(enc_launches, 1), "launches": enc_launches,
-            "tensor": {"achieved": tensor_tflops, "unit": "TFLOP/s",
-                       "peak": tf32_peak, "frac": tensor_tflops / tf32_peak,
-                       "work": "64 tf32 flop per scored pair issued (K = 32 split operands)",
-                       "algorithmic_frac": tensor_tflops / 4.0 / tf32_peak,
-                       "algorithmic_work": "2 d = 16 flop per scored pair",
-                       "peak_source": f"0.5 x bf16 {peak_src} ({peaks.get('bf16_tflops')})"}}
+            "scores_per_launch": enc_units / max(enc_launches, 1),
+            "issued": {"achieved": issued_tflops, "frac": issued_tflops / tf32_peak,
+                       "work": "64 tf32 flop per scored pair issued (K = 32 split operands)"},
+            "alu": {"achieved": alu_achieved, "peak": alu_peak, "unit": "TOP/s",
+                    "frac": alu_achieved / alu_peak,
+                    "work": "4 integer ALU ops per scored pair (key packing, min, max, min)",
+                    "peak_source": f"{nsm} SMs x 64 ALU lanes x {mhz:.0f} MHz"}}
     last = work[-1]["out"].report if len(work) == 1 else None
     line = {
         "metric": METRIC, "value": value, "unit": "scores/s", "n_gpus": ws,
@@ -458,9 +554,19 @@ def main():
                           for w in work}
     if ws == 1 and not args.no_cpu_baseline:
         w0 = work[0]
-        v, wall, cores, desc = cpu_oracle_sample(w0["cfg"], w0["Xn"], 20.0, args.ref_rows)
-        line["cpu_baseline"] = {"value": v, "unit": "scores/s", "cores": cores, "kind": "oracle",
-                                "sample": f"{desc}, {wall:.1f} s"}
+        v1, wall1, cores1, desc1 = cpu_oracle_sample(w0["cfg"], w0["Xn"], 20.0, args.ref_rows)
+        one = {"value": v1, "unit": "scores/s", "cores": cores1, "kind": "oracle",
+               "sample": f"{desc1}, {wall1:.1f} s"}
+        workers = pool_workers(w0["cfg"])
+        if workers > 1:
+            pool = OraclePool(w0["cfg"], workers)
+            v, wall, cores, desc = pool.run(15.0)
+            pool.close()
+            line["cpu_baseline"] = {"value": v, "unit": "scores/s", "cores": cores,
+                                    "kind": "oracle", "sample": f"{desc}, {wall:.1f} s",
+                                    "one_core": one}
+        else:
+            line["cpu_baseline"] = one
     print(json.dumps(line), flush=True)
 
 

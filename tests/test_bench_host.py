@@ -31,3 +31,22 @@ def test_schedule_scores_counts_what_the_schedule_scores(monkeypatch):
     monkeypatch.setattr(O, "encode_beam", counting)
     O.quantize_layer(S.gen_W(cfg), S.gen_X(cfg), cfg)
     assert sum(counted) == bench.schedule_scores(cfg, cfg.M, cfg.N)
+
+
+def test_oracle_pool_runs_one_sample_per_core_and_counts_their_scores():
+    """The all-cores CPU baseline: worker processes (spawn) each run the oracle's whole
+    schedule on their own rows; the rate counts every worker's scores over the common span."""
+    import bench
+    import synthetic as S
+    cfg = S.LayerConfig("pool", 32, 64, 32, "plain", "lognormal", 0.5, K_base=8, n_ext=1,
+                        K_ext=4, crit_frac=0.1, B=2, kmeans_iters=1)
+    assert bench.rows_needed(cfg) == 4                   # K_ext = 4 over one critical group
+    pool = bench.OraclePool(cfg, 2)
+    try:
+        rate, wall, cores, desc = pool.run(0.05)
+    finally:
+        pool.close()
+    rows = pool.rows_for(0.05)
+    assert cores == 2 and wall > 0
+    assert abs(rate * wall - 2 * bench.schedule_scores(cfg, rows, cfg.N)) <= 1e-6 * rate * wall
+    assert "2 row blocks" in desc
