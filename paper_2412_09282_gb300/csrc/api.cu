@@ -571,23 +571,29 @@ uint64_t phase_seed(uint64_t seed, int phase, int cb) {
 
 // Lloyd iterations for the last codebook of `cbs` (all earlier ones fixed), then a final
 // encode: T x (encode, LS update) + encode. Each encode accumulates the least-squares
-// statistics of the codes it writes, so the update is only the per-codeword solve.
+// statistics of the codes it writes, so the update is only the per-codeword solve, which
+// also clears the statistics it read. One scratch serves every pass, so an iteration is
+// kernels only (no allocation or memset between them in the stream).
 crvq_status lloyd(const SetView& set, CbList cbs, int iters, const EncodeExtras& ex0,
                   cudaStream_t s) {
   const int j = cbs.n - 1;
   float* C = const_cast<float*>(cbs.cb[j].C);
-  Scratch mem;
+  Scratch mem, wmem;
   StatsView st;
   CRVQ_TRY(stats_alloc(mem, cbs.cb[j].G_cov, cbs.cb[j].K, &st, s));
   CRVQ_TRY(launch_stats_prepare(set, cbs, j, st, s));  // T, H and fixed codebooks stay put
+  const size_t wbytes = argmin_scratch_bytes(set.M, cbs.cb[j].G_cov, cbs.cb[j].K);
+  CRVQ_TRY(wmem.alloc(wbytes, s));
   EncodeExtras ex = ex0;
+  ex.work = wmem.as<char>();
+  ex.work_bytes = wbytes;
+  EncodeExtras ex_last = ex;
   ex.stats = &st;
   for (int it = 0; it < iters; ++it) {
-    if (it > 0) CRVQ_TRY(stats_zero(st, s));
     CRVQ_TRY(launch_encode_beam(set, cbs, j, 1, false, nullptr, ex, s));
     CRVQ_TRY(launch_stats_solve(set, st, C, C, nullptr, s));
   }
-  return launch_encode_beam(set, cbs, j, 1, false, nullptr, ex0, s);
+  return launch_encode_beam(set, cbs, j, 1, false, nullptr, ex_last, s);
 }
 
 template <class T>

@@ -329,6 +329,7 @@ __device__ void cbmax_block(const float* __restrict__ C, int K, float* __restric
   }
 }
 
+constexpr uint32_t kKeyMask = 0xffffffe0u;       // value bits of a packed arg-min key
 constexpr int kTcCols = 128;                     // codewords per chunk (MMA N)
 constexpr int kTcBTile = kTcCols * tcenc::kK * 4;  // 16 KB
 
@@ -338,9 +339,12 @@ constexpr int kTcBTile = kTcCols * tcenc::kK * 4;  // 16 KB
 __global__ void __launch_bounds__(128)
 prep_b_kernel(SetView set, int64_t g_begin, int64_t G_range, const float* __restrict__ C,
               int K, int nchunk, float uc, char* __restrict__ out, float4* __restrict__ terms,
-              float* __restrict__ cbmax) {
+              float* __restrict__ cbmax, unsigned* __restrict__ flag_count) {
   pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
   pdl_wait();
+  // The flag list of the arg-min pass that follows starts empty. The previous pass's exact
+  // kernel, which read the count, completed before the wait above returned.
+  if (blockIdx.x == 0 && threadIdx.x == 0) *flag_count = 0u;
   if (blockIdx.x == gridDim.x - 1) {  // the last CTA: the codebook maxima
     cbmax_block(C, K, cbmax);
     return;
@@ -464,6 +468,29 @@ __device__ __forceinline__ bool less(float ah, float al, int ak, float bh, float
 // and flushed once.
 constexpr int kTcSmemStatsK = 256;  // codebooks up to this size aggregate statistics in smem
 
+// Key of a non-negative fp32 value v (its bit pattern) with column j < 32 in the low 5 bits:
+// (v & ~31) | j. `mask` = ~31 arrives as a kernel argument so that the compiler cannot fold
+// it: with the mask and the column both immediates the operation takes two ALU instructions.
+#ifndef CRVQ_KEYPACK
+#define CRVQ_KEYPACK 1
+#endif
+__device__ __forceinline__ uint32_t pack_key(uint32_t v, uint32_t j, uint32_t mask,
+                                             uint32_t m27, uint32_t m32) {
+#if CRVQ_KEYPACK == 0
+  return (v & 0xffffffe0u) | j;
+#elif CRVQ_KEYPACK == 1
+  uint32_t k;  // one three-input logic operation: (v & mask) | j
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(k) : "r"(v), "r"(mask), "r"(j));
+  return k;
+#else
+  // on the integer multiply-add path instead of the logic unit: (v >> 5) * 32 + j, with
+  // v >> 5 = the high word of v * 2^27 (m27 = 2^27 and m32 = 32, both from `mask`)
+  uint32_t hi;
+  asm("mul.hi.u32 %0, %1, %2;" : "=r"(hi) : "r"(v), "r"(m27));
+  return hi * m32 + j;
+#endif
+}
+
 // dynamic shared memory of argmin_tc_kernel<HALVES>: A tiles, two B chunks, statistics, H r,
 // alignment
 constexpr size_t argmin_smem(int halves) {
@@ -500,10 +527,11 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
                  int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
                  FlagList flags, StatsView st, const float* __restrict__ cbmax,
                  const char* __restrict__ bpre, const float4* __restrict__ terms, int tiles,
-                 unsigned* err) {
+                 uint32_t key_mask, unsigned* err) {
   pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
   pdl_wait();
   using namespace tcenc;
+  const uint32_t m32 = ~key_mask + 1u, m27 = m32 << 22;  // 32 and 2^27 for pack_key
   extern __shared__ __align__(1024) char smem_raw[];
   // 1024-byte aligned base, derived from the shared array (keeps the shared address space)
   char* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -691,8 +719,8 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
         const uint32_t* v1 = v + 32;
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
-          const uint32_t k0 = (v0[j] & 0xffffffe0u) | (uint32_t)j;
-          const uint32_t k1 = (v1[j] & 0xffffffe0u) | (uint32_t)j;
+          const uint32_t k0 = pack_key(v0[j], (uint32_t)j, key_mask, m27, m32);
+          const uint32_t k1 = pack_key(v1[j], (uint32_t)j, key_mask, m27, m32);
           const uint32_t h0 = max(a1[2 * rnd], k0), h1 = max(a1[2 * rnd + 1], k1);
           a1[2 * rnd] = min(a1[2 * rnd], k0);
           a1[2 * rnd + 1] = min(a1[2 * rnd + 1], k1);
@@ -1627,6 +1655,27 @@ crvq_status launch_beam_stage(const SetView& set, int64_t g_begin, int64_t G_ran
   return launch_beam_stage_L<17>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
 }
 
+// Scratch of one arg-min pass: codebook maxima (256 B) | B images of G_sub groups (groups
+// in sub-ranges whose images take at most 256 MB) | codeword terms | flag count (256 B) |
+// flag list (vector ids and thresholds).
+struct ArgminLayout {
+  int nchunk;
+  int64_t G_sub;
+  size_t bbytes, tbytes, fbytes, total;
+};
+
+ArgminLayout argmin_layout(int64_t M, int64_t G_range, int K) {
+  ArgminLayout L;
+  L.nchunk = (int)ceil_div(K, kTcCols);
+  const int64_t per_group = (int64_t)L.nchunk * kTcBTile;
+  L.G_sub = std::max<int64_t>(1, std::min<int64_t>(G_range, (int64_t(256) << 20) / per_group));
+  L.bbytes = (size_t)L.G_sub * per_group;
+  L.tbytes = align_up((size_t)L.G_sub * K * sizeof(float4), 256);
+  L.fbytes = align_up((size_t)M * L.G_sub * (sizeof(int64_t) + sizeof(float)), 256);
+  L.total = 256 + L.bbytes + L.tbytes + 256 + L.fbytes;
+  return L;
+}
+
 // One range of groups [g_begin, g_begin + G_range) whose searched stages are sd.st[0..S).
 crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
                          const CbList& cbs, int n_fixed, StageDesc sd, bool keep_if_better,
@@ -1664,21 +1713,22 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
     // Groups in sub-ranges whose B images (the codebook's tensor-core operand per group) take
     // at most 256 MB; per sub-range: images + per-group codeword terms (prep_b, which also
     // writes the codebook maxima), the arg-min pass, and the exact decision of flagged rows.
-    const int nchunk = (int)ceil_div(cw.K, kTcCols);
-    const int64_t per_group = (int64_t)nchunk * kTcBTile;
-    const int64_t G_sub = std::max<int64_t>(1, std::min<int64_t>(G_range, (int64_t(256) << 20) /
-                                                                              per_group));
-    const size_t bbytes = (size_t)G_sub * per_group;
-    const size_t tbytes = align_up((size_t)G_sub * cw.K * sizeof(float4), 256);
-    const size_t fbytes = align_up((size_t)set.M * G_sub * (sizeof(int64_t) + sizeof(float)), 256);
+    const ArgminLayout AL = argmin_layout(set.M, G_range, cw.K);
+    const int nchunk = AL.nchunk;
+    const int64_t G_sub = AL.G_sub;
+    const size_t bbytes = AL.bbytes, tbytes = AL.tbytes;
     Scratch bmem;
-    CRVQ_TRY(bmem.alloc(256 + bbytes + tbytes + 256 + fbytes, stream));
-    float* cbmax = bmem.as<float>();
-    char* bimg = bmem.as<char>() + 256;
+    char* wbase = ex.work;
+    if (!wbase || ex.work_bytes < AL.total) {
+      CRVQ_TRY(bmem.alloc(AL.total, stream));
+      wbase = bmem.as<char>();
+    }
+    float* cbmax = reinterpret_cast<float*>(wbase);
+    char* bimg = wbase + 256;
     float4* tout = reinterpret_cast<float4*>(bimg + bbytes);
     FlagList fl;
-    fl.count = reinterpret_cast<unsigned*>(bmem.as<char>() + 256 + bbytes + tbytes);
-    fl.vec = reinterpret_cast<int64_t*>(bmem.as<char>() + 256 + bbytes + tbytes + 256);
+    fl.count = reinterpret_cast<unsigned*>(wbase + 256 + bbytes + tbytes);
+    fl.vec = reinterpret_cast<int64_t*>(wbase + 256 + bbytes + tbytes + 256);
     fl.cap = set.M * G_sub;
     fl.thr = reinterpret_cast<float*>(fl.vec + fl.cap);
     fl.total = ex.flag_total;
@@ -1691,15 +1741,14 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
       const int64_t gn = std::min<int64_t>(G_sub, g_begin + G_range - gs);
       const int64_t nv = set.M * gn;
       fl.cap = nv;
-      fl.thr = reinterpret_cast<float*>(fl.vec + nv);
-      CRVQ_CUDA(cudaMemsetAsync(fl.count, 0, sizeof(unsigned), stream));
+      fl.thr = reinterpret_cast<float*>(fl.vec + nv);  // the count is cleared by prep_b
       {
         ProfScope pb("encode_prep_b", stream, (double)gn * nchunk * kTcCols);
         const int64_t rows = gn * nchunk * kTcCols;
         CRVQ_CUDA(launch_pdl(prep_b_kernel,
                              dim3((unsigned)std::min<int64_t>(ceil_div(rows, 128), 16 * nsm) + 1),
                              dim3(128), 0, stream, set, gs, gn, cw.C, cw.K, nchunk, uc, bimg,
-                             tout, cbmax));
+                             tout, cbmax, fl.count));
         CRVQ_LAUNCHED();
       }
       {
@@ -1719,11 +1768,11 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
         if (two_halves)
           CRVQ_CUDA(launch_pdl(argmin_tc_kernel<2>, grid, dim3(256), argmin_smem(2), stream, set,
                                gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax,
-                               bimg, tout, tiles, err));
+                               bimg, tout, tiles, kKeyMask, err));
         else
           CRVQ_CUDA(launch_pdl(argmin_tc_kernel<1>, grid, dim3(128), argmin_smem(1), stream, set,
                                gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax,
-                               bimg, tout, tiles, err));
+                               bimg, tout, tiles, kKeyMask, err));
         CRVQ_LAUNCHED();
       }
       {
@@ -1815,6 +1864,10 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
 }
 
 }  // namespace
+
+size_t argmin_scratch_bytes(int64_t M, int64_t G_range, int K) {
+  return argmin_layout(M, G_range, K).total;
+}
 
 crvq_status launch_encode_beam(const SetView& set, const CbList& cbs, int n_fixed, int B,
                                bool keep_if_better, float* vec_err, const EncodeExtras& ex,

@@ -62,7 +62,15 @@ struct EncodeExtras {
   double* scores = nullptr;                // host: += (hypothesis, codeword) pairs scored
   const StatsView* stats = nullptr;        // accumulate LS statistics of the written codes
   unsigned long long* flag_total = nullptr;  // device: += vectors sent to the fp64 fallback
+  // Scratch of the arg-min pass provided by the caller (e.g. once for a whole Lloyd loop, so
+  // that its iterations allocate nothing); used when at least argmin_scratch_bytes long.
+  char* work = nullptr;
+  size_t work_bytes = 0;
 };
+
+// Scratch of one arg-min pass over a set of M rows and G_range groups with a K-entry codebook
+// (B images, codeword terms, codebook maxima, flag list).
+size_t argmin_scratch_bytes(int64_t M, int64_t G_range, int K);
 
 // Encode / beam (see crvq_encode_beam).
 crvq_status launch_encode_beam(const SetView& set, const CbList& cbs, int n_fixed, int B,

@@ -158,6 +158,8 @@ crvq_status stats_zero(const StatsView& st, cudaStream_t s);
 // Computes the fixed-point scale for accumulating codebook `which` over `set`.
 crvq_status launch_stats_prepare(const SetView& set, const CbList& cbs, int which,
                                  const StatsView& st, cudaStream_t stream);
+// Solves every codeword from the statistics and leaves cnt and bacc zero (each is cleared
+// once read), ready for the next accumulation.
 crvq_status launch_stats_solve(const SetView& set, const StatsView& st, const float* C_old,
                                float* C_out, int32_t* counts, cudaStream_t stream);
 

@@ -336,6 +336,13 @@ stats_solve_kernel(const float* __restrict__ Hb, StatsView st, const float* C_ol
   part_h[kk][sl][e] = hi;
   part_l[kk][sl][e] = lo;
   __syncthreads();
+  // Every thread of the codeword has read its counts: clear them, so that the statistics are
+  // zero for the next accumulation (the Lloyd loop needs no memset between iterations).
+  if (e == 0 && k < K) {
+    const int64_t gper = (st.G_cov + kSolveSlices - 1) / kSolveSlices;
+    const int64_t g0 = sl * gper, g1 = min(st.G_cov, g0 + gper);
+    for (int64_t gq = g0; gq < g1; ++gq) st.cnt[gq * K + k] = 0;
+  }
   if (sl == 0 && k < K) {
     float h = part_h[kk][0][e], l = part_l[kk][0][e];
     for (int s2 = 1; s2 < kSolveSlices; ++s2) {
@@ -363,6 +370,8 @@ stats_solve_kernel(const float* __restrict__ Hb, StatsView st, const float* C_ol
     float bh[kD], bl[kD];
 #pragma unroll
     for (int j = 0; j < kD; ++j) fixed_to_pair(st.bacc[(int64_t)k * kD + j], sexp, bh[j], bl[j]);
+#pragma unroll
+    for (int j = 0; j < kD; ++j) st.bacc[(int64_t)k * kD + j] = 0;  // read: clear (see above)
     if (!solve8_pairs(Ah, Al, bh, bl, out)) {
       // no fp32 factor (cond(A) beyond fp32): the fp64 Cholesky solve
       double A[36], b[kD], x[kD];

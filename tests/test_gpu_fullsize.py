@@ -1,16 +1,24 @@
-"""Full-size workloads through the C ABI: the layer configurations of the benchmark and the
-larger LLaMA-shaped cases (4096x4096 q_proj; 4096x11008 down_proj with a 65536-entry base
-codebook; 28672x8192 up_proj with four extended codebooks), in the launch configuration the
-benchmark times. The fp64 oracle cannot run them whole, so outputs are checked on sampled
-vectors it decides one by one, and by properties that hold at any size:
+"""Full-size workloads through the C ABI, in the launch configuration the benchmark times: the
+4096x4096 q_proj (c2); the 4096x11008 down_proj with a 65536-entry base codebook (c3); the
+28672x8192 up_proj with four extended codebooks (c4); and the three distinct matrix shapes of
+the LLaMA-2-7B decoder block (c5: q_proj 4096x4096, gate_proj 11008x4096, whose 11008 rows are
+not a multiple of a CTA's row span, and down_proj 4096x11008 with two extended codebooks on 28
+critical groups).
 
-- the permutation is a bijection that sorts the importance (descending, ties by index);
-- a non-critical vector's final base code is the fp64 arg-min under the final codebook (the
-  last step of the schedule is that encode), except at fp64-level near-ties;
-- a critical vector's final tuple is no worse than the oracle's own stage-wise beam on that
-  vector (keep-if-better may keep an older, better tuple);
-- sampled rows of the reconstruction equal the sum of their codewords, bit for bit;
-- one full-size encode pass with K = 65536 returns the fp64 arg-min and its err.
+The fp64 oracle cannot run a whole schedule at these sizes, so each step is checked on the
+GPU's own full-size state (stepwise parity, the same gate as the small cases):
+- the final losses (loss_block, loss_crit, loss_full; Alg. 1 QuantLoss) against the oracle's
+  reconstruct_error of the GPU's final codebooks and codes, within 1e-4 relative;
+- one least-squares update of every codebook (Sec. 3.1 Eq. kmeans; Alg. 1 FineTuneCodebook)
+  from the final state, within 1e-4 of each codebook's largest value;
+- the arg-min encode over every row of 8 whole non-critical group columns, and the stage-wise
+  beam over every row of 2 critical group columns (Sec. 3.1 Eq. (2)-(3); Alg. 1
+  BeamSearchOptimize): codes equal the oracle's except at fp64 near-ties;
+- sampled vectors of the final codes (non-critical: the fp64 arg-min; critical: no worse than
+  the oracle's beam, since keep-if-better may keep an older, better tuple) and reconstruction
+  rows, bit for bit;
+- one full-size encode pass and one least-squares update with K = 65536 (c3).
+Hessian blocks are taken from the oracle's own H (O.hessian) in the GPU's channel order.
 """
 import numpy as np
 import pytest
@@ -18,25 +26,47 @@ import torch
 
 import synthetic as S
 from oracle import crvq_oracle as O
-from parity_util import REL_TIE, dev, host
+from parity_util import (REL_TIE, beam_boundary_gap, check_codes_with_ties, dev, host,
+                         oracle_cbs)
 
 pytestmark = pytest.mark.gpu
 
 D = 8
 
+CASES = {"c2": S.C2, "c3": S.C3, "c4": S.C4, "c5_q_proj": S.C5[0], "c5_gate_proj": S.C5[4],
+         "c5_down_proj": S.C5[6]}
+_RUNS = {}
 
-def _sorted_blocks(X, perm, groups, damp_rel):
-    """fp32 H blocks (as the oracle rounds them) of the sorted channel groups, from X in fp64."""
-    Xd = np.asarray(X, dtype=np.float64)
-    n = Xd.shape[0]
-    xsq = np.einsum("kj,kj->j", Xd, Xd) / n
-    delta = float(np.float32(damp_rel)) * xsq.mean()
-    out = {}
-    for g in groups:
-        cols = perm[g * D:(g + 1) * D]
-        Xg = Xd[:, cols]
-        out[g] = ((Xg.T @ Xg) / n + delta * np.eye(D)).astype(np.float32).astype(np.float64)
-    return out
+
+def _layer(name):
+    """The layer quantized once per module on the GPU, with the oracle's H for its X."""
+    if name not in _RUNS:
+        import paper_2412_09282_gb300 as P
+        cfg = CASES[name]
+        W, X = S.gen_W(cfg), S.gen_X(cfg)
+        out = P.crvq_quantize_layer(dev(W), dev(X), cfg)
+        P.crvq_sync()
+        H, _, _, delta = O.hessian(X, cfg.damp_rel, D)
+        perm = host(out.perm).astype(np.int64)
+        G = cfg.N // D
+        Hb = np.stack([H[np.ix_(perm[g * D:(g + 1) * D], perm[g * D:(g + 1) * D])]
+                       for g in range(G)])
+        _RUNS.clear()                                 # keep one layer's state at a time
+        _RUNS[name] = dict(cfg=cfg, W=W, X=X, out=out, H=H, delta=float(delta), perm=perm,
+                           Hb=Hb, Ws=np.ascontiguousarray(W[:, perm]))
+    return _RUNS[name]
+
+
+def _gpu_cbs(r, rows=slice(None)):
+    """The GPU's final codebooks as binding Codebooks (codes on the device) for rows `rows`."""
+    from paper_2412_09282_gb300 import Codebook
+    cfg, out = r["cfg"], r["out"]
+    G = cfg.N // D
+    Gc = out.report["n_crit_groups"]
+    cbs = [Codebook(out.C_base, out.codes_base[rows], G)]
+    for t in range(cfg.n_ext):
+        cbs.append(Codebook(out.C_ext[t].contiguous(), out.codes_ext[t][rows], Gc))
+    return cbs
 
 
 def _err(t, C, H):
@@ -44,13 +74,21 @@ def _err(t, C, H):
     return np.einsum("kd,kd->k", Dl @ H, Dl)
 
 
-@pytest.mark.parametrize("name", ["c2", "c3", "c4"])
-def test_full_size_layer_sampled_parity(name):
-    import paper_2412_09282_gb300 as P
-    cfg = S.CONFIGS[name]
-    W, X = S.gen_W(cfg), S.gen_X(cfg)
-    out = P.crvq_quantize_layer(dev(W), dev(X), cfg)
-    torch.cuda.synchronize()
+def _cmp_codebook(Cg, Co, tol=1e-4):
+    err = np.abs(Cg.astype(np.float64) - Co).max() / max(np.abs(Co).max(), 1e-30)
+    assert err <= tol, f"codebook rel err {err}"
+
+
+@pytest.mark.parametrize("name", list(CASES))
+def test_full_size_layer_parity(name):
+    """Sampled checks of the final outputs, then the stepwise checks on the GPU's state."""
+    r = _layer(name)
+    _sampled_checks(r)
+    _stepwise_checks(r, encode=r["cfg"].K_base <= 4096)
+
+
+def _sampled_checks(r):
+    cfg, out, W, Ws, Hb, perm = r["cfg"], r["out"], r["W"], r["Ws"], r["Hb"], r["perm"]
     M, N = W.shape
     G = N // D
     Gc = out.report["n_crit_groups"]
@@ -60,7 +98,6 @@ def test_full_size_layer_sampled_parity(name):
         assert np.isfinite(rep[k]) and rep[k] >= 0, k
     assert rep["loss_crit"] <= rep["loss_block"]
 
-    perm = host(out.perm).astype(np.int64)
     imp = host(out.importance).astype(np.float64)
     np.testing.assert_array_equal(np.sort(perm), np.arange(N))
     s = imp[perm]
@@ -70,8 +107,6 @@ def test_full_size_layer_sampled_parity(name):
     rows = np.sort(rng.choice(M, 6, replace=False))
     groups_nc = np.sort(rng.choice(np.arange(Gc, G), 24, replace=False))
     groups_c = np.arange(min(Gc, 6))
-    Hs = _sorted_blocks(X, perm, list(groups_nc) + list(groups_c), cfg.damp_rel)
-    Ws = W[:, perm]
     C_base = host(out.C_base)
     codes_base = host(out.codes_base)
     C_ext = [host(out.C_ext[t]) for t in range(cfg.n_ext)]
@@ -80,24 +115,25 @@ def test_full_size_layer_sampled_parity(name):
     bad = []
     for i in rows:
         for g in groups_nc:
+            H = Hb[g].astype(np.float64)
             t = Ws[i, g * D:(g + 1) * D].astype(np.float64)
-            e = _err(t, C_base, Hs[g])
+            e = _err(t, C_base, H)
             kg = int(codes_base[i, g])
             if kg != int(np.argmin(e)):
-                tt = float(t @ Hs[g] @ t)
+                tt = float(t @ H @ t)
                 if e[kg] - e.min() > REL_TIE * (e.min() + tt):
                     bad.append(("base", int(i), int(g), kg, int(np.argmin(e))))
         for g in groups_c:
-            t = Ws[i, g * D:(g + 1) * D].astype(np.float32)
+            H = Hb[g].astype(np.float64)
+            t = Ws[i, g * D:(g + 1) * D]
             cbs = [O.Codebook(C_base, None, 1)] + [O.Codebook(C, None, 1) for C in C_ext]
-            codes, verr = O.encode_beam(t[None, :], D, Hs[g][None].astype(np.float32), cbs, 0,
-                                        cfg.B)
-            r = t.astype(np.float64) - C_base[codes_base[i, g]]
+            codes, verr = O.encode_beam(t[None, :], D, Hb[g][None], cbs, 0, cfg.B)
+            rr = t.astype(np.float64) - C_base[codes_base[i, g]]
             for q in range(cfg.n_ext):
-                r = r - C_ext[q][codes_ext[q][i, g]]
-            e_gpu = float(r @ Hs[g] @ r)
+                rr = rr - C_ext[q][codes_ext[q][i, g]]
+            e_gpu = float(rr @ H @ rr)
             e_beam = float(verr[0, 0])
-            tt = float(t.astype(np.float64) @ Hs[g] @ t.astype(np.float64))
+            tt = float(t.astype(np.float64) @ H @ t.astype(np.float64))
             if e_gpu > e_beam + REL_TIE * (e_beam + tt):
                 bad.append(("beam", int(i), int(g), e_gpu, e_beam))
     assert not bad, bad[:5]
@@ -113,9 +149,82 @@ def test_full_size_layer_sampled_parity(name):
         np.testing.assert_array_equal(W_hat[i], want)
 
 
-def test_full_size_encode_pass_k65536_sampled():
+def _stepwise_checks(r, encode):
+    """Losses, least-squares updates and encodes on the GPU's final full-size state, each
+    against the oracle given the same inputs. The 28672-row up_proj (c4) takes its updates and
+    encodes on a 4096-row block (a vector set of its own); its losses are over the whole
+    matrix. With a 65536-entry base codebook (c3) the whole-column encodes are left to the
+    sampled K = 65536 test (the oracle's dense scoring of 4096 x 65536 pairs per group is too
+    slow here)."""
+    import paper_2412_09282_gb300 as P
+    from paper_2412_09282_gb300 import Codebook
+    cfg, out, Ws, Hb, X = r["cfg"], r["out"], r["Ws"], r["Hb"], r["X"]
+    M, N = Ws.shape
+    G = N // D
+    Gc = out.report["n_crit_groups"]
+    n_cb = 1 + cfg.n_ext
+
+    # S7 losses of the final state, whole matrix
+    ocbs = oracle_cbs(_gpu_cbs(r))
+    _, lb, lc, lf = O.reconstruct_error(Ws, D, Hb, r["perm"], ocbs, Gc, X, r["delta"])
+    rep = out.report
+    assert abs(rep["loss_block"] - lb) <= 1e-4 * lb
+    assert abs(rep["loss_crit"] - lc) <= 1e-4 * lc
+    assert abs(rep["loss_full"] - lf) <= 1e-4 * lf
+
+    # least-squares update of every codebook from the final state (a row block for c4)
+    rb = slice(0, min(M, 4096))
+    Ws_d = dev(Ws)
+    T = Ws_d[rb]
+    Hb_d = dev(Hb)
+    cbs = _gpu_cbs(r, rb)
+    ocbs = oracle_cbs(cbs)
+    Ws_rb = Ws[rb]
+    for j in range(n_cb):
+        Cg, cnt = P.crvq_update_codebook(T, D, Hb_d, cbs, j)
+        P.crvq_sync()
+        Co, co = O.update_codebook(Ws_rb, D, Hb, ocbs, j)
+        np.testing.assert_array_equal(host(cnt), co)
+        _cmp_codebook(host(Cg), Co.astype(np.float64))
+
+    if not encode:
+        return
+    # arg-min encode of 8 whole non-critical group columns with the final base codebook
+    g0 = Gc + (G - Gc) // 3
+    g1 = g0 + 8
+    codes = torch.zeros((T.shape[0], 8), dtype=torch.int32, device="cuda")
+    P.crvq_encode_beam(T[:, g0 * D:g1 * D], D, Hb_d[g0:g1],
+                       [Codebook(out.C_base, codes, 8)], 0, 1)
+    P.crvq_sync()
+    Tg = np.ascontiguousarray(Ws_rb[:, g0 * D:g1 * D])
+    ob = [O.Codebook(host(out.C_base), None, 8)]
+    oc, _ = O.encode_beam(Tg, D, Hb[g0:g1], ob, 0, 1)
+    check_codes_with_ties(Tg, D, Hb[g0:g1], ob, 0, [host(codes)], oc)
+
+    # stage-wise beam over every codebook on 2 whole critical group columns
+    gc = min(2, Gc)
+    new = [torch.zeros((T.shape[0], gc), dtype=torch.int32, device="cuda") for _ in range(n_cb)]
+    bcbs = [Codebook(cb.C, nc, gc) for cb, nc in zip(cbs, new)]
+    P.crvq_encode_beam(T[:, :gc * D], D, Hb_d[:gc], bcbs, 0, cfg.B)
+    P.crvq_sync()
+    Tc = np.ascontiguousarray(Ws_rb[:, :gc * D])
+    obc = [O.Codebook(cb.C, None, gc) for cb in ocbs]
+    oc, _ = O.encode_beam(Tc, D, Hb[:gc], obc, 0, cfg.B)
+    gpu = [host(c) for c in new]
+    diff = np.zeros((Tc.shape[0], gc), bool)
+    for s in range(n_cb):
+        diff |= gpu[s] != oc[s]
+    for i, g in zip(*np.nonzero(diff)):
+        gap = beam_boundary_gap(Tc[i, g * D:(g + 1) * D].astype(np.float64), Hb[g],
+                                [cb.C for cb in obc], cfg.B)
+        assert gap < REL_TIE, f"beam code differs at ({i},{g}) with gap {gap}"
+
+
+def test_full_size_encode_pass_and_update_k65536():
     """One arg-min pass at the down_proj size with a 65536-entry codebook (codeword chunks
-    streamed through the tensor-core pass; rows left open decided exactly)."""
+    streamed through the tensor-core pass; rows left open decided exactly), then the
+    least-squares update of that codebook from the codes it wrote (per-(group, code) counts
+    of 1376 x 65536 entries) against the oracle's update."""
     import paper_2412_09282_gb300 as P
     from paper_2412_09282_gb300 import Codebook
     cfg = S.C3
@@ -123,28 +232,38 @@ def test_full_size_encode_pass_k65536_sampled():
     X = S.gen_X(cfg)
     M, N = W.shape
     G = N // D
-    Hd, _, Hb, _ = P.crvq_hessian(dev(X), cfg.damp_rel, D)
+    _, _, Hb, _ = O.hessian(X, cfg.damp_rel, D)
     rng = np.random.default_rng(5)
     K = 65536
     src = rng.integers(0, M * G, K)
     C = W.reshape(M * G, D)[src] + rng.normal(0, 0.002, (K, D)).astype(np.float32)
     C = np.ascontiguousarray(C.astype(np.float32))
     codes = torch.zeros((M, G), dtype=torch.int32, device="cuda")
+    Wd, Hd = dev(W), dev(Hb)
     cb = [Codebook(dev(C), codes, G)]
-    vec_err = P.crvq_encode_beam(dev(W), D, Hb, cb, 0, 1, want_err=True)
-    torch.cuda.synchronize()
-    Hbh = host(Hb).astype(np.float64)
+    vec_err = P.crvq_encode_beam(Wd, D, Hd, cb, 0, 1, want_err=True)
+    P.crvq_sync()
     cg, eg = host(codes), host(vec_err)
     rows = np.sort(rng.choice(M, 4, replace=False))
     groups = np.sort(rng.choice(G, 8, replace=False))
     bad = []
     for i in rows:
         for g in groups:
+            H = Hb[g].astype(np.float64)
             t = W[i, g * D:(g + 1) * D].astype(np.float64)
-            e = _err(t, C, Hbh[g])
+            e = _err(t, C, H)
             k = int(cg[i, g])
-            tt = float(t @ Hbh[g] @ t)
+            tt = float(t @ H @ t)
             if k != int(np.argmin(e)) and e[k] - e.min() > REL_TIE * (e.min() + tt):
                 bad.append((int(i), int(g), k, int(np.argmin(e))))
             assert abs(float(eg[i, g]) - e[k]) <= 1e-4 * (e[k] + tt) + 1e-30
     assert not bad, bad[:5]
+
+    Cg, cnt = P.crvq_update_codebook(Wd, D, Hd, cb, 0)
+    P.crvq_sync()
+    Co, co = O.update_codebook(W, D, Hb, [O.Codebook(C, cg, G)], 0)
+    np.testing.assert_array_equal(host(cnt), co)
+    assert (co == 0).any() and (co > 1).any()        # empty and shared clusters both occur
+    _cmp_codebook(host(Cg), Co.astype(np.float64))
+    empty = co == 0
+    np.testing.assert_array_equal(host(Cg)[empty], C[empty])
