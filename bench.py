@@ -248,6 +248,55 @@ def pool_workers(cfg):
     return min(len(os.sched_getaffinity(0)), cfg.M // max(need, 1))
 
 
+def inference_matvec(P, work, flush, stream, reps=20):
+    """The inference product from codes (crvq_lut_matvec; the paper's inference setting) on each
+    distinct matrix shape of the workload, with one input (the decode matrix-vector product),
+    using the codes and codebooks the timed steps produced. Each call is timed alone with CUDA
+    events on the launching stream, the L2 flushed before it. Algorithmic bytes: every code
+    (4 B), the input, the permutation and the output once. A dense bf16 matrix-vector product
+    of the same shape (torch) is timed the same way, as context only."""
+    import torch
+    from paper_2412_09282_gb300 import Codebook
+    rows, seen = [], set()
+    for w in work:
+        cfg, out = w["cfg"], w["out"]
+        key = (cfg.M, cfg.N)
+        if key in seen:
+            continue
+        seen.add(key)
+        G = cfg.N // cfg.d
+        Gc = out.report["n_crit_groups"]
+        cbs = [Codebook(out.C_base, out.codes_base, G)] + \
+            [Codebook(out.C_ext[t].contiguous(), out.codes_ext[t], Gc) for t in range(cfg.n_ext)]
+        x = torch.randn((1, cfg.N), device=out.C_base.device)
+        y = torch.empty((1, cfg.M), device=x.device)
+        Wb = w["W_d"].to(torch.bfloat16)
+        xb = x[0].to(torch.bfloat16)
+
+        def timed(fn):
+            ts = []
+            for _ in range(reps + 3):
+                flush.fill_(1.0)
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                fn()
+                b.record(stream)
+                b.synchronize()
+                ts.append(a.elapsed_time(b))
+            return statistics.median(ts[3:])
+
+        ms = timed(lambda: P.crvq_lut_matvec(x, out.perm, cbs, cfg.M, Y=y))
+        P.crvq_sync()
+        dense = timed(lambda: torch.mv(Wb, xb))
+        nbytes = 4 * (cfg.M * G + cfg.n_ext * cfg.M * Gc) + 4 * cfg.N * 2 + 4 * cfg.M
+        rows.append({"matrix": cfg.name.split("/")[-1], "M": cfg.M, "N": cfg.N, "b": 1,
+                     "us": 1e3 * ms, "bytes": nbytes, "gbs": nbytes / (ms / 1e3) / 1e9,
+                     "dense_bf16_mv_us": 1e3 * dense})
+        del Wb
+    return rows
+
+
 def dist_init():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -369,6 +418,8 @@ def main():
     ap.add_argument("--ref-warmup", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--no-infer", action="store_true",
+                    help="skip the inference-product timing after the timed steps")
     args = ap.parse_args()
     layers = workload_layers(args.config)
     ws, rank, local = dist_init()
@@ -489,6 +540,8 @@ def main():
                "d2h_bytes_per_step": int(d2h),
                "ms_per_step": 1e3 * statistics.mean(e2e_times)}
 
+    infer = inference_matvec(P, work, flush, stream) if not args.no_infer else None
+
     if rank != 0:
         return
     peaks, peak_src = load_peaks()
@@ -544,6 +597,13 @@ def main():
                      "share": k["ms"] / total_k} for k in ks[:12]],
         "clocks": clk,
     }
+    if infer:
+        for r in infer:
+            r["hbm_frac"] = r["gbs"] / peaks.get("hbm_gbs", 6800.0)
+        line["inference_matvec"] = {
+            "call": "crvq_lut_matvec (Y = x W_hat^T from the codes, one input)",
+            "peak_gbs": peaks.get("hbm_gbs"), "peak_source": f"hbm_gbs ({peak_src}) burst",
+            "shapes": infer}
     if last is not None:
         line["losses"] = {k: last[k] for k in ("loss_pre", "loss_block", "loss_crit",
                                                 "loss_full")}

@@ -275,6 +275,27 @@ crvq_status crvq_reconstruct_error(const float* W_sorted, int64_t M, int64_t N, 
                                    double damp_delta, float* W_hat, double* losses,
                                    crvq_stream_t stream);
 
+/*
+ * Inference product of a quantized matrix, from its codes (App. "Inference Speed", Table
+ * speed: the matrix-vector product with a CRVQ layer). Y = X_in W_hat^T for b inputs, W_hat
+ * being the reconstruction in the original channel order that crvq_reconstruct_error returns,
+ * without forming it:
+ *   Y[bi][i] = sum over codebooks s and groups g < G_cov(s) of
+ *              <C_s[code_s(i, g)], x_sorted[bi][g d .. g d + d)>,  x_sorted[bi][p] = X_in[bi][perm[p]].
+ *   X_in   [b x N] device, row stride ldx >= N (floats).
+ *   perm   [N] device channel order (perm[new] = old), or NULL for the identity.
+ *   cbs    the n_cb codebooks of the M x (N/d) vector set (base first, as the layer returns
+ *          them; codes int32 on the device).
+ *   Y      [b x M] out, row stride ldy >= M.
+ * fp32 arithmetic: every codeword-input product is an 8-term FMA chain and the sums over
+ * groups follow a fixed order (no atomics), so results are identical run to run. Codes
+ * outside [0, K) and perm entries outside [0, N) are skipped and reported by crvq_sync.
+ * Requires 1 <= b <= 8, N % d == 0, 1 <= n_cb <= 8; d = 8.
+ */
+crvq_status crvq_lut_matvec(const float* X_in, int64_t ldx, int64_t b, int64_t N, int32_t d,
+                            const int32_t* perm, const crvq_codebook* cbs, int32_t n_cb,
+                            int64_t M, float* Y, int64_t ldy, crvq_stream_t stream);
+
 /* Average bits per weight (Sec. 3.2 Eq. (bitwidth); App. A.1): e-bit codes for all M N / d
  * vectors, plus m-1 extended codebooks on the lambda fraction, plus m codebooks of 2^e
  * fp16 vectors of length d, plus (include_perm) a 16-bit reorder index per channel. */

@@ -256,6 +256,21 @@ def crvq_update_codebook_noalloc(T, d, H_blocks, cbs, which, C_out=None, counts=
     return C_out, counts
 
 
+def crvq_lut_matvec(X_in, perm, cbs, M, d=8, Y=None, stream=None):
+    """Y = X_in W_hat^T (b x M) from the codes of `cbs`, X_in b x N in the original channel
+    order (a 1-D input is one row); perm None is the identity order."""
+    _need(X_in, torch.float32, "X_in")
+    X2 = X_in.unsqueeze(0) if X_in.dim() == 1 else X_in
+    _rowmajor(X2, "X_in")
+    b, N = X2.shape
+    dev = X2.device
+    Y = torch.empty((b, M), device=dev, dtype=torch.float32) if Y is None else Y
+    arr = _cb_array(cbs)
+    _check(_L().crvq_lut_matvec(_ptr(X2), X2.stride(0), b, N, d, _ptr(perm), arr, len(cbs), M,
+                                _ptr(Y), Y.stride(0), _stream(stream, dev)))
+    return Y
+
+
 def crvq_reconstruct_error(W_sorted, d, H_blocks, perm, cbs, n_crit_groups, X=None,
                            damp_delta=0.0, want_W_hat=True, stream=None):
     """Returns (W_hat or None, loss_block, loss_crit, loss_full). Synchronizes the stream."""

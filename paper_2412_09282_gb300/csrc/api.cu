@@ -540,6 +540,23 @@ crvq_status crvq_reconstruct_error(const float* W_sorted, int64_t M, int64_t N, 
   return CRVQ_OK;
 }
 
+crvq_status crvq_lut_matvec(const float* X_in, int64_t ldx, int64_t b, int64_t N, int32_t d,
+                            const int32_t* perm, const crvq_codebook* cbs, int32_t n_cb,
+                            int64_t M, float* Y, int64_t ldy, crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_TRY(check_d(d));
+  CRVQ_CHECK_ARG(X_in && Y, "X_in and Y must not be NULL");
+  CRVQ_CHECK_ARG(N >= 1 && N % d == 0 && M >= 1, "need N >= 1, N %% d == 0, M >= 1");
+  CRVQ_CHECK_ARG(b >= 1 && ldx >= N && ldy >= M, "need b >= 1, ldx >= N, ldy >= M");
+  if (b > 8) return fail(CRVQ_ERR_UNSUPPORTED, "batches of more than 8 inputs are not implemented");
+  CRVQ_CHECK_ARG(n_cb >= 1, "n_cb must be >= 1");
+  CbList cl;
+  CRVQ_TRY(make_cblist(cbs, n_cb, N / d, true, &cl));
+  CRVQ_TRY(check_dev({{X_in, "X_in"}, {perm, "perm"}, {Y, "Y"}}));
+  CRVQ_TRY(check_dev_cbs(cbs, n_cb));
+  return launch_lut_matvec(X_in, ldx, N, (int)b, perm, cl, M, Y, ldy, (cudaStream_t)stream);
+}
+
 double crvq_avg_bits(int32_t e, int32_t d, int32_t m, double lambda, int64_t M, int64_t N,
                      int32_t include_perm) {
   if (d <= 0 || M <= 0 || N <= 0 || m < 1 || e < 0) return std::nan("");

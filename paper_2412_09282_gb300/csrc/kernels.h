@@ -89,4 +89,10 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
                                      double damp_delta, const float* delta_dev, float* W_hat,
                                      double* losses_dev, cudaStream_t stream);
 
+// Y = X_in W_hat^T from the codes (see crvq_lut_matvec); b inputs of N channels (row stride
+// ldx), M output rows (Y row stride ldy).
+crvq_status launch_lut_matvec(const float* X, int64_t ldx, int64_t N, int b,
+                              const int32_t* perm, const CbList& cbs, int64_t M, float* Y,
+                              int64_t ldy, cudaStream_t stream);
+
 }  // namespace crvq

@@ -95,6 +95,12 @@ def test_validation_rejects_before_launch(lib):
     gc = c.c_int64(0)
     assert lib.crvq_select_reorder_channels(dummy, 2, 16, 8, dummy, dummy, dummy, 1.5, 0, 0,
                                             dummy, None, dummy, dummy, c.byref(gc), None) == -1
+    # inference product: more than 8 inputs unsupported; row strides below the sizes invalid
+    cb[0] = _lib.crvq_codebook(16, 4, 0, 32, 2, 2)
+    assert lib.crvq_lut_matvec(dummy, 16, 9, 16, 8, None, cb, 1, 2, dummy, 2, None) == -2
+    assert lib.crvq_lut_matvec(dummy, 8, 1, 16, 8, None, cb, 1, 2, dummy, 2, None) == -1
+    assert lib.crvq_lut_matvec(dummy, 16, 1, 16, 8, None, cb, 1, 2, dummy, 1, None) == -1
+    assert lib.crvq_lut_matvec(dummy, 16, 1, 12, 8, None, cb, 1, 2, dummy, 2, None) == -1
     # unknown importance mode
     assert lib.crvq_select_reorder_channels(dummy, 2, 16, 8, dummy, dummy, dummy, 0.5, 7, 0,
                                             dummy, None, dummy, dummy, c.byref(gc), None) == -1
@@ -120,6 +126,7 @@ def test_step_calls_refuse_host_memory_before_launch(lib):
         lambda: lib.crvq_update_codebook(host, 16, 2, 2, 8, host, cb, 1, 0, host, None, None),
         lambda: lib.crvq_update_codebook_noalloc(host, 16, 2, 2, 8, host, cb, 1, 0, host, None,
                                                  None),
+        lambda: lib.crvq_lut_matvec(host, 16, 1, 16, 8, None, cb, 1, 2, host, 2, None),
         lambda: lib.crvq_reconstruct_error(host, 2, 16, 8, host, None, cb, 1, 0, None, 0, 0.0,
                                            None, (c.c_double * 3)(), None),
     ]

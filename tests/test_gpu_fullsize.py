@@ -237,6 +237,7 @@ def test_full_size_encode_pass_and_update_k65536():
     K = 65536
     src = rng.integers(0, M * G, K)
     C = W.reshape(M * G, D)[src] + rng.normal(0, 0.002, (K, D)).astype(np.float32)
+    C[rng.choice(K, 512, replace=False)] = 7.0       # far from every vector: empty clusters
     C = np.ascontiguousarray(C.astype(np.float32))
     codes = torch.zeros((M, G), dtype=torch.int32, device="cuda")
     Wd, Hd = dev(W), dev(Hb)
