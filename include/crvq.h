@@ -276,6 +276,33 @@ crvq_status crvq_reconstruct_error(const float* W_sorted, int64_t M, int64_t N, 
                                    crvq_stream_t stream);
 
 /*
+ * Code search under the full Alg. 1 loss (QuantLoss ||W X - W_enc X||^2 = tr(dW H dW^T),
+ * cross-group terms included; the encode calls above score each vector with its own diagonal
+ * block only). Gauss-Seidel over the groups of codebook `which`, every other codebook fixed:
+ * for g = 0 .. G_cov-1 in order, each row's code of group g becomes the arg-min (as
+ * crvq_encode_beam decides it, ties to the smaller index) of err(t', c) = (t' - c)^T H_gg (t' - c)
+ * for the shifted target t' = t + H_gg^-1 b_g, where t is the row segment minus the other
+ * codebooks' codewords, b_g = sum_{g' != g} H_gg' D_g' and D = W - W_enc with every code
+ * decided so far (completing the square of the row loss in D_g). The full loss never rises.
+ *   W_sorted  [M x N] weights in the channel order of H (row-major, 16-byte aligned).
+ *   H_sorted  [N x N] the damped Hessian proxy in the same channel order (symmetric; e.g.
+ *             crvq_hessian's H taken through the layer's perm).
+ *   cbs       the n_cb codebooks of the M x (N/d) vector set; the codes of `which` are read
+ *             and rewritten in place.
+ *   sweeps    >= 0 passes over the groups.
+ *   loss      HOST out [sweeps + 1] or NULL: tr(dW H dW^T) before the first sweep and after
+ *             each (3xTF32 products, fp64 sums). Synchronizes `stream` when given.
+ * b_g comes from tensor-core products of H with D^T taken per block of 256 channels at the
+ * block's start plus the block's own earlier changes; the shift is solved in fp32 with a
+ * Cholesky factor of H_gg computed in fp64. A block without a factor is reported as
+ * CRVQ_ERR_NUMERIC by crvq_sync. Requires N % d == 0, N <= 49152; d = 8.
+ */
+crvq_status crvq_coupled_sweep(const float* W_sorted, int64_t M, int64_t N, int32_t d,
+                               const float* H_sorted, const crvq_codebook* cbs, int32_t n_cb,
+                               int32_t which, int32_t sweeps, double* loss,
+                               crvq_stream_t stream);
+
+/*
  * Inference product of a quantized matrix, from its codes (App. "Inference Speed", Table
  * speed: the matrix-vector product with a CRVQ layer). Y = X_in W_hat^T for b inputs, W_hat
  * being the reconstruction in the original channel order that crvq_reconstruct_error returns,

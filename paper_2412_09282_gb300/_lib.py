@@ -78,6 +78,9 @@ SIGNATURES = {
     "crvq_reconstruct_error": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int32, c_vp, c_vp,
                                            C.POINTER(crvq_codebook), C.c_int32, C.c_int64,
                                            c_vp, C.c_int64, C.c_double, c_vp, c_f64p, c_vp]),
+    "crvq_coupled_sweep": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int32, c_vp,
+                                       C.POINTER(crvq_codebook), C.c_int32, C.c_int32,
+                                       C.c_int32, c_f64p, c_vp]),
     "crvq_lut_matvec": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int64, C.c_int32, c_vp,
                                     C.POINTER(crvq_codebook), C.c_int32, C.c_int64, c_vp,
                                     C.c_int64, c_vp]),

@@ -256,6 +256,23 @@ def crvq_update_codebook_noalloc(T, d, H_blocks, cbs, which, C_out=None, counts=
     return C_out, counts
 
 
+def crvq_coupled_sweep(W_sorted, H_sorted, cbs, which, sweeps=1, d=8, want_loss=True,
+                       stream=None):
+    """Gauss-Seidel sweeps of codebook `which` under the full loss (codes rewritten in place);
+    returns the loss before and after each sweep (a list), or None. Synchronizes when the
+    losses are requested."""
+    _need(W_sorted, torch.float32, "W_sorted")
+    _rowmajor(W_sorted, "W_sorted")
+    _need(H_sorted, torch.float32, "H_sorted")
+    M, N = W_sorted.shape
+    arr = _cb_array(cbs)
+    loss = (C.c_double * (sweeps + 1))() if want_loss else None
+    _check(_L().crvq_coupled_sweep(_ptr(W_sorted), M, N, d, _ptr(H_sorted.contiguous()), arr,
+                                   len(cbs), which, sweeps, loss,
+                                   _stream(stream, W_sorted.device)))
+    return list(loss) if want_loss else None
+
+
 def crvq_lut_matvec(X_in, perm, cbs, M, d=8, Y=None, stream=None):
     """Y = X_in W_hat^T (b x M) from the codes of `cbs`, X_in b x N in the original channel
     order (a 1-D input is one row); perm None is the identity order."""

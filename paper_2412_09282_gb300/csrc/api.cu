@@ -540,6 +540,37 @@ crvq_status crvq_reconstruct_error(const float* W_sorted, int64_t M, int64_t N, 
   return CRVQ_OK;
 }
 
+crvq_status crvq_coupled_sweep(const float* W_sorted, int64_t M, int64_t N, int32_t d,
+                               const float* H_sorted, const crvq_codebook* cbs, int32_t n_cb,
+                               int32_t which, int32_t sweeps, double* loss,
+                               crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_TRY(check_d(d));
+  CRVQ_CHECK_ARG(N >= 1 && N % d == 0, "N must be a positive multiple of d");
+  CRVQ_CHECK_ARG(N <= 49152, "N must be <= 49152");
+  CRVQ_TRY(check_set(W_sorted, N, M, N / d, H_sorted));
+  CRVQ_CHECK_ARG(n_cb >= 1 && which >= 0 && which < n_cb, "which must be in [0, n_cb)");
+  CRVQ_CHECK_ARG(sweeps >= 0, "sweeps must be >= 0");
+  CbList cl;
+  CRVQ_TRY(make_cblist(cbs, n_cb, N / d, true, &cl));
+  CRVQ_TRY(check_dev({{W_sorted, "W_sorted"}, {H_sorted, "H_sorted"}}));
+  CRVQ_TRY(check_dev_cbs(cbs, n_cb));
+  cudaStream_t s = (cudaStream_t)stream;
+  Scratch mem;
+  double* ld = nullptr;
+  if (loss) {
+    CRVQ_TRY(mem.alloc((size_t)(sweeps + 1) * sizeof(double), s));
+    ld = mem.as<double>();
+  }
+  CRVQ_TRY(launch_coupled_sweep(W_sorted, M, N, H_sorted, cl, which, sweeps, ld, s));
+  if (loss) {
+    CRVQ_CUDA(cudaMemcpyAsync(loss, ld, (size_t)(sweeps + 1) * sizeof(double),
+                              cudaMemcpyDeviceToHost, s));
+    CRVQ_CUDA(cudaStreamSynchronize(s));
+  }
+  return CRVQ_OK;
+}
+
 crvq_status crvq_lut_matvec(const float* X_in, int64_t ldx, int64_t b, int64_t N, int32_t d,
                             const int32_t* perm, const crvq_codebook* cbs, int32_t n_cb,
                             int64_t M, float* Y, int64_t ldy, crvq_stream_t stream) {

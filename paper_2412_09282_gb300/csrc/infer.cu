@@ -29,6 +29,7 @@ constexpr int kSliceG = 32;     // groups per CTA slice (one per lane)
 constexpr int kMvThreads = 256;
 constexpr int kMaxBatch = 8;
 constexpr size_t kLutSmemCap = 160 * 1024;  // shared memory for lookup tables per CTA
+constexpr int kRowBatch = 8;    // rows a warp reads codes for before using any
 
 struct MatvecArgs {
   const float* X;       // b x N, row stride ldx
@@ -50,7 +51,7 @@ __device__ __forceinline__ float warp_sum(float v) {
 }
 
 // Partial products of one (row block, group slice): part[slice][bi][i].
-template <int BMAX>
+template <int BMAX, int MAXCB>
 __global__ void __launch_bounds__(kMvThreads)
 matvec_slice_kernel(MatvecArgs a, int rows_per_cta, unsigned* err) {
   extern __shared__ __align__(16) float sm[];
@@ -81,7 +82,8 @@ matvec_slice_kernel(MatvecArgs a, int rows_per_cta, unsigned* err) {
     xs[e] = v;
   }
   __syncthreads();
-  // lookup tables of the codebooks that have one: lut[g][k][bi] = <C[k], xs[bi][g]>
+  // lookup tables of the codebooks that have one: lut[g][k][bi] = <C[k], xs[bi][g]>; a thread
+  // takes one codeword (loaded once) across the slice's groups
   {
     float* t = lut;
     for (int s = 0; s < a.cbs.n; ++s) {
@@ -89,50 +91,70 @@ matvec_slice_kernel(MatvecArgs a, int rows_per_cta, unsigned* err) {
       const CbView& cb = a.cbs.cb[s];
       const int64_t gcov = cb.G_cov - g0;
       const int gc = gcov <= 0 ? 0 : (int)(gcov < gn ? gcov : gn);
-      for (int e = tid; e < gc * cb.K; e += blockDim.x) {
-        const int gl = e / cb.K, k = e % cb.K;
+      for (int k = tid; k < cb.K && gc > 0; k += blockDim.x) {
         const float4 c0 = __ldg(reinterpret_cast<const float4*>(cb.C + (int64_t)k * kD));
         const float4 c1 = __ldg(reinterpret_cast<const float4*>(cb.C + (int64_t)k * kD + 4));
-        for (int bi = 0; bi < a.b; ++bi) {
-          const float* x = xs + (bi * kSliceG + gl) * kD;
-          float v = c0.x * x[0];
-          v = fmaf(c0.y, x[1], v);
-          v = fmaf(c0.z, x[2], v);
-          v = fmaf(c0.w, x[3], v);
-          v = fmaf(c1.x, x[4], v);
-          v = fmaf(c1.y, x[5], v);
-          v = fmaf(c1.z, x[6], v);
-          v = fmaf(c1.w, x[7], v);
-          t[((int64_t)gl * cb.K + k) * a.b + bi] = v;
-        }
+        for (int gl = 0; gl < gc; ++gl)
+          for (int bi = 0; bi < a.b; ++bi) {
+            const float* x = xs + (bi * kSliceG + gl) * kD;
+            float v = c0.x * x[0];
+            v = fmaf(c0.y, x[1], v);
+            v = fmaf(c0.z, x[2], v);
+            v = fmaf(c0.w, x[3], v);
+            v = fmaf(c1.x, x[4], v);
+            v = fmaf(c1.y, x[5], v);
+            v = fmaf(c1.z, x[6], v);
+            v = fmaf(c1.w, x[7], v);
+            t[((int64_t)gl * cb.K + k) * a.b + bi] = v;
+          }
       }
       t += (int64_t)kSliceG * cb.K * a.b;
     }
   }
   __syncthreads();
 
-  // rows of this block: a warp per row, lane = group g0 + lane
+  // rows of this block: a warp takes kRowBatch rows at a time, lane = group g0 + lane; the
+  // codes of every row and codebook of the batch are loaded before any is used, so that each
+  // warp keeps kRowBatch x n_cb coalesced 128-byte reads in flight (the kernel is bound by the
+  // latency of these reads otherwise)
   const int64_t r0 = (int64_t)blockIdx.x * rows_per_cta;
   const int64_t r1 = a.M < r0 + rows_per_cta ? a.M : r0 + rows_per_cta;
   const int nwarps = blockDim.x >> 5;
-  for (int64_t i = r0 + warp; i < r1; i += nwarps) {
-    float acc[BMAX];
+  const int64_t g = g0 + lane;
+  for (int64_t ib = r0 + (int64_t)warp * kRowBatch; ib < r1; ib += (int64_t)nwarps * kRowBatch) {
+    int32_t kc[MAXCB][kRowBatch];
 #pragma unroll
-    for (int bi = 0; bi < BMAX; ++bi) acc[bi] = 0.f;
+    for (int s = 0; s < MAXCB; ++s) {
+      const bool cov = s < a.cbs.n && lane < gn && g < a.cbs.cb[s].G_cov;
+#pragma unroll
+      for (int u = 0; u < kRowBatch; ++u) {
+        const int64_t i = ib + u;
+        kc[s][u] = (cov && i < r1) ? __ldg(a.cbs.cb[s].codes + i * a.cbs.cb[s].ld + g) : -1;
+      }
+    }
+    float acc[kRowBatch][BMAX];
+#pragma unroll
+    for (int u = 0; u < kRowBatch; ++u)
+#pragma unroll
+      for (int bi = 0; bi < BMAX; ++bi) acc[u][bi] = 0.f;
     const float* t = lut;
-    for (int s = 0; s < a.cbs.n; ++s) {
+#pragma unroll
+    for (int s = 0; s < MAXCB; ++s) {
+      if (s >= a.cbs.n) break;
       const CbView& cb = a.cbs.cb[s];
+      const bool cov = lane < gn && g < cb.G_cov;
       const bool has_lut = (a.lut_mask >> s) & 1;
-      const int64_t g = g0 + lane;
-      if (lane < gn && g < cb.G_cov) {
-        const int32_t k = cb.codes[i * cb.ld + g];
+#pragma unroll
+      for (int u = 0; u < kRowBatch; ++u) {
+        const int32_t k = kc[s][u];
+        if (!cov || ib + u >= r1) continue;
         if (k < 0 || k >= cb.K) {
           raise_error(err, ERRBIT_INDEX);
         } else if (has_lut) {
           const float* e = t + ((int64_t)lane * cb.K + k) * a.b;
 #pragma unroll
           for (int bi = 0; bi < BMAX; ++bi)
-            if (bi < a.b) acc[bi] += e[bi];
+            if (bi < a.b) acc[u][bi] += e[bi];
         } else {
           const float4 c0 = __ldg(reinterpret_cast<const float4*>(cb.C + (int64_t)k * kD));
           const float4 c1 = __ldg(reinterpret_cast<const float4*>(cb.C + (int64_t)k * kD + 4));
@@ -148,17 +170,21 @@ matvec_slice_kernel(MatvecArgs a, int rows_per_cta, unsigned* err) {
             v = fmaf(c1.y, x[5], v);
             v = fmaf(c1.z, x[6], v);
             v = fmaf(c1.w, x[7], v);
-            acc[bi] += v;
+            acc[u][bi] += v;
           }
         }
       }
       if (has_lut) t += (int64_t)kSliceG * cb.K * a.b;
     }
 #pragma unroll
-    for (int bi = 0; bi < BMAX; ++bi) {
-      if (bi >= a.b) break;
-      const float v = warp_sum(acc[bi]);
-      if (lane == 0) a.part[(slice * a.b + bi) * a.M + i] = v;
+    for (int u = 0; u < kRowBatch; ++u) {
+      const int64_t i = ib + u;
+#pragma unroll
+      for (int bi = 0; bi < BMAX; ++bi) {
+        if (bi >= a.b) break;
+        const float v = warp_sum(acc[u][bi]);
+        if (lane == 0 && i < r1) a.part[(slice * a.b + bi) * a.M + i] = v;
+      }
     }
   }
 }
@@ -222,18 +248,20 @@ crvq_status launch_lut_matvec(const float* X, int64_t ldx, int64_t N, int b,
   const dim3 grid((unsigned)ceil_div(M, rows_per_cta), (unsigned)a.n_slices);
   {
     ProfScope ps("matvec_slices", stream, (double)M * G * cbs.n);
-    if (b == 1) {
-      CRVQ_CUDA(cudaFuncSetAttribute(matvec_slice_kernel<1>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-      matvec_slice_kernel<1><<<grid, kMvThreads, smem, stream>>>(a, rows_per_cta, err);
-    } else if (b <= 4) {
-      CRVQ_CUDA(cudaFuncSetAttribute(matvec_slice_kernel<4>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-      matvec_slice_kernel<4><<<grid, kMvThreads, smem, stream>>>(a, rows_per_cta, err);
+    auto go = [&](auto kernel) -> crvq_status {
+      CRVQ_CUDA(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)smem));
+      kernel<<<grid, kMvThreads, smem, stream>>>(a, rows_per_cta, err);
+      return CRVQ_OK;
+    };
+    if (b == 1 && cbs.n <= 4) {
+      CRVQ_TRY(go(matvec_slice_kernel<1, 4>));
+    } else if (b == 1) {
+      CRVQ_TRY(go(matvec_slice_kernel<1, kMaxCodebooks>));
+    } else if (b <= 4 && cbs.n <= 4) {
+      CRVQ_TRY(go(matvec_slice_kernel<4, 4>));
     } else {
-      CRVQ_CUDA(cudaFuncSetAttribute(matvec_slice_kernel<kMaxBatch>,
-                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-      matvec_slice_kernel<kMaxBatch><<<grid, kMvThreads, smem, stream>>>(a, rows_per_cta, err);
+      CRVQ_TRY(go(matvec_slice_kernel<kMaxBatch, kMaxCodebooks>));
     }
     CRVQ_LAUNCHED();
   }

@@ -47,6 +47,12 @@ crvq_status launch_tc_sumsq(const float* A, const float* A_sub, int64_t M, const
                             const int32_t* B_cols, int64_t Nb, int64_t K, double* part,
                             int64_t part_cap, int64_t* nparts, cudaStream_t stream);
 
+// C = A B^T on the tensor cores (3xTF32; K in chunks of 1024 added in order): A M x K
+// (leading dimension lda), B Nb x K (ldb), C M x Nb (ldc); all row-major, 16-byte aligned rows.
+crvq_status launch_tc_gemm_nt(const float* A, int64_t lda, int64_t M, const float* B,
+                              int64_t ldb, int64_t Nb, int64_t K, float* C, int64_t ldc,
+                              cudaStream_t stream);
+
 crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
                                   const float* W_pre, const float* xsq, const float* H,
                                   int mode, uint64_t seed, int32_t* perm, float* importance,
@@ -88,6 +94,12 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
                                      int64_t n_crit_groups, const float* X, int64_t n_tok,
                                      double damp_delta, const float* delta_dev, float* W_hat,
                                      double* losses_dev, cudaStream_t stream);
+
+// Gauss-Seidel sweeps of codebook `which` under the full loss (see crvq_coupled_sweep); W and
+// H (N x N) in the sorted channel order; loss_dev: sweeps + 1 doubles on the device or null.
+crvq_status launch_coupled_sweep(const float* W, int64_t M, int64_t N, const float* H,
+                                 const CbList& cbs, int which, int sweeps, double* loss_dev,
+                                 cudaStream_t stream);
 
 // Y = X_in W_hat^T from the codes (see crvq_lut_matvec); b inputs of N channels (row stride
 // ldx), M output rows (Y row stride ldy).

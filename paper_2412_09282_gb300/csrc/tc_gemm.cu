@@ -33,6 +33,17 @@ sum_partials_kernel(const float* __restrict__ P, int64_t count, int chunks, int6
     out[e] = chunk_sum(P, chunks, stride, e, scale);
 }
 
+// out[m][n] (leading dimension ldo) = sum of the chunk partials P[c][m][n] (M x Nb each), in
+// chunk order.
+__global__ void __launch_bounds__(256)
+sum_partials_strided_kernel(const float* __restrict__ P, int64_t M, int64_t Nb, int chunks,
+                            float* __restrict__ out, int64_t ldo) {
+  const int64_t count = M * Nb;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < count;
+       e += (int64_t)gridDim.x * blockDim.x)
+    out[(e / Nb) * ldo + e % Nb] = chunk_sum(P, chunks, count, e, 1.f);
+}
+
 // Original-order blocks, one CTA: xsq[i] = the undamped diagonal, delta = damp_rel * mean(xsq)
 // by the dense path's fixed-order fp64 reduction (1024 strided partials, then a tree), and the
 // blocks with delta added on their diagonals (rounded once from fp64, as the dense path does).
@@ -376,6 +387,47 @@ crvq_status launch_tc_syrk(const float* X, int64_t n, int64_t N, float* S, cudaS
     const int blocks = (int)std::min<int64_t>(ceil_div(N * N, 256), 16 * sm_count());
     sum_partials_kernel<<<blocks, 256, 0, stream>>>(P, N * N, (int)chunks, N * N,
                                                     (float)(1.0 / (double)n), S);
+    CRVQ_LAUNCHED();
+  }
+  return CRVQ_OK;
+}
+
+// C = A B^T (A: M x K, B: Nb x K, both row-major with leading dimensions lda, ldb; C: M x Nb
+// row-major, leading dimension ldc) on the tensor cores (3xTF32), K in chunks of at most 1024
+// whose partials are added in chunk order (the rounding sequence of the Hessian products).
+crvq_status launch_tc_gemm_nt(const float* A, int64_t lda, int64_t M, const float* B,
+                              int64_t ldb, int64_t Nb, int64_t K, float* C, int64_t ldc,
+                              cudaStream_t stream) {
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
+  const int64_t chunks = std::max<int64_t>(1, ceil_div(K, kKChunk));
+  Scratch mem;
+  float* P = C;
+  int64_t ldp = ldc;
+  if (chunks > 1) {
+    CRVQ_TRY(mem.alloc((size_t)chunks * M * Nb * sizeof(float), stream));
+    P = mem.as<float>();
+    ldp = Nb;
+  }
+  tc::GemmArgs g{};
+  g.A = tc::Operand{A, lda, M, true};
+  g.B = tc::Operand{B, ldb, Nb, true};
+  g.K = K;
+  g.k_chunk = kKChunk;
+  g.c_chunk_stride = M * Nb;
+  g.mode = tc::kStorePlain;
+  g.C = P;
+  g.ldc = ldp;
+  g.alpha = 1.f;
+  g.err = err;
+  {
+    ProfScope ps("gemm_nt_tc", stream, 2.0 * (double)M * Nb * K);
+    CRVQ_TRY(launch_gemm(g, chunks, stream));
+  }
+  if (chunks > 1) {
+    ProfScope ps("gemm_nt_sum_partials", stream, (double)chunks * M * Nb * 4.0);
+    const int blocks = (int)std::min<int64_t>(ceil_div(M * Nb, 256), 16 * sm_count());
+    sum_partials_strided_kernel<<<blocks, 256, 0, stream>>>(P, M, Nb, (int)chunks, C, ldc);
     CRVQ_LAUNCHED();
   }
   return CRVQ_OK;

@@ -106,7 +106,7 @@ __device__ __forceinline__ void split_store(const float v[R / kThreads][kBK], ch
 }
 
 // Epilogues.
-enum Mode { kStoreSymmetric = 0 };
+enum Mode { kStoreSymmetric = 0, kStorePlain = 1 };
 
 struct GemmArgs {
   Operand A, B;   // D[m][n] = sum_k A(m, k) B(n, k); M = A.rows, N = B.rows
@@ -117,6 +117,7 @@ struct GemmArgs {
   int64_t c_chunk_stride;
   int mode;
   // kStoreSymmetric: C[m][n] = C[n][m] = alpha * D[m][n] for n >= m (row-major, ldc)
+  // kStorePlain:     C[m][n] = alpha * D[m][n] (row-major, ldc)
   float* C;
   int64_t ldc;
   float alpha;
@@ -215,7 +216,13 @@ __global__ void __launch_bounds__(kThreads, 1) gemm3xtf32_kernel(GemmArgs a) {
     for (int c0 = 0; c0 < kBN; c0 += 32) {
       float v[32];
       tmem_ld32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
-      if (m < a.A.rows) {
+      if (m < a.A.rows && a.mode == kStorePlain) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+          const int64_t n = n0 + c0 + j;
+          if (n < a.B.rows) C[m * a.ldc + n] = a.alpha * v[j];
+        }
+      } else if (m < a.A.rows) {
 #pragma unroll
         for (int j = 0; j < 32; ++j) {
           const int64_t n = n0 + c0 + j;

@@ -103,7 +103,7 @@ def test_lut_matvec_is_deterministic_and_reports_bad_codes():
     M, N = 64, 256
     perm, cbs, G = _case(7, M, N, [256], [32])
     X = dev(np.random.default_rng(8).standard_normal((2, N)).astype(np.float32))
-    codes = dev(cbs[0].codes)
+    codes = dev(cbs[0].codes.astype(np.int32))
     gcbs = [Codebook(dev(cbs[0].C), codes, G)]
     a = P.crvq_lut_matvec(X, dev(perm), gcbs, M)
     b = P.crvq_lut_matvec(X, dev(perm), gcbs, M)
