@@ -251,10 +251,11 @@ def pool_workers(cfg):
 def inference_matvec(P, work, flush, stream, reps=20):
     """The inference product from codes (crvq_lut_matvec; the paper's inference setting) on each
     distinct matrix shape of the workload, with one input (the decode matrix-vector product),
-    using the codes and codebooks the timed steps produced. Each call is timed alone with CUDA
-    events on the launching stream, the L2 flushed before it. Algorithmic bytes: every code
-    (4 B), the input, the permutation and the output once. A dense bf16 matrix-vector product
-    of the same shape (torch) is timed the same way, as context only."""
+    using the codes and codebooks the timed steps produced. The L2 is flushed before every
+    call; the time is the library's CUDA events around its two kernels (slice products and the
+    ordered reduction) on the launching stream. Algorithmic bytes: every code (4 B), the input,
+    the permutation and the output once. A dense bf16 matrix-vector product of the same shape
+    (torch), timed with events around the call, is given as context only."""
     import torch
     from paper_2412_09282_gb300 import Codebook
     rows, seen = [], set()
@@ -270,31 +271,74 @@ def inference_matvec(P, work, flush, stream, reps=20):
             [Codebook(out.C_ext[t].contiguous(), out.codes_ext[t], Gc) for t in range(cfg.n_ext)]
         x = torch.randn((1, cfg.N), device=out.C_base.device)
         y = torch.empty((1, cfg.M), device=x.device)
+        for _ in range(3):
+            P.crvq_lut_matvec(x, out.perm, cbs, cfg.M, Y=y)
+        P.crvq_profile_filter("matvec")
+        P.crvq_profile_begin()
+        for _ in range(reps):
+            flush.fill_(1.0)
+            P.crvq_lut_matvec(x, out.perm, cbs, cfg.M, Y=y)
+        torch.cuda.synchronize()
+        st = P.crvq_profile_end()
+        P.crvq_profile_filter(None)
+        P.crvq_sync()
+        ms = sum(k["ms"] for k in st) / reps
+        kern = {k["name"]: 1e3 * k["ms"] / reps for k in st}
         Wb = w["W_d"].to(torch.bfloat16)
         xb = x[0].to(torch.bfloat16)
-
-        def timed(fn):
-            ts = []
-            for _ in range(reps + 3):
-                flush.fill_(1.0)
-                a = torch.cuda.Event(enable_timing=True)
-                b = torch.cuda.Event(enable_timing=True)
-                a.record(stream)
-                fn()
-                b.record(stream)
-                b.synchronize()
-                ts.append(a.elapsed_time(b))
-            return statistics.median(ts[3:])
-
-        ms = timed(lambda: P.crvq_lut_matvec(x, out.perm, cbs, cfg.M, Y=y))
-        P.crvq_sync()
-        dense = timed(lambda: torch.mv(Wb, xb))
+        ts = []
+        for _ in range(reps + 3):
+            flush.fill_(1.0)
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            torch.mv(Wb, xb)
+            b.record(stream)
+            b.synchronize()
+            ts.append(a.elapsed_time(b))
+        dense = statistics.median(ts[3:])
         nbytes = 4 * (cfg.M * G + cfg.n_ext * cfg.M * Gc) + 4 * cfg.N * 2 + 4 * cfg.M
         rows.append({"matrix": cfg.name.split("/")[-1], "M": cfg.M, "N": cfg.N, "b": 1,
-                     "us": 1e3 * ms, "bytes": nbytes, "gbs": nbytes / (ms / 1e3) / 1e9,
-                     "dense_bf16_mv_us": 1e3 * dense})
+                     "us": 1e3 * ms, "kernels_us": kern, "bytes": nbytes,
+                     "gbs": nbytes / (ms / 1e3) / 1e9, "dense_bf16_mv_us": 1e3 * dense})
         del Wb
     return rows
+
+
+def coupled_sweep_line(P, work, stream):
+    """One Gauss-Seidel sweep of the base codebook under the full loss (crvq_coupled_sweep) on
+    the workload's first matrix, from the codes the timed steps produced (on a copy): the dense
+    H of its X taken to the layer's channel order, the sweep timed with CUDA events around the
+    call (its kernels and their launches), the full loss tr(dW H dW^T) before and after."""
+    import torch
+    from paper_2412_09282_gb300 import Codebook
+    w = work[0]
+    cfg, out = w["cfg"], w["out"]
+    G, Gc = cfg.N // cfg.d, out.report["n_crit_groups"]
+    H, _, _, _ = P.crvq_hessian(w["X_d"], cfg.damp_rel, cfg.d)
+    perm = out.perm.long()
+    Hs = H[perm][:, perm].contiguous()
+    del H
+    Ws = w["W_d"][:, perm].contiguous()
+    cbs = [Codebook(out.C_base, out.codes_base.clone(), G)] + \
+        [Codebook(out.C_ext[t].contiguous(), out.codes_ext[t].clone(), Gc)
+         for t in range(cfg.n_ext)]
+    l0 = P.crvq_coupled_sweep(Ws, Hs, cbs, 0, sweeps=0)[0]
+    torch.cuda.synchronize()
+    a = torch.cuda.Event(enable_timing=True)
+    b = torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    P.crvq_coupled_sweep(Ws, Hs, cbs, 0, sweeps=1, want_loss=False)
+    b.record(stream)
+    b.synchronize()
+    P.crvq_sync()
+    ms = a.elapsed_time(b)
+    l1 = P.crvq_coupled_sweep(Ws, Hs, cbs, 0, sweeps=0)[0]
+    return {"call": "crvq_coupled_sweep (one sweep of the base codebook, cross-group terms)",
+            "matrix": cfg.name.split("/")[-1], "M": cfg.M, "N": cfg.N, "groups": G,
+            "sweep_ms": ms, "loss_full_before": l0, "loss_full_after": l1,
+            "loss_full_reduction": 1.0 - l1 / l0,
+            "tensor_work": "2 M N^2 flop per sweep (the lazy block products H[block] D^T)"}
 
 
 def dist_init():
@@ -419,7 +463,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--no-infer", action="store_true",
-                    help="skip the inference-product timing after the timed steps")
+                    help="skip the inference-product and coupled-sweep lines after the timed "
+                         "steps")
     args = ap.parse_args()
     layers = workload_layers(args.config)
     ws, rank, local = dist_init()
@@ -541,6 +586,7 @@ def main():
                "ms_per_step": 1e3 * statistics.mean(e2e_times)}
 
     infer = inference_matvec(P, work, flush, stream) if not args.no_infer else None
+    coupled = coupled_sweep_line(P, work, stream) if not args.no_infer else None
 
     if rank != 0:
         return
@@ -604,6 +650,8 @@ def main():
             "call": "crvq_lut_matvec (Y = x W_hat^T from the codes, one input)",
             "peak_gbs": peaks.get("hbm_gbs"), "peak_source": f"hbm_gbs ({peak_src}) burst",
             "shapes": infer}
+    if coupled:
+        line["coupled_sweep"] = coupled
     if last is not None:
         line["losses"] = {k: last[k] for k in ("loss_pre", "loss_block", "loss_crit",
                                                 "loss_full")}

@@ -15,45 +15,6 @@ namespace crvq {
 
 namespace {
 
-// Reconstruction of vector (i, g): the sum of the covering codebooks' codewords (codebook
-// order), correctly rounded to fp32 like the fp64 sum rounded once. With at most two terms the
-// fp32 sum is that value (the exact sum of two fp32 values rounds to fp32 the same way
-// whether or not it first passes through fp64); three or more terms are summed in fp64.
-__device__ __forceinline__ void recon(const CbList& cbs, int64_t i, int64_t g, float r[kD],
-                                      unsigned* err) {
-  const float* cw[kMaxCodebooks];
-  int n = 0;
-  for (int s = 0; s < cbs.n; ++s) {
-    const CbView& cb = cbs.cb[s];
-    if (g >= cb.G_cov) continue;
-    const int32_t k = cb.codes[i * cb.ld + g];
-    if (k < 0 || k >= cb.K) {
-      raise_error(err, ERRBIT_INDEX);
-      continue;
-    }
-    cw[n++] = cb.C + (int64_t)k * kD;
-  }
-  if (n <= 2) {
-#pragma unroll
-    for (int j = 0; j < kD; ++j) r[j] = 0.f;
-    for (int q = 0; q < n; ++q) {
-      const float4 a = *reinterpret_cast<const float4*>(cw[q]);
-      const float4 b = *reinterpret_cast<const float4*>(cw[q] + 4);
-      r[0] += a.x; r[1] += a.y; r[2] += a.z; r[3] += a.w;
-      r[4] += b.x; r[5] += b.y; r[6] += b.z; r[7] += b.w;
-    }
-  } else {
-    double d[kD];
-#pragma unroll
-    for (int j = 0; j < kD; ++j) d[j] = 0.0;
-    for (int q = 0; q < n; ++q)
-#pragma unroll
-      for (int j = 0; j < kD; ++j) d[j] += (double)cw[q][j];
-#pragma unroll
-    for (int j = 0; j < kD; ++j) r[j] = (float)d[j];
-  }
-}
-
 // Unevaluated fp32 pair (h, l) += x, and the merge of two pairs (TwoSum of the high parts).
 __device__ __forceinline__ void pair_add(float& h, float& l, float x) {
   const float s = __fadd_rn(h, x);
@@ -68,97 +29,180 @@ __device__ __forceinline__ void pair_merge(float& h, float& l, float oh, float o
   l = __fadd_rn(l, ol);
 }
 
-constexpr int kDecRows = 4;   // rows per warp: each H block is loaded once for all of them
-constexpr int kDecWarps = 8;  // warps per CTA
+constexpr int kDecRows = 16;     // rows per warp (the CTA's H blocks are staged once for all)
+constexpr int kDecBatch = 2;     // rows whose codes are loaded together
+constexpr int kDecWarps = 8;     // warps per CTA
+constexpr int kDecHStride = 260; // floats per staged H block (256 + 4: conflict-free float4)
+constexpr int kDecSmemCb = 48 * 1024;  // codebooks staged in shared memory up to this size
 
-// One warp = kDecRows rows x one slice of the groups, lanes across the groups: the
-// reconstruction in the sorted order (32-byte stores, consecutive lanes on consecutive
-// vectors), each vector's error under H_g (the block loaded once for the warp's rows; the
-// quadratic form as two FMA chains in fp32) and, per (row, slice), the block loss, the
-// critical loss and ||dW||^2 as fp32 pairs in a fixed order:
-// row_part[(row * slices + slice) * 3 + {0, 1, 2}] = (hi, lo). No shared memory and no block
-// barrier:
-// the kernel is bound by the latency of its loads, which full occupancy hides.
+// Reconstruction of a vector from its codes (k[s] < 0: codebook s does not cover it), with the
+// codewords read from `cw[s]` (shared memory or global): the sum in codebook order, correctly
+// rounded to fp32 like the fp64 sum rounded once (two terms in fp32 give that value exactly;
+// three or more are summed in fp64).
+template <int MAXCB>
+__device__ __forceinline__ void recon_codes(const float* const* cw, const int32_t* k, int ncb,
+                                            float r[kD]) {
+  int n = 0;
+#pragma unroll
+  for (int s = 0; s < MAXCB; ++s) n += (s < ncb && k[s] >= 0) ? 1 : 0;
+  if (n <= 2) {
+#pragma unroll
+    for (int j = 0; j < kD; ++j) r[j] = 0.f;
+#pragma unroll
+    for (int s = 0; s < MAXCB; ++s) {
+      if (s >= ncb || k[s] < 0) continue;
+      const float4 a = *reinterpret_cast<const float4*>(cw[s] + (int64_t)k[s] * kD);
+      const float4 b = *reinterpret_cast<const float4*>(cw[s] + (int64_t)k[s] * kD + 4);
+      r[0] += a.x; r[1] += a.y; r[2] += a.z; r[3] += a.w;
+      r[4] += b.x; r[5] += b.y; r[6] += b.z; r[7] += b.w;
+    }
+  } else {
+    double d[kD];
+#pragma unroll
+    for (int j = 0; j < kD; ++j) d[j] = 0.0;
+#pragma unroll
+    for (int s = 0; s < MAXCB; ++s) {
+      if (s >= ncb || k[s] < 0) continue;
+      const float* c = cw[s] + (int64_t)k[s] * kD;
+#pragma unroll
+      for (int j = 0; j < kD; ++j) d[j] += (double)c[j];
+    }
+#pragma unroll
+    for (int j = 0; j < kD; ++j) r[j] = (float)d[j];
+  }
+}
+
+// One warp = kDecRows rows x one slice of 32 groups, lane = group: the reconstruction in the
+// sorted order (32-byte stores, consecutive lanes on consecutive vectors), each vector's error
+// under H_g (the quadratic form as two FMA chains in fp32) and, per (row, slice), the block
+// loss, the critical loss and ||dW||^2 as fp32 pairs in a fixed order:
+// row_part[(row * slices + slice) * 3 + {0, 1, 2}] = (hi, lo). A CTA's warps share one slice:
+// its H blocks are staged in shared memory once for the CTA's kDecWarps x kDecRows rows; the
+// codebooks sit in shared memory when they fit, so the codeword lookup is not a dependent
+// global load; the codes of kDecBatch rows are loaded before any is used.
+template <int MAXCB>
 __global__ void __launch_bounds__(kDecWarps * 32)
 decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
                   const float* __restrict__ Hb, CbList cbs, int64_t n_crit_groups, int slices,
-                  float* __restrict__ W_rec, float2* __restrict__ row_part, unsigned* err) {
-  const int lane = threadIdx.x & 31;
-  const int64_t wid = (int64_t)blockIdx.x * kDecWarps + (threadIdx.x >> 5);
-  const int64_t G = N / kD;
-  const int64_t row_blocks = (M + kDecRows - 1) / kDecRows;
-  if (wid >= row_blocks * slices) return;  // whole warps
-  const int64_t rb = wid / slices;
-  const int sl = (int)(wid % slices);
-  const int64_t gs = (G + slices - 1) / slices;
-  const int64_t g0 = sl * gs, g1 = min(G, g0 + gs);
-  const int64_t i0 = rb * kDecRows;
-  const int nr = (int)min((int64_t)kDecRows, M - i0);
-  float lb[kDecRows], lbl[kDecRows], lc[kDecRows], lcl[kDecRows], sq[kDecRows], sql[kDecRows];
+                  int cb_in_smem, float* __restrict__ W_rec, float2* __restrict__ row_part,
+                  unsigned* err) {
+  extern __shared__ __align__(16) float s_dyn[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float* sH = s_dyn;                         // the CTA slice's 32 H blocks
+  float* s_cb = s_dyn + 32 * kDecHStride;    // codebooks (when staged)
+  const float* cw[MAXCB];
+  {
+    int64_t off = 0;
 #pragma unroll
-  for (int r = 0; r < kDecRows; ++r) lb[r] = lbl[r] = lc[r] = lcl[r] = sq[r] = sql[r] = 0.f;
-  for (int64_t g = g0 + lane; g < g1; g += 32) {
-    float4 H4[2 * kD];
-#pragma unroll
-    for (int q = 0; q < 2 * kD; ++q) H4[q] = __ldg(reinterpret_cast<const float4*>(Hb + g * kD * kD) + q);
-#pragma unroll
-    for (int r = 0; r < kDecRows; ++r) {
-      if (r >= nr) break;
-      const int64_t i = i0 + r;
-      float rv[kD], dl[kD];
-      recon(cbs, i, g, rv, err);
-      const float4 t0 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD);
-      const float4 t1 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD + 4);
-      const float t[kD] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w};
-      float q2 = 0.f;
-#pragma unroll
-      for (int j = 0; j < kD; ++j) {
-        dl[j] = t[j] - rv[j];
-        q2 = fmaf(dl[j], dl[j], q2);
-      }
-      float e = 0.f;
-#pragma unroll
-      for (int a = 0; a < kD; ++a) {
-        const float4 h0 = H4[2 * a], h1 = H4[2 * a + 1];
-        float hb = dl[0] * h0.x;
-        hb = fmaf(dl[1], h0.y, hb);
-        hb = fmaf(dl[2], h0.z, hb);
-        hb = fmaf(dl[3], h0.w, hb);
-        hb = fmaf(dl[4], h1.x, hb);
-        hb = fmaf(dl[5], h1.y, hb);
-        hb = fmaf(dl[6], h1.z, hb);
-        hb = fmaf(dl[7], h1.w, hb);
-        e = fmaf(hb, dl[a], e);
-      }
-      pair_add(lb[r], lbl[r], e);
-      if (g < n_crit_groups) pair_add(lc[r], lcl[r], e);
-      pair_add(sq[r], sql[r], q2);
-      if (W_rec) {
-        float* o = W_rec + i * N + g * kD;
-        *reinterpret_cast<float4*>(o) = make_float4(rv[0], rv[1], rv[2], rv[3]);
-        *reinterpret_cast<float4*>(o + 4) = make_float4(rv[4], rv[5], rv[6], rv[7]);
+    for (int s = 0; s < MAXCB; ++s) {
+      if (s >= cbs.n) break;
+      const int64_t n = (int64_t)cbs.cb[s].K * kD;
+      if (cb_in_smem) {
+        for (int64_t e = threadIdx.x * 4; e < n; e += blockDim.x * 4)
+          *reinterpret_cast<float4*>(s_cb + off + e) =
+              __ldg(reinterpret_cast<const float4*>(cbs.cb[s].C + e));
+        cw[s] = s_cb + off;
+        off += n;
+      } else {
+        cw[s] = cbs.cb[s].C;
       }
     }
+    if (cb_in_smem) __syncthreads();
   }
+  // CTA = (slice of 32 groups, kDecWarps x kDecRows rows); warp w takes kDecRows rows
+  const int64_t G = N / kD;
+  const int sl = (int)(blockIdx.x % slices);
+  const int64_t rb = (int64_t)(blockIdx.x / slices) * kDecWarps + warp;
+  const int64_t g = (int64_t)sl * 32 + lane;
+  const bool gok = g < G;
+  // stage the H blocks of the slice (256 bytes per group, 16 floats of padding between)
+  for (int e = threadIdx.x; e < 32 * 2 * kD; e += blockDim.x) {
+    const int gl = e / (2 * kD), q = e % (2 * kD);
+    if ((int64_t)sl * 32 + gl < G)
+      *reinterpret_cast<float4*>(sH + gl * kDecHStride + 4 * q) =
+          __ldg(reinterpret_cast<const float4*>(Hb + ((int64_t)sl * 32 + gl) * kD * kD) + q);
+  }
+  __syncthreads();
+  const int64_t i0 = rb * kDecRows;
+  if (i0 >= M) return;  // whole warps (no block barrier follows)
+  const int nr = (int)min((int64_t)kDecRows, M - i0);
+  const float4* H4 = reinterpret_cast<const float4*>(sH + lane * kDecHStride);
+  for (int r0 = 0; r0 < nr; r0 += kDecBatch) {
+    int32_t kc[kDecBatch][MAXCB];
 #pragma unroll
-  for (int r = 0; r < kDecRows; ++r) {
+    for (int u = 0; u < kDecBatch; ++u) {
+      const int64_t i = i0 + min(r0 + u, nr - 1);
 #pragma unroll
-    for (int off = 16; off > 0; off >>= 1) {
-      const float a0 = __shfl_xor_sync(0xffffffffu, lb[r], off);
-      const float a1 = __shfl_xor_sync(0xffffffffu, lbl[r], off);
-      const float b0 = __shfl_xor_sync(0xffffffffu, lc[r], off);
-      const float b1 = __shfl_xor_sync(0xffffffffu, lcl[r], off);
-      const float c0 = __shfl_xor_sync(0xffffffffu, sq[r], off);
-      const float c1 = __shfl_xor_sync(0xffffffffu, sql[r], off);
-      pair_merge(lb[r], lbl[r], a0, a1);
-      pair_merge(lc[r], lcl[r], b0, b1);
-      pair_merge(sq[r], sql[r], c0, c1);
+      for (int s = 0; s < MAXCB; ++s) {
+        kc[u][s] = -1;
+        if (gok && s < cbs.n && g < cbs.cb[s].G_cov)
+          kc[u][s] = cbs.cb[s].codes[i * cbs.cb[s].ld + g];
+      }
     }
-    if (lane == 0 && r < nr) {
-      float2* o = row_part + ((i0 + r) * slices + sl) * 3;
-      o[0] = make_float2(lb[r], lbl[r]);
-      o[1] = make_float2(lc[r], lcl[r]);
-      o[2] = make_float2(sq[r], sql[r]);
+#pragma unroll
+    for (int u = 0; u < kDecBatch; ++u) {
+      if (r0 + u >= nr) break;
+      const int64_t i = i0 + r0 + u;
+      float lb = 0.f, lc = 0.f, sq = 0.f;
+      if (gok) {
+#pragma unroll
+        for (int s = 0; s < MAXCB; ++s) {
+          if (s >= cbs.n || g >= cbs.cb[s].G_cov) continue;
+          if (kc[u][s] < 0 || kc[u][s] >= cbs.cb[s].K) {
+            raise_error(err, ERRBIT_INDEX);
+            kc[u][s] = -1;
+          }
+        }
+        float rv[kD], dl[kD];
+        recon_codes<MAXCB>(cw, kc[u], cbs.n, rv);
+        const float4 t0 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD);
+        const float4 t1 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD + 4);
+        const float t[kD] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w};
+#pragma unroll
+        for (int j = 0; j < kD; ++j) {
+          dl[j] = t[j] - rv[j];
+          sq = fmaf(dl[j], dl[j], sq);
+        }
+#pragma unroll
+        for (int a = 0; a < kD; ++a) {
+          const float4 h0 = H4[2 * a], h1 = H4[2 * a + 1];
+          float hb = dl[0] * h0.x;
+          hb = fmaf(dl[1], h0.y, hb);
+          hb = fmaf(dl[2], h0.z, hb);
+          hb = fmaf(dl[3], h0.w, hb);
+          hb = fmaf(dl[4], h1.x, hb);
+          hb = fmaf(dl[5], h1.y, hb);
+          hb = fmaf(dl[6], h1.z, hb);
+          hb = fmaf(dl[7], h1.w, hb);
+          lb = fmaf(hb, dl[a], lb);
+        }
+        if (g < n_crit_groups) lc = lb;
+        if (W_rec) {
+          float* o = W_rec + i * N + g * kD;
+          *reinterpret_cast<float4*>(o) = make_float4(rv[0], rv[1], rv[2], rv[3]);
+          *reinterpret_cast<float4*>(o + 4) = make_float4(rv[4], rv[5], rv[6], rv[7]);
+        }
+      }
+      // the 32 vectors of this (row, slice) summed as fp32 pairs in a fixed tree
+      float lbl = 0.f, lcl = 0.f, sql = 0.f;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) {
+        const float a0 = __shfl_xor_sync(0xffffffffu, lb, off);
+        const float a1 = __shfl_xor_sync(0xffffffffu, lbl, off);
+        const float b0 = __shfl_xor_sync(0xffffffffu, lc, off);
+        const float b1 = __shfl_xor_sync(0xffffffffu, lcl, off);
+        const float c0 = __shfl_xor_sync(0xffffffffu, sq, off);
+        const float c1 = __shfl_xor_sync(0xffffffffu, sql, off);
+        pair_merge(lb, lbl, a0, a1);
+        pair_merge(lc, lcl, b0, b1);
+        pair_merge(sq, sql, c0, c1);
+      }
+      if (lane == 0) {
+        float2* o = row_part + (i * slices + sl) * 3;
+        o[0] = make_float2(lb, lbl);
+        o[1] = make_float2(lc, lcl);
+        o[2] = make_float2(sq, sql);
+      }
     }
   }
 }
@@ -228,6 +272,21 @@ finalize_losses_kernel(const float2* __restrict__ row_part, int64_t n_rows,
   }
 }
 
+// The decode kernel's dynamic shared memory (staged H blocks + codebooks) exceeds the default
+// 48 KB: raise its limit once per device.
+template <class K>
+crvq_status dec_smem_attr(K kernel) {
+  static bool done[64] = {};
+  int dev = 0;
+  CRVQ_CUDA(cudaGetDevice(&dev));
+  if (dev < 64 && done[dev]) return CRVQ_OK;
+  CRVQ_CUDA(cudaFuncSetAttribute(
+      kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+      (int)((size_t)32 * kDecHStride * sizeof(float) + kDecSmemCb)));
+  if (dev < 64) done[dev] = true;
+  return CRVQ_OK;
+}
+
 }  // namespace
 
 crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N,
@@ -239,11 +298,9 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   CRVQ_TRY(device_error_word(&err));
   const int nsm = sm_count();
   const int64_t G = N / kD;
-  // warps: kDecRows rows x a slice of the groups; enough slices for ~16 warps per SM
+  // warps: kDecRows rows x a slice of 32 groups
   const int64_t row_blocks = ceil_div(M, (int64_t)kDecRows);
-  const int slices = (int)std::max<int64_t>(
-      1, std::min<int64_t>(ceil_div(16 * (int64_t)nsm * kDecWarps, row_blocks),
-                           ceil_div(G, (int64_t)32)));
+  const int slices = (int)ceil_div(G, (int64_t)32);
   // partial sums of the full loss: one per 128 x 256 tile of dW X^T
   const int64_t n_gemm_cap = X ? ceil_div(M, (int64_t)128) * ceil_div(n_tok, (int64_t)256) : 0;
   int64_t n_gemm = 0;
@@ -265,10 +322,22 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   {
     ProfScope ps("decode_rows", stream,
                  (double)M * N * 4.0 * (1.0 + (W_rec ? 1.0 : 0.0)));
-    const int64_t warps = row_blocks * slices;
-    decode_vec_kernel<<<(unsigned)ceil_div(warps, (int64_t)kDecWarps), kDecWarps * 32, 0,
-                        stream>>>(W_sorted, M, N, Hb, cbs, n_crit_groups, slices, W_rec,
-                                  row_part, err);
+    const int64_t ctas = ceil_div(row_blocks, (int64_t)kDecWarps) * slices;
+    int64_t cb_bytes = 0;
+    for (int s = 0; s < cbs.n; ++s) cb_bytes += (int64_t)cbs.cb[s].K * kD * sizeof(float);
+    const int in_smem = cb_bytes <= kDecSmemCb ? 1 : 0;
+    const size_t smem = (size_t)32 * kDecHStride * sizeof(float) +
+                        (in_smem ? (size_t)cb_bytes : 0);
+    const dim3 grid((unsigned)ctas);
+    if (cbs.n <= 4) {
+      CRVQ_TRY(dec_smem_attr(decode_vec_kernel<4>));
+      decode_vec_kernel<4><<<grid, kDecWarps * 32, smem, stream>>>(
+          W_sorted, M, N, Hb, cbs, n_crit_groups, slices, in_smem, W_rec, row_part, err);
+    } else {
+      CRVQ_TRY(dec_smem_attr(decode_vec_kernel<kMaxCodebooks>));
+      decode_vec_kernel<kMaxCodebooks><<<grid, kDecWarps * 32, smem, stream>>>(
+          W_sorted, M, N, Hb, cbs, n_crit_groups, slices, in_smem, W_rec, row_part, err);
+    }
     CRVQ_LAUNCHED();
   }
   if (W_hat && perm) {  // back to the original channel order: W_hat[:, c] = W_rec[:, inv[c]]
