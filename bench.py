@@ -341,6 +341,57 @@ def coupled_sweep_line(P, work, stream):
             "tensor_work": "2 M N^2 flop per sweep (the lazy block products H[block] D^T)"}
 
 
+def sweep_grid(name):
+    """The synthetic analogs of the paper's ablations on one matrix (no datasets: the block
+    losses stand in for perplexity): Table 2's reorder strategies (random, W-only, W-A), the
+    critical ratio lambda and the number of extended codebooks m - 1 (Sec. 6.3-6.4)."""
+    base = S.C5[0] if name == "c5" else S.CONFIGS[name]
+    grid = []
+    for mode in (2, 1, 0):                                   # Table 2: random, W-only, W-A
+        grid.append(("reorder", base.with_(importance_mode=mode, n_ext=1, crit_frac=0.02)))
+    for lam in (0.01, 0.02, 0.05, 0.10):                     # lambda
+        grid.append(("lambda", base.with_(crit_frac=lam, n_ext=1)))
+    for n_ext in (0, 1, 2, 4):                               # m - 1 extended codebooks
+        grid.append(("m", base.with_(n_ext=n_ext, crit_frac=0.02 if n_ext else 0.02)))
+    return grid
+
+
+def run_sweep(args):
+    """One JSON line per grid point of sweep_grid: losses of the quantized matrix, its time
+    (CUDA events around crvq_quantize_layer, inputs resident) and the average bits per weight
+    of the setting (Eq. bitwidth with e = log2 K, d = 8, the reorder index included)."""
+    import torch
+    import paper_2412_09282_gb300 as P
+    from paper_2412_09282_gb300 import build as B
+    B.build()
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(dev)
+    cache = {}
+    for axis, cfg in sweep_grid(args.config):
+        key = (cfg.name, cfg.x_tag)
+        if key not in cache:
+            cache[key] = (torch.from_numpy(S.gen_W(cfg)).to(dev),
+                          torch.from_numpy(S.gen_X(cfg)).to(dev))
+        W, X = cache[key]
+        out = P.crvq_quantize_layer(W, X, cfg)                # captured / warm
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        out = P.crvq_quantize_layer(W, X, cfg, out=out)
+        b.record(stream)
+        b.synchronize()
+        P.crvq_sync()
+        rep = out.report
+        e = int(np.log2(cfg.K_base))
+        bits = P.crvq_avg_bits(e, cfg.d, 1 + cfg.n_ext, float(cfg.crit_frac), cfg.M, cfg.N, True)
+        print(json.dumps({"sweep": axis, "matrix": cfg.name, "importance_mode": cfg.importance_mode,
+                          "crit_frac": cfg.crit_frac, "n_ext": cfg.n_ext,
+                          "n_crit_groups": rep["n_crit_groups"], "avg_bits": bits,
+                          "loss_block": rep["loss_block"], "loss_crit": rep["loss_crit"],
+                          "loss_full": rep["loss_full"], "loss_pre": rep["loss_pre"],
+                          "ms": a.elapsed_time(b)}), flush=True)
+
+
 def dist_init():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -465,7 +516,13 @@ def main():
     ap.add_argument("--no-infer", action="store_true",
                     help="skip the inference-product and coupled-sweep lines after the timed "
                          "steps")
+    ap.add_argument("--sweep", action="store_true",
+                    help="run the reorder / lambda / m sweep on the workload's first matrix "
+                         "instead of the benchmark (one JSON line per setting)")
     args = ap.parse_args()
+    if args.sweep:
+        run_sweep(args)
+        return
     layers = workload_layers(args.config)
     ws, rank, local = dist_init()
     if args.impl == "reference":

@@ -68,8 +68,14 @@ enum {
   CRVQ_ERR_DEVICE = -7       /* a device-side index check failed (access skipped) */
 };
 
-/* Importance modes (Sec. 4.1; Table 2 "Reorder Strategy"). */
-enum { CRVQ_IMPORTANCE_WA = 0, CRVQ_IMPORTANCE_W_ONLY = 1, CRVQ_IMPORTANCE_RANDOM = 2 };
+/* Importance modes (Sec. 4.1; Table 2 "Reorder Strategy"). WA is the App. A.2 form (the
+ * diagonal of X^T X); WA_INV is Eq. (wa) as printed, with the inverse-Hessian diagonal. */
+enum {
+  CRVQ_IMPORTANCE_WA = 0,
+  CRVQ_IMPORTANCE_W_ONLY = 1,
+  CRVQ_IMPORTANCE_RANDOM = 2,
+  CRVQ_IMPORTANCE_WA_INV = 3
+};
 
 /* One codebook of a vector set (see "Codebooks" above). */
 typedef struct crvq_codebook {
@@ -162,10 +168,25 @@ crvq_status crvq_hessian_blocks(const float* X, int64_t n_tok, int64_t N, int32_
                                 float* H_blocks, crvq_stream_t stream);
 
 /*
+ * The diagonal of the inverse of a symmetric positive definite H (the denominator of Sec. 4.1
+ * Eq. (wa)): hinv[i] = [H^-1]_ii in fp64, from a blocked fp64 Cholesky factor H = L L^T as the
+ * squared column norms of L^-1 (about 2 N^3 / 3 fp64 flops; fp64 because the channel order
+ * it decides must match an fp64 evaluation while cond(H) reaches 1e4 and more).
+ *   H     [N x N] device, symmetric (the lower triangle is read), e.g. crvq_hessian's H.
+ *   hinv  [N] device out (fp64).
+ * A non-positive pivot (H not SPD) is reported as CRVQ_ERR_NUMERIC by crvq_sync.
+ * Requires 1 <= N <= 49152. Scratch: two (N rounded up to 64)^2 fp64 matrices.
+ */
+crvq_status crvq_hessian_inverse_diag(const float* H, int64_t N, double* hinv,
+                                      crvq_stream_t stream);
+
+/*
  * S3. Channel importance and reordering (Alg. 1 ComputeImportance, ReorderChannels;
  * Sec. 4.1-4.2; App. A.2).
  *   mode W-A:    I_i = 1/2 * xsq_i * max_j (W_ji - W_pre_ji)^2 (App. A.2 form; W_pre is the
  *                prequantized W, original order).
+ *   mode W-A inverse: I_i = max_j (W_ji - W_pre_ji)^2 / (2 [H^-1]_ii) (Eq. (wa) as printed;
+ *                diag(H^-1) as crvq_hessian_inverse_diag computes it from H; xsq may be NULL).
  *   mode W-only: I_i = max_j W_ji^2 (Sec. 4.1). W_pre and xsq may be NULL.
  *   mode random: I_i = (SplitMix64(seed, i) >> 40) * 2^-24 (Table 2 "Random").
  * perm sorts channels by I descending, ties by original index (perm[new] = old).

@@ -7,11 +7,12 @@ step of the method on the host; if the library is missing, importing `api` raise
 """
 from .api import (  # noqa: F401
     Codebook, LayerOutputs, crvq_avg_bits, crvq_coupled_sweep, crvq_encode_beam, crvq_hessian,
-    crvq_hessian_blocks,
+    crvq_hessian_blocks, crvq_hessian_inverse_diag,
     crvq_kmeans_init, crvq_lut_matvec, crvq_n_crit_groups, crvq_quantize_layer,
     crvq_reconstruct_error,
     crvq_select_reorder_channels, crvq_sync, crvq_update_codebook_noalloc, crvq_profile_begin,
     crvq_profile_end, crvq_profile_filter, crvq_launch_count, crvq_selftest_bounded_wait,
     crvq_update_codebook,
-    crvq_version, CrvqError, IMPORTANCE_WA, IMPORTANCE_W_ONLY, IMPORTANCE_RANDOM, library_path,
+    crvq_version, CrvqError, IMPORTANCE_WA, IMPORTANCE_W_ONLY, IMPORTANCE_RANDOM,
+    IMPORTANCE_WA_INV, library_path,
 )

@@ -60,6 +60,7 @@ SIGNATURES = {
                                  c_vp, c_vp, c_vp]),
     "crvq_hessian_blocks": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int32, C.c_float,
                                         c_vp, c_vp, c_vp, c_vp, c_vp]),
+    "crvq_hessian_inverse_diag": (C.c_int32, [c_vp, C.c_int64, c_vp, c_vp]),
     "crvq_select_reorder_channels": (C.c_int32, [c_vp, C.c_int64, C.c_int64, C.c_int32, c_vp,
                                                  c_vp, c_vp, C.c_float, C.c_int32, C.c_uint64,
                                                  c_vp, c_vp, c_vp, c_vp, c_i64p, c_vp]),

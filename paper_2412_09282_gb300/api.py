@@ -14,7 +14,7 @@ import torch
 
 from . import _lib
 
-IMPORTANCE_WA, IMPORTANCE_W_ONLY, IMPORTANCE_RANDOM = 0, 1, 2
+IMPORTANCE_WA, IMPORTANCE_W_ONLY, IMPORTANCE_RANDOM, IMPORTANCE_WA_INV = 0, 1, 2, 3
 STATUS = {0: "OK", -1: "INVALID_ARG", -2: "UNSUPPORTED", -3: "CUDA", -4: "NOMEM",
           -5: "TIMEOUT", -6: "NUMERIC", -7: "DEVICE"}
 
@@ -168,6 +168,16 @@ def crvq_hessian_blocks(X, damp_rel, d=8, perm=None, xsq=None, delta=None, H_blo
                                     _ptr(perm), _ptr(xsq),
                                     _ptr(delta), _ptr(H_blocks), _stream(stream, dev)))
     return H_blocks, xsq, delta
+
+
+def crvq_hessian_inverse_diag(H, hinv=None, stream=None):
+    """[H^-1]_ii (fp64, length N) of a symmetric positive definite N x N H (device, fp32)."""
+    _need(H, torch.float32, "H")
+    H = H.contiguous()
+    N = H.shape[0]
+    hinv = torch.empty(N, device=H.device, dtype=torch.float64) if hinv is None else hinv
+    _check(_L().crvq_hessian_inverse_diag(_ptr(H), N, _ptr(hinv), _stream(stream, H.device)))
+    return hinv
 
 
 def crvq_select_reorder_channels(W, d, W_pre, xsq, H, crit_frac, mode=IMPORTANCE_WA, seed=0,

@@ -76,6 +76,33 @@ int sm_count() {
   return g_sm[dev];
 }
 
+namespace {
+struct SmemLimit {
+  const void* kernel;
+  int dev;
+  size_t bytes;
+};
+std::vector<SmemLimit> g_smem_limits;
+}  // namespace
+
+crvq_status smem_limit(const void* kernel, size_t bytes) {
+  int dev = 0;
+  CRVQ_CUDA(cudaGetDevice(&dev));
+  std::lock_guard<std::mutex> lk(g_mu);
+  for (auto& e : g_smem_limits)
+    if (e.kernel == kernel && e.dev == dev) {
+      if (e.bytes >= bytes) return CRVQ_OK;
+      CRVQ_CUDA(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                     (int)bytes));
+      e.bytes = bytes;
+      return CRVQ_OK;
+    }
+  CRVQ_CUDA(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)bytes));
+  g_smem_limits.push_back(SmemLimit{kernel, dev, bytes});
+  return CRVQ_OK;
+}
+
 // ------------------------------------------------------------------------- launch stats
 namespace {
 std::atomic<long long> g_launches{0};
@@ -420,6 +447,15 @@ crvq_status crvq_hessian_blocks(const float* X, int64_t n_tok, int64_t N, int32_
   return CRVQ_OK;
 }
 
+crvq_status crvq_hessian_inverse_diag(const float* H, int64_t N, double* hinv,
+                                      crvq_stream_t stream) {
+  clear_last_error();
+  CRVQ_CHECK_ARG(H && hinv, "H and hinv must not be NULL");
+  CRVQ_CHECK_ARG(N >= 1 && N <= 49152, "N must be in [1, 49152]");
+  CRVQ_TRY(check_dev({{H, "H"}, {hinv, "hinv"}}));
+  return launch_hinv_diag(H, N, hinv, (cudaStream_t)stream);
+}
+
 int64_t crvq_n_crit_groups(int64_t N, int32_t d, float crit_frac) {
   if (d <= 0 || N <= 0 || !(crit_frac > 0.f)) return 0;
   const int64_t G = N / d;
@@ -439,8 +475,9 @@ crvq_status crvq_select_reorder_channels(const float* W, int64_t M, int64_t N, i
   CRVQ_CHECK_ARG(M >= 1 && N >= 1 && N % d == 0, "need M >= 1, N >= 1, N %% d == 0");
   CRVQ_CHECK_ARG(N <= 49152, "N must be <= 49152");
   CRVQ_CHECK_ARG(crit_frac >= 0.f && crit_frac <= 1.f, "crit_frac must be in [0, 1]");
-  CRVQ_CHECK_ARG(mode >= 0 && mode <= 2, "unknown importance mode %d", mode);
+  CRVQ_CHECK_ARG(mode >= 0 && mode <= 3, "unknown importance mode %d", mode);
   if (mode == CRVQ_IMPORTANCE_WA) CRVQ_CHECK_ARG(W_pre && xsq, "W-A mode needs W_pre and xsq");
+  if (mode == CRVQ_IMPORTANCE_WA_INV) CRVQ_CHECK_ARG(W_pre, "W-A inverse mode needs W_pre");
   CRVQ_CHECK_ARG(aligned16(W) && aligned16(W_sorted) && (!W_pre || aligned16(W_pre)),
                  "W, W_pre and W_sorted must be 16-byte aligned");
   CRVQ_TRY(check_dev({{W, "W"}, {W_pre, "W_pre"}, {xsq, "xsq"}, {H, "H"}, {perm, "perm"},
@@ -747,8 +784,18 @@ crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, i
     CRVQ_TRY(launch_reconstruct_error(W, M, N, Hb0, nullptr, cl, 0, nullptr, 0, 0.0, nullptr,
                                       Wpre, losses + 3, s));
   }
-  // S3: importance and reordering (Alg. 1, importance and reordering steps)
-  CRVQ_TRY(launch_select_reorder(W, M, N, d, Wpre, xsq, nullptr, cfg->importance_mode,
+  // S3: importance and reordering (Alg. 1, importance and reordering steps); Eq. (wa) as
+  // printed needs diag(H^-1), hence the dense H
+  Buf bHd;
+  float* Hd = nullptr;
+  if (cfg->importance_mode == CRVQ_IMPORTANCE_WA_INV) {
+    CRVQ_TRY(bHd.get(&Hd, (size_t)N * N, s));
+    Buf bx2;
+    float* xsq2 = nullptr;
+    CRVQ_TRY(bx2.get(&xsq2, N, s));
+    CRVQ_TRY(launch_hessian(X, n_tok, N, d, cfg->damp_rel, Hd, xsq2, nullptr, nullptr, s));
+  }
+  CRVQ_TRY(launch_select_reorder(W, M, N, d, Wpre, xsq, Hd, cfg->importance_mode,
                                  phase_seed(cfg->seed, 4, 0), o.perm, o.imp, Ws, nullptr, s));
   CRVQ_TRY(launch_tc_hessian_blocks(Xt, ldt, n_tok, N, o.perm, true, 0.f, nullptr, nullptr,
                                     delta64, Hb, s));
@@ -1092,7 +1139,7 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   CRVQ_CHECK_ARG(cfg->crit_frac >= 0.f && cfg->crit_frac <= 1.f, "crit_frac must be in [0, 1]");
   CRVQ_CHECK_ARG(cfg->B >= 1 && cfg->B <= 16, "B must be in [1, 16]");
   CRVQ_CHECK_ARG(cfg->kmeans_iters >= 0 && cfg->refine_rounds >= 0, "negative iteration count");
-  CRVQ_CHECK_ARG(cfg->importance_mode >= 0 && cfg->importance_mode <= 2, "bad importance mode");
+  CRVQ_CHECK_ARG(cfg->importance_mode >= 0 && cfg->importance_mode <= 3, "bad importance mode");
   CRVQ_CHECK_ARG(std::isfinite(cfg->damp_rel) && cfg->damp_rel >= 0.f, "bad damp_rel");
   const int64_t Gc = crvq_n_crit_groups(N, d, cfg->crit_frac);
   if (cfg->n_ext > 0) {

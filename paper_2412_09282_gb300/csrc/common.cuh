@@ -128,6 +128,11 @@ inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 // Number of SMs of the current device (cached per device).
 int sm_count();
 
+// Raises `kernel`'s dynamic shared-memory limit on the current device to at least `bytes`,
+// calling cudaFuncSetAttribute only when a larger limit than before is needed (remembered per
+// kernel address and device).
+crvq_status smem_limit(const void* kernel, size_t bytes);
+
 // ---------------------------------------------------------------- device helpers
 // SplitMix64 (Steele, Lea & Flood 2014): output `ctr` (0-based) of the stream `stream`.
 __host__ __device__ inline uint64_t splitmix64(uint64_t stream, uint64_t ctr) {

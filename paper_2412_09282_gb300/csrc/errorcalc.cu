@@ -272,21 +272,6 @@ finalize_losses_kernel(const float2* __restrict__ row_part, int64_t n_rows,
   }
 }
 
-// The decode kernel's dynamic shared memory (staged H blocks + codebooks) exceeds the default
-// 48 KB: raise its limit once per device.
-template <class K>
-crvq_status dec_smem_attr(K kernel) {
-  static bool done[64] = {};
-  int dev = 0;
-  CRVQ_CUDA(cudaGetDevice(&dev));
-  if (dev < 64 && done[dev]) return CRVQ_OK;
-  CRVQ_CUDA(cudaFuncSetAttribute(
-      kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-      (int)((size_t)32 * kDecHStride * sizeof(float) + kDecSmemCb)));
-  if (dev < 64) done[dev] = true;
-  return CRVQ_OK;
-}
-
 }  // namespace
 
 crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N,
@@ -330,11 +315,11 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
                         (in_smem ? (size_t)cb_bytes : 0);
     const dim3 grid((unsigned)ctas);
     if (cbs.n <= 4) {
-      CRVQ_TRY(dec_smem_attr(decode_vec_kernel<4>));
+      CRVQ_TRY(smem_limit((const void*)decode_vec_kernel<4>, smem));
       decode_vec_kernel<4><<<grid, kDecWarps * 32, smem, stream>>>(
           W_sorted, M, N, Hb, cbs, n_crit_groups, slices, in_smem, W_rec, row_part, err);
     } else {
-      CRVQ_TRY(dec_smem_attr(decode_vec_kernel<kMaxCodebooks>));
+      CRVQ_TRY(smem_limit((const void*)decode_vec_kernel<kMaxCodebooks>, smem));
       decode_vec_kernel<kMaxCodebooks><<<grid, kDecWarps * 32, smem, stream>>>(
           W_sorted, M, N, Hb, cbs, n_crit_groups, slices, in_smem, W_rec, row_part, err);
     }

@@ -203,19 +203,6 @@ matvec_reduce_kernel(const float* __restrict__ part, int64_t n_slices, int64_t M
   }
 }
 
-// Raises a slice kernel's dynamic shared-memory limit to the per-CTA cap, once per device.
-template <class K>
-crvq_status smem_attr_once(K kernel) {
-  static bool done[64] = {};
-  int dev = 0;
-  CRVQ_CUDA(cudaGetDevice(&dev));
-  if (dev < 64 && done[dev]) return CRVQ_OK;
-  CRVQ_CUDA(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)(kLutSmemCap + kMaxBatch * kSliceG * kD * sizeof(float))));
-  if (dev < 64) done[dev] = true;
-  return CRVQ_OK;
-}
-
 }  // namespace
 
 size_t lut_matvec_smem(const CbList& cbs, int b, int* lut_mask) {
@@ -262,7 +249,7 @@ crvq_status launch_lut_matvec(const float* X, int64_t ldx, int64_t N, int b,
   {
     ProfScope ps("matvec_slices", stream, (double)M * G * cbs.n);
     auto go = [&](auto kernel) -> crvq_status {
-      CRVQ_TRY(smem_attr_once(kernel));
+      CRVQ_TRY(smem_limit((const void*)kernel, smem));
       kernel<<<grid, kMvThreads, smem, stream>>>(a, rows_per_cta, err);
       return CRVQ_OK;
     };

@@ -53,6 +53,10 @@ crvq_status launch_tc_gemm_nt(const float* A, int64_t lda, int64_t M, const floa
                               int64_t ldb, int64_t Nb, int64_t K, float* C, int64_t ldc,
                               cudaStream_t stream);
 
+// hinv[i] = [H^-1]_ii (fp64) of a symmetric positive definite H (N x N fp32): blocked fp64
+// Cholesky, the inverse factor by blocked forward substitution, squared column norms.
+crvq_status launch_hinv_diag(const float* H, int64_t N, double* hinv, cudaStream_t stream);
+
 crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
                                   const float* W_pre, const float* xsq, const float* H,
                                   int mode, uint64_t seed, int32_t* perm, float* importance,

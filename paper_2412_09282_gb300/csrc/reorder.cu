@@ -61,13 +61,18 @@ colmax_kernel(const float* __restrict__ W, const float* __restrict__ W_pre, int6
 }
 
 __global__ void importance_kernel(const unsigned* __restrict__ maxbits,
-                                  const float* __restrict__ xsq, int64_t N, int mode,
+                                  const float* __restrict__ xsq,
+                                  const double* __restrict__ hinv, int64_t N, int mode,
                                   uint64_t seed, float* __restrict__ I) {
   for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < N;
        i += (int64_t)gridDim.x * blockDim.x) {
     float v;
     if (mode == CRVQ_IMPORTANCE_RANDOM) {
       v = (float)(splitmix64(seed, (uint64_t)i) >> 40) * 5.9604645e-08f;  // 24 bits * 2^-24
+    } else if (mode == CRVQ_IMPORTANCE_WA_INV) {
+      // Eq. (wa): max_j dw_ji^2 / (2 [H^-1]_ii), in fp64, rounded once
+      const double m = (double)__uint_as_float(maxbits[i]);
+      v = (float)(m * m / (2.0 * hinv[i]));
     } else {
       const float m = __uint_as_float(maxbits[i]);
       v = m * m;
@@ -134,10 +139,17 @@ crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
   unsigned* err = nullptr;
   CRVQ_TRY(device_error_word(&err));
   const int nsm = sm_count();
-  Scratch mem;
+  Scratch mem, mh;
   CRVQ_TRY(mem.alloc((size_t)N * (sizeof(unsigned) + sizeof(float)), stream));
   unsigned* maxbits = mem.as<unsigned>();
   float* I = importance ? importance : reinterpret_cast<float*>(maxbits + N);
+  double* hinv = nullptr;
+  if (mode == CRVQ_IMPORTANCE_WA_INV) {
+    CRVQ_TRY(mh.alloc((size_t)N * sizeof(double), stream));
+    hinv = mh.as<double>();
+    CRVQ_TRY(launch_hinv_diag(H, N, hinv, stream));
+  }
+  const bool with_pre = mode == CRVQ_IMPORTANCE_WA || mode == CRVQ_IMPORTANCE_WA_INV;
   if (mode != CRVQ_IMPORTANCE_RANDOM) {
     CRVQ_CUDA(cudaMemsetAsync(maxbits, 0, (size_t)N * sizeof(unsigned), stream));
     const int64_t col_blocks = ceil_div(N, kColThreads * 4);
@@ -146,13 +158,12 @@ crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
     row_blocks = std::min<int64_t>(row_blocks, ceil_div(M, kRowThreads));
     const int64_t rows_per = ceil_div(M, row_blocks);
     dim3 grid((unsigned)col_blocks, (unsigned)ceil_div(M, rows_per));
-    ProfScope ps("reorder_colmax", stream,
-                 (double)M * N * 4.0 * (mode == CRVQ_IMPORTANCE_WA ? 2.0 : 1.0));
+    ProfScope ps("reorder_colmax", stream, (double)M * N * 4.0 * (with_pre ? 2.0 : 1.0));
     colmax_kernel<<<grid, kColThreads * kRowThreads, 0, stream>>>(
-        W, mode == CRVQ_IMPORTANCE_WA ? W_pre : nullptr, M, N, rows_per, maxbits, err);
+        W, with_pre ? W_pre : nullptr, M, N, rows_per, maxbits, err);
     CRVQ_LAUNCHED();
   }
-  importance_kernel<<<(unsigned)ceil_div(N, 256), 256, 0, stream>>>(maxbits, xsq, N, mode,
+  importance_kernel<<<(unsigned)ceil_div(N, 256), 256, 0, stream>>>(maxbits, xsq, hinv, N, mode,
                                                                      seed, I);
   CRVQ_LAUNCHED();
   {

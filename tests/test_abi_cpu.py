@@ -165,7 +165,7 @@ def test_quantize_layer_rejects_bad_shapes_and_options_before_launch(lib):
     assert call(crit_frac=1.5) == -1
     assert call(B=17) == -1
     assert call(kmeans_iters=-1) == -1
-    assert call(importance_mode=3) == -1
+    assert call(importance_mode=4) == -1
     assert call(damp_rel=-1.0) == -1
     assert call(crit_frac=0.0) == -1              # extended codebooks need a critical group
     assert b"critical" in lib.crvq_last_error()
