@@ -260,9 +260,9 @@ crvq_status crvq_update_codebook(const float* T, int64_t ldT, int64_t M, int64_t
  * CRVQ_ERR_INVALID_ARG), results and rounding are those of crvq_update_codebook; the caller
  * still passes the inputs and outputs. Its scratch is one file-scope device array of 4 MiB,
  * held by every GPU that loads the library until the process exits:
- *  - sizes whose statistics exceed it (G_cov * K * 4 + K * 64 + 256 bytes, each part rounded
- *    up to 256 bytes, above 4 MiB; e.g. K = 256 with more than ~4000 covered groups)
- *    return CRVQ_ERR_UNSUPPORTED before anything is enqueued;
+ *  - sizes whose statistics exceed it (G_cov * K * 4 + K * 64 + 256 + K * 296 bytes, each
+ *    part rounded up to 256 bytes, above 4 MiB; e.g. K = 256 with more than ~3900 covered
+ *    groups) return CRVQ_ERR_UNSUPPORTED before anything is enqueued;
  *  - every call shares the array and it keeps the last call's contents: each call clears
  *    what must start at zero, and calls that overlap on the GPU (on different streams, or
  *    host threads enqueueing on one device without ordering) race;

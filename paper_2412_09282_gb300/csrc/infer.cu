@@ -6,16 +6,17 @@
 //   y[bi][i] = sum over codebooks s and groups g < G_cov(s) of <C_s[codes_s(i, g)], xs[bi][g]>,
 //   xs[bi][p] = X_in[bi][perm[p]]   (the inputs taken once in the sorted channel order).
 //
-// Layout: a CTA owns one slice of 32 groups and a block of rows. It gathers its slice of the
-// inputs through the permutation into shared memory and, for codebooks small enough, the
-// lookup tables lut[g][k][bi] = <C[k], xs[bi][g]> of its 32 groups (codewords read from L2
-// once per CTA); a warp then takes one row at a time with lane l on group g0 + l, so that the
-// 32 codes of a row slice are one coalesced 128-byte read and each lookup is one shared-memory
-// load. Codebooks whose tables do not fit are dotted directly (the codeword from L2, eight FMAs
-// per input). Each row slice is reduced across the warp (shuffles, a fixed tree) into a
-// partial; a second kernel adds the partials of a row in slice order, so results are
-// identical on every run. The codes are the only per-element stream from HBM (4 bytes per
-// code), which makes the kernel bound by HBM bandwidth.
+// Layout: a CTA owns one slice of 32 groups and a block of 128 rows. It first issues every
+// load it needs at once: the base codebook's codes of its tile (128 rows x 32 codes, coalesced
+// 128-byte reads, into shared memory) and its slice of the inputs through the permutation.
+// It then builds the slice's lookup tables lut[g][k][bi] = <C_base[k], xs[bi][g]> in shared
+// memory (a thread per codeword, loaded once; tables that would not fit are skipped and the
+// codewords dotted from L2). A warp takes one row at a time, lane = group: a shared-memory
+// code, a shared-memory table entry; the extended codebooks, which cover only the first G_c
+// groups, are dotted from L2. Each row slice is reduced across the warp (a fixed shuffle tree)
+// into a partial, and the last CTA of a row block to finish adds the partials of its rows in
+// slice order, so results are identical on every run. The codes are the only per-element
+// stream from HBM (4 bytes per code).
 #include <algorithm>
 
 #include "common.cuh"
@@ -27,9 +28,9 @@ namespace {
 
 constexpr int kSliceG = 32;     // groups per CTA slice (one per lane)
 constexpr int kMvThreads = 256;
+constexpr int kMvRows = 128;    // rows per CTA
 constexpr int kMaxBatch = 8;
-constexpr size_t kLutSmemCap = 160 * 1024;  // shared memory for lookup tables per CTA
-constexpr int kRowBatch = 8;    // rows a warp reads codes for before using any
+constexpr size_t kLutSmemCap = 96 * 1024;  // the base codebook's tables per CTA at most
 
 struct MatvecArgs {
   const float* X;       // b x N, row stride ldx
@@ -39,9 +40,12 @@ struct MatvecArgs {
   CbList cbs;
   int64_t M;
   int b;
-  int lut_mask;         // bit s: codebook s uses a shared-memory lookup table
+  int base_lut;         // the base codebook (cbs.cb[0]) uses shared-memory lookup tables
   int64_t n_slices;
   float* part;          // [n_slices][b][M]
+  unsigned* done;       // per row block: CTAs finished (zero on entry)
+  float* Y;             // b x M, row stride ldy
+  int64_t ldy;
 };
 
 __device__ __forceinline__ float warp_sum(float v) {
@@ -50,28 +54,52 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// Partial products of one (row block, group slice): part[slice][bi][i].
-template <int BMAX, int MAXCB>
+__device__ __forceinline__ float dot8(const float* __restrict__ c, const float* x) {
+  const float4 c0 = __ldg(reinterpret_cast<const float4*>(c));
+  const float4 c1 = __ldg(reinterpret_cast<const float4*>(c + 4));
+  float v = c0.x * x[0];
+  v = fmaf(c0.y, x[1], v);
+  v = fmaf(c0.z, x[2], v);
+  v = fmaf(c0.w, x[3], v);
+  v = fmaf(c1.x, x[4], v);
+  v = fmaf(c1.y, x[5], v);
+  v = fmaf(c1.z, x[6], v);
+  v = fmaf(c1.w, x[7], v);
+  return v;
+}
+
+// Partial products of one (row block, group slice), and the ordered sum of a row block's
+// partials by the last of its CTAs.
+template <int BMAX>
 __global__ void __launch_bounds__(kMvThreads)
-matvec_slice_kernel(MatvecArgs a, int rows_per_cta, unsigned* err) {
+matvec_slice_kernel(MatvecArgs a, unsigned* err) {
   extern __shared__ __align__(16) float sm[];
-  float* xs = sm;                             // [b][kSliceG][8]
-  float* lut = sm + a.b * kSliceG * kD;       // per LUT codebook: [kSliceG][K][b]
-  const int64_t slice = blockIdx.y;
+  float* xs = sm;                                          // [b][kSliceG][8]
+  int32_t* scode = reinterpret_cast<int32_t*>(xs + kMaxBatch * kSliceG * kD);  // [rows][32]
+  float* lut = reinterpret_cast<float*>(scode + kMvRows * kSliceG);            // [32][K][b]
+  __shared__ int s_last;
+  const int64_t slice = blockIdx.y, rblk = blockIdx.x;
   const int64_t g0 = slice * kSliceG;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int64_t G = a.N / kD;
   const int gn = (int)(G - g0 < kSliceG ? G - g0 : kSliceG);
+  const int64_t r0 = rblk * kMvRows;
+  const int nr = (int)(a.M - r0 < kMvRows ? a.M - r0 : kMvRows);
+  const CbView& cb0 = a.cbs.cb[0];
 
-  // inputs of this slice in the sorted order
+  // every load of the tile at once: the base codes (coalesced rows of 32 codes) and the inputs
+  for (int e = tid; e < nr * kSliceG; e += blockDim.x) {
+    const int r = e / kSliceG, l = e % kSliceG;
+    const int64_t g = g0 + l;
+    scode[e] = (l < gn && g < cb0.G_cov) ? cb0.codes[(r0 + r) * cb0.ld + g] : -1;
+  }
   for (int e = tid; e < a.b * kSliceG * kD; e += blockDim.x) {
     const int bi = e / (kSliceG * kD), r = e % (kSliceG * kD);
-    const int64_t p = g0 * kD + r;
     float v = 0.f;
     if (r < gn * kD) {
-      int64_t src = p;
+      int64_t src = g0 * kD + r;
       if (a.perm) {
-        src = a.perm[p];
+        src = a.perm[src];
         if (src < 0 || src >= a.N) {
           raise_error(err, ERRBIT_INDEX);
           src = -1;
@@ -82,142 +110,74 @@ matvec_slice_kernel(MatvecArgs a, int rows_per_cta, unsigned* err) {
     xs[e] = v;
   }
   __syncthreads();
-  // lookup tables of the codebooks that have one: lut[g][k][bi] = <C[k], xs[bi][g]>; a thread
-  // takes one codeword (loaded once) across the slice's groups
-  {
-    float* t = lut;
-    for (int s = 0; s < a.cbs.n; ++s) {
-      if (!((a.lut_mask >> s) & 1)) continue;
-      const CbView& cb = a.cbs.cb[s];
-      const int64_t gcov = cb.G_cov - g0;
-      const int gc = gcov <= 0 ? 0 : (int)(gcov < gn ? gcov : gn);
-      for (int k = tid; k < cb.K && gc > 0; k += blockDim.x) {
-        const float4 c0 = __ldg(reinterpret_cast<const float4*>(cb.C + (int64_t)k * kD));
-        const float4 c1 = __ldg(reinterpret_cast<const float4*>(cb.C + (int64_t)k * kD + 4));
-        for (int gl = 0; gl < gc; ++gl)
-          for (int bi = 0; bi < a.b; ++bi) {
-            const float* x = xs + (bi * kSliceG + gl) * kD;
-            float v = c0.x * x[0];
-            v = fmaf(c0.y, x[1], v);
-            v = fmaf(c0.z, x[2], v);
-            v = fmaf(c0.w, x[3], v);
-            v = fmaf(c1.x, x[4], v);
-            v = fmaf(c1.y, x[5], v);
-            v = fmaf(c1.z, x[6], v);
-            v = fmaf(c1.w, x[7], v);
-            t[((int64_t)gl * cb.K + k) * a.b + bi] = v;
-          }
-      }
-      t += (int64_t)kSliceG * cb.K * a.b;
+  // the base codebook's tables: a thread per codeword, loaded once, across the slice's groups
+  if (a.base_lut) {
+    for (int k = tid; k < cb0.K; k += blockDim.x) {
+      const float* c = cb0.C + (int64_t)k * kD;
+      for (int gl = 0; gl < gn; ++gl)
+        for (int bi = 0; bi < a.b; ++bi)
+          lut[((int64_t)gl * cb0.K + k) * a.b + bi] = dot8(c, xs + (bi * kSliceG + gl) * kD);
     }
+    __syncthreads();
   }
-  __syncthreads();
 
-  // rows of this block: a warp takes kRowBatch rows at a time, lane = group g0 + lane; the
-  // codes of every row and codebook of the batch are loaded before any is used, so that each
-  // warp keeps kRowBatch x n_cb coalesced 128-byte reads in flight (the kernel is bound by the
-  // latency of these reads otherwise)
-  const int64_t r0 = (int64_t)blockIdx.x * rows_per_cta;
-  const int64_t r1 = a.M < r0 + rows_per_cta ? a.M : r0 + rows_per_cta;
-  const int nwarps = blockDim.x >> 5;
   const int64_t g = g0 + lane;
-  for (int64_t ib = r0 + (int64_t)warp * kRowBatch; ib < r1; ib += (int64_t)nwarps * kRowBatch) {
-    int32_t kc[MAXCB][kRowBatch];
+  for (int r = warp; r < nr; r += kMvThreads / 32) {
+    const int64_t i = r0 + r;
+    float acc[BMAX];
 #pragma unroll
-    for (int s = 0; s < MAXCB; ++s) {
-      const bool cov = s < a.cbs.n && lane < gn && g < a.cbs.cb[s].G_cov;
+    for (int bi = 0; bi < BMAX; ++bi) acc[bi] = 0.f;
+    const int32_t k = scode[r * kSliceG + lane];
+    if (lane < gn && g < cb0.G_cov) {
+      if (k < 0 || k >= cb0.K) {
+        raise_error(err, ERRBIT_INDEX);
+      } else if (a.base_lut) {
+        const float* e = lut + ((int64_t)lane * cb0.K + k) * a.b;
 #pragma unroll
-      for (int u = 0; u < kRowBatch; ++u) {
-        const int64_t i = ib + u;
-        kc[s][u] = (cov && i < r1) ? __ldg(a.cbs.cb[s].codes + i * a.cbs.cb[s].ld + g) : -1;
+        for (int bi = 0; bi < BMAX; ++bi)
+          if (bi < a.b) acc[bi] += e[bi];
+      } else {
+#pragma unroll
+        for (int bi = 0; bi < BMAX; ++bi)
+          if (bi < a.b) acc[bi] += dot8(cb0.C + (int64_t)k * kD, xs + (bi * kSliceG + lane) * kD);
       }
     }
-    float acc[kRowBatch][BMAX];
-#pragma unroll
-    for (int u = 0; u < kRowBatch; ++u)
-#pragma unroll
-      for (int bi = 0; bi < BMAX; ++bi) acc[u][bi] = 0.f;
-    const float* t = lut;
-#pragma unroll
-    for (int s = 0; s < MAXCB; ++s) {
-      if (s >= a.cbs.n) break;
+    for (int s = 1; s < a.cbs.n; ++s) {  // extended codebooks: the first G_c groups only
       const CbView& cb = a.cbs.cb[s];
-      const bool cov = lane < gn && g < cb.G_cov;
-      const bool has_lut = (a.lut_mask >> s) & 1;
-#pragma unroll
-      for (int u = 0; u < kRowBatch; ++u) {
-        const int32_t k = kc[s][u];
-        if (!cov || ib + u >= r1) continue;
-        if (k < 0 || k >= cb.K) {
-          raise_error(err, ERRBIT_INDEX);
-        } else if (has_lut) {
-          const float* e = t + ((int64_t)lane * cb.K + k) * a.b;
-#pragma unroll
-          for (int bi = 0; bi < BMAX; ++bi)
-            if (bi < a.b) acc[u][bi] += e[bi];
-        } else {
-          const float4 c0 = __ldg(reinterpret_cast<const float4*>(cb.C + (int64_t)k * kD));
-          const float4 c1 = __ldg(reinterpret_cast<const float4*>(cb.C + (int64_t)k * kD + 4));
-#pragma unroll
-          for (int bi = 0; bi < BMAX; ++bi) {
-            if (bi >= a.b) break;
-            const float* x = xs + (bi * kSliceG + lane) * kD;
-            float v = c0.x * x[0];
-            v = fmaf(c0.y, x[1], v);
-            v = fmaf(c0.z, x[2], v);
-            v = fmaf(c0.w, x[3], v);
-            v = fmaf(c1.x, x[4], v);
-            v = fmaf(c1.y, x[5], v);
-            v = fmaf(c1.z, x[6], v);
-            v = fmaf(c1.w, x[7], v);
-            acc[u][bi] += v;
-          }
-        }
+      if (!(lane < gn && g < cb.G_cov)) continue;
+      const int32_t ke = cb.codes[i * cb.ld + g];
+      if (ke < 0 || ke >= cb.K) {
+        raise_error(err, ERRBIT_INDEX);
+        continue;
       }
-      if (has_lut) t += (int64_t)kSliceG * cb.K * a.b;
+#pragma unroll
+      for (int bi = 0; bi < BMAX; ++bi)
+        if (bi < a.b) acc[bi] += dot8(cb.C + (int64_t)ke * kD, xs + (bi * kSliceG + lane) * kD);
     }
 #pragma unroll
-    for (int u = 0; u < kRowBatch; ++u) {
-      const int64_t i = ib + u;
-#pragma unroll
-      for (int bi = 0; bi < BMAX; ++bi) {
-        if (bi >= a.b) break;
-        const float v = warp_sum(acc[u][bi]);
-        if (lane == 0 && i < r1) a.part[(slice * a.b + bi) * a.M + i] = v;
-      }
+    for (int bi = 0; bi < BMAX; ++bi) {
+      if (bi >= a.b) break;
+      const float v = warp_sum(acc[bi]);
+      if (lane == 0) a.part[(slice * a.b + bi) * a.M + i] = v;
     }
   }
-}
-
-// y[bi][i] = sum of the slice partials in slice order.
-__global__ void __launch_bounds__(256)
-matvec_reduce_kernel(const float* __restrict__ part, int64_t n_slices, int64_t M, int b,
-                     float* __restrict__ Y, int64_t ldy) {
-  const int64_t n = (int64_t)b * M;
-  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n;
-       e += (int64_t)gridDim.x * blockDim.x) {
-    const int64_t bi = e / M, i = e % M;
-    float s = 0.f;
-    for (int64_t q = 0; q < n_slices; ++q) s += part[(q * b + bi) * M + i];
-    Y[bi * ldy + i] = s;
+  // the last CTA of this row block adds the slices' partials of its rows, in slice order
+  __threadfence();
+  __syncthreads();
+  if (tid == 0) s_last = atomicAdd(&a.done[rblk], 1u) == (unsigned)(a.n_slices - 1);
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  for (int e = tid; e < nr * a.b; e += blockDim.x) {
+    const int bi = e / nr;
+    const int64_t i = r0 + e % nr;
+    float sum = 0.f;
+    for (int64_t q = 0; q < a.n_slices; ++q) sum += __ldcg(a.part + (q * a.b + bi) * a.M + i);
+    a.Y[bi * a.ldy + i] = sum;
   }
 }
 
 }  // namespace
-
-size_t lut_matvec_smem(const CbList& cbs, int b, int* lut_mask) {
-  size_t bytes = (size_t)b * kSliceG * kD * sizeof(float);
-  int mask = 0;
-  for (int s = 0; s < cbs.n; ++s) {
-    const size_t t = (size_t)kSliceG * cbs.cb[s].K * b * sizeof(float);
-    if (bytes + t <= kLutSmemCap) {
-      bytes += t;
-      mask |= 1 << s;
-    }
-  }
-  if (lut_mask) *lut_mask = mask;
-  return bytes;
-}
 
 crvq_status launch_lut_matvec(const float* X, int64_t ldx, int64_t N, int b,
                               const int32_t* perm, const CbList& cbs, int64_t M, float* Y,
@@ -237,40 +197,33 @@ crvq_status launch_lut_matvec(const float* X, int64_t ldx, int64_t N, int b,
   a.M = M;
   a.b = b;
   a.n_slices = ceil_div(G, kSliceG);
-  const size_t smem = lut_matvec_smem(cbs, b, &a.lut_mask);
-  Scratch part;
-  CRVQ_TRY(part.alloc((size_t)a.n_slices * b * M * sizeof(float), stream));
-  a.part = part.as<float>();
-  const int nsm = sm_count();
-  const int64_t row_blocks = std::max<int64_t>(
-      1, std::min<int64_t>(ceil_div(M, 8), ceil_div(2 * (int64_t)nsm, a.n_slices)));
-  const int rows_per_cta = (int)ceil_div(M, row_blocks);
-  const dim3 grid((unsigned)ceil_div(M, rows_per_cta), (unsigned)a.n_slices);
-  {
-    ProfScope ps("matvec_slices", stream, (double)M * G * cbs.n);
-    auto go = [&](auto kernel) -> crvq_status {
-      CRVQ_TRY(smem_limit((const void*)kernel, smem));
-      kernel<<<grid, kMvThreads, smem, stream>>>(a, rows_per_cta, err);
-      return CRVQ_OK;
-    };
-    if (b == 1 && cbs.n <= 4) {
-      CRVQ_TRY(go(matvec_slice_kernel<1, 4>));
-    } else if (b == 1) {
-      CRVQ_TRY(go(matvec_slice_kernel<1, kMaxCodebooks>));
-    } else if (b <= 4 && cbs.n <= 4) {
-      CRVQ_TRY(go(matvec_slice_kernel<4, 4>));
-    } else {
-      CRVQ_TRY(go(matvec_slice_kernel<kMaxBatch, kMaxCodebooks>));
-    }
-    CRVQ_LAUNCHED();
-  }
-  {
-    ProfScope ps("matvec_reduce", stream, (double)b * M);
-    const int64_t n = (int64_t)b * M;
-    matvec_reduce_kernel<<<(unsigned)std::min<int64_t>(ceil_div(n, 256), 8 * nsm), 256, 0,
-                           stream>>>(a.part, a.n_slices, M, b, Y, ldy);
-    CRVQ_LAUNCHED();
-  }
+  a.Y = Y;
+  a.ldy = ldy;
+  const size_t lut_bytes = (size_t)kSliceG * cbs.cb[0].K * b * sizeof(float);
+  a.base_lut = lut_bytes <= kLutSmemCap ? 1 : 0;
+  const size_t smem = (size_t)kMaxBatch * kSliceG * kD * sizeof(float) +
+                      (size_t)kMvRows * kSliceG * sizeof(int32_t) + (a.base_lut ? lut_bytes : 0);
+  const int64_t row_blocks = ceil_div(M, (int64_t)kMvRows);
+  const size_t part_bytes = align_up((size_t)a.n_slices * b * M * sizeof(float), 256);
+  Scratch mem;
+  CRVQ_TRY(mem.alloc(part_bytes + (size_t)row_blocks * sizeof(unsigned), stream));
+  a.part = mem.as<float>();
+  a.done = reinterpret_cast<unsigned*>(mem.as<char>() + part_bytes);
+  CRVQ_CUDA(cudaMemsetAsync(a.done, 0, (size_t)row_blocks * sizeof(unsigned), stream));
+  const dim3 grid((unsigned)row_blocks, (unsigned)a.n_slices);
+  ProfScope ps("matvec_slices", stream, (double)M * G * cbs.n);
+  auto go = [&](auto kernel) -> crvq_status {
+    CRVQ_TRY(smem_limit((const void*)kernel, smem));
+    kernel<<<grid, kMvThreads, smem, stream>>>(a, err);
+    return CRVQ_OK;
+  };
+  if (b == 1)
+    CRVQ_TRY(go(matvec_slice_kernel<1>));
+  else if (b <= 4)
+    CRVQ_TRY(go(matvec_slice_kernel<4>));
+  else
+    CRVQ_TRY(go(matvec_slice_kernel<kMaxBatch>));
+  CRVQ_LAUNCHED();
   return CRVQ_OK;
 }
 

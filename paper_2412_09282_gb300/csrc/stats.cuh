@@ -15,20 +15,21 @@
 
 namespace crvq {
 
+constexpr int kNA = 37;  // packed lower triangle of the 8 x 8 A_k (36 entries) + the count
+
 struct StatsView {
   int32_t* cnt;     // [G_cov][K]
   long long* bacc;  // [K][d]
   double* scale;    // device scalar (followed by the maxima of the scale bound)
+  float2* apair;    // [K][kNA]: A_k and the count as fp32 pairs, between the two solve kernels
   int64_t G_cov;
   int K;
 };
 
-constexpr int kNA = 37;  // packed lower triangle of the 8 x 8 A_k (36 entries) + the count
-
-// Memory of the statistics of one codebook: cnt | bacc | scale + maxima (256 B), each part
-// 256-byte aligned.
+// Memory of the statistics of one codebook: cnt | bacc | scale + maxima (256 B) | apair, each
+// part 256-byte aligned.
 struct StatsLayout {
-  size_t cnt, bacc, head, total;
+  size_t cnt, bacc, head, apair, total;
 };
 
 inline StatsLayout stats_layout(int64_t G_cov, int K) {
@@ -37,7 +38,8 @@ inline StatsLayout stats_layout(int64_t G_cov, int K) {
   L.cnt = align_up((size_t)G * K * sizeof(int32_t), 256);
   L.bacc = align_up((size_t)K * kD * sizeof(long long), 256);
   L.head = 256;
-  L.total = L.cnt + L.bacc + L.head;
+  L.apair = align_up((size_t)K * kNA * sizeof(float2), 256);
+  L.total = L.cnt + L.bacc + L.head + L.apair;
   return L;
 }
 
@@ -48,6 +50,7 @@ inline void stats_bind(void* base, int64_t G_cov, int K, StatsView* st) {
   st->cnt = reinterpret_cast<int32_t*>(p);
   st->bacc = reinterpret_cast<long long*>(p + L.cnt);
   st->scale = reinterpret_cast<double*>(p + L.cnt + L.bacc);
+  st->apair = reinterpret_cast<float2*>(p + L.cnt + L.bacc + L.head);
   st->G_cov = G_cov;
   st->K = K;
 }

@@ -275,91 +275,97 @@ __device__ __forceinline__ void fixed_to_pair(long long v, int sexp, float& h, f
   l = ldexpf(__fadd_rn(t, t2), -sexp);
 }
 
-// The least-squares solve of every codeword, one kernel. CTA = kSolveK codewords; thread =
-// (codeword, entry e of A_k's packed lower triangle or the count, slice of the groups). Each
-// thread sums cnt[g][k] * H_g[e] over its slice as an unevaluated fp32 pair (every product is
-// split exactly: cnt < 2^24; TwoSum for the high part), so no fp64 arithmetic runs per group;
-// the slices are added in a fixed order as fp32 pairs; then one thread per codeword solves
+// The least-squares solve of every codeword, in two kernels. stats_sum_kernel: CTA = one
+// codeword; thread = (entry e of A_k's packed lower triangle or the count, slice of the
+// groups). Each thread sums cnt[g][k] * H_g[e] over its slice as an unevaluated fp32 pair
+// (every product is split exactly: cnt < 2^24; TwoSum for the high part), so no fp64
+// arithmetic runs per group; the slices are added in a fixed order as fp32 pairs, and the
+// pairs of A_k go to st.apair. stats_solve_kernel: one thread per codeword solves
 // A_k c_k = b_k (b_k from the fixed point) by Cholesky with refinement in fp32 pairs. The
-// fixed assignment and order make the result identical on every run. Codewords without
-// members keep their old value.
-constexpr int kSolveK = 1;        // one codeword per CTA: K CTAs share the GPU
+// summing threads carry none of the solve's registers, so every codeword's CTA is resident at
+// once. The fixed assignment and order make the result identical on every run. Codewords
+// without members keep their old value.
 constexpr int kSolveSlices = 16;  // groups split 16 ways: short dependent chains per thread
-constexpr int kSolveThreads = kSolveK * kSolveSlices * kNA;  // 592
+constexpr int kSumThreads = kSolveSlices * kNA;  // 592
+constexpr int kSolveThreads = 128;
 
-__global__ void __launch_bounds__(kSolveThreads)
-stats_solve_kernel(const float* __restrict__ Hb, StatsView st, const float* C_old, float* C_out,
-                   int32_t* __restrict__ counts_out, unsigned* err) {
+__global__ void __launch_bounds__(kSumThreads, 2)
+stats_sum_kernel(const float* __restrict__ Hb, StatsView st) {
   pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
   pdl_wait();
-  __shared__ float part_h[kSolveK][kSolveSlices][kNA], part_l[kSolveK][kSolveSlices][kNA];
+  __shared__ float part_h[kSolveSlices][kNA], part_l[kSolveSlices][kNA];
   const int tid = threadIdx.x;
-  const int kk = tid / (kSolveSlices * kNA);
-  const int sl = (tid / kNA) % kSolveSlices;
+  const int sl = tid / kNA;
   const int e = tid % kNA;
   const int K = st.K;
-  const int k = blockIdx.x * kSolveK + kk;
+  const int k = blockIdx.x;
   // entry e of the packed lower triangle: row r, column c (c <= r); e = 36 is the count
   int r = 0;
   while ((r + 1) * (r + 2) / 2 <= e && r < kD - 1) ++r;
   const int c = e - r * (r + 1) / 2;
   const int hoff = r * kD + c;
   float hi = 0.f, lo = 0.f;
-  if (k < K) {
-    const int64_t gper = (st.G_cov + kSolveSlices - 1) / kSolveSlices;
-    const int64_t g0 = sl * gper, g1 = min(st.G_cov, g0 + gper);
-    constexpr int kBatch = 16;  // loads of 16 groups in flight together; no branches
-    for (int64_t gb = g0; gb < g1; gb += kBatch) {
-      float fc[kBatch], h[kBatch];
+  const int64_t gper = (st.G_cov + kSolveSlices - 1) / kSolveSlices;
+  const int64_t g0 = sl * gper, g1 = min(st.G_cov, g0 + gper);
+  constexpr int kBatch = 8;  // loads of 8 groups in flight together; no branches
+  for (int64_t gb = g0; gb < g1; gb += kBatch) {
+    float fc[kBatch], h[kBatch];
 #pragma unroll
-      for (int u = 0; u < kBatch; ++u) {
-        const int64_t g = gb + u;
-        const bool in = g < g1;
-        fc[u] = in ? (float)st.cnt[g * K + k] : 0.f;  // exact: counts stay below 2^24
-        h[u] = in ? (e < 36 ? __ldg(Hb + g * kD * kD + hoff) : 1.f) : 0.f;
-      }
+    for (int u = 0; u < kBatch; ++u) {
+      const int64_t g = gb + u;
+      const bool in = g < g1;
+      fc[u] = in ? (float)st.cnt[g * K + k] : 0.f;  // exact: counts stay below 2^24
+      h[u] = in ? (e < 36 ? __ldg(Hb + g * kD * kD + hoff) : 1.f) : 0.f;
+    }
 #pragma unroll
-      for (int u = 0; u < kBatch; ++u) {
-        const float p = __fmul_rn(fc[u], h[u]);
-        const float pe = __fmaf_rn(fc[u], h[u], -p);  // fc h = p + pe exactly
-        const float sum = __fadd_rn(hi, p);            // TwoSum(hi, p) = sum + t exactly
-        const float bp = __fsub_rn(sum, hi);
-        const float t = __fadd_rn(__fsub_rn(hi, __fsub_rn(sum, bp)), __fsub_rn(p, bp));
-        hi = sum;
-        lo = __fadd_rn(lo, __fadd_rn(t, pe));
-      }
+    for (int u = 0; u < kBatch; ++u) {
+      const float p = __fmul_rn(fc[u], h[u]);
+      const float pe = __fmaf_rn(fc[u], h[u], -p);  // fc h = p + pe exactly
+      const float sum = __fadd_rn(hi, p);            // TwoSum(hi, p) = sum + t exactly
+      const float bp = __fsub_rn(sum, hi);
+      const float t = __fadd_rn(__fsub_rn(hi, __fsub_rn(sum, bp)), __fsub_rn(p, bp));
+      hi = sum;
+      lo = __fadd_rn(lo, __fadd_rn(t, pe));
     }
   }
   // Slices are merged per entry by its own thread in fp32 pairs (TwoSum of the high parts, low
   // parts added), in slice order: no serial fp64 chain (a dependent fp64 operation costs
   // about 180 cycles on this part).
-  part_h[kk][sl][e] = hi;
-  part_l[kk][sl][e] = lo;
+  part_h[sl][e] = hi;
+  part_l[sl][e] = lo;
   __syncthreads();
   // Every thread of the codeword has read its counts: clear them, so that the statistics are
   // zero for the next accumulation (the Lloyd loop needs no memset between iterations).
-  if (e == 0 && k < K) {
-    const int64_t gper = (st.G_cov + kSolveSlices - 1) / kSolveSlices;
-    const int64_t g0 = sl * gper, g1 = min(st.G_cov, g0 + gper);
+  if (e == 0)
     for (int64_t gq = g0; gq < g1; ++gq) st.cnt[gq * K + k] = 0;
-  }
-  if (sl == 0 && k < K) {
-    float h = part_h[kk][0][e], l = part_l[kk][0][e];
+  if (sl == 0) {
+    float h = part_h[0][e], l = part_l[0][e];
     for (int s2 = 1; s2 < kSolveSlices; ++s2) {
-      const float p = part_h[kk][s2][e];
+      const float p = part_h[s2][e];
       const float sum = __fadd_rn(h, p);
       const float bp = __fsub_rn(sum, h);
       const float t = __fadd_rn(__fsub_rn(h, __fsub_rn(sum, bp)), __fsub_rn(p, bp));
       h = sum;
-      l = __fadd_rn(l, __fadd_rn(t, part_l[kk][s2][e]));
+      l = __fadd_rn(l, __fadd_rn(t, part_l[s2][e]));
     }
-    part_h[kk][0][e] = h;
-    part_l[kk][0][e] = l;
+    st.apair[(int64_t)k * kNA + e] = make_float2(h, l);
   }
-  __syncthreads();
-  if (sl != 0 || e != 0 || k >= K) return;
-  const float* Ah = part_h[kk][0];
-  const float* Al = part_l[kk][0];
+}
+
+__global__ void __launch_bounds__(kSolveThreads)
+stats_solve_kernel(StatsView st, const float* C_old, float* C_out,
+                   int32_t* __restrict__ counts_out, unsigned* err) {
+  pdl_trigger();
+  pdl_wait();
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= st.K) return;
+  float Ah[kNA], Al[kNA];
+#pragma unroll
+  for (int e = 0; e < kNA; ++e) {
+    const float2 v = st.apair[(int64_t)k * kNA + e];
+    Ah[e] = v.x;
+    Al[e] = v.y;
+  }
   // the count: an exact integer held by the pair
   const int64_t count = (int64_t)__float2int_rn(Ah[36]) + (int64_t)__float2int_rn(Al[36]);
   if (counts_out) counts_out[k] = (int32_t)count;
@@ -399,8 +405,11 @@ crvq_status launch_solve_kernels(const float* Hb, const StatsView& st, const flo
                                  float* C_out, int32_t* counts, unsigned* err,
                                  cudaStream_t stream) {
   ProfScope ps("update_solve", stream, (double)st.K);
-  CRVQ_CUDA(launch_pdl(stats_solve_kernel, dim3((unsigned)ceil_div(st.K, kSolveK)),
-                       dim3(kSolveThreads), 0, stream, Hb, st, C_old, C_out, counts, err));
+  CRVQ_CUDA(launch_pdl(stats_sum_kernel, dim3((unsigned)st.K), dim3(kSumThreads), 0, stream,
+                       Hb, st));
+  CRVQ_LAUNCHED();
+  CRVQ_CUDA(launch_pdl(stats_solve_kernel, dim3((unsigned)ceil_div(st.K, kSolveThreads)),
+                       dim3(kSolveThreads), 0, stream, st, C_old, C_out, counts, err));
   CRVQ_LAUNCHED();
   return CRVQ_OK;
 }
@@ -471,7 +480,7 @@ crvq_status launch_update_codebook(const SetView& set, const CbList& cbs, int wh
 namespace crvq {
 
 // The update of launch_update_codebook on caller-provided scratch (no allocation): `scratch`
-// (256-byte aligned, `bytes` long) holds cnt | bacc | scale + maxima, and `err` is the error
+// (256-byte aligned, `bytes` long) holds cnt | bacc | scale + maxima | apair, and `err` is the error
 // word the kernels report to. Returns CRVQ_ERR_UNSUPPORTED when the statistics of this
 // codebook do not fit in `bytes`.
 size_t update_scratch_bytes(int64_t G_cov, int K) { return stats_layout(G_cov, K).total; }
@@ -485,7 +494,7 @@ crvq_status launch_update_codebook_on(const SetView& set, const CbList& cbs, int
   if (need > bytes)
     return fail(CRVQ_ERR_UNSUPPORTED,
                 "statistics of this codebook need %zu bytes of scratch, the limit is %zu "
-                "(G_cov * K * 4 + K * 64 + 256 bytes, each part 256-byte aligned)",
+                "(G_cov * K * 4 + K * 64 + 256 + K * 296 bytes, each part 256-byte aligned)",
                 need, bytes);
   const StatsLayout L = stats_layout(cw.G_cov, cw.K);
   StatsView st;
