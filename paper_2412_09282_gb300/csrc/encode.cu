@@ -1160,20 +1160,29 @@ __device__ __forceinline__ void hyp_terms_pair(const float rh[kD], const float r
   }
 }
 
-// Fast stage: one thread per vector, the stage codebook chunked through shared memory, a
-// sorted top-L list (L >= Bs + 1) of lower bounds low = approx_err - Et in registers.
+// Fast stage: kBeamLanes threads per vector, the stage codebook chunked through shared
+// memory. Each thread scores every hypothesis against every kBeamLanes-th codeword of a chunk
+// and keeps its own sorted top-L list (L >= Bs + 1) of lower bounds low = approx_err - Et;
+// the lists of a vector are then merged in (low, hypothesis, codeword) order, and the
+// vector's first thread carries on with the merged list alone (certificate, exact path,
+// output).
+constexpr int kBeamLanes = 8;
+constexpr int kBeamVecs = kThreads / kBeamLanes;  // vectors per CTA
+
 template <int L>
 __global__ void __launch_bounds__(kThreads, L <= 9 ? 3 : 2)
 beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc sd,
                   BeamBufs bb, FlagList flags, unsigned* err) {
   const int64_t g = g_begin + blockIdx.y;
   const int64_t G_range = gridDim.y;
-  const int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x;
+  const int sub = threadIdx.x % kBeamLanes;
+  const int64_t i = (int64_t)blockIdx.x * kBeamVecs + threadIdx.x / kBeamLanes;
   const bool live = i < set.M;
   const int64_t vi = live ? i * G_range + (g - g_begin) : 0;
   __shared__ float sH[kD * kD];
-  __shared__ __align__(16) float sC[kChunk * kD];
+  __shared__ __align__(16) float sC[kChunk * kD];  // the chunk; after the scan, the lists
   __shared__ float sN[kChunk], sL[kChunk];
+  static_assert(kBeamVecs * kBeamLanes * 17 * 3 * 4 <= kChunk * kD * 4, "merge buffer");
   if (threadIdx.x < kD * kD) sH[threadIdx.x] = set.Hb[g * kD * kD + threadIdx.x];
   __syncthreads();
 
@@ -1212,7 +1221,7 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
       hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
       const float base = rr - kU * cmul * ra;
       const float nbeta = -2.f * kU * cmul * pmax;
-      for (int k = 0; k < nk; ++k) {
+      for (int k = sub; k < nk; k += kBeamLanes) {
         const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
         const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
         float s = base + sN[k];
@@ -1241,7 +1250,41 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
       }
     }
   }
-  if (!live) return;
+  // Merge the vector's kBeamLanes lists (in the chunk buffer, free now) into its first
+  // thread's, ordered by (low, hypothesis, codeword): the same list whatever the split.
+  __syncthreads();
+  {
+    float* mv = sC + (size_t)threadIdx.x * L * 3;
+    int* mi = reinterpret_cast<int*>(mv);
+#pragma unroll
+    for (int j = 0; j < L; ++j) {
+      mv[3 * j] = topv[j];
+      mi[3 * j + 1] = toph[j];
+      mi[3 * j + 2] = topk[j];
+    }
+  }
+  __syncthreads();
+  if (!live || sub != 0) return;
+  for (int t = 1; t < kBeamLanes; ++t) {
+    const float* mv = sC + (size_t)(threadIdx.x + t) * L * 3;
+    const int* mi = reinterpret_cast<const int*>(mv);
+    for (int jj = 0; jj < L; ++jj) {
+      float sv = mv[3 * jj];
+      int sh = mi[3 * jj + 1], sk = mi[3 * jj + 2];
+      if (!(sv <= topv[L - 1])) break;  // sorted: nothing after enters either
+#pragma unroll
+      for (int j = 0; j < L; ++j) {
+        const bool before = sv < topv[j] ||
+                            (sv == topv[j] && (sh < toph[j] || (sh == toph[j] && sk < topk[j])));
+        if (before) {
+          const float tv = topv[j];
+          const int th = toph[j], tk = topk[j];
+          topv[j] = sv; toph[j] = sh; topk[j] = sk;
+          sv = tv; sh = th; sk = tk;
+        }
+      }
+    }
+  }
 
   const int64_t total = (int64_t)Bh * cw.K;
   const int nkept = (int)min((int64_t)L, total);
@@ -1635,7 +1678,7 @@ crvq_status launch_beam_stage_L(const SetView& set, int64_t g_begin, int64_t G_r
                                 const CbList& cbs, int n_fixed, const StageDesc& sd,
                                 const BeamBufs& bb, const FlagList& fl, unsigned* err,
                                 double units, cudaStream_t stream) {
-  dim3 grid((unsigned)ceil_div(set.M, kThreads), (unsigned)G_range);
+  dim3 grid((unsigned)ceil_div(set.M, kBeamVecs), (unsigned)G_range);
   ProfScope ps("encode_beam_stage", stream, units);
   beam_stage_kernel<L><<<grid, kThreads, 0, stream>>>(set, g_begin, cbs, n_fixed, sd, bb, fl,
                                                      err);

@@ -42,6 +42,7 @@ struct MatvecArgs {
   int b;
   int base_lut;         // the base codebook (cbs.cb[0]) uses shared-memory lookup tables
   int64_t n_slices;
+  const float* lut;     // [G][K_base][b] base-codebook tables (when base_lut)
   float* part;          // [n_slices][b][M]
   unsigned* done;       // per row block: CTAs finished (zero on entry)
   float* Y;             // b x M, row stride ldy
@@ -66,6 +67,40 @@ __device__ __forceinline__ float dot8(const float* __restrict__ c, const float* 
   v = fmaf(c1.z, x[6], v);
   v = fmaf(c1.w, x[7], v);
   return v;
+}
+
+// The base codebook's lookup tables of every group, once per call: lut[g][k][bi] =
+// <C_base[k], xs[bi][g]>, one thread per (group, codeword), the group's inputs taken through
+// the permutation.
+__global__ void __launch_bounds__(256)
+lut_build_kernel(const float* __restrict__ X, int64_t ldx, int64_t N,
+                 const int32_t* __restrict__ perm, CbView cb0, int b, float* __restrict__ lut,
+                 unsigned* err) {
+  const int64_t G = N / kD;
+  const int64_t total = G * cb0.K;
+  for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < total;
+       e += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t g = e / cb0.K;
+    const int k = (int)(e % cb0.K);
+    int64_t src[kD];
+#pragma unroll
+    for (int j = 0; j < kD; ++j) {
+      src[j] = g * kD + j;
+      if (perm) {
+        src[j] = perm[g * kD + j];
+        if (src[j] < 0 || src[j] >= N) {
+          if (k == 0) raise_error(err, ERRBIT_INDEX);
+          src[j] = -1;
+        }
+      }
+    }
+    for (int bi = 0; bi < b; ++bi) {
+      float x[kD];
+#pragma unroll
+      for (int j = 0; j < kD; ++j) x[j] = src[j] >= 0 ? X[bi * ldx + src[j]] : 0.f;
+      lut[e * b + bi] = dot8(cb0.C + (int64_t)k * kD, x);
+    }
+  }
 }
 
 // Partial products of one (row block, group slice), and the ordered sum of a row block's
@@ -110,14 +145,11 @@ matvec_slice_kernel(MatvecArgs a, unsigned* err) {
     xs[e] = v;
   }
   __syncthreads();
-  // the base codebook's tables: a thread per codeword, loaded once, across the slice's groups
+  // the slice's base-codebook tables, copied from the per-call build (L2-resident)
   if (a.base_lut) {
-    for (int k = tid; k < cb0.K; k += blockDim.x) {
-      const float* c = cb0.C + (int64_t)k * kD;
-      for (int gl = 0; gl < gn; ++gl)
-        for (int bi = 0; bi < a.b; ++bi)
-          lut[((int64_t)gl * cb0.K + k) * a.b + bi] = dot8(c, xs + (bi * kSliceG + gl) * kD);
-    }
+    const int64_t n4 = (int64_t)gn * cb0.K * a.b / 4;  // K * b is a multiple of 4 here
+    const float4* src = reinterpret_cast<const float4*>(a.lut + g0 * cb0.K * a.b);
+    for (int64_t e = tid; e < n4; e += blockDim.x) reinterpret_cast<float4*>(lut)[e] = src[e];
     __syncthreads();
   }
 
@@ -200,16 +232,26 @@ crvq_status launch_lut_matvec(const float* X, int64_t ldx, int64_t N, int b,
   a.Y = Y;
   a.ldy = ldy;
   const size_t lut_bytes = (size_t)kSliceG * cbs.cb[0].K * b * sizeof(float);
-  a.base_lut = lut_bytes <= kLutSmemCap ? 1 : 0;
+  a.base_lut = (lut_bytes <= kLutSmemCap && (cbs.cb[0].K * b) % 4 == 0) ? 1 : 0;
   const size_t smem = (size_t)kMaxBatch * kSliceG * kD * sizeof(float) +
                       (size_t)kMvRows * kSliceG * sizeof(int32_t) + (a.base_lut ? lut_bytes : 0);
   const int64_t row_blocks = ceil_div(M, (int64_t)kMvRows);
   const size_t part_bytes = align_up((size_t)a.n_slices * b * M * sizeof(float), 256);
+  const size_t lutg_bytes = a.base_lut ? align_up((size_t)G * cbs.cb[0].K * b * 4, 256) : 0;
   Scratch mem;
-  CRVQ_TRY(mem.alloc(part_bytes + (size_t)row_blocks * sizeof(unsigned), stream));
+  CRVQ_TRY(mem.alloc(part_bytes + lutg_bytes + (size_t)row_blocks * sizeof(unsigned), stream));
   a.part = mem.as<float>();
-  a.done = reinterpret_cast<unsigned*>(mem.as<char>() + part_bytes);
+  a.lut = reinterpret_cast<float*>(mem.as<char>() + part_bytes);
+  a.done = reinterpret_cast<unsigned*>(mem.as<char>() + part_bytes + lutg_bytes);
   CRVQ_CUDA(cudaMemsetAsync(a.done, 0, (size_t)row_blocks * sizeof(unsigned), stream));
+  const int nsm = sm_count();
+  if (a.base_lut) {
+    ProfScope pl("matvec_tables", stream, (double)G * cbs.cb[0].K * b);
+    const int64_t total = G * cbs.cb[0].K;
+    lut_build_kernel<<<(unsigned)std::min<int64_t>(ceil_div(total, 256), 8 * nsm), 256, 0,
+                       stream>>>(X, ldx, N, perm, cbs.cb[0], b, const_cast<float*>(a.lut), err);
+    CRVQ_LAUNCHED();
+  }
   const dim3 grid((unsigned)row_blocks, (unsigned)a.n_slices);
   ProfScope ps("matvec_slices", stream, (double)M * G * cbs.n);
   auto go = [&](auto kernel) -> crvq_status {
