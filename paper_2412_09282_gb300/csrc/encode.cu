@@ -954,6 +954,7 @@ argmin_exact_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs, i
 // (value, index) is reduced across the warp with the same total order, so the decision is the
 // one argmin_exact_kernel makes.
 constexpr int kExactWarpK = 1024;
+constexpr int kExactBatch = 2;  // codewords a lane loads before using them
 
 __global__ void __launch_bounds__(128)
 argmin_exact_warp_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList cbs,
@@ -982,19 +983,33 @@ argmin_exact_warp_kernel(SetView set, int64_t g_begin, int64_t G_range, CbList c
     vector_terms(rv, av, sH, m2q, pmax);
     const float nbeta = -2.f * kU * cmul * pmax;
     const float4* gt = terms ? terms + grel * cw.K : nullptr;
+    // a lane takes codewords lane, lane + 32, ...; kExactBatch of them are loaded before any is
+    // used, so their L2 round trips overlap
     float U = thr;
-    for (int k = lane; k < cw.K; k += 32) {
-      float cv[kD], nn, na, l1;
-      load_vec(cw.C + (int64_t)k * kD, cv);
-      if (gt) {
-        const float4 t = gt[k];
-        nn = t.x;
-        na = t.y;
-        l1 = t.z;
-      } else {
-        codeword_terms(cv, sH, nn, na, l1);
+    for (int k0 = lane; k0 < cw.K; k0 += 32 * kExactBatch) {
+      float cv[kExactBatch][kD];
+      float4 tt[kExactBatch];
+#pragma unroll
+      for (int u = 0; u < kExactBatch; ++u) {
+        const int k = k0 + 32 * u;
+        if (k < cw.K) {
+          load_vec(cw.C + (int64_t)k * kD, cv[u]);
+          if (gt) tt[u] = gt[k];
+        }
       }
-      U = fminf(U, up_from(nn, na, l1, cv, m2q, pmax, cmul));
+#pragma unroll
+      for (int u = 0; u < kExactBatch; ++u) {
+        if (k0 + 32 * u >= cw.K) break;
+        float nn, na, l1;
+        if (gt) {
+          nn = tt[u].x;
+          na = tt[u].y;
+          l1 = tt[u].z;
+        } else {
+          codeword_terms(cv[u], sH, nn, na, l1);
+        }
+        U = fminf(U, up_from(nn, na, l1, cv[u], m2q, pmax, cmul));
+      }
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) U = fminf(U, __shfl_xor_sync(0xffffffffu, U, o));
@@ -1160,29 +1175,20 @@ __device__ __forceinline__ void hyp_terms_pair(const float rh[kD], const float r
   }
 }
 
-// Fast stage: kBeamLanes threads per vector, the stage codebook chunked through shared
-// memory. Each thread scores every hypothesis against every kBeamLanes-th codeword of a chunk
-// and keeps its own sorted top-L list (L >= Bs + 1) of lower bounds low = approx_err - Et;
-// the lists of a vector are then merged in (low, hypothesis, codeword) order, and the
-// vector's first thread carries on with the merged list alone (certificate, exact path,
-// output).
-constexpr int kBeamLanes = 8;
-constexpr int kBeamVecs = kThreads / kBeamLanes;  // vectors per CTA
-
+// Fast stage: one thread per vector, the stage codebook chunked through shared memory, a
+// sorted top-L list (L >= Bs + 1) of lower bounds low = approx_err - Et in registers.
 template <int L>
-__global__ void __launch_bounds__(kThreads, L <= 9 ? 3 : 2)
+__global__ void __launch_bounds__(kThreads, L < 9 ? 3 : 2)
 beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc sd,
                   BeamBufs bb, FlagList flags, unsigned* err) {
   const int64_t g = g_begin + blockIdx.y;
   const int64_t G_range = gridDim.y;
-  const int sub = threadIdx.x % kBeamLanes;
-  const int64_t i = (int64_t)blockIdx.x * kBeamVecs + threadIdx.x / kBeamLanes;
+  const int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x;
   const bool live = i < set.M;
   const int64_t vi = live ? i * G_range + (g - g_begin) : 0;
   __shared__ float sH[kD * kD];
-  __shared__ __align__(16) float sC[kChunk * kD];  // the chunk; after the scan, the lists
+  __shared__ __align__(16) float sC[kChunk * kD];
   __shared__ float sN[kChunk], sL[kChunk];
-  static_assert(kBeamVecs * kBeamLanes * 17 * 3 * 4 <= kChunk * kD * 4, "merge buffer");
   if (threadIdx.x < kD * kD) sH[threadIdx.x] = set.Hb[g * kD * kD + threadIdx.x];
   __syncthreads();
 
@@ -1221,7 +1227,9 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
       hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
       const float base = rr - kU * cmul * ra;
       const float nbeta = -2.f * kU * cmul * pmax;
-      for (int k = sub; k < nk; k += kBeamLanes) {
+      // two codewords per step: their FMA chains are independent, so they overlap (the chain
+      // of one score is ten dependent operations)
+      auto score = [&](int k) {
         const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
         const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
         float s = base + sN[k];
@@ -1233,7 +1241,9 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
         s = fmaf(m2q[5], c1.y, s);
         s = fmaf(m2q[6], c1.z, s);
         s = fmaf(m2q[7], c1.w, s);
-        s = fmaf(nbeta, sL[k], s);
+        return fmaf(nbeta, sL[k], s);
+      };
+      auto insert = [&](float s, int k) {
         if (s < topv[L - 1]) {
           float sv = s;
           int sh = h, sk = k0 + k;
@@ -1247,44 +1257,17 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
             }
           }
         }
+      };
+      int k = 0;
+      for (; k + 1 < nk; k += 2) {
+        const float sa = score(k), sb = score(k + 1);
+        insert(sa, k);  // in codeword order, as one at a time
+        insert(sb, k + 1);
       }
+      if (k < nk) insert(score(k), k);
     }
   }
-  // Merge the vector's kBeamLanes lists (in the chunk buffer, free now) into its first
-  // thread's, ordered by (low, hypothesis, codeword): the same list whatever the split.
-  __syncthreads();
-  {
-    float* mv = sC + (size_t)threadIdx.x * L * 3;
-    int* mi = reinterpret_cast<int*>(mv);
-#pragma unroll
-    for (int j = 0; j < L; ++j) {
-      mv[3 * j] = topv[j];
-      mi[3 * j + 1] = toph[j];
-      mi[3 * j + 2] = topk[j];
-    }
-  }
-  __syncthreads();
-  if (!live || sub != 0) return;
-  for (int t = 1; t < kBeamLanes; ++t) {
-    const float* mv = sC + (size_t)(threadIdx.x + t) * L * 3;
-    const int* mi = reinterpret_cast<const int*>(mv);
-    for (int jj = 0; jj < L; ++jj) {
-      float sv = mv[3 * jj];
-      int sh = mi[3 * jj + 1], sk = mi[3 * jj + 2];
-      if (!(sv <= topv[L - 1])) break;  // sorted: nothing after enters either
-#pragma unroll
-      for (int j = 0; j < L; ++j) {
-        const bool before = sv < topv[j] ||
-                            (sv == topv[j] && (sh < toph[j] || (sh == toph[j] && sk < topk[j])));
-        if (before) {
-          const float tv = topv[j];
-          const int th = toph[j], tk = topk[j];
-          topv[j] = sv; toph[j] = sh; topk[j] = sk;
-          sv = tv; sh = th; sk = tk;
-        }
-      }
-    }
-  }
+  if (!live) return;
 
   const int64_t total = (int64_t)Bh * cw.K;
   const int nkept = (int)min((int64_t)L, total);
@@ -1678,7 +1661,7 @@ crvq_status launch_beam_stage_L(const SetView& set, int64_t g_begin, int64_t G_r
                                 const CbList& cbs, int n_fixed, const StageDesc& sd,
                                 const BeamBufs& bb, const FlagList& fl, unsigned* err,
                                 double units, cudaStream_t stream) {
-  dim3 grid((unsigned)ceil_div(set.M, kBeamVecs), (unsigned)G_range);
+  dim3 grid((unsigned)ceil_div(set.M, kThreads), (unsigned)G_range);
   ProfScope ps("encode_beam_stage", stream, units);
   beam_stage_kernel<L><<<grid, kThreads, 0, stream>>>(set, g_begin, cbs, n_fixed, sd, bb, fl,
                                                      err);
@@ -1819,7 +1802,7 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
         CRVQ_LAUNCHED();
       }
       {
-        ProfScope pf("encode_argmin_exact", stream, 0.0);
+        ProfScope pf("encode_exact", stream, 0.0);
         if (cw.K <= kExactWarpK) {
           CRVQ_CUDA(launch_pdl(argmin_exact_warp_kernel,
                                dim3((unsigned)std::min<int64_t>(ceil_div(nv, 4), 16 * nsm)),

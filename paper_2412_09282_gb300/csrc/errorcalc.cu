@@ -30,7 +30,7 @@ __device__ __forceinline__ void pair_merge(float& h, float& l, float oh, float o
 }
 
 constexpr int kDecRows = 16;     // rows per warp (the CTA's H blocks are staged once for all)
-constexpr int kDecBatch = 2;     // rows whose codes are loaded together
+constexpr int kDecBatch = 4;     // rows whose codes and vectors are loaded together
 constexpr int kDecWarps = 8;     // warps per CTA
 constexpr int kDecHStride = 260; // floats per staged H block (256 + 4: conflict-free float4)
 constexpr int kDecSmemCb = 48 * 1024;  // codebooks staged in shared memory up to this size
@@ -129,6 +129,7 @@ decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
   const float4* H4 = reinterpret_cast<const float4*>(sH + lane * kDecHStride);
   for (int r0 = 0; r0 < nr; r0 += kDecBatch) {
     int32_t kc[kDecBatch][MAXCB];
+    float4 tv[kDecBatch][2];
 #pragma unroll
     for (int u = 0; u < kDecBatch; ++u) {
       const int64_t i = i0 + min(r0 + u, nr - 1);
@@ -137,6 +138,11 @@ decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
         kc[u][s] = -1;
         if (gok && s < cbs.n && g < cbs.cb[s].G_cov)
           kc[u][s] = cbs.cb[s].codes[i * cbs.cb[s].ld + g];
+      }
+      tv[u][0] = tv[u][1] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (gok) {
+        tv[u][0] = *reinterpret_cast<const float4*>(Ws + i * N + g * kD);
+        tv[u][1] = *reinterpret_cast<const float4*>(Ws + i * N + g * kD + 4);
       }
     }
 #pragma unroll
@@ -155,9 +161,8 @@ decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
         }
         float rv[kD], dl[kD];
         recon_codes<MAXCB>(cw, kc[u], cbs.n, rv);
-        const float4 t0 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD);
-        const float4 t1 = *reinterpret_cast<const float4*>(Ws + i * N + g * kD + 4);
-        const float t[kD] = {t0.x, t0.y, t0.z, t0.w, t1.x, t1.y, t1.z, t1.w};
+        const float t[kD] = {tv[u][0].x, tv[u][0].y, tv[u][0].z, tv[u][0].w,
+                             tv[u][1].x, tv[u][1].y, tv[u][1].z, tv[u][1].w};
 #pragma unroll
         for (int j = 0; j < kD; ++j) {
           dl[j] = t[j] - rv[j];

@@ -28,7 +28,8 @@ namespace {
 
 constexpr int kSliceG = 32;     // groups per CTA slice (one per lane)
 constexpr int kMvThreads = 256;
-constexpr int kMvRows = 128;    // rows per CTA
+constexpr int kMvRows = 64;     // rows per CTA
+constexpr int kStageCb = 4;     // codebooks whose codes of the tile are staged in shared memory
 constexpr int kMaxBatch = 8;
 constexpr size_t kLutSmemCap = 96 * 1024;  // the base codebook's tables per CTA at most
 
@@ -110,8 +111,9 @@ __global__ void __launch_bounds__(kMvThreads)
 matvec_slice_kernel(MatvecArgs a, unsigned* err) {
   extern __shared__ __align__(16) float sm[];
   float* xs = sm;                                          // [b][kSliceG][8]
-  int32_t* scode = reinterpret_cast<int32_t*>(xs + kMaxBatch * kSliceG * kD);  // [rows][32]
-  float* lut = reinterpret_cast<float*>(scode + kMvRows * kSliceG);            // [32][K][b]
+  // codes of the tile, codebook-major: [kStageCb][rows][32]
+  int32_t* scode = reinterpret_cast<int32_t*>(xs + kMaxBatch * kSliceG * kD);
+  float* lut = reinterpret_cast<float*>(scode + kStageCb * kMvRows * kSliceG);  // [32][K][b]
   __shared__ int s_last;
   const int64_t slice = blockIdx.y, rblk = blockIdx.x;
   const int64_t g0 = slice * kSliceG;
@@ -122,11 +124,18 @@ matvec_slice_kernel(MatvecArgs a, unsigned* err) {
   const int nr = (int)(a.M - r0 < kMvRows ? a.M - r0 : kMvRows);
   const CbView& cb0 = a.cbs.cb[0];
 
-  // every load of the tile at once: the base codes (coalesced rows of 32 codes) and the inputs
-  for (int e = tid; e < nr * kSliceG; e += blockDim.x) {
-    const int r = e / kSliceG, l = e % kSliceG;
-    const int64_t g = g0 + l;
-    scode[e] = (l < gn && g < cb0.G_cov) ? cb0.codes[(r0 + r) * cb0.ld + g] : -1;
+  // every load of the tile at once: the codes of the staged codebooks that cover the slice
+  // (coalesced rows of 32 codes) and the inputs
+  const int nst = a.cbs.n < kStageCb ? a.cbs.n : kStageCb;
+  for (int s = 0; s < nst; ++s) {
+    const CbView& cb = a.cbs.cb[s];
+    if (cb.G_cov <= g0) continue;
+    int32_t* sc = scode + s * kMvRows * kSliceG;
+    for (int e = tid; e < nr * kSliceG; e += blockDim.x) {
+      const int r = e / kSliceG, l = e % kSliceG;
+      const int64_t g = g0 + l;
+      sc[e] = (l < gn && g < cb.G_cov) ? cb.codes[(r0 + r) * cb.ld + g] : -1;
+    }
   }
   for (int e = tid; e < a.b * kSliceG * kD; e += blockDim.x) {
     const int bi = e / (kSliceG * kD), r = e % (kSliceG * kD);
@@ -177,7 +186,8 @@ matvec_slice_kernel(MatvecArgs a, unsigned* err) {
     for (int s = 1; s < a.cbs.n; ++s) {  // extended codebooks: the first G_c groups only
       const CbView& cb = a.cbs.cb[s];
       if (!(lane < gn && g < cb.G_cov)) continue;
-      const int32_t ke = cb.codes[i * cb.ld + g];
+      const int32_t ke = s < kStageCb ? scode[(s * kMvRows + r) * kSliceG + lane]
+                                      : cb.codes[i * cb.ld + g];
       if (ke < 0 || ke >= cb.K) {
         raise_error(err, ERRBIT_INDEX);
         continue;
@@ -204,7 +214,15 @@ matvec_slice_kernel(MatvecArgs a, unsigned* err) {
     const int bi = e / nr;
     const int64_t i = r0 + e % nr;
     float sum = 0.f;
-    for (int64_t q = 0; q < a.n_slices; ++q) sum += __ldcg(a.part + (q * a.b + bi) * a.M + i);
+    int64_t q = 0;
+    for (; q + 8 <= a.n_slices; q += 8) {  // eight loads in flight, added in slice order
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) v[u] = __ldcg(a.part + ((q + u) * a.b + bi) * a.M + i);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) sum += v[u];
+    }
+    for (; q < a.n_slices; ++q) sum += __ldcg(a.part + (q * a.b + bi) * a.M + i);
     a.Y[bi * a.ldy + i] = sum;
   }
 }
@@ -234,7 +252,8 @@ crvq_status launch_lut_matvec(const float* X, int64_t ldx, int64_t N, int b,
   const size_t lut_bytes = (size_t)kSliceG * cbs.cb[0].K * b * sizeof(float);
   a.base_lut = (lut_bytes <= kLutSmemCap && (cbs.cb[0].K * b) % 4 == 0) ? 1 : 0;
   const size_t smem = (size_t)kMaxBatch * kSliceG * kD * sizeof(float) +
-                      (size_t)kMvRows * kSliceG * sizeof(int32_t) + (a.base_lut ? lut_bytes : 0);
+                      (size_t)kStageCb * kMvRows * kSliceG * sizeof(int32_t) +
+                      (a.base_lut ? lut_bytes : 0);
   const int64_t row_blocks = ceil_div(M, (int64_t)kMvRows);
   const size_t part_bytes = align_up((size_t)a.n_slices * b * M * sizeof(float), 256);
   const size_t lutg_bytes = a.base_lut ? align_up((size_t)G * cbs.cb[0].K * b * 4, 256) : 0;
