@@ -228,20 +228,19 @@ __device__ __forceinline__ float low_score(const float c[kD], const float* H, co
 //   A row (vector):   [q_hi x8 | q_hi x8 | q_lo x8 | 1 1 | beta_hi beta_hi beta_lo | off_hi off_lo | 0]
 //   B row (codeword): [c_hi x8 | c_lo x8 | c_hi x8 | n'_hi n'_lo | L1_hi L1_lo L1_hi | 1 1 | 0]
 // One tcgen05.mma M = 128 vectors x N = 128 codewords x K = 8, four per chunk (K = 32), fp32
-// accumulator in tensor memory. The epilogue reads each row's 128 scores in blocks of 32,
-// packs the column within its block into the low 5 mantissa bits of the (non-negative) fp32
-// bound (a truncation of at most 2^-18 relative) and keeps the two smallest keys of each
-// block with integer min / max; the block is tracked by the merge. The certificate and the
-// fp64 fallback are those of the fp32 pass, with the bound multiplier raised to cover the
+// accumulator in tensor memory. The epilogue reads each row's scores in blocks of 16: per block
+// its minimum (integer minima of the non-negative fp32 bit patterns); per row the block with the
+// smallest minimum, kept whole, and the second smallest block minimum. The row's winner and
+// second smallest score come from those 17 values, exact (no packed index). The certificate and
+// the fp64 fallback are those of the fp32 pass, with the bound multiplier raised to cover the
 // tensor-core products and accumulation (about 2^-22 per split product and fp32 accumulation
-// over 32 terms) and the packing.
+// over 32 terms).
 namespace tcenc {
 
 constexpr int kRows = 128;        // vectors per row tile (TMEM lanes)
 constexpr int kK = 32;            // tf32 columns per row
 constexpr int kATile = kRows * kK * 4;   // 16 KB
 constexpr float kCmul = 256.f;           // bound multiplier (about twice the analysis)
-constexpr float kPack = 3.8146973e-06f;  // 2^-18: relative truncation of the packed key
 
 __device__ __forceinline__ uint32_t koff(int r, int k) {
   return (uint32_t)(((r >> 3) * (kK / 4) + (k >> 2)) * 128 + (r & 7) * 16 + (k & 3) * 4);
@@ -329,7 +328,6 @@ __device__ void cbmax_block(const float* __restrict__ C, int K, float* __restric
   }
 }
 
-constexpr uint32_t kKeyMask = 0xffffffe0u;       // value bits of a packed arg-min key
 constexpr int kTcCols = 128;                     // codewords per chunk (MMA N)
 constexpr int kTcBTile = kTcCols * tcenc::kK * 4;  // 16 KB
 
@@ -461,35 +459,23 @@ __device__ __forceinline__ bool less(float ah, float al, int ak, float bh, float
 // halves of 128 that run independently (each its own tiles, named barriers, MMA issue and
 // accumulator) and share the resident codebook operand and the statistics; two CTAs per SM,
 // so four tile pipelines per SM interleave their phases (A rows, MMA, epilogue, certificate).
-// Keys carry the column within a 32-column block in their low 5 bits (2^-18 relative
-// truncation); the block is tracked by the merge. Rows the bounds do not certify go to the flag
-// list (decided exactly by the exact kernels). The Lloyd statistics of certified rows are summed
+// The sweep keeps per row the 16-column block with the smallest minimum and the second
+// smallest block minimum. Rows the bounds do not certify go to the flag list (decided exactly
+// by the exact kernels). The Lloyd statistics of certified rows are summed
 // in shared memory (integer atomics, [component][code] so that a warp's lanes hit spread banks)
 // and flushed once.
 constexpr int kTcSmemStatsK = 256;  // codebooks up to this size aggregate statistics in smem
 
-// Key of a non-negative fp32 value v (its bit pattern) with column j < 32 in the low 5 bits:
-// (v & ~31) | j. `mask` = ~31 arrives as a kernel argument so that the compiler cannot fold
-// it: with the mask and the column both immediates the operation takes two ALU instructions.
-#ifndef CRVQ_KEYPACK
-#define CRVQ_KEYPACK 1
-#endif
-__device__ __forceinline__ uint32_t pack_key(uint32_t v, uint32_t j, uint32_t mask,
-                                             uint32_t m27, uint32_t m32) {
-#if CRVQ_KEYPACK == 0
-  return (v & 0xffffffe0u) | j;
-#elif CRVQ_KEYPACK == 1
-  uint32_t k;  // one three-input logic operation: (v & mask) | j
-  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(k) : "r"(v), "r"(mask), "r"(j));
-  return k;
-#else
-  // on the integer multiply-add path instead of the logic unit: (v >> 5) * 32 + j, with
-  // v >> 5 = the high word of v * 2^27 (m27 = 2^27 and m32 = 32, both from `mask`)
-  uint32_t hi;
-  asm("mul.hi.u32 %0, %1, %2;" : "=r"(hi) : "r"(v), "r"(m27));
-  return hi * m32 + j;
-#endif
+// Minimum of 16 non-negative fp32 values by their bit patterns (which order like the values),
+// as three-input integer minima.
+__device__ __forceinline__ uint32_t min16_bits(const uint32_t* x) {
+  const uint32_t a = __vimin3_u32(x[0], x[1], x[2]), b = __vimin3_u32(x[3], x[4], x[5]),
+                 c = __vimin3_u32(x[6], x[7], x[8]), d = __vimin3_u32(x[9], x[10], x[11]),
+                 e = __vimin3_u32(x[12], x[13], x[14]);
+  return min(__vimin3_u32(a, b, c), __vimin3_u32(d, e, x[15]));
 }
+
+constexpr int kBlk = 16;  // columns per block of the arg-min sweep
 
 // dynamic shared memory of argmin_tc_kernel<HALVES>: A tiles, two B chunks, statistics, H r,
 // alignment
@@ -527,11 +513,10 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
                  int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
                  FlagList flags, StatsView st, const float* __restrict__ cbmax,
                  const char* __restrict__ bpre, const float4* __restrict__ terms, int tiles,
-                 uint32_t key_mask, unsigned* err) {
+                 unsigned* err) {
   pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
   pdl_wait();
   using namespace tcenc;
-  const uint32_t m32 = ~key_mask + 1u, m27 = m32 << 22;  // 32 and 2^27 for pack_key
   extern __shared__ __align__(1024) char smem_raw[];
   // 1024-byte aligned base, derived from the shared array (keeps the shared address space)
   char* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -665,8 +650,13 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
     tc::fence_async_smem();
     half_sync<HALVES>(half);
 
-    uint32_t g1 = 0xffffffffu, g2 = 0xffffffffu;
-    int gidx = 0;
+    // as fp32 bits: the smallest block minimum, its block and the block's 16 values; the
+    // second smallest block minimum
+    uint32_t v1 = 0xffffffffu, v2 = 0xffffffffu;
+    int b1 = 0;
+    uint32_t bv[kBlk];
+#pragma unroll
+    for (int e = 0; e < kBlk; ++e) bv[e] = 0xffffffffu;
     for (int c = 0; c < nchunk; ++c) {
       const int u = t * nchunk + c;
       const int buf = resident ? c : (u & 1);
@@ -702,40 +692,25 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       if (!ok) break;
       if (bimg && !resident && u + 2 < n_uses) fetch(u + 2);  // this buffer is free again
       tc::tc_fence_after();
-      // Epilogue: this warp's 32 rows x 128 columns, four 32-column blocks, one top-2 chain
-      // each.
-      uint32_t a1[4], a2[4];
-#pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        a1[b] = 0xffffffffu;
-        a2[b] = 0xffffffffu;
-      }
+      // Epilogue: this warp's 32 rows x 128 columns as eight blocks of 16. Per block its
+      // minimum (every D >= 0, so the bit patterns order like the values); a block whose
+      // minimum is the row's smallest so far is kept whole (16 selects), the previous best
+      // block's minimum moves to the second smallest. No per-score index.
       const uint32_t base = tmem + ((uint32_t)((warp & 3) * 32) << 16);
 #pragma unroll
-      for (int rnd = 0; rnd < 2; ++rnd) {
-        uint32_t v[64];
-        tc::tmem_ld64_wait(base + 64 * rnd, v);
-        const uint32_t* v0 = v;
-        const uint32_t* v1 = v + 32;
+      for (int rnd = 0; rnd < 4; ++rnd) {
+        uint32_t v[32];
+        tc::tmem_ld32_nowait(base + 32 * rnd, v);
+        tc::tmem_wait_ld_dep(v);
 #pragma unroll
-        for (int j = 0; j < 32; ++j) {
-          const uint32_t k0 = pack_key(v0[j], (uint32_t)j, key_mask, m27, m32);
-          const uint32_t k1 = pack_key(v1[j], (uint32_t)j, key_mask, m27, m32);
-          const uint32_t h0 = max(a1[2 * rnd], k0), h1 = max(a1[2 * rnd + 1], k1);
-          a1[2 * rnd] = min(a1[2 * rnd], k0);
-          a1[2 * rnd + 1] = min(a1[2 * rnd + 1], k1);
-          a2[2 * rnd] = min(a2[2 * rnd], h0);
-          a2[2 * rnd + 1] = min(a2[2 * rnd + 1], h1);
-        }
-      }
+        for (int q = 0; q < 32 / kBlk; ++q) {
+          const uint32_t m = min16_bits(v + kBlk * q);
+          v2 = min(v2, max(v1, m));
+          const bool lt = m < v1;
+          v1 = lt ? m : v1;
+          b1 = lt ? (c * kTcCols + 32 * rnd + kBlk * q) / kBlk : b1;
 #pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        if (a1[b] < g1) {
-          g2 = min(g1, a2[b]);
-          g1 = a1[b];
-          gidx = c * kTcCols + 32 * b + (int)(a1[b] & 31u);
-        } else {
-          g2 = min(g2, a1[b]);
+          for (int e = 0; e < kBlk; ++e) bv[e] = lt ? v[kBlk * q + e] : bv[e];
         }
       }
       tc::tc_fence_before();
@@ -743,10 +718,23 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
     }
     if (!ok) break;
 
-    // Certificate, code, flag and statistics of this thread's row.
+    // Certificate, code, flag and statistics of this thread's row. j = the smallest D (ties to
+    // the smaller column), k2 = the second smallest D over the row (the winning block's second
+    // value or the other blocks' smallest minimum).
     if (row_ok) {
-      int j = gidx;
-      const float k1 = __uint_as_float(g1), k2 = __uint_as_float(g2);
+      uint32_t w1 = bv[0], w2 = 0xffffffffu;
+      int jb = 0;
+#pragma unroll
+      for (int e = 1; e < kBlk; ++e) {
+        w2 = min(w2, max(w1, bv[e]));
+        const bool lt = bv[e] < w1;
+        w1 = lt ? bv[e] : w1;
+        jb = lt ? e : jb;
+      }
+      int j = b1 * kBlk + jb;
+      const uint32_t s2 = min(v2, w2);
+      const float k1 = __uint_as_float(w1);
+      const float k2 = s2 == 0xffffffffu ? INFINITY : __uint_as_float(s2);
       bool cert = false;
       float thr = INFINITY;
       if (j < cw.K) {
@@ -761,10 +749,11 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
           load_vec(cw.C + (int64_t)j * kD, cv);
           codeword_terms(cv, sH, n, na, l1);
         }
-        // |key - D| <= 2^-18 D; D_k <= s_k + off (every k); s_j + off <= D_j + e2 (winner).
+        // D_k <= s_k + off (every k); s_j + off <= D_j + e2 (the winner): no other codeword's
+        // exact score reaches s_j when k2 > D_j + e2 (the sum rounded up).
         const float e2 = 2.f * uc * (na + 2.f * pmax * l1 + off);
-        const float top = k1 * (1.f + 2.5f * kPack) + e2;   // >= s_j + off
-        cert = cw.K == 1 || (k2 * (1.f - kPack) > top);
+        const float top = __fadd_ru(k1, e2);   // >= s_j + off
+        cert = cw.K == 1 || k2 > top;
         thr = top - off;
         thr += 4.f * kU * (k1 + off + e2);
       } else {
@@ -1178,7 +1167,7 @@ __device__ __forceinline__ void hyp_terms_pair(const float rh[kD], const float r
 // Fast stage: one thread per vector, the stage codebook chunked through shared memory, a
 // sorted top-L list (L >= Bs + 1) of lower bounds low = approx_err - Et in registers.
 template <int L>
-__global__ void __launch_bounds__(kThreads, L < 9 ? 3 : 2)
+__global__ void __launch_bounds__(kThreads, L <= 9 ? 3 : 2)
 beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc sd,
                   BeamBufs bb, FlagList flags, unsigned* err) {
   const int64_t g = g_begin + blockIdx.y;
@@ -1227,9 +1216,7 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
       hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
       const float base = rr - kU * cmul * ra;
       const float nbeta = -2.f * kU * cmul * pmax;
-      // two codewords per step: their FMA chains are independent, so they overlap (the chain
-      // of one score is ten dependent operations)
-      auto score = [&](int k) {
+      for (int k = 0; k < nk; ++k) {
         const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
         const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
         float s = base + sN[k];
@@ -1241,9 +1228,7 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
         s = fmaf(m2q[5], c1.y, s);
         s = fmaf(m2q[6], c1.z, s);
         s = fmaf(m2q[7], c1.w, s);
-        return fmaf(nbeta, sL[k], s);
-      };
-      auto insert = [&](float s, int k) {
+        s = fmaf(nbeta, sL[k], s);
         if (s < topv[L - 1]) {
           float sv = s;
           int sh = h, sk = k0 + k;
@@ -1257,14 +1242,7 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
             }
           }
         }
-      };
-      int k = 0;
-      for (; k + 1 < nk; k += 2) {
-        const float sa = score(k), sb = score(k + 1);
-        insert(sa, k);  // in codeword order, as one at a time
-        insert(sb, k + 1);
       }
-      if (k < nk) insert(score(k), k);
     }
   }
   if (!live) return;
@@ -1794,11 +1772,11 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
         if (two_halves)
           CRVQ_CUDA(launch_pdl(argmin_tc_kernel<2>, grid, dim3(256), argmin_smem(2), stream, set,
                                gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax,
-                               bimg, tout, tiles, kKeyMask, err));
+                               bimg, tout, tiles, err));
         else
           CRVQ_CUDA(launch_pdl(argmin_tc_kernel<1>, grid, dim3(128), argmin_smem(1), stream, set,
                                gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax,
-                               bimg, tout, tiles, kKeyMask, err));
+                               bimg, tout, tiles, err));
         CRVQ_LAUNCHED();
       }
       {

@@ -268,3 +268,30 @@ def test_full_size_encode_pass_and_update_k65536():
     _cmp_codebook(host(Cg), Co.astype(np.float64))
     empty = co == 0
     np.testing.assert_array_equal(host(Cg)[empty], C[empty])
+
+
+@pytest.mark.parametrize("name", ["c2", "c3", "c4"])
+def test_full_size_dense_hessian(name):
+    """The dense crvq_hessian (S1, H = X^T X / n + delta I with delta a fraction of the mean
+    diagonal; Sec. 3.1 and Alg. 1) at full size: N = 4096 from 4096 tokens, N = 11008 (a ragged
+    last 128-channel tile) and N = 8192 from 2048 tokens, against the oracle's fp64 H entry by
+    entry at 2e-5 sqrt(H_aa H_bb), with delta, xsq and the stored diagonal blocks."""
+    import paper_2412_09282_gb300 as P
+    cfg = CASES[name]
+    X = S.gen_X(cfg)
+    H, xsq, Hb, delta = P.crvq_hessian(dev(X), cfg.damp_rel, D)
+    P.crvq_sync()
+    Ho, xo, _, do = O.hessian(X, cfg.damp_rel, D)
+    del X
+    Hg = host(H)
+    del H
+    dg = np.sqrt(np.diag(Ho))
+    for a in range(0, cfg.N, 1024):                 # row slabs bound the temporaries
+        sl = slice(a, min(a + 1024, cfg.N))
+        assert np.all(np.abs(Hg[sl] - Ho[sl]) <= 2e-5 * np.outer(dg[sl], dg) + 1e-30), a
+        np.testing.assert_array_equal(Hg[sl], Hg[:, sl].T)
+    np.testing.assert_allclose(host(xsq), xo, rtol=2e-5)
+    assert abs(float(host(delta)[0]) - float(do)) <= 2e-5 * abs(float(do))
+    Hbg = host(Hb)
+    for g in np.random.default_rng(5).choice(cfg.N // D, 64, replace=False):
+        np.testing.assert_array_equal(Hbg[g], Hg[g * D:(g + 1) * D, g * D:(g + 1) * D])
