@@ -27,7 +27,7 @@ namespace crvq {
 namespace {
 
 constexpr int kThreads = 128;
-constexpr int kChunk = 1024;            // codewords staged per shared-memory chunk
+constexpr int kChunk = 256;             // codewords staged per shared-memory chunk
 constexpr float kU = 5.9604645e-08f;    // 2^-24
 
 // Error-bound multiplier: about twice the worst-case FMA-chain analysis (<= 37 + 2 n_fixed).
@@ -177,11 +177,11 @@ __device__ __forceinline__ void vector_terms_rr(const float r[kD], const float a
   }
 }
 
-// Stage the codewords [k0, k0 + nk): sC = c, sN = n - u C Na (the lower-bound offset of the
-// codeword part), sL = ||c||_1.
+// Stage the codewords [k0, k0 + nk): sC = c, sNL = (n - u C Na, ||c||_1) (the lower-bound
+// offset of the codeword part and its L1 norm), sNa = Na.
 __device__ __forceinline__ void stage_chunk(const float* __restrict__ C, int k0, int nk,
-                                            const float* sH, float cmul, float* sC, float* sN,
-                                            float* sL) {
+                                            const float* sH, float cmul, float* sC, float2* sNL,
+                                            float* sNa) {
   for (int k = threadIdx.x; k < nk; k += blockDim.x) {
     float c[kD];
     load_vec(C + (int64_t)(k0 + k) * kD, c);
@@ -189,8 +189,8 @@ __device__ __forceinline__ void stage_chunk(const float* __restrict__ C, int k0,
     codeword_terms(c, sH, n, na, l1);
     *reinterpret_cast<float4*>(sC + k * kD) = make_float4(c[0], c[1], c[2], c[3]);
     *reinterpret_cast<float4*>(sC + k * kD + 4) = make_float4(c[4], c[5], c[6], c[7]);
-    sN[k] = n - kU * cmul * na;
-    sL[k] = l1;
+    sNL[k] = make_float2(n - kU * cmul * na, l1);
+    sNa[k] = na;
   }
 }
 
@@ -1164,6 +1164,9 @@ __device__ __forceinline__ void hyp_terms_pair(const float rh[kD], const float r
   }
 }
 
+constexpr int kBeamCand = 16;  // candidate buffer slots per thread
+constexpr int kBeamScan = 8;   // scores between two overflow checks
+
 // Fast stage: one thread per vector, the stage codebook chunked through shared memory, a
 // sorted top-L list (L >= Bs + 1) of lower bounds low = approx_err - Et in registers.
 template <int L>
@@ -1177,7 +1180,11 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
   const int64_t vi = live ? i * G_range + (g - g_begin) : 0;
   __shared__ float sH[kD * kD];
   __shared__ __align__(16) float sC[kChunk * kD];
-  __shared__ float sN[kChunk], sL[kChunk];
+  __shared__ __align__(8) float2 sNL[kChunk];
+  __shared__ float sNa[kChunk];
+  // candidate buffers, [slot][thread]: (score bits, (h << 16) | k)
+  __shared__ uint2 cand[kBeamCand * kThreads];
+  __shared__ float sRa[16 * kThreads], sPm[16 * kThreads];  // Ra_h, Pmax_h, [h][thread]
   if (threadIdx.x < kD * kD) sH[threadIdx.x] = set.Hb[g * kD * kD + threadIdx.x];
   __syncthreads();
 
@@ -1194,18 +1201,47 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
   }
 
   float topv[L];
-  int toph[L], topk[L];
+  int topi[L];  // (h << 16) | k: B <= 16 hypotheses, K <= 65536 codewords
 #pragma unroll
   for (int j = 0; j < L; ++j) {
     topv[j] = INFINITY;
-    toph[j] = 0x7fffffff;
-    topk[j] = 0x7fffffff;
+    topi[j] = 0x7fffffff;
   }
 
+  // Scores below the list's last entry (as of the last flush) are appended to this thread's
+  // candidate buffer in shared memory: a predicated store per score, no branch. Every kBeamScan
+  // scores the warp flushes when any lane's buffer could overflow within the next stretch:
+  // the buffered candidates, in (h, k) order, go through the sorted insertion (ties keep the
+  // earlier candidate ahead, as inserting every score in order would). The insertion network,
+  // which the compiler predicates, thus runs per candidate instead of per score.
+  int nc = 0;
+  float thr = INFINITY;
+  auto flush = [&]() {
+    for (int e = 0; e < nc; ++e) {
+      const uint2 ce = cand[e * kThreads + threadIdx.x];
+      float sv = __uint_as_float(ce.x);
+      int si = (int)ce.y;
+      if (sv < topv[L - 1]) {
+#pragma unroll
+        for (int j = 0; j < L; ++j) {
+          if (sv < topv[j]) {
+            const float tv = topv[j];
+            const int ti = topi[j];
+            topv[j] = sv;
+            topi[j] = si;
+            sv = tv;
+            si = ti;
+          }
+        }
+      }
+    }
+    nc = 0;
+    thr = topv[L - 1];
+  };
   for (int k0 = 0; k0 < cw.K; k0 += kChunk) {
     const int nk = min(kChunk, cw.K - k0);
     __syncthreads();
-    stage_chunk(cw.C, k0, nk, sH, cmul, sC, sN, sL);
+    stage_chunk(cw.C, k0, nk, sH, cmul, sC, sNL, sNa);
     __syncthreads();
     if (!live) continue;
     for (int h = 0; h < Bh; ++h) {
@@ -1214,36 +1250,62 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
       hyp_residual_pair(th, tl, cbs, sd, pc, rh, rl, err);
       float m2q[kD], rr, ra, pmax;
       hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
+      sRa[h * kThreads + threadIdx.x] = ra;  // the same values in every chunk
+      sPm[h * kThreads + threadIdx.x] = pmax;
       const float base = rr - kU * cmul * ra;
       const float nbeta = -2.f * kU * cmul * pmax;
-      for (int k = 0; k < nk; ++k) {
+      // One score: a chain of ten dependent operations; four independent chains per step.
+      // Every score is stored into slot nc, which advances only for a candidate (no branch);
+      // nc <= kBeamCand - kBeamScan after each check, so the at most kBeamScan stores that
+      // follow stay below kBeamCand.
+      auto score_at = [&](int k) {
         const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
         const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
-        float s = base + sN[k];
-        s = fmaf(m2q[0], c0.x, s);
-        s = fmaf(m2q[1], c0.y, s);
-        s = fmaf(m2q[2], c0.z, s);
-        s = fmaf(m2q[3], c0.w, s);
-        s = fmaf(m2q[4], c1.x, s);
-        s = fmaf(m2q[5], c1.y, s);
-        s = fmaf(m2q[6], c1.z, s);
-        s = fmaf(m2q[7], c1.w, s);
-        s = fmaf(nbeta, sL[k], s);
-        if (s < topv[L - 1]) {
-          float sv = s;
-          int sh = h, sk = k0 + k;
+        const float2 nl = sNL[k];
+        float sc = base + nl.x;
+        sc = fmaf(m2q[0], c0.x, sc);
+        sc = fmaf(m2q[1], c0.y, sc);
+        sc = fmaf(m2q[2], c0.z, sc);
+        sc = fmaf(m2q[3], c0.w, sc);
+        sc = fmaf(m2q[4], c1.x, sc);
+        sc = fmaf(m2q[5], c1.y, sc);
+        sc = fmaf(m2q[6], c1.z, sc);
+        sc = fmaf(m2q[7], c1.w, sc);
+        return fmaf(nbeta, nl.y, sc);
+      };
+      const uint32_t hk = ((uint32_t)h << 16) | (uint32_t)k0;
+      for (int kb = 0; kb < nk; kb += kBeamScan) {
+        if (__any_sync(__activemask(), nc > kBeamCand - kBeamScan)) flush();
+        if (kb + kBeamScan <= nk) {
 #pragma unroll
-          for (int j = 0; j < L; ++j) {
-            if (sv < topv[j]) {
-              const float tv = topv[j];
-              const int th = toph[j], tk = topk[j];
-              topv[j] = sv; toph[j] = sh; topk[j] = sk;
-              sv = tv; sh = th; sk = tk;
+          for (int e0 = 0; e0 < kBeamScan; e0 += 4) {
+            float sc[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) sc[e] = score_at(kb + e0 + e);
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              cand[nc * kThreads + threadIdx.x] =
+                  make_uint2(__float_as_uint(sc[e]), hk + (uint32_t)(kb + e0 + e));
+              nc += sc[e] < thr ? 1 : 0;
             }
+          }
+        } else {
+          for (int k = kb; k < nk; ++k) {
+            const float s1 = score_at(k);
+            cand[nc * kThreads + threadIdx.x] =
+                make_uint2(__float_as_uint(s1), hk + (uint32_t)k);
+            nc += s1 < thr ? 1 : 0;
           }
         }
       }
     }
+  }
+  if (live) flush();
+  int toph[L], topk[L];
+#pragma unroll
+  for (int j = 0; j < L; ++j) {
+    toph[j] = topi[j] == 0x7fffffff ? 0x7fffffff : (topi[j] >> 16);
+    topk[j] = topi[j] == 0x7fffffff ? 0x7fffffff : (topi[j] & 0xffff);
   }
   if (!live) return;
 
@@ -1259,20 +1321,26 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
       topk[j] = 0;
     }
   }
-  // Per-entry bound Et = u C (Ra_h + Na_k + 2 Pmax_h L1_k) for the listed entries.
+  // Per-entry bound Et = u C (Ra_h + Na_k + 2 Pmax_h L1_k) for the listed entries, from the
+  // hypothesis terms kept in the sweep and the staged codeword terms (recomputed when the
+  // codebook spans several chunks).
+  const bool one_chunk = cw.K <= kChunk;
   float et[L];
 #pragma unroll
   for (int j = 0; j < L; ++j) {
     et[j] = 0.f;
     if (j < nkept) {
-      float rh[kD], rl[kD];
-      const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
-      hyp_residual_pair(th, tl, cbs, sd, pc, rh, rl, err);
-      float m2q[kD], rr, ra, pmax;
-      hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
-      float c[kD], n, na, l1;
-      load_vec(cw.C + (int64_t)topk[j] * kD, c);
-      codeword_terms(c, sH, n, na, l1);
+      const float ra = sRa[toph[j] * kThreads + threadIdx.x];
+      const float pmax = sPm[toph[j] * kThreads + threadIdx.x];
+      float na, l1;
+      if (one_chunk) {
+        na = sNa[topk[j]];
+        l1 = sNL[topk[j]].y;
+      } else {
+        float c[kD], n;
+        load_vec(cw.C + (int64_t)topk[j] * kD, c);
+        codeword_terms(c, sH, n, na, l1);
+      }
       et[j] = kU * cmul * (ra + na + 2.f * pmax * l1);
     }
   }
