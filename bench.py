@@ -60,7 +60,7 @@ def schedule_scores(cfg, M, N):
 # the two DRAM counters; the summary is kept with the other profiles). None for a workload
 # whose counters have not been taken, and whenever the kernel changes until they are taken
 # again.
-ARGMIN_TRAFFIC = {"c5": 77.53e6}
+ARGMIN_TRAFFIC = {}
 
 # The tf32 tensor rate relative to bf16 (nominal dense figures of the part: 1.1 vs 2.25
 # PFLOP/s). Only the bf16 rate is measured; the arg-min's MMAs are kind::tf32.

@@ -669,9 +669,14 @@ crvq_status lloyd(const SetView& set, CbList cbs, int iters, const EncodeExtras&
   CRVQ_TRY(launch_stats_prepare(set, cbs, j, st, s));  // T, H and fixed codebooks stay put
   const size_t wbytes = argmin_scratch_bytes(set.M, cbs.cb[j].G_cov, cbs.cb[j].K);
   CRVQ_TRY(wmem.alloc(wbytes, s));
+  // the arg-min's per-vector terms, once for all iterations
+  Scratch rmem;
+  CRVQ_TRY(rmem.alloc((size_t)3 * set.M * set.G_sub * sizeof(float4), s));
+  CRVQ_TRY(launch_row_terms(set, cbs, j, rmem.as<float4>(), s));
   EncodeExtras ex = ex0;
   ex.work = wmem.as<char>();
   ex.work_bytes = wbytes;
+  ex.rowterms = rmem.as<float4>();
   EncodeExtras ex_last = ex;
   ex.stats = &st;
   for (int it = 0; it < iters; ++it) {

@@ -451,6 +451,29 @@ __device__ __forceinline__ bool less(float ah, float al, int ak, float bh, float
 
 }  // namespace dfl
 
+// Per-vector terms of the arg-min's A rows that do not change while one codebook's Lloyd
+// iterations run (the target, H_g and the fixed codebooks stay put): m2q = -2 H_g r and rr,
+// Ra, Pmax (vector_terms_rr of target32), as three planes of M float4 per group,
+// rt[(3 g + p) M + i]: p = 0, 1 the two halves of m2q, p = 2 (rr, Ra, Pmax, 0). The arg-min
+// pass reads them instead of recomputing them, with bit-identical values.
+__global__ void __launch_bounds__(128)
+row_terms_kernel(SetView set, CbList cbs, int n_fixed, float4* __restrict__ rt,
+                 unsigned* err) {
+  pdl_trigger();
+  pdl_wait();
+  const int64_t nvec = set.M * set.G_sub;
+  for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < nvec;
+       v += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t g = v / set.M, i = v - g * set.M;
+    float rv[kD], a[kD], m2q[kD], pmax, rr, ra;
+    target32(set, cbs, n_fixed, i, g, rv, a, err);
+    vector_terms_rr(rv, a, set.Hb + g * kD * kD, m2q, pmax, rr, ra);  // H_g 16-byte aligned
+    rt[(3 * g) * set.M + i] = make_float4(m2q[0], m2q[1], m2q[2], m2q[3]);
+    rt[(3 * g + 1) * set.M + i] = make_float4(m2q[4], m2q[5], m2q[6], m2q[7]);
+    rt[(3 * g + 2) * set.M + i] = make_float4(rr, ra, pmax, 0.f);
+  }
+}
+
 // Arg-min over one codebook on the tensor cores. A CTA walks `tiles` consecutive row tiles of
 // one group (thread = row = tensor-memory lane) with a 128-column accumulator per tile in
 // flight. HALVES = 1: 128 threads, three CTAs per SM, any codebook size (codeword chunks of 128
@@ -512,8 +535,8 @@ __global__ void __launch_bounds__(128 * HALVES, HALVES == 1 ? 3 : 2)
 argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_idx,
                  int32_t* __restrict__ out_code, int64_t out_ld, int64_t out_g0,
                  FlagList flags, StatsView st, const float* __restrict__ cbmax,
-                 const char* __restrict__ bpre, const float4* __restrict__ terms, int tiles,
-                 unsigned* err) {
+                 const char* __restrict__ bpre, const float4* __restrict__ terms,
+                 const float4* __restrict__ rowterms, int tiles, unsigned* err) {
   pdl_trigger();  // dependents may launch; this grid waits for its predecessor first
   pdl_wait();
   using namespace tcenc;
@@ -610,15 +633,29 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
     // Prologue: this thread's A row.
     float pmax, off;
     {
-      float rv[kD], a[kD], m2q[kD];
-      if (row_ok) {
-        target32(set, cbs, n_fixed, i, g, rv, a, err);
+      float m2q[kD], rr, ra;
+      if (rowterms) {  // precomputed for this Lloyd loop (row_terms_kernel)
+        float4 q0 = make_float4(0.f, 0.f, 0.f, 0.f), q1 = q0, t2 = q0;
+        if (row_ok) {
+          q0 = rowterms[(3 * g) * set.M + i];
+          q1 = rowterms[(3 * g + 1) * set.M + i];
+          t2 = rowterms[(3 * g + 2) * set.M + i];
+        }
+        m2q[0] = q0.x; m2q[1] = q0.y; m2q[2] = q0.z; m2q[3] = q0.w;
+        m2q[4] = q1.x; m2q[5] = q1.y; m2q[6] = q1.z; m2q[7] = q1.w;
+        rr = t2.x;
+        ra = t2.y;
+        pmax = t2.z;
       } else {
+        float rv[kD], a[kD];
+        if (row_ok) {
+          target32(set, cbs, n_fixed, i, g, rv, a, err);
+        } else {
 #pragma unroll
-        for (int j = 0; j < kD; ++j) rv[j] = a[j] = 0.f;
+          for (int j = 0; j < kD; ++j) rv[j] = a[j] = 0.f;
+        }
+        vector_terms_rr(rv, a, sH, m2q, pmax, rr, ra);
       }
-      float rr, ra;
-      vector_terms_rr(rv, a, sH, m2q, pmax, rr, ra);
       // offset making every D = low + off >= 0, with margins for every rounding involved
       off = (rr + 32.f * kU * ra + 2.f * uc * (hrow * l1max * cinf + 2.f * pmax * l1max)) *
                 (1.f + 4.f * uc) + 1e-30f;
@@ -1840,11 +1877,11 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
         if (two_halves)
           CRVQ_CUDA(launch_pdl(argmin_tc_kernel<2>, grid, dim3(256), argmin_smem(2), stream, set,
                                gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax,
-                               bimg, tout, tiles, err));
+                               bimg, tout, ex.rowterms, tiles, err));
         else
           CRVQ_CUDA(launch_pdl(argmin_tc_kernel<1>, grid, dim3(128), argmin_smem(1), stream, set,
                                gs, cbs, n_fixed, s_idx, out, out_ld, out_g0, fl, st, cbmax,
-                               bimg, tout, tiles, err));
+                               bimg, tout, ex.rowterms, tiles, err));
         CRVQ_LAUNCHED();
       }
       {
@@ -1936,6 +1973,19 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
 }
 
 }  // namespace
+
+crvq_status launch_row_terms(const SetView& set, const CbList& cbs, int n_fixed, float4* rt,
+                             cudaStream_t stream) {
+  const int64_t nvec = set.M * set.G_sub;
+  if (nvec == 0) return CRVQ_OK;
+  unsigned* err = nullptr;
+  CRVQ_TRY(device_error_word(&err));
+  const unsigned blocks = (unsigned)std::min<int64_t>(ceil_div(nvec, 128), 16 * sm_count());
+  CRVQ_CUDA(launch_pdl(row_terms_kernel, dim3(blocks), dim3(128), 0, stream, set, cbs, n_fixed,
+                       rt, err));
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
+}
 
 size_t argmin_scratch_bytes(int64_t M, int64_t G_range, int K) {
   return argmin_layout(M, G_range, K).total;

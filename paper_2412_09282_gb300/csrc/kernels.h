@@ -76,7 +76,15 @@ struct EncodeExtras {
   // that its iterations allocate nothing); used when at least argmin_scratch_bytes long.
   char* work = nullptr;
   size_t work_bytes = 0;
+  // Per-vector A-row terms of the arg-min pass for every group of the set (launch_row_terms),
+  // valid while the target, the H blocks and the fixed codebooks stay put; null: computed in
+  // the pass.
+  const float4* rowterms = nullptr;
 };
+
+// The arg-min pass's per-vector terms for all M x G_sub vectors of the set (3 M G_sub float4).
+crvq_status launch_row_terms(const SetView& set, const CbList& cbs, int n_fixed, float4* rt,
+                             cudaStream_t stream);
 
 // Scratch of one arg-min pass over a set of M rows and G_range groups with a K-entry codebook
 // (B images, codeword terms, codebook maxima, flag list).
