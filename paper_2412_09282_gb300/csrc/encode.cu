@@ -1201,6 +1201,132 @@ __device__ __forceinline__ void hyp_terms_pair(const float rh[kD], const float r
   }
 }
 
+// The end of a fast stage for one vector, given its sorted top-L list (topv, topi) of fp32
+// lower bounds low = approx_err - Et built in (h, k) order: bounds of the listed entries, the
+// fast certificate, the fp32-pair exact path, the flag for the fallback, and the kept tuples.
+// sRa / sPm: Ra_h, Pmax_h of this thread's hypotheses at [h * stride]; sNL / sNa: the staged
+// codeword terms (used when the whole codebook was staged, else recomputed).
+template <int L>
+__device__ __forceinline__ void beam_list_finish(
+    const SetView& set, const CbList& cbs, const StageDesc& sd, const BeamBufs& bb,
+    const FlagList& flags, int64_t i, int64_t g, int64_t vi, int Bh, float cmul,
+    const float th[kD], const float tl[kD], const float* sH, const float2* sNL,
+    const float* sNa, bool one_chunk, const float* sRa, const float* sPm, int stride,
+    float topv[L], int topi[L], unsigned* err) {
+  const CbView cw = cbs.cb[sd.st[sd.s]];
+  const int S = sd.S, B = sd.B, Bs = sd.Bs;
+  int toph[L], topk[L];
+#pragma unroll
+  for (int j = 0; j < L; ++j) {
+    toph[j] = topi[j] == 0x7fffffff ? 0x7fffffff : (topi[j] >> 16);
+    topk[j] = topi[j] == 0x7fffffff ? 0x7fffffff : (topi[j] & 0xffff);
+  }
+  const int64_t total = (int64_t)Bh * cw.K;
+  const int nkept = (int)min((int64_t)L, total);
+  const int keep = (int)min((int64_t)Bs, total);
+  // Non-finite scores never enter the list; keep indices valid and report it.
+#pragma unroll
+  for (int j = 0; j < L; ++j) {
+    if (j < nkept && (toph[j] >= Bh || topk[j] >= cw.K)) {
+      raise_error(err, ERRBIT_NUMERIC);
+      toph[j] = 0;
+      topk[j] = 0;
+    }
+  }
+  // Per-entry bound Et = u C (Ra_h + Na_k + 2 Pmax_h L1_k) for the listed entries, from the
+  // hypothesis terms kept in the sweep and the staged codeword terms (recomputed when the
+  // codebook spans several chunks).
+  float et[L];
+#pragma unroll
+  for (int j = 0; j < L; ++j) {
+    et[j] = 0.f;
+    if (j < nkept) {
+      const float ra = sRa[toph[j] * stride];
+      const float pmax = sPm[toph[j] * stride];
+      float na, l1;
+      if (one_chunk) {
+        na = sNa[topk[j]];
+        l1 = sNL[topk[j]].y;
+      } else {
+        float c[kD], n;
+        load_vec(cw.C + (int64_t)topk[j] * kD, c);
+        codeword_terms(c, sH, n, na, l1);
+      }
+      et[j] = kU * cmul * (ra + na + 2.f * pmax * l1);
+    }
+  }
+  // Fast certificate: low_{j+1} - low_j > 2 Et_j for j < min(keep, total - 1) (every
+  // candidate outside the list has low >= the last list entry).
+  bool ok = true;
+  const int lim = (int)min((int64_t)keep, total - 1);
+#pragma unroll
+  for (int j = 0; j < L - 1; ++j)
+    if (j < lim && !(topv[j + 1] - topv[j] > 2.f * et[j])) ok = false;
+
+  int32_t* out = bb.hyp_out + vi * B * S;
+  if (!ok) {
+    // Exact path on the listed candidates: errs as fp32 pairs (about 2^-44 relative; no fp64),
+    // (err, h, k) order; then every unlisted candidate must have low >= the last listed low,
+    // which must exceed an upper bound of the keep-th err.
+    float evh[L], evl[L];
+#pragma unroll
+    for (int j = 0; j < L; ++j) {
+      evh[j] = INFINITY;
+      evl[j] = 0.f;
+      if (j < nkept) {
+        float rh[kD], rl[kD], c[kD];
+        const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
+        hyp_residual_pair(th, tl, cbs, sd, pc, rh, rl, err);
+        load_vec(cw.C + (int64_t)topk[j] * kD, c);
+        dfl::quad_err(rh, rl, c, sH, evh[j], evl[j]);
+      }
+    }
+    const float last_low = topv[nkept - 1];
+#pragma unroll
+    for (int a = 1; a < L; ++a) {
+#pragma unroll
+      for (int b = a; b > 0; --b) {
+        const bool sw = (evh[b] < evh[b - 1]) ||
+                        (evh[b] == evh[b - 1] &&
+                         (evl[b] < evl[b - 1] ||
+                          (evl[b] == evl[b - 1] &&
+                           (toph[b] < toph[b - 1] ||
+                            (toph[b] == toph[b - 1] && topk[b] < topk[b - 1])))));
+        if (sw) {
+          const float t0 = evh[b]; evh[b] = evh[b - 1]; evh[b - 1] = t0;
+          const float t1 = evl[b]; evl[b] = evl[b - 1]; evl[b - 1] = t1;
+          const int th_ = toph[b]; toph[b] = toph[b - 1]; toph[b - 1] = th_;
+          const int tk = topk[b]; topk[b] = topk[b - 1]; topk[b - 1] = tk;
+        }
+      }
+    }
+    // upper bound of the keep-th listed err (the pair's own error is far below 1e-7)
+    const float ev_up = isfinite(evh[keep - 1])
+                            ? __fmul_ru(__fadd_ru(evh[keep - 1], evl[keep - 1]), 1.0000002f)
+                            : INFINITY;
+    const bool cert = total <= L || last_low > ev_up;
+    if (!cert) {
+      const unsigned slot = atomicAdd(flags.count, 1u);
+      if (slot < flags.cap) {
+        flags.vec[slot] = vi;
+        // every member of the exact top-keep has err <= the keep-th listed err
+        flags.thr[slot] = ev_up;
+      } else {
+        raise_error(err, ERRBIT_INDEX);
+      }
+      return;
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < L; ++j) {
+    if (j >= keep) break;
+    const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
+    for (int q = 0; q < sd.s; ++q) out[j * S + q] = pc[q];
+    out[j * S + sd.s] = topk[j];
+  }
+  bb.n_out[vi] = keep;
+}
+
 constexpr int kBeamCand = 16;  // candidate buffer slots per thread
 constexpr int kBeamScan = 8;   // scores between two overflow checks
 
@@ -1226,7 +1352,7 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
   __syncthreads();
 
   const CbView cw = cbs.cb[sd.st[sd.s]];
-  const int S = sd.S, B = sd.B, Bs = sd.Bs;
+  const int S = sd.S, B = sd.B;
   const float cmul = bound_mult(n_fixed + sd.s);
   const int Bh = (sd.s == 0) ? 1 : (live ? bb.n_in[vi] : 1);
   float th[kD], tl[kD];  // target as an fp32 pair (t - the fixed codebooks' codewords)
@@ -1337,120 +1463,271 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
       }
     }
   }
-  if (live) flush();
-  int toph[L], topk[L];
-#pragma unroll
-  for (int j = 0; j < L; ++j) {
-    toph[j] = topi[j] == 0x7fffffff ? 0x7fffffff : (topi[j] >> 16);
-    topk[j] = topi[j] == 0x7fffffff ? 0x7fffffff : (topi[j] & 0xffff);
-  }
   if (!live) return;
+  flush();
+  beam_list_finish<L>(set, cbs, sd, bb, flags, i, g, vi, Bh, cmul, th, tl, sH, sNL, sNa,
+                      cw.K <= kChunk, sRa + threadIdx.x, sPm + threadIdx.x, kThreads, topv,
+                      topi, err);
+}
 
-  const int64_t total = (int64_t)Bh * cw.K;
-  const int nkept = (int)min((int64_t)L, total);
-  const int keep = (int)min((int64_t)Bs, total);
-  // Non-finite scores never enter the list; keep indices valid and report it.
+// Fast stage with the scores on the tensor cores (codebooks of at most 256 codewords, L <= 16).
+// Thread = vector, as in beam_stage_kernel; the CTA's 128 vectors take the hypotheses in turn:
+// for hypothesis h every thread writes its A row, one tcgen05.mma pass computes
+//   y(h, k) = base_h + sN_k + m2q_h . c_k + nbeta_h L1_k
+// for all 128 vectors x 256 codewords (3xTF32 operands: the B images of prep_b built with the
+// stage's bound multiplier), and each thread reads its row from tensor memory. y differs from
+// the fast stage's fp32 chain x(h, k) (the same linear form) by at most eps_h = 2^-12 S_h,
+// S_h = |base_h| + Na_max + 2 Pmax_h L1max + |nbeta_h| L1max, which bounds every term's
+// magnitude (the split products lose about 2^-22 and the fp32 accumulation of 32 terms about
+// 2^-19 of it). A pair whose x could enter the list has y <= (the list's last x, or the bound
+// tau below) + eps_h; only those are buffered, then scored again with exactly the fast stage's
+// chain and inserted in (h, k) order with its rule. Every member of the final top-L is
+// buffered, so the list, and everything after it (beam_list_finish), equals beam_stage_kernel's.
+// tau: for h = 0, the L-th smallest of the 16-column block minima of y: at least L pairs have
+// y <= tau, so the L-th smallest x is at most tau + eps_0.
+constexpr int kTcCand = 64;   // candidate slots per thread (codeword indices, one byte each)
+constexpr size_t kBeamTcSmem = 1024 + (size_t)tcenc::kATile + 2 * (size_t)kTcBTile +
+                               (size_t)kChunk * kD * 4 + (size_t)kChunk * 8 + (size_t)kChunk * 4 +
+                               (size_t)kTcCand * kThreads + 2 * 16 * (size_t)kThreads * 4;
+
+template <int L>
+__global__ void __launch_bounds__(kThreads, 2)
+beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc sd,
+               BeamBufs bb, const char* __restrict__ bimg, const float* __restrict__ cbmax,
+               FlagList flags, unsigned* err) {
+  using namespace tcenc;
+  extern __shared__ __align__(1024) char smem_raw[];
+  char* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
+  char* Atile = smem;
+  char* Bbuf = Atile + kATile;
+  float* sC = reinterpret_cast<float*>(Bbuf + 2 * kTcBTile);
+  float2* sNL = reinterpret_cast<float2*>(sC + kChunk * kD);
+  float* sNa = reinterpret_cast<float*>(sNL + kChunk);
+  uint8_t* cand = reinterpret_cast<uint8_t*>(sNa + kChunk);  // [slot][thread]
+  float* sRa = reinterpret_cast<float*>(cand + kTcCand * kThreads);  // [h][thread]
+  float* sPm = sRa + 16 * kThreads;
+  __shared__ __align__(16) float sH[kD * kD];
+  __shared__ __align__(8) uint64_t bar_b, bar_mma;
+  __shared__ uint32_t tmem_slot;
+
+  const int tid = threadIdx.x, warp = tid >> 5;
+  const int64_t g = g_begin + blockIdx.y;
+  const int64_t G_range = gridDim.y;
+  const int64_t i = (int64_t)blockIdx.x * kThreads + tid;
+  const bool live = i < set.M;
+  const int64_t vi = live ? i * G_range + (g - g_begin) : 0;
+  const CbView cw = cbs.cb[sd.st[sd.s]];
+  const int nchunk = (cw.K + kTcCols - 1) / kTcCols;  // 1 or 2
+  const int S = sd.S, B = sd.B;
+  const float cmul = bound_mult(n_fixed + sd.s);
+
+  if (tid < kD * kD) sH[tid] = set.Hb[g * kD * kD + tid];
+  if (warp == 0) tc::tmem_alloc(&tmem_slot, 2 * kTcCols);
+  if (tid == 0) {
+    tc::mbar_init(tc::smem_u32(&bar_b), 1);
+    tc::mbar_init(tc::smem_u32(&bar_mma), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  tc::tc_fence_before();
+  __syncthreads();
+  tc::tc_fence_after();
+  const uint32_t tmem = tmem_slot;
+  if (tid == 0) {  // this group's B images, one bulk copy per 128-codeword chunk
+    tc::mbar_expect_tx(tc::smem_u32(&bar_b), (uint32_t)(nchunk * kTcBTile));
+    for (int c = 0; c < nchunk; ++c)
+      tc::bulk_copy_g2s(tc::smem_u32(Bbuf + c * kTcBTile),
+                        bimg + ((size_t)(g - g_begin) * nchunk + c) * kTcBTile, kTcBTile,
+                        tc::smem_u32(&bar_b));
+  }
+  stage_chunk(cw.C, 0, cw.K, sH, cmul, sC, sNL, sNa);
+  __syncthreads();
+
+  // Na <= max row sum of |H_g| * L1max * cinf over the codebook (cbmax: L1max, cinf)
+  float hrow = 0.f;
+#pragma unroll
+  for (int a = 0; a < kD; ++a) {
+    float rs = 0.f;
+#pragma unroll
+    for (int b = 0; b < kD; ++b) rs += fabsf(sH[a * kD + b]);
+    hrow = fmaxf(hrow, rs);
+  }
+  const float l1max = cbmax[0], cinf = cbmax[1];
+  const float na_max = hrow * l1max * cinf * (1.f + kU * cmul) * 1.0001f;
+  constexpr uint32_t idesc = tc::idesc_tf32(kRows, kTcCols);
+
+  const int Bh = (sd.s == 0) ? 1 : (live ? bb.n_in[vi] : 1);
+  const int Bmax = (sd.s == 0) ? 1 : B;  // uniform hypothesis loop bound of the CTA
+  float th[kD], tl[kD];
+  if (live) {
+    dfl::target(set, cbs, n_fixed, i, g, th, tl, err);
+  } else {
+#pragma unroll
+    for (int j = 0; j < kD; ++j) th[j] = tl[j] = 0.f;
+  }
+  float topv[L];
+  int topi[L];
 #pragma unroll
   for (int j = 0; j < L; ++j) {
-    if (j < nkept && (toph[j] >= Bh || topk[j] >= cw.K)) {
-      raise_error(err, ERRBIT_NUMERIC);
-      toph[j] = 0;
-      topk[j] = 0;
-    }
+    topv[j] = INFINITY;
+    topi[j] = 0x7fffffff;
   }
-  // Per-entry bound Et = u C (Ra_h + Na_k + 2 Pmax_h L1_k) for the listed entries, from the
-  // hypothesis terms kept in the sweep and the staged codeword terms (recomputed when the
-  // codebook spans several chunks).
-  const bool one_chunk = cw.K <= kChunk;
-  float et[L];
-#pragma unroll
-  for (int j = 0; j < L; ++j) {
-    et[j] = 0.f;
-    if (j < nkept) {
-      const float ra = sRa[toph[j] * kThreads + threadIdx.x];
-      const float pmax = sPm[toph[j] * kThreads + threadIdx.x];
-      float na, l1;
-      if (one_chunk) {
-        na = sNa[topk[j]];
-        l1 = sNL[topk[j]].y;
-      } else {
-        float c[kD], n;
-        load_vec(cw.C + (int64_t)topk[j] * kD, c);
-        codeword_terms(c, sH, n, na, l1);
-      }
-      et[j] = kU * cmul * (ra + na + 2.f * pmax * l1);
-    }
-  }
-  // Fast certificate: low_{j+1} - low_j > 2 Et_j for j < min(keep, total - 1) (every
-  // candidate outside the list has low >= the last list entry).
+  float tau_x = INFINITY;
   bool ok = true;
-  const int lim = (int)min((int64_t)keep, total - 1);
+  const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+  for (int h = 0; h < Bmax && ok; ++h) {
+    const bool act = live && h < Bh;
+    float m2q[kD], base = 0.f, nbeta = 0.f, eps = 0.f;
+    {
+      float rr = 0.f, ra = 0.f, pmax = 0.f;
 #pragma unroll
-  for (int j = 0; j < L - 1; ++j)
-    if (j < lim && !(topv[j + 1] - topv[j] > 2.f * et[j])) ok = false;
-
-  int32_t* out = bb.hyp_out + vi * B * S;
-  if (!ok) {
-    // Exact path on the listed candidates: errs as fp32 pairs (about 2^-44 relative; no fp64),
-    // (err, h, k) order; then every unlisted candidate must have low >= the last listed low,
-    // which must exceed an upper bound of the keep-th err.
-    float evh[L], evl[L];
-#pragma unroll
-    for (int j = 0; j < L; ++j) {
-      evh[j] = INFINITY;
-      evl[j] = 0.f;
-      if (j < nkept) {
-        float rh[kD], rl[kD], c[kD];
-        const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
+      for (int p = 0; p < kD; ++p) m2q[p] = 0.f;
+      if (act) {
+        float rh[kD], rl[kD];
+        const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
         hyp_residual_pair(th, tl, cbs, sd, pc, rh, rl, err);
-        load_vec(cw.C + (int64_t)topk[j] * kD, c);
-        dfl::quad_err(rh, rl, c, sH, evh[j], evl[j]);
+        hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
+        sRa[h * kThreads + tid] = ra;
+        sPm[h * kThreads + tid] = pmax;
+        base = rr - kU * cmul * ra;
+        nbeta = -2.f * kU * cmul * pmax;
+        eps = 2.44140625e-04f *  // 2^-12
+              (fabsf(base) + na_max + 2.f * pmax * l1max * 1.0001f + fabsf(nbeta) * l1max);
       }
+      uint32_t row[kK];
+#pragma unroll
+      for (int p = 0; p < kD; ++p) {
+        uint32_t hh, ll;
+        split(m2q[p], hh, ll);
+        row[p] = hh;
+        row[8 + p] = hh;
+        row[16 + p] = ll;
+      }
+      const uint32_t one = __float_as_uint(1.f);
+      row[24] = one;
+      row[25] = one;
+      split(nbeta, row[26], row[28]);
+      row[27] = row[26];
+      split(base, row[29], row[30]);
+      row[31] = 0u;
+      put_row(Atile, tid, row);
     }
-    const float last_low = topv[nkept - 1];
+    tc::fence_async_smem();
+    tc::tc_fence_before();
+    __syncthreads();
+    if (tid == 0) {
+      bool bok = true;
+      if (h == 0) bok = tc::mbar_wait(tc::smem_u32(&bar_b), 0u, err);
+      if (bok) {
+        tc::tc_fence_after();
+        const uint32_t a0 = tc::smem_u32(Atile);
+        for (int c = 0; c < nchunk; ++c) {
+          const uint32_t b0 = tc::smem_u32(Bbuf + c * kTcBTile);
 #pragma unroll
-    for (int a = 1; a < L; ++a) {
+          for (int ks = 0; ks < kK / 8; ++ks)
+            tc::mma_tf32(tmem + (uint32_t)(c * kTcCols),
+                         tc::smem_desc(a0 + ks * 256, 128, (kK / 4) * 128),
+                         tc::smem_desc(b0 + ks * 256, 128, (kK / 4) * 128), idesc,
+                         ks > 0 ? 1u : 0u);
+        }
+        tc::mma_commit(tc::smem_u32(&bar_mma));
+      } else {
+        tc::mbar_arrive(tc::smem_u32(&bar_mma));  // release the waiters; ok turns false
+      }
+      if (!bok) raise_error(err, ERRBIT_TIMEOUT);
+    }
+    bool wok = tc::mbar_wait(tc::smem_u32(&bar_mma), (uint32_t)(h & 1), err);
+    if (h == 0 && tid == 0) wok = wok && tc::mbar_try_wait(tc::smem_u32(&bar_b), 0u);
+    ok = __syncthreads_and(wok);
+    if (!ok) break;
+    tc::tc_fence_after();
+
+    const int ncol = nchunk * kTcCols;
+    if (h == 0) {  // tau from the block minima of y for hypothesis 0
+      float bl[L];
 #pragma unroll
-      for (int b = a; b > 0; --b) {
-        const bool sw = (evh[b] < evh[b - 1]) ||
-                        (evh[b] == evh[b - 1] &&
-                         (evl[b] < evl[b - 1] ||
-                          (evl[b] == evl[b - 1] &&
-                           (toph[b] < toph[b - 1] ||
-                            (toph[b] == toph[b - 1] && topk[b] < topk[b - 1])))));
-        if (sw) {
-          const float t0 = evh[b]; evh[b] = evh[b - 1]; evh[b - 1] = t0;
-          const float t1 = evl[b]; evl[b] = evl[b - 1]; evl[b - 1] = t1;
-          const int th_ = toph[b]; toph[b] = toph[b - 1]; toph[b - 1] = th_;
-          const int tk = topk[b]; topk[b] = topk[b - 1]; topk[b - 1] = tk;
+      for (int j = 0; j < L; ++j) bl[j] = INFINITY;
+      for (int q = 0; q < ncol / 32; ++q) {
+        uint32_t v[32];
+        __syncwarp();
+        tc::tmem_ld32_nowait(trow + 32 * q, v);
+        tc::tmem_wait_ld_dep(v);
+#pragma unroll
+        for (int b2 = 0; b2 < 2; ++b2) {
+          float m = __uint_as_float(v[16 * b2]);
+#pragma unroll
+          for (int e = 1; e < 16; ++e) m = fminf(m, __uint_as_float(v[16 * b2 + e]));
+          m = (m == m) ? m : INFINITY;  // a block of NaNs holds no bound
+#pragma unroll
+          for (int j = 0; j < L; ++j) {
+            const float t = fmaxf(bl[j], m);
+            bl[j] = fminf(bl[j], m);
+            m = t;
+          }
         }
       }
+      if (act) tau_x = __fadd_ru(bl[L - 1], eps);
     }
-    // upper bound of the keep-th listed err (the pair's own error is far below 1e-7)
-    const float ev_up = isfinite(evh[keep - 1])
-                            ? __fmul_ru(__fadd_ru(evh[keep - 1], evl[keep - 1]), 1.0000002f)
-                            : INFINITY;
-    const bool cert = total <= L || last_low > ev_up;
-    if (!cert) {
-      const unsigned slot = atomicAdd(flags.count, 1u);
-      if (slot < flags.cap) {
-        flags.vec[slot] = vi;
-        // every member of the exact top-keep has err <= the keep-th listed err
-        flags.thr[slot] = ev_up;
-      } else {
-        raise_error(err, ERRBIT_INDEX);
-      }
-      return;
-    }
-  }
+    // candidates of hypothesis h, flushed in (h, k) order
+    int nc = 0;
+    // NaN for a thread without this hypothesis: no value compares below it
+    float thrD = act ? __fadd_ru(fminf(topv[L - 1], tau_x), eps) : __int_as_float(0x7fffffff);
+    auto flush = [&]() {
+      for (int e = 0; e < nc; ++e) {
+        const int k = cand[e * kThreads + tid];
+        if (k >= cw.K) continue;  // padding columns (only with an unbounded threshold)
+        const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
+        const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
+        const float2 nl = sNL[k];
+        float sv = base + nl.x;
+        sv = fmaf(m2q[0], c0.x, sv);
+        sv = fmaf(m2q[1], c0.y, sv);
+        sv = fmaf(m2q[2], c0.z, sv);
+        sv = fmaf(m2q[3], c0.w, sv);
+        sv = fmaf(m2q[4], c1.x, sv);
+        sv = fmaf(m2q[5], c1.y, sv);
+        sv = fmaf(m2q[6], c1.z, sv);
+        sv = fmaf(m2q[7], c1.w, sv);
+        sv = fmaf(nbeta, nl.y, sv);
+        int si = (h << 16) | k;
+        if (sv < topv[L - 1]) {
 #pragma unroll
-  for (int j = 0; j < L; ++j) {
-    if (j >= keep) break;
-    const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + toph[j]) * S : nullptr;
-    for (int q = 0; q < sd.s; ++q) out[j * S + q] = pc[q];
-    out[j * S + sd.s] = topk[j];
+          for (int j = 0; j < L; ++j) {
+            if (sv < topv[j]) {
+              const float tv = topv[j];
+              const int ti = topi[j];
+              topv[j] = sv;
+              topi[j] = si;
+              sv = tv;
+              si = ti;
+            }
+          }
+        }
+      }
+      nc = 0;
+      if (act) thrD = __fadd_ru(fminf(topv[L - 1], tau_x), eps);
+    };
+    for (int q = 0; q < ncol / 32; ++q) {
+      if (__any_sync(0xffffffffu, nc > kTcCand - 32)) flush();
+      uint32_t v[32];
+      __syncwarp();
+      tc::tmem_ld32_nowait(trow + 32 * q, v);
+      tc::tmem_wait_ld_dep(v);
+#pragma unroll
+      for (int e = 0; e < 32; ++e) {
+        cand[nc * kThreads + tid] = (uint8_t)(32 * q + e);
+        nc += (__uint_as_float(v[e]) <= thrD) ? 1 : 0;
+      }
+    }
+    flush();
+    tc::tc_fence_before();
   }
-  bb.n_out[vi] = keep;
+  // let the codebook copy land before the CTA ends (bounded), then free the tensor memory
+  if (!ok && tid == 0) tc::mbar_wait(tc::smem_u32(&bar_b), 0u, err);
+  __syncthreads();
+  if (warp == 0) tc::tmem_dealloc(tmem, 2 * kTcCols);
+  if (!live) return;
+  beam_list_finish<L>(set, cbs, sd, bb, flags, i, g, vi, Bh, cmul, th, tl, sH, sNL, sNa, true,
+                      sRa + tid, sPm + tid, kThreads, topv, topi, err);
 }
 
 // Exact stage for flagged vectors: one warp per vector; the lanes stride over the (h, k)
@@ -1752,6 +2029,63 @@ crvq_status launch_beam_stage_L(const SetView& set, int64_t g_begin, int64_t G_r
   return CRVQ_OK;
 }
 
+template <int L>
+crvq_status launch_beam_tc_L(const SetView& set, int64_t g_begin, int64_t G_range,
+                             const CbList& cbs, int n_fixed, const StageDesc& sd,
+                             const BeamBufs& bb, const char* bimg, const float* cbmax,
+                             const FlagList& fl, unsigned* err, double units,
+                             cudaStream_t stream) {
+  CRVQ_TRY(set_smem_attr(beam_tc_kernel<L>, kBeamTcSmem));
+  dim3 grid((unsigned)ceil_div(set.M, kThreads), (unsigned)G_range);
+  ProfScope ps("encode_beam_stage", stream, units);
+  beam_tc_kernel<L><<<grid, kThreads, kBeamTcSmem, stream>>>(set, g_begin, cbs, n_fixed, sd, bb,
+                                                             bimg, cbmax, fl, err);
+  CRVQ_LAUNCHED();
+  return CRVQ_OK;
+}
+
+// The tensor-core stage for codebooks of at most 256 codewords and lists of at most 9 entries
+// (beam width up to 8): B images of the stage codebook for the group range (prep_b with the
+// stage's bound multiplier), then beam_tc_kernel. `work` holds beam_tc_scratch_bytes.
+size_t beam_tc_scratch_bytes(int64_t G_range, int K) {
+  const int nchunk = (int)ceil_div(K, kTcCols);
+  return 256 + (size_t)G_range * nchunk * kTcBTile +
+         align_up((size_t)G_range * K * sizeof(float4), 256) + 256;
+}
+
+bool beam_tc_applies(const StageDesc& sd, const CbList& cbs, int64_t G_range) {
+  const int K = cbs.cb[sd.st[sd.s]].K;
+  return K <= 2 * kTcCols && sd.Bs + 1 <= 9 &&
+         (size_t)G_range * ceil_div(K, kTcCols) * kTcBTile <= (size_t(256) << 20);
+}
+
+crvq_status launch_beam_stage_tc(const SetView& set, int64_t g_begin, int64_t G_range,
+                                 const CbList& cbs, int n_fixed, const StageDesc& sd,
+                                 const BeamBufs& bb, const FlagList& fl, unsigned* err,
+                                 char* work, double units, cudaStream_t stream) {
+  const CbView& cw = cbs.cb[sd.st[sd.s]];
+  const int nchunk = (int)ceil_div(cw.K, kTcCols);
+  float* cbmax = reinterpret_cast<float*>(work);
+  char* bimg = work + 256;
+  float4* tout = reinterpret_cast<float4*>(bimg + (size_t)G_range * nchunk * kTcBTile);
+  const float uc = kU * bound_mult(n_fixed + sd.s);
+  {
+    ProfScope pb("encode_prep_b", stream, (double)G_range * nchunk * kTcCols);
+    const int64_t rows = G_range * nchunk * kTcCols;
+    CRVQ_CUDA(launch_pdl(prep_b_kernel,
+                         dim3((unsigned)std::min<int64_t>(ceil_div(rows, 128), 16 * sm_count()) +
+                              1),
+                         dim3(128), 0, stream, set, g_begin, G_range, cw.C, cw.K, nchunk, uc,
+                         bimg, tout, cbmax, fl.count));
+    CRVQ_LAUNCHED();
+  }
+  const int need = sd.Bs + 1;
+  if (need <= 2) return launch_beam_tc_L<2>(set, g_begin, G_range, cbs, n_fixed, sd, bb, bimg, cbmax, fl, err, units, stream);
+  if (need <= 3) return launch_beam_tc_L<3>(set, g_begin, G_range, cbs, n_fixed, sd, bb, bimg, cbmax, fl, err, units, stream);
+  if (need <= 5) return launch_beam_tc_L<5>(set, g_begin, G_range, cbs, n_fixed, sd, bb, bimg, cbmax, fl, err, units, stream);
+  return launch_beam_tc_L<9>(set, g_begin, G_range, cbs, n_fixed, sd, bb, bimg, cbmax, fl, err, units, stream);
+}
+
 crvq_status launch_beam_stage(const SetView& set, int64_t g_begin, int64_t G_range,
                               const CbList& cbs, int n_fixed, const StageDesc& sd,
                               const BeamBufs& bb, const FlagList& fl, unsigned* err,
@@ -1943,14 +2277,29 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
   int32_t* out_n = nA;
   double sc = 0.0;
   int64_t parents = 1;
+  // scratch of the tensor-core stages (B images and terms of one stage codebook)
+  size_t tc_bytes = 0;
+  for (int s = 0; s < S; ++s) {
+    StageDesc d = sd;
+    d.s = s;
+    d.Bs = (s == S - 1) ? 1 : B;
+    if (beam_tc_applies(d, cbs, G_range))
+      tc_bytes = std::max(tc_bytes, beam_tc_scratch_bytes(G_range, cbs.cb[sd.st[s]].K));
+  }
+  Scratch tc_mem;
+  if (tc_bytes) CRVQ_TRY(tc_mem.alloc(tc_bytes, stream));
   for (int s = 0; s < S; ++s) {
     sd.s = s;
     sd.Bs = (s == S - 1) ? 1 : B;  // only the best tuple of the last stage is used
     CRVQ_CUDA(cudaMemsetAsync(fl.count, 0, sizeof(unsigned), stream));
     BeamBufs bb{in_h, in_n, out_h, out_n};
     const int K = cbs.cb[sd.st[s]].K;
-    CRVQ_TRY(launch_beam_stage(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err,
-                               (double)nvec * parents * K, stream));
+    if (beam_tc_applies(sd, cbs, G_range))
+      CRVQ_TRY(launch_beam_stage_tc(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err,
+                                    tc_mem.as<char>(), (double)nvec * parents * K, stream));
+    else
+      CRVQ_TRY(launch_beam_stage(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err,
+                                 (double)nvec * parents * K, stream));
     {
       ProfScope ps("encode_beam_fallback", stream, 0.0);
       beam_stage_fallback_kernel<<<4 * nsm, kThreads, 0, stream>>>(
