@@ -1470,7 +1470,7 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
                       topi, err);
 }
 
-// Fast stage with the scores on the tensor cores (codebooks of at most 256 codewords, L <= 16).
+// Fast stage with the scores on the tensor cores (codebooks of at most 256 codewords, L <= 9).
 // Thread = vector, as in beam_stage_kernel; the CTA's 128 vectors take the hypotheses in turn:
 // for hypothesis h every thread writes its A row, one tcgen05.mma pass computes
 //   y(h, k) = base_h + sN_k + m2q_h . c_k + nbeta_h L1_k
@@ -1480,21 +1480,22 @@ beam_stage_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDe
 // S_h = |base_h| + Na_max + 2 Pmax_h L1max + |nbeta_h| L1max, which bounds every term's
 // magnitude (the split products lose about 2^-22 and the fp32 accumulation of 32 terms about
 // 2^-19 of it). A pair whose x could enter the list has y <= (the list's last x, or the bound
-// tau below) + eps_h; only those are buffered, then scored again with exactly the fast stage's
-// chain and inserted in (h, k) order with its rule. Every member of the final top-L is
-// buffered, so the list, and everything after it (beam_list_finish), equals beam_stage_kernel's.
-// tau: for h = 0, the L-th smallest of the 16-column block minima of y: at least L pairs have
-// y <= tau, so the L-th smallest x is at most tau + eps_0.
-constexpr int kTcCand = 64;   // candidate slots per thread (codeword indices, one byte each)
+// tau below) + eps_h; only those are kept (a bit mask per thread), scored again with exactly
+// the fast stage's chain and inserted in (h, k) order with its rule (strictly below the last
+// entry, before the first entry strictly above). Every member of the final
+// top-L is among them, so the list, and everything after it (beam_list_finish), equals
+// beam_stage_kernel's. tau: for h = 0, the L-th smallest of the 16-column block minima of y:
+// at least L pairs have y <= tau, so the L-th smallest x is at most tau + eps_0.
 constexpr size_t kBeamTcSmem = 1024 + (size_t)tcenc::kATile + 2 * (size_t)kTcBTile +
                                (size_t)kChunk * kD * 4 + (size_t)kChunk * 8 + (size_t)kChunk * 4 +
-                               (size_t)kTcCand * kThreads + 2 * 16 * (size_t)kThreads * 4;
+                               2 * 16 * (size_t)kThreads * 4 + 2 * 9 * (size_t)kThreads * 4;
 
 template <int L>
 __global__ void __launch_bounds__(kThreads, 2)
 beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc sd,
                BeamBufs bb, const char* __restrict__ bimg, const float* __restrict__ cbmax,
                FlagList flags, unsigned* err) {
+  static_assert(L <= 9, "the shared-memory list holds 9 entries");
   using namespace tcenc;
   extern __shared__ __align__(1024) char smem_raw[];
   char* smem = smem_raw + ((1024u - (tc::smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -1503,9 +1504,10 @@ beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc 
   float* sC = reinterpret_cast<float*>(Bbuf + 2 * kTcBTile);
   float2* sNL = reinterpret_cast<float2*>(sC + kChunk * kD);
   float* sNa = reinterpret_cast<float*>(sNL + kChunk);
-  uint8_t* cand = reinterpret_cast<uint8_t*>(sNa + kChunk);  // [slot][thread]
-  float* sRa = reinterpret_cast<float*>(cand + kTcCand * kThreads);  // [h][thread]
+  float* sRa = sNa + kChunk;  // [h][thread]
   float* sPm = sRa + 16 * kThreads;
+  float* sTopV = sPm + 16 * kThreads;                          // [j][thread]
+  int* sTopI = reinterpret_cast<int*>(sTopV + 9 * kThreads);  // [j][thread]
   __shared__ __align__(16) float sH[kD * kD];
   __shared__ __align__(8) uint64_t bar_b, bar_mma;
   __shared__ uint32_t tmem_slot;
@@ -1564,13 +1566,15 @@ beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc 
 #pragma unroll
     for (int j = 0; j < kD; ++j) th[j] = tl[j] = 0.f;
   }
-  float topv[L];
-  int topi[L];
+  // The sorted top-L list lives in shared memory ([j][thread]), `last` = its last value: a
+  // candidate that does not enter costs one compare, one that does only the shifts it needs
+  // (a register list would be updated by a predicated network for every candidate).
 #pragma unroll
   for (int j = 0; j < L; ++j) {
-    topv[j] = INFINITY;
-    topi[j] = 0x7fffffff;
+    sTopV[j * kThreads + tid] = INFINITY;
+    sTopI[j * kThreads + tid] = 0x7fffffff;
   }
+  float last = INFINITY;
   float tau_x = INFINITY;
   bool ok = true;
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
@@ -1641,21 +1645,20 @@ beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc 
     if (!ok) break;
     tc::tc_fence_after();
 
-    const int ncol = nchunk * kTcCols;
+    const int nq = nchunk * 2;  // 64-column loads
     if (h == 0) {  // tau from the block minima of y for hypothesis 0
       float bl[L];
 #pragma unroll
       for (int j = 0; j < L; ++j) bl[j] = INFINITY;
-      for (int q = 0; q < ncol / 32; ++q) {
-        uint32_t v[32];
-        __syncwarp();
-        tc::tmem_ld32_nowait(trow + 32 * q, v);
-        tc::tmem_wait_ld_dep(v);
+#pragma unroll 1
+      for (int q = 0; q < nq; ++q) {
+        uint32_t v[64];
+        tc::tmem_ld64_wait(trow + 64 * q, v);
 #pragma unroll
-        for (int b2 = 0; b2 < 2; ++b2) {
-          float m = __uint_as_float(v[16 * b2]);
+        for (int b4 = 0; b4 < 4; ++b4) {
+          float m = __uint_as_float(v[16 * b4]);
 #pragma unroll
-          for (int e = 1; e < 16; ++e) m = fminf(m, __uint_as_float(v[16 * b2 + e]));
+          for (int e = 1; e < 16; ++e) m = fminf(m, __uint_as_float(v[16 * b4 + e]));
           m = (m == m) ? m : INFINITY;  // a block of NaNs holds no bound
 #pragma unroll
           for (int j = 0; j < L; ++j) {
@@ -1667,58 +1670,61 @@ beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc 
       }
       if (act) tau_x = __fadd_ru(bl[L - 1], eps);
     }
-    // candidates of hypothesis h, flushed in (h, k) order
-    int nc = 0;
-    // NaN for a thread without this hypothesis: no value compares below it
-    float thrD = act ? __fadd_ru(fminf(topv[L - 1], tau_x), eps) : __int_as_float(0x7fffffff);
-    auto flush = [&]() {
-      for (int e = 0; e < nc; ++e) {
-        const int k = cand[e * kThreads + tid];
-        if (k >= cw.K) continue;  // padding columns (only with an unbounded threshold)
-        const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
-        const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
-        const float2 nl = sNL[k];
-        float sv = base + nl.x;
-        sv = fmaf(m2q[0], c0.x, sv);
-        sv = fmaf(m2q[1], c0.y, sv);
-        sv = fmaf(m2q[2], c0.z, sv);
-        sv = fmaf(m2q[3], c0.w, sv);
-        sv = fmaf(m2q[4], c1.x, sv);
-        sv = fmaf(m2q[5], c1.y, sv);
-        sv = fmaf(m2q[6], c1.z, sv);
-        sv = fmaf(m2q[7], c1.w, sv);
-        sv = fmaf(nbeta, nl.y, sv);
-        int si = (h << 16) | k;
-        if (sv < topv[L - 1]) {
+    // Candidates of hypothesis h, 64 columns at a time: a mask (a compare and a predicated or
+    // per score), then its members in codeword order, scored again with the fast stage's chain
+    // and inserted; the threshold tightens after every 64 columns. NaN threshold for a thread
+    // without this hypothesis: no value compares below it.
+#pragma unroll 1
+    for (int q = 0; q < nq; ++q) {
+      const float thrD =
+          act ? __fadd_ru(fminf(last, tau_x), eps) : __int_as_float(0x7fffffff);
+      uint32_t m0 = 0u, m1 = 0u;
+      {
+        uint32_t v[64];
+        tc::tmem_ld64_wait(trow + 64 * q, v);
 #pragma unroll
-          for (int j = 0; j < L; ++j) {
-            if (sv < topv[j]) {
-              const float tv = topv[j];
-              const int ti = topi[j];
-              topv[j] = sv;
-              topi[j] = si;
-              sv = tv;
-              si = ti;
+        for (int e = 0; e < 32; ++e) {
+          if (__uint_as_float(v[e]) <= thrD) m0 |= 1u << e;
+          if (__uint_as_float(v[32 + e]) <= thrD) m1 |= 1u << e;
+        }
+      }
+#pragma unroll
+      for (int w = 0; w < 2; ++w) {
+        uint32_t m = w ? m1 : m0;
+        while (m) {
+          const int k = 64 * q + 32 * w + __ffs(m) - 1;
+          m &= m - 1u;
+          if (k >= cw.K) break;  // padding columns (only with an unbounded threshold)
+          const float4 c0 = *reinterpret_cast<const float4*>(sC + k * kD);
+          const float4 c1 = *reinterpret_cast<const float4*>(sC + k * kD + 4);
+          const float2 nl = sNL[k];
+          float sv = base + nl.x;
+          sv = fmaf(m2q[0], c0.x, sv);
+          sv = fmaf(m2q[1], c0.y, sv);
+          sv = fmaf(m2q[2], c0.z, sv);
+          sv = fmaf(m2q[3], c0.w, sv);
+          sv = fmaf(m2q[4], c1.x, sv);
+          sv = fmaf(m2q[5], c1.y, sv);
+          sv = fmaf(m2q[6], c1.z, sv);
+          sv = fmaf(m2q[7], c1.w, sv);
+          sv = fmaf(nbeta, nl.y, sv);
+          if (sv < last) {  // insert before the first entry strictly above sv
+            int j = L - 1;
+            while (j > 0) {
+              const float pv = sTopV[(j - 1) * kThreads + tid];
+              if (!(sv < pv)) break;
+              sTopV[j * kThreads + tid] = pv;
+              sTopI[j * kThreads + tid] = sTopI[(j - 1) * kThreads + tid];
+              --j;
             }
+            sTopV[j * kThreads + tid] = sv;
+            sTopI[j * kThreads + tid] = (h << 16) | k;
+            last = sTopV[(L - 1) * kThreads + tid];
           }
         }
       }
-      nc = 0;
-      if (act) thrD = __fadd_ru(fminf(topv[L - 1], tau_x), eps);
-    };
-    for (int q = 0; q < ncol / 32; ++q) {
-      if (__any_sync(0xffffffffu, nc > kTcCand - 32)) flush();
-      uint32_t v[32];
       __syncwarp();
-      tc::tmem_ld32_nowait(trow + 32 * q, v);
-      tc::tmem_wait_ld_dep(v);
-#pragma unroll
-      for (int e = 0; e < 32; ++e) {
-        cand[nc * kThreads + tid] = (uint8_t)(32 * q + e);
-        nc += (__uint_as_float(v[e]) <= thrD) ? 1 : 0;
-      }
     }
-    flush();
     tc::tc_fence_before();
   }
   // let the codebook copy land before the CTA ends (bounded), then free the tensor memory
@@ -1726,6 +1732,13 @@ beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc 
   __syncthreads();
   if (warp == 0) tc::tmem_dealloc(tmem, 2 * kTcCols);
   if (!live) return;
+  float topv[L];
+  int topi[L];
+#pragma unroll
+  for (int j = 0; j < L; ++j) {
+    topv[j] = sTopV[j * kThreads + tid];
+    topi[j] = sTopI[j * kThreads + tid];
+  }
   beam_list_finish<L>(set, cbs, sd, bb, flags, i, g, vi, Bh, cmul, th, tl, sH, sNL, sNa, true,
                       sRa + tid, sPm + tid, kThreads, topv, topi, err);
 }
