@@ -1578,43 +1578,50 @@ beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc 
   float tau_x = INFINITY;
   bool ok = true;
   const uint32_t trow = tmem + ((uint32_t)(warp * 32) << 16);
+  // Terms of hypothesis h (zero for a thread without it) and its A row. The terms of h + 1
+  // are computed while the tensor cores run the pass of h, its row written once that pass
+  // has completed.
+  auto hyp_terms = [&](int h, float m2q[kD], float& base, float& nbeta, float& eps) {
+#pragma unroll
+    for (int p = 0; p < kD; ++p) m2q[p] = 0.f;
+    base = nbeta = eps = 0.f;
+    if (live && h < Bh) {
+      float rh[kD], rl[kD], rr, ra, pmax;
+      const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
+      hyp_residual_pair(th, tl, cbs, sd, pc, rh, rl, err);
+      hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
+      sRa[h * kThreads + tid] = ra;
+      sPm[h * kThreads + tid] = pmax;
+      base = rr - kU * cmul * ra;
+      nbeta = -2.f * kU * cmul * pmax;
+      eps = 2.44140625e-04f *  // 2^-12
+            (fabsf(base) + na_max + 2.f * pmax * l1max * 1.0001f + fabsf(nbeta) * l1max);
+    }
+  };
+  auto write_a = [&](const float m2q[kD], float base, float nbeta) {
+    uint32_t row[kK];
+#pragma unroll
+    for (int p = 0; p < kD; ++p) {
+      uint32_t hh, ll;
+      split(m2q[p], hh, ll);
+      row[p] = hh;
+      row[8 + p] = hh;
+      row[16 + p] = ll;
+    }
+    const uint32_t one = __float_as_uint(1.f);
+    row[24] = one;
+    row[25] = one;
+    split(nbeta, row[26], row[28]);
+    row[27] = row[26];
+    split(base, row[29], row[30]);
+    row[31] = 0u;
+    put_row(Atile, tid, row);
+  };
+  float m2q[kD], base, nbeta, eps;
+  hyp_terms(0, m2q, base, nbeta, eps);
+  write_a(m2q, base, nbeta);
   for (int h = 0; h < Bmax && ok; ++h) {
     const bool act = live && h < Bh;
-    float m2q[kD], base = 0.f, nbeta = 0.f, eps = 0.f;
-    {
-      float rr = 0.f, ra = 0.f, pmax = 0.f;
-#pragma unroll
-      for (int p = 0; p < kD; ++p) m2q[p] = 0.f;
-      if (act) {
-        float rh[kD], rl[kD];
-        const int32_t* pc = bb.hyp_in ? bb.hyp_in + (vi * B + h) * S : nullptr;
-        hyp_residual_pair(th, tl, cbs, sd, pc, rh, rl, err);
-        hyp_terms_pair(rh, rl, sH, m2q, rr, ra, pmax);
-        sRa[h * kThreads + tid] = ra;
-        sPm[h * kThreads + tid] = pmax;
-        base = rr - kU * cmul * ra;
-        nbeta = -2.f * kU * cmul * pmax;
-        eps = 2.44140625e-04f *  // 2^-12
-              (fabsf(base) + na_max + 2.f * pmax * l1max * 1.0001f + fabsf(nbeta) * l1max);
-      }
-      uint32_t row[kK];
-#pragma unroll
-      for (int p = 0; p < kD; ++p) {
-        uint32_t hh, ll;
-        split(m2q[p], hh, ll);
-        row[p] = hh;
-        row[8 + p] = hh;
-        row[16 + p] = ll;
-      }
-      const uint32_t one = __float_as_uint(1.f);
-      row[24] = one;
-      row[25] = one;
-      split(nbeta, row[26], row[28]);
-      row[27] = row[26];
-      split(base, row[29], row[30]);
-      row[31] = 0u;
-      put_row(Atile, tid, row);
-    }
     tc::fence_async_smem();
     tc::tc_fence_before();
     __syncthreads();
@@ -1639,6 +1646,8 @@ beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc 
       }
       if (!bok) raise_error(err, ERRBIT_TIMEOUT);
     }
+    float nm2q[kD], nbase, nnbeta, neps;
+    if (h + 1 < Bmax) hyp_terms(h + 1, nm2q, nbase, nnbeta, neps);
     bool wok = tc::mbar_wait(tc::smem_u32(&bar_mma), (uint32_t)(h & 1), err);
     if (h == 0 && tid == 0) wok = wok && tc::mbar_try_wait(tc::smem_u32(&bar_b), 0u);
     ok = __syncthreads_and(wok);
@@ -1726,6 +1735,14 @@ beam_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, StageDesc 
       __syncwarp();
     }
     tc::tc_fence_before();
+    if (h + 1 < Bmax) {  // the pass of h has completed: its A tile is free
+      write_a(nm2q, nbase, nnbeta);
+#pragma unroll
+      for (int p = 0; p < kD; ++p) m2q[p] = nm2q[p];
+      base = nbase;
+      nbeta = nnbeta;
+      eps = neps;
+    }
   }
   // let the codebook copy land before the CTA ends (bounded), then free the tensor memory
   if (!ok && tid == 0) tc::mbar_wait(tc::smem_u32(&bar_b), 0u, err);
