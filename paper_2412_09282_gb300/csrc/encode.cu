@@ -501,10 +501,11 @@ __device__ __forceinline__ uint32_t min16_bits(const uint32_t* x) {
 constexpr int kBlk = 16;  // columns per block of the arg-min sweep
 
 // dynamic shared memory of argmin_tc_kernel<HALVES>: A tiles, two B chunks, statistics, H r,
-// alignment
+// with two halves the codeword terms (Na, L1) of the group, alignment
 constexpr size_t argmin_smem(int halves) {
   return (size_t)halves * tcenc::kATile + 2 * (size_t)kTcBTile +
-         (size_t)kTcSmemStatsK * (kD * 8 + 4) + (size_t)halves * tcenc::kRows * kD * 4 + 1024;
+         (size_t)kTcSmemStatsK * (kD * 8 + 4) + (size_t)halves * tcenc::kRows * kD * 4 +
+         (halves == 2 ? (size_t)kTcSmemStatsK * 8 : 0) + 1024;
 }
 
 // Barrier over this half's 128 threads (named barrier 1 + half), or the whole CTA.
@@ -548,6 +549,7 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
   long long* s_bacc = reinterpret_cast<long long*>(Bbuf + 2 * kTcBTile);  // [8][256]
   int* s_cnt = reinterpret_cast<int*>(s_bacc + kTcSmemStatsK * kD);       // [256]
   float* sQ = reinterpret_cast<float*>(s_cnt + kTcSmemStatsK);            // [128 HALVES][8]
+  float2* sNaL1 = reinterpret_cast<float2*>(sQ + HALVES * kRows * kD);     // [256] (2 halves)
   __shared__ __align__(16) float sH[kD * kD];
   __shared__ __align__(8) uint64_t bar_mma_s[HALVES], bar_b[2];
   __shared__ uint32_t tmem_slot;
@@ -569,9 +571,20 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
 
   if (tid < kD * kD) sH[tid] = set.Hb[g * kD * kD + tid];
   if (smem_stats) {
-    for (int e = tid; e < kTcSmemStatsK * kD; e += blockDim.x) s_bacc[e] = 0;
+    for (int e = tid; e < kTcSmemStatsK * kD; e += blockDim.x) s_bacc[e] = 0;  // (= s_b32)
     for (int e = tid; e < kTcSmemStatsK; e += blockDim.x) s_cnt[e] = 0;
   }
+  // Statistics terms (|v| < 2^30) split as v = 2^15 vh + vl, 0 <= vl < 2^15, into two 32-bit
+  // shared sums [component][vh, vl][code] (native 32-bit atomics instead of 64-bit ones): exact,
+  // since the host gives a CTA with these sums fewer than 2^16 rows (|sum| < 2^31).
+  int* s_b32 = reinterpret_cast<int*>(s_bacc);  // [8][2][256] in the 64-bit sums' space
+  // the winner's terms for the certificate, from shared memory (K <= 256 with two halves)
+  const bool smem_terms = HALVES == 2 && gterms != nullptr;
+  if (smem_terms)
+    for (int k = tid; k < cw.K; k += blockDim.x) {
+      const float4 tk = gterms[k];
+      sNaL1[k] = make_float2(tk.y, tk.z);
+    }
   if (warp == 0) tc::tmem_alloc(&tmem_slot, HALVES * kTcCols);
   if (tid == 0) {
     for (int h = 0; h < HALVES; ++h) tc::mbar_init(tc::smem_u32(&bar_mma_s[h]), 1);
@@ -776,7 +789,11 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       float thr = INFINITY;
       if (j < cw.K) {
         float n, na, l1;
-        if (gterms) {
+        if (smem_terms) {
+          const float2 tj = sNaL1[j];
+          na = tj.x;
+          l1 = tj.y;
+        } else if (gterms) {
           const float4 tj = gterms[j];
           n = tj.x;
           na = tj.y;
@@ -816,9 +833,11 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
         if (smem_stats) {
           atomicAdd(&s_cnt[j], 1);
 #pragma unroll
-          for (int p = 0; p < kD; ++p)
-            atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[p * kTcSmemStatsK + j]),
-                      (unsigned long long)fix_rn_small(q[p], sscale));
+          for (int p = 0; p < kD; ++p) {
+            const long long v = fix_rn_small(q[p], sscale);
+            atomicAdd(&s_b32[(2 * p) * kTcSmemStatsK + j], (int)(v >> 15));
+            atomicAdd(&s_b32[(2 * p + 1) * kTcSmemStatsK + j], (int)(v & 0x7fff));
+          }
         } else {
           stats_add(st, sscale, g, j, q);
         }
@@ -837,9 +856,12 @@ argmin_tc_kernel(SetView set, int64_t g_begin, CbList cbs, int n_fixed, int s_id
       if (c == 0) continue;
       atomicAdd(&st.cnt[g * st.K + k], c);
 #pragma unroll
-      for (int p = 0; p < kD; ++p)
+      for (int p = 0; p < kD; ++p) {
+        const long long v = (long long)s_b32[(2 * p) * kTcSmemStatsK + k] * 32768 +
+                            s_b32[(2 * p + 1) * kTcSmemStatsK + k];
         atomicAdd(reinterpret_cast<unsigned long long*>(&st.bacc[(int64_t)k * kD + p]),
-                  (unsigned long long)s_bacc[p * kTcSmemStatsK + k]);
+                  (unsigned long long)v);
+      }
     }
   }
   tc::tc_fence_before();
@@ -2235,6 +2257,8 @@ crvq_status encode_range(const SetView& set, int64_t g_begin, int64_t G_range,
         const int64_t per_group = std::max<int64_t>(1, want_ctas / std::max<int64_t>(1, gn));
         int tiles = (int)std::max<int64_t>(1, ceil_div(row_tiles, per_group));
         if (two_halves) tiles += tiles & 1;
+        // fused statistics in 32-bit shared sums: fewer than 2^16 rows per CTA
+        if (st.cnt && cw.K <= kTcSmemStatsK) tiles = std::min(tiles, 510);
         const dim3 grid((unsigned)ceil_div(row_tiles, tiles), (unsigned)gn);
         ProfScope ps(st.cnt ? "encode_argmin_lloyd" : "encode_argmin", stream,
                      (double)nv * cw.K);
