@@ -91,15 +91,18 @@ __global__ void stats_scale_kernel(const unsigned* __restrict__ maxbits, int n_c
 }
 
 // Statistics of every covered vector from its current code. CTA (x, y): groups y,
-// y + gridDim.y, ..., rows x, x + gridDim.x, ... of each; with K <= kSmemStatsK the CTA sums its counts and fixed-point terms
-// in shared memory (integer atomics) and adds them to the global sums once; larger codebooks
-// add each vector's terms to the global sums directly. Integer sums: the order is immaterial.
+// y + gridDim.y, ..., rows x, x + gridDim.x, ... of each; with K <= kSmemStatsK the CTA sums
+// its counts and fixed-point terms in shared memory and adds them to the global sums once;
+// larger codebooks add each vector's terms to the global sums directly. A term (|v| < 2^30)
+// enters shared memory as v = 2^15 vh + vl (0 <= vl < 2^15) in two 32-bit sums (native 32-bit
+// atomics): exact, as accumulate_grid gives a CTA fewer than 2^16 rows of a group. Integer
+// sums: the order is immaterial.
 constexpr int kSmemStatsK = 256;
 
 __global__ void __launch_bounds__(256)
 accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsigned* err) {
-  __shared__ long long s_bacc[kD * kSmemStatsK];  // [component][code]: lanes of a warp
-                                                  // adding one component hit spread banks
+  // [component][vh, vl][code]: lanes of a warp adding one component hit spread banks
+  __shared__ int s_b32[kD * 2 * kSmemStatsK];
   __shared__ int s_cnt[kSmemStatsK];
   const CbView cw = cbs.cb[which];
   const float sscale = stats_scale_f(st);
@@ -107,7 +110,7 @@ accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsign
   for (int64_t g = blockIdx.y; g < cw.G_cov; g += gridDim.y) {
     if (smem) {
       __syncthreads();  // the previous group's flush has read the sums
-      for (int e = threadIdx.x; e < kSmemStatsK * kD; e += blockDim.x) s_bacc[e] = 0;
+      for (int e = threadIdx.x; e < kSmemStatsK * kD * 2; e += blockDim.x) s_b32[e] = 0;
       for (int e = threadIdx.x; e < kSmemStatsK; e += blockDim.x) s_cnt[e] = 0;
       __syncthreads();
     }
@@ -124,9 +127,11 @@ accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsign
       if (smem) {
         atomicAdd(&s_cnt[k], 1);
 #pragma unroll
-        for (int j = 0; j < kD; ++j)
-          atomicAdd(reinterpret_cast<unsigned long long*>(&s_bacc[j * kSmemStatsK + k]),
-                    (unsigned long long)fix_rn_small(q[j], sscale));
+        for (int j = 0; j < kD; ++j) {
+          const long long v = fix_rn_small(q[j], sscale);
+          atomicAdd(&s_b32[(2 * j) * kSmemStatsK + k], (int)(v >> 15));
+          atomicAdd(&s_b32[(2 * j + 1) * kSmemStatsK + k], (int)(v & 0x7fff));
+        }
       } else {
         stats_add(st, sscale, g, k, q);
       }
@@ -138,19 +143,25 @@ accumulate_stats_kernel(SetView set, CbList cbs, int which, StatsView st, unsign
         if (c == 0) continue;
         atomicAdd(&st.cnt[g * st.K + k], c);
 #pragma unroll
-        for (int j = 0; j < kD; ++j)
+        for (int j = 0; j < kD; ++j) {
+          const long long v = (long long)s_b32[(2 * j) * kSmemStatsK + k] * 32768 +
+                              s_b32[(2 * j + 1) * kSmemStatsK + k];
           atomicAdd(reinterpret_cast<unsigned long long*>(&st.bacc[(int64_t)k * kD + j]),
-                    (unsigned long long)s_bacc[j * kSmemStatsK + k]);
+                    (unsigned long long)v);
+        }
       }
     }
   }
 }
 
 // Grid of accumulate_stats_kernel: one column of CTAs per group, enough rows per CTA that
-// the flush stays small, at least ~4 CTAs per SM overall.
+// the flush stays small, at least ~4 CTAs per SM overall, and fewer than 2^16 rows per CTA
+// (the 32-bit shared sums).
 dim3 accumulate_grid(int64_t M, int64_t G_cov, int nsm) {
-  const int64_t want = std::max<int64_t>(1, ceil_div(4 * (int64_t)nsm, std::max<int64_t>(G_cov, 1)));
-  const int64_t rows_x = std::max<int64_t>(1, std::min<int64_t>(want, ceil_div(M, 1024)));
+  const int64_t want =
+      std::max<int64_t>(1, ceil_div(4 * (int64_t)nsm, std::max<int64_t>(G_cov, 1)));
+  const int64_t rows_x = std::max<int64_t>(
+      ceil_div(M, 65000), std::max<int64_t>(1, std::min<int64_t>(want, ceil_div(M, 1024))));
   return dim3((unsigned)rows_x, (unsigned)std::min<int64_t>(std::max<int64_t>(G_cov, 1), 65535));
 }
 
