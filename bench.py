@@ -520,6 +520,8 @@ def main():
     ap.add_argument("--ref-warmup", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--streams", type=int, default=3,
+                    help="streams (and host threads) the matrices of a step run on")
     ap.add_argument("--no-infer", action="store_true",
                     help="skip the inference-product and coupled-sweep lines after the timed "
                          "steps")
@@ -558,18 +560,58 @@ def main():
                      "Xn": Xn, "out": None, "h_out": None})
     flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
+    # The matrices of a step are independent problems. With --streams S > 1 they run on S
+    # streams from S host threads (the library replays each matrix's graph on its own stream
+    # without holding its cache lock), balanced by size, largest first.
+    nstr = max(1, min(args.streams, len(work)))
+    lanes = [[] for _ in range(nstr)]
+    load = [0] * nstr
+    for j in sorted(range(len(work)), key=lambda j: -work[j]["cfg"].M * work[j]["cfg"].N):
+        q = load.index(min(load))
+        lanes[q].append(j)
+        load[q] += work[j]["cfg"].M * work[j]["cfg"].N
+    streams = [stream] if nstr == 1 else [torch.cuda.Stream(dev) for _ in range(nstr)]
+    pool = None
+    if nstr > 1:
+        from concurrent.futures import ThreadPoolExecutor
+        pool = ThreadPoolExecutor(nstr)
 
-    def run_step(host=False):
+    def run_lane(q, host, start):
+        s = streams[q]
+        sc = 0.0
+        with torch.cuda.device(dev):
+            if start is not None:
+                s.wait_event(start)
+            for j in lanes[q]:
+                w = work[j]
+                if host:
+                    w["h_out"] = P.crvq_quantize_layer(w["W_h"], w["X_h"], w["cfg"],
+                                                       out=w["h_out"], stream=s, device=dev)
+                    sc += w["h_out"].report["scores"]
+                else:
+                    w["out"] = P.crvq_quantize_layer(w["W_d"], w["X_d"], w["cfg"],
+                                                     out=w["out"], stream=s)
+                    sc += w["out"].report["scores"]
+        return sc
+
+    def run_step(host=False, sequential=False):
         """One step: every matrix of the workload through crvq_quantize_layer. Returns the
         scores of the step."""
-        sc = 0.0
-        for w in work:
-            if host:
-                w["h_out"] = P.crvq_quantize_layer(w["W_h"], w["X_h"], w["cfg"], out=w["h_out"])
-                sc += w["h_out"].report["scores"]
-            else:
-                w["out"] = P.crvq_quantize_layer(w["W_d"], w["X_d"], w["cfg"], out=w["out"])
+        if sequential:  # the matrices one after another on the main stream
+            sc = 0.0
+            for w in work:
+                w["out"] = P.crvq_quantize_layer(w["W_d"], w["X_d"], w["cfg"], out=w["out"],
+                                                 stream=stream)
                 sc += w["out"].report["scores"]
+            return sc
+        if pool is None:
+            return run_lane(0, host, None)
+        start = torch.cuda.Event()
+        start.record(stream)
+        sc = sum(f.result() for f in [pool.submit(run_lane, q, host, start)
+                                      for q in range(nstr)])
+        for s in streams:  # every call has synchronized its stream; order the main one after
+            stream.wait_stream(s)
         return sc
 
     for _ in range(args.warmup):
@@ -615,10 +657,22 @@ def main():
                     if k["name"] in ("encode_argmin", "encode_argmin_lloyd")]
     launches = P.crvq_launch_count() - launches0
     clk = clocks.stop()
-    # per-kernel breakdown: one more step, untimed, every launch bracketed
+    # With several streams the arg-min launches of the timed steps share the GPU with the other
+    # streams' kernels. One more step, untimed, runs the matrices one after another for the
+    # kernel's own launch time beside the live one.
+    iso_stats = None
+    if nstr > 1:
+        P.crvq_profile_filter("encode_argmin")
+        P.crvq_profile_begin()
+        run_step(sequential=True)
+        torch.cuda.synchronize()
+        iso_stats = [k for k in P.crvq_profile_end()
+                     if k["name"] in ("encode_argmin", "encode_argmin_lloyd")]
+    # per-kernel breakdown: one more step, untimed, the matrices one after another, every
+    # launch bracketed
     P.crvq_profile_filter(None)
     P.crvq_profile_begin()
-    run_step()
+    run_step(sequential=True)
     torch.cuda.synchronize()
     kstats = P.crvq_profile_end()
     tot_ms_max, scores_all = rank_aggregate(sum(step_ms), scores, ws, dev)
@@ -693,12 +747,27 @@ def main():
                     "work": (f"{ALU_OPS_PER_SCORE} integer ALU ops per scored pair (the "
                              "kernel's ALU pipe instructions, measured by ncu)"),
                     "peak_source": f"{nsm} SMs x 64 ALU lanes x {mhz:.0f} MHz"}}
+    if iso_stats:
+        roof["streams"] = nstr
+        roof["note"] = (f"live: the timed steps, the matrices on {nstr} streams, so arg-min "
+                        "launches share the GPU with other streams' kernels; isolated: one "
+                        "untimed step with the matrices one after another")
+        i_ms = sum(k["ms"] for k in iso_stats)
+        i_units = sum(k["units"] for k in iso_stats)
+        i_launches = sum(k["launches"] for k in iso_stats)
+        i_sec = i_ms / 1e3 if i_ms > 0 else float("inf")
+        i_alg = i_units * 16.0 / i_sec / 1e12
+        roof["isolated"] = {
+            "achieved": i_alg, "frac": i_alg / tf32_peak,
+            "avg_launch_ms": i_ms / max(i_launches, 1), "launches": i_launches,
+            "issued_frac": i_units * 64.0 / i_sec / 1e12 / tf32_peak,
+            "alu_frac": i_units * ALU_OPS_PER_SCORE / i_sec / 1e12 / alu_peak}
     last = work[-1]["out"].report if len(work) == 1 else None
     line = {
         "metric": METRIC, "value": value, "unit": "scores/s", "n_gpus": ws,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": tot_ms_max / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-        "data": DATA, "config": workload_dict(args.config, layers),
+        "data": DATA, "config": dict(workload_dict(args.config, layers), streams=nstr),
         "layer_time_s": tot_ms_max / args.steps / 1e3 / len(work),
         "roofline": roof,
         "e2e": e2e,

@@ -887,7 +887,9 @@ void fill_report(crvq_layer_report* report, const double hl[12], unsigned long l
 // runs without host synchronisation between its ~240 launches; it is captured once into a
 // CUDA graph per (device, stream, shapes, configuration, pointers, profiling state) and
 // replayed, which removes the host launch gaps. Up to kGraphs graphs are kept (least recently
-// used evicted). CRVQ_GRAPHS=0 in the environment turns this off.
+// used evicted, never one being replayed). Calls on different streams from different host
+// threads run concurrently: the cache lock covers the lookup (and a capture), not the replay.
+// CRVQ_GRAPHS=0 in the environment turns this off.
 struct LayerGraph {
   int dev = -1;
   cudaStream_t stream = nullptr;
@@ -906,8 +908,11 @@ struct LayerGraph {
   int64_t launches = 0;                     // kernels in the graph
   CapturedEvents events;                    // arg-min event nodes when captured while profiling
   uint64_t used = 0;
+  int users = 0;                            // replays in flight (never evicted meanwhile)
 };
-constexpr int kGraphs = 16;  // a 7-matrix decoder block in both profiling states
+// A 7-matrix decoder block in both profiling states on its streams, plus the host-buffer and
+// single-stream variants of the same matrices.
+constexpr int kGraphs = 48;
 std::mutex g_graph_mu;
 std::vector<LayerGraph*> g_graphs;
 uint64_t g_graph_clock = 0;
@@ -952,7 +957,7 @@ crvq_status run_graph(const float* W, const float* X, int64_t M, int64_t N, int6
   int dev = 0;
   CRVQ_CUDA(cudaGetDevice(&dev));
   const bool prof = g_prof.load();
-  std::lock_guard<std::mutex> lk(g_graph_mu);
+  std::unique_lock<std::mutex> lk(g_graph_mu);
   LayerGraph* e = nullptr;
   for (auto* c : g_graphs)
     if (same_key(*c, dev, s, M, N, n_tok, cfg, W, X, o, prof)) e = c;
@@ -1003,15 +1008,27 @@ crvq_status run_graph(const float* W, const float* X, int64_t M, int64_t N, int6
       return CRVQ_OK;
     }
     if ((int)g_graphs.size() >= kGraphs) {
-      size_t lru = 0;
-      for (size_t q = 1; q < g_graphs.size(); ++q)
-        if (g_graphs[q]->used < g_graphs[lru]->used) lru = q;
-      destroy_graph(g_graphs[lru]);
-      g_graphs.erase(g_graphs.begin() + lru);
+      int lru = -1;
+      for (int q = 0; q < (int)g_graphs.size(); ++q)
+        if (g_graphs[q]->users == 0 && (lru < 0 || g_graphs[q]->used < g_graphs[lru]->used))
+          lru = q;
+      if (lru >= 0) {
+        destroy_graph(g_graphs[lru]);
+        g_graphs.erase(g_graphs.begin() + lru);
+      }
     }
     g_graphs.push_back(e);
   }
   e->used = ++g_graph_clock;
+  ++e->users;
+  lk.unlock();
+  struct Unpin {  // the entry may be evicted again once this replay is done
+    LayerGraph* e;
+    ~Unpin() {
+      std::lock_guard<std::mutex> l(g_graph_mu);
+      --e->users;
+    }
+  } unpin{e};
   CRVQ_CUDA(cudaGraphLaunch(e->exec, s));
   g_launches.fetch_add(e->launches);
   double hl[12];
@@ -1040,7 +1057,8 @@ crvq_status run_graph(const float* W, const float* X, int64_t M, int64_t N, int6
 // Persistent device staging for layers called with host inputs or outputs: the host data is
 // copied into buffers that outlive the call, so that the graph captured on them (keyed by
 // pointers) is replayed by later calls of the same shapes, as for device buffers. Up to
-// kStagings sets are kept (least recently used freed; never one a call is using).
+// kStagings sets are kept (least recently used freed; never one a call is using): calls of one
+// shape running concurrently on several streams each take their own set.
 struct Staging {
   int dev = -1;
   int64_t M = 0, N = 0, n_tok = 0, K_base = 0, n_ext = 0, K_ext = 0, Gc = 0;
@@ -1050,7 +1068,7 @@ struct Staging {
   uint64_t used = 0;
   int users = 0;
 };
-constexpr int kStagings = 4;
+constexpr int kStagings = 8;
 std::mutex g_stage_mu;
 std::vector<Staging*> g_stagings;
 uint64_t g_stage_clock = 0;
