@@ -30,7 +30,7 @@ __device__ __forceinline__ void pair_merge(float& h, float& l, float oh, float o
 }
 
 constexpr int kDecRows = 16;     // rows per warp (the CTA's H blocks are staged once for all)
-constexpr int kDecBatch = 4;     // rows whose codes and vectors are loaded together
+constexpr int kDecBatch = 2;     // rows whose codes and vectors are loaded together
 constexpr int kDecWarps = 8;     // warps per CTA
 constexpr int kDecHStride = 260; // floats per staged H block (256 + 4: conflict-free float4)
 constexpr int kDecSmemCb = 48 * 1024;  // codebooks staged in shared memory up to this size
@@ -73,13 +73,14 @@ __device__ __forceinline__ void recon_codes(const float* const* cw, const int32_
 }
 
 // One warp = kDecRows rows x one slice of 32 groups, lane = group: the reconstruction in the
-// sorted order (32-byte stores, consecutive lanes on consecutive vectors), each vector's error
-// under H_g (the quadratic form as two FMA chains in fp32) and, per (row, slice), the block
-// loss, the critical loss and ||dW||^2 as fp32 pairs in a fixed order:
-// row_part[(row * slices + slice) * 3 + {0, 1, 2}] = (hi, lo). A CTA's warps share one slice:
-// its H blocks are staged in shared memory once for the CTA's kDecWarps x kDecRows rows; the
-// codebooks sit in shared memory when they fit, so the codeword lookup is not a dependent
-// global load; the codes of kDecBatch rows are loaded before any is used.
+// sorted order (32-byte stores, consecutive lanes on consecutive vectors) and, per (row block,
+// slice), the block loss, the critical loss and ||dW||^2 as fp32 pairs in a fixed order:
+// row_part[(row_block * slices + slice) * 3 + {0, 1, 2}] = (hi, lo). A lane sums its group's
+// S = sum over its rows of dl dl^T (dl = w - w_hat; the 36 entries of the symmetric 8 x 8), then
+// takes the loss as tr(H_g S) = sum_v dl_v^T H_g dl_v once, and ||dW||^2 as tr(S). A CTA's warps
+// share one slice: its H blocks are staged in shared memory once; the codebooks sit in shared
+// memory when they fit, so the codeword lookup is not a dependent global load; the codes of
+// kDecBatch rows are loaded before any is used.
 template <int MAXCB>
 __global__ void __launch_bounds__(kDecWarps * 32)
 decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
@@ -126,7 +127,9 @@ decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
   const int64_t i0 = rb * kDecRows;
   if (i0 >= M) return;  // whole warps (no block barrier follows)
   const int nr = (int)min((int64_t)kDecRows, M - i0);
-  const float4* H4 = reinterpret_cast<const float4*>(sH + lane * kDecHStride);
+  float S[kD * (kD + 1) / 2];  // sum of dl dl^T over this warp's rows, packed lower triangle
+#pragma unroll
+  for (int e = 0; e < kD * (kD + 1) / 2; ++e) S[e] = 0.f;
   for (int r0 = 0; r0 < nr; r0 += kDecBatch) {
     int32_t kc[kDecBatch][MAXCB];
     float4 tv[kDecBatch][2];
@@ -147,68 +150,73 @@ decode_vec_kernel(const float* __restrict__ Ws, int64_t M, int64_t N,
     }
 #pragma unroll
     for (int u = 0; u < kDecBatch; ++u) {
-      if (r0 + u >= nr) break;
+      if (r0 + u >= nr || !gok) break;
       const int64_t i = i0 + r0 + u;
-      float lb = 0.f, lc = 0.f, sq = 0.f;
-      if (gok) {
 #pragma unroll
-        for (int s = 0; s < MAXCB; ++s) {
-          if (s >= cbs.n || g >= cbs.cb[s].G_cov) continue;
-          if (kc[u][s] < 0 || kc[u][s] >= cbs.cb[s].K) {
-            raise_error(err, ERRBIT_INDEX);
-            kc[u][s] = -1;
-          }
-        }
-        float rv[kD], dl[kD];
-        recon_codes<MAXCB>(cw, kc[u], cbs.n, rv);
-        const float t[kD] = {tv[u][0].x, tv[u][0].y, tv[u][0].z, tv[u][0].w,
-                             tv[u][1].x, tv[u][1].y, tv[u][1].z, tv[u][1].w};
-#pragma unroll
-        for (int j = 0; j < kD; ++j) {
-          dl[j] = t[j] - rv[j];
-          sq = fmaf(dl[j], dl[j], sq);
-        }
-#pragma unroll
-        for (int a = 0; a < kD; ++a) {
-          const float4 h0 = H4[2 * a], h1 = H4[2 * a + 1];
-          float hb = dl[0] * h0.x;
-          hb = fmaf(dl[1], h0.y, hb);
-          hb = fmaf(dl[2], h0.z, hb);
-          hb = fmaf(dl[3], h0.w, hb);
-          hb = fmaf(dl[4], h1.x, hb);
-          hb = fmaf(dl[5], h1.y, hb);
-          hb = fmaf(dl[6], h1.z, hb);
-          hb = fmaf(dl[7], h1.w, hb);
-          lb = fmaf(hb, dl[a], lb);
-        }
-        if (g < n_crit_groups) lc = lb;
-        if (W_rec) {
-          float* o = W_rec + i * N + g * kD;
-          *reinterpret_cast<float4*>(o) = make_float4(rv[0], rv[1], rv[2], rv[3]);
-          *reinterpret_cast<float4*>(o + 4) = make_float4(rv[4], rv[5], rv[6], rv[7]);
+      for (int s = 0; s < MAXCB; ++s) {
+        if (s >= cbs.n || g >= cbs.cb[s].G_cov) continue;
+        if (kc[u][s] < 0 || kc[u][s] >= cbs.cb[s].K) {
+          raise_error(err, ERRBIT_INDEX);
+          kc[u][s] = -1;
         }
       }
-      // the 32 vectors of this (row, slice) summed as fp32 pairs in a fixed tree
-      float lbl = 0.f, lcl = 0.f, sql = 0.f;
+      float rv[kD], dl[kD];
+      recon_codes<MAXCB>(cw, kc[u], cbs.n, rv);
+      const float t[kD] = {tv[u][0].x, tv[u][0].y, tv[u][0].z, tv[u][0].w,
+                           tv[u][1].x, tv[u][1].y, tv[u][1].z, tv[u][1].w};
 #pragma unroll
-      for (int off = 16; off > 0; off >>= 1) {
-        const float a0 = __shfl_xor_sync(0xffffffffu, lb, off);
-        const float a1 = __shfl_xor_sync(0xffffffffu, lbl, off);
-        const float b0 = __shfl_xor_sync(0xffffffffu, lc, off);
-        const float b1 = __shfl_xor_sync(0xffffffffu, lcl, off);
-        const float c0 = __shfl_xor_sync(0xffffffffu, sq, off);
-        const float c1 = __shfl_xor_sync(0xffffffffu, sql, off);
-        pair_merge(lb, lbl, a0, a1);
-        pair_merge(lc, lcl, b0, b1);
-        pair_merge(sq, sql, c0, c1);
-      }
-      if (lane == 0) {
-        float2* o = row_part + (i * slices + sl) * 3;
-        o[0] = make_float2(lb, lbl);
-        o[1] = make_float2(lc, lcl);
-        o[2] = make_float2(sq, sql);
+      for (int j = 0; j < kD; ++j) dl[j] = t[j] - rv[j];
+      int e = 0;
+#pragma unroll
+      for (int a2 = 0; a2 < kD; ++a2)
+#pragma unroll
+        for (int b2 = 0; b2 <= a2; ++b2, ++e) S[e] = fmaf(dl[a2], dl[b2], S[e]);
+      if (W_rec) {
+        float* o = W_rec + i * N + g * kD;
+        *reinterpret_cast<float4*>(o) = make_float4(rv[0], rv[1], rv[2], rv[3]);
+        *reinterpret_cast<float4*>(o + 4) = make_float4(rv[4], rv[5], rv[6], rv[7]);
       }
     }
+  }
+  // lb = tr(H_g S) (H_g symmetric: diagonal once, each off-diagonal pair twice), sq = tr(S)
+  float lb = 0.f, lc = 0.f, sq = 0.f;
+  if (gok) {
+    const float* Hl = sH + lane * kDecHStride;
+    float off = 0.f;
+    int e = 0;
+#pragma unroll
+    for (int a2 = 0; a2 < kD; ++a2)
+#pragma unroll
+      for (int b2 = 0; b2 <= a2; ++b2, ++e) {
+        if (a2 == b2) {
+          lb = fmaf(Hl[a2 * kD + b2], S[e], lb);
+          sq += S[e];
+        } else {
+          off = fmaf(Hl[a2 * kD + b2], S[e], off);
+        }
+      }
+    lb = fmaf(2.f, off, lb);
+    if (g < n_crit_groups) lc = lb;
+  }
+  // the 32 groups of this (row block, slice) summed as fp32 pairs in a fixed tree
+  float lbl = 0.f, lcl = 0.f, sql = 0.f;
+#pragma unroll
+  for (int o2 = 16; o2 > 0; o2 >>= 1) {
+    const float a0 = __shfl_xor_sync(0xffffffffu, lb, o2);
+    const float a1 = __shfl_xor_sync(0xffffffffu, lbl, o2);
+    const float b0 = __shfl_xor_sync(0xffffffffu, lc, o2);
+    const float b1 = __shfl_xor_sync(0xffffffffu, lcl, o2);
+    const float c0 = __shfl_xor_sync(0xffffffffu, sq, o2);
+    const float c1 = __shfl_xor_sync(0xffffffffu, sql, o2);
+    pair_merge(lb, lbl, a0, a1);
+    pair_merge(lc, lcl, b0, b1);
+    pair_merge(sq, sql, c0, c1);
+  }
+  if (lane == 0) {
+    float2* o = row_part + (rb * slices + sl) * 3;
+    o[0] = make_float2(lb, lbl);
+    o[1] = make_float2(lc, lcl);
+    o[2] = make_float2(sq, sql);
   }
 }
 
@@ -226,7 +234,7 @@ __global__ void invert_perm_kernel(const int32_t* __restrict__ perm, int64_t N,
   }
 }
 
-// One CTA of 1024 threads: the (row, slice) partials summed as fp32 pairs (strided, then a
+// One CTA of 1024 threads: the (row block, slice) partials summed as fp32 pairs (strided, then a
 // tree; no dependent fp64 chain), the loss-product partials in fp64 (a few per thread).
 __global__ void __launch_bounds__(1024)
 finalize_losses_kernel(const float2* __restrict__ row_part, int64_t n_rows,
@@ -300,7 +308,7 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   const bool rec_is_out = W_hat && !perm;
   const size_t rec_bytes = (need_rec && !rec_is_out) ? align_up((size_t)M * N * 4, 256) : 0;
   const size_t inv_bytes = (W_hat && perm) ? align_up((size_t)N * 4, 256) : 0;
-  const size_t part_bytes = align_up((size_t)M * slices * 3 * sizeof(float2), 256) +
+  const size_t part_bytes = align_up((size_t)row_blocks * slices * 3 * sizeof(float2), 256) +
                             (size_t)(n_gemm_cap + 1) * sizeof(double);
   Scratch mem;
   CRVQ_TRY(mem.alloc(rec_bytes + inv_bytes + part_bytes, stream));
@@ -308,7 +316,8 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
   int32_t* inv = inv_bytes ? reinterpret_cast<int32_t*>(mem.as<char>() + rec_bytes) : nullptr;
   float2* row_part = reinterpret_cast<float2*>(mem.as<char>() + rec_bytes + inv_bytes);
   double* gemm_part = reinterpret_cast<double*>(
-      reinterpret_cast<char*>(row_part) + align_up((size_t)M * slices * 3 * sizeof(float2), 256));
+      reinterpret_cast<char*>(row_part) +
+      align_up((size_t)row_blocks * slices * 3 * sizeof(float2), 256));
   {
     ProfScope ps("decode_rows", stream,
                  (double)M * N * 4.0 * (1.0 + (W_rec ? 1.0 : 0.0)));
@@ -343,7 +352,8 @@ crvq_status launch_reconstruct_error(const float* W_sorted, int64_t M, int64_t N
     CRVQ_TRY(launch_tc_sumsq(W_sorted, W_rec, M, X, perm, n_tok, N, gemm_part, n_gemm_cap,
                              &n_gemm, stream));
   }
-  finalize_losses_kernel<<<1, 1024, 0, stream>>>(row_part, M * slices, X ? gemm_part : nullptr,
+  finalize_losses_kernel<<<1, 1024, 0, stream>>>(row_part, row_blocks * slices,
+                                                 X ? gemm_part : nullptr,
                                                  n_gemm, n_tok, damp_delta, delta_dev,
                                                  losses_dev);
   CRVQ_LAUNCHED();
