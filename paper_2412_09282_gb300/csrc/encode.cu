@@ -15,6 +15,7 @@
 // Codes therefore equal the fp64 arg-min (ties to the smaller index) except for ties at fp64
 // rounding level. Beam stages use the same bounds on a sorted top-(B+1) list.
 #include <algorithm>
+#include <type_traits>
 #include <vector>
 
 #include "common.cuh"
@@ -2131,23 +2132,32 @@ crvq_status launch_beam_stage_tc(const SetView& set, int64_t g_begin, int64_t G_
                          bimg, tout, cbmax, fl.count));
     CRVQ_LAUNCHED();
   }
+  // the list length L = Bs + 1, rounded up to an instantiated size
+  auto go = [&](auto L) {
+    return launch_beam_tc_L<decltype(L)::value>(set, g_begin, G_range, cbs, n_fixed, sd, bb,
+                                                 bimg, cbmax, fl, err, units, stream);
+  };
   const int need = sd.Bs + 1;
-  if (need <= 2) return launch_beam_tc_L<2>(set, g_begin, G_range, cbs, n_fixed, sd, bb, bimg, cbmax, fl, err, units, stream);
-  if (need <= 3) return launch_beam_tc_L<3>(set, g_begin, G_range, cbs, n_fixed, sd, bb, bimg, cbmax, fl, err, units, stream);
-  if (need <= 5) return launch_beam_tc_L<5>(set, g_begin, G_range, cbs, n_fixed, sd, bb, bimg, cbmax, fl, err, units, stream);
-  return launch_beam_tc_L<9>(set, g_begin, G_range, cbs, n_fixed, sd, bb, bimg, cbmax, fl, err, units, stream);
+  if (need <= 2) return go(std::integral_constant<int, 2>{});
+  if (need <= 3) return go(std::integral_constant<int, 3>{});
+  if (need <= 5) return go(std::integral_constant<int, 5>{});
+  return go(std::integral_constant<int, 9>{});
 }
 
 crvq_status launch_beam_stage(const SetView& set, int64_t g_begin, int64_t G_range,
                               const CbList& cbs, int n_fixed, const StageDesc& sd,
                               const BeamBufs& bb, const FlagList& fl, unsigned* err,
                               double units, cudaStream_t stream) {
+  auto go = [&](auto L) {
+    return launch_beam_stage_L<decltype(L)::value>(set, g_begin, G_range, cbs, n_fixed, sd, bb,
+                                                   fl, err, units, stream);
+  };
   const int need = sd.Bs + 1;
-  if (need <= 2) return launch_beam_stage_L<2>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
-  if (need <= 3) return launch_beam_stage_L<3>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
-  if (need <= 5) return launch_beam_stage_L<5>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
-  if (need <= 9) return launch_beam_stage_L<9>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
-  return launch_beam_stage_L<17>(set, g_begin, G_range, cbs, n_fixed, sd, bb, fl, err, units, stream);
+  if (need <= 2) return go(std::integral_constant<int, 2>{});
+  if (need <= 3) return go(std::integral_constant<int, 3>{});
+  if (need <= 5) return go(std::integral_constant<int, 5>{});
+  if (need <= 9) return go(std::integral_constant<int, 9>{});
+  return go(std::integral_constant<int, 17>{});
 }
 
 // Scratch of one arg-min pass: codebook maxima (256 B) | B images of G_sub groups (groups
