@@ -82,24 +82,21 @@ __global__ void importance_kernel(const unsigned* __restrict__ maxbits,
   }
 }
 
+// perm[rank(i)] = i, rank(i) = #{j : I_j > I_i or (I_j == I_i and j < i)} (descending order,
+// ties to the smaller index). One warp per channel: the lanes count over j, a warp sum.
 __global__ void __launch_bounds__(256)
 rank_kernel(const float* __restrict__ I, int64_t N, int32_t* __restrict__ perm) {
-  __shared__ float tile[1024];
-  const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const float Ii = i < N ? I[i] : 0.f;
-  int64_t rank = 0;
-  for (int64_t j0 = 0; j0 < N; j0 += 1024) {
-    __syncthreads();
-    for (int t = threadIdx.x; t < 1024; t += blockDim.x)
-      tile[t] = (j0 + t < N) ? I[j0 + t] : -INFINITY;
-    __syncthreads();
-    const int lim = (int)min((int64_t)1024, N - j0);
-    for (int t = 0; t < lim; ++t) {
-      const float Ij = tile[t];
-      rank += (Ij > Ii) || (Ij == Ii && j0 + t < i);
-    }
+  const int lane = threadIdx.x & 31;
+  const int64_t i = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  if (i >= N) return;  // whole warps
+  const float Ii = I[i];
+  int rank = 0;
+  for (int64_t j = lane; j < N; j += 32) {
+    const float Ij = I[j];
+    rank += (Ij > Ii) || (Ij == Ii && j < i);
   }
-  if (i < N) perm[rank] = (int32_t)i;
+  rank = __reduce_add_sync(0xffffffffu, rank);
+  if (lane == 0) perm[rank] = (int32_t)i;
 }
 
 __global__ void __launch_bounds__(256)
@@ -168,7 +165,7 @@ crvq_status launch_select_reorder(const float* W, int64_t M, int64_t N, int d,
   CRVQ_LAUNCHED();
   {
     ProfScope ps("reorder_rank", stream, (double)N * N);
-    rank_kernel<<<(unsigned)ceil_div(N, 256), 256, 0, stream>>>(I, N, perm);
+    rank_kernel<<<(unsigned)ceil_div(N, 8), 256, 0, stream>>>(I, N, perm);
     CRVQ_LAUNCHED();
   }
   {
