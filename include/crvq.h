@@ -409,9 +409,15 @@ typedef struct crvq_layer_report {
  * When W, X and every output are device pointers and refine_rounds <= 1, the schedule has no
  * host synchronisation inside: it is captured into a CUDA graph on the first call for a given
  * (device, stream, shapes, configuration, pointers, profiling state) and replayed on later
- * calls, which reads the current contents of W and X (up to 16 graphs are kept per process,
- * least recently used evicted; their scratch stays reserved while they are kept). Setting
- * CRVQ_GRAPHS=0 in the environment runs every call directly. Results are identical either way.
+ * calls, which reads the current contents of W and X (up to 48 graphs are kept per process,
+ * least recently used evicted, never one being replayed; their scratch stays reserved while
+ * they are kept). Setting CRVQ_GRAPHS=0 in the environment runs every call directly. Results
+ * are identical either way.
+ * Calls for different matrices may run concurrently from different host threads, each on its
+ * own stream and with its own output buffers: a replay does not hold the library's graph lock,
+ * and a host-buffer call stages its data in buffers no running call holds (up to eight sets
+ * kept). Their results equal those of the same calls one after another. Concurrent calls that
+ * share output buffers, or share one stream, race.
  * What the kernels report on the device (a non-finite input, a refused index, a bounded wait
  * that ran out) is returned by the next crvq_sync on the device, not by this call.
  */
