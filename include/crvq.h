@@ -417,7 +417,7 @@ typedef struct crvq_layer_report {
  * own stream and with its own output buffers: a replay does not hold the library's graph lock,
  * and a host-buffer call stages its data in buffers no running call holds (up to eight sets
  * kept). Their results equal those of the same calls one after another. Concurrent calls that
- * share output buffers, or share one stream, race.
+ * share output buffers race; calls on one stream run one after another.
  * What the kernels report on the device (a non-finite input, a refused index, a bounded wait
  * that ran out) is returned by the next crvq_sync on the device, not by this call.
  */
