@@ -15,6 +15,7 @@
 // Codes therefore equal the fp64 arg-min (ties to the smaller index) except for ties at fp64
 // rounding level. Beam stages use the same bounds on a sorted top-(B+1) list.
 #include <algorithm>
+#include <cstdlib>
 #include <type_traits>
 #include <vector>
 
@@ -2106,7 +2107,11 @@ size_t beam_tc_scratch_bytes(int64_t G_range, int K) {
          align_up((size_t)G_range * K * sizeof(float4), 256) + 256;
 }
 
+// CRVQ_BEAM_TC=0 in the environment (read at every call) keeps every stage on the SIMT kernel:
+// the two forms give the same lists, which tests compare.
 bool beam_tc_applies(const StageDesc& sd, const CbList& cbs, int64_t G_range) {
+  const char* v = getenv("CRVQ_BEAM_TC");
+  if (v && v[0] == '0') return false;
   const int K = cbs.cb[sd.st[sd.s]].K;
   return K <= 2 * kTcCols && sd.Bs + 1 <= 9 &&
          (size_t)G_range * ceil_div(K, kTcCols) * kTcBTile <= (size_t(256) << 20);
