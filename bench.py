@@ -477,6 +477,19 @@ DATA = ("synthetic: seeded SplitMix64/Box-Muller LLaMA-2-shaped weights and cali
         "activations (no real weights or Red_Pajama text)")
 
 
+def assign_lanes(sizes, streams):
+    """Matrices (by size) to at most `streams` lanes: largest first, each to the least loaded
+    lane. Returns the lanes' matrix indices, in the order each lane runs them."""
+    n = max(1, min(streams, len(sizes)))
+    lanes = [[] for _ in range(n)]
+    load = [0] * n
+    for j in sorted(range(len(sizes)), key=lambda j: (-sizes[j], j)):
+        q = load.index(min(load))
+        lanes[q].append(j)
+        load[q] += sizes[j]
+    return lanes
+
+
 def config_dict(cfg, rows_note=None):
     c = {"workload": cfg.name, "M": cfg.M, "N": cfg.N, "n_tok": cfg.n_tok, "d": cfg.d,
          "K_base": cfg.K_base, "n_ext": cfg.n_ext, "K_ext": cfg.K_ext,
@@ -563,13 +576,8 @@ def main():
     # The matrices of a step are independent problems. With --streams S > 1 they run on S
     # streams from S host threads (the library replays each matrix's graph on its own stream
     # without holding its cache lock), balanced by size, largest first.
-    nstr = max(1, min(args.streams, len(work)))
-    lanes = [[] for _ in range(nstr)]
-    load = [0] * nstr
-    for j in sorted(range(len(work)), key=lambda j: -work[j]["cfg"].M * work[j]["cfg"].N):
-        q = load.index(min(load))
-        lanes[q].append(j)
-        load[q] += work[j]["cfg"].M * work[j]["cfg"].N
+    lanes = assign_lanes([w["cfg"].M * w["cfg"].N for w in work], args.streams)
+    nstr = len(lanes)
     streams = [stream] if nstr == 1 else [torch.cuda.Stream(dev) for _ in range(nstr)]
     pool = None
     if nstr > 1:

@@ -1,5 +1,6 @@
 """Host-side logic of bench.py on the CPU: the score count that the CPU baseline's rate
-divides by is the number of (hypothesis, codeword) pairs the schedule actually scores."""
+divides by is the number of (hypothesis, codeword) pairs the schedule actually scores; the
+oracle pool; and the assignment of a block's matrices to streams."""
 import numpy as np
 
 
@@ -50,3 +51,23 @@ def test_oracle_pool_runs_one_sample_per_core_and_counts_their_scores():
     assert cores == 2 and wall > 0
     assert abs(rate * wall - 2 * bench.schedule_scores(cfg, rows, cfg.N)) <= 1e-6 * rate * wall
     assert "2 row blocks" in desc
+
+
+def test_lanes_cover_every_matrix_once_largest_first():
+    import bench
+    import synthetic as S
+    sizes = [c.M * c.N for c in S.C5]
+    for streams in (1, 2, 3, 4, 7, 12):
+        lanes = bench.assign_lanes(sizes, streams)
+        assert len(lanes) == min(streams, len(sizes))
+        assert sorted(j for lane in lanes for j in lane) == list(range(len(sizes)))
+        loads = [sum(sizes[j] for j in lane) for lane in lanes]
+        # greedy longest-first: no lane exceeds the lightest by more than one matrix
+        assert max(loads) - min(loads) <= max(sizes)
+        for lane in lanes:  # each lane runs its largest matrix first
+            assert [sizes[j] for j in lane] == sorted((sizes[j] for j in lane), reverse=True)
+    # the block's three 11008 x 4096 / 4096 x 11008 matrices go to different lanes with 3
+    big = [j for j, s in enumerate(sizes) if s == max(sizes)]
+    lanes = bench.assign_lanes(sizes, 3)
+    assert sorted(lane[0] for lane in lanes) == sorted(big)
+    assert bench.assign_lanes([5], 3) == [[0]]
