@@ -230,6 +230,9 @@ crvq_status crvq_kmeans_init(const float* T, int64_t ldT, int64_t M, int64_t G_s
  *   vec_err         [M x G_sub] out or NULL: err of the written tuple (fp64, rounded).
  * Requires 1 <= B <= 16, 0 <= n_fixed < n_cb <= 8. Sets of more than 65535 groups return
  * CRVQ_ERR_UNSUPPORTED (a beam stage launches one grid row per group).
+ * Beam stages over codebooks of at most 256 codewords with B <= 8 score on the tensor cores and
+ * keep exactly the lists of the SIMT stages; CRVQ_BEAM_TC=0 in the environment (read at every
+ * call) keeps every stage on the SIMT kernels. The results are identical either way.
  */
 crvq_status crvq_encode_beam(const float* T, int64_t ldT, int64_t M, int64_t G_sub, int32_t d,
                              const float* H_blocks, const crvq_codebook* cbs, int32_t n_cb,
