@@ -16,8 +16,9 @@ Data model (shared vocabulary with the C-ABI):
   * A vector set is a row-major M x (G_sub*d) block of a matrix with leading dimension ldT;
     vector (i, g) is scored with the d x d Hessian block H_blocks[g].
   * A codebook is (C: K x d, codes: M x G_cov int, G_cov): it covers groups g < G_cov of the
-    set. The base codebook covers every group; the extended codebooks cover only the first
-    G_c groups, which hold the reordered critical channels (Sec. 4.3, Fig. 2). The
+    set. The base codebook (each of them, with several, Sec. 6.4) covers every group; the
+    extended codebooks cover only the first G_c groups, which hold the reordered critical
+    channels (Sec. 4.3, Fig. 2). The
     reconstruction of vector (i, g) is the sum of C_s[codes_s[i, g]] over the codebooks
     that cover g (additive VQ, Sec. 3.1 last paragraph and Sec. 4.3).
 
@@ -41,7 +42,7 @@ Readings where the paper is silent or ambiguous (all listed in the design notes)
   * BeamSearchOptimize (Alg. 1) is a stage-wise beam over the codebooks that cover a
     vector, in codebook order, keeping the B best partial tuples by (err, parent rank, k).
 
-Beyond the current GPU path (each pinned in the tests, ahead of its kernel):
+Beyond the per-matrix schedule (each pinned in the tests):
   * MODE_WA_INV / hinv_diag: Eq. (wa) with the inverse-Hessian diagonal;
   * coupled_sweep / full_loss: code search under the full Alg. 1 loss, cross-group terms
     included (Gauss-Seidel over groups);
@@ -483,7 +484,9 @@ def quantize_layer(W, X, cfg):
     with the readings above.
 
     cfg has attributes d, K_base, n_ext, K_ext, crit_frac, B, kmeans_iters, refine_rounds,
-    eps_rel, damp_rel, importance_mode, seed. Returns a dict of every intermediate result."""
+    eps_rel, damp_rel, importance_mode, seed, and optionally n_base (base codebooks, default
+    1). Returns a dict of every intermediate result; out["codebooks"] lists the n_base base
+    codebooks, then the extended ones."""
     d = cfg.d
     W = np.asarray(W, dtype=np.float32)
     M, N = W.shape
@@ -502,11 +505,16 @@ def quantize_layer(W, X, cfg):
         W, d, W_pre, xsq, H, cfg.crit_frac, cfg.importance_mode,
         phase_seed(cfg.seed, PHASE_RANDOM, 0))
     out.update(perm=perm, importance=I, W_sorted=Ws, H_blocks=Hb, n_crit_groups=Gc)
-    # S4 (Alg. 1, base codebook steps)
-    Cb0 = kmeans_init(Ws, d, G, cfg.K_base, phase_seed(cfg.seed, PHASE_BASE, 0))
-    base, obj = lloyd(Ws, d, Hb, [], Cb0, G, cfg.kmeans_iters)
-    out["base_objective"] = obj
-    cbs = [base]
+    # S4 (Alg. 1, base codebook steps). With several base codebooks (Sec. 6.4, the m = 2
+    # setting) base codebook b covers every group and is fitted on the residual of bases
+    # 0..b-1, as the extended loop does on the critical groups; cfg.n_base defaults to one.
+    cbs = []
+    for b in range(getattr(cfg, "n_base", 1)):
+        Cb0 = kmeans_init(Ws, d, G, cfg.K_base, phase_seed(cfg.seed, PHASE_BASE, b), cbs)
+        base, obj = lloyd(Ws, d, Hb, cbs, Cb0, G, cfg.kmeans_iters)
+        if b == 0:
+            out["base_objective"] = obj
+        cbs.append(base)
     # S5 (Alg. 1, extended-codebook loop): extended codebooks on the critical residual
     crit_losses = [reconstruct_error(Ws, d, Hb, perm, cbs, Gc)[2]]
     Tc = Ws[:, :Gc * d]

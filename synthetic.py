@@ -111,6 +111,7 @@ class LayerConfig:
     importance_mode: int = 0  # 0 = W-A (App. A.2), 1 = W-only, 2 = random
     seed: int = 0
     x_tag: str = ""           # layers that share X use the same tag
+    n_base: int = 1           # base codebooks over every group (Sec. 6.4's m = 2 setting)
 
     @property
     def G(self) -> int:

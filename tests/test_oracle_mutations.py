@@ -290,8 +290,10 @@ def _schedule_variant(slip):
     """The per-matrix schedule with one wiring slip: the base codebook fitted on W instead of
     the reordered W ("base_on_W"), warm-started from the prequantize codebook ("warm_start"),
     extended codebooks fitted on the raw critical vectors instead of the residual of the base
-    ("ext_without_base"), or the refinement updating the codebooks in reverse order
-    ("refine_reversed"). Otherwise the same steps as the oracle's quantize_layer."""
+    ("ext_without_base"), the refinement updating the codebooks in reverse order
+    ("refine_reversed"), a second base codebook fitted on the reordered W instead of the
+    residual of the first ("base2_on_W_sorted") or on the critical groups only
+    ("base2_critical_only"). Otherwise the same steps as the oracle's quantize_layer."""
     def plant(orig):
         def f(W, X, cfg):
             d = cfg.d
@@ -317,6 +319,18 @@ def _schedule_variant(slip):
             base, obj = O.lloyd(T_base, d, Hb, [], Cb0, G, cfg.kmeans_iters)
             out["base_objective"] = obj
             cbs = [base]
+            for b in range(1, getattr(cfg, "n_base", 1)):
+                if slip == "base2_on_W_sorted":        # not on the residual of base 1
+                    fixed, Gb = [], G
+                elif slip == "base2_critical_only":    # only the critical groups
+                    fixed, Gb = [O.Codebook(cb.C, cb.codes[:, :Gc], Gc) for cb in cbs], Gc
+                else:
+                    fixed, Gb = list(cbs), G
+                Tb = Ws[:, :Gb * d]
+                Cb0 = O.kmeans_init(Tb, d, Gb, cfg.K_base,
+                                    O.phase_seed(cfg.seed, O.PHASE_BASE, b), fixed)
+                nb, _ = O.lloyd(Tb, d, Hb[:Gb], fixed, Cb0, Gb, cfg.kmeans_iters)
+                cbs.append(nb)
             Tc, Hbc = Ws[:, :Gc * d], Hb[:Gc]
             for t in range(1, cfg.n_ext + 1):
                 fixed = [] if slip == "ext_without_base" else \
@@ -347,6 +361,8 @@ def _schedule_variant(slip):
 _SCHEDULE_PINS = ["test_schedule_with_one_codeword_per_codebook_is_a_sequence_of_weighted_means",
                   "test_schedule_without_lloyd_iterations_keeps_the_sampled_codewords",
                   "test_schedule_with_a_codeword_per_vector_reconstructs_exactly"]
+_TWO_BASE_PINS = ["test_schedule_with_two_base_codebooks_of_one_codeword_each",
+                  "test_schedule_with_two_base_codebooks_without_lloyd_iterations"]
 
 
 # (name, oracle attribute, planted version, pins that must catch it: a test name, or a test
@@ -430,6 +446,10 @@ MUTATIONS = [
      _schedule_variant("ext_without_base"), _SCHEDULE_PINS),
     ("schedule: refinement updates the codebooks in reverse order", "quantize_layer",
      _schedule_variant("refine_reversed"), _SCHEDULE_PINS),
+    ("schedule: second base codebook fitted on the reordered W, not the residual",
+     "quantize_layer", _schedule_variant("base2_on_W_sorted"), _TWO_BASE_PINS),
+    ("schedule: second base codebook on the critical groups only", "quantize_layer",
+     _schedule_variant("base2_critical_only"), _TWO_BASE_PINS),
 ]
 
 

@@ -634,6 +634,90 @@ def test_schedule_without_lloyd_iterations_keeps_the_sampled_codewords():
         np.testing.assert_array_equal(cbs[t + 1].codes, code_e[t])
 
 
+def test_schedule_with_two_base_codebooks_of_one_codeword_each():
+    """Two base codebooks (Sec. 6.4's m = 2 setting) with one codeword each, one extended
+    codebook of one codeword: the second base is the H-weighted mean of the residual of the
+    first over every group (which is zero), the extended codebook that of the residual of both
+    on the critical groups, and the refinement round updates base 1, base 2, ext 1 in that
+    order with the others fixed."""
+    cfg = S.LayerConfig("pin_m2_k1", 6, 32, 48, "outlier_cols", "lognormal", 0.5,
+                        n_outlier_cols=2, K_base=1, n_ext=1, K_ext=1, crit_frac=0.3, B=2,
+                        kmeans_iters=2, refine_rounds=1, n_base=2)
+    W, X = S.gen_W(cfg), S.gen_X(cfg)
+    out = O.quantize_layer(W, X, cfg)
+    d, M, N = 8, cfg.M, cfg.N
+    G, Gc = N // d, 2
+    H, xsq, _ = _h64(X, cfg.damp_rel)
+    W64 = W.astype(np.float64)
+    vec = lambda A, i, g: A[i, g * d:(g + 1) * d]
+    H0 = _blocks(H, np.arange(N), d)
+    c_pre = _wmean([(H0[g], vec(W64, i, g)) for i in range(M) for g in range(G)])
+    perm = _importance_perm(W, np.tile(c_pre, G)[None, :], xsq)
+    Ws = W64[:, perm]
+    Hs = _blocks(H, perm, d)
+    every = [(i, g) for i in range(M) for g in range(G)]
+    crit = [(i, g) for i in range(M) for g in range(Gc)]
+    c_1 = _wmean([(Hs[g], vec(Ws, i, g)) for i, g in every])
+    c_2 = _wmean([(Hs[g], vec(Ws, i, g) - c_1) for i, g in every])
+    c_e = _wmean([(Hs[g], vec(Ws, i, g) - c_1 - c_2) for i, g in crit])
+    ext = lambda g: c_e if g < Gc else 0.0
+    c_1 = _wmean([(Hs[g], vec(Ws, i, g) - c_2 - ext(g)) for i, g in every])
+    c_2 = _wmean([(Hs[g], vec(Ws, i, g) - c_1 - ext(g)) for i, g in every])
+    c_e = _wmean([(Hs[g], vec(Ws, i, g) - c_1 - c_2) for i, g in crit])
+    scale = np.abs(c_pre).max()
+    cbs = out["codebooks"]
+    assert len(cbs) == 3 and [cb.G_cov for cb in cbs] == [G, G, Gc]
+    for cb, c in zip(cbs, (c_1, c_2, c_e)):
+        np.testing.assert_allclose(np.asarray(cb.C, np.float64).reshape(-1), c, rtol=0,
+                                   atol=2e-5 * scale)
+    rec = np.tile(c_1 + c_2, G)
+    rec[:Gc * d] += np.tile(c_e, Gc)
+    D = Ws - rec[None, :]
+    lb = sum(float(vec(D, i, g) @ Hs[g] @ vec(D, i, g)) for i, g in every)
+    assert out["loss_block"] == pytest.approx(lb, rel=1e-5)
+
+
+def test_schedule_with_two_base_codebooks_without_lloyd_iterations():
+    """Two base codebooks, kmeans_iters = 0, no refinement: base 2 is drawn (phase 2,
+    codebook 1) from the residual of base 1 over every group and encodes that residual; the
+    extended codebook is drawn (phase 3, codebook 1) from the critical residual of both."""
+    cfg = S.LayerConfig("pin_m2_t0", 8, 32, 40, "outlier_cols", "lognormal", 0.5,
+                        n_outlier_cols=2, K_base=8, n_ext=1, K_ext=4, crit_frac=0.3, B=2,
+                        kmeans_iters=0, refine_rounds=0, seed=7, n_base=2)
+    W, X = S.gen_W(cfg), S.gen_X(cfg)
+    out = O.quantize_layer(W, X, cfg)
+    d, M, N = 8, cfg.M, cfg.N
+    G, Gc = N // d, 2
+    H, xsq, _ = _h64(X, cfg.damp_rel)
+    W64 = W.astype(np.float64)
+    vec = lambda A, v, Gs: A[v // Gs, (v % Gs) * d:(v % Gs + 1) * d]
+    H0 = _blocks(H, np.arange(N), d)
+    C_pre = np.stack([vec(W64, v, G) for v in _strata(M * G, 8, _seed(7, 1, 0))])
+    W_pre = np.concatenate([C_pre[[_nearest(vec(W64, i * G + g, G), C_pre, H0[g])
+                                   for i in range(M)]] for g in range(G)], axis=1)
+    perm = _importance_perm(W, W_pre, xsq)
+    Ws = W64[:, perm]
+    Hs = _blocks(H, perm, d)
+    res = np.stack([vec(Ws, v, G) for v in range(M * G)])      # vector v = i * G + g
+    C_b, code_b = [], []
+    for b in (0, 1):
+        Cb = res[_strata(M * G, 8, _seed(7, 2, b))]
+        cb = np.array([_nearest(res[v], Cb, Hs[v % G]) for v in range(M * G)])
+        res = res - Cb[cb]
+        C_b.append(Cb)
+        code_b.append(cb.reshape(M, G))
+    rc = np.stack([res[i * G + g] for i in range(M) for g in range(Gc)])
+    C_e = rc[_strata(M * Gc, 4, _seed(7, 3, 1))]
+    code_e = np.array([_nearest(rc[v], C_e, Hs[v % Gc]) for v in range(M * Gc)])
+    np.testing.assert_array_equal(out["perm"], perm)
+    cbs = out["codebooks"]
+    for b in (0, 1):
+        np.testing.assert_allclose(cbs[b].C, C_b[b], rtol=0, atol=1e-7)
+        np.testing.assert_array_equal(cbs[b].codes, code_b[b])
+    np.testing.assert_allclose(cbs[2].C, C_e, rtol=0, atol=1e-7)
+    np.testing.assert_array_equal(cbs[2].codes, code_e.reshape(M, Gc))
+
+
 def test_schedule_with_a_codeword_per_vector_reconstructs_exactly():
     """K_base equal to the number of vectors: the strata hold one vector each, so the base
     k-means starts from every vector of the reordered W and the reconstruction is exact; the
