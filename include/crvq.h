@@ -369,7 +369,8 @@ typedef struct crvq_config {
   float eps_rel;           /* stop refining when loss_block > (1 - eps_rel) * previous */
   float damp_rel;          /* Hessian damping, relative to the mean diagonal */
   int32_t importance_mode; /* CRVQ_IMPORTANCE_* */
-  int32_t _pad;
+  int32_t n_base;          /* base codebooks over every group, 0 or 1 = one (Sec. 6.4 uses
+                              two, "m = 2"); n_base + n_ext <= 8 */
   uint64_t seed;
 } crvq_config;
 
@@ -377,8 +378,8 @@ typedef struct crvq_config {
  * through the device inside the call). */
 typedef struct crvq_layer_outputs {
   int32_t* perm;       /* [N] channel order, perm[new] = old */
-  float* C_base;       /* [K_base x d] */
-  int32_t* codes_base; /* [M x N/d], vector (i, g) in the sorted order */
+  float* C_base;       /* [n_base x K_base x d] */
+  int32_t* codes_base; /* [n_base x M x N/d], vector (i, g) in the sorted order */
   float* C_ext;        /* [n_ext x K_ext x d] */
   int32_t* codes_ext;  /* [n_ext x M x G_c] */
   float* W_hat;        /* [M x N] reconstruction in the original order, or NULL */
@@ -402,12 +403,15 @@ typedef struct crvq_layer_report {
  * One weight matrix through Alg. 1, prequantization through the refinement loop (everything
  * but block / end-to-end fine-tuning):
  * S1 Hessian; S2 prequantize (k-means + encode in the original order); S3 importance and
- * reorder; S4 base codebook (k-means over all vectors); S5 each extended codebook (k-means
- * on the critical residual, greedy encode); S6 up to refine_rounds rounds of
+ * reorder; S4 base codebook (k-means over all vectors; with n_base > 1 each further base
+ * codebook is fitted the same way on the residual of the earlier ones over every vector);
+ * S5 each extended codebook (k-means on the critical residual of every earlier codebook,
+ * greedy encode); S6 up to refine_rounds rounds of
  * least-squares updates of every codebook followed by a joint beam re-encode (keep-if-better);
  * S7 losses and the reconstruction in the original order. Per-phase seeds are
- * SplitMix64(cfg->seed, phase * 1024 + codebook) with phase 1 = prequantize, 2 = base,
- * 3 = extended, 4 = random importance. W [M x N], X [n_tok x N] may be host or device
+ * SplitMix64(cfg->seed, phase * 1024 + codebook) with phase 1 = prequantize, 2 = base
+ * (codebook b = 0 .. n_base - 1), 3 = extended (codebook t = 1 .. n_ext), 4 = random
+ * importance. The refinement updates the base codebooks, then the extended ones, in order. W [M x N], X [n_tok x N] may be host or device
  * pointers. Synchronizes `stream` (the report is host memory).
  * When W, X and every output are device pointers and refine_rounds <= 1, the schedule has no
  * host synchronisation inside: it is captured into a CUDA graph on the first call for a given

@@ -24,7 +24,7 @@ class crvq_config(C.Structure):
                 ("K_ext", C.c_int32), ("crit_frac", C.c_float), ("B", C.c_int32),
                 ("kmeans_iters", C.c_int32), ("refine_rounds", C.c_int32),
                 ("eps_rel", C.c_float), ("damp_rel", C.c_float),
-                ("importance_mode", C.c_int32), ("_pad", C.c_int32), ("seed", C.c_uint64)]
+                ("importance_mode", C.c_int32), ("n_base", C.c_int32), ("seed", C.c_uint64)]
 
 
 class crvq_layer_outputs(C.Structure):

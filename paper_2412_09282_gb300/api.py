@@ -332,13 +332,15 @@ class LayerOutputs:
 def _cfg_struct(cfg) -> _lib.crvq_config:
     return _lib.crvq_config(cfg.d, cfg.K_base, cfg.n_ext, cfg.K_ext, cfg.crit_frac, cfg.B,
                             cfg.kmeans_iters, cfg.refine_rounds, cfg.eps_rel, cfg.damp_rel,
-                            cfg.importance_mode, 0, int(cfg.seed) & (2**64 - 1))
+                            cfg.importance_mode, getattr(cfg, "n_base", 1),
+                            int(cfg.seed) & (2**64 - 1))
 
 
 def crvq_quantize_layer(W, X, cfg, want_W_hat=True, out=None, stream=None, device=None):
     """Alg. 1, prequantization through the refinement loop, for one matrix. W, X: torch
     tensors on the GPU, or pinned/pageable CPU tensors (then the library stages them and the
-    outputs are CPU tensors)."""
+    outputs are CPU tensors). With cfg.n_base > 1 base codebooks, C_base and codes_base gain a
+    leading axis of that length."""
     M, N = W.shape
     n_tok = X.shape[0]
     d = cfg.d
@@ -351,10 +353,13 @@ def crvq_quantize_layer(W, X, cfg, want_W_hat=True, out=None, stream=None, devic
     def alloc(shape, dtype):
         return torch.empty(shape, dtype=dtype, device=dev, pin_memory=pin)
 
+    n_base = getattr(cfg, "n_base", 1)
+    lead = (n_base,) if n_base > 1 else ()
+
     if out is None:
         out = LayerOutputs(
-            perm=alloc((N,), torch.int32), C_base=alloc((cfg.K_base, d), torch.float32),
-            codes_base=alloc((M, G), torch.int32),
+            perm=alloc((N,), torch.int32), C_base=alloc(lead + (cfg.K_base, d), torch.float32),
+            codes_base=alloc(lead + (M, G), torch.int32),
             C_ext=alloc((max(cfg.n_ext, 0), cfg.K_ext, d), torch.float32),
             codes_ext=alloc((max(cfg.n_ext, 0), M, Gc), torch.int32),
             W_hat=alloc((M, N), torch.float32) if want_W_hat else None,

@@ -727,8 +727,11 @@ struct OutBuf {
 
 namespace {
 
+// Base codebooks of a configuration (n_base 0 reads as one).
+int n_base_of(const crvq_config* cfg) { return cfg->n_base > 1 ? cfg->n_base : 1; }
+
 // Device outputs of one layer (every pointer on the device; C_ext / codes_ext NULL when
-// n_ext = 0, W_hat and imp may be NULL).
+// n_ext = 0, W_hat and imp may be NULL). C_base / codes_base hold n_base codebooks back to back.
 struct LayerDev {
   int32_t* perm;
   float* C_base;
@@ -804,37 +807,46 @@ crvq_status run_schedule(const float* W, const float* X, int64_t M, int64_t N, i
                                  phase_seed(cfg->seed, 4, 0), o.perm, o.imp, Ws, nullptr, s));
   CRVQ_TRY(launch_tc_hessian_blocks(Xt, ldt, n_tok, N, o.perm, true, 0.f, nullptr, nullptr,
                                     delta64, Hb, s));
-  // S4: base codebook over all vectors (Alg. 1, base codebook steps)
+  // S4: base codebooks over all vectors (Alg. 1, base codebook steps). With several (Sec. 6.4,
+  // the m = 2 setting) base b is fitted on the residual of bases 0..b-1 over every group.
+  const int nb = n_base_of(cfg);
   CbList all{};
-  all.n = 1 + cfg->n_ext;
-  all.cb[0] = CbView{o.C_base, o.codes_base, G, G, cfg->K_base};
+  all.n = nb + cfg->n_ext;
+  for (int b = 0; b < nb; ++b)
+    all.cb[b] = CbView{o.C_base + (size_t)b * cfg->K_base * d, o.codes_base + (size_t)b * M * G,
+                       G, G, cfg->K_base};
   for (int t = 1; t <= cfg->n_ext; ++t)
-    all.cb[t] = CbView{o.C_ext + (size_t)(t - 1) * cfg->K_ext * d,
-                       o.codes_ext + (size_t)(t - 1) * M * Gc, Gc, Gc, cfg->K_ext};
+    all.cb[nb + t - 1] = CbView{o.C_ext + (size_t)(t - 1) * cfg->K_ext * d,
+                                o.codes_ext + (size_t)(t - 1) * M * Gc, Gc, Gc, cfg->K_ext};
   const SetView full{Ws, N, M, G, Hb};
-  {
+  for (int b = 0; b < nb; ++b) {
     CbList cl{};
-    cl.n = 1;
-    cl.cb[0] = all.cb[0];
-    CRVQ_TRY(launch_kmeans_init(full, CbList{}, cfg->K_base, phase_seed(cfg->seed, 2, 0),
-                                o.C_base, s));
+    cl.n = b + 1;
+    for (int q = 0; q <= b; ++q) cl.cb[q] = all.cb[q];
+    CbList fixed{};
+    fixed.n = b;
+    for (int q = 0; q < b; ++q) fixed.cb[q] = all.cb[q];
+    CRVQ_TRY(launch_kmeans_init(full, fixed, cfg->K_base, phase_seed(cfg->seed, 2, b),
+                                const_cast<float*>(all.cb[b].C), s));
     CRVQ_TRY(lloyd(full, cl, cfg->kmeans_iters, ex, s));
   }
-  // S5: extended codebooks on the critical residual (Alg. 1, extended-codebook loop)
+  // S5: extended codebooks on the critical residual of every earlier codebook (Alg. 1,
+  // extended-codebook loop)
   if (cfg->n_ext > 0) {
     const SetView crit{Ws, N, M, Gc, Hb};
     for (int t = 1; t <= cfg->n_ext; ++t) {
+      const int j = nb + t - 1;
       CbList cl{};
-      cl.n = t + 1;
-      for (int q = 0; q <= t; ++q) {
+      cl.n = j + 1;
+      for (int q = 0; q <= j; ++q) {
         cl.cb[q] = all.cb[q];
         cl.cb[q].G_cov = Gc;
       }
       CbList fixed{};
-      fixed.n = t;
-      for (int q = 0; q < t; ++q) fixed.cb[q] = cl.cb[q];
+      fixed.n = j;
+      for (int q = 0; q < j; ++q) fixed.cb[q] = cl.cb[q];
       CRVQ_TRY(launch_kmeans_init(crit, fixed, cfg->K_ext, phase_seed(cfg->seed, 3, t),
-                                  const_cast<float*>(all.cb[t].C), s));
+                                  const_cast<float*>(all.cb[j].C), s));
       CRVQ_TRY(lloyd(crit, cl, cfg->kmeans_iters, ex, s));
     }
   }
@@ -1061,7 +1073,7 @@ crvq_status run_graph(const float* W, const float* X, int64_t M, int64_t N, int6
 // shape running concurrently on several streams each take their own set.
 struct Staging {
   int dev = -1;
-  int64_t M = 0, N = 0, n_tok = 0, K_base = 0, n_ext = 0, K_ext = 0, Gc = 0;
+  int64_t M = 0, N = 0, n_tok = 0, n_base = 0, K_base = 0, n_ext = 0, K_ext = 0, Gc = 0;
   float *W = nullptr, *X = nullptr, *C_base = nullptr, *C_ext = nullptr, *W_hat = nullptr,
         *imp = nullptr;
   int32_t *perm = nullptr, *codes_base = nullptr, *codes_ext = nullptr;
@@ -1086,9 +1098,10 @@ crvq_status acquire_staging(int dev, int64_t M, int64_t N, int64_t n_tok, const 
                             int64_t Gc, Staging** out) {
   std::lock_guard<std::mutex> lk(g_stage_mu);
   const int d = cfg->d;
+  const int nb = n_base_of(cfg);
   for (auto* sg : g_stagings)
     if (sg->dev == dev && sg->M == M && sg->N == N && sg->n_tok == n_tok &&
-        sg->K_base == cfg->K_base && sg->n_ext == cfg->n_ext &&
+        sg->n_base == nb && sg->K_base == cfg->K_base && sg->n_ext == cfg->n_ext &&
         sg->K_ext == (cfg->n_ext ? cfg->K_ext : 0) && sg->Gc == Gc && sg->users == 0) {
       sg->used = ++g_stage_clock;
       sg->users = 1;
@@ -1110,6 +1123,7 @@ crvq_status acquire_staging(int dev, int64_t M, int64_t N, int64_t n_tok, const 
   sg->M = M;
   sg->N = N;
   sg->n_tok = n_tok;
+  sg->n_base = nb;
   sg->K_base = cfg->K_base;
   sg->n_ext = cfg->n_ext;
   sg->K_ext = cfg->n_ext ? cfg->K_ext : 0;
@@ -1117,11 +1131,11 @@ crvq_status acquire_staging(int dev, int64_t M, int64_t N, int64_t n_tok, const 
   const int64_t G = N / d;
   bool ok = cudaMalloc(&sg->W, (size_t)M * N * 4) == cudaSuccess &&
             cudaMalloc(&sg->X, (size_t)n_tok * N * 4) == cudaSuccess &&
-            cudaMalloc(&sg->C_base, (size_t)cfg->K_base * d * 4) == cudaSuccess &&
+            cudaMalloc(&sg->C_base, (size_t)nb * cfg->K_base * d * 4) == cudaSuccess &&
             cudaMalloc(&sg->W_hat, (size_t)M * N * 4) == cudaSuccess &&
             cudaMalloc(&sg->imp, (size_t)N * 4) == cudaSuccess &&
             cudaMalloc(&sg->perm, (size_t)N * 4) == cudaSuccess &&
-            cudaMalloc(&sg->codes_base, (size_t)M * G * 4) == cudaSuccess;
+            cudaMalloc(&sg->codes_base, (size_t)nb * M * G * 4) == cudaSuccess;
   if (ok && cfg->n_ext > 0)
     ok = cudaMalloc(&sg->C_ext, (size_t)cfg->n_ext * cfg->K_ext * d * 4) == cudaSuccess &&
          cudaMalloc(&sg->codes_ext, (size_t)cfg->n_ext * M * Gc * 4) == cudaSuccess;
@@ -1159,6 +1173,9 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   CRVQ_CHECK_ARG(cfg->K_base >= 1 && cfg->K_base <= 65536 && cfg->K_base <= M * G,
                  "K_base out of range");
   CRVQ_CHECK_ARG(cfg->n_ext >= 0 && cfg->n_ext <= kMaxCodebooks - 1, "n_ext must be in [0, 7]");
+  CRVQ_CHECK_ARG(cfg->n_base >= 0 && n_base_of(cfg) + cfg->n_ext <= kMaxCodebooks,
+                 "n_base must be >= 0 with n_base + n_ext <= 8");
+  const int nb = n_base_of(cfg);
   CRVQ_CHECK_ARG(cfg->crit_frac >= 0.f && cfg->crit_frac <= 1.f, "crit_frac must be in [0, 1]");
   CRVQ_CHECK_ARG(cfg->B >= 1 && cfg->B <= 16, "B must be in [1, 16]");
   CRVQ_CHECK_ARG(cfg->kmeans_iters >= 0 && cfg->refine_rounds >= 0, "negative iteration count");
@@ -1234,8 +1251,8 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
       };
       LayerDev o{};
       o.perm = place(out->perm, sg->perm, (size_t)N);
-      o.C_base = place(out->C_base, sg->C_base, (size_t)cfg->K_base * d);
-      o.codes_base = place(out->codes_base, sg->codes_base, (size_t)M * G);
+      o.C_base = place(out->C_base, sg->C_base, (size_t)nb * cfg->K_base * d);
+      o.codes_base = place(out->codes_base, sg->codes_base, (size_t)nb * M * G);
       if (cfg->n_ext) {
         o.C_ext = place(out->C_ext, sg->C_ext, (size_t)cfg->n_ext * cfg->K_ext * d);
         o.codes_ext = place(out->codes_ext, sg->codes_ext, (size_t)cfg->n_ext * M * Gc);
@@ -1261,8 +1278,8 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   OutBuf<int32_t> o_perm, o_codes_base, o_codes_ext;
   OutBuf<float> o_C_base, o_C_ext, o_W_hat, o_imp;
   CRVQ_TRY(o_perm.init(out->perm, N, s));
-  CRVQ_TRY(o_C_base.init(out->C_base, (size_t)cfg->K_base * d, s));
-  CRVQ_TRY(o_codes_base.init(out->codes_base, (size_t)M * G, s));
+  CRVQ_TRY(o_C_base.init(out->C_base, (size_t)nb * cfg->K_base * d, s));
+  CRVQ_TRY(o_codes_base.init(out->codes_base, (size_t)nb * M * G, s));
   CRVQ_TRY(o_C_ext.init(out->C_ext, (size_t)cfg->n_ext * cfg->K_ext * d, s));
   CRVQ_TRY(o_codes_ext.init(out->codes_ext, (size_t)cfg->n_ext * M * Gc, s));
   if (out->W_hat) CRVQ_TRY(o_W_hat.init(out->W_hat, (size_t)M * N, s));

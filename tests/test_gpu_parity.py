@@ -457,10 +457,11 @@ def _gpu_schedule_with_checks(W, X, cfg):
                                    cfg.importance_mode, seed(4, 0))
     np.testing.assert_array_equal(host(perm), po[0])
     Ws_np, Hb_np = host(Ws), host(Hb)
-    # S4
-    Cb0 = P.crvq_kmeans_init(Ws, d, G, cfg.K_base, seed(2, 0))
-    base = lloyd(Ws, Hb, [], Cb0, G, Ws_np, Hb_np)
-    cbs = [base]
+    # S4: base codebook b on the residual of bases 0..b-1 over every group
+    cbs = []
+    for b in range(getattr(cfg, "n_base", 1)):
+        Cb0 = P.crvq_kmeans_init(Ws, d, G, cfg.K_base, seed(2, b), fixed=list(cbs))
+        cbs.append(lloyd(Ws, Hb, list(cbs), Cb0, G, Ws_np, Hb_np))
     # S5
     crit = Ws[:, :Gc * d]
     for t in range(1, cfg.n_ext + 1):
@@ -485,7 +486,7 @@ def _gpu_schedule_with_checks(W, X, cfg):
         for s in range(len(cbs)):
             diff[:, :cbs[s].G_cov] |= gpu[s] != oc[s]
         for i, g in zip(*np.nonzero(diff)):
-            Cs = [before[0].C] + ([cb.C for cb in before[1:]] if g < Gc else [])
+            Cs = [cb.C for cb in before if g < cb.G_cov]
             gap = beam_boundary_gap(Ws_np[i, g * d:(g + 1) * d].astype(np.float64), Hb_np[g],
                                     Cs, cfg.B)
             assert gap < 1e-6, f"refinement code differs at ({i},{g}) with gap {gap}"
@@ -500,27 +501,34 @@ def _gpu_schedule_with_checks(W, X, cfg):
                 losses=(lb, lc, lf))
 
 
-@pytest.mark.parametrize("name", ["c1", "small_B8_3ext"])
+@pytest.mark.parametrize("name", ["c1", "small_B8_3ext", "two_base_2ext"])
 def test_quantize_layer_matches_resynced_stepwise_schedule(c1, name):
     """Every step of the schedule agrees with the oracle given the GPU's state, and the
     one-call crvq_quantize_layer reproduces that trajectory exactly (same kernels, same
-    order; the fused Lloyd statistics equal the standalone update's, bit for bit)."""
+    order; the fused Lloyd statistics equal the standalone update's, bit for bit). The
+    two-base case has two base codebooks over every group (Sec. 6.4's m = 2 setting)."""
     if name == "c1":
         cfg, W, X = c1["cfg"], c1["W"], c1["X"]
     else:
         cfg = S.LayerConfig("pin_med", 256, 192, 300, "outlier_cols", "lognormal", 0.5,
                             n_outlier_cols=5, K_base=128, n_ext=3, K_ext=32, crit_frac=0.1,
                             B=8, kmeans_iters=5)
+        if name == "two_base_2ext":
+            cfg = cfg.with_(n_base=2, K_base=64, n_ext=2, B=4, kmeans_iters=3)
         W, X = S.gen_W(cfg), S.gen_X(cfg)
     ref = _gpu_schedule_with_checks(W, X, cfg)
     out = P.crvq_quantize_layer(dev(W), dev(X), cfg)
     torch.cuda.synchronize()
     np.testing.assert_array_equal(host(out.perm), ref["perm"])
-    np.testing.assert_array_equal(host(out.C_base), ref["cbs"][0][0])
-    np.testing.assert_array_equal(host(out.codes_base), ref["cbs"][0][1])
+    nb = cfg.n_base
+    C_base = host(out.C_base).reshape(nb, cfg.K_base, cfg.d)
+    codes_base = host(out.codes_base).reshape(nb, *ref["cbs"][0][1].shape)
+    for b in range(nb):
+        np.testing.assert_array_equal(C_base[b], ref["cbs"][b][0])
+        np.testing.assert_array_equal(codes_base[b], ref["cbs"][b][1])
     for t in range(cfg.n_ext):
-        np.testing.assert_array_equal(host(out.C_ext[t]), ref["cbs"][t + 1][0])
-        np.testing.assert_array_equal(host(out.codes_ext[t]), ref["cbs"][t + 1][1])
+        np.testing.assert_array_equal(host(out.C_ext[t]), ref["cbs"][nb + t][0])
+        np.testing.assert_array_equal(host(out.codes_ext[t]), ref["cbs"][nb + t][1])
     lb, lc, lf = ref["losses"]
     assert out.report["loss_block"] == pytest.approx(lb, rel=1e-12)
     assert out.report["loss_full"] == pytest.approx(lf, rel=1e-12)
@@ -564,6 +572,32 @@ def test_quantize_layer_host_buffers_match_device(c1):
     np.testing.assert_array_equal(host(a.codes_base), b.codes_base.numpy())
     np.testing.assert_array_equal(host(a.C_ext), b.C_ext.numpy())
     assert a.report["loss_full"] == b.report["loss_full"]
+
+
+def test_quantize_layer_two_base_codebooks_host_direct_and_graph_agree(c1, monkeypatch):
+    """Two base codebooks: the graph replay on device buffers, the staged host-buffer call and
+    the direct (uncaptured) run give the same outputs bit for bit, and each base codebook's
+    codes stay in range with every group covered."""
+    cfg = c1["cfg"].with_(kmeans_iters=2, n_base=2, K_base=64)
+    a = P.crvq_quantize_layer(dev(c1["W"]), dev(c1["X"]), cfg)
+    torch.cuda.synchronize()
+    Wh = torch.from_numpy(c1["W"]).pin_memory()
+    Xh = torch.from_numpy(c1["X"]).pin_memory()
+    b = P.crvq_quantize_layer(Wh, Xh, cfg)
+    monkeypatch.setenv("CRVQ_GRAPHS", "0")
+    c = P.crvq_quantize_layer(dev(c1["W"]), dev(c1["X"]), cfg)
+    torch.cuda.synchronize()
+    M, N = c1["W"].shape
+    assert tuple(a.C_base.shape) == (2, 64, cfg.d)
+    assert tuple(a.codes_base.shape) == (2, M, N // cfg.d)
+    codes = host(a.codes_base)
+    assert codes.min() >= 0 and codes.max() < 64
+    for k in ("perm", "C_base", "codes_base", "C_ext", "codes_ext", "W_hat"):
+        ref = host(getattr(a, k))
+        np.testing.assert_array_equal(ref, getattr(b, k).numpy(), err_msg=k)
+        np.testing.assert_array_equal(ref, host(getattr(c, k)), err_msg=k)
+    for k in ("loss_block", "loss_crit", "loss_full", "loss_pre"):
+        assert a.report[k] == b.report[k] == c.report[k], k
 
 
 def test_quantize_layer_graph_replay_matches_direct_run(c1, monkeypatch):
