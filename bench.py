@@ -44,14 +44,19 @@ def schedule_scores(cfg, M, N):
     G = N // d
     Gc = min(G, int(np.ceil(np.float32(cfg.crit_frac) * N / d - 1e-12))) if cfg.crit_frac > 0 else 0
     n_all, n_crit = M * G, M * Gc
-    s = 2 * (T + 1) * n_all * cfg.K_base                  # prequantize + base k-means
+    n_base = getattr(cfg, "n_base", 1)
+
+    def beam(stages):                                      # pairs per vector of a beam pass
+        total, parents = 0, 1
+        for K in stages:
+            total += parents * K
+            parents = min(cfg.B, parents * K)
+        return total
+
+    s = (1 + n_base) * (T + 1) * n_all * cfg.K_base       # prequantize + base k-means
     s += cfg.n_ext * (T + 1) * n_crit * cfg.K_ext          # extended k-means
-    beam = cfg.K_base
-    parents = min(cfg.B, cfg.K_base)
-    for _ in range(cfg.n_ext):
-        beam += parents * cfg.K_ext
-        parents = min(cfg.B, parents * cfg.K_ext)
-    s += cfg.refine_rounds * (n_crit * beam + (n_all - n_crit) * cfg.K_base)
+    s += cfg.refine_rounds * (n_crit * beam([cfg.K_base] * n_base + [cfg.K_ext] * cfg.n_ext) +
+                              (n_all - n_crit) * beam([cfg.K_base] * n_base))
     return float(s)
 
 
@@ -351,7 +356,8 @@ def coupled_sweep_line(P, work, stream):
 def sweep_grid(name):
     """The synthetic analogs of the paper's ablations on one matrix (no datasets: the block
     losses stand in for perplexity): Table 2's reorder strategies (random, W-only, W-A), the
-    critical ratio lambda and the number of extended codebooks m - 1 (Sec. 6.3-6.4)."""
+    critical ratio lambda, the number of extended codebooks m - 1 (Sec. 6.3-6.4) and two base
+    codebooks, alone and with three extended ones (Sec. 6.4's m = 2 setting at d = 8)."""
     base = S.C5[0] if name == "c5" else S.CONFIGS[name]
     grid = []
     for mode in (2, 1, 0):                                   # Table 2: random, W-only, W-A
@@ -359,8 +365,20 @@ def sweep_grid(name):
     for lam in (0.01, 0.02, 0.05, 0.10):                     # lambda
         grid.append(("lambda", base.with_(crit_frac=lam, n_ext=1)))
     for n_ext in (0, 1, 2, 4):                               # m - 1 extended codebooks
-        grid.append(("m", base.with_(n_ext=n_ext, crit_frac=0.02 if n_ext else 0.02)))
+        grid.append(("m", base.with_(n_ext=n_ext, crit_frac=0.02)))
+    for n_ext in (0, 3):                                     # two base codebooks
+        grid.append(("m_base", base.with_(n_base=2, n_ext=n_ext, crit_frac=0.02)))
     return grid
+
+
+def avg_bits_of(P, cfg):
+    """Bits per weight of a setting (Sec. 3.2 Eq. (bitwidth), App. A.1, the reorder index
+    included): crvq_avg_bits for one base and n_ext extended codebooks of 2^e codewords, plus
+    for each further base codebook e / d code bits per weight and its 2^e fp16 codewords."""
+    e = int(np.log2(cfg.K_base))
+    bits = P.crvq_avg_bits(e, cfg.d, 1 + cfg.n_ext, float(cfg.crit_frac), cfg.M, cfg.N, True)
+    extra = cfg.n_base - 1
+    return bits + extra * (e / cfg.d + (2 ** e) * cfg.d * 16 / (cfg.M * cfg.N))
 
 
 def run_sweep(args):
@@ -389,10 +407,9 @@ def run_sweep(args):
         b.synchronize()
         P.crvq_sync()
         rep = out.report
-        e = int(np.log2(cfg.K_base))
-        bits = P.crvq_avg_bits(e, cfg.d, 1 + cfg.n_ext, float(cfg.crit_frac), cfg.M, cfg.N, True)
+        bits = avg_bits_of(P, cfg)
         print(json.dumps({"sweep": axis, "matrix": cfg.name, "importance_mode": cfg.importance_mode,
-                          "crit_frac": cfg.crit_frac, "n_ext": cfg.n_ext,
+                          "crit_frac": cfg.crit_frac, "n_base": cfg.n_base, "n_ext": cfg.n_ext,
                           "n_crit_groups": rep["n_crit_groups"], "avg_bits": bits,
                           "loss_block": rep["loss_block"], "loss_crit": rep["loss_crit"],
                           "loss_full": rep["loss_full"], "loss_pre": rep["loss_pre"],

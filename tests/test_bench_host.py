@@ -1,10 +1,12 @@
 """Host-side logic of bench.py on the CPU: the score count that the CPU baseline's rate
 divides by is the number of (hypothesis, codeword) pairs the schedule actually scores; the
-oracle pool; and the assignment of a block's matrices to streams."""
+oracle pool; the assignment of a block's matrices to streams; the sweep's bit-widths."""
 import numpy as np
+import pytest
 
 
-def test_schedule_scores_counts_what_the_schedule_scores(monkeypatch):
+@pytest.mark.parametrize("n_base", [1, 2])
+def test_schedule_scores_counts_what_the_schedule_scores(monkeypatch, n_base):
     """bench.schedule_scores (the CPU baseline's numerator) against the pairs the oracle's
     schedule actually scores: every encode call is counted from its arguments (per group, each
     searched stage scores parents x K pairs per vector, parents = min(B, parents x K))."""
@@ -12,7 +14,7 @@ def test_schedule_scores_counts_what_the_schedule_scores(monkeypatch):
     from oracle import crvq_oracle as O
     import synthetic as S
     cfg = S.LayerConfig("count", 16, 64, 32, "plain", "lognormal", 0.5, K_base=8, n_ext=2,
-                        K_ext=4, crit_frac=0.1, B=2, kmeans_iters=2)
+                        K_ext=4, crit_frac=0.1, B=2, kmeans_iters=2, n_base=n_base)
     counted = []
     orig = O.encode_beam
 
@@ -71,3 +73,25 @@ def test_lanes_cover_every_matrix_once_largest_first():
     lanes = bench.assign_lanes(sizes, 3)
     assert sorted(lane[0] for lane in lanes) == sorted(big)
     assert bench.assign_lanes([5], 3) == [[0]]
+
+
+def test_sweep_bit_width_with_two_base_codebooks_follows_eq_bitwidth():
+    """With no extended codebooks (lambda = 0) and no reorder index the setting is plain
+    additive VQ, and Sec. 3.2 Eq. (bitwidth) for a 4096 x 4096 matrix gives
+    n = m e / d + 2^(e - 20) m d (m = 2, e = 8, d = 8: 2 + 2^-12 * 16); the reorder index adds
+    16 bits per channel (App. A.1)."""
+    import bench
+    import synthetic as S
+    import paper_2412_09282_gb300 as P
+    try:
+        P.crvq_version()
+    except (ImportError, OSError):
+        pytest.skip("libcrvq.so not built")
+    cfg = S.LayerConfig("bits", 4096, 4096, 8, "plain", "lognormal", 0.5, K_base=256, n_ext=0,
+                        crit_frac=0.0, n_base=2)
+    perm_bits = 16 * 4096 / 4096 ** 2
+    assert bench.avg_bits_of(P, cfg) == pytest.approx(2 * 8 / 8 + 2 ** -12 * 2 * 8 + perm_bits,
+                                                      rel=1e-12)
+    cfg3 = cfg.with_(n_ext=3, crit_frac=0.02)
+    one = bench.avg_bits_of(P, cfg3.with_(n_base=1))
+    assert bench.avg_bits_of(P, cfg3) == pytest.approx(one + 1 + 2 ** -12 * 8, rel=1e-12)
