@@ -360,7 +360,7 @@ int64_t crvq_n_crit_groups(int64_t N, int32_t d, float crit_frac);
 typedef struct crvq_config {
   int32_t d;               /* vector length (8) */
   int32_t K_base;          /* base codebook size 2^e */
-  int32_t n_ext;           /* extended codebooks (m - 1), 0..7 */
+  int32_t n_ext;           /* extended codebooks (m - 1), 0..7, n_base + n_ext <= 8 */
   int32_t K_ext;           /* extended codebook size */
   float crit_frac;         /* lambda */
   int32_t B;               /* beam width of the refinement re-encode, 1..16 */
