@@ -640,13 +640,22 @@ def test_schedule_with_two_base_codebooks_of_one_codeword_each():
     first over every group (which is zero), the extended codebook that of the residual of both
     on the critical groups, and the refinement round updates base 1, base 2, ext 1 in that
     order with the others fixed."""
+    _two_base_one_codeword(8)
+
+
+def test_schedule_with_two_base_codebooks_of_one_codeword_each_at_d16():
+    """The same at d = 16, the vector length of Sec. 6.4's m = 2 setting."""
+    _two_base_one_codeword(16)
+
+
+def _two_base_one_codeword(d):
     cfg = S.LayerConfig("pin_m2_k1", 6, 32, 48, "outlier_cols", "lognormal", 0.5,
                         n_outlier_cols=2, K_base=1, n_ext=1, K_ext=1, crit_frac=0.3, B=2,
-                        kmeans_iters=2, refine_rounds=1, n_base=2)
+                        kmeans_iters=2, refine_rounds=1, n_base=2, d=d)
     W, X = S.gen_W(cfg), S.gen_X(cfg)
     out = O.quantize_layer(W, X, cfg)
-    d, M, N = 8, cfg.M, cfg.N
-    G, Gc = N // d, 2
+    M, N = cfg.M, cfg.N
+    G, Gc = N // d, -(-3 * N // (10 * d))             # ceil(0.3 * N / d)
     H, xsq, _ = _h64(X, cfg.damp_rel)
     W64 = W.astype(np.float64)
     vec = lambda A, i, g: A[i, g * d:(g + 1) * d]
