@@ -1173,7 +1173,8 @@ crvq_status crvq_quantize_layer(const float* W_in, const float* X_in, int64_t M,
   CRVQ_CHECK_ARG(cfg->K_base >= 1 && cfg->K_base <= 65536 && cfg->K_base <= M * G,
                  "K_base out of range");
   CRVQ_CHECK_ARG(cfg->n_ext >= 0 && cfg->n_ext <= kMaxCodebooks - 1, "n_ext must be in [0, 7]");
-  CRVQ_CHECK_ARG(cfg->n_base >= 0 && n_base_of(cfg) + cfg->n_ext <= kMaxCodebooks,
+  CRVQ_CHECK_ARG(cfg->n_base >= 0 && cfg->n_base <= kMaxCodebooks &&
+                     n_base_of(cfg) + cfg->n_ext <= kMaxCodebooks,
                  "n_base must be >= 0 with n_base + n_ext <= 8");
   const int nb = n_base_of(cfg);
   CRVQ_CHECK_ARG(cfg->crit_frac >= 0.f && cfg->crit_frac <= 1.f, "crit_frac must be in [0, 1]");

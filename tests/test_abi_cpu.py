@@ -164,6 +164,7 @@ def test_quantize_layer_rejects_bad_shapes_and_options_before_launch(lib):
     assert call(n_ext=8) == -1                    # at most 7 extended codebooks
     assert call(n_base=-1) == -1
     assert call(n_base=2, n_ext=7) == -1          # at most 8 codebooks in all
+    assert call(n_base=2**31 - 1) == -1
     assert b"n_base" in lib.crvq_last_error()
     assert call(crit_frac=1.5) == -1
     assert call(B=17) == -1
