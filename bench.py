@@ -373,12 +373,10 @@ def sweep_grid(name):
 
 def avg_bits_of(P, cfg):
     """Bits per weight of a setting (Sec. 3.2 Eq. (bitwidth), App. A.1, the reorder index
-    included): crvq_avg_bits for one base and n_ext extended codebooks of 2^e codewords, plus
-    for each further base codebook e / d code bits per weight and its 2^e fp16 codewords."""
+    included), with e = log2 K_base for every codebook."""
     e = int(np.log2(cfg.K_base))
-    bits = P.crvq_avg_bits(e, cfg.d, 1 + cfg.n_ext, float(cfg.crit_frac), cfg.M, cfg.N, True)
-    extra = cfg.n_base - 1
-    return bits + extra * (e / cfg.d + (2 ** e) * cfg.d * 16 / (cfg.M * cfg.N))
+    return P.crvq_avg_bits_bases(e, cfg.d, cfg.n_base, cfg.n_ext, float(cfg.crit_frac), cfg.M,
+                                 cfg.N, True)
 
 
 def run_sweep(args):

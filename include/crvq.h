@@ -353,6 +353,14 @@ crvq_status crvq_lut_matvec(const float* X_in, int64_t ldx, int64_t b, int64_t N
 double crvq_avg_bits(int32_t e, int32_t d, int32_t m, double lambda, int64_t M, int64_t N,
                      int32_t include_perm);
 
+/* The same with n_base base codebooks (crvq_config.n_base) and n_ext extended ones: e-bit codes
+ * for all vectors per base codebook (Sec. 3.2 Eq. (bitwidth) counts m of them), n_ext on the
+ * lambda fraction, n_base + n_ext codebooks of 2^e fp16 vectors of length d, and (include_perm)
+ * the reorder index. n_base = 1 equals crvq_avg_bits with m = 1 + n_ext. NaN for d, M, N or
+ * n_base below 1, or e or n_ext below 0. */
+double crvq_avg_bits_bases(int32_t e, int32_t d, int32_t n_base, int32_t n_ext, double lambda,
+                           int64_t M, int64_t N, int32_t include_perm);
+
 /* G_c = min(N/d, ceil(crit_frac * N / d)) (0 when crit_frac == 0). */
 int64_t crvq_n_crit_groups(int64_t N, int32_t d, float crit_frac);
 

@@ -440,13 +440,15 @@ def reconstruct_error(W_sorted, d, H_blocks, perm, cbs, G_c, X=None, delta=0.0):
 # --------------------------------------------------------------------------------------
 # Average bit-width (Sec. 3.2 Eq. (bitwidth); App. A.1)
 # --------------------------------------------------------------------------------------
-def avg_bits(e, d, m, lam, M=4096, N=4096, include_perm=False):
-    """Bits per weight of an M x N matrix with one base and m-1 extended codebooks.
+def avg_bits(e, d, m, lam, M=4096, N=4096, include_perm=False, n_base=1):
+    """Bits per weight of an M x N matrix with n_base base and m-1 extended codebooks.
 
-    Codes: e bits per vector for the base codebook on all M N / d vectors, and for each of
-    the m-1 extended codebooks on the lambda fraction of critical vectors; codebooks: m of
-    2^e fp16 vectors of length d; optional 16-bit reorder index per channel (App. A.1)."""
-    bits = (M * N / d) * e + (m - 1) * lam * (M * N / d) * e + m * (2 ** e) * d * 16
+    Codes: e bits per vector for each base codebook on all M N / d vectors (Sec. 3.2 Eq.
+    (bitwidth) counts m such codebooks), and for each of the m-1 extended codebooks on the
+    lambda fraction of critical vectors (App. A.1); codebooks: n_base + m - 1 of 2^e fp16
+    vectors of length d; optional 16-bit reorder index per channel (App. A.1)."""
+    nvec = M * N / d
+    bits = n_base * nvec * e + (m - 1) * lam * nvec * e + (n_base + m - 1) * (2 ** e) * d * 16
     if include_perm:
         bits += 16 * N
     return bits / (M * N)

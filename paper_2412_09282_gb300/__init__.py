@@ -6,7 +6,7 @@ torch tensors (device memory and streams) into pointers and sizes. Nothing here 
 step of the method on the host; if the library is missing, importing `api` raises.
 """
 from .api import (  # noqa: F401
-    Codebook, LayerOutputs, crvq_avg_bits, crvq_coupled_sweep, crvq_encode_beam, crvq_hessian,
+    Codebook, LayerOutputs, crvq_avg_bits, crvq_avg_bits_bases, crvq_coupled_sweep, crvq_encode_beam, crvq_hessian,
     crvq_hessian_blocks, crvq_hessian_inverse_diag,
     crvq_kmeans_init, crvq_lut_matvec, crvq_n_crit_groups, crvq_quantize_layer,
     crvq_reconstruct_error,

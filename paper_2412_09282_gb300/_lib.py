@@ -87,6 +87,8 @@ SIGNATURES = {
                                     C.c_int64, c_vp]),
     "crvq_avg_bits": (C.c_double, [C.c_int32, C.c_int32, C.c_int32, C.c_double, C.c_int64,
                                    C.c_int64, C.c_int32]),
+    "crvq_avg_bits_bases": (C.c_double, [C.c_int32, C.c_int32, C.c_int32, C.c_int32,
+                                         C.c_double, C.c_int64, C.c_int64, C.c_int32]),
     "crvq_n_crit_groups": (C.c_int64, [C.c_int64, C.c_int32, C.c_float]),
     "crvq_quantize_layer": (C.c_int32, [c_vp, c_vp, C.c_int64, C.c_int64, C.c_int64,
                                         C.POINTER(crvq_config), C.POINTER(crvq_layer_outputs),

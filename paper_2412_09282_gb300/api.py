@@ -130,6 +130,11 @@ def crvq_avg_bits(e, d, m, lam, M=4096, N=4096, include_perm=False) -> float:
     return float(_L().crvq_avg_bits(e, d, m, lam, M, N, int(bool(include_perm))))
 
 
+def crvq_avg_bits_bases(e, d, n_base, n_ext, lam, M=4096, N=4096, include_perm=False) -> float:
+    return float(_L().crvq_avg_bits_bases(e, d, n_base, n_ext, lam, M, N,
+                                          int(bool(include_perm))))
+
+
 def crvq_n_crit_groups(N, d, crit_frac) -> int:
     return int(_L().crvq_n_crit_groups(N, d, crit_frac))
 

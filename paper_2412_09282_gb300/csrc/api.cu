@@ -635,6 +635,16 @@ double crvq_avg_bits(int32_t e, int32_t d, int32_t m, double lambda, int64_t M, 
   return bits / ((double)M * (double)N);
 }
 
+double crvq_avg_bits_bases(int32_t e, int32_t d, int32_t n_base, int32_t n_ext, double lambda,
+                           int64_t M, int64_t N, int32_t include_perm) {
+  if (d <= 0 || M <= 0 || N <= 0 || n_base < 1 || n_ext < 0 || e < 0) return std::nan("");
+  const double nvec = (double)M * (double)N / (double)d;
+  double bits = (double)n_base * nvec * e + (double)n_ext * lambda * nvec * e +
+                (double)(n_base + n_ext) * std::ldexp(1.0, e) * d * 16.0;
+  if (include_perm) bits += 16.0 * (double)N;
+  return bits / ((double)M * (double)N);
+}
+
 }  // extern "C"
 
 // ------------------------------------------------------------------------- layer schedule

@@ -5,6 +5,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 from oracle import crvq_oracle as O
@@ -47,6 +48,11 @@ def test_avg_bits_and_crit_groups_match_oracle(lib):
             for ip in (False, True):
                 assert P.crvq_avg_bits(e, d, m, lam, M, N, ip) == pytest.approx(
                     O.avg_bits(e, d, m, lam, M, N, ip), rel=1e-12)
+                for nb in (1, 2, 3):
+                    assert P.crvq_avg_bits_bases(e, d, nb, m - 1, lam, M, N, ip) == \
+                        pytest.approx(O.avg_bits(e, d, m, lam, M, N, ip, n_base=nb), rel=1e-12)
+    assert np.isnan(P.crvq_avg_bits_bases(8, 8, 0, 1, 0.02))
+    assert np.isnan(P.crvq_avg_bits_bases(8, 8, 1, -1, 0.02))
     for N, d, lam in [(512, 8, 0.02), (4096, 8, 0.02), (11008, 8, 0.01), (8192, 8, 0.05),
                       (64, 8, 0.0), (64, 8, 1.0), (64, 8, 0.125), (8, 8, 0.5)]:
         assert P.crvq_n_crit_groups(N, d, lam) == O.n_crit_groups(N, d, lam)

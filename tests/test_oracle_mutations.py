@@ -162,8 +162,15 @@ def _init_residual_sign(orig):
 
 
 def _avg_bits_without_extended(orig):
-    def f(e, d, m, lam, M=4096, N=4096, include_perm=False):
-        return orig(e, d, 1, lam, M, N, include_perm)
+    def f(e, d, m, lam, M=4096, N=4096, include_perm=False, n_base=1):
+        return orig(e, d, 1, lam, M, N, include_perm, n_base)
+    return f
+
+
+def _avg_bits_one_base(orig):
+    """Every further base codebook's codes and codewords left out of the count."""
+    def f(e, d, m, lam, M=4096, N=4096, include_perm=False, n_base=1):
+        return orig(e, d, m, lam, M, N, include_perm, 1)
     return f
 
 
@@ -406,6 +413,8 @@ MUTATIONS = [
      ["test_kmeans_init_takes_sampled_vectors_and_residuals"]),
     ("bit-width: extended codebooks dropped", "avg_bits", _avg_bits_without_extended,
      ["test_avg_bits_paper_values"]),
+    ("bit-width: one base codebook counted", "avg_bits", _avg_bits_one_base,
+     ["test_avg_bits_of_base_codebooks_alone_is_sec_3_2_eq_bitwidth"]),
     ("critical groups: floor instead of ceiling", "n_crit_groups", _crit_groups_floor,
      ["test_n_crit_groups_closed_form"]),
     ("splitmix64: wrong output", "splitmix64", _splitmix64_wrong_constant,

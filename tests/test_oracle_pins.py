@@ -462,6 +462,19 @@ def test_avg_bits_paper_values():
         assert round(v, int(dec)) == pytest.approx(float(exp))
 
 
+def test_avg_bits_of_base_codebooks_alone_is_sec_3_2_eq_bitwidth():
+    """m base codebooks and no extended ones: the App. A.1 count reduces to Sec. 3.2 Eq.
+    (bitwidth) for a 4096 x 4096 matrix, n = m e / d + 2^(e - 20) m d; the two 1-bit settings
+    Sec. 3.2 names for e = 8 (m = 1, d = 8 and m = 2, d = 16) both come to 1 bit and a
+    fraction of a percent."""
+    for e, d, m in [(8, 8, 1), (8, 16, 2), (10, 8, 2), (12, 16, 3), (8, 8, 4)]:
+        eq = m * e / d + 2.0 ** (e - 20) * m * d
+        assert O.avg_bits(e, d, 1, 0.0, n_base=m) == pytest.approx(eq, rel=1e-12)
+        assert O.avg_bits(e, d, 1, 0.3, n_base=m) == pytest.approx(eq, rel=1e-12)
+    for d, m in [(8, 1), (16, 2)]:
+        assert 1.0 < O.avg_bits(8, d, 1, 0.0, n_base=m) < 1.01
+
+
 # ---------------------------------------------------------------- schedule invariants
 def test_schedule_invariants_small():
     """Extended codebooks never raise the critical-channel loss (LS optimality vs c = 0
